@@ -1,0 +1,331 @@
+"""Python access to the plain CPU oracle (``oracle/ilw_oracle.cpp``).
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s
+CPU-baseline / reference arm may import this package.  It never imports the product package
+and the product package never imports it.
+
+Every function takes and returns numpy arrays; the integer semantics are those of the C++
+oracle (see ``ilw_oracle.h``): Algorithm 1 (ShiftExp, SD-ShiftGELU), Algorithm 2
+(CalibrateShift, Constrained Shiftmax), Sec. 3.2 (integer linear layers, split convolution),
+Sec. 3.3 (I-LayerNorm) and Sec. 3.1.1 (nearest-neighbour deformable sampling).
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "ilw_oracle.cpp")
+_LIB_PATH = os.path.join(_HERE, "libilw_oracle.so")
+_lib = None
+
+i8p = C.POINTER(C.c_int8)
+u8p = C.POINTER(C.c_uint8)
+i16p = C.POINTER(C.c_int16)
+i32p = C.POINTER(C.c_int32)
+i64p = C.POINTER(C.c_int64)
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with g++ (C++20, -O2) into ``oracle/libilw_oracle.so``."""
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < max(
+        os.path.getmtime(_SRC), os.path.getmtime(os.path.join(_HERE, "ilw_oracle.h"))
+    ):
+        tmp = _LIB_PATH + ".tmp%d" % os.getpid()
+        subprocess.check_call(
+            ["g++", "-std=c++20", "-O2", "-fPIC", "-shared", "-Wall", "-o", tmp, _SRC]
+        )
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+class ShiftmaxParams(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in ("I0", "k_inter", "k_out", "s_d", "m_p", "M_hw")]
+
+
+class BlockParams(C.Structure):
+    _fields_ = [
+        ("d", C.c_int32), ("H", C.c_int32), ("F", C.c_int32), ("win_side", C.c_int32),
+        ("ln_iters", C.c_int32),
+        ("ln1_beta", i32p), ("ln1_mult", i32p), ("ln1_shift", i32p),
+        ("ln2_beta", i32p), ("ln2_mult", i32p), ("ln2_shift", i32p),
+        ("w_qkv", i8p), ("b_qkv", i32p), ("m_qkv", i32p), ("s_qkv", i32p),
+        ("smx", ShiftmaxParams),
+        ("m_o", C.c_int32), ("s_o", C.c_int32),
+        ("w_proj", i8p), ("b_proj", i32p), ("m_proj", i32p), ("s_proj", i32p),
+        ("m_r1", C.c_int32), ("s_r1", C.c_int32),
+        ("w_fc1", i8p), ("b_fc1", i32p), ("m_fc1", i32p), ("s_fc1", i32p),
+        ("gelu_I0", C.c_int32), ("gelu_k_inter", C.c_int32), ("gelu_k_out", C.c_int32),
+        ("m_g", C.c_int32), ("s_g", C.c_int32),
+        ("w_fc2", i8p), ("b_fc2", i32p), ("m_fc2", i32p), ("s_fc2", i32p),
+        ("m_r2", C.c_int32), ("s_r2", C.c_int32),
+    ]
+
+
+class BlockTaps(C.Structure):
+    _fields_ = [("a1", i8p), ("qkv", i8p), ("o", i8p), ("x1", i16p), ("a2", i8p),
+                ("g", i16p), ("h", i8p)]
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        build()
+        L = C.CDLL(_LIB_PATH)
+        L.orc_rq.restype = C.c_int64
+        L.orc_rq.argtypes = [C.c_int64, C.c_int32, C.c_int32]
+        L.orc_sat.restype = C.c_int64
+        L.orc_sat.argtypes = [C.c_int64, C.c_int32]
+        L.orc_shiftexp.restype = C.c_int64
+        L.orc_shiftexp.argtypes = [C.c_int64, C.c_int64, C.c_int32]
+        L.orc_calibrate_shift.restype = C.c_int32
+        L.orc_calibrate_shift.argtypes = [C.c_int64, C.c_int32, C.c_int32]
+        L.orc_sdshiftgelu_idiv.restype = C.c_int64
+        L.orc_sdshiftgelu_idiv.argtypes = [C.c_int64, C.c_int32, C.c_int32, C.c_int32]
+        L.orc_newton_isqrt.restype = C.c_int64
+        L.orc_newton_isqrt.argtypes = [C.c_int64, C.c_int32]
+        L.orc_shiftexp_vec.restype = None
+        L.orc_shiftexp_vec.argtypes = [i32p, C.c_int64, C.c_int32, C.c_int32, i64p]
+        L.orc_shiftmax_rows.restype = C.c_int
+        L.orc_shiftmax_rows.argtypes = [i32p, C.c_int64, C.c_int64, C.c_int64,
+                                        C.POINTER(ShiftmaxParams), u8p, C.c_int64, i64p, i32p, i64p]
+        L.orc_sdshiftgelu.restype = C.c_int
+        L.orc_sdshiftgelu.argtypes = [i32p, i32p, C.c_int64, C.c_int32, C.c_int32, C.c_int32]
+        L.orc_int_layernorm.restype = C.c_int
+        L.orc_int_layernorm.argtypes = [i32p, C.c_int64, C.c_int64, C.c_int64, i32p, i32p, i32p,
+                                        C.c_int32, C.c_int32, i32p, C.c_int64]
+        L.orc_gemm_requant.restype = C.c_int
+        L.orc_gemm_requant.argtypes = [i8p, C.c_int64, i8p, C.c_int64, i32p, i32p, i32p,
+                                       C.c_int64, C.c_int64, C.c_int64, C.c_int32,
+                                       i16p, C.c_int64, C.c_int64, C.c_int32, C.c_int32,
+                                       i32p, C.c_int64]
+        L.orc_attention.restype = C.c_int
+        L.orc_attention.argtypes = [i8p, i8p, i8p, C.c_int64, C.c_int32, C.c_int32, C.c_int32,
+                                    C.c_int32, C.c_int32, C.POINTER(ShiftmaxParams), C.c_int32,
+                                    C.c_int32, i8p, C.c_int64]
+        L.orc_block_forward.restype = C.c_int
+        L.orc_block_forward.argtypes = [C.POINTER(BlockParams), i16p, i16p, C.c_int32, C.c_int32,
+                                        C.POINTER(BlockTaps)]
+        L.orc_split_conv.restype = C.c_int
+        L.orc_split_conv.argtypes = [C.POINTER(i8p), i64p, C.c_int32, C.c_int64, i32p,
+                                     C.POINTER(i8p), i32p, i32p, i32p, i32p, i32p, C.c_int64,
+                                     i8p, C.c_int64]
+        L.orc_deform_attn.restype = C.c_int
+        L.orc_deform_attn.argtypes = [i8p, i32p, C.c_int32, i32p, i32p, u8p, C.c_int32,
+                                      C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int64,
+                                      C.c_int32, C.c_int32, i8p]
+        _lib = L
+    return _lib
+
+
+def _p(a: np.ndarray, ptype):
+    assert a.flags["C_CONTIGUOUS"], "oracle wants C-contiguous arrays"
+    return a.ctypes.data_as(ptype)
+
+
+def _check(rc: int, what: str) -> None:
+    if rc != 0:
+        raise ValueError(f"oracle {what} rejected its arguments (rc={rc})")
+
+
+# ---------------------------------------------------------------- scalar building blocks
+def rq(v: int, m: int, s: int) -> int:
+    return int(lib().orc_rq(int(v), int(m), int(s)))
+
+
+def sat(v: int, bits: int) -> int:
+    return int(lib().orc_sat(int(v), int(bits)))
+
+
+def shiftexp(I: int, I0: int, k_inter: int = 16) -> int:
+    return int(lib().orc_shiftexp(int(I), int(I0), int(k_inter)))
+
+
+def calibrate_shift(S_sum: int, m_p: int = 4, M_hw: int = 31) -> int:
+    return int(lib().orc_calibrate_shift(int(S_sum), int(m_p), int(M_hw)))
+
+
+def sdshiftgelu_idiv(x: int, I0: int, k_inter: int = 16, k_out: int = 8) -> int:
+    return int(lib().orc_sdshiftgelu_idiv(int(x), int(I0), int(k_inter), int(k_out)))
+
+
+def newton_isqrt(V: int, iters: int) -> int:
+    return int(lib().orc_newton_isqrt(int(V), int(iters)))
+
+
+# ---------------------------------------------------------------- tensor operators
+def shiftexp_vec(I: np.ndarray, I0: int, k_inter: int = 16) -> np.ndarray:
+    I = np.ascontiguousarray(I, dtype=np.int32)
+    out = np.empty(I.shape, dtype=np.int64)
+    lib().orc_shiftexp_vec(_p(I, i32p), I.size, I0, k_inter, _p(out, i64p))
+    return out
+
+
+def shiftmax_rows(X: np.ndarray, I0: int, k_inter: int = 16, k_out: int = 8, s_d: int = -1,
+                  m_p: int = 4, M_hw: int = 31):
+    """Constrained Shiftmax (Algorithm 2) on every row of a 2-D int32 array.
+
+    Returns (P u8 [rows, len], S_sum int64 [rows], s_d int32 [rows], S_R int64 [rows])."""
+    X = np.ascontiguousarray(X, dtype=np.int32)
+    rows, n = X.shape
+    P = np.zeros((rows, n), dtype=np.uint8)
+    S = np.zeros(rows, dtype=np.int64)
+    sd = np.zeros(rows, dtype=np.int32)
+    SR = np.zeros(rows, dtype=np.int64)
+    prm = ShiftmaxParams(I0, k_inter, k_out, s_d, m_p, M_hw)
+    _check(lib().orc_shiftmax_rows(_p(X, i32p), n, rows, n, C.byref(prm), _p(P, u8p), n,
+                                   _p(S, i64p), _p(sd, i32p), _p(SR, i64p)), "shiftmax_rows")
+    return P, S, sd, SR
+
+
+def sdshiftgelu(X: np.ndarray, I0: int, k_inter: int = 16, k_out: int = 8) -> np.ndarray:
+    """SD-ShiftGELU (Algorithm 1): returns I_out = x * I_div as int32 (scale S_x 2^-(k_out-1))."""
+    X = np.ascontiguousarray(X, dtype=np.int32)
+    Y = np.empty_like(X)
+    _check(lib().orc_sdshiftgelu(_p(X, i32p), _p(Y, i32p), X.size, I0, k_inter, k_out),
+           "sdshiftgelu")
+    return Y
+
+
+def int_layernorm(X: np.ndarray, beta, mult, shift, iters: int = 10, out_bits: int = 8):
+    """I-LayerNorm over the last axis of a 2-D integer array; returns int32 values."""
+    X = np.ascontiguousarray(X, dtype=np.int32)
+    rows, Cn = X.shape
+    beta = np.ascontiguousarray(beta, dtype=np.int32)
+    mult = np.ascontiguousarray(mult, dtype=np.int32)
+    shift = np.ascontiguousarray(shift, dtype=np.int32)
+    Y = np.empty((rows, Cn), dtype=np.int32)
+    _check(lib().orc_int_layernorm(_p(X, i32p), Cn, rows, Cn, _p(beta, i32p), _p(mult, i32p),
+                                   _p(shift, i32p), iters, out_bits, _p(Y, i32p), Cn),
+           "int_layernorm")
+    return Y
+
+
+def gemm_requant(A: np.ndarray, W: np.ndarray, bias, mult, shift, out_bits: int = 8,
+                 res: np.ndarray | None = None, m_r: int = 0, s_r: int = 0) -> np.ndarray:
+    """Integer linear layer: A int8 [M,K], W int8 [N,K] -> int32 [M,N] holding the result."""
+    A = np.ascontiguousarray(A, dtype=np.int8)
+    W = np.ascontiguousarray(W, dtype=np.int8)
+    M, K = A.shape
+    N = W.shape[0]
+    assert W.shape[1] == K
+    bias = None if bias is None else np.ascontiguousarray(bias, dtype=np.int32)
+    mult = np.ascontiguousarray(mult if mult is not None else np.zeros(N), dtype=np.int32)
+    shift = np.ascontiguousarray(shift if shift is not None else np.zeros(N), dtype=np.int32)
+    Cm = np.empty((M, N), dtype=np.int32)
+    if res is not None:
+        res = np.ascontiguousarray(res, dtype=np.int16)
+        rp, ldr, rrows = _p(res, i16p), res.shape[1], res.shape[0]
+    else:
+        rp, ldr, rrows = None, 0, 1
+    _check(lib().orc_gemm_requant(_p(A, i8p), K, _p(W, i8p), K,
+                                  None if bias is None else _p(bias, i32p), _p(mult, i32p),
+                                  _p(shift, i32p), M, N, K, out_bits, rp, ldr, rrows, m_r, s_r,
+                                  _p(Cm, i32p), N), "gemm_requant")
+    return Cm
+
+
+def attention(qkv: np.ndarray, B: int, T: int, H: int, dh: int, win_side: int, smx: dict,
+              m_o: int, s_o: int) -> np.ndarray:
+    """Attention over a token-major [B*T, 3*H*dh] int8 q|k|v buffer -> int8 O [B*T, H*dh]."""
+    qkv = np.ascontiguousarray(qkv, dtype=np.int8)
+    d = H * dh
+    ld = qkv.shape[1]
+    O = np.zeros((B * T, d), dtype=np.int8)
+    prm = ShiftmaxParams(smx["I0"], smx.get("k_inter", 16), smx.get("k_out", 8),
+                         smx.get("s_d", -1), smx.get("m_p", 4), smx.get("M_hw", 31))
+    base = qkv.ctypes.data
+    _check(lib().orc_attention(C.cast(base, i8p), C.cast(base + d, i8p), C.cast(base + 2 * d, i8p),
+                               ld, B, T, H, dh, win_side, C.byref(prm), m_o, s_o, _p(O, i8p), d),
+           "attention")
+    return O
+
+
+def _block_struct(bp: dict, keep: list) -> BlockParams:
+    def arr(name, dt):
+        a = np.ascontiguousarray(bp[name], dtype=dt)
+        keep.append(a)
+        return _p(a, i8p if dt == np.int8 else i32p)
+
+    s = bp["smx"]
+    return BlockParams(
+        bp["d"], bp["H"], bp["F"], bp["win_side"], bp["ln_iters"],
+        arr("ln1_beta", np.int32), arr("ln1_mult", np.int32), arr("ln1_shift", np.int32),
+        arr("ln2_beta", np.int32), arr("ln2_mult", np.int32), arr("ln2_shift", np.int32),
+        arr("w_qkv", np.int8), arr("b_qkv", np.int32), arr("m_qkv", np.int32), arr("s_qkv", np.int32),
+        ShiftmaxParams(s["I0"], s["k_inter"], s["k_out"], s["s_d"], s["m_p"], s["M_hw"]),
+        bp["m_o"], bp["s_o"],
+        arr("w_proj", np.int8), arr("b_proj", np.int32), arr("m_proj", np.int32), arr("s_proj", np.int32),
+        bp["m_r1"], bp["s_r1"],
+        arr("w_fc1", np.int8), arr("b_fc1", np.int32), arr("m_fc1", np.int32), arr("s_fc1", np.int32),
+        bp["gelu_I0"], bp["gelu_k_inter"], bp["gelu_k_out"], bp["m_g"], bp["s_g"],
+        arr("w_fc2", np.int8), arr("b_fc2", np.int32), arr("m_fc2", np.int32), arr("s_fc2", np.int32),
+        bp["m_r2"], bp["s_r2"],
+    )
+
+
+def block_forward(bp: dict, x: np.ndarray, B: int, T: int, taps: bool = False):
+    """One integer encoder block on int16 x [B*T, d]; returns y (and a dict of taps)."""
+    keep: list = []
+    st = _block_struct(bp, keep)
+    x = np.ascontiguousarray(x, dtype=np.int16)
+    y = np.empty_like(x)
+    d, F = bp["d"], bp["F"]
+    M = B * T
+    tp = None
+    out = {}
+    if taps:
+        out = {"a1": np.empty((M, d), np.int8), "qkv": np.empty((M, 3 * d), np.int8),
+               "o": np.empty((M, d), np.int8), "x1": np.empty((M, d), np.int16),
+               "a2": np.empty((M, d), np.int8), "g": np.empty((M, F), np.int16),
+               "h": np.empty((M, F), np.int8)}
+        tp = BlockTaps(*[_p(out[k], i16p if out[k].dtype == np.int16 else i8p)
+                         for k in ("a1", "qkv", "o", "x1", "a2", "g", "h")])
+    _check(lib().orc_block_forward(C.byref(st), _p(x, i16p), _p(y, i16p), B, T,
+                                   None if tp is None else C.byref(tp)), "block_forward")
+    return (y, out) if taps else y
+
+
+def split_conv(Xs: list, Ws: list, m_b, s_b, bias, mult, shift) -> np.ndarray:
+    """Scale-preserving split convolution (Sec. 3.2.2) over nb branches of int8 [M, K_b]."""
+    nb = len(Xs)
+    Xs = [np.ascontiguousarray(x, dtype=np.int8) for x in Xs]
+    Ws = [np.ascontiguousarray(w, dtype=np.int8) for w in Ws]
+    M = Xs[0].shape[0]
+    N = Ws[0].shape[0]
+    Kb = np.array([x.shape[1] for x in Xs], dtype=np.int32)
+    ldx = np.array([x.shape[1] for x in Xs], dtype=np.int64)
+    xp = (i8p * nb)(*[_p(x, i8p) for x in Xs])
+    wp = (i8p * nb)(*[_p(w, i8p) for w in Ws])
+    m_b = np.ascontiguousarray(m_b, dtype=np.int32)
+    s_b = np.ascontiguousarray(s_b, dtype=np.int32)
+    bias = np.ascontiguousarray(bias, dtype=np.int32)
+    mult = np.ascontiguousarray(mult, dtype=np.int32)
+    shift = np.ascontiguousarray(shift, dtype=np.int32)
+    Y = np.empty((M, N), dtype=np.int8)
+    _check(lib().orc_split_conv(xp, _p(ldx, i64p), nb, M, _p(Kb, i32p), wp, _p(m_b, i32p),
+                                _p(s_b, i32p), _p(bias, i32p), _p(mult, i32p), _p(shift, i32p),
+                                N, _p(Y, i8p), N), "split_conv")
+    return Y
+
+
+def deform_attn(value: np.ndarray, level_hw, ref_q16: np.ndarray, off_q8: np.ndarray,
+                w: np.ndarray, m: int, s: int) -> np.ndarray:
+    """Nearest-neighbour deformable sampling: value int8 [B, S, H*dh]; ref [B,Q,2];
+    off [B,Q,H,L,P,2]; w u8 [B,Q,H,L*P] -> int8 [B, Q, H*dh]."""
+    value = np.ascontiguousarray(value, dtype=np.int8)
+    lhw = np.ascontiguousarray(level_hw, dtype=np.int32).reshape(-1, 2)
+    ref_q16 = np.ascontiguousarray(ref_q16, dtype=np.int32)
+    off_q8 = np.ascontiguousarray(off_q8, dtype=np.int32)
+    w = np.ascontiguousarray(w, dtype=np.uint8)
+    B, S, Dm = value.shape
+    _, Q, H, L, P, _ = off_q8.shape
+    dh = Dm // H
+    out = np.empty((B, Q, Dm), dtype=np.int8)
+    _check(lib().orc_deform_attn(_p(value, i8p), _p(lhw, i32p), L, _p(ref_q16, i32p),
+                                 _p(off_q8, i32p), _p(w, u8p), B, Q, H, P, dh, S, m, s,
+                                 _p(out, i8p)), "deform_attn")
+    return out

@@ -1,0 +1,550 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself.
+
+Each test names what fixes the expected value: exact rational arithmetic (Python integers and
+fractions), closed forms derived by hand from Algorithms 1 and 2, a library routine (numpy
+int64 matmul, math.isqrt, math.exp), invariants the paper states (the quotient-remainder
+identity, I_delta <= 0, element-wise independence of SD-ShiftGELU), or brute force over every
+input of a small range.  The tolerances of the float comparisons are derived in the docstrings.
+"""
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+from paper_2607_24981_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+LOG2E = 1.0 / math.log(2.0)
+
+
+def exact_rq(v: int, m: int, s: int) -> int:
+    """floor(v*m / 2^s + 1/2) with exact rationals (round half up)."""
+    return math.floor(Fraction(v * m, 1 << s) + Fraction(1, 2)) if s > 0 else v * m
+
+
+# ----------------------------------------------------------------------------- requant / sat
+def test_rq_matches_exact_rational(orc):
+    rng = np.random.default_rng(1)
+    cases = [(0, 1 << 30, 30), (1, 1 << 30, 30), (-1, 1 << 30, 31), (-(1 << 31), (1 << 31) - 1, 40),
+             ((1 << 31) - 1, (1 << 31) - 1, 31), (-3, 1, 1), (3, 1, 1), (-5, 3, 2)]
+    for _ in range(2000):
+        v = int(rng.integers(-(1 << 31), 1 << 31))
+        m = int(rng.integers(-(1 << 31), 1 << 31))
+        s = int(rng.integers(1, 62))
+        cases.append((v, m, s))
+    for v, m, s in cases:
+        assert orc.rq(v, m, s) == exact_rq(v, m, s), (v, m, s)
+
+
+def test_rq_identity_and_halves(orc):
+    # m = 2^30, s = 30 is the identity; exact halves round up (towards +inf)
+    for v in range(-1000, 1001):
+        assert orc.rq(v, 1 << 30, 30) == v
+    assert orc.rq(1, 1, 1) == 1 and orc.rq(-1, 1, 1) == 0 and orc.rq(-3, 1, 1) == -1
+
+
+def test_sat_symmetric(orc):
+    assert orc.sat(200, 8) == 127 and orc.sat(-200, 8) == -127 and orc.sat(-128, 8) == -127
+    assert orc.sat(40000, 16) == 32767 and orc.sat(-40000, 16) == -32767
+    assert orc.sat(5, 8) == 5
+
+
+# ----------------------------------------------------------------------------- ShiftExp
+def test_shiftexp_closed_form_multiples(orc):
+    """I = -16 j with I0 = 23: I_e = -16j - 8j + j = -23 j = -j I0 exactly, so q = j, r = 0,
+    I_b = I0 and I_exp = 23 * 2^(16-j) for j <= 16 and the clamp value I0 beyond."""
+    for j in range(0, 40):
+        want = 23 * (1 << (16 - j)) if j <= 16 else 23
+        assert orc.shiftexp(-16 * j, 23, 16) == want, j
+
+
+def test_shiftexp_brute_force_properties(orc):
+    """Every Delta in [-1.5 k I0, 0] for several I0: top value I0 2^k, monotone, clamp value I0
+    below the threshold, and the float bound of the shift-add exponential:
+      S_exp I_exp / exp(Delta/I0) = 2^((I_e - log2e Delta)/I0) * (1 - f/2)/2^-f * (I_b/(I0(1-f/2)))
+    with |I_e - 1.4375 Delta| < 1, (1 - f/2)/2^-f in [1, 1.0614] and |I_b - I0(1-f/2)| <= 1/2."""
+    k = 16
+    for I0 in (1, 2, 3, 7, 23, 256, 1023, 4096):
+        lo = -int(1.5 * k * I0) - 16
+        D = np.arange(lo, 1, dtype=np.int32)
+        e = orc.shiftexp_vec(D, I0, k)
+        assert e[-1] == I0 << k
+        assert np.all(np.diff(e) >= 0), "ShiftExp must be non-decreasing"
+        assert e.min() == I0
+        # unclamped region: -I_e < k I0  <=>  1.4375 |Delta| < k I0 - 1
+        Df = D.astype(np.float64)
+        un = (1.4375 * -Df + 1.0) < k * I0
+        x = Df[un] / I0
+        ratio = (e[un].astype(np.float64) / (I0 * 2.0 ** k)) / np.exp(x)
+        drift = (1.4375 - LOG2E) * Df[un] / I0  # >= 0 since Delta <= 0
+        upper = 1.0614 * 2.0 ** (drift + 1.0 / I0) * (1.0 + 1.0 / I0)
+        lower = 2.0 ** (drift - 1.0 / I0) * (1.0 - 1.0 / I0)
+        assert np.all(ratio <= upper + 1e-12), I0
+        assert np.all(ratio >= lower - 1e-12), I0
+
+
+def test_shiftexp_relative_error_grows_with_magnitude(orc):
+    """Sec. 3.3.1 / Fig. 3: the relative error of ShiftExp increases as the input becomes more
+    negative (1.4375 < log2 e).  The linear 2^-f part repeats with period 1 in 1.4375 x, so the
+    mean error over bins of two whole periods rises from bin to bin by the drift factor."""
+    I0, k = 4096, 16
+    D = np.arange(-11 * I0, 1, dtype=np.int32)
+    e = orc.shiftexp_vec(D, I0, k)
+    rel = e / (I0 * 2.0 ** k) / np.exp(D / I0) - 1.0
+    u = -1.4375 * D / I0  # exponent in periods
+    bins = [rel[(u >= 2 * b) & (u < 2 * b + 2)].mean() for b in range(7)]
+    assert all(b2 > b1 for b1, b2 in zip(bins, bins[1:])), bins
+
+
+# ----------------------------------------------------------------------------- CalibrateShift
+def test_calibrate_shift_powers_of_two(orc):
+    """M_req = ceil(log2 S): 2^j -> j and 2^j + 1 -> j + 1; s_d = max(M_req + 4 - 31, 0)."""
+    for j in range(0, 61):
+        assert orc.calibrate_shift(1 << j, 4, 31) == max(j + 4 - 31, 0)
+        if j >= 1:
+            assert orc.calibrate_shift((1 << j) + 1, 4, 31) == max(j + 1 + 4 - 31, 0)
+        assert orc.calibrate_shift((1 << (j + 1)) - 1 if j >= 1 else 1, 4, 31) == max(
+            (j + 1 if j >= 1 else 0) + 4 - 31, 0)
+
+
+def test_calibrate_shift_keeps_shifted_sum_below_target(orc):
+    """After the shift, S_sum / 2^s_d < 2^(M_hw - m_p) and (when s_d > 0) the shift is minimal."""
+    rng = np.random.default_rng(2)
+    for _ in range(3000):
+        S = int(rng.integers(1, 1 << 62))
+        sd = orc.calibrate_shift(S, 4, 31)
+        assert Fraction(S, 1 << sd) <= (1 << 27)
+        if sd > 0:
+            assert Fraction(S, 1 << (sd - 1)) > (1 << 27)
+
+
+# ----------------------------------------------------------------------------- Constrained Shiftmax
+def _golden_rows():
+    rows = []
+    with open(os.path.join(GOLDEN, "shiftmax_closed_forms.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                rows.append([int(t) for t in line.split()])
+    return rows
+
+
+def test_shiftmax_uniform_row_closed_forms(orc):
+    for n, I0, Iexp, Ssum, sd, SR, F, out in _golden_rows():
+        X = np.full((1, n), 12345, dtype=np.int32)
+        P, S, sdv, SRv = orc.shiftmax_rows(X, I0)
+        assert S[0] == Ssum and sdv[0] == sd and SRv[0] == SR
+        assert (2**31 - 1) // SRv[0] == F
+        assert np.all(P == out)
+
+
+def test_shiftmax_qr_identity_and_range(orc):
+    """Quotient-remainder accumulation (Sec. 3.3.2) equals floor(S_sum / 2^s_d); every output is
+    in [0, 2^k_out) and F >= 2^m_p - 1 in per-row mode (S_R < 2^(31 - m_p))."""
+    for L, I0 in ((1, 4096), (3, 17), (64, 1 << 12), (400, 1 << 13), (1600, 1 << 14), (65, 1000)):
+        X = synth.uniform_int(5, f"smx{L}", (64, L), -(1 << 15), 1 << 15)
+        P, S, sd, SR = orc.shiftmax_rows(X, I0)
+        for r in range(X.shape[0]):
+            assert SR[r] == min(max(S[r] >> sd[r], 1), 2**31 - 1)
+            assert (2**31 - 1) // SR[r] >= 15
+            e = orc.shiftexp_vec(X[r] - X[r].max(), I0)
+            assert int(e.sum()) == S[r]
+        assert P.max() < 256
+
+
+def test_shiftmax_monotone_and_shift_invariant(orc):
+    X = synth.uniform_int(6, "smxm", (32, 400), -(1 << 15), 1 << 15)
+    P, *_ = orc.shiftmax_rows(X, 3000)
+    P2, *_ = orc.shiftmax_rows(X + 777, 3000)
+    assert np.array_equal(P, P2)
+    for r in range(X.shape[0]):
+        order = np.argsort(X[r], kind="stable")
+        assert np.all(np.diff(P[r][order].astype(int)) >= 0)
+
+
+def test_shiftmax_sd0_is_ivit_shiftmax(orc):
+    """Static s_d = 0 is I-ViT's Shiftmax with M = 31:
+    out = (floor((2^31-1)/S_sum) * I_exp) >> (M - (k_out - 1)); when S_sum > 2^31 - 1 the
+    normaliser collapses (S_R clamps to 2^31-1, F = 1) and the outputs fall to ~0 (Table 9)."""
+    X = synth.uniform_int(7, "ivit", (16, 64), -20000, 20000)
+    for I0 in (64, 256, 1 << 12):
+        P, S, sd, SR = orc.shiftmax_rows(X, I0, s_d=0)
+        for r in range(X.shape[0]):
+            e = orc.shiftexp_vec(X[r] - X[r].max(), I0).astype(object)
+            Ssum = int(sum(e))
+            if Ssum <= 2**31 - 1:
+                want = [((2**31 - 1) // Ssum * int(v)) >> (31 - 7) for v in e]
+            else:
+                want = [int(v) >> (31 - 7) for v in e]  # F = 1
+            assert list(P[r]) == want
+    # collapse: a 1600-long row of equal scores at I0 = 2^12 has S_sum = 1600 * 2^28 > 2^31
+    Pc, S, _, _ = orc.shiftmax_rows(np.zeros((1, 1600), np.int32), 1 << 12, s_d=0)
+    assert S[0] > 2**31 and Pc.max() == (1 << 28) >> 24
+    Pr, *_ = orc.shiftmax_rows(np.zeros((1, 1600), np.int32), 1 << 12)
+    assert Pr.sum() < Pc.sum()
+
+
+def test_shiftmax_output_budget(orc):
+    """sum_i out_i <= floor(S_sum * F / 2^(24 + s_d)) <= 2^(k_out-1) (1 + 1/S_R)."""
+    X = synth.uniform_int(8, "budget", (200, 400), -(1 << 15), 1 << 15)
+    for I0 in (1 << 11, 1 << 13):
+        P, S, sd, SR = orc.shiftmax_rows(X, I0)
+        for r in range(X.shape[0]):
+            F = (2**31 - 1) // int(SR[r])
+            tot = int(P[r].astype(np.int64).sum())
+            assert tot <= (int(S[r]) * F) >> (24 + int(sd[r]))
+            assert Fraction(tot) <= Fraction(128) * (1 + Fraction(1, int(SR[r])))
+
+
+def test_shiftmax_close_to_float_softmax(orc):
+    """Float bound: I_exp_i = c exp(x_i) rho_i with rho in [rho_lo, rho_hi] (ShiftExp bound above),
+    so I_exp_i / S_sum is within the factor rho_hi/rho_lo of softmax_i; F = floor((2^31-1)/S_R)
+    loses at most the factor (1 - S_R/2^31); the final shift floors by < 1/128 and the
+    quotient-remainder shift by S_R/(S_R+1).  Hence
+      |out_i/128 - p_i| <= p_i (rho_hi/rho_lo - 1 + S_R/2^31 + 1/F + 1/S_R) + 1/128."""
+    I0 = 1 << 12
+    X = synth.uniform_int(9, "float", (100, 400), -(1 << 14), 1 << 14)
+    P, S, sd, SR = orc.shiftmax_rows(X, I0)
+    for r in range(X.shape[0]):
+        z = (X[r] - X[r].max()) / I0
+        p = np.exp(z) / np.exp(z).sum()
+        zmax = -z.min()
+        drift_hi = (1.4375 - LOG2E) * (-zmax)  # ratio drift is 2^(|1.4375-log2e| |z|)
+        rho = 1.0614 * 2 ** (-drift_hi + 2.0 / I0) * (1 + 2.0 / I0)
+        F = (2**31 - 1) // int(SR[r])
+        tol = p * (rho - 1 + int(SR[r]) / 2**31 + 1.0 / F + 1.0 / int(SR[r])) + 1 / 128 + 1e-9
+        assert np.all(np.abs(P[r] / 128.0 - p) <= tol)
+
+
+# ----------------------------------------------------------------------------- SD-ShiftGELU
+def _gelu_parts(x, I0):
+    """The algebraic pieces of the sigmoid the paper states (Sec. 3.3.1): I_p = 1.6875x with
+    floor shifts, the sign-split sigmoid with both exponent inputs <= 0."""
+    Ip = x + (x >> 1) + (x >> 3) + (x >> 4)
+    return Ip
+
+
+@pytest.mark.parametrize("I0", [1, 2, 3, 7, 64, 256, 512, 1023, 2048])
+def test_sdshiftgelu_brute_force(orc, I0):
+    """Every x in [-2^12, 2^12] (which contains every int8 value):
+    sign(out) in {sign(x), 0}; I_div in [0, 2^(k_out-1) - 1]; I_div(x) + I_div(-x) <= 127
+    (floor shifts give I_p(-x) <= -I_p(x)); monotone I_div when F keeps >= 8 bits (I0 <= 256);
+    and I_div equals 128 E/(E+E') up to the floors of IntDiv: |I_div - 128 sigma| <= 1 + I0/256."""
+    xs = np.arange(-4096, 4097, dtype=np.int32)
+    out = orc.sdshiftgelu(xs, I0)
+    idiv = np.array([orc.sdshiftgelu_idiv(int(x), I0) for x in xs])
+    assert np.array_equal(out, xs * idiv)
+    assert np.all((np.sign(out) == np.sign(xs)) | (out == 0))
+    assert idiv.min() >= 0 and idiv.max() <= 127
+    assert np.all(idiv + idiv[::-1] <= 127)
+    if I0 <= 256:
+        assert np.all(np.diff(idiv) >= 0)
+    for x, v in zip(xs[::7], idiv[::7]):
+        Ip = int(_gelu_parts(int(x), I0))
+        E = orc.shiftexp(min(Ip, 0), I0)
+        E2 = orc.shiftexp(-max(Ip, 0), I0)
+        sig = Fraction(128 * E, E + E2)
+        assert abs(Fraction(int(v)) - sig) <= 1 + Fraction(I0, 256)
+
+
+def test_sdshiftgelu_sigmoid_is_sign_split(orc):
+    """Sec. 3.3.1: sigma(z) = 1/(1+exp(-z)) for z >= 0 and exp(z)/(1+exp(z)) for z < 0 — both
+    exponent inputs non-positive; for x >= 0 the numerator is ShiftExp(0) = I0 2^k."""
+    I0 = 100
+    for x in (0, 1, 50, 300, 5000):
+        Ip = _gelu_parts(x, I0)
+        assert Ip >= 0 and orc.shiftexp(min(Ip, 0), I0) == I0 << 16
+    for x in (-1, -50, -300, -5000):
+        Ip = _gelu_parts(x, I0)
+        assert Ip < 0 and orc.shiftexp(-max(Ip, 0), I0) == I0 << 16
+
+
+def test_sdshiftgelu_elementwise_independence(orc):
+    """The paper's point against I-ViT's row-max ShiftGELU: each output depends on its own input
+    only, so permuting / embedding the input permutes / embeds the output."""
+    x = synth.uniform_int(10, "gind", (5000,), -4096, 4096)
+    y = orc.sdshiftgelu(x, 700)
+    perm = np.argsort(synth.uniform_int(10, "gperm", (5000,), 0, 1 << 30), kind="stable")
+    assert np.array_equal(orc.sdshiftgelu(x[perm], 700), y[perm])
+    big = x.copy()
+    big[0] = 4000000
+    assert np.array_equal(orc.sdshiftgelu(big, 700)[1:], y[1:])
+
+
+def test_sdshiftgelu_close_to_float_gelu(orc):
+    """Against x sigma(1.702 x) (the paper's GELU form, Eq. for GELU): the sigmoid argument uses
+    1.6875 x (|1.702 - 1.6875| |x| / 4 slope bound), ShiftExp ratios rho in [1, 1.0614 ...]
+    change sigma by <= sigma(1-sigma) ln(rho_hi/rho_lo) <= 0.25 ln 1.07, IntDiv floors cost
+    <= (1 + I0/256)/128.  Tolerance per element (real units, x = I_x / I0):
+      |x| (0.0145 |x| / 4 + 0.25 ln(1.07) + (1 + I0/256)/128 + 2/I0)."""
+    for I0 in (64, 256, 1024):
+        xs = np.arange(-8 * I0, 8 * I0 + 1, max(1, I0 // 64), dtype=np.int32)
+        out = orc.sdshiftgelu(xs, I0).astype(np.float64) / 128.0 / I0
+        x = xs / I0
+        ref = x / (1.0 + np.exp(-1.702 * x))
+        tol = np.abs(x) * (0.0145 * np.minimum(np.abs(x), 8) / 4 + 0.25 * math.log(1.07)
+                           + (1 + I0 / 256) / 128 + 2.0 / I0) + 1e-12
+        assert np.all(np.abs(out - ref) <= tol), I0
+
+
+# ----------------------------------------------------------------------------- Newton isqrt / LN
+def test_newton_isqrt_converges_to_isqrt(orc):
+    """With enough iterations the integer Newton iteration ends at isqrt(V) or isqrt(V)+1
+    (math.isqrt is the reference); after >= 1 step it never goes below isqrt(V)."""
+    vals = list(range(0, 5000)) + [int(v) for v in np.random.default_rng(3).integers(1, 1 << 40, 3000)]
+    for V in vals:
+        r = math.isqrt(V)
+        R = orc.newton_isqrt(V, 60)
+        assert R in (max(r, 1), r + 1), V
+        for n in (1, 10, 20):
+            assert orc.newton_isqrt(V, n) >= max(r, 1)
+
+
+def test_newton_isqrt_is_floored_real_newton(orc):
+    """Newton's method for x^2 = V is x <- (x + V/x)/2; the integer version floors each step.
+    Rebuild every iterate with exact rationals from the start 2^16 (one floor of the real step,
+    no nested floors) and compare the unconverged values after N = 1..12 steps."""
+    rng = np.random.default_rng(4)
+    for V in [1, 2, 3, 1000, 65535, 10**10, 2**39 - 5] + [int(v) for v in rng.integers(1, 1 << 40, 200)]:
+        x = 1 << 16
+        for n in range(1, 13):
+            x = math.floor((Fraction(x) + Fraction(V, x)) / 2)
+            assert orc.newton_isqrt(V, n) == max(x, 1), (V, n)
+
+
+def test_newton_isqrt_unconverged_closed_form(orc):
+    """V = 0: the iteration halves 2^16 each step: 2^(16-N) for N <= 16, then 0 -> clamp 1.
+    V = 2^32: 2^16 is already the fixed point."""
+    for n in range(0, 25):
+        assert orc.newton_isqrt(0, n) == max(1 << (16 - n), 1) if n <= 16 else 1
+    assert orc.newton_isqrt(1 << 32, 10) == 1 << 16
+
+
+def test_layernorm_constant_row_is_beta(orc):
+    """Constant row: y = 0, n = 0, out = sat(rq(beta))."""
+    d = 8
+    beta = np.array([100, -100, 5000, -5000, 0, 1, -1, 1 << 20], np.int32)
+    mult = np.array([1 << 30] * 4 + [-(1 << 30)] * 4, np.int32)
+    shift = np.full(d, 30, np.int32)
+    X = np.full((3, d), 77, np.int32)
+    Y = orc.int_layernorm(X, beta, mult, shift, 10, 16)
+    want = [max(-32767, min(32767, exact_rq(int(b), int(m), 30))) for b, m in zip(beta, mult)]
+    assert np.all(Y == np.array(want))
+
+
+def test_layernorm_mean_rounds_half_up(orc):
+    """Row [0, 1]: mean 1/2 rounds up to 1, y = [-1, 0], V = 1 -> R = 1 after >= 17 steps,
+    F = 2^31-1, n = [floor(-(2^31-1)/2), 0] = [-2^30, 0]."""
+    beta = np.zeros(2, np.int32)
+    mult = np.full(2, 1 << 30, np.int32)
+    shift = np.full(2, 46, np.int32)
+    Y = orc.int_layernorm(np.array([[0, 1]], np.int32), beta, mult, shift, 20, 16)
+    assert list(Y[0]) == [exact_rq(-(1 << 30), 1 << 30, 46), 0] == [-16384, 0]
+
+
+def test_layernorm_matches_float_normalisation(orc):
+    """n = (y F) >> 1 with F = floor((2^31-1)/R) approximates 2^30 y / sqrt(V); reading it out
+    through rq(.; 2^30, 45) gives 2^15 y / sqrt(V) within
+      2^15 (|y|/sqrt(V)) (|sqrt(V)/R - 1| + R/2^31) + 1.5 (floors and rounding)."""
+    C = 384
+    X = synth.uniform_int(11, "lnf", (200, C), -(1 << 14), 1 << 14)
+    beta = np.zeros(C, np.int32)
+    mult = np.full(C, 1 << 30, np.int32)
+    shift = np.full(C, 45, np.int32)
+    for iters in (10, 20):
+        Y = orc.int_layernorm(X, beta, mult, shift, iters, 16)
+        for r in range(X.shape[0]):
+            x = X[r].astype(np.int64)
+            mu = math.floor(Fraction(int(x.sum()), C) + Fraction(1, 2))
+            y = x - mu
+            V = int((y * y).sum())
+            R = orc.newton_isqrt(V, iters)
+            ref = 2.0 ** 15 * y / math.sqrt(V)
+            tol = 2.0 ** 15 * np.abs(y) / math.sqrt(V) * (abs(math.sqrt(V) / R - 1) + R / 2**31) + 1.5
+            assert np.all(np.abs(Y[r] - ref) <= tol)
+            assert R in (math.isqrt(V), math.isqrt(V) + 1) or iters == 10
+
+
+def test_layernorm_gamma_sign(orc):
+    C = 64
+    X = synth.uniform_int(12, "lns", (10, C), -2000, 2000)
+    beta = np.zeros(C, np.int32)
+    shift = np.full(C, 50, np.int32)
+    Yp = orc.int_layernorm(X, beta, np.full(C, 1 << 30, np.int32), shift, 10, 8)
+    Yn = orc.int_layernorm(X, beta, np.full(C, -(1 << 30), np.int32), shift, 10, 8)
+    # rq rounds half up, so negation is exact except at exact halves (off by one there)
+    assert np.all(np.abs(Yp + Yn) <= 1)
+
+
+# ----------------------------------------------------------------------------- GEMM
+@pytest.mark.parametrize("out_bits", [8, 16, 32])
+def test_gemm_matches_numpy_int64_and_exact_rq(orc, out_bits):
+    """Sec. 3.2.1: MAC in the integer domain, scale after accumulation.  Reference: numpy int64
+    matmul + exact rational rq + symmetric saturation."""
+    M, N, K = 37, 29, 70
+    A = synth.uniform_int(13, "A", (M, K), -127, 127, np.int8)
+    W, b, m, s = synth.gemm_params(13, "g", N, K, 73.0, 30.0, mode="literal")
+    res = synth.uniform_int(13, "res", (M, N), -30000, 30000, np.int16)
+    C = orc.gemm_requant(A, W, b, m, s, out_bits, res if out_bits != 32 else None, 1 << 30, 31)
+    acc = A.astype(np.int64) @ W.astype(np.int64).T + b
+    for i in range(M):
+        for c in range(N):
+            if out_bits == 32:
+                want = int(acc[i, c])
+            else:
+                v = exact_rq(int(acc[i, c]), int(m[c]), int(s[c])) + exact_rq(int(res[i, c]), 1 << 30, 31)
+                lim = (1 << (out_bits - 1)) - 1
+                want = max(-lim, min(lim, v))
+            assert C[i, c] == want
+
+
+# ----------------------------------------------------------------------------- attention
+def _smx(I0):
+    return {"I0": I0, "k_inter": 16, "k_out": 8, "s_d": -1, "m_p": 4, "M_hw": 31}
+
+
+def test_attention_matches_composed_reference(orc):
+    """scores = q k^T (numpy int64), P = Constrained Shiftmax (pinned above), O = P V (numpy),
+    O8 = sat8(exact rq)."""
+    B, T, H, dh = 2, 40, 2, 32
+    d = H * dh
+    qkv = synth.uniform_int(14, "qkv", (B * T, 3 * d), -127, 127, np.int8)
+    O = orc.attention(qkv, B, T, H, dh, 0, _smx(3000), 1 << 30, 38)
+    for b in range(B):
+        for h in range(H):
+            rows = slice(b * T, (b + 1) * T)
+            q = qkv[rows, h * dh:(h + 1) * dh].astype(np.int64)
+            k = qkv[rows, d + h * dh:d + (h + 1) * dh].astype(np.int64)
+            v = qkv[rows, 2 * d + h * dh:2 * d + (h + 1) * dh].astype(np.int64)
+            S = (q @ k.T).astype(np.int32)
+            P, *_ = orc.shiftmax_rows(S, 3000)
+            o = P.astype(np.int64) @ v
+            want = np.array([[max(-127, min(127, exact_rq(int(t), 1 << 30, 38))) for t in row] for row in o])
+            assert np.array_equal(O[rows, h * dh:(h + 1) * dh], want)
+
+
+def test_window_attention_is_global_attention_per_window(orc):
+    """Windowed attention on a 6x6 token grid with 2x2 windows equals global attention run on
+    each window's gathered tokens (numpy fancy indexing, independent of the oracle's index maths)."""
+    B, G, H, dh, nw = 2, 6, 2, 32, 2
+    T, d, ws = G * G, H * dh, G // nw
+    qkv = synth.uniform_int(15, "wqkv", (B * T, 3 * d), -127, 127, np.int8)
+    Ow = orc.attention(qkv, B, T, H, dh, nw, _smx(2000), 1 << 30, 37)
+    for b in range(B):
+        for wy in range(nw):
+            for wx in range(nw):
+                idx = np.array([b * T + (wy * ws + ly) * G + wx * ws + lx
+                                for ly in range(ws) for lx in range(ws)])
+                Og = orc.attention(qkv[idx], 1, ws * ws, H, dh, 0, _smx(2000), 1 << 30, 37)
+                assert np.array_equal(Ow[idx], Og)
+
+
+# ----------------------------------------------------------------------------- split conv
+def test_split_conv_equal_scales_is_concat_conv(orc):
+    """Table 7's baseline: with equal branch scales (m_b = 2^30, s_b = 30 is the identity) the
+    split convolution equals the single convolution over the concatenated channels."""
+    M, N, Ks = 50, 24, (16, 32, 48, 8)
+    Xs = [synth.uniform_int(16, f"x{i}", (M, k), -127, 127, np.int8) for i, k in enumerate(Ks)]
+    Ws = [synth.uniform_int(16, f"w{i}", (N, k), -127, 127, np.int8) for i, k in enumerate(Ks)]
+    bias = synth.uniform_int(16, "bias", (N,), -(1 << 15), 1 << 15)
+    mult = synth.uniform_int(16, "mult", (N,), 1 << 30, (1 << 31) - 1)
+    shift = np.full(N, 36, np.int32)
+    Y = orc.split_conv(Xs, Ws, [1 << 30] * 4, [30] * 4, bias, mult, shift)
+    Yc = orc.gemm_requant(np.concatenate(Xs, 1), np.concatenate(Ws, 1), bias, mult, shift, 8)
+    assert np.array_equal(Y, Yc.astype(np.int8))
+
+
+def test_split_conv_branch_rescale(orc):
+    """Each branch partial is rescaled by its own dyadic ratio before the integer sum."""
+    M, N = 20, 8
+    Xs = [synth.uniform_int(17, f"x{i}", (M, 16), -127, 127, np.int8) for i in range(2)]
+    Ws = [synth.uniform_int(17, f"w{i}", (N, 16), -127, 127, np.int8) for i in range(2)]
+    bias = np.zeros(N, np.int32)
+    mult = np.full(N, 1 << 30, np.int32)
+    shift = np.full(N, 38, np.int32)
+    mb, sb = [1 << 30, 3 << 28], [30, 31]  # ratios 1 and 3/8
+    Y = orc.split_conv(Xs, Ws, mb, sb, bias, mult, shift)
+    for i in range(M):
+        for c in range(N):
+            t = sum(exact_rq(int(Xs[b][i].astype(np.int64) @ Ws[b][c].astype(np.int64)), mb[b], sb[b])
+                    for b in range(2))
+            assert Y[i, c] == max(-127, min(127, exact_rq(t, 1 << 30, 38)))
+
+
+# ----------------------------------------------------------------------------- deformable sampling
+def test_deform_nearest_neighbour_cases(orc):
+    """Sec. 3.1.1: zero offsets at a pixel centre gather that pixel; a single weight-128 sample
+    returns rq(128 v); samples outside every map give 0; brute force against numpy gathers."""
+    B, Q, H, L, P, dh = 2, 5, 2, 2, 3, 16
+    hw = np.array([[4, 6], [2, 3]], np.int32)
+    S = int((hw[:, 0] * hw[:, 1]).sum())
+    value = synth.uniform_int(18, "val", (B, S, H * dh), -127, 127, np.int8)
+    # reference at the centre of pixel (ix=2, iy=1) of level 0: x = (2 + 0.5)/6, y = (1 + 0.5)/4
+    ref = np.zeros((B, Q, 2), np.int32)
+    ref[..., 0] = int((2.5 / 6) * 65536)
+    ref[..., 1] = int((1.5 / 4) * 65536)
+    off = np.zeros((B, Q, H, L, P, 2), np.int32)
+    w = np.zeros((B, Q, H, L * P), np.uint8)
+    w[..., 0] = 128  # level 0, point 0 only
+    out = orc.deform_attn(value, hw, ref, off, w, 1 << 30, 37)  # rq(128 v; 2^30, 37) = v
+    for b in range(B):
+        want = value[b, 1 * 6 + 2].astype(np.int64)
+        assert np.all(out[b] == want[None, :])
+    # all samples pushed outside -> zeros
+    off_far = np.full((B, Q, H, L, P, 2), -(1 << 16), np.int32)
+    w_all = np.full((B, Q, H, L * P), 20, np.uint8)
+    assert np.all(orc.deform_attn(value, hw, ref, off_far, w_all, 1 << 30, 30) == 0)
+    # random offsets: brute force with numpy gathers
+    off_r = synth.uniform_int(18, "off", (B, Q, H, L, P, 2), -(3 << 8), 3 << 8)
+    ref_r = synth.uniform_int(18, "ref", (B, Q, 2), 0, 65535)
+    w_r = synth.uniform_int(18, "w", (B, Q, H, L * P), 0, 60, np.uint8)
+    got = orc.deform_attn(value, hw, ref_r, off_r, w_r, 1 << 30, 34)
+    starts = [0, 24]
+    for b in range(B):
+        for q in range(Q):
+            for h in range(H):
+                acc = np.zeros(dh, np.int64)
+                for l in range(L):
+                    Hl, Wl = hw[l]
+                    for p in range(P):
+                        locx = Fraction(int(ref_r[b, q, 0]) * int(Wl), 65536) + Fraction(int(off_r[b, q, h, l, p, 0]), 256)
+                        locy = Fraction(int(ref_r[b, q, 1]) * int(Hl), 65536) + Fraction(int(off_r[b, q, h, l, p, 1]), 256)
+                        # the reference position is truncated to Q8 before the offset is added
+                        px = (int(ref_r[b, q, 0]) * int(Wl)) // 256 + int(off_r[b, q, h, l, p, 0])
+                        py = (int(ref_r[b, q, 1]) * int(Hl)) // 256 + int(off_r[b, q, h, l, p, 1])
+                        ix, iy = px // 256, py // 256
+                        assert abs(Fraction(px, 256) - locx) < 1 and abs(Fraction(py, 256) - locy) < 1
+                        if 0 <= ix < Wl and 0 <= iy < Hl:
+                            acc += int(w_r[b, q, h, l * P + p]) * value[b, starts[l] + iy * Wl + ix, h * dh:(h + 1) * dh].astype(np.int64)
+                want = [max(-127, min(127, exact_rq(int(a), 1 << 30, 34))) for a in acc]
+                assert list(got[b, q, h * dh:(h + 1) * dh]) == want
+
+
+# ----------------------------------------------------------------------------- block composition
+def test_block_equals_composition_of_pinned_parts(orc):
+    """orc_block_forward is parity-unpinned beyond its parts; this checks that it is exactly the
+    stated composition of the parts pinned above (LN -> QKV -> attention -> proj + residual ->
+    LN -> FC1 -> SD-ShiftGELU -> FC2 + residual)."""
+    B, T, d, H, F = 1, 16, 64, 2, 128
+    bp = synth.block_params(19, 0, d, H, F, 0, "calibrated")
+    x = synth.block_input(19, B, T, d)
+    y, taps = orc.block_forward(bp, x, B, T, taps=True)
+    a1 = orc.int_layernorm(x, bp["ln1_beta"], bp["ln1_mult"], bp["ln1_shift"], 10, 8)
+    assert np.array_equal(a1, taps["a1"])
+    qkv = orc.gemm_requant(a1, bp["w_qkv"], bp["b_qkv"], bp["m_qkv"], bp["s_qkv"], 8)
+    assert np.array_equal(qkv, taps["qkv"])
+    o = orc.attention(qkv, B, T, H, d // H, 0, bp["smx"], bp["m_o"], bp["s_o"])
+    assert np.array_equal(o, taps["o"])
+    x1 = orc.gemm_requant(o, bp["w_proj"], bp["b_proj"], bp["m_proj"], bp["s_proj"], 16, x,
+                          bp["m_r1"], bp["s_r1"])
+    assert np.array_equal(x1, taps["x1"])
+    a2 = orc.int_layernorm(x1, bp["ln2_beta"], bp["ln2_mult"], bp["ln2_shift"], 10, 8)
+    g = orc.gemm_requant(a2, bp["w_fc1"], bp["b_fc1"], bp["m_fc1"], bp["s_fc1"], 16)
+    assert np.array_equal(g, taps["g"])
+    gi = orc.sdshiftgelu(g, bp["gelu_I0"]).astype(np.int64)
+    h = np.array([[max(-127, min(127, exact_rq(int(v), bp["m_g"], bp["s_g"]))) for v in row] for row in gi])
+    assert np.array_equal(h, taps["h"])
+    y2 = orc.gemm_requant(h, bp["w_fc2"], bp["b_fc2"], bp["m_fc2"], bp["s_fc2"], 16, x1,
+                          bp["m_r2"], bp["s_r2"])
+    assert np.array_equal(y2, y)
