@@ -1,0 +1,444 @@
+#!/usr/bin/env python
+"""Throughput of the integer-only I-LW-DETR encoder on GB300.
+
+Default workload (N=1): the Medium-scale integer ViT backbone of the paper's Table 1 -- patch
+embedding of a 640x640 int8 image (1600 tokens of dim 384) followed by 10 encoder blocks (6
+heads, MLP 1536; global attention at layers 2, 4, 5, 9, 2x2-window attention elsewhere), batch
+8, seeded synthetic int8 inputs and weights.  One step = one backbone forward of the batch.
+The metric counts encoder-block tokens: value = blocks * B * T / step time.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Under torchrun (N > 1) every rank runs its own replica on its own batch (no data-path
+collective: the path shards by image); the step time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "int-only encoder block tokens/s (1600 tok, d=384)"
+UNIT = "block-tokens/s"
+WORKLOAD = "medium_c2"
+SEED = 0
+# cpu baseline / reference arm sample: one image through blocks 0..4 (3 window + 2 global, the
+# backbone's 6:4 window/global ratio)
+CPU_SAMPLE_BLOCKS = 5
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ilw", choices=["ilw", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args(argv)
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def max_over_ranks(value: float, world: int) -> float:
+    """Max of a per-rank float over the process group (identity for one process)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int) -> None:
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+# ------------------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples (every 200 ms) of SM clock and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.p = None
+
+    def __enter__(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+        return self
+
+    def __exit__(self, *a):
+        if self.p is not None:
+            self.p.terminate()
+            try:
+                self.p.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.p.kill()
+
+    def summary(self) -> dict:
+        self.f.flush()
+        self.f.seek(0)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.f.read().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.f.name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------ workload
+def workload_cfg():
+    from paper_2607_24981_gb300 import synth
+
+    return dict(synth.CONFIGS[WORKLOAD])
+
+
+def build_host_params():
+    from paper_2607_24981_gb300 import synth
+
+    cfg = workload_cfg()
+    blocks = synth.backbone_params(SEED, cfg)
+    pe = synth.patch_embed_params(SEED, cfg["d"], mode=cfg["mode"])
+    return cfg, pe, blocks
+
+
+class Instrumented:
+    """The backbone forward issued as the same sequence of ABI calls that ilwdetr_patch_embed and
+    ilwdetr_block_forward make, with CUDA events around each call so every kernel class gets its
+    own device time inside the timed region."""
+
+    def __init__(self, bb, torch):
+        self.bb, self.torch = bb, torch
+        M, d, F = bb.B * bb.T, bb.d, bb.F
+        dev = bb.x[0].device
+        self.a1 = torch.empty((M, d), dtype=torch.int8, device=dev)
+        self.qkv = torch.empty((M, 3 * d), dtype=torch.int8, device=dev)
+        self.o = torch.empty((M, d), dtype=torch.int8, device=dev)
+        self.x1 = torch.empty((M, d), dtype=torch.int16, device=dev)
+        self.a2 = torch.empty((M, d), dtype=torch.int8, device=dev)
+        self.h = torch.empty((M, F), dtype=torch.int8, device=dev)
+        self.xs = [torch.empty((M, d), dtype=torch.int16, device=dev) for _ in range(2)]
+        self.records = []  # (kernel class, start event, end event, launches)
+
+    def _ev(self):
+        e = self.torch.cuda.Event(enable_timing=True)
+        e.record()
+        return e
+
+    def _rec(self, name, fn, launches=1):
+        s = self._ev()
+        out = fn()
+        self.records.append((name, s, self._ev(), launches))
+        return out
+
+    def forward(self, img):
+        import paper_2607_24981_gb300 as ilw
+
+        bb, pe = self.bb, self.bb.pe
+        B, T, d, F = bb.B, bb.T, bb.d, bb.F
+        M = B * T
+        x = self._rec("patch_embed", lambda: ilw.patch_embed(
+            img, bb.p, pe["w_p"], d, pe["b"], pe["m"], pe["s"], pe["pos"], bb.pe_s["m_pos"],
+            bb.pe_s["s_pos"], bb.ws_pe, self.xs[0]), launches=2)
+        for i, bw in enumerate(bb.blocks):
+            t, p = bw.t, bw.bp
+            y = self.xs[(i + 1) % 2]
+            self._rec("layernorm", lambda: ilw.int_layernorm(x, t["ln1_beta"], t["ln1_mult"], t["ln1_shift"],
+                                                             p["ln_iters"], 8, out=self.a1))
+            self._rec("gemm_qkv", lambda: ilw.gemm_requant(self.a1, t["w_qkv_p"], 3 * d, t["b_qkv"], t["m_qkv"],
+                                                           t["s_qkv"], 8, out=self.qkv))
+            kind = "attention_global" if p["win_side"] <= 1 else "attention_window"
+            self._rec(kind, lambda: ilw.shiftmax_attn(self.qkv, B, T, p["H"], d // p["H"], p["win_side"], p["smx"],
+                                                      p["m_o"], p["s_o"], out=self.o))
+            self._rec("gemm_proj", lambda: ilw.gemm_requant(self.o, t["w_proj_p"], d, t["b_proj"], t["m_proj"],
+                                                            t["s_proj"], 16, res=x, m_r=p["m_r1"], s_r=p["s_r1"],
+                                                            out=self.x1))
+            self._rec("layernorm", lambda: ilw.int_layernorm(self.x1, t["ln2_beta"], t["ln2_mult"], t["ln2_shift"],
+                                                             p["ln_iters"], 8, out=self.a2))
+            self._rec("gemm_fc1_gelu", lambda: ilw.gemm_gelu(self.a2, t["w_fc1_p"], F, t["b_fc1"], t["m_fc1"],
+                                                             t["s_fc1"], {"I0": p["gelu_I0"]}, p["m_g"], p["s_g"],
+                                                             out=self.h))
+            self._rec("gemm_fc2", lambda: ilw.gemm_requant(self.h, t["w_fc2_p"], d, t["b_fc2"], t["m_fc2"], t["s_fc2"],
+                                                           16, res=self.x1, m_r=p["m_r2"], s_r=p["s_r2"], out=y))
+            x = y
+        return x
+
+
+def kernel_work(cfg, B):
+    """Algorithmic work per launch of each kernel class (one backbone step)."""
+    T, d, F, H = cfg["T"], cfg["d"], cfg["F"], cfg["H"]
+    M = B * T
+    dh = d // H
+    Tw = T // 4  # 2x2 windows
+    return {
+        # tensor classes: 2*M*N*K integer multiply-adds per launch
+        "gemm_qkv": ("tensor", 2.0 * M * 3 * d * d),
+        "gemm_proj": ("tensor", 2.0 * M * d * d),
+        "gemm_fc1_gelu": ("tensor", 2.0 * M * F * d),
+        "gemm_fc2": ("tensor", 2.0 * M * d * F),
+        "patch_embed": ("tensor", 2.0 * M * d * 768),
+        # attention: scores per launch (q.k^T, Shiftmax, P.V), see the ALU roofline
+        "attention_global": ("alu", float(B * H * T * T)),
+        "attention_window": ("alu", float(B * H * 4 * Tw * Tw)),
+        # I-LayerNorm: int16 in (2 B) + int8 out (1 B) per element
+        "layernorm": ("hbm", 3.0 * M * d),
+    }
+
+
+def run_cpu_sample(cfg, pe, blocks) -> dict:
+    """The oracle as it stands, single-threaded: one image through blocks 0..CPU_SAMPLE_BLOCKS-1."""
+    import numpy as np
+
+    import oracle
+    from paper_2607_24981_gb300 import synth
+
+    oracle.build()
+    img = synth.image_input(SEED, 1)
+    x = oracle.patch_embed(img, pe["p"], pe["w"], pe["b"], pe["m"], pe["s"], pe["pos"], pe["m_pos"], pe["s_pos"])
+    t0 = time.perf_counter()
+    for bp in blocks[:CPU_SAMPLE_BLOCKS]:
+        x = oracle.block_forward(bp, x, 1, cfg["T"])
+    dt = time.perf_counter() - t0
+    units = CPU_SAMPLE_BLOCKS * cfg["T"]
+    assert np.isfinite(dt)
+    return {"value": units / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"1 image x encoder blocks 0-{CPU_SAMPLE_BLOCKS - 1} (3 window + 2 global), "
+                      f"{units} block-tokens, {dt:.1f} s, single-threaded C++ oracle (-O2)"}
+
+
+# ------------------------------------------------------------------------------ reference arm
+def run_reference(args) -> None:
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    cfg, pe, blocks = build_host_params()
+    import oracle
+    from paper_2607_24981_gb300 import synth
+
+    oracle.build()
+    img = synth.image_input(SEED, 1)
+    x0 = oracle.patch_embed(img, pe["p"], pe["w"], pe["b"], pe["m"], pe["s"], pe["pos"], pe["m_pos"], pe["s_pos"])
+    times = []
+    for step in range(args.warmup + args.steps):
+        bp = blocks[step % len(blocks)]
+        t0 = time.perf_counter()
+        oracle.block_forward(bp, x0, 1, cfg["T"])
+        if step >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    ms = 1000.0 * statistics.mean(times)
+    value = cfg["T"] / (ms / 1000.0)
+    sample = (f"per step: 1 image (1600 tokens) through one encoder block, cycling over the 10 "
+              f"blocks (6 window, 4 global) step by step; single-threaded C++ oracle")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": "medium_c2 backbone (CPU oracle sample)", "B": 1, "T": cfg["T"],
+                       "d": cfg["d"], "H": cfg["H"], "F": cfg["F"]},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------ main arm
+def main(argv=None):
+    args = parse_args(argv)
+    if args.impl == "reference":
+        return run_reference(args)
+    rank, world, local = dist_env()
+    import torch
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    import numpy as np
+
+    import paper_2607_24981_gb300 as ilw
+    from paper_2607_24981_gb300 import synth
+
+    ilw.lib()
+    cfg, pe, blocks = build_host_params()
+    B, T, L = cfg["B"], cfg["T"], cfg["layers"]
+    units_per_step = L * B * T
+    dev = torch.device("cuda", local)
+    bb = ilw.Backbone(pe, blocks, B, device=dev)
+    img_h = synth.image_input(SEED + rank, B)
+    img = torch.from_numpy(img_h).to(dev)
+    inst = Instrumented(bb, torch)
+
+    # the instrumented sequence and the public Backbone.forward must agree bit for bit
+    ref_out = bb.forward(img).clone()
+    out = inst.forward(img)
+    torch.cuda.synchronize()
+    assert torch.equal(ref_out, out), "instrumented launch sequence differs from the public API path"
+    inst.records.clear()
+
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB L2
+
+    for _ in range(args.warmup):
+        inst.forward(img)
+    torch.cuda.synchronize()
+    inst.records.clear()
+
+    step_ms = []
+    barrier(world)
+    with ClockSampler(local) as clk:
+        for _ in range(args.steps):
+            flush.fill_(1)  # evict L2 between timed steps
+            s = torch.cuda.Event(enable_timing=True)
+            e = torch.cuda.Event(enable_timing=True)
+            s.record()
+            inst.forward(img)
+            e.record()
+            e.synchronize()
+            step_ms.append(s.elapsed_time(e))
+        torch.cuda.synchronize()
+    barrier(world)
+    ilw.device_status()
+    ms_local = statistics.mean(step_ms)
+    ms = max_over_ranks(ms_local, world)
+    value = world * units_per_step / (ms / 1000.0)
+
+    # per-kernel device times (average launch duration per class, over the timed region)
+    per = {}
+    for name, s, e, n in inst.records:
+        d_ms = s.elapsed_time(e)
+        tot, cnt, ln = per.get(name, (0.0, 0, 0))
+        per[name] = (tot + d_ms, cnt + 1, ln + n)
+    launches_per_step = sum(v[2] for v in per.values()) // args.steps
+    step_total = sum(v[0] for v in per.values())
+    work = kernel_work(cfg, B)
+    peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))) if os.path.exists(
+        os.path.join(ROOT, "MEASURED_PEAKS.json")) else {}
+    clocks = clk.summary()
+    kernels = {}
+    for name, (tot, cnt, _) in per.items():
+        avg_ms = tot / cnt
+        bound, w = work[name]
+        kernels[name] = {"share": tot / step_total, "avg_ms": avg_ms, "launches_per_step": cnt // args.steps,
+                         "bound": bound}
+        if bound == "tensor":
+            kernels[name]["tops"] = w / (avg_ms / 1000.0) / 1e12
+        elif bound == "hbm":
+            kernels[name]["gbs"] = w / (avg_ms / 1000.0) / 1e9
+        else:
+            kernels[name]["gscores_s"] = w / (avg_ms / 1000.0) / 1e9
+    dom = max(per, key=lambda k: per[k][0])
+    roofline = roofline_entry(dom, kernels[dom], work[dom], peaks, clocks)
+
+    # end to end through the public API: pinned host image -> device, backbone, result -> host
+    pin_in = torch.from_numpy(img_h).pin_memory()
+    pin_out = torch.empty((B * T, cfg["d"]), dtype=torch.int16).pin_memory()
+    dimg = torch.empty_like(img)
+    e2e_ms = []
+    for i in range(args.warmup + args.steps):
+        flush.fill_(1)
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record()
+        dimg.copy_(pin_in, non_blocking=True)
+        y = bb.forward(dimg)
+        pin_out.copy_(y, non_blocking=True)
+        e.record()
+        e.synchronize()
+        if i >= args.warmup:
+            e2e_ms.append(s.elapsed_time(e))
+    assert np.array_equal(pin_out.numpy(), ref_out.cpu().numpy())
+    e2e_t = max_over_ranks(statistics.mean(e2e_ms), world)
+    e2e = {"value": world * units_per_step / (e2e_t / 1000.0), "unit": UNIT,
+           "h2d_bytes_per_step": int(pin_in.numel()), "d2h_bytes_per_step": int(pin_out.numel() * 2)}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = run_cpu_sample(cfg, pe, blocks)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+            "config": {"workload": "medium_c2: Medium integer ViT backbone (patch embed + 10 blocks)",
+                       "B": B, "T": T, "d": cfg["d"], "H": cfg["H"], "F": cfg["F"], "blocks": L,
+                       "global_layers": list(cfg["global_layers"]), "window": "2x2 windows of 400 tokens",
+                       "image": "640x640 int8, 16x16 patches", "per_gpu_batch": B,
+                       "units": "block-tokens = blocks x images x tokens per step",
+                       "l2": "flushed between timed steps (256 MB write)", "parallelism": f"replicas x{world}"},
+            "clocks": clocks, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
+            "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+def roofline_entry(name, k, work, peaks, clocks):
+    bound, w = work
+    avg_s = k["avg_ms"] / 1000.0
+    if bound == "hbm":
+        peak = peaks.get("hbm_gbs")
+        src = "measured" if peak else "fallback"
+        peak = peak or 6800.0
+        a = w / avg_s / 1e9
+        return {"kernel": name, "bound": "hbm", "achieved": a, "peak": peak, "unit": "GB/s", "frac": a / peak,
+                "traffic": None, "peak_source": src}
+    if bound == "tensor":
+        peak = peaks.get("bf16_tflops_sustained")
+        src = "measured bf16 sustained (same rate as fp16 kind::f16)" if peak else "fallback"
+        peak = peak or 1700.0
+        a = w / avg_s / 1e12
+        return {"kernel": name, "bound": "tensor", "achieved": a, "peak": peak, "unit": "TFLOP/s",
+                "frac": a / peak, "traffic": None, "peak_source": src}
+    # ALU: integer ops per score (minimum the method needs with ShiftExp evaluated once per score:
+    # max 1, ShiftExp 12, sum 1, output multiply+shift 2) against SMs x 128 lanes x SM clock
+    ops_per_score = 16.0
+    mhz = clocks.get("sm_mhz") or 1500.0
+    peak = 152 * 128 * mhz * 1e6 / 1e12
+    a = w * ops_per_score / avg_s / 1e12
+    return {"kernel": name, "bound": "alu", "achieved": a, "peak": peak, "unit": "Tops/s", "frac": a / peak,
+            "traffic": None, "peak_source": f"derived: 152 SMs x 128 int32 lanes x {mhz:.0f} MHz (median SM clock)",
+            "ops_per_score": ops_per_score}
+
+
+if __name__ == "__main__":
+    main()

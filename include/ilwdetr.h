@@ -1,0 +1,228 @@
+/*
+ * ilwdetr.h -- C-ABI of the GB300 (sm_103a) integer-only I-LW-DETR forward path.
+ *
+ * Every entry point computes one integer operator of "Enabling Fully Integer-Only Inference for
+ * Lightweight Detection Transformers" exactly (bit for bit) as the paper defines it; the
+ * passages are cited beside each declaration.  All arithmetic on the device is integer.
+ *
+ * Conventions (apply to every call unless a declaration says otherwise)
+ *   - Pointers to tensors are DEVICE pointers owned by the caller; the library never frees or
+ *     keeps them.  Arrays described as "host" are read during the call only.
+ *   - Layouts are row-major with an explicit leading dimension (elements between rows).
+ *   - Every call is asynchronous on `stream` (0 = the legacy default stream) and returns an
+ *     int status: ILW_OK, or a negative ILW_ERR_* code with a message available from
+ *     ilwdetr_last_error() (thread-local).  Argument errors are reported before anything is
+ *     launched.  Device-side failures that the kernels detect (a bounded wait that ran out)
+ *     are latched in a device status word and reported by ilwdetr_device_status().
+ *   - rq(v; m, s) = (v*m + 2^(s-1)) >> s, arithmetic shift (dyadic requantisation, Sec. 3.2.2,
+ *     round half up); satN clips to the symmetric range [-(2^(N-1)-1), 2^(N-1)-1] (Sec. 3.2.1).
+ *     Per-channel `mult` is int32 (sign allowed), `shift` is int32 in [1, 62]; values outside
+ *     that domain give unspecified results.
+ *   - The caller passes integer parameters only (I0 = round(1/S), dyadic pairs, shifts): the
+ *     float scales of calibration never reach the device.
+ */
+#ifndef ILWDETR_H
+#define ILWDETR_H
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *ilw_stream_t; /* identical to cudaStream_t */
+
+enum {
+    ILW_OK = 0,
+    ILW_ERR_INVALID_ARG = -1, /* null / misaligned pointer, bad size, parameter out of domain */
+    ILW_ERR_UNSUPPORTED = -2, /* valid but outside what the kernels implement (e.g. head dim) */
+    ILW_ERR_CUDA = -3,        /* a CUDA runtime call or launch failed */
+    ILW_ERR_TIMEOUT = -4      /* a kernel's bounded wait expired (see ilwdetr_device_status) */
+};
+
+/* Library version string, e.g. "ilwdetr 0.1 sm_103a". */
+const char *ilwdetr_version(void);
+/* Message of the last failing call on this thread ("" if none). */
+const char *ilwdetr_last_error(void);
+/* Synchronises `stream`, then reads and clears the device status word of the current device:
+ * ILW_OK, or ILW_ERR_TIMEOUT if a kernel gave up a bounded wait since the last read. */
+int ilwdetr_device_status(ilw_stream_t stream);
+
+/* Constrained Shiftmax parameters (Algorithm 2 inputs; Sec. 3.3.2).
+ *   I0      round(1/S_x) of the score scale, 1 <= I0 < 2^15 (ShiftExp, Algorithm 1)
+ *   k_inter intermediate precision, 0 <= k_inter <= 16, I0 * 2^k_inter < 2^31
+ *   k_out   output bits, 1 <= k_out <= 8 (outputs are u8 with scale 2^-(k_out-1))
+ *   s_d     < 0: per-row CalibrateShift (Algorithm 2); >= 0: static shift (<= 31)
+ *   m_p     precision margin (the paper uses 4); M_hw hardware division precision (31) */
+typedef struct {
+    int32_t I0, k_inter, k_out, s_d, m_p, M_hw;
+} ilw_shiftmax_t;
+
+/* SD-ShiftGELU parameters (Algorithm 1 inputs; Sec. 3.3.1).  1 <= I0, I0 * 2^(k_inter+1) < 2^31,
+ * 1 <= k_out <= 8. */
+typedef struct {
+    int32_t I0, k_inter, k_out;
+} ilw_gelu_t;
+
+/* Residual term of a two-term requantised sum: out = sat(rq(acc) + rq(x[row % rows]; mult, shift)).
+ * x is an int16 device tensor [rows, >= N] with leading dimension ldx. */
+typedef struct {
+    const int16_t *x;
+    int64_t ldx;
+    int64_t rows;
+    int32_t mult, shift;
+} ilw_residual_t;
+
+/* ------------------------------------------------------------------ integer linear layers */
+
+/* Bytes of the packed form of an int8 weight W[N, K] (row-major, K contiguous). */
+size_t ilwdetr_packed_weight_bytes(int32_t N, int32_t K);
+/* Packs W (device, int8 [N, K], leading dimension K) into `packed` (device, bytes given by
+ * ilwdetr_packed_weight_bytes).  Done once per weight; the values stay the same integers.
+ * K must be a multiple of 16. */
+int ilwdetr_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, ilw_stream_t stream);
+
+/* Integer linear layer with fused bias and dyadic requantisation (Sec. 3.2.1, the equation
+ * Y ~ S_x S_w (I_x I_w) + b: the MAC is integer, the scale is applied after accumulation).
+ *   A      int8 [M, K] (lda >= K, lda and the base 16-byte aligned)
+ *   Wp     packed weight of W int8 [N, K]
+ *   acc[i,c] = sum_k A[i,k] W[c,k] + bias[c]      (exact; must fit int32)
+ *   out_bits 8 / 16: C[i,c] = satN(rq(acc; mult[c], shift[c]) [+ rq(res...)]) (int8 / int16)
+ *   out_bits 32    : C[i,c] = acc (int32; mult, shift and res ignored and may be NULL)
+ *   bias may be NULL (0).  C has leading dimension ldc (elements). */
+int ilwdetr_gemm_requant(const int8_t *A, int64_t lda, const void *Wp, const int32_t *bias,
+                         const int32_t *mult, const int32_t *shift, int32_t M, int32_t N,
+                         int32_t K, int32_t out_bits, void *C, int64_t ldc,
+                         const ilw_residual_t *res /* nullable, host struct */,
+                         ilw_stream_t stream);
+
+/* Integer linear layer followed by SD-ShiftGELU (Sec. 3.3.1, Algorithm 1) in the epilogue:
+ *   g = sat16(rq(acc; mult[c], shift[c]));  I_out = g * I_div(g)  (Algorithm 1, scale 2^-(k_out-1))
+ *   H[i,c] = sat8(rq(I_out; m_g, s_g))  (int8, leading dimension ldh). */
+int ilwdetr_gemm_gelu(const int8_t *A, int64_t lda, const void *Wp, const int32_t *bias,
+                      const int32_t *mult, const int32_t *shift, int32_t M, int32_t N, int32_t K,
+                      const ilw_gelu_t *gelu, int32_t m_g, int32_t s_g, int8_t *H, int64_t ldh,
+                      ilw_stream_t stream);
+
+/* Scale-preserving split convolution (Sec. 3.2.2, Fig. 2(b)), 1x1 kernels (a per-pixel GEMM):
+ *   y[i,c] = sat8(rq( sum_b rq(X_b[i,:] . W_b[c,:]; m_b[b], s_b[b]) + bias[c]; mult[c], shift[c] ))
+ * Each branch keeps its own activation scale; (m_b, s_b) is the dyadic ratio S_b / max_b S_b
+ * (must satisfy m_b <= 2^s_b).  X, ldx, Kb, Wp, m_b, s_b are HOST arrays of nb entries holding
+ * device pointers / values; 1 <= nb <= 8, every K_b a multiple of 16. */
+int ilwdetr_split_conv(const int8_t *const *X, const int64_t *ldx, int32_t nb, int32_t M,
+                       const int32_t *Kb, const void *const *Wp, const int32_t *m_b,
+                       const int32_t *s_b, const int32_t *bias, const int32_t *mult,
+                       const int32_t *shift, int32_t N, int8_t *Y, int64_t ldy,
+                       ilw_stream_t stream);
+
+/* ------------------------------------------------------------------ nonlinear operators */
+
+/* Constrained Shiftmax over rows (Algorithm 2; Sec. 3.3.2): X int32 [rows, len] (ldx) ->
+ * P u8 [rows, len] (ldp), scale 2^-(k_out-1).  Per row: max, ShiftExp of the differences,
+ * S_sum (int64), s_d, the exact shifted denominator S_R = floor(S_sum / 2^s_d) (quotient-
+ * remainder accumulation), F = floor((2^31-1)/clamp(S_R,1,2^31-1)), out = (I_exp F) >> (32-k_out+s_d). */
+int ilwdetr_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, int32_t len,
+                          const ilw_shiftmax_t *p, uint8_t *P, int64_t ldp, ilw_stream_t stream);
+
+/* SD-ShiftGELU (Algorithm 1; Sec. 3.3.1), element-wise: Y[i] = X[i] * I_div(X[i]) (int32, scale
+ * S_x 2^-(k_out-1)); IntDiv is Algorithm 2's fixed-point division with s_d = 0.
+ * Values must satisfy |X[i]| * 2^(k_out-1) < 2^31. */
+int ilwdetr_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const ilw_gelu_t *p,
+                        ilw_stream_t stream);
+
+/* I-LayerNorm (Sec. 3.3: I-ViT's integer LayerNorm with a Newton integer square root; 10
+ * iterations in the encoder, 20 in the decoder).  Per row of C values:
+ *   mu = floor((2 sum x + C) / (2C)); y = x - mu; V = sum y^2; R = Newton(V) from 2^16, `iters`
+ *   steps; F = floor((2^31-1)/max(R,1)); n = (y F) >> 1; out = sat_{out_bits}(rq(n + beta[c];
+ *   mult[c], shift[c])).
+ *   X: in_bits 16 (int16) or 32 (int32, |x| < 2^24), [rows, C] with leading dimension ldx.
+ *   Y: out_bits 8 (int8) or 16 (int16), leading dimension ldy.  1 <= C <= 4096. */
+int ilwdetr_int_layernorm(const void *X, int32_t in_bits, int64_t ldx, int64_t rows, int32_t C,
+                          const int32_t *beta, const int32_t *mult, const int32_t *shift,
+                          int32_t iters, void *Y, int32_t out_bits, int64_t ldy,
+                          ilw_stream_t stream);
+
+/* ------------------------------------------------------------------ attention */
+
+/* Multi-head attention with Constrained Shiftmax (Sec. 3.2.1 integer MatMul, Sec. 3.3.2):
+ *   scores = q k^T (int32; 1/sqrt(dh) is folded into the score scale, hence into p->I0),
+ *   P = ConstrainedShiftmax(scores) (u8), O = P V (int32), out = sat8(rq(O; m_o, s_o)).
+ * Q, K, V: token-major int8, element (b, t, h, e) at [(b*T + t) * ld_qkv + h*dh + e]
+ * (16-byte aligned rows; q|k|v of one [B*T, 3*H*dh] buffer is the usual case).
+ * O: int8, element (b, t, h, e) at [(b*T + t) * ld_o + h*dh + e].
+ * win_side <= 1: global attention over the T tokens; win_side = n >= 2: the sqrt(T) x sqrt(T)
+ * token grid (row-major) is cut into n x n windows and tokens attend within their window
+ * (LW-DETR's window attention, Table 1).  dh must be 32 or 64. */
+int ilwdetr_shiftmax_attn(const int8_t *Q, const int8_t *K, const int8_t *V, int64_t ld_qkv,
+                          int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side,
+                          const ilw_shiftmax_t *p, int32_t m_o, int32_t s_o, int8_t *O,
+                          int64_t ld_o, ilw_stream_t stream);
+
+/* Integer deformable-attention sampling with nearest-neighbour lookup (Sec. 3.1.1): for each
+ * (b, q, h) and sample (l, p): loc = ((ref * W_l) >> 8) + off (Q8 pixels), index = loc >> 8
+ * (the nearest grid point, pixel centres at i + 1/2); samples outside the map contribute 0;
+ * acc = sum w * value (int32); out = sat8(rq(acc; m, s)).
+ *   value   int8 [B, S_total, H*dh], levels concatenated row-major (S_total = sum H_l W_l)
+ *   level_hw HOST int32 [L, 2] = (H_l, W_l); 1 <= L <= 8
+ *   ref_q16 int32 [B, Q, 2] = (x, y) in [0, 2^16) of the map; off_q8 int32 [B, Q, H, L, P, 2]
+ *   w       u8 [B, Q, H, L*P] (Shiftmax outputs over the L*P samples)
+ *   out     int8 [B, Q, H*dh].  dh must be a multiple of 4. */
+int ilwdetr_deform_attn(const int8_t *value, const int32_t *level_hw, int32_t L,
+                        const int32_t *ref_q16, const int32_t *off_q8, const uint8_t *w,
+                        int32_t B, int32_t Q, int32_t H, int32_t P, int32_t dh, int32_t m,
+                        int32_t s, int8_t *out, ilw_stream_t stream);
+
+/* ------------------------------------------------------------------ patch embedding */
+
+/* Workspace bytes of ilwdetr_patch_embed (the gathered patch matrix, B*T x Cin*p*p int8). */
+size_t ilwdetr_patch_embed_workspace_bytes(int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p);
+/* ViT patch embedding: a p x p convolution with stride p of the int8 image (an integer linear
+ * layer on each non-overlapping patch, Sec. 3.2.1; Table 10 maps it to CONV_2D):
+ *   x0[b*T + t, c] = sat16(rq(acc; mult[c], shift[c]) + rq(pos[t, c]; m_pos, s_pos)),
+ *   acc = bias[c] + sum_{ch,ky,kx} W[c, (ch*p + ky)*p + kx] img[b, ch, py*p + ky, px*p + kx],
+ *   t = py*(Ww/p) + px, T = (Hh/p)(Ww/p).
+ *   img  int8 [B, Cin, Hh, Ww] (NCHW, 16-byte aligned), Ww and p multiples of 16, p | Hh, p | Ww
+ *   Wp   packed weight of W int8 [d, Cin*p*p];  pos int16 [T, d] or NULL
+ *   x0   int16 [B*T, d];  workspace: >= ilwdetr_patch_embed_workspace_bytes, 256-byte aligned */
+int ilwdetr_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
+                        const void *Wp, const int32_t *bias, const int32_t *mult, const int32_t *shift,
+                        int32_t d, const int16_t *pos, int32_t m_pos, int32_t s_pos, int16_t *x0,
+                        void *workspace, size_t workspace_bytes, ilw_stream_t stream);
+
+/* ------------------------------------------------------------------ encoder block */
+
+/* Integer parameters of one encoder block (all pointers are device pointers; weights packed
+ * with ilwdetr_pack_weight).  The block computes (a reading of LW-DETR's plain ViT block with
+ * the paper's integer operators):
+ *   a1 = LN1(x) (int8); qkv = sat8(rq(a1 Wqkv^T + b)) (token-major q|k|v);
+ *   O = Attention(q, k, v) (int8); x1 = sat16(rq(O Wproj^T + b) + rq(x; m_r1, s_r1));
+ *   a2 = LN2(x1); g = sat16(rq(a2 W1^T + b)); h = sat8(rq(g * I_div(g); m_g, s_g));
+ *   y = sat16(rq(h W2^T + b) + rq(x1; m_r2, s_r2)). */
+typedef struct {
+    uint32_t struct_size; /* sizeof(ilw_block_params_t) */
+    int32_t d, H, F, win_side, ln_iters;
+    const int32_t *ln1_beta, *ln1_mult, *ln1_shift;
+    const int32_t *ln2_beta, *ln2_mult, *ln2_shift;
+    const void *w_qkv; const int32_t *b_qkv, *m_qkv, *s_qkv;
+    ilw_shiftmax_t smx;
+    int32_t m_o, s_o;
+    const void *w_proj; const int32_t *b_proj, *m_proj, *s_proj;
+    int32_t m_r1, s_r1;
+    const void *w_fc1; const int32_t *b_fc1, *m_fc1, *s_fc1;
+    ilw_gelu_t gelu;
+    int32_t m_g, s_g;
+    const void *w_fc2; const int32_t *b_fc2, *m_fc2, *s_fc2;
+    int32_t m_r2, s_r2;
+} ilw_block_params_t;
+
+/* Workspace bytes ilwdetr_block_forward needs for B*T tokens. */
+size_t ilwdetr_block_workspace_bytes(int32_t B, int32_t T, int32_t d, int32_t F);
+/* One encoder block: x int16 [B*T, d] -> y int16 [B*T, d] (x and y may not alias).
+ * `workspace` is a device buffer of at least ilwdetr_block_workspace_bytes (256-byte aligned). */
+int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t *y, int32_t B,
+                          int32_t T, void *workspace, size_t workspace_bytes, ilw_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

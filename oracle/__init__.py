@@ -102,6 +102,10 @@ def lib():
                                        C.c_int64, C.c_int64, C.c_int64, C.c_int32,
                                        i16p, C.c_int64, C.c_int64, C.c_int32, C.c_int32,
                                        i32p, C.c_int64]
+        L.orc_patch_embed.restype = C.c_int
+        L.orc_patch_embed.argtypes = [i8p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
+                                      i8p, i32p, i32p, i32p, C.c_int32, i16p, C.c_int32,
+                                      C.c_int32, i16p]
         L.orc_attention.restype = C.c_int
         L.orc_attention.argtypes = [i8p, i8p, i8p, C.c_int64, C.c_int32, C.c_int32, C.c_int32,
                                     C.c_int32, C.c_int32, C.POINTER(ShiftmaxParams), C.c_int32,
@@ -226,6 +230,28 @@ def gemm_requant(A: np.ndarray, W: np.ndarray, bias, mult, shift, out_bits: int 
                                   _p(shift, i32p), M, N, K, out_bits, rp, ldr, rrows, m_r, s_r,
                                   _p(Cm, i32p), N), "gemm_requant")
     return Cm
+
+
+def patch_embed(img: np.ndarray, p: int, W: np.ndarray, bias, mult, shift,
+                pos: np.ndarray | None = None, m_pos: int = 0, s_pos: int = 0) -> np.ndarray:
+    """p x p stride-p integer convolution of int8 img [B, C, H, W] -> int16 [B*T, d]."""
+    img = np.ascontiguousarray(img, dtype=np.int8)
+    B, Cin, Hh, Ww = img.shape
+    W = np.ascontiguousarray(W, dtype=np.int8)
+    d = W.shape[0]
+    bias = np.ascontiguousarray(bias, dtype=np.int32)
+    mult = np.ascontiguousarray(mult, dtype=np.int32)
+    shift = np.ascontiguousarray(shift, dtype=np.int32)
+    T = (Hh // p) * (Ww // p)
+    x0 = np.empty((B * T, d), dtype=np.int16)
+    pp = None
+    if pos is not None:
+        pos = np.ascontiguousarray(pos, dtype=np.int16)
+        pp = _p(pos, i16p)
+    _check(lib().orc_patch_embed(_p(img, i8p), B, Cin, Hh, Ww, p, _p(W, i8p), _p(bias, i32p),
+                                 _p(mult, i32p), _p(shift, i32p), d, pp, m_pos, s_pos,
+                                 _p(x0, i16p)), "patch_embed")
+    return x0
 
 
 def attention(qkv: np.ndarray, B: int, T: int, H: int, dh: int, win_side: int, smx: dict,

@@ -240,6 +240,37 @@ int orc_gemm_requant(const int8_t *A, int64_t lda, const int8_t *W, int64_t ldw,
     return 0;
 }
 
+// Patch embedding of the ViT encoder (Table 1: 640x640 input, 16x16 patches -> 1600 tokens):
+// an integer convolution with kernel = stride = p (Sec. 3.2.1: integer MAC, scale after
+// accumulation; Table 10 maps it to CONV_2D), written as the direct convolution sum.  The
+// position term is a second requantised addend (the same two-term form as the residuals).
+int orc_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
+                    const int8_t *W, const int32_t *bias, const int32_t *mult, const int32_t *shift,
+                    int32_t d, const int16_t *pos, int32_t m_pos, int32_t s_pos, int16_t *x0) {
+    if (p < 1 || Hh % p || Ww % p) return -1;
+    const int32_t Gh = Hh / p, Gw = Ww / p, T = Gh * Gw, Kc = Cin * p * p;
+    for (int32_t b = 0; b < B; ++b) {
+        for (int32_t py = 0; py < Gh; ++py) {
+            for (int32_t px = 0; px < Gw; ++px) {
+                const int32_t t = py * Gw + px;
+                for (int32_t c = 0; c < d; ++c) {
+                    int64_t acc = bias ? bias[c] : 0;
+                    for (int32_t ch = 0; ch < Cin; ++ch)
+                        for (int32_t ky = 0; ky < p; ++ky)
+                            for (int32_t kx = 0; kx < p; ++kx)
+                                acc += (int64_t)W[(int64_t)c * Kc + (ch * p + ky) * p + kx] *
+                                       img[(((int64_t)b * Cin + ch) * Hh + py * p + ky) * Ww + px * p + kx];
+                    if (acc < INT32_MIN || acc > INT32_MAX) return -2;
+                    int64_t v = orc_rq(acc, mult[c], shift[c]);
+                    if (pos) v += orc_rq(pos[(int64_t)t * d + c], m_pos, s_pos);
+                    x0[((int64_t)b * T + t) * d + c] = (int16_t)orc_sat(v, 16);
+                }
+            }
+        }
+    }
+    return 0;
+}
+
 // Multi-head attention with Constrained Shiftmax.  Scores are the integer q.k^T (the 1/sqrt(dh)
 // factor lives in the score scale, hence in I0); P = ConstrainedShiftmax(scores) (u8, scale
 // 2^-(k_out-1)); O = P.V accumulated in int64, O8 = sat8(rq(O; m_o, s_o)).

@@ -107,6 +107,15 @@ int orc_gemm_requant(const int8_t *A, int64_t lda, const int8_t *W, int64_t ldw,
                      const int16_t *res, int64_t ldr, int64_t res_rows, int32_t m_r, int32_t s_r,
                      int32_t *C, int64_t ldc);
 
+/* Patch embedding: a p x p, stride-p integer convolution of the int8 image (NCHW), bias and
+ * per-channel requantisation, plus the requantised position term, saturated to 16 bits:
+ *   x0[b*T + t, c] = sat16(rq(acc; mult[c], shift[c]) + rq(pos[t, c]; m_pos, s_pos)),
+ *   acc = bias[c] + sum_{ch,ky,kx} W[c, ch*p*p + ky*p + kx] * img[b, ch, py*p + ky, px*p + kx],
+ * t = py * (Ww/p) + px.  pos may be NULL. */
+int orc_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
+                    const int8_t *W, const int32_t *bias, const int32_t *mult, const int32_t *shift,
+                    int32_t d, const int16_t *pos, int32_t m_pos, int32_t s_pos, int16_t *x0);
+
 /* Multi-head attention on token-major q, k, v ([B*T, ld], head h at columns h*dh..h*dh+dh-1). */
 int orc_attention(const int8_t *Q, const int8_t *K, const int8_t *V, int64_t ld,
                   int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side,

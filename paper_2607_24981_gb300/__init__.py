@@ -1,0 +1,382 @@
+"""GB300 (sm_103a) integer-only I-LW-DETR forward path.
+
+Python names mirror the C-ABI of ``include/ilwdetr.h`` (``libilwdetr.so`` in this directory).
+This module only marshals arguments: torch tensors provide device memory and the current CUDA
+stream; every step of the computation runs in the library's CUDA kernels.  There is no CPU
+fallback: if the library is missing or cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+__all__ = [
+    "lib", "IlwError", "version", "pack_weight", "gemm_requant", "gemm_gelu", "split_conv",
+    "shiftmax_rows", "sdshiftgelu", "int_layernorm", "shiftmax_attn", "deform_attn",
+    "BlockWeights", "block_forward", "block_workspace_bytes", "device_status",
+    "patch_embed", "patch_embed_workspace_bytes", "Backbone",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libilwdetr.so")
+_lib = None
+
+
+class IlwError(RuntimeError):
+    pass
+
+
+class ShiftmaxT(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in ("I0", "k_inter", "k_out", "s_d", "m_p", "M_hw")]
+
+
+class GeluT(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in ("I0", "k_inter", "k_out")]
+
+
+class ResidualT(C.Structure):
+    _fields_ = [("x", C.c_void_p), ("ldx", C.c_int64), ("rows", C.c_int64),
+                ("mult", C.c_int32), ("shift", C.c_int32)]
+
+
+class BlockParamsT(C.Structure):
+    _fields_ = [
+        ("struct_size", C.c_uint32),
+        ("d", C.c_int32), ("H", C.c_int32), ("F", C.c_int32), ("win_side", C.c_int32),
+        ("ln_iters", C.c_int32),
+        ("ln1_beta", C.c_void_p), ("ln1_mult", C.c_void_p), ("ln1_shift", C.c_void_p),
+        ("ln2_beta", C.c_void_p), ("ln2_mult", C.c_void_p), ("ln2_shift", C.c_void_p),
+        ("w_qkv", C.c_void_p), ("b_qkv", C.c_void_p), ("m_qkv", C.c_void_p), ("s_qkv", C.c_void_p),
+        ("smx", ShiftmaxT), ("m_o", C.c_int32), ("s_o", C.c_int32),
+        ("w_proj", C.c_void_p), ("b_proj", C.c_void_p), ("m_proj", C.c_void_p), ("s_proj", C.c_void_p),
+        ("m_r1", C.c_int32), ("s_r1", C.c_int32),
+        ("w_fc1", C.c_void_p), ("b_fc1", C.c_void_p), ("m_fc1", C.c_void_p), ("s_fc1", C.c_void_p),
+        ("gelu", GeluT), ("m_g", C.c_int32), ("s_g", C.c_int32),
+        ("w_fc2", C.c_void_p), ("b_fc2", C.c_void_p), ("m_fc2", C.c_void_p), ("s_fc2", C.c_void_p),
+        ("m_r2", C.c_int32), ("s_r2", C.c_int32),
+    ]
+
+
+# C signatures (argtypes, restype) of every export declared in include/ilwdetr.h
+_VP, _I32, _I64 = C.c_void_p, C.c_int32, C.c_int64
+SIGNATURES = {
+    "ilwdetr_version": ([], C.c_char_p),
+    "ilwdetr_last_error": ([], C.c_char_p),
+    "ilwdetr_device_status": ([_VP], C.c_int),
+    "ilwdetr_packed_weight_bytes": ([_I32, _I32], C.c_size_t),
+    "ilwdetr_pack_weight": ([_VP, _I32, _I32, _VP, _VP], C.c_int),
+    "ilwdetr_gemm_requant": ([_VP, _I64, _VP, _VP, _VP, _VP, _I32, _I32, _I32, _I32, _VP, _I64,
+                              C.POINTER(ResidualT), _VP], C.c_int),
+    "ilwdetr_gemm_gelu": ([_VP, _I64, _VP, _VP, _VP, _VP, _I32, _I32, _I32, C.POINTER(GeluT),
+                           _I32, _I32, _VP, _I64, _VP], C.c_int),
+    "ilwdetr_split_conv": ([C.POINTER(_VP), C.POINTER(_I64), _I32, _I32, C.POINTER(_I32),
+                            C.POINTER(_VP), C.POINTER(_I32), C.POINTER(_I32), _VP, _VP, _VP, _I32,
+                            _VP, _I64, _VP], C.c_int),
+    "ilwdetr_shiftmax_rows": ([_VP, _I64, _I64, _I32, C.POINTER(ShiftmaxT), _VP, _I64, _VP], C.c_int),
+    "ilwdetr_sdshiftgelu": ([_VP, _VP, _I64, C.POINTER(GeluT), _VP], C.c_int),
+    "ilwdetr_int_layernorm": ([_VP, _I32, _I64, _I64, _I32, _VP, _VP, _VP, _I32, _VP, _I32, _I64,
+                               _VP], C.c_int),
+    "ilwdetr_shiftmax_attn": ([_VP, _VP, _VP, _I64, _I32, _I32, _I32, _I32, _I32,
+                               C.POINTER(ShiftmaxT), _I32, _I32, _VP, _I64, _VP], C.c_int),
+    "ilwdetr_deform_attn": ([_VP, C.POINTER(_I32), _I32, _VP, _VP, _VP, _I32, _I32, _I32, _I32,
+                             _I32, _I32, _I32, _VP, _VP], C.c_int),
+    "ilwdetr_patch_embed_workspace_bytes": ([_I32, _I32, _I32, _I32, _I32], C.c_size_t),
+    "ilwdetr_patch_embed": ([_VP, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _VP, _VP, _I32, _VP, _I32,
+                             _I32, _VP, _VP, C.c_size_t, _VP], C.c_int),
+    "ilwdetr_block_workspace_bytes": ([_I32, _I32, _I32, _I32], C.c_size_t),
+    "ilwdetr_block_forward": ([C.POINTER(BlockParamsT), _VP, _VP, _I32, _I32, _VP, C.c_size_t, _VP],
+                              C.c_int),
+}
+
+
+def lib():
+    """Load libilwdetr.so (raises IlwError if it is missing: there is no fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise IlwError(f"{LIB_PATH} is missing: build it with __graft_entry__.build()")
+        L = C.CDLL(LIB_PATH)
+        for name, (args, res) in SIGNATURES.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = L
+    return _lib
+
+
+def _check(rc: int, what: str) -> None:
+    if rc != 0:
+        msg = lib().ilwdetr_last_error().decode()
+        raise IlwError(f"{what} failed ({rc}): {msg}")
+
+
+def _stream():
+    import torch
+
+    return C.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _dev(t, dtype):
+    import torch
+
+    assert isinstance(t, torch.Tensor) and t.is_cuda and t.dtype == dtype, (t.dtype, dtype)
+    return t
+
+
+def version() -> str:
+    return lib().ilwdetr_version().decode()
+
+
+def device_status() -> None:
+    _check(lib().ilwdetr_device_status(_stream()), "device_status")
+
+
+# ---------------------------------------------------------------------------- linear layers
+def pack_weight(W):
+    """Pack an int8 [N, K] CUDA weight once (ilwdetr_pack_weight)."""
+    import torch
+
+    _dev(W, torch.int8)
+    N, K = W.shape
+    W = W.contiguous()
+    nbytes = lib().ilwdetr_packed_weight_bytes(N, K)
+    out = torch.empty(nbytes, dtype=torch.uint8, device=W.device)
+    _check(lib().ilwdetr_pack_weight(_ptr(W), N, K, _ptr(out), _stream()), "pack_weight")
+    return out
+
+
+def gemm_requant(A, Wp, N, bias, mult, shift, out_bits=8, res=None, m_r=0, s_r=0, out=None):
+    """ilwdetr_gemm_requant: A int8 [M, K] x packed W [N, K] -> int8/int16/int32 [M, N]."""
+    import torch
+
+    M, K = A.shape
+    dt = {8: torch.int8, 16: torch.int16, 32: torch.int32}[out_bits]
+    if out is None:
+        out = torch.empty((M, N), dtype=dt, device=A.device)
+    r = None
+    if res is not None:
+        r = ResidualT(res.data_ptr(), res.stride(0), res.shape[0], m_r, s_r)
+    _check(lib().ilwdetr_gemm_requant(_ptr(A), A.stride(0), _ptr(Wp), _ptr(bias), _ptr(mult),
+                                      _ptr(shift), M, N, K, out_bits, _ptr(out), out.stride(0),
+                                      None if r is None else C.byref(r), _stream()), "gemm_requant")
+    return out
+
+
+def gemm_gelu(A, Wp, N, bias, mult, shift, gelu: dict, m_g, s_g, out=None):
+    """ilwdetr_gemm_gelu: linear + SD-ShiftGELU epilogue -> int8 [M, N]."""
+    import torch
+
+    M, K = A.shape
+    if out is None:
+        out = torch.empty((M, N), dtype=torch.int8, device=A.device)
+    g = GeluT(gelu["I0"], gelu.get("k_inter", 16), gelu.get("k_out", 8))
+    _check(lib().ilwdetr_gemm_gelu(_ptr(A), A.stride(0), _ptr(Wp), _ptr(bias), _ptr(mult),
+                                   _ptr(shift), M, N, K, C.byref(g), m_g, s_g, _ptr(out),
+                                   out.stride(0), _stream()), "gemm_gelu")
+    return out
+
+
+def split_conv(Xs, Wps, N, m_b, s_b, bias, mult, shift, out=None):
+    """ilwdetr_split_conv over nb branches of int8 [M, K_b] with packed weights [N, K_b]."""
+    import torch
+
+    nb = len(Xs)
+    M = Xs[0].shape[0]
+    if out is None:
+        out = torch.empty((M, N), dtype=torch.int8, device=Xs[0].device)
+    xp = (C.c_void_p * nb)(*[x.data_ptr() for x in Xs])
+    ld = (C.c_int64 * nb)(*[x.stride(0) for x in Xs])
+    kb = (C.c_int32 * nb)(*[x.shape[1] for x in Xs])
+    wp = (C.c_void_p * nb)(*[w.data_ptr() for w in Wps])
+    mb = (C.c_int32 * nb)(*[int(v) for v in m_b])
+    sb = (C.c_int32 * nb)(*[int(v) for v in s_b])
+    _check(lib().ilwdetr_split_conv(xp, ld, nb, M, kb, wp, mb, sb, _ptr(bias), _ptr(mult),
+                                    _ptr(shift), N, _ptr(out), out.stride(0), _stream()),
+           "split_conv")
+    return out
+
+
+# ---------------------------------------------------------------------------- nonlinear ops
+def _smx(p: dict) -> ShiftmaxT:
+    return ShiftmaxT(p["I0"], p.get("k_inter", 16), p.get("k_out", 8), p.get("s_d", -1),
+                     p.get("m_p", 4), p.get("M_hw", 31))
+
+
+def shiftmax_rows(X, smx: dict, out=None):
+    """ilwdetr_shiftmax_rows: int32 [rows, len] -> u8 [rows, len]."""
+    import torch
+
+    rows, n = X.shape
+    if out is None:
+        out = torch.empty((rows, n), dtype=torch.uint8, device=X.device)
+    p = _smx(smx)
+    _check(lib().ilwdetr_shiftmax_rows(_ptr(X), X.stride(0), rows, n, C.byref(p), _ptr(out),
+                                       out.stride(0), _stream()), "shiftmax_rows")
+    return out
+
+
+def sdshiftgelu(X, gelu: dict, out=None):
+    """ilwdetr_sdshiftgelu: int32 -> int32 (x * I_div)."""
+    import torch
+
+    if out is None:
+        out = torch.empty_like(X)
+    g = GeluT(gelu["I0"], gelu.get("k_inter", 16), gelu.get("k_out", 8))
+    _check(lib().ilwdetr_sdshiftgelu(_ptr(X), _ptr(out), X.numel(), C.byref(g), _stream()),
+           "sdshiftgelu")
+    return out
+
+
+def int_layernorm(X, beta, mult, shift, iters=10, out_bits=8, out=None):
+    """ilwdetr_int_layernorm: int16/int32 [rows, C] -> int8/int16 [rows, C]."""
+    import torch
+
+    rows, Cn = X.shape
+    in_bits = {torch.int16: 16, torch.int32: 32}[X.dtype]
+    if out is None:
+        out = torch.empty((rows, Cn), dtype=torch.int8 if out_bits == 8 else torch.int16,
+                          device=X.device)
+    _check(lib().ilwdetr_int_layernorm(_ptr(X), in_bits, X.stride(0), rows, Cn, _ptr(beta),
+                                       _ptr(mult), _ptr(shift), iters, _ptr(out), out_bits,
+                                       out.stride(0), _stream()), "int_layernorm")
+    return out
+
+
+def shiftmax_attn(qkv, B, T, H, dh, win_side, smx: dict, m_o, s_o, out=None):
+    """ilwdetr_shiftmax_attn on a token-major [B*T, 3*H*dh] int8 q|k|v buffer -> [B*T, H*dh]."""
+    import torch
+
+    d = H * dh
+    if out is None:
+        out = torch.empty((B * T, d), dtype=torch.int8, device=qkv.device)
+    base = qkv.data_ptr()
+    p = _smx(smx)
+    _check(lib().ilwdetr_shiftmax_attn(C.c_void_p(base), C.c_void_p(base + d), C.c_void_p(base + 2 * d),
+                                       qkv.stride(0), B, T, H, dh, win_side, C.byref(p), m_o, s_o,
+                                       _ptr(out), out.stride(0), _stream()), "shiftmax_attn")
+    return out
+
+
+def deform_attn(value, level_hw, ref_q16, off_q8, w, m, s, out=None):
+    """ilwdetr_deform_attn: value int8 [B,S,H*dh]; ref int32 [B,Q,2]; off int32 [B,Q,H,L,P,2];
+    w u8 [B,Q,H,L*P] -> int8 [B,Q,H*dh]."""
+    import torch
+
+    B, S, Dm = value.shape
+    _, Q, H, L, P, _ = off_q8.shape
+    dh = Dm // H
+    if out is None:
+        out = torch.empty((B, Q, Dm), dtype=torch.int8, device=value.device)
+    hw = [int(v) for pair in level_hw for v in pair]
+    arr = (C.c_int32 * len(hw))(*hw)
+    _check(lib().ilwdetr_deform_attn(_ptr(value), arr, L, _ptr(ref_q16), _ptr(off_q8), _ptr(w), B,
+                                     Q, H, P, dh, m, s, _ptr(out), _stream()), "deform_attn")
+    return out
+
+
+# ---------------------------------------------------------------------------- encoder block
+class BlockWeights:
+    """Device copies of one block's integer parameters (from a dict of numpy arrays / ints, as
+    produced by ``synth.block_params``) plus its ilw_block_params_t."""
+
+    def __init__(self, bp: dict, device="cuda"):
+        import numpy as np
+        import torch
+
+        self.bp = bp
+        self.t = {}
+        for k, v in bp.items():
+            if isinstance(v, np.ndarray):
+                self.t[k] = torch.from_numpy(np.ascontiguousarray(v)).to(device)
+        for k in ("w_qkv", "w_proj", "w_fc1", "w_fc2"):
+            self.t[k + "_p"] = pack_weight(self.t[k])
+        s, T = bp["smx"], self.t
+        self.params = BlockParamsT(
+            C.sizeof(BlockParamsT), bp["d"], bp["H"], bp["F"], bp["win_side"], bp["ln_iters"],
+            T["ln1_beta"].data_ptr(), T["ln1_mult"].data_ptr(), T["ln1_shift"].data_ptr(),
+            T["ln2_beta"].data_ptr(), T["ln2_mult"].data_ptr(), T["ln2_shift"].data_ptr(),
+            T["w_qkv_p"].data_ptr(), T["b_qkv"].data_ptr(), T["m_qkv"].data_ptr(), T["s_qkv"].data_ptr(),
+            ShiftmaxT(s["I0"], s["k_inter"], s["k_out"], s["s_d"], s["m_p"], s["M_hw"]),
+            bp["m_o"], bp["s_o"],
+            T["w_proj_p"].data_ptr(), T["b_proj"].data_ptr(), T["m_proj"].data_ptr(), T["s_proj"].data_ptr(),
+            bp["m_r1"], bp["s_r1"],
+            T["w_fc1_p"].data_ptr(), T["b_fc1"].data_ptr(), T["m_fc1"].data_ptr(), T["s_fc1"].data_ptr(),
+            GeluT(bp["gelu_I0"], bp["gelu_k_inter"], bp["gelu_k_out"]), bp["m_g"], bp["s_g"],
+            T["w_fc2_p"].data_ptr(), T["b_fc2"].data_ptr(), T["m_fc2"].data_ptr(), T["s_fc2"].data_ptr(),
+            bp["m_r2"], bp["s_r2"],
+        )
+
+
+def block_workspace_bytes(B, T, d, F) -> int:
+    return int(lib().ilwdetr_block_workspace_bytes(B, T, d, F))
+
+
+def block_forward(bw: BlockWeights, x, B, T, workspace, out=None):
+    """ilwdetr_block_forward: int16 [B*T, d] -> int16 [B*T, d]."""
+    import torch
+
+    if out is None:
+        out = torch.empty_like(x)
+    _check(lib().ilwdetr_block_forward(C.byref(bw.params), _ptr(x), _ptr(out), B, T,
+                                       _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                       _stream()), "block_forward")
+    return out
+
+
+# ---------------------------------------------------------------------------- patch embedding
+def patch_embed_workspace_bytes(B, Cin, Hh, Ww, p) -> int:
+    return int(lib().ilwdetr_patch_embed_workspace_bytes(B, Cin, Hh, Ww, p))
+
+
+def patch_embed(img, p, Wp, d, bias, mult, shift, pos=None, m_pos=0, s_pos=0, workspace=None, out=None):
+    """ilwdetr_patch_embed: int8 image [B, C, H, W] -> int16 x0 [B*T, d]."""
+    import torch
+
+    B, Cin, Hh, Ww = img.shape
+    T = (Hh // p) * (Ww // p)
+    if workspace is None:
+        workspace = torch.empty(patch_embed_workspace_bytes(B, Cin, Hh, Ww, p), dtype=torch.uint8,
+                                device=img.device)
+    if out is None:
+        out = torch.empty((B * T, d), dtype=torch.int16, device=img.device)
+    _check(lib().ilwdetr_patch_embed(_ptr(img), B, Cin, Hh, Ww, p, _ptr(Wp), _ptr(bias), _ptr(mult),
+                                     _ptr(shift), d, _ptr(pos), m_pos, s_pos, _ptr(out),
+                                     _ptr(workspace), workspace.numel(), _stream()), "patch_embed")
+    return out
+
+
+class Backbone:
+    """The integer ViT encoder of one configuration on the device: patch embedding followed by
+    ``len(blocks)`` encoder blocks (each an ilwdetr_block_forward call), with its buffers."""
+
+    def __init__(self, pe: dict, blocks: list, B: int, img_hw=(640, 640), device="cuda"):
+        import numpy as np
+        import torch
+
+        self.B, self.p, self.hw = B, pe["p"], img_hw
+        self.d, self.F = blocks[0]["d"], blocks[0]["F"]
+        self.T = (img_hw[0] // self.p) * (img_hw[1] // self.p)
+        self.pe = {k: torch.from_numpy(np.ascontiguousarray(v)).to(device)
+                   for k, v in pe.items() if isinstance(v, np.ndarray)}
+        self.pe_s = pe
+        self.pe["w_p"] = pack_weight(self.pe["w"])
+        self.blocks = [BlockWeights(bp, device) for bp in blocks]
+        M = B * self.T
+        self.ws_pe = torch.empty(patch_embed_workspace_bytes(B, 3, img_hw[0], img_hw[1], self.p),
+                                 dtype=torch.uint8, device=device)
+        self.ws_blk = torch.empty(block_workspace_bytes(B, self.T, self.d, self.F), dtype=torch.uint8,
+                                  device=device)
+        self.x = [torch.empty((M, self.d), dtype=torch.int16, device=device) for _ in range(2)]
+
+    def forward(self, img):
+        """img int8 [B, 3, H, W] (device) -> x_L int16 [B*T, d] (a buffer owned by the backbone)."""
+        pe = self.pe
+        x = patch_embed(img, self.p, pe["w_p"], self.d, pe["b"], pe["m"], pe["s"], pe["pos"],
+                        self.pe_s["m_pos"], self.pe_s["s_pos"], self.ws_pe, self.x[0])
+        for i, bw in enumerate(self.blocks):
+            x = block_forward(bw, x, self.B, self.T, self.ws_blk, out=self.x[(i + 1) % 2])
+        return x

@@ -1,0 +1,124 @@
+// ilw_kernels.h -- internal launch interface between the C-ABI layer and the kernels.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "ilw_device.cuh"
+
+namespace ilw {
+
+// Host-side construction of the per-launch ShiftExp constants (Algorithm 1).
+inline ShiftExpC make_shiftexp(int32_t I0, int32_t k) {
+    ShiftExpC c;
+    c.I0 = I0;
+    c.kI0 = k * I0;
+    uint64_t M = (((uint64_t)1 << 40) + (uint64_t)I0 - 1) / (uint64_t)I0;  // ceil(2^40 / I0)
+    c.m_lo = (uint32_t)(M & 0xffffffffull);
+    c.m_hi = (uint32_t)(M >> 32);
+    c.k = k;
+    return c;
+}
+inline GeluC make_gelu(const ilw_gelu_t &g) {
+    GeluC c;
+    c.se = make_shiftexp(g.I0, g.k_inter);
+    c.out_sh = 31 - g.k_out + 1;
+    return c;
+}
+
+// ---------------------------------------------------------------- GEMM
+constexpr int kMaxBranches = 8;
+struct GemmBranch {
+    const int8_t *A;   // [M, K] row-major, lda
+    int64_t lda;
+    const int8_t *W;   // [N, K] row-major (ld = K)
+    const void *Wp;    // packed weight (tensor-core operand form)
+    int32_t K;
+    int32_t m_b, s_b;  // split-conv branch rescale (ignored for a plain GEMM)
+};
+struct GemmProblem {
+    int32_t M, N;
+    int32_t nb;        // branches; 1 = plain GEMM
+    bool branch_rq;    // rq each branch partial with (m_b, s_b) before the integer sum
+    GemmBranch br[kMaxBranches];
+};
+enum EpiKind { EPI_REQUANT = 0, EPI_GELU = 1 };
+struct EpiParams {
+    EpiKind kind;
+    const int32_t *bias, *mult, *shift;
+    int32_t out_bits;  // 8, 16, 32 (EPI_REQUANT)
+    void *C;
+    int64_t ldc;
+    // residual (EPI_REQUANT, out_bits 8/16)
+    const int16_t *res;
+    int64_t ldr, res_rows;
+    int32_t m_r, s_r;
+    // GELU (EPI_GELU): int8 output in C
+    GeluC gelu;
+    int32_t m_g, s_g;
+};
+
+// Packed weight layout: [int8 W, N*K bytes][pad to 256][fp16 W, N*K*2 bytes].
+size_t packed_weight_bytes(int32_t N, int32_t K);
+inline const int8_t *packed_i8(const void *p) { return (const int8_t *)p; }
+inline const void *packed_f16(const void *p, int32_t N, int32_t K) {
+    size_t off = (((size_t)N * K) + 255) & ~(size_t)255;
+    return (const char *)p + off;
+}
+cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, cudaStream_t s);
+cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s);
+
+// ---------------------------------------------------------------- row / element kernels
+struct ShiftmaxC {
+    ShiftExpC se;
+    int32_t s_d, m_p, M_hw, k_out;
+};
+cudaError_t launch_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, int32_t len,
+                                 const ShiftmaxC &c, uint8_t *P, int64_t ldp, cudaStream_t s);
+cudaError_t launch_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const GeluC &c, cudaStream_t s);
+struct LnParams {
+    const void *X;
+    int32_t in_bits;
+    int64_t ldx, rows;
+    int32_t C;
+    const int32_t *beta, *mult, *shift;
+    int32_t iters;
+    void *Y;
+    int32_t out_bits;
+    int64_t ldy;
+};
+cudaError_t launch_layernorm(const LnParams &p, cudaStream_t s);
+
+// ---------------------------------------------------------------- attention
+struct AttnParams {
+    const int8_t *Q, *K, *V;
+    int64_t ld_qkv;
+    int32_t B, T, H, dh;
+    int32_t nw;        // windows per side (1 = global)
+    int32_t grid_side; // sqrt(T) when nw > 1
+    ShiftmaxC smx;
+    int32_t m_o, s_o;
+    int8_t *O;
+    int64_t ld_o;
+};
+cudaError_t launch_attention(const AttnParams &p, cudaStream_t s);
+
+// ---------------------------------------------------------------- deformable sampling
+struct DeformParams {
+    const int8_t *value;
+    int32_t L;
+    int32_t lh[8], lw[8];
+    int64_t lstart[8];
+    int64_t S_total;
+    const int32_t *ref, *off;
+    const uint8_t *w;
+    int32_t B, Q, H, P, dh;
+    int32_t m, s;
+    int8_t *out;
+};
+cudaError_t launch_deform(const DeformParams &p, cudaStream_t s);
+
+// ---------------------------------------------------------------- patch embedding
+cudaError_t launch_patchify(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
+                            int8_t *A, cudaStream_t s);
+
+}  // namespace ilw

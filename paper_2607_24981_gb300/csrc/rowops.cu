@@ -1,0 +1,240 @@
+// rowops.cu -- bandwidth-bound integer nonlinearities: Constrained Shiftmax over rows
+// (Algorithm 2), SD-ShiftGELU (Algorithm 1) and I-LayerNorm (Sec. 3.3).
+//
+// One warp owns one row; the row stays in registers between the two dependent reductions, so
+// HBM sees each input byte once.  Rows are read with 128-bit loads when the layout allows.
+#include <climits>
+#include <cstdint>
+
+#include "ilw_kernels.h"
+
+namespace ilw {
+namespace {
+
+__device__ __forceinline__ int32_t warp_max(int32_t v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ uint64_t warp_sum_u64(uint64_t v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ int64_t warp_sum_i64(int64_t v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// ------------------------------------------------------------------ Constrained Shiftmax rows
+// NCH = 4-element chunks per lane (row length <= 128 * NCH); vector loads need len % 4 == 0
+// and 16-byte aligned rows.
+template <int NCH>
+__global__ void __launch_bounds__(256) shiftmax_rows_vec(const int32_t *__restrict__ X, int64_t ldx,
+                                                          int64_t rows, int32_t len, const ShiftmaxC c,
+                                                          uint8_t *__restrict__ P, int64_t ldp) {
+    const int lane = threadIdx.x & 31;
+    const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (row >= rows) return;
+    const int nch = len >> 2;
+    const int4 *xr = (const int4 *)(X + row * ldx);
+    int4 v[NCH];
+    int32_t mx = INT_MIN;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+        int ch = lane + 32 * j;
+        if (ch < nch) {
+            v[j] = __ldcs(xr + ch);
+            mx = max(mx, max(max(v[j].x, v[j].y), max(v[j].z, v[j].w)));
+        }
+    }
+    mx = warp_max(mx);
+    // differences below -2^30 are deep in ShiftExp's clamp region: use -2^30 there
+    const int32_t lowb = mx > INT_MIN + (1 << 30) ? mx - (1 << 30) : INT_MIN;
+    uint64_t sum = 0;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+        int ch = lane + 32 * j;
+        if (ch < nch) {
+            int32_t *e = (int32_t *)&v[j];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                int32_t d = e[q] > lowb ? e[q] - mx : -(1 << 30);
+                uint32_t ex = shift_exp(d, c.se);
+                e[q] = (int32_t)ex;
+                sum += ex;
+            }
+        }
+    }
+    sum = warp_sum_u64(sum);
+    const RowNorm rn = shiftmax_norm(sum, c.s_d, c.m_p, c.M_hw, c.k_out);
+    uint32_t *pr = (uint32_t *)(P + row * ldp);
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+        int ch = lane + 32 * j;
+        if (ch < nch) {
+            const int32_t *e = (const int32_t *)&v[j];
+            uint32_t o = shiftmax_out((uint32_t)e[0], rn) | (shiftmax_out((uint32_t)e[1], rn) << 8) |
+                         (shiftmax_out((uint32_t)e[2], rn) << 16) | (shiftmax_out((uint32_t)e[3], rn) << 24);
+            __stcs(pr + ch, o);
+        }
+    }
+}
+
+// Any length / alignment: three passes over the row from global memory (L1/L2 resident).
+__global__ void __launch_bounds__(256) shiftmax_rows_generic(const int32_t *__restrict__ X, int64_t ldx,
+                                                              int64_t rows, int32_t len, const ShiftmaxC c,
+                                                              uint8_t *__restrict__ P, int64_t ldp) {
+    const int lane = threadIdx.x & 31;
+    const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (row >= rows) return;
+    const int32_t *x = X + row * ldx;
+    int32_t mx = INT_MIN;
+    for (int i = lane; i < len; i += 32) mx = max(mx, x[i]);
+    mx = warp_max(mx);
+    const int32_t lowb = mx > INT_MIN + (1 << 30) ? mx - (1 << 30) : INT_MIN;
+    uint64_t sum = 0;
+    for (int i = lane; i < len; i += 32) {
+        int32_t d = x[i] > lowb ? x[i] - mx : -(1 << 30);
+        sum += shift_exp(d, c.se);
+    }
+    sum = warp_sum_u64(sum);
+    const RowNorm rn = shiftmax_norm(sum, c.s_d, c.m_p, c.M_hw, c.k_out);
+    for (int i = lane; i < len; i += 32) {
+        int32_t d = x[i] > lowb ? x[i] - mx : -(1 << 30);
+        P[row * ldp + i] = (uint8_t)shiftmax_out(shift_exp(d, c.se), rn);
+    }
+}
+
+// ------------------------------------------------------------------ SD-ShiftGELU
+__device__ __forceinline__ int32_t gelu_one(int32_t x, const GeluC &c) {
+    int32_t xc = min(max(x, -(1 << 26)), 1 << 26);  // I_div is constant beyond |x| = 2^19
+    return x * gelu_idiv(xc, c);
+}
+
+__global__ void __launch_bounds__(256) sdshiftgelu_vec(const int4 *__restrict__ X, int4 *__restrict__ Y,
+                                                        int64_t n4, const GeluC c) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+        int4 v = __ldcs(X + i);
+        int4 o;
+        o.x = gelu_one(v.x, c);
+        o.y = gelu_one(v.y, c);
+        o.z = gelu_one(v.z, c);
+        o.w = gelu_one(v.w, c);
+        __stcs(Y + i, o);
+    }
+}
+__global__ void sdshiftgelu_tail(const int32_t *X, int32_t *Y, int64_t start, int64_t n, const GeluC c) {
+    int64_t i = start + (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) Y[i] = gelu_one(X[i], c);
+}
+
+// ------------------------------------------------------------------ I-LayerNorm
+template <typename TIn, typename TOut, int EPL>
+__global__ void __launch_bounds__(256) layernorm_kernel(const LnParams p) {
+    const int lane = threadIdx.x & 31;
+    const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (row >= p.rows) return;
+    const TIn *x = (const TIn *)p.X + row * p.ldx;
+    const int C = p.C;
+    int32_t v[EPL];
+    int64_t s = 0;
+#pragma unroll
+    for (int j = 0; j < EPL; ++j) {
+        int c = lane + 32 * j;
+        v[j] = c < C ? (int32_t)x[c] : 0;
+        s += v[j];
+    }
+    s = warp_sum_i64(s);
+    // mu = floor((2 sum + C) / (2C))
+    const int64_t num = 2 * s + C, den = 2 * (int64_t)C;
+    int64_t mu = num / den;
+    if ((num % den) != 0 && num < 0) mu -= 1;
+    uint64_t V = 0;
+#pragma unroll
+    for (int j = 0; j < EPL; ++j) {
+        int c = lane + 32 * j;
+        if (c < C) {
+            int64_t y = (int64_t)v[j] - mu;
+            V += (uint64_t)(y * y);
+        }
+    }
+    V = warp_sum_u64(V);
+    // Newton integer square root from 2^16, exactly `iters` steps (stops at 0 only if V = 0)
+    uint64_t r = 1ull << 16;
+    for (int it = 0; it < p.iters; ++it) {
+        if (r == 0) break;
+        r = (r + V / r) >> 1;
+    }
+    if (r < 1) r = 1;
+    const int64_t F = (int64_t)(0x7fffffffull / r);
+    TOut *yo = (TOut *)p.Y + row * p.ldy;
+#pragma unroll
+    for (int j = 0; j < EPL; ++j) {
+        int c = lane + 32 * j;
+        if (c < C) {
+            int64_t y = (int64_t)v[j] - mu;
+            int64_t n = (y * F) >> 1;
+            int64_t o = rq(n + p.beta[c], p.mult[c], p.shift[c]);
+            yo[c] = (TOut)(sizeof(TOut) == 1 ? sat8(o) : sat16(o));
+        }
+    }
+}
+
+template <typename TIn, typename TOut>
+cudaError_t ln_dispatch(const LnParams &p, cudaStream_t s) {
+    const int rows_per_block = 8;
+    dim3 grid((unsigned)((p.rows + rows_per_block - 1) / rows_per_block));
+    if (p.C <= 128) layernorm_kernel<TIn, TOut, 4><<<grid, 256, 0, s>>>(p);
+    else if (p.C <= 256) layernorm_kernel<TIn, TOut, 8><<<grid, 256, 0, s>>>(p);
+    else if (p.C <= 384) layernorm_kernel<TIn, TOut, 12><<<grid, 256, 0, s>>>(p);
+    else if (p.C <= 512) layernorm_kernel<TIn, TOut, 16><<<grid, 256, 0, s>>>(p);
+    else if (p.C <= 1024) layernorm_kernel<TIn, TOut, 32><<<grid, 256, 0, s>>>(p);
+    else if (p.C <= 2048) layernorm_kernel<TIn, TOut, 64><<<grid, 256, 0, s>>>(p);
+    else layernorm_kernel<TIn, TOut, 128><<<grid, 256, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, int32_t len,
+                                 const ShiftmaxC &c, uint8_t *P, int64_t ldp, cudaStream_t s) {
+    if (rows == 0 || len == 0) return cudaSuccess;
+    dim3 grid((unsigned)((rows + 7) / 8));
+    bool vec = (len % 4 == 0) && (ldx % 4 == 0) && (ldp % 4 == 0) && (((uintptr_t)X & 15) == 0) &&
+               (((uintptr_t)P & 3) == 0);
+    if (vec && len <= 128) shiftmax_rows_vec<1><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 512) shiftmax_rows_vec<4><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 1024) shiftmax_rows_vec<8><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 1664) shiftmax_rows_vec<13><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 2048) shiftmax_rows_vec<16><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else shiftmax_rows_generic<<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const GeluC &c, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    int64_t n4 = 0;
+    if ((((uintptr_t)X | (uintptr_t)Y) & 15) == 0) {
+        n4 = n / 4;
+        if (n4) {
+            int64_t blocks = (n4 + 255) / 256;
+            if (blocks > 152 * 16) blocks = 152 * 16;
+            sdshiftgelu_vec<<<(unsigned)blocks, 256, 0, s>>>((const int4 *)X, (int4 *)Y, n4, c);
+        }
+    }
+    int64_t start = n4 * 4;
+    if (start < n) sdshiftgelu_tail<<<(unsigned)((n - start + 255) / 256), 256, 0, s>>>(X, Y, start, n, c);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_layernorm(const LnParams &p, cudaStream_t s) {
+    if (p.rows == 0) return cudaSuccess;
+    if (p.in_bits == 16 && p.out_bits == 8) return ln_dispatch<int16_t, int8_t>(p, s);
+    if (p.in_bits == 16 && p.out_bits == 16) return ln_dispatch<int16_t, int16_t>(p, s);
+    if (p.in_bits == 32 && p.out_bits == 8) return ln_dispatch<int32_t, int8_t>(p, s);
+    return ln_dispatch<int32_t, int16_t>(p, s);
+}
+
+}  // namespace ilw

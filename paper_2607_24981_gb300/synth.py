@@ -166,6 +166,19 @@ CONFIGS = {
 }
 
 
+def image_input(seed: int, B: int, H: int = 640, W: int = 640) -> np.ndarray:
+    """int8 image [B, 3, H, W], uniform in [-127, 127]."""
+    return uniform_int(seed, "img", (B, 3, H, W), -127, 127, np.int8)
+
+
+def patch_embed_params(seed: int, d: int, p: int = 16, T: int = 1600, mode: str = "calibrated",
+                       sigma_x: float = 64.0) -> dict:
+    """Patch-embedding conv weight [d, 3*p*p], bias, per-channel dyadic pair, position term."""
+    W, b, m, s = gemm_params(seed, "pe", d, 3 * p * p, 127.0 / math.sqrt(3.0), sigma_x, mode)
+    pos = uniform_int(seed, "pe.pos", (T, d), -64, 64, np.int16)
+    return {"p": p, "w": W, "b": b, "m": m, "s": s, "pos": pos, "m_pos": 1 << 30, "s_pos": 31}
+
+
 def backbone_params(seed: int, cfg: dict) -> list:
     out = []
     for layer in range(cfg["layers"]):

@@ -1,0 +1,67 @@
+"""The C-ABI library builds, loads without a GPU and exports every entry point declared in
+include/ilwdetr.h; the Python binding covers the same names.  No compute call is made here."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_symbols():
+    src = open(os.path.join(ROOT, "include", "ilwdetr.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(ilwdetr_\w+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def built_lib():
+    from paper_2607_24981_gb300 import build
+
+    path = build.build()
+    return path
+
+
+def test_header_declares_the_paths_entry_points():
+    syms = declared_symbols()
+    for name in ("ilwdetr_gemm_requant", "ilwdetr_shiftmax_attn", "ilwdetr_sdshiftgelu",
+                 "ilwdetr_int_layernorm", "ilwdetr_split_conv", "ilwdetr_deform_attn",
+                 "ilwdetr_block_forward", "ilwdetr_shiftmax_rows"):
+        assert name in syms
+
+
+def test_library_exports_every_declared_symbol(built_lib):
+    L = ctypes.CDLL(built_lib)
+    missing = [s for s in declared_symbols() if not hasattr(L, s)]
+    assert not missing, missing
+
+
+def test_binding_signatures_cover_the_header(built_lib):
+    import paper_2607_24981_gb300 as ilw
+
+    assert set(ilw.SIGNATURES) == set(declared_symbols())
+    ilw.lib()
+    assert ilw.version().startswith("ilwdetr")
+
+
+def test_host_side_validation_without_gpu(built_lib):
+    """Argument errors are reported before any launch, so they work with no device at all."""
+    import paper_2607_24981_gb300 as ilw
+
+    L = ilw.lib()
+    bad = ilw.ShiftmaxT(0, 16, 8, -1, 4, 31)  # I0 = 0 is outside the domain of ShiftExp
+    rc = L.ilwdetr_shiftmax_rows(ctypes.c_void_p(16), 4, 1, 4, ctypes.byref(bad), ctypes.c_void_p(16), 4, None)
+    assert rc == -1 and b"I0" in L.ilwdetr_last_error()
+    g = ilw.GeluT(1 << 14, 16, 8)  # I0 * 2^(k+1) = 2^31: overflows
+    rc = L.ilwdetr_sdshiftgelu(ctypes.c_void_p(16), ctypes.c_void_p(16), 4, ctypes.byref(g), None)
+    assert rc == -1
+    smx = ilw.ShiftmaxT(100, 16, 8, -1, 4, 31)
+    rc = L.ilwdetr_shiftmax_attn(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), 48, 1, 64, 1, 48,
+                                 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 48, None)
+    assert rc == -2  # dh = 48 unsupported
+    rc = L.ilwdetr_gemm_requant(ctypes.c_void_p(16), 24, ctypes.c_void_p(256), None, None, None, 4, 4, 24, 8,
+                                ctypes.c_void_p(16), 4, None, None)
+    assert rc == -2  # K % 16 != 0
+    assert L.ilwdetr_packed_weight_bytes(3, 32) > 0
+    assert L.ilwdetr_block_workspace_bytes(8, 1600, 384, 1536) > 8 * 1600 * 384 * 8

@@ -548,3 +548,23 @@ def test_block_equals_composition_of_pinned_parts(orc):
     y2 = orc.gemm_requant(h, bp["w_fc2"], bp["b_fc2"], bp["m_fc2"], bp["s_fc2"], 16, x1,
                           bp["m_r2"], bp["s_r2"])
     assert np.array_equal(y2, y)
+
+
+# ----------------------------------------------------------------------------- patch embedding
+def test_patch_embed_is_patch_matmul(orc):
+    """A stride-p, kernel-p convolution equals a matmul of non-overlapping patches: numpy
+    reshape/transpose into [B*T, C*p*p] rows, int64 matmul with the flattened weight, exact rq
+    of the accumulator plus exact rq of the position term, 16-bit saturation."""
+    B, Cin, Hh, Ww, p, d = 2, 3, 32, 48, 16, 40
+    img = synth.uniform_int(20, "img", (B, Cin, Hh, Ww), -127, 127, np.int8)
+    W, b, m, s = synth.gemm_params(20, "pe", d, Cin * p * p, 73.0, 256.0, "calibrated")
+    pos = synth.uniform_int(20, "pos", ((Hh // p) * (Ww // p), d), -3000, 3000, np.int16)
+    x0 = orc.patch_embed(img, p, W, b, m, s, pos, 3 << 29, 31)
+    patches = img.reshape(B, Cin, Hh // p, p, Ww // p, p).transpose(0, 2, 4, 1, 3, 5)
+    patches = patches.reshape(B * (Hh // p) * (Ww // p), Cin * p * p).astype(np.int64)
+    acc = patches @ W.astype(np.int64).T + b
+    T = (Hh // p) * (Ww // p)
+    for i in range(0, B * T, 3):
+        for c in range(d):
+            v = exact_rq(int(acc[i, c]), int(m[c]), int(s[c])) + exact_rq(int(pos[i % T, c]), 3 << 29, 31)
+            assert x0[i, c] == max(-32767, min(32767, v))
