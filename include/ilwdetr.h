@@ -189,6 +189,27 @@ int ilwdetr_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, i
                         int32_t d, const int16_t *pos, int32_t m_pos, int32_t s_pos, int16_t *x0,
                         void *workspace, size_t workspace_bytes, ilw_stream_t stream);
 
+/* Allocation-free patch embedding.  The paper has no counterpart: this entry point exists for
+ * callers that cannot provide device memory to the library -- a host runtime that owns the
+ * whole device-memory budget and forbids allocations inside its inference loop, or a
+ * latency-critical loop that cannot afford cudaMalloc/cudaFree and their implicit
+ * synchronisation.  It computes exactly what ilwdetr_patch_embed computes, with the same
+ * arguments minus the workspace, and allocates nothing: the gathered patch matrix lives in a
+ * fixed 8 MiB device array inside the library (ilwdetr_patch_embed_noalloc_max_bytes()),
+ * which every GPU that loads the library holds until the process exits.
+ *   - Batches needing more than that (B * (Hh/p) * (Ww/p) * Cin * p * p bytes; e.g. more than
+ *     6 images of 3 x 640 x 640) are rejected with ILW_ERR_UNSUPPORTED and a message.
+ *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress)
+ *     with that device current; make that first call before any stream capture.
+ *   - All calls share the one array and it keeps the last call's contents (each call overwrites
+ *     every byte it reads, so nothing needs clearing).  Calls whose execution overlaps on the
+ *     GPU (other streams, other threads) race on it: serialise them. */
+size_t ilwdetr_patch_embed_noalloc_max_bytes(void);
+int ilwdetr_patch_embed_noalloc(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww,
+                                int32_t p, const void *Wp, const int32_t *bias, const int32_t *mult,
+                                const int32_t *shift, int32_t d, const int16_t *pos, int32_t m_pos,
+                                int32_t s_pos, int16_t *x0, ilw_stream_t stream);
+
 /* ------------------------------------------------------------------ encoder block */
 
 /* Integer parameters of one encoder block (all pointers are device pointers; weights packed

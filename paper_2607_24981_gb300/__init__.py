@@ -83,6 +83,9 @@ SIGNATURES = {
     "ilwdetr_patch_embed_workspace_bytes": ([_I32, _I32, _I32, _I32, _I32], C.c_size_t),
     "ilwdetr_patch_embed": ([_VP, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _VP, _VP, _I32, _VP, _I32,
                              _I32, _VP, _VP, C.c_size_t, _VP], C.c_int),
+    "ilwdetr_patch_embed_noalloc_max_bytes": ([], C.c_size_t),
+    "ilwdetr_patch_embed_noalloc": ([_VP, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _VP, _VP, _I32, _VP,
+                                     _I32, _I32, _VP, _VP], C.c_int),
     "ilwdetr_block_workspace_bytes": ([_I32, _I32, _I32, _I32], C.c_size_t),
     "ilwdetr_block_forward": ([C.POINTER(BlockParamsT), _VP, _VP, _I32, _I32, _VP, C.c_size_t, _VP],
                               C.c_int),

@@ -88,6 +88,8 @@ int gemm_common(const int8_t *A, int64_t lda, const void *Wp, int32_t M, int32_t
 
 }  // namespace
 
+int ilw::report_error(int code, const char *msg) { return fail(code, "%s", msg); }
+
 extern "C" {
 
 const char *ilwdetr_version(void) { return "ilwdetr 0.1 sm_103a"; }

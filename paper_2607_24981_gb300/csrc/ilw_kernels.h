@@ -7,6 +7,9 @@
 
 namespace ilw {
 
+// Records `msg` as this thread's ilwdetr_last_error() text and returns `code`.
+int report_error(int code, const char *msg);
+
 // Host-side construction of the per-launch ShiftExp constants (Algorithm 1).
 inline ShiftExpC make_shiftexp(int32_t I0, int32_t k) {
     ShiftExpC c;
