@@ -9,10 +9,6 @@
 #include "ilw_kernels.h"
 #include "ilwdetr.h"
 
-namespace ilw {
-__device__ int g_device_status;  // latched by kernels whose bounded waits expire
-}
-
 namespace {
 
 thread_local std::string g_err;
@@ -98,11 +94,9 @@ const char *ilwdetr_last_error(void) { return g_err.c_str(); }
 int ilwdetr_device_status(ilw_stream_t stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_status(e, "cudaStreamSynchronize");
-    int v = 0, zero = 0;
-    e = cudaMemcpyFromSymbol(&v, ilw::g_device_status, sizeof(int));
+    int v = 0;
+    e = ilw::read_and_clear_status(&v);
     if (e != cudaSuccess) return cuda_status(e, "read device status");
-    e = cudaMemcpyToSymbol(ilw::g_device_status, &zero, sizeof(int));
-    if (e != cudaSuccess) return cuda_status(e, "clear device status");
     if (v) return fail(ILW_ERR_TIMEOUT, "a kernel's bounded wait expired (code %d)", v);
     return ILW_OK;
 }
@@ -204,6 +198,7 @@ int ilwdetr_split_conv(const int8_t *const *X, const int64_t *ldx, int32_t nb, i
         int rc = gemm_common(X[b], ldx[b], Wp[b], M, N, Kb[b]);
         if (rc) return rc;
         if ((rc = check_rq_scalar(s_b[b], "branch"))) return rc;
+        if (Kb[b] > 1024) return fail(ILW_ERR_UNSUPPORTED, "split_conv: branch %d has K=%d > 1024", b, Kb[b]);
         if (m_b[b] < 0 || (s_b[b] <= 31 && (int64_t)m_b[b] > ((int64_t)1 << s_b[b])))
             return fail(ILW_ERR_INVALID_ARG, "branch %d: ratio m_b / 2^s_b must be in [0, 1]", b);
         gp.br[b] = {X[b], ldx[b], ilw::packed_i8(Wp[b]), ilw::packed_f16(Wp[b], N, Kb[b]), Kb[b], m_b[b], s_b[b]};

@@ -173,8 +173,14 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt) {
             int key = kb * KB + nt * 8 + 2 * t;
-            if (key < Tg) { sum0 += shift_exp(S[nt][0] - mx0, se); sum1 += shift_exp(S[nt][2] - mx1, se); }
-            if (key + 1 < Tg) { sum0 += shift_exp(S[nt][1] - mx0, se); sum1 += shift_exp(S[nt][3] - mx1, se); }
+            if (key < Tg) {
+                sum0 += shift_exp_mag((uint32_t)(mx0 - S[nt][0]), se);
+                sum1 += shift_exp_mag((uint32_t)(mx1 - S[nt][2]), se);
+            }
+            if (key + 1 < Tg) {
+                sum0 += shift_exp_mag((uint32_t)(mx0 - S[nt][1]), se);
+                sum1 += shift_exp_mag((uint32_t)(mx1 - S[nt][3]), se);
+            }
         }
         __syncthreads();
     }
@@ -221,10 +227,10 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
         for (int nt = 0; nt < 8; ++nt) {
             int key = kb * KB + nt * 8 + 2 * t;
             bool v0 = key < Tg, v1 = key + 1 < Tg;
-            pv[nt][0] = v0 ? shiftmax_out(shift_exp(S[nt][0] - mx0, se), rn0) : 0u;
-            pv[nt][1] = v1 ? shiftmax_out(shift_exp(S[nt][1] - mx0, se), rn0) : 0u;
-            pv[nt][2] = v0 ? shiftmax_out(shift_exp(S[nt][2] - mx1, se), rn1) : 0u;
-            pv[nt][3] = v1 ? shiftmax_out(shift_exp(S[nt][3] - mx1, se), rn1) : 0u;
+            pv[nt][0] = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(mx0 - S[nt][0]), se), rn0) : 0u;
+            pv[nt][1] = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(mx0 - S[nt][1]), se), rn0) : 0u;
+            pv[nt][2] = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(mx1 - S[nt][2]), se), rn1) : 0u;
+            pv[nt][3] = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(mx1 - S[nt][3]), se), rn1) : 0u;
         }
 #pragma unroll
         for (int ch = 0; ch < 2; ++ch) {

@@ -189,7 +189,7 @@ cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *pack
     return cudaGetLastError();
 }
 
-cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
+cudaError_t launch_gemm_mma(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     if (gp.M == 0 || gp.N == 0) return cudaSuccess;
     dim3 grid((gp.M + BM - 1) / BM, (gp.N + BN - 1) / BN);
     bool split = gp.nb > 1 || gp.branch_rq;

@@ -1,0 +1,556 @@
+// gemm_tc.cu -- exact integer GEMM on the 5th-generation tensor cores (tcgen05.mma, sm_103a)
+// with the bias / dyadic requantisation / residual / SD-ShiftGELU / split-convolution epilogues
+// fused (Sec. 3.2.1, 3.2.2, 3.3.1).
+//
+// Exactness.  sm_103a has no int8 tcgen05 MMA, so the int8 values are carried in fp16 (every
+// integer of magnitude <= 2048 is exact in fp16) and multiplied by tcgen05.mma.kind::f16 with
+// fp32 accumulation in tensor memory.  Each product |a w| <= 127^2 < 2^14 is exact, and every
+// partial sum of an accumulator is an integer of magnitude <= 127^2 * 1024 < 2^24, exactly
+// representable in fp32, so the accumulation is exact as long as one accumulator never sees more
+// than 1024 terms of K.  Longer K is cut into segments of <= 1024, each with its own TMEM
+// accumulator; the epilogue converts every segment to int32 (exact) and adds them in integers.
+// Split-convolution branches are segments too, each rescaled by its own dyadic (m_b, s_b)
+// before the integer sum.
+//
+// Persistent kernel, one CTA per SM, 128 x BN output tiles, 14 warps:
+//   warp 0      TMA producer: int8 activation tile (128 x 64 bytes) and fp16 weight tile
+//               (BN x 64, 128-byte swizzle) per K stage, STAGES stages ahead; TMEM allocation
+//   warp 1      MMA issuer (one thread): 4 x (128 x BN x 16) MMAs per 64-wide K stage
+//   warps 2-5   operand converters: int8 activation rows (smem) -> fp16 rows in the same 128-byte
+//               swizzled K-major layout TMA produces for the weights
+//   warps 6-13  epilogue: TMEM -> registers -> integer epilogue -> HBM, one row per thread and
+//               half of the tile's columns per warp
+// Two TMEM accumulator sets (when they fit) let the epilogue of tile i overlap the MMAs of tile
+// i+1.  HBM sees the activations as int8 (half the bytes of fp16).
+// Every mbarrier wait is bounded (about one second); on expiry the kernel latches the device
+// status word, stops issuing work, drains the loads it issued and frees its TMEM.
+#include <cuda.h>
+
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include "ilw_kernels.h"
+
+namespace ilw {
+namespace {
+
+constexpr int BM = 128, BK = 64;
+constexpr int kThreads = 448;
+constexpr int kMaxSeg = 8;
+constexpr int kSegK = 1024;  // max K per accumulator for exact fp32 accumulation
+constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
+
+struct Seg {
+    int32_t k0, klen;   // K range of this accumulator (same columns of A and W)
+    int32_t map;        // index of the activation / weight tensor maps
+    int32_t m_b, s_b;   // split-conv rescale of the branch partial
+};
+
+struct TcParams {  // CUtensorMap members keep the 64-byte alignment TMA needs
+    CUtensorMap amap[kMaxBranches];
+    CUtensorMap wmap[kMaxBranches];
+    Seg seg[kMaxSeg];
+    int32_t nseg;
+    int32_t branch_rq;
+    int32_t M, N;
+    int32_t tiles_n, tiles;
+    int32_t nbuf;       // TMEM accumulator sets (1 or 2)
+    int32_t tmem_cols;
+    int *status;
+    EpiParams ep;
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred P;\n mbarrier.try_wait.parity.shared::cta.b64 P, [%1], %2;\n selp.b32 %0, 1, 0, P;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait: true when the phase completed; false (after latching `code` in the status word
+// and raising the CTA's abort flag) when it ran out, or when another role already aborted.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort, int *status, int code) {
+    long long t0 = clock64();
+    for (uint32_t i = 0;; ++i) {
+        if (mbar_try(bar, parity)) return true;
+        if ((i & 255) == 255) {
+            if (*abort) return false;
+            if (clock64() - t0 > kWaitCycles) {
+                if (status) atomicExch(status, code);
+                *abort = 1;
+                return false;
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int32_t x, int32_t y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 bytes apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    uint64_t d = (uint64_t)((saddr >> 4) & 0x3FFFu);
+    d |= (uint64_t)1 << 16;             // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024 >> 4) << 32;   // stride byte offset: next 8-row group
+    d |= (uint64_t)1 << 46;             // descriptor version
+    d |= (uint64_t)2 << 61;             // 128-byte swizzle
+    return d;
+}
+
+__device__ __forceinline__ void tc_mma(uint32_t dtmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(dtmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(acc)
+        : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+#define ILW_LD32_REGS(v)                                                                                          \
+    "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),     \
+        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]),     \
+        "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),    \
+        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+        "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : ILW_LD32_REGS(v)
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),
+          "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// 4 int8 (one word) -> 2 words of fp16x2, exact: fp16 bits 0x6400 | (b ^ 0x80) encode 1152 + b.
+__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
+    const uint32_t x = w ^ 0x80808080u;
+    uint32_t a = __byte_perm(x, 0x64646464u, 0x4140);
+    uint32_t b = __byte_perm(x, 0x64646464u, 0x4342);
+    const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
+    __half2 ha = __hsub2(*reinterpret_cast<__half2 *>(&a), k1152);
+    __half2 hb = __hsub2(*reinterpret_cast<__half2 *>(&b), k1152);
+    lo = *reinterpret_cast<uint32_t *>(&ha);
+    hi = *reinterpret_cast<uint32_t *>(&hb);
+}
+
+// Shared memory per pipeline stage: fp16 A (128 rows x 128 B, swizzled), fp16 W (BN rows x 128 B,
+// swizzled by TMA), int8 A staging (128 rows x 64 B, written by TMA).
+template <int BN>
+struct Smem {
+    static constexpr int kA16 = BM * 128;
+    static constexpr int kW = BN * 128;
+    static constexpr int kA8 = BM * 64;
+    static constexpr int kStage = kA16 + kW + kA8;
+};
+
+// Output kinds: one compact epilogue per kernel instantiation.
+enum { KIND_RQ8 = 0, KIND_RQ16 = 1, KIND_RAW32 = 2, KIND_GELU8 = 3 };
+
+template <int KIND>
+__device__ __forceinline__ int32_t epi_one(const EpiParams &ep, int64_t row, int32_t acc, int32_t bias, int32_t mult,
+                                           int32_t shift, int32_t col) {
+    const int64_t v = (int64_t)acc + bias;
+    if (KIND == KIND_RAW32) return (int32_t)v;
+    if (KIND == KIND_GELU8) {
+        const int32_t g = sat16(rq(v, mult, shift));
+        return sat8(rq((int64_t)g * gelu_idiv(g, ep.gelu), ep.m_g, ep.s_g));
+    }
+    int64_t o = rq(v, mult, shift);
+    if (ep.res) o += rq((int64_t)ep.res[(row % ep.res_rows) * ep.ldr + col], ep.m_r, ep.s_r);
+    return KIND == KIND_RQ8 ? sat8(o) : sat16(o);
+}
+
+template <int BN, int STAGES, int KIND>
+__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    constexpr int kStage = Smem<BN>::kStage;
+    uint64_t *bars = (uint64_t *)(smem + STAGES * kStage);
+    // barriers: full[S], a_ready[S], empty[S], acc_full[2], acc_empty[2]
+    uint32_t *tmem_slot = (uint32_t *)(bars + 3 * STAGES + 4);
+    volatile int *abort = (volatile int *)(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t bar0 = smem_u32(bars);
+    auto full = [&](int s) { return bar0 + 8u * s; };
+    auto a_ready = [&](int s) { return bar0 + 8u * (STAGES + s); };
+    auto empty = [&](int s) { return bar0 + 8u * (2 * STAGES + s); };
+    auto acc_full = [&](int b) { return bar0 + 8u * (3 * STAGES + b); };
+    auto acc_empty = [&](int b) { return bar0 + 8u * (3 * STAGES + 2 + b); };
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(full(s), 1);
+            mbar_init(a_ready(s), 4);
+            mbar_init(empty(s), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(acc_full(b), 1);
+            mbar_init(acc_empty(b), 8);
+        }
+        *abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(p.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int acc_cols = p.nseg * BN;  // columns of one accumulator set
+
+    if (warp == 0) {
+        // ---------------------------------------------------------------- TMA producer
+        if (lane == 0) {
+            int it = 0;  // global K-block counter (ring position)
+            bool ok = true;
+            for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x) {
+                const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN;
+                for (int sg = 0; sg < p.nseg && ok; ++sg) {
+                    const Seg &S = p.seg[sg];
+                    const int nk = (S.klen + BK - 1) / BK;
+                    for (int kk = 0; kk < nk; ++kk, ++it) {
+                        const int s = it % STAGES;
+                        const uint32_t ph = (it / STAGES) & 1;
+                        if (!mbar_wait(empty(s), ph ^ 1, abort, p.status, kStatusTimeoutFree)) {
+                            ok = false;
+                            break;
+                        }
+                        uint8_t *st = smem + s * kStage;
+                        mbar_expect_tx(full(s), Smem<BN>::kW + Smem<BN>::kA8);
+                        tma_load_2d(smem_u32(st + Smem<BN>::kA16 + Smem<BN>::kW), &p.amap[S.map], S.k0 + kk * BK, m0,
+                                    full(s));
+                        tma_load_2d(smem_u32(st + Smem<BN>::kA16), &p.wmap[S.map], S.k0 + kk * BK, n0, full(s));
+                    }
+                }
+            }
+            if (!ok) {  // drain the loads still in flight (bounded) before the CTA can exit
+                long long t0 = clock64();
+                for (int j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
+                    while (!mbar_try(full(j % STAGES), (j / STAGES) & 1) && clock64() - t0 < kWaitCycles) {
+                    }
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+            int it = 0, tl = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++tl) {
+                const int b = tl % p.nbuf;
+                const uint32_t use = (uint32_t)(tl / p.nbuf);
+                if (!mbar_wait(acc_empty(b), (use & 1) ^ 1, abort, p.status, kStatusTimeoutMma)) break;
+                tc_fence_after();
+                for (int sg = 0; sg < p.nseg && ok; ++sg) {
+                    const Seg &S = p.seg[sg];
+                    const int nk = (S.klen + BK - 1) / BK;
+                    const uint32_t dt = tmem + (uint32_t)(b * acc_cols + sg * BN);
+                    for (int kk = 0; kk < nk; ++kk, ++it) {
+                        const int s = it % STAGES;
+                        const uint32_t ph = (it / STAGES) & 1;
+                        if (!mbar_wait(a_ready(s), ph, abort, p.status, kStatusTimeoutOperand)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a0 = smem_u32(smem + s * kStage), w0 = a0 + Smem<BN>::kA16;
+#pragma unroll
+                        for (int k16 = 0; k16 < BK / 16; ++k16)
+                            tc_mma(dt, sw128_desc(a0 + 32 * k16), sw128_desc(w0 + 32 * k16), idesc,
+                                   (kk > 0 || k16 > 0) ? 1u : 0u);
+                        tc_commit(empty(s));
+                    }
+                }
+                tc_commit(acc_full(b));  // arrives once every MMA of this tile has completed
+            }
+        }
+    } else if (warp < 6) {
+        // ---------------------------------------------------------------- operand converters
+        const int r = (warp - 2) * 32 + lane;  // row of the 128-row A tile
+        const int sw = (r >> 1) & 3;           // TMA's 64-byte swizzle of the int8 staging rows
+        int it = 0;
+        for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
+            for (int sg = 0; sg < p.nseg; ++sg) {
+                const int nk = (p.seg[sg].klen + BK - 1) / BK;
+                for (int kk = 0; kk < nk; ++kk, ++it) {
+                    const int s = it % STAGES;
+                    const uint32_t ph = (it / STAGES) & 1;
+                    if (!mbar_wait(full(s), ph, abort, p.status, kStatusTimeoutTma)) goto conv_done;
+                    uint8_t *st = smem + s * kStage;
+                    const uint8_t *a8 = st + Smem<BN>::kA16 + Smem<BN>::kW + r * 64;
+                    uint8_t *a16 = st + r * 128;
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {  // 16 int8 = K elements 16j .. 16j+15
+                        const uint4 v = *(const uint4 *)(a8 + 16 * (j ^ sw));
+                        uint4 o0, o1;
+                        i8x4_to_f16x4(v.x, o0.x, o0.y);
+                        i8x4_to_f16x4(v.y, o0.z, o0.w);
+                        i8x4_to_f16x4(v.z, o1.x, o1.y);
+                        i8x4_to_f16x4(v.w, o1.z, o1.w);
+                        *(uint4 *)(a16 + (((2 * j) ^ (r & 7)) << 4)) = o0;
+                        *(uint4 *)(a16 + (((2 * j + 1) ^ (r & 7)) << 4)) = o1;
+                    }
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(a_ready(s));
+                }
+            }
+        }
+    conv_done:;
+    } else {
+        // ---------------------------------------------------------------- epilogue
+        // 8 warps: warp w reads TMEM lanes 32q..32q+31 (q = w % 4) and owns half h of the columns
+        constexpr int HALF = BN / 2;
+        const int q = warp & 3, h = (warp - 6) >> 2;
+        const EpiParams &ep = p.ep;
+        int32_t *s_bias = (int32_t *)(tmem_slot + 4) + (warp - 6) * 3 * HALF;  // this warp's copy of
+        int32_t *s_mult = s_bias + HALF;                                       // the tile's per-column
+        int32_t *s_shift = s_mult + HALF;                                      // epilogue parameters
+        constexpr int bits = KIND == KIND_RQ16 ? 16 : (KIND == KIND_RAW32 ? 32 : 8);
+        int tl = 0;
+        for (int t = blockIdx.x; t < p.tiles; t += gridDim.x, ++tl) {
+            const int b = tl % p.nbuf;
+            const uint32_t use = (uint32_t)(tl / p.nbuf);
+            const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN + h * HALF;
+            __syncwarp();  // this warp is done with the previous tile's parameters
+            for (int c = lane; c < HALF; c += 32) {
+                const int col = n0 + c;
+                const bool ok = col < p.N;
+                s_bias[c] = (ok && ep.bias) ? ep.bias[col] : 0;
+                s_mult[c] = (ok && ep.mult) ? ep.mult[col] : 0;
+                s_shift[c] = (ok && ep.shift) ? ep.shift[col] : 1;
+            }
+            __syncwarp();
+            if (!mbar_wait(acc_full(b), use & 1, abort, p.status, kStatusTimeoutMma)) break;
+            tc_fence_after();
+            const int64_t row = (int64_t)m0 + 32 * q + lane;
+            const bool row_ok = row < p.M;
+            for (int c0 = 0; c0 < HALF; c0 += 16) {
+                int32_t acc[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) acc[i] = 0;
+                for (int sg = 0; sg < p.nseg; ++sg) {
+                    uint32_t v[16];
+                    tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * acc_cols + sg * BN + h * HALF + c0), v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        int32_t a = __float2int_rn(__uint_as_float(v[i]));  // exact: integer < 2^24
+                        acc[i] += p.branch_rq ? (int32_t)rq(a, p.seg[sg].m_b, p.seg[sg].s_b) : a;
+                    }
+                }
+                if (c0 + 16 >= HALF) {  // every TMEM read of this warp in this accumulator set is done
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(acc_empty(b));
+                }
+                const int ncol = min(16, p.N - (n0 + c0));
+                if (row_ok && ncol > 0) {
+                    int32_t out[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i)
+                        out[i] = epi_one<KIND>(ep, row, acc[i], s_bias[c0 + i], s_mult[c0 + i], s_shift[c0 + i],
+                                               min(n0 + c0 + i, p.N - 1));
+                    char *dst = (char *)ep.C + (row * ep.ldc + n0 + c0) * (bits / 8);
+                    const bool vec = ncol == 16 && (((uintptr_t)dst & 15) == 0);
+                    if constexpr (bits == 8) {
+                        if (vec) {
+                            uint32_t w[4];
+#pragma unroll
+                            for (int u = 0; u < 4; ++u)
+                                w[u] = (uint32_t)(uint8_t)out[4 * u] | ((uint32_t)(uint8_t)out[4 * u + 1] << 8) |
+                                       ((uint32_t)(uint8_t)out[4 * u + 2] << 16) | ((uint32_t)(uint8_t)out[4 * u + 3] << 24);
+                            *(uint4 *)dst = make_uint4(w[0], w[1], w[2], w[3]);
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i)
+                                if (i < ncol) ((int8_t *)dst)[i] = (int8_t)out[i];
+                        }
+                    } else if constexpr (bits == 16) {
+                        if (vec) {
+#pragma unroll
+                            for (int j = 0; j < 2; ++j) {
+                                uint32_t w[4];
+#pragma unroll
+                                for (int u = 0; u < 4; ++u)
+                                    w[u] = (uint32_t)(uint16_t)out[8 * j + 2 * u] | ((uint32_t)(uint16_t)out[8 * j + 2 * u + 1] << 16);
+                                ((uint4 *)dst)[j] = make_uint4(w[0], w[1], w[2], w[3]);
+                            }
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i)
+                                if (i < ncol) ((int16_t *)dst)[i] = (int16_t)out[i];
+                        }
+                    } else {
+                        if (vec) {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j)
+                                ((int4 *)dst)[j] = make_int4(out[4 * j], out[4 * j + 1], out[4 * j + 2], out[4 * j + 3]);
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i)
+                                if (i < ncol) ((int32_t *)dst)[i] = out[i];
+                        }
+                    }
+                }
+                __syncwarp();  // reconverge before the next warp-synchronous tcgen05.ld
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        __syncwarp();
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(p.tmem_cols) : "memory");
+    }
+}
+
+// ------------------------------------------------------------------ host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static std::once_flag once;
+    static EncodeTiledFn fn = nullptr;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiledFn)f;
+    });
+    return fn;
+}
+
+// 2-D tensor map over a row-major [rows, cols] matrix (cols contiguous), boxes of box_cols x box_rows
+bool make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int esize, int64_t rows, int64_t cols,
+              int64_t ld, int box_cols, int box_rows, CUtensorMapSwizzle sw) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)(ld * esize)};
+    cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int num_sms() {
+    static std::once_flag once;
+    static int n = 148;
+    std::call_once(once, [] {
+        int dev = 0, v = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+            n = v;
+    });
+    return n;
+}
+
+template <int BN, int STAGES, int KIND>
+cudaError_t launch_tc(TcParams &tp, cudaStream_t s) {
+    const size_t smem = 1024 + (size_t)STAGES * Smem<BN>::kStage + 8 * (3 * STAGES + 4) + 16 + 4 * 3 * BN * 4;
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)smem);
+    });
+    if (attr_err != cudaSuccess) return attr_err;
+    const int grid = tp.tiles < num_sms() ? tp.tiles : num_sms();
+    gemm_tc_kernel<BN, STAGES, KIND><<<grid, kThreads, smem, s>>>(tp);
+    return cudaGetLastError();
+}
+
+template <int BN, int STAGES>
+cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
+    TcParams tp;
+    memset(&tp, 0, sizeof(tp));
+    tp.M = gp.M;
+    tp.N = gp.N;
+    tp.branch_rq = gp.branch_rq ? 1 : 0;
+    tp.ep = ep;
+    tp.status = status_word_ptr();
+    int nseg = 0;
+    for (int b = 0; b < gp.nb; ++b) {
+        const GemmBranch &br = gp.br[b];
+        if (!make_map(&tp.amap[b], br.A, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, gp.M, br.K, br.lda, BK, BM,
+                      CU_TENSOR_MAP_SWIZZLE_64B) ||
+            !make_map(&tp.wmap[b], br.Wp, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, gp.N, br.K, br.K, BK, BN,
+                      CU_TENSOR_MAP_SWIZZLE_128B))
+            return cudaErrorInvalidValue;
+        // cut K into near-equal segments of at most kSegK (multiples of 64)
+        const int parts = (br.K + kSegK - 1) / kSegK;
+        if (gp.branch_rq && parts != 1) return cudaErrorInvalidValue;
+        const int per = ((br.K + parts - 1) / parts + BK - 1) / BK * BK;
+        for (int k0 = 0; k0 < br.K; k0 += per) {
+            if (nseg >= kMaxSeg) return cudaErrorInvalidValue;
+            Seg &S = tp.seg[nseg++];
+            S.k0 = k0;
+            S.klen = min(per, br.K - k0);
+            S.map = b;
+            S.m_b = br.m_b;
+            S.s_b = br.s_b;
+        }
+    }
+    tp.nseg = nseg;
+    tp.tiles_n = (gp.N + BN - 1) / BN;
+    tp.tiles = ((gp.M + BM - 1) / BM) * tp.tiles_n;
+    const int one = nseg * BN;
+    tp.nbuf = 2 * one <= 512 ? 2 : 1;
+    int alloc = 32;
+    while (alloc < tp.nbuf * one) alloc <<= 1;
+    if (alloc > 512) return cudaErrorInvalidValue;
+    tp.tmem_cols = alloc;
+    if (ep.kind == EPI_GELU) return launch_tc<BN, STAGES, KIND_GELU8>(tp, s);
+    if (ep.out_bits == 8) return launch_tc<BN, STAGES, KIND_RQ8>(tp, s);
+    if (ep.out_bits == 16) return launch_tc<BN, STAGES, KIND_RQ16>(tp, s);
+    return launch_tc<BN, STAGES, KIND_RAW32>(tp, s);
+}
+
+}  // namespace
+
+cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
+    if (gp.M == 0 || gp.N == 0) return cudaSuccess;
+    // 192-wide tiles when N splits evenly into them (fewer re-reads of A per flop), else 128
+    if (gp.N % 192 == 0 && gp.N >= 768 && gp.nb == 1) return run<192, 4>(gp, ep, s);
+    return run<128, 5>(gp, ep, s);
+}
+
+}  // namespace ilw

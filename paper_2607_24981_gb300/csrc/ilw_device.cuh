@@ -35,11 +35,24 @@ struct ShiftExpC {
     int32_t k;      // k_inter
 };
 
-// I_exp = ShiftExp(delta) for delta <= 0 with delta >= -2^30 (callers clamp below that: every
-// such delta is already in the clamp region, where the result is the constant I0).
-__device__ __forceinline__ uint32_t shift_exp(int32_t delta, const ShiftExpC &c) {
-    int32_t Ie = delta + (delta >> 1) - (delta >> 4);  // I * log2(e) with shifts
-    uint32_t n = (uint32_t)min(-Ie, c.kI0);            // -clamp_min(I_e, -k I0)
+// Arithmetic (flooring) right shift of a signed value.
+__device__ __forceinline__ int32_t asr(int32_t v, int32_t s) {
+    int32_t r;
+    asm("shr.s32 %0, %1, %2;" : "=r"(r) : "r"(v), "r"(s));
+    return r;
+}
+
+// I_exp = ShiftExp(-a) for a magnitude a = -I >= 0 with a <= 2^30 (callers clamp above that:
+// every such input is already in the clamp region, where the result is the constant I0).
+// Algorithm 1's I_e = I + (I >> 1) - (I >> 4) floors negative values; with I = -a,
+// floor(-a/2) = -((a+1) >> 1) and floor(-a/16) = -((a+15) >> 4), so
+//   -I_e = a + ((a+1) >> 1) - ((a+15) >> 4)
+// exactly, and every shift here acts on a non-negative value.  (Shifting the negated value
+// directly is not safe to leave to the compiler: CUDA 13.0 turned (-|x|) >> 4 into a truncating
+// shift when it could infer the operand's sign.)
+__device__ __forceinline__ uint32_t shift_exp_mag(uint32_t a, const ShiftExpC &c) {
+    uint32_t n = a + ((a + 1u) >> 1) - ((a + 15u) >> 4);  // -I_e (I * log2 e with shifts)
+    n = min(n, (uint32_t)c.kI0);                            // -clamp_min(I_e, -k I0)
     uint32_t q = (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
     uint32_t r = n - q * (uint32_t)c.I0;               // decimal part, in [0, I0)
     uint32_t Ib = (uint32_t)c.I0 - ((r + 1u) >> 1);    // ((-r) >> 1) + I0
@@ -75,13 +88,27 @@ struct GeluC {
     ShiftExpC se;
     int32_t out_sh;  // 31 - k_out + 1
 };
+// floor((2^31 - 1) / den) for den >= 1, exact.  For den >= 2^16 the quotient is < 2^15 and a
+// float estimate (relative error < 2^-21, so absolute error < 2^-6) rounded to the nearest
+// integer is q or q + 1; one integer remainder test corrects it.  Smaller denominators use the
+// integer divide.
+__device__ __forceinline__ uint32_t div_int31(uint32_t den) {
+    if (den < 65536u) return kInt31Max / den;
+    uint32_t q = __float2uint_rn(__fdividef(2147483647.0f, __uint2float_rn(den)));
+    const int64_t r = (int64_t)kInt31Max - (int64_t)q * den;
+    if (r < 0) --q;
+    else if (r >= (int64_t)den) ++q;
+    return q;
+}
+
+// With I_shift = ReLU(I_p) and I_delta = I_p - I_shift, one of the two ShiftExp inputs is always
+// 0, and ShiftExp(0) = I0 * 2^k exactly; so a single ShiftExp of -|I_p| gives both E and E'.
 __device__ __forceinline__ int32_t gelu_idiv(int32_t x, const GeluC &c) {
-    int32_t Ip = x + (x >> 1) + (x >> 3) + (x >> 4);  // 1.702 x
-    int32_t Ish = max(Ip, 0);                          // ReLU(I_p)
-    int32_t Id = Ip - Ish;                             // <= 0
-    uint32_t E = shift_exp(Id, c.se);
-    uint32_t E2 = shift_exp(-Ish, c.se);
-    uint32_t F = kInt31Max / (E + E2);  // IntDiv: Algorithm 2's fixed-point division, s_d = 0
+    int32_t Ip = x + asr(x, 1) + asr(x, 3) + asr(x, 4);  // 1.702 x
+    uint32_t e = shift_exp_mag((uint32_t)abs(Ip), c.se);   // ShiftExp(I_delta) or ShiftExp(-I_shift)
+    uint32_t top = (uint32_t)c.se.I0 << c.se.k;         // ShiftExp(0)
+    uint32_t E = Ip >= 0 ? top : e;                    // numerator: ShiftExp(I_delta)
+    uint32_t F = div_int31(top + e);  // IntDiv: Algorithm 2's fixed-point division, s_d = 0
     return (int32_t)(((uint64_t)E * F) >> c.out_sh);
 }
 

@@ -10,6 +10,15 @@ namespace ilw {
 // Records `msg` as this thread's ilwdetr_last_error() text and returns `code`.
 int report_error(int code, const char *msg);
 
+// Device status word (latched by kernels whose bounded waits expire): its device address on
+// the current device (nullptr on failure), and a synchronous read-and-clear.
+int *status_word_ptr();
+cudaError_t read_and_clear_status(int *value);
+constexpr int kStatusTimeoutTma = 1;     // a wait for a TMA load ran out
+constexpr int kStatusTimeoutMma = 2;     // a wait for tensor-core completion ran out
+constexpr int kStatusTimeoutOperand = 3; // a wait for the converted operand ran out
+constexpr int kStatusTimeoutFree = 4;    // a wait for a free pipeline stage ran out
+
 // Host-side construction of the per-launch ShiftExp constants (Algorithm 1).
 inline ShiftExpC make_shiftexp(int32_t I0, int32_t k) {
     ShiftExpC c;
@@ -60,6 +69,23 @@ struct EpiParams {
     int32_t m_g, s_g;
 };
 
+// The fused epilogue value of output (row, col) from the exact integer accumulator (bias not
+// yet added), given the column's bias/mult/shift: Sec. 3.2.1 (bias, per-channel dyadic
+// requantisation), the two-term residual form, and SD-ShiftGELU (Algorithm 1) for EPI_GELU.
+__device__ __forceinline__ int32_t epi_value(const EpiParams &ep, int64_t row, int32_t acc, int32_t bias,
+                                             int32_t mult, int32_t shift, int32_t col) {
+    int64_t v = (int64_t)acc + bias;
+    if (ep.kind == EPI_GELU) {
+        int32_t g = sat16(rq(v, mult, shift));
+        int32_t idiv = gelu_idiv(g, ep.gelu);
+        return sat8(rq((int64_t)g * idiv, ep.m_g, ep.s_g));
+    }
+    if (ep.out_bits == 32) return (int32_t)v;
+    int64_t o = rq(v, mult, shift);
+    if (ep.res) o += rq((int64_t)ep.res[(row % ep.res_rows) * ep.ldr + col], ep.m_r, ep.s_r);
+    return ep.out_bits == 8 ? sat8(o) : sat16(o);
+}
+
 // Packed weight layout: [int8 W, N*K bytes][pad to 256][fp16 W, N*K*2 bytes].
 size_t packed_weight_bytes(int32_t N, int32_t K);
 inline const int8_t *packed_i8(const void *p) { return (const int8_t *)p; }
@@ -68,7 +94,10 @@ inline const void *packed_f16(const void *p, int32_t N, int32_t K) {
     return (const char *)p + off;
 }
 cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, cudaStream_t s);
+// tcgen05 tensor-core GEMM (exact integer via fp16 operands, fp32 TMEM accumulators)
 cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s);
+// warp-level int8 MMA GEMM (mma.sync m16n8k32), kept as the measured legacy-path baseline
+cudaError_t launch_gemm_mma(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s);
 
 // ---------------------------------------------------------------- row / element kernels
 struct ShiftmaxC {

@@ -60,8 +60,8 @@ __global__ void __launch_bounds__(256) shiftmax_rows_vec(const int32_t *__restri
             int32_t *e = (int32_t *)&v[j];
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                int32_t d = e[q] > lowb ? e[q] - mx : -(1 << 30);
-                uint32_t ex = shift_exp(d, c.se);
+                uint32_t a = e[q] > lowb ? (uint32_t)(mx - e[q]) : (1u << 30);
+                uint32_t ex = shift_exp_mag(a, c.se);
                 e[q] = (int32_t)ex;
                 sum += ex;
             }
@@ -96,14 +96,14 @@ __global__ void __launch_bounds__(256) shiftmax_rows_generic(const int32_t *__re
     const int32_t lowb = mx > INT_MIN + (1 << 30) ? mx - (1 << 30) : INT_MIN;
     uint64_t sum = 0;
     for (int i = lane; i < len; i += 32) {
-        int32_t d = x[i] > lowb ? x[i] - mx : -(1 << 30);
-        sum += shift_exp(d, c.se);
+        uint32_t a = x[i] > lowb ? (uint32_t)(mx - x[i]) : (1u << 30);
+        sum += shift_exp_mag(a, c.se);
     }
     sum = warp_sum_u64(sum);
     const RowNorm rn = shiftmax_norm(sum, c.s_d, c.m_p, c.M_hw, c.k_out);
     for (int i = lane; i < len; i += 32) {
-        int32_t d = x[i] > lowb ? x[i] - mx : -(1 << 30);
-        P[row * ldp + i] = (uint8_t)shiftmax_out(shift_exp(d, c.se), rn);
+        uint32_t a = x[i] > lowb ? (uint32_t)(mx - x[i]) : (1u << 30);
+        P[row * ldp + i] = (uint8_t)shiftmax_out(shift_exp_mag(a, c.se), rn);
     }
 }
 

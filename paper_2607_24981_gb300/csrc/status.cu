@@ -1,0 +1,39 @@
+// status.cu -- the device status word that kernels with bounded waits latch when a wait runs
+// out, and the host side that reads and clears it (ilwdetr_device_status).
+#include <cstdint>
+#include <mutex>
+
+#include "ilw_kernels.h"
+
+namespace ilw {
+namespace {
+
+__device__ int g_status_word;
+
+constexpr int kMaxDev = 64;
+std::mutex g_mu;
+int *g_addr[kMaxDev] = {};
+
+}  // namespace
+
+int *status_word_ptr() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return nullptr;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (!g_addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+        g_addr[dev] = (int *)p;
+    }
+    return g_addr[dev];
+}
+
+cudaError_t read_and_clear_status(int *value) {
+    *value = 0;
+    int zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(value, g_status_word, sizeof(int));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_status_word, &zero, sizeof(int));
+}
+
+}  // namespace ilw
