@@ -5,11 +5,13 @@
 // maximum must be known before any exponential.  Each CTA therefore streams the keys of its
 // attention group three times (they stay in L2): pass 1 takes the exact row max, pass 2 sums
 // ShiftExp (int64), which fixes s_d and F, pass 3 forms P (u8) and accumulates P V.
-// Scores and P V run on the int8 tensor-core MMA (m16n8k32, s8.s8 and u8.s8 -> s32), exact.
 //
-// P V reuses the score fragments as the A operand without shuffles: the MMA's k order is
-// permuted (k-slot 4t + {0,1,2,3} <-> key 2t + {0,1,8,9} within each 16-key half), and V is
-// transposed into shared memory with the same permutation.
+// Tensor cores: the int8 q, k, v and the u8 P are carried exactly in fp16 and multiplied with the
+// warp-level fp16 MMA (m16n8k16, fp32 accumulation).  Every score |q.k| <= 64 * 127^2 < 2^20 and
+// every partial sum of P V (|.| <= 255 * 127 * (sum of P <= 2^8)) is an integer below 2^24, so the
+// fp32 accumulation is exact.  (On this GPU the fp16 warp MMA is about 3.8x faster than the int8
+// one.)  Q, K, V are read from HBM as int8 and converted while staged into shared memory; the
+// score fragments of pass 3 are already laid out as the A operand of P V.
 #include <climits>
 #include <cstdint>
 
@@ -22,27 +24,45 @@ constexpr int QT = 64;   // query rows per CTA (4 warps x 16)
 constexpr int KB = 64;   // keys per block
 constexpr int THREADS = 128;
 
-__device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool valid) {
-    uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
-    int n = valid ? 16 : 0;
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
+__device__ __forceinline__ void mma_f16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
 
-__device__ __forceinline__ void mma_s8s8(int32_t (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k32.row.col.s32.s8.s8.s32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-        "{%0,%1,%2,%3};\n"
-        : "+r"(c[0]), "+r"(c[1]), "+r"(c[2]), "+r"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+// two int8 (low bytes of w >> 0 and w >> 8) -> fp16x2, exact: 0x6400 | (b ^ 0x80) is 1152 + b
+__device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t w) {
+    uint32_t x = __byte_perm(w ^ 0x8080u, 0x64646464u, 0x4140);
+    __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), __half2half2(__ushort_as_half((unsigned short)0x6480)));
+    return *reinterpret_cast<uint32_t *>(&h);
 }
-__device__ __forceinline__ void mma_u8s8(int32_t (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k32.row.col.s32.u8.s8.s32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-        "{%0,%1,%2,%3};\n"
-        : "+r"(c[0]), "+r"(c[1]), "+r"(c[2]), "+r"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+// 16 int8 -> 16 fp16 (two uint4)
+__device__ __forceinline__ void i8x16_to_h16(const uint4 v, uint4 &lo, uint4 &hi) {
+    lo.x = i8x2_to_h2(v.x);
+    lo.y = i8x2_to_h2(v.x >> 16);
+    lo.z = i8x2_to_h2(v.y);
+    lo.w = i8x2_to_h2(v.y >> 16);
+    hi.x = i8x2_to_h2(v.z);
+    hi.y = i8x2_to_h2(v.z >> 16);
+    hi.z = i8x2_to_h2(v.w);
+    hi.w = i8x2_to_h2(v.w >> 16);
+}
+// two integers in [0, 1024) -> fp16x2, exact: 0x6400 | p is 1024 + p
+__device__ __forceinline__ uint32_t u10x2_to_h2(uint32_t p0, uint32_t p1) {
+    uint32_t x = (0x6400u | p0) | ((0x6400u | p1) << 16);
+    __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), __half2half2(__ushort_as_half((unsigned short)0x6400)));
+    return *reinterpret_cast<uint32_t *>(&h);
 }
 
 struct Group {
@@ -57,14 +77,12 @@ struct Group {
 
 template <int DH>
 __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
-    constexpr int LDK = DH + 16;  // padded q/k/v smem row (bytes)
-    constexpr int LDV = KB + 16;  // padded transposed-V row (bytes)
-    constexpr int KS = DH / 32;   // k32 steps of q k^T
-    constexpr int NT = DH / 8;    // n-tiles of P V
-    __shared__ __align__(16) int8_t Qs[QT * LDK];
-    __shared__ __align__(16) int8_t Ks[KB * LDK];
-    __shared__ __align__(16) int8_t Vr[KB * LDK];
-    __shared__ __align__(16) int8_t Vt[DH * LDV];
+    constexpr int LDH = DH * 2 + 16;  // padded fp16 row (bytes): conflict-free ldmatrix
+    constexpr int KS = DH / 16;       // k16 steps of q k^T
+    constexpr int NT = DH / 8;        // n-tiles of P V
+    constexpr int CH = DH / 16;       // 16-byte int8 chunks per row
+    __shared__ __align__(16) uint8_t Ks[KB * LDH];
+    __shared__ __align__(16) uint8_t Vs[KB * LDH];
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, t = lane & 3;
@@ -78,108 +96,123 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
         gr.nw = p.nw;
         gr.gs = p.grid_side;
         gr.ws = p.nw > 1 ? p.grid_side / p.nw : 0;
-        gr.wy = w / (p.nw > 0 ? p.nw : 1);
-        gr.wx = w % (p.nw > 0 ? p.nw : 1);
+        gr.wy = w / p.nw;
+        gr.wx = w % p.nw;
         gr.Tg = p.nw > 1 ? gr.ws * gr.ws : p.T;
     }
     const int Tg = gr.Tg;
     const int q0 = blockIdx.x * QT;
     const int hoff = h * DH;
 
-    // ---- Q tile -> registers (A fragments of the score MMA)
-    for (int c = tid; c < QT * (DH / 16); c += THREADS) {
-        int r = c / (DH / 16), kc = (c % (DH / 16)) * 16;
-        bool v = (q0 + r) < Tg;
-        const int8_t *src = v ? p.Q + gr.token(q0 + r) * p.ld_qkv + hoff + kc : p.Q;
-        cp_async16(Qs + r * LDK + kc, src, v);
-    }
-    cp_async_commit();
-    cp_async_wait_all();
-    __syncthreads();
+    // ---- Q rows of this warp -> fp16 A fragments (rows g and g + 8 of the warp's 16)
     uint32_t qa[KS][4];
+    {
+        const int r0 = q0 + warp * 16 + g, r1 = r0 + 8;
+        const int8_t *Q0 = r0 < Tg ? p.Q + gr.token(r0) * p.ld_qkv + hoff : nullptr;
+        const int8_t *Q1 = r1 < Tg ? p.Q + gr.token(r1) * p.ld_qkv + hoff : nullptr;
 #pragma unroll
-    for (int ks = 0; ks < KS; ++ks) {
-        const int8_t *q = Qs + (warp * 16 + g) * LDK + ks * 32 + 4 * t;
-        qa[ks][0] = *(const uint32_t *)(q);
-        qa[ks][1] = *(const uint32_t *)(q + 8 * LDK);
-        qa[ks][2] = *(const uint32_t *)(q + 16);
-        qa[ks][3] = *(const uint32_t *)(q + 8 * LDK + 16);
+        for (int ks = 0; ks < KS; ++ks) {
+            const int c = ks * 16 + 2 * t;
+            uint32_t w00 = Q0 ? *(const uint16_t *)(Q0 + c) : 0u, w01 = Q0 ? *(const uint16_t *)(Q0 + c + 8) : 0u;
+            uint32_t w10 = Q1 ? *(const uint16_t *)(Q1 + c) : 0u, w11 = Q1 ? *(const uint16_t *)(Q1 + c + 8) : 0u;
+            qa[ks][0] = i8x2_to_h2(w00);
+            qa[ks][1] = i8x2_to_h2(w10);
+            qa[ks][2] = i8x2_to_h2(w01);
+            qa[ks][3] = i8x2_to_h2(w11);
+        }
     }
 
     const int nkb = (Tg + KB - 1) / KB;
-    auto load_k = [&](int kb) {
-        for (int c = tid; c < KB * (DH / 16); c += THREADS) {
-            int r = c / (DH / 16), kc = (c % (DH / 16)) * 16;
-            int key = kb * KB + r;
-            bool v = key < Tg;
-            const int8_t *src = v ? p.K + gr.token(key) * p.ld_qkv + hoff + kc : p.K;
-            cp_async16(Ks + r * LDK + kc, src, v);
+    // stage one 64-key block of K (and V) as fp16 rows
+    auto stage = [&](int kb, bool with_v) {
+        for (int c = tid; c < KB * CH; c += THREADS) {
+            const int r = c / CH, ch = c % CH;
+            const int key = kb * KB + r;
+            uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+            if (key < Tg) {
+                const int64_t off = gr.token(key) * p.ld_qkv + hoff + ch * 16;
+                kv = __ldg((const uint4 *)(p.K + off));
+                if (with_v) vv = __ldg((const uint4 *)(p.V + off));
+            }
+            uint4 lo, hi;
+            i8x16_to_h16(kv, lo, hi);
+            *(uint4 *)(Ks + r * LDH + ch * 32) = lo;
+            *(uint4 *)(Ks + r * LDH + ch * 32 + 16) = hi;
+            if (with_v) {
+                i8x16_to_h16(vv, lo, hi);
+                *(uint4 *)(Vs + r * LDH + ch * 32) = lo;
+                *(uint4 *)(Vs + r * LDH + ch * 32 + 16) = hi;
+            }
         }
     };
-    auto load_v = [&](int kb) {
-        for (int c = tid; c < KB * (DH / 16); c += THREADS) {
-            int r = c / (DH / 16), kc = (c % (DH / 16)) * 16;
-            int key = kb * KB + r;
-            bool v = key < Tg;
-            const int8_t *src = v ? p.V + gr.token(key) * p.ld_qkv + hoff + kc : p.V;
-            cp_async16(Vr + r * LDK + kc, src, v);
-        }
-    };
-    // scores of this warp's 16 rows x the 64 keys of the block in Ks
-    auto scores = [&](int32_t (&S)[8][4]) {
+    const uint32_t ks_base = (uint32_t)__cvta_generic_to_shared(Ks);
+    const uint32_t vs_base = (uint32_t)__cvta_generic_to_shared(Vs);
+    // scores of this warp's 16 rows x the 64 keys of the staged block (exact integers in fp32)
+    auto scores = [&](float (&S)[8][4]) {
 #pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            S[nt][0] = S[nt][1] = S[nt][2] = S[nt][3] = 0;
+        for (int nt = 0; nt < 8; ++nt) S[nt][0] = S[nt][1] = S[nt][2] = S[nt][3] = 0.f;
 #pragma unroll
-            for (int ks = 0; ks < KS; ++ks) {
-                const int8_t *k = Ks + (nt * 8 + g) * LDK + ks * 32 + 4 * t;
-                mma_s8s8(S[nt], qa[ks], *(const uint32_t *)k, *(const uint32_t *)(k + 16));
+        for (int np = 0; np < 4; ++np) {      // pairs of n-tiles (16 keys)
+#pragma unroll
+            for (int kp = 0; kp < KS; kp += 2) {  // pairs of k16 steps (32 dims)
+                // matrices: keys [16np + 8(i&1) ...], dims [16kp + 8(i>>1) ...]
+                uint32_t b[4][2];
+                const int i = lane >> 3;
+                const uint32_t row = 16 * np + 8 * (i & 1) + (lane & 7);
+                const uint32_t addr = ks_base + row * LDH + (16 * kp + 8 * (i >> 1)) * 2;
+                uint32_t r0, r1, r2, r3;
+                ldsm_x4(addr, r0, r1, r2, r3);  // r0: n-tile 2np, k lo; r1: 2np+1, k lo; r2, r3: k hi
+                b[0][0] = r0; b[1][0] = r1; b[0][1] = r2; b[1][1] = r3;
+                mma_f16(S[2 * np], qa[kp], b[0][0], b[0][1]);
+                mma_f16(S[2 * np + 1], qa[kp], b[1][0], b[1][1]);
+                if (kp + 1 < KS) {
+                    ldsm_x4(addr + 16 * 2, r0, r1, r2, r3);  // next k16 step: 16 dims further
+                    mma_f16(S[2 * np], qa[kp + 1], r0, r2);
+                    mma_f16(S[2 * np + 1], qa[kp + 1], r1, r3);
+                }
             }
         }
     };
 
     // ---- pass 1: exact row maxima
-    int32_t mx0 = INT_MIN, mx1 = INT_MIN;
+    float mx0 = -3.0e38f, mx1 = -3.0e38f;
     for (int kb = 0; kb < nkb; ++kb) {
-        load_k(kb);
-        cp_async_commit();
-        cp_async_wait_all();
+        stage(kb, false);
         __syncthreads();
-        int32_t S[8][4];
+        float S[8][4];
         scores(S);
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt) {
-            int key = kb * KB + nt * 8 + 2 * t;
-            if (key < Tg) { mx0 = max(mx0, S[nt][0]); mx1 = max(mx1, S[nt][2]); }
-            if (key + 1 < Tg) { mx0 = max(mx0, S[nt][1]); mx1 = max(mx1, S[nt][3]); }
+            const int key = kb * KB + nt * 8 + 2 * t;
+            if (key < Tg) { mx0 = fmaxf(mx0, S[nt][0]); mx1 = fmaxf(mx1, S[nt][2]); }
+            if (key + 1 < Tg) { mx0 = fmaxf(mx0, S[nt][1]); mx1 = fmaxf(mx1, S[nt][3]); }
         }
         __syncthreads();
     }
-    mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-    mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-    mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+    const int32_t imx0 = __float2int_rn(mx0), imx1 = __float2int_rn(mx1);
 
-    // ---- pass 2: S_sum = sum ShiftExp(s - max) (|scores| <= dh 127^2 < 2^20: no clamp needed)
+    // ---- pass 2: S_sum = sum ShiftExp(s - max)
     const ShiftExpC se = p.smx.se;
     uint64_t sum0 = 0, sum1 = 0;
     for (int kb = 0; kb < nkb; ++kb) {
-        load_k(kb);
-        cp_async_commit();
-        cp_async_wait_all();
+        stage(kb, false);
         __syncthreads();
-        int32_t S[8][4];
+        float S[8][4];
         scores(S);
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt) {
-            int key = kb * KB + nt * 8 + 2 * t;
+            const int key = kb * KB + nt * 8 + 2 * t;
             if (key < Tg) {
-                sum0 += shift_exp_mag((uint32_t)(mx0 - S[nt][0]), se);
-                sum1 += shift_exp_mag((uint32_t)(mx1 - S[nt][2]), se);
+                sum0 += shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][0])), se);
+                sum1 += shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][2])), se);
             }
             if (key + 1 < Tg) {
-                sum0 += shift_exp_mag((uint32_t)(mx0 - S[nt][1]), se);
-                sum1 += shift_exp_mag((uint32_t)(mx1 - S[nt][3]), se);
+                sum0 += shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][1])), se);
+                sum1 += shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][3])), se);
             }
         }
         __syncthreads();
@@ -188,62 +221,46 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
     sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
     sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
     sum1 += __shfl_xor_sync(0xffffffffu, sum1, 2);
-    // rows past Tg have sum 0: give them a harmless normaliser (their outputs are not stored)
+    // rows past Tg see sum >= 1 too (their max is over valid keys); their outputs are not stored
     const RowNorm rn0 = shiftmax_norm(sum0 ? sum0 : 1, p.smx.s_d, p.smx.m_p, p.smx.M_hw, p.smx.k_out);
     const RowNorm rn1 = shiftmax_norm(sum1 ? sum1 : 1, p.smx.s_d, p.smx.m_p, p.smx.M_hw, p.smx.k_out);
 
-    // ---- pass 3: P = (I_exp F) >> sh, O += P V
-    int32_t o[NT][4];
+    // ---- pass 3: P = (I_exp F) >> sh (exact integers < 256), O += P V
+    float o[NT][4];
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0;
+    for (int nt = 0; nt < NT; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
     for (int kb = 0; kb < nkb; ++kb) {
-        load_k(kb);
-        load_v(kb);
-        cp_async_commit();
-        cp_async_wait_all();
+        stage(kb, true);
         __syncthreads();
-        // transpose V into Vt[dim][slot] with the k-slot permutation of the P fragments
-        for (int m = tid; m < 16 * (DH / 4); m += THREADS) {
-            int kg = m & 15, dq = m >> 4;
-            int ch = kg >> 3, half = (kg >> 2) & 1, tt = kg & 3;
-            int k0 = ch * 32 + half * 16 + 2 * tt;
-            uint32_t w0 = *(const uint32_t *)(Vr + (k0 + 0) * LDK + 4 * dq);
-            uint32_t w1 = *(const uint32_t *)(Vr + (k0 + 1) * LDK + 4 * dq);
-            uint32_t w2 = *(const uint32_t *)(Vr + (k0 + 8) * LDK + 4 * dq);
-            uint32_t w3 = *(const uint32_t *)(Vr + (k0 + 9) * LDK + 4 * dq);
-            uint32_t t0 = __byte_perm(w0, w1, 0x5140), t1 = __byte_perm(w2, w3, 0x5140);
-            uint32_t t2 = __byte_perm(w0, w1, 0x7362), t3 = __byte_perm(w2, w3, 0x7362);
-            int sw = ch * 8 + half * 4 + tt;
-            *(uint32_t *)(Vt + (4 * dq + 0) * LDV + 4 * sw) = __byte_perm(t0, t1, 0x5410);
-            *(uint32_t *)(Vt + (4 * dq + 1) * LDV + 4 * sw) = __byte_perm(t0, t1, 0x7632);
-            *(uint32_t *)(Vt + (4 * dq + 2) * LDV + 4 * sw) = __byte_perm(t2, t3, 0x5410);
-            *(uint32_t *)(Vt + (4 * dq + 3) * LDV + 4 * sw) = __byte_perm(t2, t3, 0x7632);
-        }
-        __syncthreads();
-        int32_t S[8][4];
+        float S[8][4];
         scores(S);
-        uint32_t pv[8][4];
+        uint32_t pa[4][4];  // A fragments of P for the 4 k16 steps (16 keys each)
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt) {
-            int key = kb * KB + nt * 8 + 2 * t;
-            bool v0 = key < Tg, v1 = key + 1 < Tg;
-            pv[nt][0] = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(mx0 - S[nt][0]), se), rn0) : 0u;
-            pv[nt][1] = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(mx0 - S[nt][1]), se), rn0) : 0u;
-            pv[nt][2] = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(mx1 - S[nt][2]), se), rn1) : 0u;
-            pv[nt][3] = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(mx1 - S[nt][3]), se), rn1) : 0u;
+            const int key = kb * KB + nt * 8 + 2 * t;
+            const bool v0 = key < Tg, v1 = key + 1 < Tg;
+            const uint32_t p0 = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][0])), se), rn0) : 0u;
+            const uint32_t p1 = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][1])), se), rn0) : 0u;
+            const uint32_t p2 = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][2])), se), rn1) : 0u;
+            const uint32_t p3 = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][3])), se), rn1) : 0u;
+            // n-tile nt covers keys 8nt..8nt+7 = half (nt & 1) of k16 step nt >> 1
+            pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(p0, p1);  // row g
+            pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(p2, p3);  // row g + 8
         }
 #pragma unroll
-        for (int ch = 0; ch < 2; ++ch) {
-            uint32_t a[4];
-            const int n0 = 4 * ch;
-            a[0] = pv[n0][0] | (pv[n0][1] << 8) | (pv[n0 + 1][0] << 16) | (pv[n0 + 1][1] << 24);
-            a[1] = pv[n0][2] | (pv[n0][3] << 8) | (pv[n0 + 1][2] << 16) | (pv[n0 + 1][3] << 24);
-            a[2] = pv[n0 + 2][0] | (pv[n0 + 2][1] << 8) | (pv[n0 + 3][0] << 16) | (pv[n0 + 3][1] << 24);
-            a[3] = pv[n0 + 2][2] | (pv[n0 + 2][3] << 8) | (pv[n0 + 3][2] << 16) | (pv[n0 + 3][3] << 24);
+        for (int kk = 0; kk < 4; ++kk) {
+            // A fragment order for m16n8k16: {row g k lo, row g+8 k lo, row g k hi, row g+8 k hi}
+            const uint32_t a[4] = {pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3]};
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const int8_t *v = Vt + (nt * 8 + g) * LDV + ch * 32 + 4 * t;
-                mma_u8s8(o[nt], a, *(const uint32_t *)v, *(const uint32_t *)(v + 16));
+            for (int np = 0; np < NT / 2; ++np) {
+                // V rows = keys 16kk.., cols = dims 16np..: transposed 8x8 matrices give B fragments
+                const int i = lane >> 3;
+                const uint32_t row = 16 * kk + 8 * (i & 1) + (lane & 7);
+                const uint32_t addr = vs_base + row * LDH + (16 * np + 8 * (i >> 1)) * 2;
+                uint32_t r0, r1, r2, r3;
+                ldsm_x4_t(addr, r0, r1, r2, r3);  // r0: k lo, n 16np..; r1: k hi, n 16np..; r2/r3: n 16np+8..
+                mma_f16(o[2 * np], a, r0, r1);
+                mma_f16(o[2 * np + 1], a, r2, r3);
             }
         }
         __syncthreads();
@@ -256,14 +273,16 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
     int8_t *O1 = ok1 ? p.O + gr.token(r1) * p.ld_o + hoff : nullptr;
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
-        int col = nt * 8 + 2 * t;
+        const int col = nt * 8 + 2 * t;
         if (ok0) {
-            O0[col] = (int8_t)sat8(rq(o[nt][0], p.m_o, p.s_o));
-            O0[col + 1] = (int8_t)sat8(rq(o[nt][1], p.m_o, p.s_o));
+            const int32_t a0 = sat8(rq(__float2int_rn(o[nt][0]), p.m_o, p.s_o));
+            const int32_t a1 = sat8(rq(__float2int_rn(o[nt][1]), p.m_o, p.s_o));
+            *(uint16_t *)(O0 + col) = (uint16_t)((uint8_t)a0 | ((uint32_t)(uint8_t)a1 << 8));
         }
         if (ok1) {
-            O1[col] = (int8_t)sat8(rq(o[nt][2], p.m_o, p.s_o));
-            O1[col + 1] = (int8_t)sat8(rq(o[nt][3], p.m_o, p.s_o));
+            const int32_t a2 = sat8(rq(__float2int_rn(o[nt][2]), p.m_o, p.s_o));
+            const int32_t a3 = sat8(rq(__float2int_rn(o[nt][3]), p.m_o, p.s_o));
+            *(uint16_t *)(O1 + col) = (uint16_t)((uint8_t)a2 | ((uint32_t)(uint8_t)a3 << 8));
         }
     }
 }
