@@ -1,0 +1,121 @@
+"""Single-kernel workloads of the path, for timing and for profiler captures.
+
+  python -m paper_2607_24981_gb300.cases <case> [--reps N]
+
+Each case builds its seeded inputs (shapes of the paper's Medium model and of the nonlinearity
+sweep), runs the entry point `reps` times after 3 warm-up calls and prints the mean device time
+with the case's algorithmic work.  Cases:
+  attn_global   attention, 2 images x 1600 tokens, 6 heads, dh 64, global
+  attn_window   attention, 8 images x 1600 tokens, 6 heads, 2x2 windows of 400
+  gemm_qkv / gemm_proj / gemm_fc1_gelu / gemm_fc2
+                the block GEMMs at 12800 tokens, d 384, MLP 1536
+  ln_c2         I-LayerNorm on the int16 residual stream, 12800 x 384
+  smx_64 / smx_400 / smx_1600
+                Constrained Shiftmax over 2^27 int32 scores in rows of 64 / 400 / 1600
+  gelu_c3       SD-ShiftGELU over 2^28 int32 values
+  ln_192 / ln_384
+                I-LayerNorm over 2^20 int32 rows of dim 192 / 384
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+import numpy as np
+
+from . import synth
+
+
+def _dev(a):
+    import torch
+
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def build(case: str):
+    """Returns (fn, work dict) for a case; fn() launches the entry point once."""
+    import torch
+
+    import paper_2607_24981_gb300 as ilw
+
+    ilw.lib()
+    if case.startswith("attn"):
+        B, T, H, dh = (2, 1600, 6, 64) if case == "attn_global" else (8, 1600, 6, 64)
+        win = 0 if case == "attn_global" else 2
+        qkv = _dev(synth.uniform_int(0, "case.qkv", (B * T, 3 * H * dh), -127, 127, np.int8))
+        out = torch.empty((B * T, H * dh), dtype=torch.int8, device="cuda")
+        scores = B * H * (T * T if win == 0 else 4 * (T // 4) ** 2)
+        return (lambda: ilw.shiftmax_attn(qkv, B, T, H, dh, win, {"I0": 6000}, 3 << 29, 36, out=out),
+                {"scores": scores})
+    if case.startswith("gemm"):
+        M, d, F = 12800, 384, 1536
+        N, K = {"gemm_qkv": (3 * d, d), "gemm_proj": (d, d), "gemm_fc1_gelu": (F, d), "gemm_fc2": (d, F)}[case]
+        A = _dev(synth.uniform_int(1, "case.A", (M, K), -127, 127, np.int8))
+        W, b, m, s = synth.gemm_params(1, "case.W", N, K, 40.0, 40.0)
+        Wp = ilw.pack_weight(_dev(W))
+        b, m, s = _dev(b), _dev(m), _dev(s)
+        if case == "gemm_fc1_gelu":
+            out = torch.empty((M, N), dtype=torch.int8, device="cuda")
+            fn = lambda: ilw.gemm_gelu(A, Wp, N, b, m, s, {"I0": 1000}, 3 << 29, 40, out=out)
+        elif case == "gemm_qkv":
+            out = torch.empty((M, N), dtype=torch.int8, device="cuda")
+            fn = lambda: ilw.gemm_requant(A, Wp, N, b, m, s, 8, out=out)
+        else:
+            res = _dev(synth.uniform_int(1, "case.res", (M, N), -3000, 3000, np.int16))
+            out = torch.empty((M, N), dtype=torch.int16, device="cuda")
+            fn = lambda: ilw.gemm_requant(A, Wp, N, b, m, s, 16, res=res, m_r=1 << 30, s_r=31, out=out)
+        return fn, {"flops": 2.0 * M * N * K}
+    if case.startswith("smx"):
+        L = int(case.split("_")[1])
+        X = _dev(synth.uniform_int(30, f"c3smx{L}", ((1 << 27) // L, L), -(1 << 15), 1 << 15))
+        P = torch.empty(X.shape, dtype=torch.uint8, device="cuda")
+        return (lambda: ilw.shiftmax_rows(X, {"I0": 3000}, out=P)), {"bytes": 5.0 * X.numel()}
+    if case == "gelu_c3":
+        X = _dev(synth.uniform_int(32, "c3gelu", (1 << 28,), -(1 << 12), 1 << 12))
+        Y = torch.empty_like(X)
+        return (lambda: ilw.sdshiftgelu(X, {"I0": 600}, out=Y)), {"bytes": 8.0 * X.numel()}
+    if case.startswith("ln"):
+        if case == "ln_c2":
+            X = _dev(synth.uniform_int(34, "case.ln", (12800, 384), -3000, 3000, np.int16))
+            per = 3.0
+        else:
+            C = int(case.split("_")[1])
+            X = _dev(synth.uniform_int(34, f"c3ln{C}", (1 << 20, C), -(1 << 14), 1 << 14))
+            per = 5.0
+        C = X.shape[1]
+        beta, mult, shift = (_dev(a) for a in synth.ln_params(34, f"c3lnp{C}", C))
+        Y = torch.empty(X.shape, dtype=torch.int8, device="cuda")
+        return (lambda: ilw.int_layernorm(X, beta, mult, shift, 10, 8, out=Y)), {"bytes": per * X.numel()}
+    raise SystemExit(f"unknown case {case}")
+
+
+def main(argv=None):
+    import torch
+
+    ap = argparse.ArgumentParser()
+    ap.add_argument("case")
+    ap.add_argument("--reps", type=int, default=10)
+    a = ap.parse_args(argv)
+    fn, work = build(a.case)
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(a.reps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / max(a.reps, 1)
+    out = {"case": a.case, "us": ms * 1000.0}
+    if "flops" in work:
+        out["tflops"] = work["flops"] / (ms / 1000.0) / 1e12
+    if "bytes" in work:
+        out["gbs"] = work["bytes"] / (ms / 1000.0) / 1e9
+    if "scores" in work:
+        out["gscores_s"] = work["scores"] / (ms / 1000.0) / 1e9
+    print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -441,6 +441,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     }
 }
 
+// int8 weight -> fp16 operand copy (|w| <= 127: exact)
+__global__ void pack_weight_kernel(const int8_t *W, int64_t n, __half *w16) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) w16[i] = __int2half_rn((int)W[i]);
+}
+
 // ------------------------------------------------------------------ host side
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
@@ -545,6 +551,12 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
 }
 
 }  // namespace
+
+cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, cudaStream_t s) {
+    const int64_t n = (int64_t)N * K;
+    pack_weight_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(W, n, (__half *)packed);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     if (gp.M == 0 || gp.N == 0) return cudaSuccess;

@@ -86,18 +86,13 @@ __device__ __forceinline__ int32_t epi_value(const EpiParams &ep, int64_t row, i
     return ep.out_bits == 8 ? sat8(o) : sat16(o);
 }
 
-// Packed weight layout: [int8 W, N*K bytes][pad to 256][fp16 W, N*K*2 bytes].
-size_t packed_weight_bytes(int32_t N, int32_t K);
-inline const int8_t *packed_i8(const void *p) { return (const int8_t *)p; }
-inline const void *packed_f16(const void *p, int32_t N, int32_t K) {
-    size_t off = (((size_t)N * K) + 255) & ~(size_t)255;
-    return (const char *)p + off;
-}
+// Packed weight layout: the same integers as fp16 [N, K] (row-major), the tensor-core operand.
+inline size_t packed_weight_bytes(int32_t N, int32_t K) { return (size_t)N * K * 2; }
+inline const int8_t *packed_i8(const void *) { return nullptr; }
+inline const void *packed_f16(const void *p, int32_t, int32_t) { return p; }
 cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, cudaStream_t s);
 // tcgen05 tensor-core GEMM (exact integer via fp16 operands, fp32 TMEM accumulators)
 cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s);
-// warp-level int8 MMA GEMM (mma.sync m16n8k32), kept as the measured legacy-path baseline
-cudaError_t launch_gemm_mma(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s);
 
 // ---------------------------------------------------------------- row / element kernels
 struct ShiftmaxC {
