@@ -76,13 +76,14 @@ struct Group {
 };
 
 template <int DH>
-__global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
+__global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     constexpr int LDH = DH * 2 + 16;  // padded fp16 row (bytes): conflict-free ldmatrix
     constexpr int KS = DH / 16;       // k16 steps of q k^T
     constexpr int NT = DH / 8;        // n-tiles of P V
     constexpr int CH = DH / 16;       // 16-byte int8 chunks per row
-    __shared__ __align__(16) uint8_t Ks[KB * LDH];
-    __shared__ __align__(16) uint8_t Vs[KB * LDH];
+    constexpr int PER = KB * CH / THREADS;  // 16-byte int8 chunks per thread per key block
+    __shared__ __align__(16) uint8_t Ks[2][KB * LDH];
+    __shared__ __align__(16) uint8_t Vs[2][KB * LDH];
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, t = lane & 3;
@@ -123,32 +124,43 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
     }
 
     const int nkb = (Tg + KB - 1) / KB;
-    // stage one 64-key block of K (and V) as fp16 rows
-    auto stage = [&](int kb, bool with_v) {
-        for (int c = tid; c < KB * CH; c += THREADS) {
+    // Key blocks go global (int8) -> registers -> shared (fp16), double buffered: the loads of
+    // block kb+1 are in flight while block kb is computed.
+    uint4 kreg[PER], vreg[PER];
+    auto fetch = [&](int kb, bool with_v) {
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int c = tid + i * THREADS;
             const int r = c / CH, ch = c % CH;
             const int key = kb * KB + r;
-            uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
+            kreg[i] = make_uint4(0, 0, 0, 0);
+            vreg[i] = make_uint4(0, 0, 0, 0);
             if (key < Tg) {
                 const int64_t off = gr.token(key) * p.ld_qkv + hoff + ch * 16;
-                kv = __ldg((const uint4 *)(p.K + off));
-                if (with_v) vv = __ldg((const uint4 *)(p.V + off));
-            }
-            uint4 lo, hi;
-            i8x16_to_h16(kv, lo, hi);
-            *(uint4 *)(Ks + r * LDH + ch * 32) = lo;
-            *(uint4 *)(Ks + r * LDH + ch * 32 + 16) = hi;
-            if (with_v) {
-                i8x16_to_h16(vv, lo, hi);
-                *(uint4 *)(Vs + r * LDH + ch * 32) = lo;
-                *(uint4 *)(Vs + r * LDH + ch * 32 + 16) = hi;
+                kreg[i] = __ldg((const uint4 *)(p.K + off));
+                if (with_v) vreg[i] = __ldg((const uint4 *)(p.V + off));
             }
         }
     };
-    const uint32_t ks_base = (uint32_t)__cvta_generic_to_shared(Ks);
-    const uint32_t vs_base = (uint32_t)__cvta_generic_to_shared(Vs);
-    // scores of this warp's 16 rows x the 64 keys of the staged block (exact integers in fp32)
-    auto scores = [&](float (&S)[8][4]) {
+    auto commit = [&](int buf, bool with_v) {
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const int c = tid + i * THREADS;
+            const int r = c / CH, ch = c % CH;
+            uint4 lo, hi;
+            i8x16_to_h16(kreg[i], lo, hi);
+            *(uint4 *)(Ks[buf] + r * LDH + ch * 32) = lo;
+            *(uint4 *)(Ks[buf] + r * LDH + ch * 32 + 16) = hi;
+            if (with_v) {
+                i8x16_to_h16(vreg[i], lo, hi);
+                *(uint4 *)(Vs[buf] + r * LDH + ch * 32) = lo;
+                *(uint4 *)(Vs[buf] + r * LDH + ch * 32 + 16) = hi;
+            }
+        }
+    };
+    // scores of this warp's 16 rows x the 64 keys of buffer `buf` (exact integers in fp32)
+    auto scores = [&](int buf, float (&S)[8][4]) {
+        const uint32_t ks_base = (uint32_t)__cvta_generic_to_shared(Ks[buf]);
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt) S[nt][0] = S[nt][1] = S[nt][2] = S[nt][3] = 0.f;
 #pragma unroll
@@ -156,15 +168,13 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
 #pragma unroll
             for (int kp = 0; kp < KS; kp += 2) {  // pairs of k16 steps (32 dims)
                 // matrices: keys [16np + 8(i&1) ...], dims [16kp + 8(i>>1) ...]
-                uint32_t b[4][2];
                 const int i = lane >> 3;
                 const uint32_t row = 16 * np + 8 * (i & 1) + (lane & 7);
                 const uint32_t addr = ks_base + row * LDH + (16 * kp + 8 * (i >> 1)) * 2;
                 uint32_t r0, r1, r2, r3;
                 ldsm_x4(addr, r0, r1, r2, r3);  // r0: n-tile 2np, k lo; r1: 2np+1, k lo; r2, r3: k hi
-                b[0][0] = r0; b[1][0] = r1; b[0][1] = r2; b[1][1] = r3;
-                mma_f16(S[2 * np], qa[kp], b[0][0], b[0][1]);
-                mma_f16(S[2 * np + 1], qa[kp], b[1][0], b[1][1]);
+                mma_f16(S[2 * np], qa[kp], r0, r2);
+                mma_f16(S[2 * np + 1], qa[kp], r1, r3);
                 if (kp + 1 < KS) {
                     ldsm_x4(addr + 16 * 2, r0, r1, r2, r3);  // next k16 step: 16 dims further
                     mma_f16(S[2 * np], qa[kp + 1], r0, r2);
@@ -173,22 +183,40 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
             }
         }
     };
+    // one pass over the key blocks: body(kb, buf, full) with the block staged in buffer buf
+    auto sweep = [&](bool with_v, auto &&body) {
+        fetch(0, with_v);
+        commit(0, with_v);
+        __syncthreads();
+        for (int kb = 0; kb < nkb; ++kb) {
+            const int buf = kb & 1;
+            if (kb + 1 < nkb) fetch(kb + 1, with_v);
+            body(kb, buf, (kb + 1) * KB <= Tg);
+            if (kb + 1 < nkb) commit(buf ^ 1, with_v);  // buffer buf^1 was released by the last sync
+            __syncthreads();
+        }
+    };
 
     // ---- pass 1: exact row maxima
     float mx0 = -3.0e38f, mx1 = -3.0e38f;
-    for (int kb = 0; kb < nkb; ++kb) {
-        stage(kb, false);
-        __syncthreads();
+    sweep(false, [&](int kb, int buf, bool full) {
         float S[8][4];
-        scores(S);
+        scores(buf, S);
+        if (full) {
 #pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            const int key = kb * KB + nt * 8 + 2 * t;
-            if (key < Tg) { mx0 = fmaxf(mx0, S[nt][0]); mx1 = fmaxf(mx1, S[nt][2]); }
-            if (key + 1 < Tg) { mx0 = fmaxf(mx0, S[nt][1]); mx1 = fmaxf(mx1, S[nt][3]); }
+            for (int nt = 0; nt < 8; ++nt) {
+                mx0 = fmaxf(mx0, fmaxf(S[nt][0], S[nt][1]));
+                mx1 = fmaxf(mx1, fmaxf(S[nt][2], S[nt][3]));
+            }
+        } else {
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                const int key = kb * KB + nt * 8 + 2 * t;
+                if (key < Tg) { mx0 = fmaxf(mx0, S[nt][0]); mx1 = fmaxf(mx1, S[nt][2]); }
+                if (key + 1 < Tg) { mx0 = fmaxf(mx0, S[nt][1]); mx1 = fmaxf(mx1, S[nt][3]); }
+            }
         }
-        __syncthreads();
-    }
+    });
     mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
     mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
     mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
@@ -198,25 +226,21 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
     // ---- pass 2: S_sum = sum ShiftExp(s - max)
     const ShiftExpC se = p.smx.se;
     uint64_t sum0 = 0, sum1 = 0;
-    for (int kb = 0; kb < nkb; ++kb) {
-        stage(kb, false);
-        __syncthreads();
+    sweep(false, [&](int kb, int buf, bool full) {
         float S[8][4];
-        scores(S);
+        scores(buf, S);
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt) {
             const int key = kb * KB + nt * 8 + 2 * t;
-            if (key < Tg) {
-                sum0 += shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][0])), se);
-                sum1 += shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][2])), se);
-            }
-            if (key + 1 < Tg) {
-                sum0 += shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][1])), se);
-                sum1 += shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][3])), se);
-            }
+            const bool v0 = full || key < Tg, v1 = full || key + 1 < Tg;
+            const uint32_t e0 = shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][0])), se);
+            const uint32_t e1 = shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][1])), se);
+            const uint32_t e2 = shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][2])), se);
+            const uint32_t e3 = shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][3])), se);
+            sum0 += (uint64_t)(v0 ? e0 : 0u) + (v1 ? e1 : 0u);
+            sum1 += (uint64_t)(v0 ? e2 : 0u) + (v1 ? e3 : 0u);
         }
-        __syncthreads();
-    }
+    });
     sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
     sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
     sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
@@ -229,16 +253,14 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
     float o[NT][4];
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
-    for (int kb = 0; kb < nkb; ++kb) {
-        stage(kb, true);
-        __syncthreads();
+    sweep(true, [&](int kb, int buf, bool full) {
         float S[8][4];
-        scores(S);
+        scores(buf, S);
         uint32_t pa[4][4];  // A fragments of P for the 4 k16 steps (16 keys each)
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt) {
             const int key = kb * KB + nt * 8 + 2 * t;
-            const bool v0 = key < Tg, v1 = key + 1 < Tg;
+            const bool v0 = full || key < Tg, v1 = full || key + 1 < Tg;
             const uint32_t p0 = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][0])), se), rn0) : 0u;
             const uint32_t p1 = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][1])), se), rn0) : 0u;
             const uint32_t p2 = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][2])), se), rn1) : 0u;
@@ -247,6 +269,7 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
             pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(p0, p1);  // row g
             pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(p2, p3);  // row g + 8
         }
+        const uint32_t vs_base = (uint32_t)__cvta_generic_to_shared(Vs[buf]);
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
             // A fragment order for m16n8k16: {row g k lo, row g+8 k lo, row g k hi, row g+8 k hi}
@@ -263,8 +286,7 @@ __global__ void __launch_bounds__(THREADS) attn_kernel(const AttnParams p) {
                 mma_f16(o[2 * np + 1], a, r2, r3);
             }
         }
-        __syncthreads();
-    }
+    });
 
     // ---- epilogue: sat8(rq(O; m_o, s_o)), written back at the tokens' own positions
     const int r0 = q0 + warp * 16 + g, r1 = r0 + 8;

@@ -57,6 +57,7 @@ struct TcParams {  // CUtensorMap members keep the 64-byte alignment TMA needs
     int32_t tiles_n, tiles;
     int32_t nbuf;       // TMEM accumulator sets (1 or 2)
     int32_t tmem_cols;
+    int32_t gelu_T;     // SD-ShiftGELU table covers g in [-gelu_T, gelu_T] (constant beyond)
     int *status;
     EpiParams ep;
 };
@@ -177,12 +178,13 @@ enum { KIND_RQ8 = 0, KIND_RQ16 = 1, KIND_RAW32 = 2, KIND_GELU8 = 3 };
 
 template <int KIND>
 __device__ __forceinline__ int32_t epi_one(const EpiParams &ep, int64_t row, int32_t acc, int32_t bias, int32_t mult,
-                                           int32_t shift, int32_t col) {
+                                           int32_t shift, int32_t col, const uint8_t *gtab, int32_t gT) {
     const int64_t v = (int64_t)acc + bias;
     if (KIND == KIND_RAW32) return (int32_t)v;
     if (KIND == KIND_GELU8) {
         const int32_t g = sat16(rq(v, mult, shift));
-        return sat8(rq((int64_t)g * gelu_idiv(g, ep.gelu), ep.m_g, ep.s_g));
+        const int32_t idiv = gtab[min(max(g, -gT), gT) + gT];  // = gelu_idiv(g) (tabulated below)
+        return sat8(rq((int64_t)g * idiv, ep.m_g, ep.s_g));
     }
     int64_t o = rq(v, mult, shift);
     if (ep.res) o += rq((int64_t)ep.res[(row % ep.res_rows) * ep.ldr + col], ep.m_r, ep.s_r);
@@ -230,6 +232,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // SD-ShiftGELU: I_div depends on the int16 value g alone and is constant once both ShiftExp
+    // inputs are clamped (|g| > gelu_T), so the epilogue warps tabulate it once per CTA with the
+    // same device function (exact by construction) and then look it up.
+    uint8_t *gtab = (uint8_t *)((int32_t *)(tmem_slot + 4) + 12 * BN);
+    if (KIND == KIND_GELU8 && warp >= 6) {
+        for (int i = threadIdx.x - 192; i <= 2 * p.gelu_T; i += 256) gtab[i] = (uint8_t)gelu_idiv(i - p.gelu_T, p.ep.gelu);
+        asm volatile("bar.sync 1, 256;" ::: "memory");  // the 8 epilogue warps only
+    }
     const int acc_cols = p.nseg * BN;  // columns of one accumulator set
 
     if (warp == 0) {
@@ -384,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 #pragma unroll
                     for (int i = 0; i < 16; ++i)
                         out[i] = epi_one<KIND>(ep, row, acc[i], s_bias[c0 + i], s_mult[c0 + i], s_shift[c0 + i],
-                                               min(n0 + c0 + i, p.N - 1));
+                                               min(n0 + c0 + i, p.N - 1), gtab, p.gelu_T);
                     char *dst = (char *)ep.C + (row * ep.ldc + n0 + c0) * (bits / 8);
                     const bool vec = ncol == 16 && (((uintptr_t)dst & 15) == 0);
                     if constexpr (bits == 8) {
@@ -491,7 +501,8 @@ int num_sms() {
 
 template <int BN, int STAGES, int KIND>
 cudaError_t launch_tc(TcParams &tp, cudaStream_t s) {
-    const size_t smem = 1024 + (size_t)STAGES * Smem<BN>::kStage + 8 * (3 * STAGES + 4) + 16 + 4 * 3 * BN * 4;
+    const size_t smem = 1024 + (size_t)STAGES * Smem<BN>::kStage + 8 * (3 * STAGES + 4) + 16 + 4 * 3 * BN * 4 +
+                        (KIND == KIND_GELU8 ? 65536 : 0);
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
@@ -544,6 +555,13 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     while (alloc < tp.nbuf * one) alloc <<= 1;
     if (alloc > 512) return cudaErrorInvalidValue;
     tp.tmem_cols = alloc;
+    if (ep.kind == EPI_GELU) {
+        // |g| > T puts both ShiftExp inputs past the clamp: |I_p| >= 1.6875|g| - 3 and
+        // -I_e >= 1.4375|I_p| - 1 >= k I0 once |g| >= ((k I0 + 1)/1.4375 + 3)/1.6875; 0.7 (k I0 + 1) + 8
+        // is above that bound.  g is int16, so T never needs to exceed 32767.
+        const double bound = 0.7 * ((double)ep.gelu.se.kI0 + 1.0) + 8.0;
+        tp.gelu_T = bound > 32767.0 ? 32767 : (int32_t)bound;
+    }
     if (ep.kind == EPI_GELU) return launch_tc<BN, STAGES, KIND_GELU8>(tp, s);
     if (ep.out_bits == 8) return launch_tc<BN, STAGES, KIND_RQ8>(tp, s);
     if (ep.out_bits == 16) return launch_tc<BN, STAGES, KIND_RQ16>(tp, s);
@@ -561,8 +579,9 @@ cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *pack
 cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     if (gp.M == 0 || gp.N == 0) return cudaSuccess;
     // 192-wide tiles when N splits evenly into them (fewer re-reads of A per flop), else 128
-    if (gp.N % 192 == 0 && gp.N >= 768 && gp.nb == 1) return run<192, 4>(gp, ep, s);
-    return run<128, 5>(gp, ep, s);
+    if (gp.N % 192 == 0 && gp.N >= 768 && gp.nb == 1)
+        return ep.kind == EPI_GELU ? run<192, 3>(gp, ep, s) : run<192, 4>(gp, ep, s);
+    return ep.kind == EPI_GELU ? run<128, 3>(gp, ep, s) : run<128, 5>(gp, ep, s);
 }
 
 }  // namespace ilw

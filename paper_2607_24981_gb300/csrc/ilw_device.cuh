@@ -78,8 +78,11 @@ __device__ __forceinline__ RowNorm shiftmax_norm(uint64_t S_sum, int32_t s_d_sta
     rn.sh = 31 - k_out + 1 + s_d;
     return rn;
 }
+// (e * F) >> sh for e, F < 2^31 and sh >= 24 (k_out <= 8): from the 32-bit halves of the
+// product, so no 64-bit shift is needed (e * F < 2^62, so any sh >= 63 gives 0).
 __device__ __forceinline__ uint32_t shiftmax_out(uint32_t e, const RowNorm &rn) {
-    return (uint32_t)(((uint64_t)e * rn.F) >> rn.sh);
+    const uint32_t lo = e * rn.F, hi = __umulhi(e, rn.F);
+    return rn.sh < 32 ? __funnelshift_r(lo, hi, rn.sh) : (hi >> min(rn.sh - 32, 31));
 }
 
 // ---- SD-ShiftGELU sigmoid factor I_div (Algorithm 1), for |x| < 2^26 (callers clamp: beyond

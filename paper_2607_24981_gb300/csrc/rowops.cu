@@ -30,53 +30,70 @@ __device__ __forceinline__ int64_t warp_sum_i64(int64_t v) {
 // ------------------------------------------------------------------ Constrained Shiftmax rows
 // NCH = 4-element chunks per lane (row length <= 128 * NCH); vector loads need len % 4 == 0
 // and 16-byte aligned rows.
-template <int NCH>
+template <int LANES>
+__device__ __forceinline__ int32_t group_max(int32_t v) {
+#pragma unroll
+    for (int o = LANES / 2; o; o >>= 1) v = max(v, __shfl_xor_sync(0xffffffffu, v, o, LANES));
+    return v;
+}
+template <int LANES>
+__device__ __forceinline__ uint64_t group_sum_u64(uint64_t v) {
+#pragma unroll
+    for (int o = LANES / 2; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o, LANES);
+    return v;
+}
+
+// LANES lanes own one row (32 / LANES rows per warp); NCH = 4-element chunks per lane (row length
+// <= 4 * LANES * NCH).  Vector loads need len % 4 == 0 and 16-byte aligned rows.
+template <int NCH, int LANES>
 __global__ void __launch_bounds__(256) shiftmax_rows_vec(const int32_t *__restrict__ X, int64_t ldx,
                                                           int64_t rows, int32_t len, const ShiftmaxC c,
                                                           uint8_t *__restrict__ P, int64_t ldp) {
-    const int lane = threadIdx.x & 31;
-    const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (row >= rows) return;
-    const int nch = len >> 2;
-    const int4 *xr = (const int4 *)(X + row * ldx);
+    constexpr int RPW = 32 / LANES;
+    const int lane = threadIdx.x & 31, sub = lane % LANES;
+    const int64_t row = ((int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * RPW + lane / LANES;
+    const bool live = row < rows;  // every lane stays for the shuffles
+    const int nch = live ? (len >> 2) : 0;
+    const int4 *xr = (const int4 *)(X + (live ? row : 0) * ldx);
     int4 v[NCH];
     int32_t mx = INT_MIN;
 #pragma unroll
     for (int j = 0; j < NCH; ++j) {
-        int ch = lane + 32 * j;
+        const int ch = sub + LANES * j;
         if (ch < nch) {
             v[j] = __ldcs(xr + ch);
             mx = max(mx, max(max(v[j].x, v[j].y), max(v[j].z, v[j].w)));
         }
     }
-    mx = warp_max(mx);
+    mx = group_max<LANES>(mx);
     // differences below -2^30 are deep in ShiftExp's clamp region: use -2^30 there
     const int32_t lowb = mx > INT_MIN + (1 << 30) ? mx - (1 << 30) : INT_MIN;
     uint64_t sum = 0;
 #pragma unroll
     for (int j = 0; j < NCH; ++j) {
-        int ch = lane + 32 * j;
+        const int ch = sub + LANES * j;
         if (ch < nch) {
             int32_t *e = (int32_t *)&v[j];
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                uint32_t a = e[q] > lowb ? (uint32_t)(mx - e[q]) : (1u << 30);
-                uint32_t ex = shift_exp_mag(a, c.se);
+                const uint32_t a = e[q] > lowb ? (uint32_t)(mx - e[q]) : (1u << 30);
+                const uint32_t ex = shift_exp_mag(a, c.se);
                 e[q] = (int32_t)ex;
                 sum += ex;
             }
         }
     }
-    sum = warp_sum_u64(sum);
+    sum = group_sum_u64<LANES>(sum);
+    if (!live) return;
     const RowNorm rn = shiftmax_norm(sum, c.s_d, c.m_p, c.M_hw, c.k_out);
     uint32_t *pr = (uint32_t *)(P + row * ldp);
 #pragma unroll
     for (int j = 0; j < NCH; ++j) {
-        int ch = lane + 32 * j;
+        const int ch = sub + LANES * j;
         if (ch < nch) {
             const int32_t *e = (const int32_t *)&v[j];
-            uint32_t o = shiftmax_out((uint32_t)e[0], rn) | (shiftmax_out((uint32_t)e[1], rn) << 8) |
-                         (shiftmax_out((uint32_t)e[2], rn) << 16) | (shiftmax_out((uint32_t)e[3], rn) << 24);
+            const uint32_t o = shiftmax_out((uint32_t)e[0], rn) | (shiftmax_out((uint32_t)e[1], rn) << 8) |
+                               (shiftmax_out((uint32_t)e[2], rn) << 16) | (shiftmax_out((uint32_t)e[3], rn) << 24);
             __stcs(pr + ch, o);
         }
     }
@@ -125,12 +142,93 @@ __global__ void __launch_bounds__(256) sdshiftgelu_vec(const int4 *__restrict__ 
         __stcs(Y + i, o);
     }
 }
+// Table form: I_div depends on x alone and is constant for |x| >= T (both ShiftExp inputs are in
+// their clamp regions there), so each CTA tabulates I_div(x) for x in [-T, T] with the same device
+// function (exact by construction) and streams the data through lookups.
+__global__ void __launch_bounds__(256) sdshiftgelu_table(const int4 *__restrict__ X, int4 *__restrict__ Y, int64_t n4,
+                                                          const GeluC c, int32_t T) {
+    extern __shared__ uint8_t tab[];
+    for (int i = threadIdx.x; i <= 2 * T; i += blockDim.x) tab[i] = (uint8_t)gelu_idiv(i - T, c);
+    __syncthreads();
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+        const int4 v = __ldcs(X + i);
+        int4 o;
+        o.x = v.x * (int32_t)tab[min(max(v.x, -T), T) + T];
+        o.y = v.y * (int32_t)tab[min(max(v.y, -T), T) + T];
+        o.z = v.z * (int32_t)tab[min(max(v.z, -T), T) + T];
+        o.w = v.w * (int32_t)tab[min(max(v.w, -T), T) + T];
+        __stcs(Y + i, o);
+    }
+}
+
 __global__ void sdshiftgelu_tail(const int32_t *X, int32_t *Y, int64_t start, int64_t n, const GeluC c) {
     int64_t i = start + (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) Y[i] = gelu_one(X[i], c);
 }
 
 // ------------------------------------------------------------------ I-LayerNorm
+// Newton integer square root from 2^16, exactly `iters` steps, stopping only at 0 (V = 0).
+__device__ __forceinline__ uint64_t newton_isqrt(uint64_t V, int iters) {
+    uint64_t r = 1ull << 16;
+    for (int it = 0; it < iters; ++it) {
+        if (r == 0) break;
+        r = (r + V / r) >> 1;
+    }
+    return r < 1 ? 1 : r;
+}
+
+// ROWS rows per warp, held in registers: lanes share the loads and the two integer row sums,
+// then lane j runs Newton's iteration (the sequential part) for row j, so a warp pays for one
+// Newton sequence per ROWS rows.  V = sum (x - mu)^2 = sum x^2 - 2 mu sum x + C mu^2, exactly.
+template <typename TIn, typename TOut, int EPL, int ROWS>
+__global__ void __launch_bounds__(256) layernorm_multi(const LnParams p) {
+    const int lane = threadIdx.x & 31;
+    const int64_t row0 = ((int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * ROWS;
+    if (row0 >= p.rows) return;
+    const int C = p.C;
+    int32_t v[ROWS][EPL];
+    int64_t my_s = 0, my_q = 0;
+#pragma unroll
+    for (int r = 0; r < ROWS; ++r) {
+        const bool ok = row0 + r < p.rows;
+        const TIn *x = (const TIn *)p.X + (ok ? row0 + r : row0) * p.ldx;
+        int64_t s = 0, q = 0;
+#pragma unroll
+        for (int j = 0; j < EPL; ++j) {
+            const int c = lane + 32 * j;
+            v[r][j] = (ok && c < C) ? (int32_t)x[c] : 0;
+            s += v[r][j];
+            q += (int64_t)v[r][j] * v[r][j];
+        }
+        s = warp_sum_i64(s);
+        q = warp_sum_i64(q);
+        if (lane == r) { my_s = s; my_q = q; }
+    }
+    // lane r < ROWS: mean, variance and Newton for row r
+    const int64_t den = 2 * (int64_t)C, num = 2 * my_s + C;
+    int64_t mu = num / den;
+    if ((num % den) != 0 && num < 0) mu -= 1;
+    const uint64_t V = (uint64_t)(my_q - 2 * mu * my_s + (int64_t)C * mu * mu);
+    const uint64_t R = lane < ROWS ? newton_isqrt(V, p.iters) : 1;
+    const int64_t F = (int64_t)(0x7fffffffull / R);
+#pragma unroll
+    for (int r = 0; r < ROWS; ++r) {
+        if (row0 + r >= p.rows) break;
+        const int64_t mur = __shfl_sync(0xffffffffu, mu, r);
+        const int64_t Fr = __shfl_sync(0xffffffffu, F, r);
+        TOut *yo = (TOut *)p.Y + (row0 + r) * p.ldy;
+#pragma unroll
+        for (int j = 0; j < EPL; ++j) {
+            const int c = lane + 32 * j;
+            if (c < C) {
+                const int64_t n = (((int64_t)v[r][j] - mur) * Fr) >> 1;
+                const int64_t o = rq(n + p.beta[c], p.mult[c], p.shift[c]);
+                yo[c] = (TOut)(sizeof(TOut) == 1 ? sat8(o) : sat16(o));
+            }
+        }
+    }
+}
+
 template <typename TIn, typename TOut, int EPL>
 __global__ void __launch_bounds__(256) layernorm_kernel(const LnParams p) {
     const int lane = threadIdx.x & 31;
@@ -184,6 +282,15 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const LnParams p) {
 
 template <typename TIn, typename TOut>
 cudaError_t ln_dispatch(const LnParams &p, cudaStream_t s) {
+    if (p.C <= 512) {  // 4 rows per warp in registers, lane-parallel Newton
+        constexpr int ROWS = 4;
+        dim3 g4((unsigned)((p.rows + 8 * ROWS - 1) / (8 * ROWS)));
+        if (p.C <= 128) layernorm_multi<TIn, TOut, 4, ROWS><<<g4, 256, 0, s>>>(p);
+        else if (p.C <= 256) layernorm_multi<TIn, TOut, 8, ROWS><<<g4, 256, 0, s>>>(p);
+        else if (p.C <= 384) layernorm_multi<TIn, TOut, 12, ROWS><<<g4, 256, 0, s>>>(p);
+        else layernorm_multi<TIn, TOut, 16, ROWS><<<g4, 256, 0, s>>>(p);
+        return cudaGetLastError();
+    }
     const int rows_per_block = 8;
     dim3 grid((unsigned)((p.rows + rows_per_block - 1) / rows_per_block));
     if (p.C <= 128) layernorm_kernel<TIn, TOut, 4><<<grid, 256, 0, s>>>(p);
@@ -202,13 +309,15 @@ cudaError_t launch_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, in
                                  const ShiftmaxC &c, uint8_t *P, int64_t ldp, cudaStream_t s) {
     if (rows == 0 || len == 0) return cudaSuccess;
     dim3 grid((unsigned)((rows + 7) / 8));
+    dim3 grid2((unsigned)((rows + 15) / 16));
     bool vec = (len % 4 == 0) && (ldx % 4 == 0) && (ldp % 4 == 0) && (((uintptr_t)X & 15) == 0) &&
                (((uintptr_t)P & 3) == 0);
-    if (vec && len <= 128) shiftmax_rows_vec<1><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 512) shiftmax_rows_vec<4><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 1024) shiftmax_rows_vec<8><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 1664) shiftmax_rows_vec<13><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 2048) shiftmax_rows_vec<16><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    if (vec && len <= 64) shiftmax_rows_vec<1, 16><<<grid2, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 128) shiftmax_rows_vec<1, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 512) shiftmax_rows_vec<4, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 1024) shiftmax_rows_vec<8, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 1664) shiftmax_rows_vec<13, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    else if (vec && len <= 2048) shiftmax_rows_vec<16, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
     else shiftmax_rows_generic<<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
     return cudaGetLastError();
 }
@@ -216,9 +325,26 @@ cudaError_t launch_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, in
 cudaError_t launch_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const GeluC &c, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
     int64_t n4 = 0;
+    // the clamp threshold of both ShiftExp inputs: |x| >= ((k I0 + 1)/1.4375 + 3)/1.6875 (< T)
+    const double bound = 0.7 * ((double)c.se.kI0 + 1.0) + 8.0;
     if ((((uintptr_t)X | (uintptr_t)Y) & 15) == 0) {
         n4 = n / 4;
-        if (n4) {
+        if (n4 && bound <= 32767.0 && n4 >= (1 << 16)) {
+            const int32_t T = (int32_t)bound;
+            const int smem = 2 * T + 1;
+            static bool attr = false;
+            if (!attr) {
+                cudaError_t e = cudaFuncSetAttribute(sdshiftgelu_table, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536);
+                if (e != cudaSuccess) return e;
+                attr = true;
+            }
+            int dev = 0, sms = 148;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            int64_t blocks = (n4 + 255) / 256;
+            if (blocks > 3 * sms) blocks = 3 * sms;
+            sdshiftgelu_table<<<(unsigned)blocks, 256, smem, s>>>((const int4 *)X, (int4 *)Y, n4, c, T);
+        } else if (n4) {
             int64_t blocks = (n4 + 255) / 256;
             if (blocks > 152 * 16) blocks = 152 * 16;
             sdshiftgelu_vec<<<(unsigned)blocks, 256, 0, s>>>((const int4 *)X, (int4 *)Y, n4, c);

@@ -122,6 +122,17 @@ def test_sdshiftgelu_all_int16(ilw, orc, I0):
     assert_same(host(got), orc.sdshiftgelu(x, I0), f"gelu I0={I0}")
 
 
+@pytest.mark.parametrize("I0", [1, 300, 1 << 10, 2047, 4000])
+def test_sdshiftgelu_large_input(ilw, orc, I0):
+    """Large inputs take the tabulated path (I_div(x) in shared memory for |x| <= T, constant
+    beyond): every int16 value four times over, plus magnitudes far past the table's range."""
+    x = np.tile(np.arange(-(1 << 15), 1 << 15, dtype=np.int32), 4)
+    x = np.concatenate([x, np.array([1 << 20, -(1 << 20), (1 << 24) - 1, -(1 << 24) + 1, 40000, -40000], np.int32)])
+    x = np.concatenate([x, np.zeros((-len(x)) % 4, np.int32)])
+    got = ilw.sdshiftgelu(dev(x), {"I0": I0})
+    assert_same(host(got), orc.sdshiftgelu(x, I0), f"gelu table I0={I0}")
+
+
 def test_sdshiftgelu_unaligned_tail(ilw, orc):
     x = synth.uniform_int(6, "gt", (1003,), -4096, 4096)
     xd = dev(np.concatenate([np.zeros(1, np.int32), x]))[1:]  # 4-byte but not 16-byte aligned
