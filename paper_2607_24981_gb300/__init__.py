@@ -14,7 +14,7 @@ __all__ = [
     "lib", "IlwError", "version", "pack_weight", "gemm_requant", "gemm_gelu", "split_conv",
     "shiftmax_rows", "sdshiftgelu", "int_layernorm", "shiftmax_attn", "deform_attn",
     "BlockWeights", "block_forward", "block_workspace_bytes", "device_status",
-    "patch_embed", "patch_embed_workspace_bytes", "Backbone",
+    "patch_embed", "patch_embed_workspace_bytes", "Backbone", "Graphed",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -383,3 +383,32 @@ class Backbone:
         for i, bw in enumerate(self.blocks):
             x = block_forward(bw, x, self.B, self.T, self.ws_blk, out=self.x[(i + 1) % 2])
         return x
+
+    def capture(self, img) -> "Graphed":
+        """The forward of ``img`` recorded as one CUDA graph: ``replay()`` re-runs the patch
+        embedding and every block on the current contents of ``img`` (a fixed device buffer) and
+        returns the backbone's output buffer."""
+        return Graphed(lambda: self.forward(img))
+
+
+class Graphed:
+    """A CUDA graph of one sequence of library calls on fixed buffers.  The calls run once on a
+    side stream (so every lazily built table and tensor map exists), are then recorded, and each
+    ``replay()`` launches the recorded kernels on the current stream in one graph launch."""
+
+    def __init__(self, fn, warmup: int = 1):
+        import torch
+
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            for _ in range(warmup):
+                fn()
+        torch.cuda.current_stream().wait_stream(side)
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            self.out = fn()
+
+    def replay(self):
+        self.graph.replay()
+        return self.out

@@ -75,7 +75,7 @@ struct Group {
     }
 };
 
-template <int DH>
+template <int DH, bool FASTQ>
 __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     constexpr int LDH = DH * 2 + 16;  // padded fp16 row (bytes): conflict-free ldmatrix
     constexpr int KS = DH / 16;       // k16 steps of q k^T
@@ -221,24 +221,30 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
     mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
     mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    const int32_t imx0 = __float2int_rn(mx0), imx1 = __float2int_rn(mx1);
+    // ShiftExp(s - max) is read off the bits of (max + 2^23) - s (exact: integers below 2^23)
+    const float mb0 = mx0 + 8388608.0f, mb1 = mx1 + 8388608.0f;
+    const ShiftExpC se = p.smx.se;
+    auto sexp = [&](float mb, float sv) { return shift_exp_bits<FASTQ>(__float_as_uint(mb - sv), se); };
 
     // ---- pass 2: S_sum = sum ShiftExp(s - max)
-    const ShiftExpC se = p.smx.se;
     uint64_t sum0 = 0, sum1 = 0;
     sweep(false, [&](int kb, int buf, bool full) {
         float S[8][4];
         scores(buf, S);
+        if (full) {
 #pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            const int key = kb * KB + nt * 8 + 2 * t;
-            const bool v0 = full || key < Tg, v1 = full || key + 1 < Tg;
-            const uint32_t e0 = shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][0])), se);
-            const uint32_t e1 = shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][1])), se);
-            const uint32_t e2 = shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][2])), se);
-            const uint32_t e3 = shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][3])), se);
-            sum0 += (uint64_t)(v0 ? e0 : 0u) + (v1 ? e1 : 0u);
-            sum1 += (uint64_t)(v0 ? e2 : 0u) + (v1 ? e3 : 0u);
+            for (int nt = 0; nt < 8; ++nt) {
+                sum0 += (uint64_t)sexp(mb0, S[nt][0]) + sexp(mb0, S[nt][1]);
+                sum1 += (uint64_t)sexp(mb1, S[nt][2]) + sexp(mb1, S[nt][3]);
+            }
+        } else {
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                const int key = kb * KB + nt * 8 + 2 * t;
+                const bool v0 = key < Tg, v1 = key + 1 < Tg;
+                sum0 += (uint64_t)(v0 ? sexp(mb0, S[nt][0]) : 0u) + (v1 ? sexp(mb0, S[nt][1]) : 0u);
+                sum1 += (uint64_t)(v0 ? sexp(mb1, S[nt][2]) : 0u) + (v1 ? sexp(mb1, S[nt][3]) : 0u);
+            }
         }
     });
     sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
@@ -257,17 +263,27 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
         float S[8][4];
         scores(buf, S);
         uint32_t pa[4][4];  // A fragments of P for the 4 k16 steps (16 keys each)
+        // n-tile nt covers keys 8nt..8nt+7 = half (nt & 1) of k16 step nt >> 1
+        if (full) {
 #pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            const int key = kb * KB + nt * 8 + 2 * t;
-            const bool v0 = full || key < Tg, v1 = full || key + 1 < Tg;
-            const uint32_t p0 = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][0])), se), rn0) : 0u;
-            const uint32_t p1 = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(imx0 - __float2int_rn(S[nt][1])), se), rn0) : 0u;
-            const uint32_t p2 = v0 ? shiftmax_out(shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][2])), se), rn1) : 0u;
-            const uint32_t p3 = v1 ? shiftmax_out(shift_exp_mag((uint32_t)(imx1 - __float2int_rn(S[nt][3])), se), rn1) : 0u;
-            // n-tile nt covers keys 8nt..8nt+7 = half (nt & 1) of k16 step nt >> 1
-            pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(p0, p1);  // row g
-            pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(p2, p3);  // row g + 8
+            for (int nt = 0; nt < 8; ++nt) {
+                pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(shiftmax_out(sexp(mb0, S[nt][0]), rn0),
+                                                            shiftmax_out(sexp(mb0, S[nt][1]), rn0));  // row g
+                pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(shiftmax_out(sexp(mb1, S[nt][2]), rn1),
+                                                            shiftmax_out(sexp(mb1, S[nt][3]), rn1));  // row g + 8
+            }
+        } else {
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                const int key = kb * KB + nt * 8 + 2 * t;
+                const bool v0 = key < Tg, v1 = key + 1 < Tg;
+                const uint32_t p0 = v0 ? shiftmax_out(sexp(mb0, S[nt][0]), rn0) : 0u;
+                const uint32_t p1 = v1 ? shiftmax_out(sexp(mb0, S[nt][1]), rn0) : 0u;
+                const uint32_t p2 = v0 ? shiftmax_out(sexp(mb1, S[nt][2]), rn1) : 0u;
+                const uint32_t p3 = v1 ? shiftmax_out(sexp(mb1, S[nt][3]), rn1) : 0u;
+                pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(p0, p1);
+                pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(p2, p3);
+            }
         }
         const uint32_t vs_base = (uint32_t)__cvta_generic_to_shared(Vs[buf]);
 #pragma unroll
@@ -316,8 +332,14 @@ cudaError_t launch_attention(const AttnParams &p, cudaStream_t s) {
     const int Tg = p.nw > 1 ? (p.grid_side / p.nw) * (p.grid_side / p.nw) : p.T;
     if (p.B == 0 || Tg == 0) return cudaSuccess;
     dim3 grid((Tg + QT - 1) / QT, p.H, p.B * G2);
-    if (p.dh == 64) attn_kernel<64><<<grid, THREADS, 0, s>>>(p);
-    else attn_kernel<32><<<grid, THREADS, 0, s>>>(p);
+    const bool fastq = p.smx.se.m32 != 0;
+    if (p.dh == 64) {
+        if (fastq) attn_kernel<64, true><<<grid, THREADS, 0, s>>>(p);
+        else attn_kernel<64, false><<<grid, THREADS, 0, s>>>(p);
+    } else {
+        if (fastq) attn_kernel<32, true><<<grid, THREADS, 0, s>>>(p);
+        else attn_kernel<32, false><<<grid, THREADS, 0, s>>>(p);
+    }
     return cudaGetLastError();
 }
 

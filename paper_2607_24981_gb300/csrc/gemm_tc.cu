@@ -47,9 +47,10 @@ struct Seg {
     int32_t m_b, s_b;   // split-conv rescale of the branch partial
 };
 
+template <int NB>  // NB: tensor-map slots (1 for a plain GEMM, kMaxBranches for split convolution)
 struct TcParams {  // CUtensorMap members keep the 64-byte alignment TMA needs
-    CUtensorMap amap[kMaxBranches];
-    CUtensorMap wmap[kMaxBranches];
+    CUtensorMap amap[NB];
+    CUtensorMap wmap[NB];
     Seg seg[kMaxSeg];
     int32_t nseg;
     int32_t branch_rq;
@@ -150,6 +151,15 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
         : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// Waits for this thread's TMEM loads and marks the 16 destination registers as written by the
+// wait, so that no use of them can be scheduled before the data has arrived.
+__device__ __forceinline__ void tmem_wait_ld16(uint32_t (&v)[16]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
+                   "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]), "+r"(v[12]), "+r"(v[13]), "+r"(v[14]), "+r"(v[15])
+                 :
+                 : "memory");
+}
 
 // 4 int8 (one word) -> 2 words of fp16x2, exact: fp16 bits 0x6400 | (b ^ 0x80) encode 1152 + b.
 __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
@@ -176,23 +186,75 @@ struct Smem {
 // Output kinds: one compact epilogue per kernel instantiation.
 enum { KIND_RQ8 = 0, KIND_RQ16 = 1, KIND_RAW32 = 2, KIND_GELU8 = 3 };
 
-template <int KIND>
-__device__ __forceinline__ int32_t epi_one(const EpiParams &ep, int64_t row, int32_t acc, int32_t bias, int32_t mult,
-                                           int32_t shift, int32_t col, const uint8_t *gtab, int32_t gT) {
-    const int64_t v = (int64_t)acc + bias;
-    if (KIND == KIND_RAW32) return (int32_t)v;
-    if (KIND == KIND_GELU8) {
-        const int32_t g = sat16(rq(v, mult, shift));
-        const int32_t idiv = gtab[min(max(g, -gT), gT) + gT];  // = gelu_idiv(g) (tabulated below)
-        return sat8(rq((int64_t)g * idiv, ep.m_g, ep.s_g));
-    }
-    int64_t o = rq(v, mult, shift);
-    if (ep.res) o += rq((int64_t)ep.res[(row % ep.res_rows) * ep.ldr + col], ep.m_r, ep.s_r);
-    return KIND == KIND_RQ8 ? sat8(o) : sat16(o);
+// 16 consecutive int32 of shared memory (16-byte aligned) into registers: four 128-bit loads
+__device__ __forceinline__ void lds16(const int32_t *p, int32_t (&o)[16]) {
+    const uint32_t a = (uint32_t)__cvta_generic_to_shared(p);
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(o[4 * j]), "=r"(o[4 * j + 1]), "=r"(o[4 * j + 2]), "=r"(o[4 * j + 3])
+                     : "r"(a + 16 * j));
 }
 
-template <int BN, int STAGES, int KIND>
-__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
+// rq(v; m, s) for int32 v and s >= 33: with v*m = hi 2^32 + lo, lo / 2^32 < 1 added to an integer
+// numerator never changes floor(. / 2^(s-32)), so rq = (hi + 2^(s-33)) >> (s-32) exactly.
+__device__ __forceinline__ int32_t rq_hi(int32_t v, int32_t m, int32_t s) {
+    return (__mulhi(v, m) + (1 << (s - 33))) >> (s - 32);
+}
+
+// The fused epilogue of 16 consecutive columns of one row, computed stage by stage so that the
+// 16 independent elements overlap.  The fast path (every shift >= 33, the usual case) is decided
+// per chunk, which is uniform across the warp.
+template <int KIND>
+__device__ __forceinline__ void epi_chunk(const EpiParams &ep, int64_t row, const int32_t (&acc)[16],
+                                          const int32_t (&sb)[16], const int32_t (&sm)[16], const int32_t (&ss)[16],
+                                          int32_t col0,
+                                          int32_t N, const uint8_t *gtab, int32_t gT, int32_t (&out)[16]) {
+    if (KIND == KIND_RAW32) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) out[i] = acc[i] + sb[i];
+        return;
+    }
+    bool fast = true;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) fast &= ss[i] >= 33;
+    int32_t r[16];
+    if (fast) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) r[i] = rq_hi(acc[i] + sb[i], sm[i], ss[i]);  // |r| < 2^29
+    } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int64_t t = rq((int64_t)acc[i] + sb[i], sm[i], ss[i]);
+            r[i] = (int32_t)(t < -(1 << 30) ? -(1 << 30) : (t > (1 << 30) ? (1 << 30) : t));  // saturates the same
+        }
+    }
+    if (KIND == KIND_GELU8) {
+        const bool gfast = ep.s_g >= 33;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int32_t g = sat16(r[i]);
+            const int32_t gi = g * (int32_t)gtab[min(max(g, -gT), gT) + gT];  // g * I_div(g), |.| < 2^22
+            out[i] = sat8(gfast ? rq_hi(gi, ep.m_g, ep.s_g) : rq((int64_t)gi, ep.m_g, ep.s_g));
+        }
+        return;
+    }
+    if (ep.res) {
+        const int16_t *res = ep.res + (row % ep.res_rows) * ep.ldr;
+        const bool rfast = ep.s_r >= 17;  // int16 residual: res * 2^16 fits int32
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int32_t x = res[min(col0 + i, N - 1)];
+            const int32_t rr = rfast ? rq_hi(x * 65536, ep.m_r, ep.s_r + 16) : (int32_t)rq((int64_t)x, ep.m_r, ep.s_r);
+            r[i] += rr;
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i) out[i] = KIND == KIND_RQ8 ? sat8(r[i]) : sat16(r[i]);
+}
+
+template <int BN, int STAGES, int KIND, int NB>
+__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcParams<NB> p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     constexpr int kStage = Smem<BN>::kStage;
@@ -235,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     // SD-ShiftGELU: I_div depends on the int16 value g alone and is constant once both ShiftExp
     // inputs are clamped (|g| > gelu_T), so the epilogue warps tabulate it once per CTA with the
     // same device function (exact by construction) and then look it up.
-    uint8_t *gtab = (uint8_t *)((int32_t *)(tmem_slot + 4) + 12 * BN);
+    uint8_t *gtab = (uint8_t *)((int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + 12 * BN);
     if (KIND == KIND_GELU8 && warp >= 6) {
         for (int i = threadIdx.x - 192; i <= 2 * p.gelu_T; i += 256) gtab[i] = (uint8_t)gelu_idiv(i - p.gelu_T, p.ep.gelu);
         asm volatile("bar.sync 1, 256;" ::: "memory");  // the 8 epilogue warps only
@@ -347,54 +409,80 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         constexpr int HALF = BN / 2;
         const int q = warp & 3, h = (warp - 6) >> 2;
         const EpiParams &ep = p.ep;
-        int32_t *s_bias = (int32_t *)(tmem_slot + 4) + (warp - 6) * 3 * HALF;  // this warp's copy of
+        int32_t *s_bias = (int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + (warp - 6) * 3 * HALF;  // this warp's copy of
         int32_t *s_mult = s_bias + HALF;                                       // the tile's per-column
         int32_t *s_shift = s_mult + HALF;                                      // epilogue parameters
         constexpr int bits = KIND == KIND_RQ16 ? 16 : (KIND == KIND_RAW32 ? 32 : 8);
+        constexpr int PPL = HALF / 32;  // parameters per lane and per array
+        // The next tile's parameters are fetched into registers while the current tile is processed.
+        int32_t pb[PPL], pm[PPL], ps[PPL];
+        auto fetch = [&](int t) {
+            const int nn = (t % p.tiles_n) * BN + h * HALF;
+#pragma unroll
+            for (int k = 0; k < PPL; ++k) {
+                const int col = nn + lane + 32 * k;
+                const bool ok = col < p.N;
+                pb[k] = (ok && ep.bias) ? __ldg(ep.bias + col) : 0;
+                pm[k] = (ok && ep.mult) ? __ldg(ep.mult + col) : 0;
+                ps[k] = (ok && ep.shift) ? __ldg(ep.shift + col) : 1;
+            }
+        };
+        if (blockIdx.x < p.tiles) fetch(blockIdx.x);
+        const int nseg = p.nseg, nld = (HALF / 16) * nseg;  // TMEM loads per tile
         int tl = 0;
         for (int t = blockIdx.x; t < p.tiles; t += gridDim.x, ++tl) {
             const int b = tl % p.nbuf;
             const uint32_t use = (uint32_t)(tl / p.nbuf);
             const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN + h * HALF;
             __syncwarp();  // this warp is done with the previous tile's parameters
-            for (int c = lane; c < HALF; c += 32) {
-                const int col = n0 + c;
-                const bool ok = col < p.N;
-                s_bias[c] = (ok && ep.bias) ? ep.bias[col] : 0;
-                s_mult[c] = (ok && ep.mult) ? ep.mult[col] : 0;
-                s_shift[c] = (ok && ep.shift) ? ep.shift[col] : 1;
+#pragma unroll
+            for (int k = 0; k < PPL; ++k) {
+                s_bias[lane + 32 * k] = pb[k];
+                s_mult[lane + 32 * k] = pm[k];
+                s_shift[lane + 32 * k] = ps[k];
             }
             __syncwarp();
+            if (t + (int)gridDim.x < p.tiles) fetch(t + gridDim.x);
             if (!mbar_wait(acc_full(b), use & 1, abort, p.status, kStatusTimeoutMma)) break;
             tc_fence_after();
             const int64_t row = (int64_t)m0 + 32 * q + lane;
             const bool row_ok = row < p.M;
-            for (int c0 = 0; c0 < HALF; c0 += 16) {
-                int32_t acc[16];
+            const uint32_t tbase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * acc_cols + h * HALF);
+            // TMEM load i reads segment i % nseg of chunk i / nseg; load i+1 is in flight while the
+            // epilogue of load i's chunk runs.
+            uint32_t v[16];
+            tmem_ld16(tbase, v);
+            int32_t acc[16];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) acc[i] = 0;
-                for (int sg = 0; sg < p.nseg; ++sg) {
-                    uint32_t v[16];
-                    tmem_ld16(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * acc_cols + sg * BN + h * HALF + c0), v);
-                    tmem_wait_ld();
+            for (int i = 0; i < 16; ++i) acc[i] = 0;
+            for (int li = 0; li < nld; ++li) {
+                const int c0 = (li / nseg) * 16, sg = li - (li / nseg) * nseg;
+                tmem_wait_ld16(v);
+                if (p.branch_rq) {
+                    const int32_t mb = p.seg[sg].m_b, sbb = p.seg[sg].s_b;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        int32_t a = __float2int_rn(__uint_as_float(v[i]));  // exact: integer < 2^24
-                        acc[i] += p.branch_rq ? (int32_t)rq(a, p.seg[sg].m_b, p.seg[sg].s_b) : a;
-                    }
+                    for (int i = 0; i < 16; ++i) acc[i] += (int32_t)rq(__float2int_rn(__uint_as_float(v[i])), mb, sbb);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) acc[i] += __float2int_rn(__uint_as_float(v[i]));  // exact: < 2^24
                 }
-                if (c0 + 16 >= HALF) {  // every TMEM read of this warp in this accumulator set is done
+                if (li + 1 < nld) {
+                    const int c1 = ((li + 1) / nseg) * 16, sg1 = (li + 1) - ((li + 1) / nseg) * nseg;
+                    tmem_ld16(tbase + (uint32_t)(sg1 * BN + c1), v);
+                } else {  // every TMEM read of this warp in this accumulator set is done
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(acc_empty(b));
                 }
+                if (sg != nseg - 1) continue;
+                int32_t cb[16], cm[16], cs[16];  // this chunk's per-column parameters
+                lds16(s_bias + c0, cb);
+                lds16(s_mult + c0, cm);
+                lds16(s_shift + c0, cs);
                 const int ncol = min(16, p.N - (n0 + c0));
                 if (row_ok && ncol > 0) {
                     int32_t out[16];
-#pragma unroll
-                    for (int i = 0; i < 16; ++i)
-                        out[i] = epi_one<KIND>(ep, row, acc[i], s_bias[c0 + i], s_mult[c0 + i], s_shift[c0 + i],
-                                               min(n0 + c0 + i, p.N - 1), gtab, p.gelu_T);
+                    epi_chunk<KIND>(ep, row, acc, cb, cm, cs, n0 + c0, p.N, gtab, p.gelu_T, out);
                     char *dst = (char *)ep.C + (row * ep.ldc + n0 + c0) * (bits / 8);
                     const bool vec = ncol == 16 && (((uintptr_t)dst & 15) == 0);
                     if constexpr (bits == 8) {
@@ -437,7 +525,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                         }
                     }
                 }
-                __syncwarp();  // reconverge before the next warp-synchronous tcgen05.ld
+#pragma unroll
+                for (int i = 0; i < 16; ++i) acc[i] = 0;
+                __syncwarp();  // reconverge before the next warp-synchronous tcgen05 instruction
             }
         }
     }
@@ -475,17 +565,50 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
+// Recently encoded tensor maps of this host thread.  A map is a pure function of its key, so a hit
+// is the same 128 bytes cuTensorMapEncodeTiled would write; the cache only saves the encoding.
+struct MapKey {
+    const void *base;
+    int64_t rows, cols, ld;
+    int32_t dt, box_cols, box_rows, sw;
+    bool operator==(const MapKey &o) const {
+        return base == o.base && rows == o.rows && cols == o.cols && ld == o.ld && dt == o.dt &&
+               box_cols == o.box_cols && box_rows == o.box_rows && sw == o.sw;
+    }
+};
+struct MapCache {
+    static constexpr int kSlots = 64;
+    MapKey key[kSlots];
+    CUtensorMap map[kSlots];
+    bool used[kSlots] = {};
+    int next = 0;
+};
+
 // 2-D tensor map over a row-major [rows, cols] matrix (cols contiguous), boxes of box_cols x box_rows
 bool make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int esize, int64_t rows, int64_t cols,
               int64_t ld, int box_cols, int box_rows, CUtensorMapSwizzle sw) {
+    thread_local MapCache cache;
+    const MapKey k{base, rows, cols, ld, (int32_t)dt, box_cols, box_rows, (int32_t)sw};
+    for (int i = 0; i < MapCache::kSlots; ++i)
+        if (cache.used[i] && cache.key[i] == k) {
+            *m = cache.map[i];
+            return true;
+        }
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)(ld * esize)};
     cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
-    return fn(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    if (fn(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return false;
+    const int slot = cache.next;
+    cache.next = (cache.next + 1) % MapCache::kSlots;
+    cache.key[slot] = k;
+    cache.map[slot] = *m;
+    cache.used[slot] = true;
+    return true;
 }
 
 int num_sms() {
@@ -499,25 +622,26 @@ int num_sms() {
     return n;
 }
 
-template <int BN, int STAGES, int KIND>
-cudaError_t launch_tc(TcParams &tp, cudaStream_t s) {
-    const size_t smem = 1024 + (size_t)STAGES * Smem<BN>::kStage + 8 * (3 * STAGES + 4) + 16 + 4 * 3 * BN * 4 +
+template <int BN, int STAGES, int KIND, int NB>
+cudaError_t launch_tc(TcParams<NB> &tp, cudaStream_t s) {
+    const size_t smem = 1024 + (size_t)STAGES * Smem<BN>::kStage + 8 * (3 * STAGES + 4) + 32 + 4 * 3 * BN * 4 +
                         (KIND == KIND_GELU8 ? 65536 : 0);
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        attr_err = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, KIND, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)smem);
     });
     if (attr_err != cudaSuccess) return attr_err;
     const int grid = tp.tiles < num_sms() ? tp.tiles : num_sms();
-    gemm_tc_kernel<BN, STAGES, KIND><<<grid, kThreads, smem, s>>>(tp);
+    gemm_tc_kernel<BN, STAGES, KIND, NB><<<grid, kThreads, smem, s>>>(tp);
     return cudaGetLastError();
 }
 
-template <int BN, int STAGES>
+template <int BN, int STAGES, int NB>
 cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
-    TcParams tp;
+    if (gp.nb > NB) return cudaErrorInvalidValue;
+    TcParams<NB> tp;
     memset(&tp, 0, sizeof(tp));
     tp.M = gp.M;
     tp.N = gp.N;
@@ -562,10 +686,14 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
         const double bound = 0.7 * ((double)ep.gelu.se.kI0 + 1.0) + 8.0;
         tp.gelu_T = bound > 32767.0 ? 32767 : (int32_t)bound;
     }
-    if (ep.kind == EPI_GELU) return launch_tc<BN, STAGES, KIND_GELU8>(tp, s);
-    if (ep.out_bits == 8) return launch_tc<BN, STAGES, KIND_RQ8>(tp, s);
-    if (ep.out_bits == 16) return launch_tc<BN, STAGES, KIND_RQ16>(tp, s);
-    return launch_tc<BN, STAGES, KIND_RAW32>(tp, s);
+    if constexpr (NB == 1) {
+        if (ep.kind == EPI_GELU) return launch_tc<BN, STAGES, KIND_GELU8, NB>(tp, s);
+    } else {
+        if (ep.kind == EPI_GELU) return cudaErrorInvalidValue;  // split convolutions requantise only
+    }
+    if (ep.out_bits == 8) return launch_tc<BN, STAGES, KIND_RQ8, NB>(tp, s);
+    if (ep.out_bits == 16) return launch_tc<BN, STAGES, KIND_RQ16, NB>(tp, s);
+    return launch_tc<BN, STAGES, KIND_RAW32, NB>(tp, s);
 }
 
 }  // namespace
@@ -579,9 +707,10 @@ cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *pack
 cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     if (gp.M == 0 || gp.N == 0) return cudaSuccess;
     // 192-wide tiles when N splits evenly into them (fewer re-reads of A per flop), else 128
-    if (gp.N % 192 == 0 && gp.N >= 768 && gp.nb == 1)
-        return ep.kind == EPI_GELU ? run<192, 3>(gp, ep, s) : run<192, 4>(gp, ep, s);
-    return ep.kind == EPI_GELU ? run<128, 3>(gp, ep, s) : run<128, 5>(gp, ep, s);
+    if (gp.nb > 1) return run<128, 5, kMaxBranches>(gp, ep, s);
+    if (gp.N % 192 == 0 && gp.N >= 768)
+        return ep.kind == EPI_GELU ? run<192, 3, 1>(gp, ep, s) : run<192, 4, 1>(gp, ep, s);
+    return ep.kind == EPI_GELU ? run<128, 3, 1>(gp, ep, s) : run<128, 5, 1>(gp, ep, s);
 }
 
 }  // namespace ilw

@@ -33,6 +33,8 @@ struct ShiftExpC {
     uint32_t m_lo;  // low 32 bits of M
     uint32_t m_hi;  // high bits of M (M <= 2^40)
     int32_t k;      // k_inter
+    uint32_t m32;   // ceil(2^32 / I0) when k I0^2 < 2^32 (then floor(n / I0) = umulhi(n, m32) for
+                    // every n <= k I0), else 0
 };
 
 // Arithmetic (flooring) right shift of a signed value.
@@ -56,6 +58,21 @@ __device__ __forceinline__ uint32_t shift_exp_mag(uint32_t a, const ShiftExpC &c
     uint32_t q = (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
     uint32_t r = n - q * (uint32_t)c.I0;               // decimal part, in [0, I0)
     uint32_t Ib = (uint32_t)c.I0 - ((r + 1u) >> 1);    // ((-r) >> 1) + I0
+    return Ib << (c.k - (int32_t)q);
+}
+
+// The same ShiftExp of the magnitude a = max - s, taken from b = bits of the fp32 value
+// (max + 2^23) - s.  For integer scores with 0 <= a < 2^23 that value is exact and b = 0x4B000000 + a.
+// Because 0x4B000000 is a multiple of 16, ceil(b/2) and ceil(b/16) are ceil(a/2) and ceil(a/16) plus
+// fixed constants, so n = a + ceil(a/2) - ceil(a/16) is read off b with the constants folded into one
+// (1.4375 * 0x4B000000 = 1808793600).  The quotient uses the single-multiply reciprocal when c.m32 is
+// set (FASTQ), and I0 - ceil(r/2) is written as ((q + 2) I0 - n) / 2 (r = n - q I0, floored).
+template <bool FASTQ>
+__device__ __forceinline__ uint32_t shift_exp_bits(uint32_t b, const ShiftExpC &c) {
+    uint32_t n = b + ((b + 1u) >> 1) - ((b + 15u) >> 4) - 1808793600u;
+    n = min(n, (uint32_t)c.kI0);
+    const uint32_t q = FASTQ ? __umulhi(n, c.m32) : (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
+    const uint32_t Ib = ((q + 2u) * (uint32_t)c.I0 - n) >> 1;
     return Ib << (c.k - (int32_t)q);
 }
 

@@ -28,6 +28,10 @@ inline ShiftExpC make_shiftexp(int32_t I0, int32_t k) {
     c.m_lo = (uint32_t)(M & 0xffffffffull);
     c.m_hi = (uint32_t)(M >> 32);
     c.k = k;
+    const uint64_t kI0sq = (uint64_t)(k > 0 ? k : 0) * (uint64_t)I0 * (uint64_t)I0;
+    c.m32 = (I0 >= 2 && kI0sq < ((uint64_t)1 << 32))
+                ? (uint32_t)((((uint64_t)1 << 32) + (uint64_t)I0 - 1) / (uint64_t)I0)
+                : 0u;
     return c;
 }
 inline GeluC make_gelu(const ilw_gelu_t &g) {
@@ -68,23 +72,6 @@ struct EpiParams {
     GeluC gelu;
     int32_t m_g, s_g;
 };
-
-// The fused epilogue value of output (row, col) from the exact integer accumulator (bias not
-// yet added), given the column's bias/mult/shift: Sec. 3.2.1 (bias, per-channel dyadic
-// requantisation), the two-term residual form, and SD-ShiftGELU (Algorithm 1) for EPI_GELU.
-__device__ __forceinline__ int32_t epi_value(const EpiParams &ep, int64_t row, int32_t acc, int32_t bias,
-                                             int32_t mult, int32_t shift, int32_t col) {
-    int64_t v = (int64_t)acc + bias;
-    if (ep.kind == EPI_GELU) {
-        int32_t g = sat16(rq(v, mult, shift));
-        int32_t idiv = gelu_idiv(g, ep.gelu);
-        return sat8(rq((int64_t)g * idiv, ep.m_g, ep.s_g));
-    }
-    if (ep.out_bits == 32) return (int32_t)v;
-    int64_t o = rq(v, mult, shift);
-    if (ep.res) o += rq((int64_t)ep.res[(row % ep.res_rows) * ep.ldr + col], ep.m_r, ep.s_r);
-    return ep.out_bits == 8 ? sat8(o) : sat16(o);
-}
 
 // Packed weight layout: the same integers as fp16 [N, K] (row-major), the tensor-core operand.
 inline size_t packed_weight_bytes(int32_t N, int32_t K) { return (size_t)N * K * 2; }

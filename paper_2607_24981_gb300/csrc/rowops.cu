@@ -177,29 +177,65 @@ __device__ __forceinline__ uint64_t newton_isqrt(uint64_t V, int iters) {
     return r < 1 ? 1 : r;
 }
 
-// ROWS rows per warp, held in registers: lanes share the loads and the two integer row sums,
-// then lane j runs Newton's iteration (the sequential part) for row j, so a warp pays for one
-// Newton sequence per ROWS rows.  V = sum (x - mu)^2 = sum x^2 - 2 mu sum x + C mu^2, exactly.
-template <typename TIn, typename TOut, int EPL, int ROWS>
+// 4 consecutive elements of one row as int32 (vector load: int4 for int32 input, 8 bytes for int16)
+template <typename TIn>
+__device__ __forceinline__ void load4(const TIn *x, int32_t (&o)[4]);
+template <>
+__device__ __forceinline__ void load4<int32_t>(const int32_t *x, int32_t (&o)[4]) {
+    const int4 v = __ldcs((const int4 *)x);
+    o[0] = v.x; o[1] = v.y; o[2] = v.z; o[3] = v.w;
+}
+template <>
+__device__ __forceinline__ void load4<int16_t>(const int16_t *x, int32_t (&o)[4]) {
+    const uint2 v = __ldcs((const uint2 *)x);
+    o[0] = (int16_t)(v.x & 0xffff); o[1] = (int16_t)(v.x >> 16); o[2] = (int16_t)(v.y & 0xffff); o[3] = (int16_t)(v.y >> 16);
+}
+template <typename TOut>
+__device__ __forceinline__ void store4(TOut *y, const int32_t (&o)[4]);
+template <>
+__device__ __forceinline__ void store4<int8_t>(int8_t *y, const int32_t (&o)[4]) {
+    *(uint32_t *)y = (uint32_t)(uint8_t)o[0] | ((uint32_t)(uint8_t)o[1] << 8) | ((uint32_t)(uint8_t)o[2] << 16) |
+                     ((uint32_t)(uint8_t)o[3] << 24);
+}
+template <>
+__device__ __forceinline__ void store4<int16_t>(int16_t *y, const int32_t (&o)[4]) {
+    *(uint2 *)y = make_uint2((uint32_t)(uint16_t)o[0] | ((uint32_t)(uint16_t)o[1] << 16),
+                             (uint32_t)(uint16_t)o[2] | ((uint32_t)(uint16_t)o[3] << 16));
+}
+
+// ROWS rows per warp, held in registers.  Each lane owns 4-element chunks (lane + 32 j) of every
+// row; all loads of the warp's rows are issued before any reduction.  Lanes share the two integer
+// row sums, then lane r runs Newton's iteration (the sequential part) for row r, so a warp pays for
+// one Newton sequence per ROWS rows.  V = sum (x - mu)^2 = sum x^2 - 2 mu sum x + C mu^2, exactly.
+template <typename TIn, typename TOut, int NCH, int ROWS>
 __global__ void __launch_bounds__(256) layernorm_multi(const LnParams p) {
     const int lane = threadIdx.x & 31;
     const int64_t row0 = ((int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * ROWS;
     if (row0 >= p.rows) return;
-    const int C = p.C;
-    int32_t v[ROWS][EPL];
-    int64_t my_s = 0, my_q = 0;
+    const int C = p.C, nchunk = C >> 2;
+    int32_t v[ROWS][NCH][4];
 #pragma unroll
     for (int r = 0; r < ROWS; ++r) {
         const bool ok = row0 + r < p.rows;
         const TIn *x = (const TIn *)p.X + (ok ? row0 + r : row0) * p.ldx;
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) {
+            const int ch = lane + 32 * j;
+            if (ok && ch < nchunk) load4<TIn>(x + 4 * ch, v[r][j]);
+            else v[r][j][0] = v[r][j][1] = v[r][j][2] = v[r][j][3] = 0;
+        }
+    }
+    int64_t my_s = 0, my_q = 0;
+#pragma unroll
+    for (int r = 0; r < ROWS; ++r) {
         int64_t s = 0, q = 0;
 #pragma unroll
-        for (int j = 0; j < EPL; ++j) {
-            const int c = lane + 32 * j;
-            v[r][j] = (ok && c < C) ? (int32_t)x[c] : 0;
-            s += v[r][j];
-            q += (int64_t)v[r][j] * v[r][j];
-        }
+        for (int j = 0; j < NCH; ++j)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                s += v[r][j][u];
+                q += (int64_t)v[r][j][u] * v[r][j][u];
+            }
         s = warp_sum_i64(s);
         q = warp_sum_i64(q);
         if (lane == r) { my_s = s; my_q = q; }
@@ -218,12 +254,22 @@ __global__ void __launch_bounds__(256) layernorm_multi(const LnParams p) {
         const int64_t Fr = __shfl_sync(0xffffffffu, F, r);
         TOut *yo = (TOut *)p.Y + (row0 + r) * p.ldy;
 #pragma unroll
-        for (int j = 0; j < EPL; ++j) {
-            const int c = lane + 32 * j;
-            if (c < C) {
-                const int64_t n = (((int64_t)v[r][j] - mur) * Fr) >> 1;
-                const int64_t o = rq(n + p.beta[c], p.mult[c], p.shift[c]);
-                yo[c] = (TOut)(sizeof(TOut) == 1 ? sat8(o) : sat16(o));
+        for (int j = 0; j < NCH; ++j) {
+            const int ch = lane + 32 * j;
+            if (ch < nchunk) {
+                const int4 be = __ldg((const int4 *)(p.beta + 4 * ch));
+                const int4 mu4 = __ldg((const int4 *)(p.mult + 4 * ch));
+                const int4 sh4 = __ldg((const int4 *)(p.shift + 4 * ch));
+                const int32_t bb[4] = {be.x, be.y, be.z, be.w}, mm[4] = {mu4.x, mu4.y, mu4.z, mu4.w},
+                              ss[4] = {sh4.x, sh4.y, sh4.z, sh4.w};
+                int32_t o[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int64_t n = (((int64_t)v[r][j][u] - mur) * Fr) >> 1;
+                    const int64_t t = rq(n + bb[u], mm[u], ss[u]);
+                    o[u] = sizeof(TOut) == 1 ? sat8(t) : sat16(t);
+                }
+                store4<TOut>(yo + 4 * ch, o);
             }
         }
     }
@@ -282,13 +328,16 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const LnParams p) {
 
 template <typename TIn, typename TOut>
 cudaError_t ln_dispatch(const LnParams &p, cudaStream_t s) {
-    if (p.C <= 512) {  // 4 rows per warp in registers, lane-parallel Newton
+    const int eb = sizeof(TIn), ob = sizeof(TOut);
+    const bool vec = p.C % 4 == 0 && p.ldx % 4 == 0 && p.ldy % 4 == 0 && ((uintptr_t)p.X % (4 * eb)) == 0 &&
+                     ((uintptr_t)p.Y % (4 * ob)) == 0 && (((uintptr_t)p.beta | (uintptr_t)p.mult | (uintptr_t)p.shift) % 16) == 0;
+    if (vec && p.C <= 512) {  // 4 rows per warp in registers, vector loads, lane-parallel Newton
         constexpr int ROWS = 4;
         dim3 g4((unsigned)((p.rows + 8 * ROWS - 1) / (8 * ROWS)));
-        if (p.C <= 128) layernorm_multi<TIn, TOut, 4, ROWS><<<g4, 256, 0, s>>>(p);
-        else if (p.C <= 256) layernorm_multi<TIn, TOut, 8, ROWS><<<g4, 256, 0, s>>>(p);
-        else if (p.C <= 384) layernorm_multi<TIn, TOut, 12, ROWS><<<g4, 256, 0, s>>>(p);
-        else layernorm_multi<TIn, TOut, 16, ROWS><<<g4, 256, 0, s>>>(p);
+        if (p.C <= 128) layernorm_multi<TIn, TOut, 1, ROWS><<<g4, 256, 0, s>>>(p);
+        else if (p.C <= 256) layernorm_multi<TIn, TOut, 2, ROWS><<<g4, 256, 0, s>>>(p);
+        else if (p.C <= 384) layernorm_multi<TIn, TOut, 3, ROWS><<<g4, 256, 0, s>>>(p);
+        else layernorm_multi<TIn, TOut, 4, ROWS><<<g4, 256, 0, s>>>(p);
         return cudaGetLastError();
     }
     const int rows_per_block = 8;

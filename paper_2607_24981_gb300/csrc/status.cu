@@ -19,12 +19,17 @@ int *g_addr[kMaxDev] = {};
 int *status_word_ptr() {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return nullptr;
+    thread_local int last_dev = -1;
+    thread_local int *last_ptr = nullptr;
+    if (dev == last_dev) return last_ptr;
     std::lock_guard<std::mutex> lock(g_mu);
     if (!g_addr[dev]) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
         g_addr[dev] = (int *)p;
     }
+    last_dev = dev;
+    last_ptr = g_addr[dev];
     return g_addr[dev];
 }
 

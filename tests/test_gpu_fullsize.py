@@ -44,10 +44,21 @@ def test_backbone_full_batch_sampled_images(ilw, orc, workload):
     pe = synth.patch_embed_params(0, d, mode=cfg["mode"])
     img = synth.image_input(0, B)
     bb = ilw.Backbone(pe, blocks, B)
-    y = bb.forward(dev(img))
+    dimg = dev(img)
+    y = bb.forward(dimg)
     torch.cuda.synchronize()
     ilw.device_status()
     yh = y.cpu().numpy().reshape(B, T, d)
+    # the same forward recorded as a CUDA graph (Backbone.capture, the step bench.py replays):
+    # identical bytes, on a fresh input too
+    g = bb.capture(dimg)
+    same(g.replay().cpu().numpy().reshape(B, T, d), yh, f"{workload} graph replay")
+    img2 = synth.image_input(1, B)
+    dimg.copy_(dev(img2))
+    y2g = g.replay().cpu().numpy()
+    y2 = bb.forward(dimg).cpu().numpy()
+    same(y2g, y2, f"{workload} graph replay, second input")
+    assert not np.array_equal(y2, yh.reshape(y2.shape))
     pick = 5 if workload == "medium_c2" else 2
     x = orc.patch_embed(img[pick:pick + 1], pe["p"], pe["w"], pe["b"], pe["m"], pe["s"], pe["pos"],
                         pe["m_pos"], pe["s_pos"])

@@ -37,3 +37,47 @@ def test_sigmoid_uses_one_shiftexp():
     Id = Ip - Ish
     pair = np.sort(np.stack([Id, -Ish]), axis=0)
     assert np.array_equal(pair[0], -np.abs(Ip)) and np.all(pair[1] == 0)
+
+
+def test_shiftexp_exponent_from_biased_float_bits():
+    """Attention reads a = max - s off the bits of the fp32 value (max + 2^23) - s: for integer
+    scores |s|, |max| < 2^20 that value is exact, so its bits are 0x4B000000 + a; and since
+    0x4B000000 is a multiple of 16, -I_e = a + ceil(a/2) - ceil(a/16) equals
+    b + ((b+1) >> 1) - ((b+15) >> 4) - 1808793600 in wrapping 32-bit arithmetic."""
+    rng = np.random.default_rng(11)
+    s = rng.integers(-(1 << 20) + 1, 1 << 20, size=1 << 20)
+    mx = np.maximum(s, rng.integers(-(1 << 20) + 1, 1 << 20, size=s.size))
+    mb = mx.astype(np.float32) + np.float32(8388608.0)
+    bits = (mb - s.astype(np.float32)).view(np.uint32).astype(np.int64)
+    assert np.array_equal(bits, 0x4B000000 + (mx - s))
+    a = np.arange(0, 1 << 22, dtype=np.int64)
+    b = (0x4B000000 + a).astype(np.uint32)
+    n_bits = b + ((b + np.uint32(1)) >> np.uint32(1)) - ((b + np.uint32(15)) >> np.uint32(4)) - np.uint32(1808793600)
+    assert np.array_equal(n_bits.astype(np.int64), a + ((a + 1) >> 1) - ((a + 15) >> 4))
+    assert 0x4B000000 % 16 == 0 and 0x4B000000 + 0x4B000000 // 2 - 0x4B000000 // 16 == 1808793600
+
+
+@pytest.mark.parametrize("I0", [2, 3, 7, 255, 1000, 4096, 6151, 9999, 12289, 16383])
+def test_single_multiply_quotient_and_half_remainder(I0):
+    """With m32 = ceil(2^32 / I0) and k I0^2 < 2^32, umulhi(n, m32) = floor(n / I0) for every
+    n <= k I0 (the error n (m32 I0 - 2^32) / 2^32 stays below 1/I0); and I0 - ceil(r/2) for
+    r = n - q I0 equals ((q + 2) I0 - n) >> 1."""
+    k = 16
+    assert k * I0 * I0 < (1 << 32)
+    n = np.arange(0, k * I0 + 1, dtype=np.uint64)
+    m32 = np.uint64(((1 << 32) + I0 - 1) // I0)
+    q = (n * m32) >> np.uint64(32)
+    assert np.array_equal(q, n // np.uint64(I0))
+    r = n - q * np.uint64(I0)
+    assert np.array_equal(np.uint64(I0) - ((r + np.uint64(1)) >> np.uint64(1)),
+                          ((q + np.uint64(2)) * np.uint64(I0) - n) >> np.uint64(1))
+
+
+def test_single_multiply_quotient_fails_past_the_bound():
+    """The bound matters: for I0 = 30000, k = 16 (k I0^2 >= 2^32) the single multiply misreads
+    n = 359999 as 12 instead of 11, so the kernels keep the 40-bit reciprocal there."""
+    I0, k = 30000, 16
+    assert k * I0 * I0 >= (1 << 32)
+    n = np.uint64(359999)
+    m32 = np.uint64(((1 << 32) + I0 - 1) // I0)
+    assert int((n * m32) >> np.uint64(32)) == 12 and int(n) // I0 == 11
