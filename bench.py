@@ -151,7 +151,7 @@ class Instrumented:
         M, d, F = bb.B * bb.T, bb.d, bb.F
         dev = bb.x[0].device
         self.a1 = torch.empty((M, d), dtype=torch.int8, device=dev)
-        self.qkv = torch.empty((M, 3 * d), dtype=torch.int8, device=dev)
+        self.qkv = torch.empty((M, 3 * d), dtype=torch.float16, device=dev)  # int8 values, fp16 carrier
         self.o = torch.empty((M, d), dtype=torch.int8, device=dev)
         self.x1 = torch.empty((M, d), dtype=torch.int16, device=dev)
         self.a2 = torch.empty((M, d), dtype=torch.int8, device=dev)
@@ -186,7 +186,7 @@ class Instrumented:
             self._rec("layernorm", lambda: ilw.int_layernorm(x, t["ln1_beta"], t["ln1_mult"], t["ln1_shift"],
                                                              p["ln_iters"], 8, out=self.a1))
             self._rec("gemm_qkv", lambda: ilw.gemm_requant(self.a1, t["w_qkv_p"], 3 * d, t["b_qkv"], t["m_qkv"],
-                                                           t["s_qkv"], 8, out=self.qkv))
+                                                           t["s_qkv"], ilw.I8_IN_F16, out=self.qkv))
             kind = "attention_global" if p["win_side"] <= 1 else "attention_window"
             self._rec(kind, lambda: ilw.shiftmax_attn(self.qkv, B, T, p["H"], d // p["H"], p["win_side"], p["smx"],
                                                       p["m_o"], p["s_o"], out=self.o))

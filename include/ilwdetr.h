@@ -40,6 +40,12 @@ enum {
     ILW_ERR_TIMEOUT = -4      /* a kernel's bounded wait expired (see ilwdetr_device_status) */
 };
 
+/* Activation form code: int8-range integers (|v| <= 127) stored as fp16, which holds them exactly.
+ * It is the operand form of the fp16 tensor-core kernels; a producer that writes it saves its
+ * consumer the int8 -> fp16 conversion.  Accepted where an argument says so (out_bits of
+ * ilwdetr_gemm_requant, qkv_form of ilwdetr_shiftmax_attn); 8 denotes plain int8 there. */
+#define ILW_I8_IN_F16 108
+
 /* Library version string, e.g. "ilwdetr 0.1 sm_103a". */
 const char *ilwdetr_version(void);
 /* Message of the last failing call on this thread ("" if none). */
@@ -89,6 +95,7 @@ int ilwdetr_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, ilw
  *   acc[i,c] = sum_k A[i,k] W[c,k] + bias[c]      (exact; must fit int32)
  *   out_bits 8 / 16: C[i,c] = satN(rq(acc; mult[c], shift[c]) [+ rq(res...)]) (int8 / int16)
  *   out_bits 32    : C[i,c] = acc (int32; mult, shift and res ignored and may be NULL)
+ *   out_bits ILW_I8_IN_F16: the out_bits 8 values, stored as fp16 (C is fp16 [M, ldc])
  *   bias may be NULL (0).  C has leading dimension ldc (elements). */
 int ilwdetr_gemm_requant(const int8_t *A, int64_t lda, const void *Wp, const int32_t *bias,
                          const int32_t *mult, const int32_t *shift, int32_t M, int32_t N,
@@ -147,14 +154,15 @@ int ilwdetr_int_layernorm(const void *X, int32_t in_bits, int64_t ldx, int64_t r
 /* Multi-head attention with Constrained Shiftmax (Sec. 3.2.1 integer MatMul, Sec. 3.3.2):
  *   scores = q k^T (int32; 1/sqrt(dh) is folded into the score scale, hence into p->I0),
  *   P = ConstrainedShiftmax(scores) (u8), O = P V (int32), out = sat8(rq(O; m_o, s_o)).
- * Q, K, V: token-major int8, element (b, t, h, e) at [(b*T + t) * ld_qkv + h*dh + e]
- * (16-byte aligned rows; q|k|v of one [B*T, 3*H*dh] buffer is the usual case).
+ * Q, K, V: token-major, element (b, t, h, e) at [(b*T + t) * ld_qkv + h*dh + e] (elements), in
+ * the form qkv_form: 8 = int8, ILW_I8_IN_F16 = the same integers as fp16 (16-byte aligned rows;
+ * q|k|v of one [B*T, 3*H*dh] buffer is the usual case).
  * O: int8, element (b, t, h, e) at [(b*T + t) * ld_o + h*dh + e].
  * win_side <= 1: global attention over the T tokens; win_side = n >= 2: the sqrt(T) x sqrt(T)
  * token grid (row-major) is cut into n x n windows and tokens attend within their window
  * (LW-DETR's window attention, Table 1).  dh must be 32 or 64. */
-int ilwdetr_shiftmax_attn(const int8_t *Q, const int8_t *K, const int8_t *V, int64_t ld_qkv,
-                          int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side,
+int ilwdetr_shiftmax_attn(const void *Q, const void *K, const void *V, int64_t ld_qkv,
+                          int32_t qkv_form, int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side,
                           const ilw_shiftmax_t *p, int32_t m_o, int32_t s_o, int8_t *O,
                           int64_t ld_o, ilw_stream_t stream);
 

@@ -11,7 +11,7 @@ import ctypes as C
 import os
 
 __all__ = [
-    "lib", "IlwError", "version", "pack_weight", "gemm_requant", "gemm_gelu", "split_conv",
+    "lib", "IlwError", "I8_IN_F16", "version", "pack_weight", "gemm_requant", "gemm_gelu", "split_conv",
     "shiftmax_rows", "sdshiftgelu", "int_layernorm", "shiftmax_attn", "deform_attn",
     "BlockWeights", "block_forward", "block_workspace_bytes", "device_status",
     "patch_embed", "patch_embed_workspace_bytes", "Backbone", "Graphed",
@@ -24,6 +24,11 @@ _lib = None
 
 class IlwError(RuntimeError):
     pass
+
+
+# ILW_I8_IN_F16: int8-range integers carried as fp16 (an out_bits value of gemm_requant and the
+# float16 q|k|v form of shiftmax_attn)
+I8_IN_F16 = 108
 
 
 class ShiftmaxT(C.Structure):
@@ -76,7 +81,7 @@ SIGNATURES = {
     "ilwdetr_sdshiftgelu": ([_VP, _VP, _I64, C.POINTER(GeluT), _VP], C.c_int),
     "ilwdetr_int_layernorm": ([_VP, _I32, _I64, _I64, _I32, _VP, _VP, _VP, _I32, _VP, _I32, _I64,
                                _VP], C.c_int),
-    "ilwdetr_shiftmax_attn": ([_VP, _VP, _VP, _I64, _I32, _I32, _I32, _I32, _I32,
+    "ilwdetr_shiftmax_attn": ([_VP, _VP, _VP, _I64, _I32, _I32, _I32, _I32, _I32, _I32,
                                C.POINTER(ShiftmaxT), _I32, _I32, _VP, _I64, _VP], C.c_int),
     "ilwdetr_deform_attn": ([_VP, C.POINTER(_I32), _I32, _VP, _VP, _VP, _I32, _I32, _I32, _I32,
                              _I32, _I32, _I32, _VP, _VP], C.c_int),
@@ -153,11 +158,12 @@ def pack_weight(W):
 
 
 def gemm_requant(A, Wp, N, bias, mult, shift, out_bits=8, res=None, m_r=0, s_r=0, out=None):
-    """ilwdetr_gemm_requant: A int8 [M, K] x packed W [N, K] -> int8/int16/int32 [M, N]."""
+    """ilwdetr_gemm_requant: A int8 [M, K] x packed W [N, K] -> int8/int16/int32 [M, N], or, with
+    out_bits I8_IN_F16, the int8 values as float16."""
     import torch
 
     M, K = A.shape
-    dt = {8: torch.int8, 16: torch.int16, 32: torch.int32}[out_bits]
+    dt = {8: torch.int8, 16: torch.int16, 32: torch.int32, I8_IN_F16: torch.float16}[out_bits]
     if out is None:
         out = torch.empty((M, N), dtype=dt, device=A.device)
     r = None
@@ -250,16 +256,18 @@ def int_layernorm(X, beta, mult, shift, iters=10, out_bits=8, out=None):
 
 
 def shiftmax_attn(qkv, B, T, H, dh, win_side, smx: dict, m_o, s_o, out=None):
-    """ilwdetr_shiftmax_attn on a token-major [B*T, 3*H*dh] int8 q|k|v buffer -> [B*T, H*dh]."""
+    """ilwdetr_shiftmax_attn on a token-major [B*T, 3*H*dh] q|k|v buffer (int8, or float16
+    holding the int8 values) -> int8 [B*T, H*dh]."""
     import torch
 
     d = H * dh
     if out is None:
         out = torch.empty((B * T, d), dtype=torch.int8, device=qkv.device)
-    base = qkv.data_ptr()
+    form = I8_IN_F16 if qkv.dtype == torch.float16 else 8
+    base, es = qkv.data_ptr(), qkv.element_size()
     p = _smx(smx)
-    _check(lib().ilwdetr_shiftmax_attn(C.c_void_p(base), C.c_void_p(base + d), C.c_void_p(base + 2 * d),
-                                       qkv.stride(0), B, T, H, dh, win_side, C.byref(p), m_o, s_o,
+    _check(lib().ilwdetr_shiftmax_attn(C.c_void_p(base), C.c_void_p(base + d * es), C.c_void_p(base + 2 * d * es),
+                                       qkv.stride(0), form, B, T, H, dh, win_side, C.byref(p), m_o, s_o,
                                        _ptr(out), out.stride(0), _stream()), "shiftmax_attn")
     return out
 

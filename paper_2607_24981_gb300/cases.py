@@ -5,7 +5,7 @@
 Each case builds its seeded inputs (shapes of the paper's Medium model and of the nonlinearity
 sweep), runs the entry point `reps` times after 3 warm-up calls and prints the mean device time
 with the case's algorithmic work.  Cases:
-  attn_global   attention, 2 images x 1600 tokens, 6 heads, dh 64, global
+  attn_global   attention, 2 images x 1600 tokens, 6 heads, dh 64, global (fp16-carried q|k|v)
   attn_window   attention, 8 images x 1600 tokens, 6 heads, 2x2 windows of 400
   gemm_qkv / gemm_proj / gemm_fc1_gelu / gemm_fc2
                 the block GEMMs at 12800 tokens, d 384, MLP 1536
@@ -42,7 +42,8 @@ def build(case: str):
     if case.startswith("attn"):
         B, T, H, dh = (2, 1600, 6, 64) if case == "attn_global" else (8, 1600, 6, 64)
         win = 0 if case == "attn_global" else 2
-        qkv = _dev(synth.uniform_int(0, "case.qkv", (B * T, 3 * H * dh), -127, 127, np.int8))
+        # q|k|v as the QKV GEMM hands them over: the int8 values carried in float16
+        qkv = _dev(synth.uniform_int(0, "case.qkv", (B * T, 3 * H * dh), -127, 127, np.int8).astype(np.float16))
         out = torch.empty((B * T, H * dh), dtype=torch.int8, device="cuda")
         scores = B * H * (T * T if win == 0 else 4 * (T // 4) ** 2)
         return (lambda: ilw.shiftmax_attn(qkv, B, T, H, dh, win, {"I0": 6000}, 3 << 29, 36, out=out),
@@ -57,9 +58,9 @@ def build(case: str):
         if case == "gemm_fc1_gelu":
             out = torch.empty((M, N), dtype=torch.int8, device="cuda")
             fn = lambda: ilw.gemm_gelu(A, Wp, N, b, m, s, {"I0": 1000}, 3 << 29, 40, out=out)
-        elif case == "gemm_qkv":
-            out = torch.empty((M, N), dtype=torch.int8, device="cuda")
-            fn = lambda: ilw.gemm_requant(A, Wp, N, b, m, s, 8, out=out)
+        elif case == "gemm_qkv":  # q|k|v written as fp16-carried int8, as the encoder block does
+            out = torch.empty((M, N), dtype=torch.float16, device="cuda")
+            fn = lambda: ilw.gemm_requant(A, Wp, N, b, m, s, ilw.I8_IN_F16, out=out)
         else:
             res = _dev(synth.uniform_int(1, "case.res", (M, N), -3000, 3000, np.int16))
             out = torch.empty((M, N), dtype=torch.int16, device="cuda")

@@ -120,8 +120,8 @@ int ilwdetr_gemm_requant(const int8_t *A, int64_t lda, const void *Wp, const int
                          ilw_stream_t stream) {
     int rc = gemm_common(A, lda, Wp, M, N, K);
     if (rc) return rc;
-    if (out_bits != 8 && out_bits != 16 && out_bits != 32)
-        return fail(ILW_ERR_INVALID_ARG, "out_bits=%d must be 8, 16 or 32", out_bits);
+    if (out_bits != 8 && out_bits != 16 && out_bits != 32 && out_bits != ILW_I8_IN_F16)
+        return fail(ILW_ERR_INVALID_ARG, "out_bits=%d must be 8, 16, 32 or ILW_I8_IN_F16", out_bits);
     if (M == 0 || N == 0) return ILW_OK;
     if (!C || ldc < N) return fail(ILW_ERR_INVALID_ARG, "C is NULL or ldc < N");
     if (out_bits != 32 && (!mult || !shift)) return fail(ILW_ERR_INVALID_ARG, "mult/shift are NULL");
@@ -251,8 +251,8 @@ int ilwdetr_int_layernorm(const void *X, int32_t in_bits, int64_t ldx, int64_t r
     return cuda_status(ilw::launch_layernorm(lp, (cudaStream_t)stream), "int_layernorm");
 }
 
-static int attn_params(ilw::AttnParams &ap, const int8_t *Q, const int8_t *K, const int8_t *V, int64_t ld_qkv,
-                       int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side,
+static int attn_params(ilw::AttnParams &ap, const void *Q, const void *K, const void *V, int64_t ld_qkv,
+                       int32_t qkv_form, int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side,
                        const ilw_shiftmax_t *p, int32_t m_o, int32_t s_o, int8_t *O, int64_t ld_o) {
     int rc = check_shiftmax(p);
     if (rc) return rc;
@@ -260,11 +260,15 @@ static int attn_params(ilw::AttnParams &ap, const int8_t *Q, const int8_t *K, co
     if (B < 0 || T < 0 || H < 1) return fail(ILW_ERR_INVALID_ARG, "attention: bad sizes");
     if (dh != 32 && dh != 64) return fail(ILW_ERR_UNSUPPORTED, "attention: dh=%d must be 32 or 64", dh);
     if (!Q || !K || !V || !O) return fail(ILW_ERR_INVALID_ARG, "attention: NULL pointer");
-    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || ld_qkv % 16 || ld_qkv < (int64_t)H * dh)
-        return fail(ILW_ERR_INVALID_ARG, "attention: q/k/v must be 16-byte aligned with ld_qkv %% 16 == 0");
+    if (qkv_form != 8 && qkv_form != ILW_I8_IN_F16)
+        return fail(ILW_ERR_INVALID_ARG, "attention: qkv_form=%d must be 8 or ILW_I8_IN_F16", qkv_form);
+    const int64_t esz = qkv_form == 8 ? 1 : 2;
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || (ld_qkv * esz) % 16 || ld_qkv < (int64_t)H * dh)
+        return fail(ILW_ERR_INVALID_ARG, "attention: q/k/v must be 16-byte aligned with 16-byte aligned rows");
     if (ld_o < (int64_t)H * dh) return fail(ILW_ERR_INVALID_ARG, "attention: ld_o < H*dh");
     ap = {};
     ap.Q = Q; ap.K = K; ap.V = V; ap.ld_qkv = ld_qkv;
+    ap.qkv_f16 = qkv_form == ILW_I8_IN_F16 ? 1 : 0;
     ap.B = B; ap.T = T; ap.H = H; ap.dh = dh;
     ap.nw = win_side <= 1 ? 1 : win_side;
     ap.grid_side = 0;
@@ -281,12 +285,12 @@ static int attn_params(ilw::AttnParams &ap, const int8_t *Q, const int8_t *K, co
     return ILW_OK;
 }
 
-int ilwdetr_shiftmax_attn(const int8_t *Q, const int8_t *K, const int8_t *V, int64_t ld_qkv, int32_t B,
-                          int32_t T, int32_t H, int32_t dh, int32_t win_side, const ilw_shiftmax_t *p,
+int ilwdetr_shiftmax_attn(const void *Q, const void *K, const void *V, int64_t ld_qkv, int32_t qkv_form,
+                          int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side, const ilw_shiftmax_t *p,
                           int32_t m_o, int32_t s_o, int8_t *O, int64_t ld_o, ilw_stream_t stream) {
     if (B == 0 || T == 0) return ILW_OK;
     ilw::AttnParams ap;
-    int rc = attn_params(ap, Q, K, V, ld_qkv, B, T, H, dh, win_side, p, m_o, s_o, O, ld_o);
+    int rc = attn_params(ap, Q, K, V, ld_qkv, qkv_form, B, T, H, dh, win_side, p, m_o, s_o, O, ld_o);
     if (rc) return rc;
     return cuda_status(ilw::launch_attention(ap, (cudaStream_t)stream), "shiftmax_attn");
 }
@@ -355,7 +359,7 @@ int ilwdetr_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, i
 size_t ilwdetr_block_workspace_bytes(int32_t B, int32_t T, int32_t d, int32_t F) {
     if (B < 0 || T < 0 || d < 0 || F < 0) return 0;
     size_t M = (size_t)B * T;
-    return align256(M * d) /*a1*/ + align256(M * 3 * d) /*qkv*/ + align256(M * d) /*O*/ +
+    return align256(M * d) /*a1*/ + align256(M * 3 * d * 2) /*qkv (fp16)*/ + align256(M * d) /*O*/ +
            align256(M * d * 2) /*x1*/ + align256(M * d) /*a2*/ + align256(M * F) /*h*/;
 }
 
@@ -375,7 +379,7 @@ int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t
     const int32_t M = B * T;
     char *ws = (char *)workspace;
     int8_t *a1 = (int8_t *)ws; ws += align256((size_t)M * d);
-    int8_t *qkv = (int8_t *)ws; ws += align256((size_t)M * 3 * d);
+    __half *qkv = (__half *)ws; ws += align256((size_t)M * 3 * d * 2);  // q|k|v as fp16 (ILW_I8_IN_F16)
     int8_t *o = (int8_t *)ws; ws += align256((size_t)M * d);
     int16_t *x1 = (int16_t *)ws; ws += align256((size_t)M * d * 2);
     int8_t *a2 = (int8_t *)ws; ws += align256((size_t)M * d);
@@ -383,9 +387,10 @@ int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t
     int rc;
     if ((rc = ilwdetr_int_layernorm(x, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, a1, 8, d, stream)))
         return rc;
-    if ((rc = ilwdetr_gemm_requant(a1, d, p->w_qkv, p->b_qkv, p->m_qkv, p->s_qkv, M, 3 * d, d, 8, qkv, 3 * d, nullptr, stream)))
+    if ((rc = ilwdetr_gemm_requant(a1, d, p->w_qkv, p->b_qkv, p->m_qkv, p->s_qkv, M, 3 * d, d, ILW_I8_IN_F16, qkv, 3 * d,
+                                   nullptr, stream)))
         return rc;
-    if ((rc = ilwdetr_shiftmax_attn(qkv, qkv + d, qkv + 2 * d, 3 * d, B, T, H, d / H, p->win_side, &p->smx, p->m_o,
+    if ((rc = ilwdetr_shiftmax_attn(qkv, qkv + d, qkv + 2 * d, 3 * d, ILW_I8_IN_F16, B, T, H, d / H, p->win_side, &p->smx, p->m_o,
                                     p->s_o, o, d, stream)))
         return rc;
     ilw_residual_t r1{x, d, M, p->m_r1, p->s_r1};

@@ -41,6 +41,13 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t 
                  : "r"(addr));
 }
 
+// 16-byte asynchronous global -> shared copy; src_bytes 0 writes zeros (rows past the group)
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 // two int8 (low bytes of w >> 0 and w >> 8) -> fp16x2, exact: 0x6400 | (b ^ 0x80) is 1152 + b
 __device__ __forceinline__ uint32_t i8x2_to_h2(uint32_t w) {
     uint32_t x = __byte_perm(w ^ 0x8080u, 0x64646464u, 0x4140);
@@ -75,7 +82,9 @@ struct Group {
     }
 };
 
-template <int DH, bool FASTQ>
+// QF16: q, k, v arrive as fp16 (the int8 values, exact) and are copied to shared memory as they
+// are; otherwise they arrive as int8 and are converted on the way in.
+template <int DH, bool FASTQ, bool QF16>
 __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     constexpr int LDH = DH * 2 + 16;  // padded fp16 row (bytes): conflict-free ldmatrix
     constexpr int KS = DH / 16;       // k16 steps of q k^T
@@ -107,10 +116,22 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
 
     // ---- Q rows of this warp -> fp16 A fragments (rows g and g + 8 of the warp's 16)
     uint32_t qa[KS][4];
-    {
+    if constexpr (QF16) {
         const int r0 = q0 + warp * 16 + g, r1 = r0 + 8;
-        const int8_t *Q0 = r0 < Tg ? p.Q + gr.token(r0) * p.ld_qkv + hoff : nullptr;
-        const int8_t *Q1 = r1 < Tg ? p.Q + gr.token(r1) * p.ld_qkv + hoff : nullptr;
+        const __half *Q0 = r0 < Tg ? (const __half *)p.Q + gr.token(r0) * p.ld_qkv + hoff : nullptr;
+        const __half *Q1 = r1 < Tg ? (const __half *)p.Q + gr.token(r1) * p.ld_qkv + hoff : nullptr;
+#pragma unroll
+        for (int ks = 0; ks < KS; ++ks) {
+            const int c = ks * 16 + 2 * t;
+            qa[ks][0] = Q0 ? *(const uint32_t *)(Q0 + c) : 0u;
+            qa[ks][1] = Q1 ? *(const uint32_t *)(Q1 + c) : 0u;
+            qa[ks][2] = Q0 ? *(const uint32_t *)(Q0 + c + 8) : 0u;
+            qa[ks][3] = Q1 ? *(const uint32_t *)(Q1 + c + 8) : 0u;
+        }
+    } else {
+        const int r0 = q0 + warp * 16 + g, r1 = r0 + 8;
+        const int8_t *Q0 = r0 < Tg ? (const int8_t *)p.Q + gr.token(r0) * p.ld_qkv + hoff : nullptr;
+        const int8_t *Q1 = r1 < Tg ? (const int8_t *)p.Q + gr.token(r1) * p.ld_qkv + hoff : nullptr;
 #pragma unroll
         for (int ks = 0; ks < KS; ++ks) {
             const int c = ks * 16 + 2 * t;
@@ -137,8 +158,8 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
             vreg[i] = make_uint4(0, 0, 0, 0);
             if (key < Tg) {
                 const int64_t off = gr.token(key) * p.ld_qkv + hoff + ch * 16;
-                kreg[i] = __ldg((const uint4 *)(p.K + off));
-                if (with_v) vreg[i] = __ldg((const uint4 *)(p.V + off));
+                kreg[i] = __ldg((const uint4 *)((const int8_t *)p.K + off));
+                if (with_v) vreg[i] = __ldg((const uint4 *)((const int8_t *)p.V + off));
             }
         }
     };
@@ -183,16 +204,47 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
             }
         }
     };
+    // fp16 input: 16-byte asynchronous copies straight into the padded rows
+    constexpr int CH16 = DH * 2 / 16;             // 16-byte chunks per fp16 row
+    constexpr int PER16 = KB * CH16 / THREADS;    // chunks per thread per key block
+    auto issue16 = [&](int kb, int buf, bool with_v) {
+#pragma unroll
+        for (int i = 0; i < PER16; ++i) {
+            const int c = tid + i * THREADS;
+            const int r = c / CH16, ch = c % CH16;
+            const int key = kb * KB + r;
+            const bool ok = key < Tg;
+            const int64_t off = gr.token(ok ? key : 0) * p.ld_qkv + hoff + ch * 8;  // elements
+            cp_async16((uint32_t)__cvta_generic_to_shared(Ks[buf] + r * LDH + ch * 16), (const __half *)p.K + off,
+                       ok ? 16u : 0u);
+            if (with_v)
+                cp_async16((uint32_t)__cvta_generic_to_shared(Vs[buf] + r * LDH + ch * 16), (const __half *)p.V + off,
+                           ok ? 16u : 0u);
+        }
+        cp_async_commit();
+    };
     // one pass over the key blocks: body(kb, buf, full) with the block staged in buffer buf
     auto sweep = [&](bool with_v, auto &&body) {
-        fetch(0, with_v);
-        commit(0, with_v);
+        if constexpr (QF16) {
+            issue16(0, 0, with_v);
+            cp_async_wait_all();
+        } else {
+            fetch(0, with_v);
+            commit(0, with_v);
+        }
         __syncthreads();
         for (int kb = 0; kb < nkb; ++kb) {
             const int buf = kb & 1;
-            if (kb + 1 < nkb) fetch(kb + 1, with_v);
-            body(kb, buf, (kb + 1) * KB <= Tg);
-            if (kb + 1 < nkb) commit(buf ^ 1, with_v);  // buffer buf^1 was released by the last sync
+            // buffer buf^1 was released by the barrier that ended the previous block
+            if constexpr (QF16) {
+                if (kb + 1 < nkb) issue16(kb + 1, buf ^ 1, with_v);
+                body(kb, buf, (kb + 1) * KB <= Tg);
+                if (kb + 1 < nkb) cp_async_wait_all();
+            } else {
+                if (kb + 1 < nkb) fetch(kb + 1, with_v);
+                body(kb, buf, (kb + 1) * KB <= Tg);
+                if (kb + 1 < nkb) commit(buf ^ 1, with_v);
+            }
             __syncthreads();
         }
     };
@@ -333,12 +385,22 @@ cudaError_t launch_attention(const AttnParams &p, cudaStream_t s) {
     if (p.B == 0 || Tg == 0) return cudaSuccess;
     dim3 grid((Tg + QT - 1) / QT, p.H, p.B * G2);
     const bool fastq = p.smx.se.m32 != 0;
-    if (p.dh == 64) {
-        if (fastq) attn_kernel<64, true><<<grid, THREADS, 0, s>>>(p);
-        else attn_kernel<64, false><<<grid, THREADS, 0, s>>>(p);
+    if (p.qkv_f16) {
+        if (p.dh == 64) {
+            if (fastq) attn_kernel<64, true, true><<<grid, THREADS, 0, s>>>(p);
+            else attn_kernel<64, false, true><<<grid, THREADS, 0, s>>>(p);
+        } else {
+            if (fastq) attn_kernel<32, true, true><<<grid, THREADS, 0, s>>>(p);
+            else attn_kernel<32, false, true><<<grid, THREADS, 0, s>>>(p);
+        }
     } else {
-        if (fastq) attn_kernel<32, true><<<grid, THREADS, 0, s>>>(p);
-        else attn_kernel<32, false><<<grid, THREADS, 0, s>>>(p);
+        if (p.dh == 64) {
+            if (fastq) attn_kernel<64, true, false><<<grid, THREADS, 0, s>>>(p);
+            else attn_kernel<64, false, false><<<grid, THREADS, 0, s>>>(p);
+        } else {
+            if (fastq) attn_kernel<32, true, false><<<grid, THREADS, 0, s>>>(p);
+            else attn_kernel<32, false, false><<<grid, THREADS, 0, s>>>(p);
+        }
     }
     return cudaGetLastError();
 }

@@ -131,18 +131,6 @@ __device__ __forceinline__ void tc_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
 
-#define ILW_LD32_REGS(v)                                                                                          \
-    "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),     \
-        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]),     \
-        "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),    \
-        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
-        "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : ILW_LD32_REGS(v)
-        : "r"(taddr));
-}
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
@@ -150,7 +138,6 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
           "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
         : "r"(taddr));
 }
-__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 // Waits for this thread's TMEM loads and marks the 16 destination registers as written by the
 // wait, so that no use of them can be scheduled before the data has arrived.
 __device__ __forceinline__ void tmem_wait_ld16(uint32_t (&v)[16]) {
@@ -184,7 +171,7 @@ struct Smem {
 };
 
 // Output kinds: one compact epilogue per kernel instantiation.
-enum { KIND_RQ8 = 0, KIND_RQ16 = 1, KIND_RAW32 = 2, KIND_GELU8 = 3 };
+enum { KIND_RQ8 = 0, KIND_RQ16 = 1, KIND_RAW32 = 2, KIND_GELU8 = 3, KIND_F16OUT = 4 };  // F16OUT: RQ8 values as fp16
 
 // 16 consecutive int32 of shared memory (16-byte aligned) into registers: four 128-bit loads
 __device__ __forceinline__ void lds16(const int32_t *p, int32_t (&o)[16]) {
@@ -206,10 +193,10 @@ __device__ __forceinline__ int32_t rq_hi(int32_t v, int32_t m, int32_t s) {
 // 16 independent elements overlap.  The fast path (every shift >= 33, the usual case) is decided
 // per chunk, which is uniform across the warp.
 template <int KIND>
-__device__ __forceinline__ void epi_chunk(const EpiParams &ep, int64_t row, const int32_t (&acc)[16],
-                                          const int32_t (&sb)[16], const int32_t (&sm)[16], const int32_t (&ss)[16],
-                                          int32_t col0,
-                                          int32_t N, const uint8_t *gtab, int32_t gT, int32_t (&out)[16]) {
+__device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool has_res, const uint32_t (&rp)[8],
+                                          const int32_t (&acc)[16], const int32_t (&sb)[16],
+                                          const int32_t (&sm)[16], const int32_t (&ss)[16],
+                                          const uint8_t *gtab, int32_t gT, int32_t (&out)[16]) {
     if (KIND == KIND_RAW32) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) out[i] = acc[i] + sb[i];
@@ -239,18 +226,17 @@ __device__ __forceinline__ void epi_chunk(const EpiParams &ep, int64_t row, cons
         }
         return;
     }
-    if (ep.res) {
-        const int16_t *res = ep.res + (row % ep.res_rows) * ep.ldr;
-        const bool rfast = ep.s_r >= 17;  // int16 residual: res * 2^16 fits int32
+    if (has_res) {
+        // rp holds the 16 int16 residuals in pairs; x * 2^16 is the pair word masked or shifted
+        const bool rfast = ep.s_r >= 17;  // then rq(x; m_r, s_r) = rq_hi(x * 2^16; m_r, s_r + 16)
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-            const int32_t x = res[min(col0 + i, N - 1)];
-            const int32_t rr = rfast ? rq_hi(x * 65536, ep.m_r, ep.s_r + 16) : (int32_t)rq((int64_t)x, ep.m_r, ep.s_r);
-            r[i] += rr;
+            const int32_t xs = (i & 1) ? (int32_t)(rp[i >> 1] & 0xFFFF0000u) : (int32_t)(rp[i >> 1] << 16);
+            r[i] += rfast ? rq_hi(xs, ep.m_r, ep.s_r + 16) : (int32_t)rq((int64_t)(xs >> 16), ep.m_r, ep.s_r);
         }
     }
 #pragma unroll
-    for (int i = 0; i < 16; ++i) out[i] = KIND == KIND_RQ8 ? sat8(r[i]) : sat16(r[i]);
+    for (int i = 0; i < 16; ++i) out[i] = (KIND == KIND_RQ8 || KIND == KIND_F16OUT) ? sat8(r[i]) : sat16(r[i]);
 }
 
 template <int BN, int STAGES, int KIND, int NB>
@@ -412,7 +398,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         int32_t *s_bias = (int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + (warp - 6) * 3 * HALF;  // this warp's copy of
         int32_t *s_mult = s_bias + HALF;                                       // the tile's per-column
         int32_t *s_shift = s_mult + HALF;                                      // epilogue parameters
-        constexpr int bits = KIND == KIND_RQ16 ? 16 : (KIND == KIND_RAW32 ? 32 : 8);
+        constexpr int bits = (KIND == KIND_RQ16 || KIND == KIND_F16OUT) ? 16 : (KIND == KIND_RAW32 ? 32 : 8);
         constexpr int PPL = HALF / 32;  // parameters per lane and per array
         // The next tile's parameters are fetched into registers while the current tile is processed.
         int32_t pb[PPL], pm[PPL], ps[PPL];
@@ -447,6 +433,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             tc_fence_after();
             const int64_t row = (int64_t)m0 + 32 * q + lane;
             const bool row_ok = row < p.M;
+            // this row's residual (row modulo res_rows broadcasts a [res_rows, N] table)
+            const int16_t *rrow = (ep.res && row_ok) ? ep.res + (row % ep.res_rows) * ep.ldr + n0 : nullptr;
+            const bool rvec = ((uintptr_t)rrow & 15) == 0;
+            const bool has_res = ep.res != nullptr;
+            uint32_t rp[8];
             const uint32_t tbase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * acc_cols + h * HALF);
             // TMEM load i reads segment i % nseg of chunk i / nseg; load i+1 is in flight while the
             // epilogue of load i's chunk runs.
@@ -457,6 +448,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             for (int i = 0; i < 16; ++i) acc[i] = 0;
             for (int li = 0; li < nld; ++li) {
                 const int c0 = (li / nseg) * 16, sg = li - (li / nseg) * nseg;
+                if (has_res && sg == 0) {  // this chunk's residuals, in flight during the TMEM wait
+                    if (rrow && rvec && n0 + c0 + 16 <= p.N) {
+                        const uint4 a = __ldg((const uint4 *)(rrow + c0)), b = __ldg((const uint4 *)(rrow + c0) + 1);
+                        rp[0] = a.x; rp[1] = a.y; rp[2] = a.z; rp[3] = a.w;
+                        rp[4] = b.x; rp[5] = b.y; rp[6] = b.z; rp[7] = b.w;
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            const int cl = n0 + c0 + 2 * j;
+                            const uint32_t lo = (rrow && cl < p.N) ? (uint16_t)rrow[c0 + 2 * j] : 0u;
+                            const uint32_t hi = (rrow && cl + 1 < p.N) ? (uint16_t)rrow[c0 + 2 * j + 1] : 0u;
+                            rp[j] = lo | (hi << 16);
+                        }
+                    }
+                }
                 tmem_wait_ld16(v);
                 if (p.branch_rq) {
                     const int32_t mb = p.seg[sg].m_b, sbb = p.seg[sg].s_b;
@@ -482,7 +488,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 const int ncol = min(16, p.N - (n0 + c0));
                 if (row_ok && ncol > 0) {
                     int32_t out[16];
-                    epi_chunk<KIND>(ep, row, acc, cb, cm, cs, n0 + c0, p.N, gtab, p.gelu_T, out);
+                    epi_chunk<KIND>(ep, has_res, rp, acc, cb, cm, cs, gtab, p.gelu_T, out);
+                    if constexpr (KIND == KIND_F16OUT) {  // |v| <= 127: fp16 bits of 1152 + v, minus 1152
+                        const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
+#pragma unroll
+                        for (int i = 0; i < 16; i += 2) {
+                            uint32_t x = (uint32_t)(0x6480 + out[i]) | ((uint32_t)(0x6480 + out[i + 1]) << 16);
+                            __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), k1152);
+                            x = *reinterpret_cast<uint32_t *>(&h);
+                            out[i] = (int32_t)(x & 0xFFFFu);
+                            out[i + 1] = (int32_t)(x >> 16);
+                        }
+                    }
                     char *dst = (char *)ep.C + (row * ep.ldc + n0 + c0) * (bits / 8);
                     const bool vec = ncol == 16 && (((uintptr_t)dst & 15) == 0);
                     if constexpr (bits == 8) {
@@ -690,6 +707,10 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
         if (ep.kind == EPI_GELU) return launch_tc<BN, STAGES, KIND_GELU8, NB>(tp, s);
     } else {
         if (ep.kind == EPI_GELU) return cudaErrorInvalidValue;  // split convolutions requantise only
+    }
+    if (ep.out_bits == kOutI8InF16) {
+        if constexpr (NB == 1) return launch_tc<BN, STAGES, KIND_F16OUT, NB>(tp, s);
+        else return cudaErrorInvalidValue;
     }
     if (ep.out_bits == 8) return launch_tc<BN, STAGES, KIND_RQ8, NB>(tp, s);
     if (ep.out_bits == 16) return launch_tc<BN, STAGES, KIND_RQ16, NB>(tp, s);

@@ -58,10 +58,11 @@ struct GemmProblem {
     GemmBranch br[kMaxBranches];
 };
 enum EpiKind { EPI_REQUANT = 0, EPI_GELU = 1 };
+constexpr int32_t kOutI8InF16 = 108;  // the out_bits 8 values stored as fp16 (ILW_I8_IN_F16)
 struct EpiParams {
     EpiKind kind;
     const int32_t *bias, *mult, *shift;
-    int32_t out_bits;  // 8, 16, 32 (EPI_REQUANT)
+    int32_t out_bits;  // 8, 16, 32, or kOutI8InF16 (EPI_REQUANT)
     void *C;
     int64_t ldc;
     // residual (EPI_REQUANT, out_bits 8/16)
@@ -104,8 +105,9 @@ cudaError_t launch_layernorm(const LnParams &p, cudaStream_t s);
 
 // ---------------------------------------------------------------- attention
 struct AttnParams {
-    const int8_t *Q, *K, *V;
-    int64_t ld_qkv;
+    const void *Q, *K, *V;  // int8, or fp16 when qkv_f16 (the same integers)
+    int64_t ld_qkv;         // elements
+    int32_t qkv_f16;
     int32_t B, T, H, dh;
     int32_t nw;        // windows per side (1 = global)
     int32_t grid_side; // sqrt(T) when nw > 1

@@ -167,29 +167,43 @@ __global__ void sdshiftgelu_tail(const int32_t *X, int32_t *Y, int64_t start, in
 }
 
 // ------------------------------------------------------------------ I-LayerNorm
-// Newton integer square root from 2^16, exactly `iters` steps, stopping only at 0 (V = 0).
-__device__ __forceinline__ uint64_t newton_isqrt(uint64_t V, int iters) {
-    uint64_t r = 1ull << 16;
+// Newton's integer square root r <- (r + V / r) >> 1 from r = 2^16, exactly `iters` steps (the loop
+// stops at 0, which only V = 0 reaches), cut short once the rest of the sequence is known: a fixed
+// point repeats forever, and once r_{i+1} = r_{i-1} the iterates alternate between two values, so
+// r_iters is read off the parity of the steps left.  Identical result, fewer 64-bit divisions.
+__device__ __forceinline__ uint64_t newton_isqrt_early(uint64_t V, int iters) {
+    uint64_t r = 1ull << 16, prev = ~0ull;
     for (int it = 0; it < iters; ++it) {
         if (r == 0) break;
-        r = (r + V / r) >> 1;
+        const uint64_t nx = (r + V / r) >> 1;
+        if (nx == r) break;
+        if (nx == prev) {
+            r = ((iters - it - 1) & 1) ? r : nx;
+            break;
+        }
+        prev = r;
+        r = nx;
     }
     return r < 1 ? 1 : r;
 }
 
-// 4 consecutive elements of one row as int32 (vector load: int4 for int32 input, 8 bytes for int16)
-template <typename TIn>
-__device__ __forceinline__ void load4(const TIn *x, int32_t (&o)[4]);
-template <>
-__device__ __forceinline__ void load4<int32_t>(const int32_t *x, int32_t (&o)[4]) {
-    const int4 v = __ldcs((const int4 *)x);
-    o[0] = v.x; o[1] = v.y; o[2] = v.z; o[3] = v.w;
-}
-template <>
-__device__ __forceinline__ void load4<int16_t>(const int16_t *x, int32_t (&o)[4]) {
-    const uint2 v = __ldcs((const uint2 *)x);
-    o[0] = (int16_t)(v.x & 0xffff); o[1] = (int16_t)(v.x >> 16); o[2] = (int16_t)(v.y & 0xffff); o[3] = (int16_t)(v.y >> 16);
-}
+// Row storage of the multi-row kernel: int16 rows stay packed (two per 32-bit register).
+template <typename TIn> struct Chunk;
+template <> struct Chunk<int16_t> {
+    uint2 w;
+    __device__ __forceinline__ void load(const int16_t *x) { w = __ldcs((const uint2 *)x); }
+    __device__ __forceinline__ void zero() { w = make_uint2(0, 0); }
+    __device__ __forceinline__ int32_t get(int u) const {
+        const uint32_t h = u < 2 ? w.x : w.y;
+        return (u & 1) ? ((int32_t)h >> 16) : ((int32_t)(h << 16) >> 16);
+    }
+};
+template <> struct Chunk<int32_t> {
+    int4 w;
+    __device__ __forceinline__ void load(const int32_t *x) { w = __ldcs((const int4 *)x); }
+    __device__ __forceinline__ void zero() { w = make_int4(0, 0, 0, 0); }
+    __device__ __forceinline__ int32_t get(int u) const { return u == 0 ? w.x : (u == 1 ? w.y : (u == 2 ? w.z : w.w)); }
+};
 template <typename TOut>
 __device__ __forceinline__ void store4(TOut *y, const int32_t (&o)[4]);
 template <>
@@ -203,17 +217,37 @@ __device__ __forceinline__ void store4<int16_t>(int16_t *y, const int32_t (&o)[4
                              (uint32_t)(uint16_t)o[2] | ((uint32_t)(uint16_t)o[3] << 16));
 }
 
+// Sums R per-lane partials (one per row) over the warp so that lane l ends with the total of row
+// l % R: log2 R exchange steps each hand half of the rows to the partner lane (R - 1 shuffles),
+// then 5 - log2 R ordinary butterfly steps.
+template <int R, typename T>
+__device__ __forceinline__ T rows_reduce(T (&v)[R], int lane) {
+#pragma unroll
+    for (int o = 1, n = R; o < R; o <<= 1, n >>= 1) {
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < n / 2; ++i) {
+            const T keep = up ? v[2 * i + 1] : v[2 * i];
+            const T send = up ? v[2 * i] : v[2 * i + 1];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+#pragma unroll
+    for (int o = R; o < 32; o <<= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+    return v[0];
+}
+
 // ROWS rows per warp, held in registers.  Each lane owns 4-element chunks (lane + 32 j) of every
-// row; all loads of the warp's rows are issued before any reduction.  Lanes share the two integer
-// row sums, then lane r runs Newton's iteration (the sequential part) for row r, so a warp pays for
-// one Newton sequence per ROWS rows.  V = sum (x - mu)^2 = sum x^2 - 2 mu sum x + C mu^2, exactly.
+// row; all loads of the warp's rows are issued before any reduction.  Lane l then holds the sums
+// of row l % ROWS and runs Newton's iteration for it, so a warp pays for one Newton sequence per
+// ROWS rows.  V = sum (x - mu)^2 = sum x^2 - 2 mu sum x + C mu^2, exactly.
 template <typename TIn, typename TOut, int NCH, int ROWS>
 __global__ void __launch_bounds__(256) layernorm_multi(const LnParams p) {
     const int lane = threadIdx.x & 31;
     const int64_t row0 = ((int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * ROWS;
     if (row0 >= p.rows) return;
     const int C = p.C, nchunk = C >> 2;
-    int32_t v[ROWS][NCH][4];
+    Chunk<TIn> v[ROWS][NCH];
 #pragma unroll
     for (int r = 0; r < ROWS; ++r) {
         const bool ok = row0 + r < p.rows;
@@ -221,32 +255,33 @@ __global__ void __launch_bounds__(256) layernorm_multi(const LnParams p) {
 #pragma unroll
         for (int j = 0; j < NCH; ++j) {
             const int ch = lane + 32 * j;
-            if (ok && ch < nchunk) load4<TIn>(x + 4 * ch, v[r][j]);
-            else v[r][j][0] = v[r][j][1] = v[r][j][2] = v[r][j][3] = 0;
+            if (ok && ch < nchunk) v[r][j].load(x + 4 * ch);
+            else v[r][j].zero();
         }
     }
-    int64_t my_s = 0, my_q = 0;
+    int64_t ps[ROWS], pq[ROWS];
 #pragma unroll
     for (int r = 0; r < ROWS; ++r) {
-        int64_t s = 0, q = 0;
+        int64_t sr = 0, qr = 0;
 #pragma unroll
         for (int j = 0; j < NCH; ++j)
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
-                s += v[r][j][u];
-                q += (int64_t)v[r][j][u] * v[r][j][u];
+                const int32_t x = v[r][j].get(u);
+                sr += x;
+                qr += (int64_t)x * x;
             }
-        s = warp_sum_i64(s);
-        q = warp_sum_i64(q);
-        if (lane == r) { my_s = s; my_q = q; }
+        ps[r] = sr;
+        pq[r] = qr;
     }
-    // lane r < ROWS: mean, variance and Newton for row r
+    const int64_t my_s = rows_reduce<ROWS>(ps, lane), my_q = rows_reduce<ROWS>(pq, lane);
+    // lane l: mean, variance and Newton for row l % ROWS
     const int64_t den = 2 * (int64_t)C, num = 2 * my_s + C;
     int64_t mu = num / den;
     if ((num % den) != 0 && num < 0) mu -= 1;
     const uint64_t V = (uint64_t)(my_q - 2 * mu * my_s + (int64_t)C * mu * mu);
-    const uint64_t R = lane < ROWS ? newton_isqrt(V, p.iters) : 1;
-    const int64_t F = (int64_t)(0x7fffffffull / R);
+    const uint64_t R = newton_isqrt_early(V, p.iters);
+    const int64_t F = R < (1ull << 32) ? (int64_t)(0x7fffffffu / (uint32_t)R) : 0;
 #pragma unroll
     for (int r = 0; r < ROWS; ++r) {
         if (row0 + r >= p.rows) break;
@@ -265,7 +300,7 @@ __global__ void __launch_bounds__(256) layernorm_multi(const LnParams p) {
                 int32_t o[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const int64_t n = (((int64_t)v[r][j][u] - mur) * Fr) >> 1;
+                    const int64_t n = (((int64_t)v[r][j].get(u) - mur) * Fr) >> 1;
                     const int64_t t = rq(n + bb[u], mm[u], ss[u]);
                     o[u] = sizeof(TOut) == 1 ? sat8(t) : sat16(t);
                 }
@@ -305,13 +340,8 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const LnParams p) {
         }
     }
     V = warp_sum_u64(V);
-    // Newton integer square root from 2^16, exactly `iters` steps (stops at 0 only if V = 0)
-    uint64_t r = 1ull << 16;
-    for (int it = 0; it < p.iters; ++it) {
-        if (r == 0) break;
-        r = (r + V / r) >> 1;
-    }
-    if (r < 1) r = 1;
+    // Newton integer square root from 2^16, `iters` steps (stops at 0 only if V = 0)
+    const uint64_t r = newton_isqrt_early(V, p.iters);
     const int64_t F = (int64_t)(0x7fffffffull / r);
     TOut *yo = (TOut *)p.Y + row * p.ldy;
 #pragma unroll
@@ -331,8 +361,8 @@ cudaError_t ln_dispatch(const LnParams &p, cudaStream_t s) {
     const int eb = sizeof(TIn), ob = sizeof(TOut);
     const bool vec = p.C % 4 == 0 && p.ldx % 4 == 0 && p.ldy % 4 == 0 && ((uintptr_t)p.X % (4 * eb)) == 0 &&
                      ((uintptr_t)p.Y % (4 * ob)) == 0 && (((uintptr_t)p.beta | (uintptr_t)p.mult | (uintptr_t)p.shift) % 16) == 0;
-    if (vec && p.C <= 512) {  // 4 rows per warp in registers, vector loads, lane-parallel Newton
-        constexpr int ROWS = 4;
+    if (vec && p.C <= 512) {  // several rows per warp in registers, vector loads, lane-parallel Newton
+        constexpr int ROWS = sizeof(TIn) == 2 ? 8 : 4;
         dim3 g4((unsigned)((p.rows + 8 * ROWS - 1) / (8 * ROWS)));
         if (p.C <= 128) layernorm_multi<TIn, TOut, 1, ROWS><<<g4, 256, 0, s>>>(p);
         else if (p.C <= 256) layernorm_multi<TIn, TOut, 2, ROWS><<<g4, 256, 0, s>>>(p);

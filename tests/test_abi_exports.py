@@ -41,6 +41,8 @@ def test_binding_signatures_cover_the_header(built_lib):
     import paper_2607_24981_gb300 as ilw
 
     assert set(ilw.SIGNATURES) == set(declared_symbols())
+    hdr = open(os.path.join(ROOT, "include", "ilwdetr.h")).read()
+    assert int(re.search(r"#define ILW_I8_IN_F16 (\d+)", hdr).group(1)) == ilw.I8_IN_F16
     ilw.lib()
     assert ilw.version().startswith("ilwdetr")
 
@@ -57,9 +59,15 @@ def test_host_side_validation_without_gpu(built_lib):
     rc = L.ilwdetr_sdshiftgelu(ctypes.c_void_p(16), ctypes.c_void_p(16), 4, ctypes.byref(g), None)
     assert rc == -1
     smx = ilw.ShiftmaxT(100, 16, 8, -1, 4, 31)
-    rc = L.ilwdetr_shiftmax_attn(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), 48, 1, 64, 1, 48,
+    rc = L.ilwdetr_shiftmax_attn(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), 48, 8, 1, 64, 1, 48,
                                  0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 48, None)
     assert rc == -2  # dh = 48 unsupported
+    rc = L.ilwdetr_shiftmax_attn(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), 64, 16, 1, 64, 1, 64,
+                                 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 64, None)
+    assert rc == -1 and b"qkv_form" in L.ilwdetr_last_error()  # neither int8 nor ILW_I8_IN_F16
+    rc = L.ilwdetr_shiftmax_attn(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), 68, ilw.I8_IN_F16, 1,
+                                 64, 1, 64, 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 64, None)
+    assert rc == -1  # fp16 rows of 68 elements are not 16-byte aligned
     rc = L.ilwdetr_gemm_requant(ctypes.c_void_p(16), 24, ctypes.c_void_p(256), None, None, None, 4, 4, 24, 8,
                                 ctypes.c_void_p(16), 4, None, None)
     assert rc == -2  # K % 16 != 0

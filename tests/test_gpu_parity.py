@@ -44,13 +44,17 @@ def assert_same(got, want, what=""):
 # ------------------------------------------------------------------------------ GEMM
 @pytest.mark.parametrize("M,N,K", [(1, 1, 16), (37, 29, 64), (130, 200, 384), (257, 129, 80),
                                    (300, 1152, 384), (128, 384, 1536)])
-@pytest.mark.parametrize("out_bits,mode", [(8, "calibrated"), (8, "literal"), (16, "calibrated"), (32, "literal")])
+@pytest.mark.parametrize("out_bits,mode", [(8, "calibrated"), (8, "literal"), (16, "calibrated"), (32, "literal"),
+                                           (108, "calibrated")])
 def test_gemm_requant(ilw, orc, M, N, K, out_bits, mode):
+    """out_bits 108 (ILW_I8_IN_F16): the out_bits 8 result carried as float16."""
     A = synth.uniform_int(1, f"A{M}{K}", (M, K), -127, 127, np.int8)
     W, b, m, s = synth.gemm_params(1, f"W{N}{K}", N, K, 73.0, 40.0, mode)
     Wp = ilw.pack_weight(dev(W))
     got = ilw.gemm_requant(dev(A), Wp, N, dev(b), dev(m), dev(s), out_bits)
-    want = orc.gemm_requant(A, W, b, m, s, out_bits)
+    want = orc.gemm_requant(A, W, b, m, s, 8 if out_bits == ilw.I8_IN_F16 else out_bits)
+    if out_bits == ilw.I8_IN_F16:
+        assert got.dtype == torch.float16
     assert_same(host(got), want, "gemm")
 
 
@@ -162,14 +166,17 @@ def test_int_layernorm(ilw, orc, C, in_bits, out_bits, iters):
 @pytest.mark.parametrize("B,T,H,dh,win", [(1, 17, 1, 64, 0), (2, 64, 2, 64, 0), (1, 256, 3, 64, 0),
                                           (1, 300, 2, 32, 0), (2, 100, 2, 64, 2), (1, 1600, 1, 64, 2),
                                           (1, 144, 2, 32, 3), (1, 400, 1, 64, 0)])
-def test_attention(ilw, orc, B, T, H, dh, win):
+@pytest.mark.parametrize("form", ["int8", "f16"])
+def test_attention(ilw, orc, B, T, H, dh, win, form):
+    """form f16: q|k|v handed over as float16 holding the int8 values (ILW_I8_IN_F16)."""
     d = H * dh
     qkv = synth.uniform_int(8, f"qkv{T}{dh}", (B * T, 3 * d), -127, 127, np.int8)
+    q_dev = dev(qkv) if form == "int8" else dev(qkv.astype(np.float16))
     for I0, sd in ((1 << 13, -1), (1 << 12, -1), (20000, 3)):
         smx = {"I0": I0, "k_inter": 16, "k_out": 8, "s_d": sd, "m_p": 4, "M_hw": 31}
-        got = ilw.shiftmax_attn(dev(qkv), B, T, H, dh, win, smx, 3 << 29, 36)
+        got = ilw.shiftmax_attn(q_dev, B, T, H, dh, win, smx, 3 << 29, 36)
         want = orc.attention(qkv, B, T, H, dh, win, smx, 3 << 29, 36)
-        assert_same(host(got), want, f"attn T={T} win={win} I0={I0}")
+        assert_same(host(got), want, f"attn T={T} win={win} I0={I0} {form}")
 
 
 def test_attention_extreme_scores(ilw, orc):

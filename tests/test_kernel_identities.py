@@ -81,3 +81,41 @@ def test_single_multiply_quotient_fails_past_the_bound():
     n = np.uint64(359999)
     m32 = np.uint64(((1 << 32) + I0 - 1) // I0)
     assert int((n * m32) >> np.uint64(32)) == 12 and int(n) // I0 == 11
+
+
+def _newton_fixed(V, iters):
+    r = 1 << 16
+    for _ in range(iters):
+        if r == 0:
+            break
+        r = (r + V // r) >> 1
+    return max(r, 1)
+
+
+def _newton_early(V, iters):
+    """The I-LayerNorm kernels' schedule: stop at a fixed point, or resolve a 2-cycle by parity."""
+    r, prev = 1 << 16, None
+    for it in range(iters):
+        if r == 0:
+            break
+        nx = (r + V // r) >> 1
+        if nx == r:
+            break
+        if nx == prev:
+            r = r if (iters - it - 1) & 1 else nx
+            break
+        prev, r = r, nx
+    return max(r, 1)
+
+
+def test_newton_early_exit_matches_fixed_iteration_count():
+    """Cutting Newton's integer square root short (fixed point, or the s <-> s+1 alternation at
+    V = s^2 + 2s) gives exactly the value of the full `iters` steps, for every iteration count."""
+    rng = np.random.default_rng(5)
+    Vs = [0, 1, 2, 3, 8, 15, 24, 35, (1 << 32) - 1, 1 << 32, (1 << 40) - 1]
+    Vs += [s * s + 2 * s for s in (1, 2, 3, 255, 256, 65535, 65536, 70000, 1 << 19)]
+    Vs += [int(v) for v in rng.integers(0, 1 << 40, size=3000)]
+    Vs += [int(v) for v in rng.integers(0, 1 << 20, size=2000)]
+    for V in Vs:
+        for iters in range(0, 21):
+            assert _newton_early(V, iters) == _newton_fixed(V, iters), (V, iters)
