@@ -223,35 +223,52 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
         }
         cp_async_commit();
     };
-    // one pass over the key blocks: body(kb, buf, full) with the block staged in buffer buf
-    auto sweep = [&](bool with_v, auto &&body) {
-        if constexpr (QF16) {
-            issue16(0, 0, with_v);
-            cp_async_wait_all();
+    // A warp whose 16 query rows all lie past the group (the short last tile of a window) only
+    // helps stage the key blocks.
+    const bool rows_live = q0 + warp * 16 < Tg;
+    // One pass over the key blocks: body(kb, buf, full) with block kb staged in buffer buf.  While
+    // the last block of a pass is computed, the first block of the next pass (with or without V:
+    // next_v) is staged, so only the very first block of the CTA is waited for unhidden.
+    bool prestaged = false;
+    int pre_buf = 0;
+    auto sweep = [&](bool with_v, bool has_next, bool next_v, auto &&body) {
+        int b0 = 0;
+        if (prestaged) {
+            b0 = pre_buf;
         } else {
-            fetch(0, with_v);
-            commit(0, with_v);
-        }
-        __syncthreads();
-        for (int kb = 0; kb < nkb; ++kb) {
-            const int buf = kb & 1;
-            // buffer buf^1 was released by the barrier that ended the previous block
             if constexpr (QF16) {
-                if (kb + 1 < nkb) issue16(kb + 1, buf ^ 1, with_v);
-                body(kb, buf, (kb + 1) * KB <= Tg);
-                if (kb + 1 < nkb) cp_async_wait_all();
+                issue16(0, 0, with_v);
+                cp_async_wait_all();
             } else {
-                if (kb + 1 < nkb) fetch(kb + 1, with_v);
-                body(kb, buf, (kb + 1) * KB <= Tg);
-                if (kb + 1 < nkb) commit(buf ^ 1, with_v);
+                fetch(0, with_v);
+                commit(0, with_v);
             }
             __syncthreads();
         }
+        for (int kb = 0; kb < nkb; ++kb) {
+            const int buf = (b0 + kb) & 1;
+            const bool more = kb + 1 < nkb, stage = more || has_next;
+            const int nkb_ = more ? kb + 1 : 0;
+            const bool nv = more ? with_v : next_v;
+            // buffer buf^1 was released by the barrier that ended the previous block
+            if constexpr (QF16) {
+                if (stage) issue16(nkb_, buf ^ 1, nv);
+                if (rows_live) body(kb, buf, (kb + 1) * KB <= Tg);
+                if (stage) cp_async_wait_all();
+            } else {
+                if (stage) fetch(nkb_, nv);
+                if (rows_live) body(kb, buf, (kb + 1) * KB <= Tg);
+                if (stage) commit(buf ^ 1, nv);
+            }
+            __syncthreads();
+        }
+        prestaged = has_next;
+        pre_buf = (b0 + nkb) & 1;
     };
 
     // ---- pass 1: exact row maxima
     float mx0 = -3.0e38f, mx1 = -3.0e38f;
-    sweep(false, [&](int kb, int buf, bool full) {
+    sweep(false, true, false, [&](int kb, int buf, bool full) {
         float S[8][4];
         scores(buf, S);
         if (full) {
@@ -280,7 +297,7 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
 
     // ---- pass 2: S_sum = sum ShiftExp(s - max)
     uint64_t sum0 = 0, sum1 = 0;
-    sweep(false, [&](int kb, int buf, bool full) {
+    sweep(false, true, true, [&](int kb, int buf, bool full) {
         float S[8][4];
         scores(buf, S);
         if (full) {
@@ -311,7 +328,7 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     float o[NT][4];
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
-    sweep(true, [&](int kb, int buf, bool full) {
+    sweep(true, false, false, [&](int kb, int buf, bool full) {
         float S[8][4];
         scores(buf, S);
         uint32_t pa[4][4];  // A fragments of P for the 4 k16 steps (16 keys each)

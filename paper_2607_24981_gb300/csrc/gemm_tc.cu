@@ -59,6 +59,7 @@ struct TcParams {  // CUtensorMap members keep the 64-byte alignment TMA needs
     int32_t nbuf;       // TMEM accumulator sets (1 or 2)
     int32_t tmem_cols;
     int32_t gelu_T;     // SD-ShiftGELU table covers g in [-gelu_T, gelu_T] (constant beyond)
+    const uint8_t *gelu_tab;  // that table in global memory (16-byte aligned, 65536 bytes)
     int *status;
     EpiParams ep;
 };
@@ -183,17 +184,19 @@ __device__ __forceinline__ void lds16(const int32_t *p, int32_t (&o)[16]) {
                      : "r"(a + 16 * j));
 }
 
-// rq(v; m, s) for int32 v and s >= 33: with v*m = hi 2^32 + lo, lo / 2^32 < 1 added to an integer
-// numerator never changes floor(. / 2^(s-32)), so rq = (hi + 2^(s-33)) >> (s-32) exactly.
-__device__ __forceinline__ int32_t rq_hi(int32_t v, int32_t m, int32_t s) {
-    return (__mulhi(v, m) + (1 << (s - 33))) >> (s - 32);
+// rq(v; m, s) for int32 v and s >= 33, given sh1 = s - 33.  With v m = H 2^32 + L (0 <= L < 2^32),
+// L / 2^32 < 1 added to an integer numerator never changes floor(. / 2^(s-32)), so
+// rq = floor((H + 2^(s-33)) / 2^(s-32)); and floor((h + 2^(k-1)) / 2^k) = (floor(h / 2^(k-1)) + 1) >> 1
+// for k >= 1, which needs no rounding constant.
+__device__ __forceinline__ int32_t rq_hi1(int32_t v, int32_t m, int32_t sh1) {
+    return ((__mulhi(v, m) >> sh1) + 1) >> 1;
 }
 
 // The fused epilogue of 16 consecutive columns of one row, computed stage by stage so that the
-// 16 independent elements overlap.  The fast path (every shift >= 33, the usual case) is decided
-// per chunk, which is uniform across the warp.
+// 16 independent elements overlap.  fastw (uniform across the warp, decided per tile) says every
+// shift of the warp's columns is >= 33; ss then holds s - 33, else s.
 template <int KIND>
-__device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool has_res, const uint32_t (&rp)[8],
+__device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool fastw, bool has_res, const uint32_t (&rp)[8],
                                           const int32_t (&acc)[16], const int32_t (&sb)[16],
                                           const int32_t (&sm)[16], const int32_t (&ss)[16],
                                           const uint8_t *gtab, int32_t gT, int32_t (&out)[16]) {
@@ -202,13 +205,10 @@ __device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool has_res, con
         for (int i = 0; i < 16; ++i) out[i] = acc[i] + sb[i];
         return;
     }
-    bool fast = true;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) fast &= ss[i] >= 33;
     int32_t r[16];
-    if (fast) {
+    if (fastw) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) r[i] = rq_hi(acc[i] + sb[i], sm[i], ss[i]);  // |r| < 2^29
+        for (int i = 0; i < 16; ++i) r[i] = rq_hi1(acc[i] + sb[i], sm[i], ss[i]);  // |r| < 2^29
     } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -222,17 +222,17 @@ __device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool has_res, con
         for (int i = 0; i < 16; ++i) {
             const int32_t g = sat16(r[i]);
             const int32_t gi = g * (int32_t)gtab[min(max(g, -gT), gT) + gT];  // g * I_div(g), |.| < 2^22
-            out[i] = sat8(gfast ? rq_hi(gi, ep.m_g, ep.s_g) : rq((int64_t)gi, ep.m_g, ep.s_g));
+            out[i] = sat8(gfast ? rq_hi1(gi, ep.m_g, ep.s_g - 33) : rq((int64_t)gi, ep.m_g, ep.s_g));
         }
         return;
     }
     if (has_res) {
         // rp holds the 16 int16 residuals in pairs; x * 2^16 is the pair word masked or shifted
-        const bool rfast = ep.s_r >= 17;  // then rq(x; m_r, s_r) = rq_hi(x * 2^16; m_r, s_r + 16)
+        const bool rfast = ep.s_r >= 17;  // then rq(x; m_r, s_r) = rq(x * 2^16; m_r, s_r + 16), s_r + 16 >= 33
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             const int32_t xs = (i & 1) ? (int32_t)(rp[i >> 1] & 0xFFFF0000u) : (int32_t)(rp[i >> 1] << 16);
-            r[i] += rfast ? rq_hi(xs, ep.m_r, ep.s_r + 16) : (int32_t)rq((int64_t)(xs >> 16), ep.m_r, ep.s_r);
+            r[i] += rfast ? rq_hi1(xs, ep.m_r, ep.s_r - 17) : (int32_t)rq((int64_t)(xs >> 16), ep.m_r, ep.s_r);
         }
     }
 #pragma unroll
@@ -281,11 +281,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     // SD-ShiftGELU: I_div depends on the int16 value g alone and is constant once both ShiftExp
-    // inputs are clamped (|g| > gelu_T), so the epilogue warps tabulate it once per CTA with the
-    // same device function (exact by construction) and then look it up.
+    // inputs are clamped (|g| > gelu_T); the table (built once per parameter set by
+    // gelu_table_kernel with the same device function) is copied into shared memory here.
     uint8_t *gtab = (uint8_t *)((int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + 12 * BN);
     if (KIND == KIND_GELU8 && warp >= 6) {
-        for (int i = threadIdx.x - 192; i <= 2 * p.gelu_T; i += 256) gtab[i] = (uint8_t)gelu_idiv(i - p.gelu_T, p.ep.gelu);
+        const int n16 = (2 * p.gelu_T + 1 + 15) / 16;
+        for (int i = threadIdx.x - 192; i < n16; i += 256) ((uint4 *)gtab)[i] = __ldg((const uint4 *)p.gelu_tab + i);
         asm volatile("bar.sync 1, 256;" ::: "memory");  // the 8 epilogue warps only
     }
     const int acc_cols = p.nseg * BN;  // columns of one accumulator set
@@ -410,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 const bool ok = col < p.N;
                 pb[k] = (ok && ep.bias) ? __ldg(ep.bias + col) : 0;
                 pm[k] = (ok && ep.mult) ? __ldg(ep.mult + col) : 0;
-                ps[k] = (ok && ep.shift) ? __ldg(ep.shift + col) : 1;
+                ps[k] = (ok && ep.shift) ? __ldg(ep.shift + col) : 33;
             }
         };
         if (blockIdx.x < p.tiles) fetch(blockIdx.x);
@@ -421,11 +422,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint32_t use = (uint32_t)(tl / p.nbuf);
             const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN + h * HALF;
             __syncwarp();  // this warp is done with the previous tile's parameters
+            bool fast_lane = true;
+#pragma unroll
+            for (int k = 0; k < PPL; ++k) fast_lane &= ps[k] >= 33;
+            const bool fastw = __all_sync(0xffffffffu, fast_lane);  // shifts stored as s - 33 if so
 #pragma unroll
             for (int k = 0; k < PPL; ++k) {
                 s_bias[lane + 32 * k] = pb[k];
                 s_mult[lane + 32 * k] = pm[k];
-                s_shift[lane + 32 * k] = ps[k];
+                s_shift[lane + 32 * k] = fastw ? ps[k] - 33 : ps[k];
             }
             __syncwarp();
             if (t + (int)gridDim.x < p.tiles) fetch(t + gridDim.x);
@@ -488,21 +493,29 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 const int ncol = min(16, p.N - (n0 + c0));
                 if (row_ok && ncol > 0) {
                     int32_t out[16];
-                    epi_chunk<KIND>(ep, has_res, rp, acc, cb, cm, cs, gtab, p.gelu_T, out);
-                    if constexpr (KIND == KIND_F16OUT) {  // |v| <= 127: fp16 bits of 1152 + v, minus 1152
-                        const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
-#pragma unroll
-                        for (int i = 0; i < 16; i += 2) {
-                            uint32_t x = (uint32_t)(0x6480 + out[i]) | ((uint32_t)(0x6480 + out[i + 1]) << 16);
-                            __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), k1152);
-                            x = *reinterpret_cast<uint32_t *>(&h);
-                            out[i] = (int32_t)(x & 0xFFFFu);
-                            out[i + 1] = (int32_t)(x >> 16);
-                        }
-                    }
+                    epi_chunk<KIND>(ep, fastw, has_res, rp, acc, cb, cm, cs, gtab, p.gelu_T, out);
                     char *dst = (char *)ep.C + (row * ep.ldc + n0 + c0) * (bits / 8);
                     const bool vec = ncol == 16 && (((uintptr_t)dst & 15) == 0);
-                    if constexpr (bits == 8) {
+                    if constexpr (KIND == KIND_F16OUT) {
+                        // |v| <= 127: the fp16 bits of 1152 + v are 0x6480 + v; one half2 subtract of
+                        // 1152 leaves v exactly
+                        const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
+                        uint32_t hw[8];
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            uint32_t x = (uint32_t)(0x6480 + out[2 * j]) | ((uint32_t)(0x6480 + out[2 * j + 1]) << 16);
+                            __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), k1152);
+                            hw[j] = *reinterpret_cast<uint32_t *>(&h);
+                        }
+                        if (vec) {
+                            ((uint4 *)dst)[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+                            ((uint4 *)dst)[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i)
+                                if (i < ncol) ((uint16_t *)dst)[i] = (uint16_t)((i & 1) ? hw[i >> 1] >> 16 : hw[i >> 1]);
+                        }
+                    } else if constexpr (bits == 8) {
                         if (vec) {
                             uint32_t w[4];
 #pragma unroll
@@ -556,6 +569,70 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(p.tmem_cols) : "memory");
     }
+}
+
+// SD-ShiftGELU tables, one slot per parameter set: entry i is I_div(i - T) for i in [0, 2T].
+constexpr int kGeluSlots = 32;
+constexpr int kGeluTabBytes = 65536;  // 2T + 1 <= 65535 for T <= 32767, rounded up to 16 bytes
+__device__ __align__(16) uint8_t g_gelu_tab[kGeluSlots][kGeluTabBytes];
+
+__global__ void gelu_table_kernel(uint8_t *tab, int32_t T, GeluC c) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i <= 2 * T) tab[i] = (uint8_t)gelu_idiv(i - T, c);
+}
+
+// The table slot of (device, GELU constants, T), built on first use.  The first build of a slot is
+// waited for (unless the stream is being captured), so a slot marked built is complete for every
+// stream; a build recorded into a graph is repeated by each replay until an eager call builds it.
+const uint8_t *gelu_table(const GeluC &c, int32_t T, cudaStream_t s, cudaError_t *err) {
+    struct Key {
+        int dev;
+        int32_t I0, k, out_sh, T;
+        bool operator==(const Key &o) const {
+            return dev == o.dev && I0 == o.I0 && k == o.k && out_sh == o.out_sh && T == o.T;
+        }
+    };
+    static std::mutex mu;
+    static Key keys[64][kGeluSlots];
+    static bool used[64][kGeluSlots] = {}, built[64][kGeluSlots] = {};
+    static int next[64] = {};
+    static uint8_t *base[64] = {};
+    *err = cudaSuccess;
+    int dev = 0;
+    if ((*err = cudaGetDevice(&dev)) != cudaSuccess) return nullptr;
+    if (dev < 0 || dev >= 64) {
+        *err = cudaErrorInvalidDevice;
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    if (!base[dev]) {
+        void *b = nullptr;
+        if ((*err = cudaGetSymbolAddress(&b, g_gelu_tab)) != cudaSuccess) return nullptr;
+        base[dev] = (uint8_t *)b;
+    }
+    const Key key{dev, c.se.I0, c.se.k, c.out_sh, T};
+    int slot = -1;
+    for (int i = 0; i < kGeluSlots; ++i)
+        if (used[dev][i] && keys[dev][i] == key) slot = i;
+    if (slot < 0) {
+        slot = next[dev];
+        next[dev] = (next[dev] + 1) % kGeluSlots;
+        keys[dev][slot] = key;
+        used[dev][slot] = true;
+        built[dev][slot] = false;
+    }
+    uint8_t *tab = base[dev] + (size_t)slot * kGeluTabBytes;
+    if (!built[dev][slot]) {
+        gelu_table_kernel<<<(2 * T + 1 + 255) / 256, 256, 0, s>>>(tab, T, c);
+        if ((*err = cudaGetLastError()) != cudaSuccess) return nullptr;
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if ((*err = cudaStreamIsCapturing(s, &cs)) != cudaSuccess) return nullptr;
+        if (cs == cudaStreamCaptureStatusNone) {
+            if ((*err = cudaStreamSynchronize(s)) != cudaSuccess) return nullptr;
+            built[dev][slot] = true;
+        }
+    }
+    return tab;
 }
 
 // int8 weight -> fp16 operand copy (|w| <= 127: exact)
@@ -702,6 +779,9 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
         // is above that bound.  g is int16, so T never needs to exceed 32767.
         const double bound = 0.7 * ((double)ep.gelu.se.kI0 + 1.0) + 8.0;
         tp.gelu_T = bound > 32767.0 ? 32767 : (int32_t)bound;
+        cudaError_t e = cudaSuccess;
+        tp.gelu_tab = gelu_table(ep.gelu, tp.gelu_T, s, &e);
+        if (!tp.gelu_tab) return e != cudaSuccess ? e : cudaErrorUnknown;
     }
     if constexpr (NB == 1) {
         if (ep.kind == EPI_GELU) return launch_tc<BN, STAGES, KIND_GELU8, NB>(tp, s);
