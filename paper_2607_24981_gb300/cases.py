@@ -5,7 +5,8 @@
 Each case builds its seeded inputs (shapes of the paper's Medium model and of the nonlinearity
 sweep), runs the entry point `reps` times after 3 warm-up calls and prints the mean device time
 with the case's algorithmic work.  Cases:
-  attn_global   attention, 2 images x 1600 tokens, 6 heads, dh 64, global (fp16-carried q|k|v)
+  attn_global   attention, 2 images x 1600 tokens, 6 heads, dh 64, global (fp16-carried q|k|v);
+                --batch 8 gives the encoder's launch
   attn_window   attention, 8 images x 1600 tokens, 6 heads, 2x2 windows of 400
   gemm_qkv / gemm_proj / gemm_fc1_gelu / gemm_fc2
                 the block GEMMs at 12800 tokens, d 384, MLP 1536
@@ -32,8 +33,9 @@ def _dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-def build(case: str):
-    """Returns (fn, work dict) for a case; fn() launches the entry point once."""
+def build(case: str, batch: int = 0):
+    """Returns (fn, work dict) for a case; fn() launches the entry point once.  ``batch`` > 0
+    overrides the number of images of the attention cases."""
     import torch
 
     import paper_2607_24981_gb300 as ilw
@@ -41,6 +43,7 @@ def build(case: str):
     ilw.lib()
     if case.startswith("attn"):
         B, T, H, dh = (2, 1600, 6, 64) if case == "attn_global" else (8, 1600, 6, 64)
+        B = batch or B
         win = 0 if case == "attn_global" else 2
         # q|k|v as the QKV GEMM hands them over: the int8 values carried in float16
         qkv = _dev(synth.uniform_int(0, "case.qkv", (B * T, 3 * H * dh), -127, 127, np.int8).astype(np.float16))
@@ -96,8 +99,9 @@ def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("case")
     ap.add_argument("--reps", type=int, default=10)
+    ap.add_argument("--batch", type=int, default=0, help="images of the attention cases")
     a = ap.parse_args(argv)
-    fn, work = build(a.case)
+    fn, work = build(a.case, a.batch)
     for _ in range(3):
         fn()
     torch.cuda.synchronize()
