@@ -251,6 +251,86 @@ size_t ilwdetr_block_workspace_bytes(int32_t B, int32_t T, int32_t d, int32_t F)
 int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t *y, int32_t B,
                           int32_t T, void *workspace, size_t workspace_bytes, ilw_stream_t stream);
 
+/* ------------------------------------------------------------------ detector: projector, decoder */
+
+/* Per-tensor requantisation with an optional second term (the QuantAct between the int16 residual
+ * stream and the int8 input of an integer linear layer, Sec. 3.2.1; with Z, two tensors brought to
+ * one activation scale, as for a decoder query plus its positional query):
+ *   Y[r, c] = sat_{out_bits}( rq(X[r, c]; m1, s1) + rq(Z[r mod z_rows, c]; m2, s2) )
+ *   X  int16 (in_bits 16) or int32 (in_bits 32) [rows, ldx];  Z int16 [z_rows, ldz] or NULL
+ *   Y  int8 / int16 (symmetric saturation) or int32 (out_bits 32: the sum must fit int32, no
+ *      saturation) [rows, ldy].  C, ldx, ldz, ldy must be multiples of 4 and each base pointer
+ *      aligned to 4 elements.
+ * Shifts in [1, 62]; |X m1| and |Z m2| must stay below 2^62 (always so for int16 inputs);
+ * errors as for the other entry points. */
+int ilwdetr_requant(const void *X, int32_t in_bits, int64_t ldx, int64_t rows, int32_t C, int32_t m1,
+                    int32_t s1, const int16_t *Z, int64_t ldz, int64_t z_rows, int32_t m2, int32_t s2,
+                    int32_t out_bits, void *Y, int64_t ldy, ilw_stream_t stream);
+
+/* Nearest-neighbour resampling of B int8 feature maps (the projector's strides 8 / 16 / 32 read as
+ * nearest resampling of the stride-16 encoder grid; a 1x1 convolution commutes with it):
+ *   Y[b][y*Wo + x, :] = X[b][floor(y*Hi/Ho)*Wi + floor(x*Wi/Wo), :]
+ *   X int8, map b starts at row b*x_bstride of C channels; Y likewise with y_bstride (so the
+ *   levels can be written into one concatenated decoder memory).  C % 16 == 0, 16-byte aligned. */
+int ilwdetr_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int32_t Hi, int32_t Wi,
+                             int32_t C, int8_t *Y, int64_t y_bstride, int32_t Ho, int32_t Wo,
+                             ilw_stream_t stream);
+
+/* One integer decoder layer (post-norm, the Deformable-DETR order; the paper's decoder with
+ * nearest-neighbour deformable sampling, Sec. 3.1.1, and I-LayerNorm with 20 Newton steps,
+ * Sec. 3.3).  All weights are packed (ilwdetr_pack_weight) int8 [out, in]:
+ *   self-attention   qk_in = sat8(rq(tgt; m_q1,s_q1) + rq(pos; m_q2,s_q2)), v_in = sat8(rq(tgt; m_v1,s_v1));
+ *                    q|k = rq8(qk_in W_qk^T) [2d], v = rq8(v_in W_v^T) [d]; global attention over
+ *                    the Q queries (dh = d / H); x1 = sat16(rq(O W_o^T) + rq(tgt; m_r1,s_r1));
+ *                    t1 = LN1(x1) (int16)
+ *   cross-attention  qc = sat8(rq(t1; m_c1,s_c1) + rq(pos; m_c2,s_c2)); value = rq8(memory W_val^T);
+ *                    Q8 offsets = rq16(qc W_off^T) [H*L*P*2]; logits = rq16(qc W_att^T) [H*L*P];
+ *                    weights = Constrained Shiftmax (smx_w) over each head's L*P logits;
+ *                    s = ilwdetr_deform_attn(value, ..., m_s, s_s);
+ *                    x2 = sat16(rq(s W_o2^T) + rq(t1; m_r2,s_r2)); t2 = LN2(x2)
+ *   FFN              f = sat8(rq(t2; m_f,s_f)); h = GELU8(f W_fc1^T) [F];
+ *                    x3 = sat16(rq(h W_fc2^T) + rq(t2; m_r3,s_r3)); out = LN3(x3) (int16) */
+typedef struct ilw_decoder_params_t {
+    uint32_t struct_size; /* sizeof(ilw_decoder_params_t) */
+    int32_t d, H, F, L, P, ln_iters;
+    int32_t m_q1, s_q1, m_q2, s_q2, m_v1, s_v1;
+    const void *w_qk; const int32_t *b_qk, *m_qk, *s_qk;
+    const void *w_v; const int32_t *b_v, *m_v, *s_v;
+    ilw_shiftmax_t smx;
+    int32_t m_o, s_o;
+    const void *w_o; const int32_t *b_o, *m_oc, *s_oc;
+    int32_t m_r1, s_r1;
+    const int32_t *ln1_beta, *ln1_mult, *ln1_shift;
+    int32_t m_c1, s_c1, m_c2, s_c2;
+    const void *w_val; const int32_t *b_val, *m_val, *s_val;
+    const void *w_off; const int32_t *b_off, *m_off, *s_off;
+    const void *w_att; const int32_t *b_att, *m_att, *s_att;
+    ilw_shiftmax_t smx_w;
+    int32_t m_s, s_s;
+    const void *w_o2; const int32_t *b_o2, *m_o2, *s_o2;
+    int32_t m_r2, s_r2;
+    const int32_t *ln2_beta, *ln2_mult, *ln2_shift;
+    int32_t m_f, s_f;
+    const void *w_fc1; const int32_t *b_fc1, *m_fc1, *s_fc1;
+    ilw_gelu_t gelu;
+    int32_t m_g, s_g;
+    const void *w_fc2; const int32_t *b_fc2, *m_fc2, *s_fc2;
+    int32_t m_r3, s_r3;
+    const int32_t *ln3_beta, *ln3_mult, *ln3_shift;
+} ilw_decoder_params_t;
+
+/* Workspace bytes of ilwdetr_decoder_layer_forward for B*Q queries over B*S_total memory rows. */
+size_t ilwdetr_decoder_workspace_bytes(int32_t B, int32_t Q, int64_t S_total, int32_t d, int32_t F,
+                                       int32_t H, int32_t L, int32_t P);
+/* tgt, pos int16 [B*Q, d]; memory int8 [B*S_total, d] (levels concatenated per image, as
+ * ilwdetr_deform_attn reads them); level_hw HOST int32 [L, 2]; ref_q16 int32 [B, Q, 2];
+ * out int16 [B*Q, d] (may not alias tgt).  d % 16 == 0, d / H in {32, 64}, F % 16 == 0.
+ * workspace: >= ilwdetr_decoder_workspace_bytes, 256-byte aligned. */
+int ilwdetr_decoder_layer_forward(const ilw_decoder_params_t *p, const int16_t *tgt, const int16_t *pos,
+                                  const int8_t *memory, const int32_t *level_hw, int32_t L,
+                                  const int32_t *ref_q16, int32_t B, int32_t Q, int16_t *out,
+                                  void *workspace, size_t workspace_bytes, ilw_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -121,6 +121,13 @@ def lib():
         L.orc_deform_attn.argtypes = [i8p, i32p, C.c_int32, i32p, i32p, u8p, C.c_int32,
                                       C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int64,
                                       C.c_int32, C.c_int32, i8p]
+        L.orc_requant.restype = C.c_int
+        L.orc_requant.argtypes = [i32p, C.c_int64, C.c_int64, C.c_int64, C.c_int32, C.c_int32,
+                                  i32p, C.c_int64, C.c_int64, C.c_int32, C.c_int32, C.c_int32,
+                                  i32p, C.c_int64]
+        L.orc_resample_nearest.restype = C.c_int
+        L.orc_resample_nearest.argtypes = [i8p, C.c_int64, C.c_int32, C.c_int32, C.c_int32,
+                                           C.c_int32, i8p, C.c_int64, C.c_int32, C.c_int32]
         _lib = L
     return _lib
 
@@ -355,3 +362,94 @@ def deform_attn(value: np.ndarray, level_hw, ref_q16: np.ndarray, off_q8: np.nda
                                  _p(off_q8, i32p), _p(w, u8p), B, Q, H, P, dh, S, m, s,
                                  _p(out, i8p)), "deform_attn")
     return out
+
+
+# ---------------------------------------------------------------- detector: projector, decoder
+_OUT_DT = {8: np.int8, 16: np.int16, 32: np.int32}
+
+
+def requant(X: np.ndarray, m1: int, s1: int, Z: np.ndarray | None = None, m2: int = 0, s2: int = 1,
+            out_bits: int = 8) -> np.ndarray:
+    """sat_{out_bits}(rq(X; m1, s1) + rq(Z[r mod z_rows]; m2, s2)) elementwise over a 2-D X."""
+    X32 = np.ascontiguousarray(X, dtype=np.int32)
+    rows, Cn = X32.shape
+    Y = np.empty((rows, Cn), dtype=np.int32)
+    if Z is not None:
+        Z32 = np.ascontiguousarray(Z, dtype=np.int32)
+        zp, zr, zl = _p(Z32, i32p), Z32.shape[0], Z32.shape[1]
+    else:
+        zp, zr, zl = None, 1, Cn
+    _check(lib().orc_requant(_p(X32, i32p), Cn, rows, Cn, m1, s1, zp, zl, zr, m2, s2, out_bits,
+                             _p(Y, i32p), Cn), "requant")
+    return Y.astype(_OUT_DT[out_bits])
+
+
+def resample_nearest(X: np.ndarray, B: int, Hi: int, Wi: int, Ho: int, Wo: int) -> np.ndarray:
+    """B maps [Hi*Wi, C] int8 (stacked as [B*Hi*Wi, C]) -> [B*Ho*Wo, C] by nearest resampling."""
+    X = np.ascontiguousarray(X, dtype=np.int8)
+    Cn = X.shape[1]
+    Y = np.empty((B * Ho * Wo, Cn), dtype=np.int8)
+    _check(lib().orc_resample_nearest(_p(X, i8p), Hi * Wi, B, Hi, Wi, Cn, _p(Y, i8p), Ho * Wo, Ho, Wo),
+           "resample_nearest")
+    return Y
+
+
+def projector(pp: dict, taps: list, B: int, grid: int, levels) -> np.ndarray:
+    """Multi-scale projector (Sec. 3.2.2 split convolution; strides read as nearest resampling):
+    each tapped layer x_b (int16 [B*grid*grid, K]) is requantised to int8 with its own scale; per
+    level, one split convolution over the branches gives [B*grid*grid, N] int8, resampled by
+    nearest neighbour to the level's H_l x W_l (a 1x1 convolution commutes with it); the levels
+    are concatenated per image into the decoder memory [B*S, N], S = sum H_l W_l."""
+    t = [requant(x, m, s_, out_bits=8) for x, (m, s_) in zip(taps, pp["taps"])]
+    outs = []
+    for lv, (Hl, Wl) in zip(pp["levels"], levels):
+        y = split_conv(t, lv["w"], lv["m_b"], lv["s_b"], lv["b"], lv["m"], lv["s"])
+        outs.append(resample_nearest(y, B, grid, grid, Hl, Wl).reshape(B, Hl * Wl, -1))
+    return np.concatenate(outs, axis=1).reshape(B * sum(h * w for h, w in levels), -1)
+
+
+def decoder_layer(dp: dict, tgt: np.ndarray, pos: np.ndarray, memory: np.ndarray, level_hw,
+                  refs: np.ndarray, B: int, Q: int) -> np.ndarray:
+    """One integer decoder layer (post-norm, Deformable-DETR order), every step one of the pinned
+    operators above:
+      self-attention: q = k from sat8(rq(tgt) + rq(pos)), v from sat8(rq(tgt)); global
+        attention over the Q queries; output projection + residual tgt -> sat16; I-LayerNorm
+        (20 Newton steps, int16 out);
+      deformable cross-attention: query sat8(rq(t1) + rq(pos)); value = rq8(memory W_val);
+        Q8 offsets and logits = rq16 of two linear layers of the query; weights = Constrained
+        Shiftmax over the L*P logits of each head; nearest-neighbour sampling; output
+        projection + residual t1; I-LayerNorm;
+      FFN: sat8(rq(t2)) -> FC1 + SD-ShiftGELU -> FC2 + residual t2; I-LayerNorm."""
+    d, H, F, L, P = dp["d"], dp["H"], dp["F"], dp["L"], dp["P"]
+    dh = d // H
+    M = B * Q
+    lhw = np.asarray(level_hw, dtype=np.int32).reshape(-1, 2)
+    it = dp["ln_iters"]
+    # self-attention
+    qk_in = requant(tgt, dp["m_q1"], dp["s_q1"], pos, dp["m_q2"], dp["s_q2"], 8)
+    v_in = requant(tgt, dp["m_v1"], dp["s_v1"], out_bits=8)
+    qk = gemm_requant(qk_in, dp["w_qk"], dp["b_qk"], dp["m_qk"], dp["s_qk"], 8).astype(np.int8)
+    v = gemm_requant(v_in, dp["w_v"], dp["b_v"], dp["m_v"], dp["s_v"], 8).astype(np.int8)
+    o = attention(np.concatenate([qk, v], axis=1), B, Q, H, dh, 0, dp["smx"], dp["m_o"], dp["s_o"])
+    x1 = gemm_requant(o, dp["w_o"], dp["b_o"], dp["m_oc"], dp["s_oc"], 16, tgt, dp["m_r1"], dp["s_r1"])
+    t1 = int_layernorm(x1, dp["ln1_beta"], dp["ln1_mult"], dp["ln1_shift"], it, 16).astype(np.int16)
+    # deformable cross-attention
+    qc = requant(t1, dp["m_c1"], dp["s_c1"], pos, dp["m_c2"], dp["s_c2"], 8)
+    value = gemm_requant(memory, dp["w_val"], dp["b_val"], dp["m_val"], dp["s_val"], 8).astype(np.int8)
+    off = gemm_requant(qc, dp["w_off"], dp["b_off"], dp["m_off"], dp["s_off"], 16)
+    att = gemm_requant(qc, dp["w_att"], dp["b_att"], dp["m_att"], dp["s_att"], 16)
+    sw = dp["smx_w"]
+    w, *_ = shiftmax_rows(att.reshape(M * H, L * P), sw["I0"], sw["k_inter"], sw["k_out"], sw["s_d"],
+                          sw["m_p"], sw["M_hw"])
+    S = memory.shape[0] // B
+    samp = deform_attn(value.reshape(B, S, d), lhw, refs, off.reshape(B, Q, H, L, P, 2),
+                       w.reshape(B, Q, H, L * P), dp["m_s"], dp["s_s"]).reshape(M, d)
+    x2 = gemm_requant(samp, dp["w_o2"], dp["b_o2"], dp["m_o2"], dp["s_o2"], 16, t1, dp["m_r2"], dp["s_r2"])
+    t2 = int_layernorm(x2, dp["ln2_beta"], dp["ln2_mult"], dp["ln2_shift"], it, 16).astype(np.int16)
+    # FFN
+    fin = requant(t2, dp["m_f"], dp["s_f"], out_bits=8)
+    g = gemm_requant(fin, dp["w_fc1"], dp["b_fc1"], dp["m_fc1"], dp["s_fc1"], 16)
+    gi = sdshiftgelu(g, dp["gelu_I0"], dp["gelu_k_inter"], dp["gelu_k_out"])  # g * I_div(g), int32
+    h = requant(gi, dp["m_g"], dp["s_g"], out_bits=8)
+    x3 = gemm_requant(h, dp["w_fc2"], dp["b_fc2"], dp["m_fc2"], dp["s_fc2"], 16, t2, dp["m_r3"], dp["s_r3"])
+    return int_layernorm(x3, dp["ln3_beta"], dp["ln3_mult"], dp["ln3_shift"], it, 16).astype(np.int16)

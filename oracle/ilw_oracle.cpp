@@ -472,4 +472,47 @@ int orc_deform_attn(const int8_t *value, const int32_t *level_hw, int32_t L,
     return 0;
 }
 
+// Per-tensor requantisation of an activation (the QuantAct that brings the int16 residual
+// stream to the int8 input of the next integer linear layer, Sec. 3.2.1), with an optional
+// second requantised term added before saturation (two tensors brought to one activation
+// scale, as for the decoder's query plus positional query):
+//   Y[r, c] = sat_{out_bits}( rq(X[r, c]; m1, s1) + rq(Z[r mod z_rows, c]; m2, s2) ),  Z may be NULL.
+// out_bits 8 / 16 saturate symmetrically; out_bits 32 requires the sum to fit int32.
+int orc_requant(const int32_t *X, int64_t ldx, int64_t rows, int64_t C, int32_t m1, int32_t s1,
+                const int32_t *Z, int64_t ldz, int64_t z_rows, int32_t m2, int32_t s2,
+                int32_t out_bits, int32_t *Y, int64_t ldy) {
+    if (out_bits != 8 && out_bits != 16 && out_bits != 32) return -1;
+    if (Z && z_rows < 1) return -1;
+    for (int64_t r = 0; r < rows; ++r) {
+        for (int64_t c = 0; c < C; ++c) {
+            int64_t v = orc_rq(X[r * ldx + c], m1, s1);
+            if (Z) v += orc_rq(Z[(r % z_rows) * ldz + c], m2, s2);
+            if (out_bits == 32) {
+                if (v < INT32_MIN || v > INT32_MAX) return -2;
+                Y[r * ldy + c] = (int32_t)v;
+            } else {
+                Y[r * ldy + c] = (int32_t)orc_sat(v, out_bits);
+            }
+        }
+    }
+    return 0;
+}
+
+// Nearest-neighbour resampling of B feature maps (reading of the multi-scale projector's
+// strides): map b of X is [Hi, Wi] pixels of C int8 channels, pixel (y, x) at row y*Wi + x of
+// X + b*x_bstride rows; Y[b][y*Wo + x] = X[b][floor(y*Hi/Ho)*Wi + floor(x*Wi/Wo)].
+int orc_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int32_t Hi, int32_t Wi,
+                         int32_t C, int8_t *Y, int64_t y_bstride, int32_t Ho, int32_t Wo) {
+    if (B < 0 || Hi < 1 || Wi < 1 || Ho < 1 || Wo < 1 || C < 1) return -1;
+    for (int32_t b = 0; b < B; ++b)
+        for (int32_t y = 0; y < Ho; ++y)
+            for (int32_t x = 0; x < Wo; ++x) {
+                const int64_t sy = (int64_t)y * Hi / Ho, sx = (int64_t)x * Wi / Wo;
+                const int8_t *src = X + ((int64_t)b * x_bstride + sy * Wi + sx) * C;
+                int8_t *dst = Y + ((int64_t)b * y_bstride + (int64_t)y * Wo + x) * C;
+                for (int32_t c = 0; c < C; ++c) dst[c] = src[c];
+            }
+    return 0;
+}
+
 }  // extern "C"

@@ -138,6 +138,18 @@ int orc_deform_attn(const int8_t *value, const int32_t *level_hw /* [L,2] (H_l, 
                     int32_t B, int32_t Q, int32_t H, int32_t P, int32_t dh, int64_t S_total,
                     int32_t m, int32_t s, int8_t *out /* [B,Q,H*dh] */);
 
+/* Per-tensor requantisation with an optional second term:
+ *   Y[r,c] = sat_{out_bits}( rq(X[r,c]; m1, s1) + rq(Z[r mod z_rows, c]; m2, s2) ), Z may be NULL;
+ * out_bits 8 / 16 saturate, 32 must fit int32. */
+int orc_requant(const int32_t *X, int64_t ldx, int64_t rows, int64_t C, int32_t m1, int32_t s1,
+                const int32_t *Z, int64_t ldz, int64_t z_rows, int32_t m2, int32_t s2,
+                int32_t out_bits, int32_t *Y, int64_t ldy);
+
+/* Nearest-neighbour resampling of B maps [Hi, Wi, C] to [Ho, Wo, C] (batch strides in rows):
+ * Y[b][y*Wo + x] = X[b][floor(y*Hi/Ho)*Wi + floor(x*Wi/Wo)]. */
+int orc_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int32_t Hi, int32_t Wi,
+                         int32_t C, int8_t *Y, int64_t y_bstride, int32_t Ho, int32_t Wo);
+
 #ifdef __cplusplus
 }
 #endif

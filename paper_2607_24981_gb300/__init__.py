@@ -15,6 +15,8 @@ __all__ = [
     "shiftmax_rows", "sdshiftgelu", "int_layernorm", "shiftmax_attn", "deform_attn",
     "BlockWeights", "block_forward", "block_workspace_bytes", "device_status",
     "patch_embed", "patch_embed_workspace_bytes", "Backbone", "Graphed",
+    "requant", "resample_nearest", "DecoderWeights", "decoder_workspace_bytes", "decoder_layer_forward",
+    "Projector", "Detector",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -62,6 +64,36 @@ class BlockParamsT(C.Structure):
     ]
 
 
+class DecoderParamsT(C.Structure):
+    _fields_ = [
+        ("struct_size", C.c_uint32),
+        ("d", C.c_int32), ("H", C.c_int32), ("F", C.c_int32), ("L", C.c_int32), ("P", C.c_int32),
+        ("ln_iters", C.c_int32),
+        ("m_q1", C.c_int32), ("s_q1", C.c_int32), ("m_q2", C.c_int32), ("s_q2", C.c_int32),
+        ("m_v1", C.c_int32), ("s_v1", C.c_int32),
+        ("w_qk", C.c_void_p), ("b_qk", C.c_void_p), ("m_qk", C.c_void_p), ("s_qk", C.c_void_p),
+        ("w_v", C.c_void_p), ("b_v", C.c_void_p), ("m_v", C.c_void_p), ("s_v", C.c_void_p),
+        ("smx", ShiftmaxT), ("m_o", C.c_int32), ("s_o", C.c_int32),
+        ("w_o", C.c_void_p), ("b_o", C.c_void_p), ("m_oc", C.c_void_p), ("s_oc", C.c_void_p),
+        ("m_r1", C.c_int32), ("s_r1", C.c_int32),
+        ("ln1_beta", C.c_void_p), ("ln1_mult", C.c_void_p), ("ln1_shift", C.c_void_p),
+        ("m_c1", C.c_int32), ("s_c1", C.c_int32), ("m_c2", C.c_int32), ("s_c2", C.c_int32),
+        ("w_val", C.c_void_p), ("b_val", C.c_void_p), ("m_val", C.c_void_p), ("s_val", C.c_void_p),
+        ("w_off", C.c_void_p), ("b_off", C.c_void_p), ("m_off", C.c_void_p), ("s_off", C.c_void_p),
+        ("w_att", C.c_void_p), ("b_att", C.c_void_p), ("m_att", C.c_void_p), ("s_att", C.c_void_p),
+        ("smx_w", ShiftmaxT), ("m_s", C.c_int32), ("s_s", C.c_int32),
+        ("w_o2", C.c_void_p), ("b_o2", C.c_void_p), ("m_o2", C.c_void_p), ("s_o2", C.c_void_p),
+        ("m_r2", C.c_int32), ("s_r2", C.c_int32),
+        ("ln2_beta", C.c_void_p), ("ln2_mult", C.c_void_p), ("ln2_shift", C.c_void_p),
+        ("m_f", C.c_int32), ("s_f", C.c_int32),
+        ("w_fc1", C.c_void_p), ("b_fc1", C.c_void_p), ("m_fc1", C.c_void_p), ("s_fc1", C.c_void_p),
+        ("gelu", GeluT), ("m_g", C.c_int32), ("s_g", C.c_int32),
+        ("w_fc2", C.c_void_p), ("b_fc2", C.c_void_p), ("m_fc2", C.c_void_p), ("s_fc2", C.c_void_p),
+        ("m_r3", C.c_int32), ("s_r3", C.c_int32),
+        ("ln3_beta", C.c_void_p), ("ln3_mult", C.c_void_p), ("ln3_shift", C.c_void_p),
+    ]
+
+
 # C signatures (argtypes, restype) of every export declared in include/ilwdetr.h
 _VP, _I32, _I64 = C.c_void_p, C.c_int32, C.c_int64
 SIGNATURES = {
@@ -94,6 +126,12 @@ SIGNATURES = {
     "ilwdetr_block_workspace_bytes": ([_I32, _I32, _I32, _I32], C.c_size_t),
     "ilwdetr_block_forward": ([C.POINTER(BlockParamsT), _VP, _VP, _I32, _I32, _VP, C.c_size_t, _VP],
                               C.c_int),
+    "ilwdetr_requant": ([_VP, _I32, _I64, _I64, _I32, _I32, _I32, _VP, _I64, _I64, _I32, _I32, _I32, _VP,
+                         _I64, _VP], C.c_int),
+    "ilwdetr_resample_nearest": ([_VP, _I64, _I32, _I32, _I32, _I32, _VP, _I64, _I32, _I32, _VP], C.c_int),
+    "ilwdetr_decoder_workspace_bytes": ([_I32, _I32, _I64, _I32, _I32, _I32, _I32, _I32], C.c_size_t),
+    "ilwdetr_decoder_layer_forward": ([C.POINTER(DecoderParamsT), _VP, _VP, _VP, C.POINTER(_I32), _I32, _VP,
+                                       _I32, _I32, _VP, _VP, C.c_size_t, _VP], C.c_int),
 }
 
 
@@ -383,13 +421,16 @@ class Backbone:
                                   device=device)
         self.x = [torch.empty((M, self.d), dtype=torch.int16, device=device) for _ in range(2)]
 
-    def forward(self, img):
-        """img int8 [B, 3, H, W] (device) -> x_L int16 [B*T, d] (a buffer owned by the backbone)."""
+    def forward(self, img, taps: dict | None = None):
+        """img int8 [B, 3, H, W] (device) -> x_L int16 [B*T, d] (a buffer owned by the backbone).
+        ``taps`` maps block indices to int16 [B*T, d] buffers that receive those blocks' outputs."""
         pe = self.pe
         x = patch_embed(img, self.p, pe["w_p"], self.d, pe["b"], pe["m"], pe["s"], pe["pos"],
                         self.pe_s["m_pos"], self.pe_s["s_pos"], self.ws_pe, self.x[0])
         for i, bw in enumerate(self.blocks):
-            x = block_forward(bw, x, self.B, self.T, self.ws_blk, out=self.x[(i + 1) % 2])
+            # a tapped block writes straight into its tap buffer; the others ping-pong
+            out = taps[i] if taps and i in taps else (self.x[1] if x is self.x[0] else self.x[0])
+            x = block_forward(bw, x, self.B, self.T, self.ws_blk, out=out)
         return x
 
     def capture(self, img) -> "Graphed":
@@ -420,3 +461,159 @@ class Graphed:
     def replay(self):
         self.graph.replay()
         return self.out
+
+
+# ---------------------------------------------------------------------------- detector
+def requant(X, m1, s1, Z=None, m2=0, s2=1, out_bits=8, out=None):
+    """ilwdetr_requant: sat(rq(X; m1, s1) + rq(Z[r mod z_rows]; m2, s2)), X int16/int32 [rows, C],
+    Z int16 or None -> int8/int16/int32 [rows, C]."""
+    import torch
+
+    rows, Cn = X.shape
+    in_bits = {torch.int16: 16, torch.int32: 32}[X.dtype]
+    if out is None:
+        out = torch.empty((rows, Cn), dtype={8: torch.int8, 16: torch.int16, 32: torch.int32}[out_bits],
+                          device=X.device)
+    zp, ldz, zr = (None, 0, 1) if Z is None else (_ptr(Z), Z.stride(0), Z.shape[0])
+    _check(lib().ilwdetr_requant(_ptr(X), in_bits, X.stride(0), rows, Cn, m1, s1, zp, ldz, zr, m2, s2, out_bits,
+                                 _ptr(out), out.stride(0), _stream()), "requant")
+    return out
+
+
+def resample_nearest(X, B, Hi, Wi, Ho, Wo, out=None, x_bstride=None, y_bstride=None):
+    """ilwdetr_resample_nearest over B maps of int8 [Hi*Wi, C] rows -> [B*Ho*Wo, C] (or into `out`
+    with its own batch stride in rows)."""
+    import torch
+
+    Cn = X.shape[-1]
+    if out is None:
+        out = torch.empty((B * Ho * Wo, Cn), dtype=torch.int8, device=X.device)
+    xs = Hi * Wi if x_bstride is None else x_bstride
+    ys = Ho * Wo if y_bstride is None else y_bstride
+    _check(lib().ilwdetr_resample_nearest(_ptr(X), xs, B, Hi, Wi, Cn, _ptr(out), ys, Ho, Wo, _stream()),
+           "resample_nearest")
+    return out
+
+
+class DecoderWeights:
+    """Device copies of one decoder layer's integer parameters (``synth.decoder_params``) and its
+    ilw_decoder_params_t."""
+
+    _W = ("w_qk", "w_v", "w_o", "w_val", "w_off", "w_att", "w_o2", "w_fc1", "w_fc2")
+
+    def __init__(self, dp: dict, device="cuda"):
+        import numpy as np
+        import torch
+
+        self.dp = dp
+        T = self.t = {k: torch.from_numpy(np.ascontiguousarray(v)).to(device)
+                      for k, v in dp.items() if isinstance(v, np.ndarray)}
+        for k in self._W:
+            T[k + "_p"] = pack_weight(T[k])
+        a = lambda k: T[k].data_ptr()  # noqa: E731
+        self.params = DecoderParamsT(
+            C.sizeof(DecoderParamsT), dp["d"], dp["H"], dp["F"], dp["L"], dp["P"], dp["ln_iters"],
+            dp["m_q1"], dp["s_q1"], dp["m_q2"], dp["s_q2"], dp["m_v1"], dp["s_v1"],
+            a("w_qk_p"), a("b_qk"), a("m_qk"), a("s_qk"), a("w_v_p"), a("b_v"), a("m_v"), a("s_v"),
+            _smx(dp["smx"]), dp["m_o"], dp["s_o"],
+            a("w_o_p"), a("b_o"), a("m_oc"), a("s_oc"), dp["m_r1"], dp["s_r1"],
+            a("ln1_beta"), a("ln1_mult"), a("ln1_shift"),
+            dp["m_c1"], dp["s_c1"], dp["m_c2"], dp["s_c2"],
+            a("w_val_p"), a("b_val"), a("m_val"), a("s_val"),
+            a("w_off_p"), a("b_off"), a("m_off"), a("s_off"),
+            a("w_att_p"), a("b_att"), a("m_att"), a("s_att"),
+            _smx(dp["smx_w"]), dp["m_s"], dp["s_s"],
+            a("w_o2_p"), a("b_o2"), a("m_o2"), a("s_o2"), dp["m_r2"], dp["s_r2"],
+            a("ln2_beta"), a("ln2_mult"), a("ln2_shift"),
+            dp["m_f"], dp["s_f"],
+            a("w_fc1_p"), a("b_fc1"), a("m_fc1"), a("s_fc1"),
+            GeluT(dp["gelu_I0"], dp["gelu_k_inter"], dp["gelu_k_out"]), dp["m_g"], dp["s_g"],
+            a("w_fc2_p"), a("b_fc2"), a("m_fc2"), a("s_fc2"), dp["m_r3"], dp["s_r3"],
+            a("ln3_beta"), a("ln3_mult"), a("ln3_shift"),
+        )
+
+
+def decoder_workspace_bytes(B, Q, S_total, d, F, H, L, P) -> int:
+    return int(lib().ilwdetr_decoder_workspace_bytes(B, Q, S_total, d, F, H, L, P))
+
+
+def decoder_layer_forward(dw: DecoderWeights, tgt, pos, memory, level_hw, refs, B, Q, workspace, out=None):
+    """ilwdetr_decoder_layer_forward: tgt, pos int16 [B*Q, d], memory int8 [B*S, d], refs int32
+    [B, Q, 2] -> int16 [B*Q, d]."""
+    import torch
+
+    if out is None:
+        out = torch.empty_like(tgt)
+    L = len(level_hw)
+    lhw = (C.c_int32 * (2 * L))(*[int(v) for hw in level_hw for v in hw])
+    _check(lib().ilwdetr_decoder_layer_forward(C.byref(dw.params), _ptr(tgt), _ptr(pos), _ptr(memory), lhw, L,
+                                               _ptr(refs), B, Q, _ptr(out), _ptr(workspace),
+                                               workspace.numel() * workspace.element_size(), _stream()),
+           "decoder_layer_forward")
+    return out
+
+
+class Projector:
+    """The split-convolution projector on the device: the tapped encoder layers requantised to int8
+    (one scale each), one ilwdetr_split_conv per level on the stride-16 grid, and the levels
+    resampled by nearest neighbour into one concatenated decoder memory [B*S, N]."""
+
+    def __init__(self, pp: dict, B: int, grid: int, levels, K: int, device="cuda"):
+        import numpy as np
+        import torch
+
+        self.pp, self.B, self.grid, self.levels = pp, B, grid, [tuple(x) for x in levels]
+        self.N = pp["levels"][0]["w"][0].shape[0]
+        self.S = sum(h * w for h, w in self.levels)
+        dv = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)  # noqa: E731
+        self.lv = []
+        for lv in pp["levels"]:
+            self.lv.append({"w_p": [pack_weight(dv(w)) for w in lv["w"]], "b": dv(lv["b"]), "m": dv(lv["m"]),
+                            "s": dv(lv["s"]), "m_b": list(lv["m_b"]), "s_b": list(lv["s_b"])})
+        M = B * grid * grid
+        self.t = [torch.empty((M, K), dtype=torch.int8, device=device) for _ in pp["taps"]]
+        self.y = torch.empty((M, self.N), dtype=torch.int8, device=device)
+        self.memory = torch.empty((B * self.S, self.N), dtype=torch.int8, device=device)
+
+    def forward(self, taps):
+        for x, (m, s), t in zip(taps, self.pp["taps"], self.t):
+            requant(x, m, s, out_bits=8, out=t)
+        start = 0
+        for lv, (Hl, Wl) in zip(self.lv, self.levels):
+            split_conv(self.t, lv["w_p"], self.N, lv["m_b"], lv["s_b"], lv["b"], lv["m"], lv["s"], out=self.y)
+            resample_nearest(self.y, self.B, self.grid, self.grid, Hl, Wl, out=self.memory[start:],
+                             y_bstride=self.S)
+            start += Hl * Wl
+        return self.memory
+
+
+class Detector:
+    """The full integer detector forward: Backbone (with its output layers tapped) -> Projector ->
+    decoder layers (ilwdetr_decoder_layer_forward), all on fixed device buffers."""
+
+    def __init__(self, pe: dict, blocks: list, taps, pp: dict, dps: list, B: int, Q: int, levels, grid: int = 40,
+                 device="cuda"):
+        import torch
+
+        self.backbone = Backbone(pe, blocks, B, device=device)
+        self.taps = tuple(taps)
+        self.proj = Projector(pp, B, grid, levels, self.backbone.d, device)
+        self.dec = [DecoderWeights(dp, device) for dp in dps]
+        self.B, self.Q, self.levels = B, Q, [tuple(x) for x in levels]
+        d, dp0 = dps[0]["d"], dps[0]
+        self.d = d
+        M = B * self.backbone.T
+        self.tap_buf = [torch.empty((M, self.backbone.d), dtype=torch.int16, device=device) for _ in self.taps]
+        self.ws = torch.empty(decoder_workspace_bytes(B, Q, self.proj.S, d, dp0["F"], dp0["H"], dp0["L"], dp0["P"]),
+                              dtype=torch.uint8, device=device)
+        self.t = [torch.empty((B * Q, d), dtype=torch.int16, device=device) for _ in range(2)]
+
+    def forward(self, img, tgt, pos, refs):
+        """img int8 [B, 3, H, W]; tgt, pos int16 [B*Q, d]; refs int32 [B, Q, 2] -> int16 [B*Q, d]."""
+        self.backbone.forward(img, taps=dict(zip(self.taps, self.tap_buf)))
+        memory = self.proj.forward(self.tap_buf)
+        x = tgt
+        for i, dw in enumerate(self.dec):
+            x = decoder_layer_forward(dw, x, pos, memory, self.levels, refs, self.B, self.Q, self.ws,
+                                      out=self.t[i % 2])
+        return x

@@ -405,4 +405,154 @@ int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t
     return ilwdetr_gemm_requant(hbuf, F, p->w_fc2, p->b_fc2, p->m_fc2, p->s_fc2, M, d, F, 16, y, d, &r2, stream);
 }
 
+// ------------------------------------------------------------------ detector: projector, decoder
+
+int ilwdetr_requant(const void *X, int32_t in_bits, int64_t ldx, int64_t rows, int32_t C, int32_t m1,
+                    int32_t s1, const int16_t *Z, int64_t ldz, int64_t z_rows, int32_t m2, int32_t s2,
+                    int32_t out_bits, void *Y, int64_t ldy, ilw_stream_t stream) {
+    if (in_bits != 16 && in_bits != 32) return fail(ILW_ERR_INVALID_ARG, "requant: in_bits=%d must be 16 or 32", in_bits);
+    if (out_bits != 8 && out_bits != 16 && out_bits != 32)
+        return fail(ILW_ERR_INVALID_ARG, "requant: out_bits=%d must be 8, 16 or 32", out_bits);
+    if (rows < 0 || C < 0 || C % 4) return fail(ILW_ERR_UNSUPPORTED, "requant: C=%d must be a multiple of 4", C);
+    int rc;
+    if ((rc = check_rq_scalar(s1, "requant"))) return rc;
+    if (Z && (rc = check_rq_scalar(s2, "requant second term"))) return rc;
+    if (rows == 0 || C == 0) return ILW_OK;
+    const int64_t ib = in_bits / 8, ob = out_bits / 8;
+    if (!X || !Y || ldx < C || ldy < C || !aligned(X, 4 * ib) || !aligned(Y, 4 * ob) || ldx % 4 || ldy % 4)
+        return fail(ILW_ERR_INVALID_ARG, "requant: NULL, misaligned or short rows");
+    if (Z && (z_rows < 1 || ldz < C || !aligned(Z, 8) || ldz % 4))
+        return fail(ILW_ERR_INVALID_ARG, "requant: bad second term");
+    ilw::RequantParams p{X, in_bits, ldx, rows, C, m1, s1, Z, ldz, Z ? z_rows : 1, m2, Z ? s2 : 1, out_bits, Y, ldy};
+    return cuda_status(ilw::launch_requant(p, (cudaStream_t)stream), "requant");
+}
+
+int ilwdetr_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int32_t Hi, int32_t Wi,
+                             int32_t C, int8_t *Y, int64_t y_bstride, int32_t Ho, int32_t Wo,
+                             ilw_stream_t stream) {
+    if (B < 0 || Hi < 1 || Wi < 1 || Ho < 1 || Wo < 1 || C < 16 || C % 16)
+        return fail(ILW_ERR_UNSUPPORTED, "resample: bad sizes (C=%d must be a multiple of 16)", C);
+    if (B == 0) return ILW_OK;
+    if (!X || !Y || !aligned(X, 16) || !aligned(Y, 16) || x_bstride < (int64_t)Hi * Wi || y_bstride < (int64_t)Ho * Wo)
+        return fail(ILW_ERR_INVALID_ARG, "resample: NULL, misaligned or overlapping batch strides");
+    return cuda_status(ilw::launch_resample(X, x_bstride, B, Hi, Wi, C, Y, y_bstride, Ho, Wo, (cudaStream_t)stream),
+                       "resample_nearest");
+}
+
+namespace {
+struct DecBufs {
+    int8_t *qk_in, *v_in, *qkv, *o, *qc, *value, *samp, *fin, *h;
+    int16_t *x1, *t1, *off16, *att16, *x2, *t2, *x3;
+    int32_t *off32, *att32;
+    uint8_t *w;
+    size_t bytes;
+};
+DecBufs dec_layout(char *ws, int32_t B, int32_t Q, int64_t S_total, int32_t d, int32_t F, int32_t H, int32_t L,
+                   int32_t P) {
+    const size_t M = (size_t)B * Q, MS = (size_t)B * S_total, lp = (size_t)H * L * P;
+    DecBufs b{};
+    size_t off = 0;
+    auto take = [&](size_t n) {
+        char *p = ws ? ws + off : nullptr;
+        off += align256(n);
+        return p;
+    };
+    b.qk_in = (int8_t *)take(M * d);
+    b.v_in = (int8_t *)take(M * d);
+    b.qkv = (int8_t *)take(M * 3 * d);
+    b.o = (int8_t *)take(M * d);
+    b.x1 = (int16_t *)take(M * d * 2);
+    b.t1 = (int16_t *)take(M * d * 2);
+    b.qc = (int8_t *)take(M * d);
+    b.value = (int8_t *)take(MS * d);
+    b.off16 = (int16_t *)take(M * lp * 2 * 2);
+    b.off32 = (int32_t *)take(M * lp * 2 * 4);
+    b.att16 = (int16_t *)take(M * lp * 2);
+    b.att32 = (int32_t *)take(M * lp * 4);
+    b.w = (uint8_t *)take(M * lp);
+    b.samp = (int8_t *)take(M * d);
+    b.x2 = (int16_t *)take(M * d * 2);
+    b.t2 = (int16_t *)take(M * d * 2);
+    b.fin = (int8_t *)take(M * d);
+    b.h = (int8_t *)take(M * F);
+    b.x3 = (int16_t *)take(M * d * 2);
+    b.bytes = off;
+    return b;
+}
+}  // namespace
+
+size_t ilwdetr_decoder_workspace_bytes(int32_t B, int32_t Q, int64_t S_total, int32_t d, int32_t F,
+                                       int32_t H, int32_t L, int32_t P) {
+    if (B < 0 || Q < 0 || S_total < 0 || d < 0 || F < 0 || H < 1 || L < 1 || P < 1) return 0;
+    return dec_layout(nullptr, B, Q, S_total, d, F, H, L, P).bytes;
+}
+
+int ilwdetr_decoder_layer_forward(const ilw_decoder_params_t *p, const int16_t *tgt, const int16_t *pos,
+                                  const int8_t *memory, const int32_t *level_hw, int32_t L,
+                                  const int32_t *ref_q16, int32_t B, int32_t Q, int16_t *out,
+                                  void *workspace, size_t workspace_bytes, ilw_stream_t stream) {
+    if (!p || p->struct_size != sizeof(ilw_decoder_params_t))
+        return fail(ILW_ERR_INVALID_ARG, "decoder params NULL or struct_size mismatch");
+    const int32_t d = p->d, H = p->H, F = p->F, P = p->P;
+    if (d < 16 || d % 16 || H < 1 || d % H || (d / H != 32 && d / H != 64) || F < 16 || F % 16 || P < 1)
+        return fail(ILW_ERR_INVALID_ARG, "decoder: d=%d H=%d F=%d P=%d unsupported", d, H, F, P);
+    if (L != p->L || L < 1 || L > 8 || !level_hw) return fail(ILW_ERR_INVALID_ARG, "decoder: bad levels");
+    if (B < 0 || Q < 0) return fail(ILW_ERR_INVALID_ARG, "decoder: negative sizes");
+    if (B == 0 || Q == 0) return ILW_OK;
+    if (!tgt || !pos || !memory || !ref_q16 || !out || (const void *)out == (const void *)tgt)
+        return fail(ILW_ERR_INVALID_ARG, "decoder: NULL or aliased tensors");
+    int64_t S_total = 0;
+    for (int l = 0; l < L; ++l) S_total += (int64_t)level_hw[2 * l] * level_hw[2 * l + 1];
+    const size_t need = ilwdetr_decoder_workspace_bytes(B, Q, S_total, d, F, H, L, P);
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < need)
+        return fail(ILW_ERR_INVALID_ARG, "decoder: workspace NULL, misaligned or smaller than %zu bytes", need);
+    const DecBufs b = dec_layout((char *)workspace, B, Q, S_total, d, F, H, L, P);
+    const int32_t M = B * Q, LP = L * P, HLP = H * LP;
+    const int64_t MS = (int64_t)B * S_total;
+    int rc;
+#define ILW_TRY(x) \
+    if ((rc = (x))) return rc
+    // self-attention
+    ILW_TRY(ilwdetr_requant(tgt, 16, d, M, d, p->m_q1, p->s_q1, pos, d, M, p->m_q2, p->s_q2, 8, b.qk_in, d, stream));
+    ILW_TRY(ilwdetr_requant(tgt, 16, d, M, d, p->m_v1, p->s_v1, nullptr, 0, 1, 0, 1, 8, b.v_in, d, stream));
+    ILW_TRY(ilwdetr_gemm_requant(b.qk_in, d, p->w_qk, p->b_qk, p->m_qk, p->s_qk, M, 2 * d, d, 8, b.qkv, 3 * d, nullptr,
+                                 stream));
+    ILW_TRY(ilwdetr_gemm_requant(b.v_in, d, p->w_v, p->b_v, p->m_v, p->s_v, M, d, d, 8, b.qkv + 2 * d, 3 * d, nullptr,
+                                 stream));
+    ILW_TRY(ilwdetr_shiftmax_attn(b.qkv, b.qkv + d, b.qkv + 2 * d, 3 * d, 8, B, Q, H, d / H, 0, &p->smx, p->m_o, p->s_o,
+                                  b.o, d, stream));
+    ilw_residual_t r1{tgt, d, M, p->m_r1, p->s_r1};
+    ILW_TRY(ilwdetr_gemm_requant(b.o, d, p->w_o, p->b_o, p->m_oc, p->s_oc, M, d, d, 16, b.x1, d, &r1, stream));
+    ILW_TRY(ilwdetr_int_layernorm(b.x1, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, b.t1, 16, d,
+                                  stream));
+    // deformable cross-attention
+    ILW_TRY(ilwdetr_requant(b.t1, 16, d, M, d, p->m_c1, p->s_c1, pos, d, M, p->m_c2, p->s_c2, 8, b.qc, d, stream));
+    ILW_TRY(ilwdetr_gemm_requant(memory, d, p->w_val, p->b_val, p->m_val, p->s_val, (int32_t)MS, d, d, 8, b.value, d,
+                                 nullptr, stream));
+    ILW_TRY(ilwdetr_gemm_requant(b.qc, d, p->w_off, p->b_off, p->m_off, p->s_off, M, 2 * HLP, d, 16, b.off16, 2 * HLP,
+                                 nullptr, stream));
+    ILW_TRY(ilwdetr_gemm_requant(b.qc, d, p->w_att, p->b_att, p->m_att, p->s_att, M, HLP, d, 16, b.att16, HLP, nullptr,
+                                 stream));
+    // int16 -> int32 containers (rq with m = 2^30, s = 30 is the identity)
+    ILW_TRY(ilwdetr_requant(b.off16, 16, 2 * HLP, M, 2 * HLP, 1 << 30, 30, nullptr, 0, 1, 0, 1, 32, b.off32, 2 * HLP,
+                            stream));
+    ILW_TRY(ilwdetr_requant(b.att16, 16, HLP, M, HLP, 1 << 30, 30, nullptr, 0, 1, 0, 1, 32, b.att32, HLP, stream));
+    ILW_TRY(ilwdetr_shiftmax_rows(b.att32, LP, (int64_t)M * H, LP, &p->smx_w, b.w, LP, stream));
+    ILW_TRY(ilwdetr_deform_attn(b.value, level_hw, L, ref_q16, b.off32, b.w, B, Q, H, P, d / H, p->m_s, p->s_s, b.samp,
+                                stream));
+    ilw_residual_t r2{b.t1, d, M, p->m_r2, p->s_r2};
+    ILW_TRY(ilwdetr_gemm_requant(b.samp, d, p->w_o2, p->b_o2, p->m_o2, p->s_o2, M, d, d, 16, b.x2, d, &r2, stream));
+    ILW_TRY(ilwdetr_int_layernorm(b.x2, 16, d, M, d, p->ln2_beta, p->ln2_mult, p->ln2_shift, p->ln_iters, b.t2, 16, d,
+                                  stream));
+    // FFN
+    ILW_TRY(ilwdetr_requant(b.t2, 16, d, M, d, p->m_f, p->s_f, nullptr, 0, 1, 0, 1, 8, b.fin, d, stream));
+    ILW_TRY(ilwdetr_gemm_gelu(b.fin, d, p->w_fc1, p->b_fc1, p->m_fc1, p->s_fc1, M, F, d, &p->gelu, p->m_g, p->s_g, b.h,
+                              F, stream));
+    ilw_residual_t r3{b.t2, d, M, p->m_r3, p->s_r3};
+    ILW_TRY(ilwdetr_gemm_requant(b.h, F, p->w_fc2, p->b_fc2, p->m_fc2, p->s_fc2, M, d, F, 16, b.x3, d, &r3, stream));
+    return ilwdetr_int_layernorm(b.x3, 16, d, M, d, p->ln3_beta, p->ln3_mult, p->ln3_shift, p->ln_iters, out, 16, d,
+                                 stream);
+#undef ILW_TRY
+}
+
 }  // extern "C"

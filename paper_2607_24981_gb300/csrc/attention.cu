@@ -30,6 +30,15 @@ __device__ __forceinline__ void mma_f16(float (&c)[4], const uint32_t (&a)[4], u
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+// D = A B + C with C = {c0, c0, c1, c1} (rows g and g + 8 of the fragment): starts an accumulation
+// without a separate initialisation of D.
+__device__ __forceinline__ void mma_f16_init(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1, float c0,
+                                             float c1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%11,%11};\n"
+        : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(c0), "f"(c1));
+}
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
                  : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
@@ -72,6 +81,28 @@ __device__ __forceinline__ uint32_t u10x2_to_h2(uint32_t p0, uint32_t p1) {
     return *reinterpret_cast<uint32_t *>(&h);
 }
 
+// Logical right shift whose amount saturates at 32 (PTX shr clamps the shift amount to the
+// register width, so any amount >= 32 gives 0).
+__device__ __forceinline__ uint32_t shr_sat(uint32_t v, uint32_t n) {
+    uint32_t r;
+    asm("shr.u32 %0, %1, %2;" : "=r"(r) : "r"(v), "r"(n));
+    return r;
+}
+
+// Constrained Shiftmax output straight from ShiftExp's parts.  With e = I_b 2^(k-q) and
+// sh = 31 - k_out + 1 + s_d >= k, floor(e F / 2^sh) = floor(I_b F / 2^(sh - k + q)) exactly, and
+// I_b F < 2^32 when s_d is chosen per row and m_p <= M_hw - 15 (then F <= 2^(32 + m_p - M_hw), or
+// S_R >= I0 2^k when s_d = 0); the host selects this form (DIRECT) only under those conditions.
+// b: bits of the fp32 value (max + 2^23) - s, as for shift_exp_bits.
+template <bool FASTQ>
+__device__ __forceinline__ uint32_t smx_out_direct(uint32_t b, const ShiftExpC &c, uint32_t F, uint32_t sh0) {
+    uint32_t n = b + ((b + 1u) >> 1) - ((b + 15u) >> 4) - 1808793600u;
+    n = min(n, (uint32_t)c.kI0);
+    const uint32_t q = FASTQ ? __umulhi(n, c.m32) : (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
+    const uint32_t Ib = ((q + 2u) * (uint32_t)c.I0 - n) >> 1;
+    return shr_sat(Ib * F, sh0 + q);
+}
+
 struct Group {
     int64_t base;  // b * T
     int32_t Tg;
@@ -84,7 +115,7 @@ struct Group {
 
 // QF16: q, k, v arrive as fp16 (the int8 values, exact) and are copied to shared memory as they
 // are; otherwise they arrive as int8 and are converted on the way in.
-template <int DH, bool FASTQ, bool QF16>
+template <int DH, bool FASTQ, bool QF16, bool DIRECT>
 __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     constexpr int LDH = DH * 2 + 16;  // padded fp16 row (bytes): conflict-free ldmatrix
     constexpr int KS = DH / 16;       // k16 steps of q k^T
@@ -144,6 +175,13 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
         }
     }
 
+    // q is negated (exact in fp16), so that the MMAs produce C - s: with C = 0 the row maximum is
+    // minus the minimum of pass 1, and with C = max + 2^23 passes 2 and 3 get (max + 2^23) - s directly.
+#pragma unroll
+    for (int ks = 0; ks < KS; ++ks)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) qa[ks][i] ^= 0x80008000u;
+
     const int nkb = (Tg + KB - 1) / KB;
     // Key blocks go global (int8) -> registers -> shared (fp16), double buffered: the loads of
     // block kb+1 are in flight while block kb is computed.
@@ -179,11 +217,10 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
             }
         }
     };
-    // scores of this warp's 16 rows x the 64 keys of buffer `buf` (exact integers in fp32)
-    auto scores = [&](int buf, float (&S)[8][4]) {
+    // c - s for this warp's 16 rows x the 64 keys of buffer `buf` (c0 for row g, c1 for row g + 8;
+    // exact integers in fp32, below 2^24 in magnitude)
+    auto scores = [&](int buf, float (&S)[8][4], float c0, float c1) {
         const uint32_t ks_base = (uint32_t)__cvta_generic_to_shared(Ks[buf]);
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) S[nt][0] = S[nt][1] = S[nt][2] = S[nt][3] = 0.f;
 #pragma unroll
         for (int np = 0; np < 4; ++np) {      // pairs of n-tiles (16 keys)
 #pragma unroll
@@ -194,8 +231,13 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
                 const uint32_t addr = ks_base + row * LDH + (16 * kp + 8 * (i >> 1)) * 2;
                 uint32_t r0, r1, r2, r3;
                 ldsm_x4(addr, r0, r1, r2, r3);  // r0: n-tile 2np, k lo; r1: 2np+1, k lo; r2, r3: k hi
-                mma_f16(S[2 * np], qa[kp], r0, r2);
-                mma_f16(S[2 * np + 1], qa[kp], r1, r3);
+                if (kp == 0) {
+                    mma_f16_init(S[2 * np], qa[kp], r0, r2, c0, c1);
+                    mma_f16_init(S[2 * np + 1], qa[kp], r1, r3, c0, c1);
+                } else {
+                    mma_f16(S[2 * np], qa[kp], r0, r2);
+                    mma_f16(S[2 * np + 1], qa[kp], r1, r3);
+                }
                 if (kp + 1 < KS) {
                     ldsm_x4(addr + 16 * 2, r0, r1, r2, r3);  // next k16 step: 16 dims further
                     mma_f16(S[2 * np], qa[kp + 1], r0, r2);
@@ -266,53 +308,54 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
         pre_buf = (b0 + nkb) & 1;
     };
 
-    // ---- pass 1: exact row maxima
-    float mx0 = -3.0e38f, mx1 = -3.0e38f;
+    // ---- pass 1: exact row maxima (the MMAs give -s; max s = -min)
+    float mn0 = 3.0e38f, mn1 = 3.0e38f;
     sweep(false, true, false, [&](int kb, int buf, bool full) {
         float S[8][4];
-        scores(buf, S);
+        scores(buf, S, 0.f, 0.f);
         if (full) {
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
-                mx0 = fmaxf(mx0, fmaxf(S[nt][0], S[nt][1]));
-                mx1 = fmaxf(mx1, fmaxf(S[nt][2], S[nt][3]));
+                mn0 = fminf(mn0, fminf(S[nt][0], S[nt][1]));
+                mn1 = fminf(mn1, fminf(S[nt][2], S[nt][3]));
             }
         } else {
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
                 const int key = kb * KB + nt * 8 + 2 * t;
-                if (key < Tg) { mx0 = fmaxf(mx0, S[nt][0]); mx1 = fmaxf(mx1, S[nt][2]); }
-                if (key + 1 < Tg) { mx0 = fmaxf(mx0, S[nt][1]); mx1 = fmaxf(mx1, S[nt][3]); }
+                if (key < Tg) { mn0 = fminf(mn0, S[nt][0]); mn1 = fminf(mn1, S[nt][2]); }
+                if (key + 1 < Tg) { mn0 = fminf(mn0, S[nt][1]); mn1 = fminf(mn1, S[nt][3]); }
             }
         }
     });
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    // ShiftExp(s - max) is read off the bits of (max + 2^23) - s (exact: integers below 2^23)
-    const float mb0 = mx0 + 8388608.0f, mb1 = mx1 + 8388608.0f;
+    mn0 = fminf(mn0, __shfl_xor_sync(0xffffffffu, mn0, 1));
+    mn0 = fminf(mn0, __shfl_xor_sync(0xffffffffu, mn0, 2));
+    mn1 = fminf(mn1, __shfl_xor_sync(0xffffffffu, mn1, 1));
+    mn1 = fminf(mn1, __shfl_xor_sync(0xffffffffu, mn1, 2));
+    // ShiftExp(s - max) is read off the bits of (max + 2^23) - s (exact: integers below 2^23), which
+    // the MMAs of passes 2 and 3 produce with C = max + 2^23
+    const float mb0 = 8388608.0f - mn0, mb1 = 8388608.0f - mn1;
     const ShiftExpC se = p.smx.se;
-    auto sexp = [&](float mb, float sv) { return shift_exp_bits<FASTQ>(__float_as_uint(mb - sv), se); };
+    auto sexp = [&](float d) { return shift_exp_bits<FASTQ>(__float_as_uint(d), se); };
 
     // ---- pass 2: S_sum = sum ShiftExp(s - max)
     uint64_t sum0 = 0, sum1 = 0;
     sweep(false, true, true, [&](int kb, int buf, bool full) {
         float S[8][4];
-        scores(buf, S);
+        scores(buf, S, mb0, mb1);
         if (full) {
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
-                sum0 += (uint64_t)sexp(mb0, S[nt][0]) + sexp(mb0, S[nt][1]);
-                sum1 += (uint64_t)sexp(mb1, S[nt][2]) + sexp(mb1, S[nt][3]);
+                sum0 += (uint64_t)sexp(S[nt][0]) + sexp(S[nt][1]);
+                sum1 += (uint64_t)sexp(S[nt][2]) + sexp(S[nt][3]);
             }
         } else {
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
                 const int key = kb * KB + nt * 8 + 2 * t;
                 const bool v0 = key < Tg, v1 = key + 1 < Tg;
-                sum0 += (uint64_t)(v0 ? sexp(mb0, S[nt][0]) : 0u) + (v1 ? sexp(mb0, S[nt][1]) : 0u);
-                sum1 += (uint64_t)(v0 ? sexp(mb1, S[nt][2]) : 0u) + (v1 ? sexp(mb1, S[nt][3]) : 0u);
+                sum0 += (uint64_t)(v0 ? sexp(S[nt][0]) : 0u) + (v1 ? sexp(S[nt][1]) : 0u);
+                sum1 += (uint64_t)(v0 ? sexp(S[nt][2]) : 0u) + (v1 ? sexp(S[nt][3]) : 0u);
             }
         }
     });
@@ -323,6 +366,7 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     // rows past Tg see sum >= 1 too (their max is over valid keys); their outputs are not stored
     const RowNorm rn0 = shiftmax_norm(sum0 ? sum0 : 1, p.smx.s_d, p.smx.m_p, p.smx.M_hw, p.smx.k_out);
     const RowNorm rn1 = shiftmax_norm(sum1 ? sum1 : 1, p.smx.s_d, p.smx.m_p, p.smx.M_hw, p.smx.k_out);
+    const uint32_t sh00 = (uint32_t)(rn0.sh - se.k), sh01 = (uint32_t)(rn1.sh - se.k);  // >= 8
 
     // ---- pass 3: P = (I_exp F) >> sh (exact integers < 256), O += P V
     float o[NT][4];
@@ -330,26 +374,29 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     for (int nt = 0; nt < NT; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
     sweep(true, false, false, [&](int kb, int buf, bool full) {
         float S[8][4];
-        scores(buf, S);
+        scores(buf, S, mb0, mb1);
         uint32_t pa[4][4];  // A fragments of P for the 4 k16 steps (16 keys each)
+        // P of one score: (I_exp F) >> sh, or its direct form from ShiftExp's parts
+        auto pout0 = [&](float d) { return DIRECT ? smx_out_direct<FASTQ>(__float_as_uint(d), se, rn0.F, sh00)
+                                                  : shiftmax_out(sexp(d), rn0); };
+        auto pout1 = [&](float d) { return DIRECT ? smx_out_direct<FASTQ>(__float_as_uint(d), se, rn1.F, sh01)
+                                                  : shiftmax_out(sexp(d), rn1); };
         // n-tile nt covers keys 8nt..8nt+7 = half (nt & 1) of k16 step nt >> 1
         if (full) {
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
-                pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(shiftmax_out(sexp(mb0, S[nt][0]), rn0),
-                                                            shiftmax_out(sexp(mb0, S[nt][1]), rn0));  // row g
-                pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(shiftmax_out(sexp(mb1, S[nt][2]), rn1),
-                                                            shiftmax_out(sexp(mb1, S[nt][3]), rn1));  // row g + 8
+                pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(pout0(S[nt][0]), pout0(S[nt][1]));  // row g
+                pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(pout1(S[nt][2]), pout1(S[nt][3]));  // row g + 8
             }
         } else {
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
                 const int key = kb * KB + nt * 8 + 2 * t;
                 const bool v0 = key < Tg, v1 = key + 1 < Tg;
-                const uint32_t p0 = v0 ? shiftmax_out(sexp(mb0, S[nt][0]), rn0) : 0u;
-                const uint32_t p1 = v1 ? shiftmax_out(sexp(mb0, S[nt][1]), rn0) : 0u;
-                const uint32_t p2 = v0 ? shiftmax_out(sexp(mb1, S[nt][2]), rn1) : 0u;
-                const uint32_t p3 = v1 ? shiftmax_out(sexp(mb1, S[nt][3]), rn1) : 0u;
+                const uint32_t p0 = v0 ? pout0(S[nt][0]) : 0u;
+                const uint32_t p1 = v1 ? pout0(S[nt][1]) : 0u;
+                const uint32_t p2 = v0 ? pout1(S[nt][2]) : 0u;
+                const uint32_t p3 = v1 ? pout1(S[nt][3]) : 0u;
                 pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(p0, p1);
                 pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(p2, p3);
             }
@@ -402,23 +449,23 @@ cudaError_t launch_attention(const AttnParams &p, cudaStream_t s) {
     if (p.B == 0 || Tg == 0) return cudaSuccess;
     dim3 grid((Tg + QT - 1) / QT, p.H, p.B * G2);
     const bool fastq = p.smx.se.m32 != 0;
+    // the direct output form needs per-row s_d and I_b F < 2^32 (m_p <= M_hw - 15), and sh >= k
+    const bool direct = p.smx.s_d < 0 && p.smx.m_p + 15 <= p.smx.M_hw && 32 - p.smx.k_out >= p.smx.se.k;
+#define ILW_ATTN(DH, QF)                                                                          \
+    do {                                                                                          \
+        if (fastq && direct) attn_kernel<DH, true, QF, true><<<grid, THREADS, 0, s>>>(p);         \
+        else if (fastq) attn_kernel<DH, true, QF, false><<<grid, THREADS, 0, s>>>(p);             \
+        else if (direct) attn_kernel<DH, false, QF, true><<<grid, THREADS, 0, s>>>(p);            \
+        else attn_kernel<DH, false, QF, false><<<grid, THREADS, 0, s>>>(p);                       \
+    } while (0)
     if (p.qkv_f16) {
-        if (p.dh == 64) {
-            if (fastq) attn_kernel<64, true, true><<<grid, THREADS, 0, s>>>(p);
-            else attn_kernel<64, false, true><<<grid, THREADS, 0, s>>>(p);
-        } else {
-            if (fastq) attn_kernel<32, true, true><<<grid, THREADS, 0, s>>>(p);
-            else attn_kernel<32, false, true><<<grid, THREADS, 0, s>>>(p);
-        }
+        if (p.dh == 64) ILW_ATTN(64, true);
+        else ILW_ATTN(32, true);
     } else {
-        if (p.dh == 64) {
-            if (fastq) attn_kernel<64, true, false><<<grid, THREADS, 0, s>>>(p);
-            else attn_kernel<64, false, false><<<grid, THREADS, 0, s>>>(p);
-        } else {
-            if (fastq) attn_kernel<32, true, false><<<grid, THREADS, 0, s>>>(p);
-            else attn_kernel<32, false, false><<<grid, THREADS, 0, s>>>(p);
-        }
+        if (p.dh == 64) ILW_ATTN(64, false);
+        else ILW_ATTN(32, false);
     }
+#undef ILW_ATTN
     return cudaGetLastError();
 }
 

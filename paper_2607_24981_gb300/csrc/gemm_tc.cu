@@ -29,6 +29,7 @@
 #include <cstdint>
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 
 #include "ilw_kernels.h"
 
@@ -58,8 +59,7 @@ struct TcParams {  // CUtensorMap members keep the 64-byte alignment TMA needs
     int32_t tiles_n, tiles;
     int32_t nbuf;       // TMEM accumulator sets (1 or 2)
     int32_t tmem_cols;
-    int32_t gelu_T;     // SD-ShiftGELU table covers g in [-gelu_T, gelu_T] (constant beyond)
-    const uint8_t *gelu_tab;  // that table in global memory (16-byte aligned, 65536 bytes)
+    const int8_t *gelu_tab;  // SD-ShiftGELU output table in global memory (16-byte aligned, 65536 bytes)
     int *status;
     EpiParams ep;
 };
@@ -184,31 +184,24 @@ __device__ __forceinline__ void lds16(const int32_t *p, int32_t (&o)[16]) {
                      : "r"(a + 16 * j));
 }
 
-// rq(v; m, s) for int32 v and s >= 33, given sh1 = s - 33.  With v m = H 2^32 + L (0 <= L < 2^32),
-// L / 2^32 < 1 added to an integer numerator never changes floor(. / 2^(s-32)), so
-// rq = floor((H + 2^(s-33)) / 2^(s-32)); and floor((h + 2^(k-1)) / 2^k) = (floor(h / 2^(k-1)) + 1) >> 1
-// for k >= 1, which needs no rounding constant.
-__device__ __forceinline__ int32_t rq_hi1(int32_t v, int32_t m, int32_t sh1) {
-    return ((__mulhi(v, m) >> sh1) + 1) >> 1;
-}
-
 // The fused epilogue of 16 consecutive columns of one row, computed stage by stage so that the
-// 16 independent elements overlap.  fastw (uniform across the warp, decided per tile) says every
-// shift of the warp's columns is >= 33; ss then holds s - 33, else s.
-template <int KIND>
-__device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool fastw, bool has_res, const uint32_t (&rp)[8],
+// 16 independent elements overlap.  FAST (uniform across the warp, decided per tile) says every
+// shift of the warp's columns is >= 33; ss then holds s - 32 and sr 2^(s-33) (rq_hi), else ss
+// holds s.  RFAST: the residual's shift s_r is >= 17.  gtab points at entry 0 of the SD-ShiftGELU output table (index -32767 .. 32767).
+template <int KIND, bool FAST, bool RFAST>
+__device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool has_res, const uint32_t (&rp)[8],
                                           const int32_t (&acc)[16], const int32_t (&sb)[16],
                                           const int32_t (&sm)[16], const int32_t (&ss)[16],
-                                          const uint8_t *gtab, int32_t gT, int32_t (&out)[16]) {
+                                          const int32_t (&sr)[16], const int8_t *gtab, int32_t (&out)[16]) {
     if (KIND == KIND_RAW32) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) out[i] = acc[i] + sb[i];
         return;
     }
     int32_t r[16];
-    if (fastw) {
+    if (FAST) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) r[i] = rq_hi1(acc[i] + sb[i], sm[i], ss[i]);  // |r| < 2^29
+        for (int i = 0; i < 16; ++i) r[i] = rq_hi(acc[i] + sb[i], sm[i], sr[i], ss[i]);  // |r| < 2^29
     } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -217,26 +210,22 @@ __device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool fastw, bool 
         }
     }
     if (KIND == KIND_GELU8) {
-        const bool gfast = ep.s_g >= 33;
+        // g = sat16(r); the table holds sat8(rq(g * I_div(g); m_g, s_g)) for every int16 g
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            const int32_t g = sat16(r[i]);
-            const int32_t gi = g * (int32_t)gtab[min(max(g, -gT), gT) + gT];  // g * I_div(g), |.| < 2^22
-            out[i] = sat8(gfast ? rq_hi1(gi, ep.m_g, ep.s_g - 33) : rq((int64_t)gi, ep.m_g, ep.s_g));
-        }
+        for (int i = 0; i < 16; ++i) out[i] = gtab[clamp16(r[i])];
         return;
     }
     if (has_res) {
         // rp holds the 16 int16 residuals in pairs; x * 2^16 is the pair word masked or shifted
-        const bool rfast = ep.s_r >= 17;  // then rq(x; m_r, s_r) = rq(x * 2^16; m_r, s_r + 16), s_r + 16 >= 33
+        // (RFAST: rq(x; m_r, s_r) = rq(x * 2^16; m_r, s_r + 16) with s_r + 16 >= 33)
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             const int32_t xs = (i & 1) ? (int32_t)(rp[i >> 1] & 0xFFFF0000u) : (int32_t)(rp[i >> 1] << 16);
-            r[i] += rfast ? rq_hi1(xs, ep.m_r, ep.s_r - 17) : (int32_t)rq((int64_t)(xs >> 16), ep.m_r, ep.s_r);
+            r[i] += RFAST ? rq_hi(xs, ep.m_r, 1 << (ep.s_r - 17), ep.s_r - 16) : (int32_t)rq((int64_t)(xs >> 16), ep.m_r, ep.s_r);
         }
     }
 #pragma unroll
-    for (int i = 0; i < 16; ++i) out[i] = (KIND == KIND_RQ8 || KIND == KIND_F16OUT) ? sat8(r[i]) : sat16(r[i]);
+    for (int i = 0; i < 16; ++i) out[i] = (KIND == KIND_RQ8 || KIND == KIND_F16OUT) ? clamp8(r[i]) : clamp16(r[i]);
 }
 
 template <int BN, int STAGES, int KIND, int NB>
@@ -280,13 +269,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    // SD-ShiftGELU: I_div depends on the int16 value g alone and is constant once both ShiftExp
-    // inputs are clamped (|g| > gelu_T); the table (built once per parameter set by
-    // gelu_table_kernel with the same device function) is copied into shared memory here.
-    uint8_t *gtab = (uint8_t *)((int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + 12 * BN);
+    // SD-ShiftGELU and its output requantisation depend on the int16 value g alone: the table of
+    // sat8(rq(g * I_div(g); m_g, s_g)) (built once per parameter set by gelu_table_kernel) is
+    // copied into shared memory here.
+    int8_t *gtab = (int8_t *)((int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + 16 * BN);
     if (KIND == KIND_GELU8 && warp >= 6) {
-        const int n16 = (2 * p.gelu_T + 1 + 15) / 16;
-        for (int i = threadIdx.x - 192; i < n16; i += 256) ((uint4 *)gtab)[i] = __ldg((const uint4 *)p.gelu_tab + i);
+        for (int i = threadIdx.x - 192; i < 65536 / 16; i += 256) ((uint4 *)gtab)[i] = __ldg((const uint4 *)p.gelu_tab + i);
         asm volatile("bar.sync 1, 256;" ::: "memory");  // the 8 epilogue warps only
     }
     const int acc_cols = p.nseg * BN;  // columns of one accumulator set
@@ -396,9 +384,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         constexpr int HALF = BN / 2;
         const int q = warp & 3, h = (warp - 6) >> 2;
         const EpiParams &ep = p.ep;
-        int32_t *s_bias = (int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + (warp - 6) * 3 * HALF;  // this warp's copy of
+        int32_t *s_bias = (int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + (warp - 6) * 4 * HALF;  // this warp's copy of
         int32_t *s_mult = s_bias + HALF;                                       // the tile's per-column
         int32_t *s_shift = s_mult + HALF;                                      // epilogue parameters
+        int32_t *s_rnd = s_shift + HALF;                                       // (rq_hi rounding constants)
         constexpr int bits = (KIND == KIND_RQ16 || KIND == KIND_F16OUT) ? 16 : (KIND == KIND_RAW32 ? 32 : 8);
         constexpr int PPL = HALF / 32;  // parameters per lane and per array
         // The next tile's parameters are fetched into registers while the current tile is processed.
@@ -425,12 +414,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             bool fast_lane = true;
 #pragma unroll
             for (int k = 0; k < PPL; ++k) fast_lane &= ps[k] >= 33;
-            const bool fastw = __all_sync(0xffffffffu, fast_lane);  // shifts stored as s - 33 if so
+            const bool fastw = __all_sync(0xffffffffu, fast_lane);  // shifts stored as s - 32 if so
 #pragma unroll
             for (int k = 0; k < PPL; ++k) {
                 s_bias[lane + 32 * k] = pb[k];
                 s_mult[lane + 32 * k] = pm[k];
-                s_shift[lane + 32 * k] = fastw ? ps[k] - 33 : ps[k];
+                s_shift[lane + 32 * k] = fastw ? ps[k] - 32 : ps[k];
+                s_rnd[lane + 32 * k] = fastw ? 1 << (ps[k] - 33) : 0;
             }
             __syncwarp();
             if (t + (int)gridDim.x < p.tiles) fetch(t + gridDim.x);
@@ -442,122 +432,137 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const int16_t *rrow = (ep.res && row_ok) ? ep.res + (row % ep.res_rows) * ep.ldr + n0 : nullptr;
             const bool rvec = ((uintptr_t)rrow & 15) == 0;
             const bool has_res = ep.res != nullptr;
+            const bool rfast = has_res && ep.s_r >= 17;
             uint32_t rp[8];
             const uint32_t tbase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * acc_cols + h * HALF);
-            // TMEM load i reads segment i % nseg of chunk i / nseg; load i+1 is in flight while the
-            // epilogue of load i's chunk runs.
-            uint32_t v[16];
-            tmem_ld16(tbase, v);
-            int32_t acc[16];
+            // The tile's chunks, with the requantisation forms fixed for the whole tile (a branch per
+            // tile instead of both forms predicated per element).  TMEM load i reads segment i % nseg
+            // of chunk i / nseg; load i+1 is in flight while the epilogue of load i's chunk runs.
+            auto chunks = [&](auto fast_c, auto rfast_c) {
+                constexpr bool FAST = decltype(fast_c)::value, RFAST = decltype(rfast_c)::value;
+                uint32_t v[16];
+                tmem_ld16(tbase, v);
+                int32_t acc[16];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) acc[i] = 0;
-            for (int li = 0; li < nld; ++li) {
-                const int c0 = (li / nseg) * 16, sg = li - (li / nseg) * nseg;
-                if (has_res && sg == 0) {  // this chunk's residuals, in flight during the TMEM wait
-                    if (rrow && rvec && n0 + c0 + 16 <= p.N) {
-                        const uint4 a = __ldg((const uint4 *)(rrow + c0)), b = __ldg((const uint4 *)(rrow + c0) + 1);
-                        rp[0] = a.x; rp[1] = a.y; rp[2] = a.z; rp[3] = a.w;
-                        rp[4] = b.x; rp[5] = b.y; rp[6] = b.z; rp[7] = b.w;
-                    } else {
+                for (int i = 0; i < 16; ++i) acc[i] = 0;
+                for (int li = 0; li < nld; ++li) {
+                    const int c0 = (li / nseg) * 16, sg = li - (li / nseg) * nseg;
+                    if (has_res && sg == 0) {  // this chunk's residuals, in flight during the TMEM wait
+                        if (rrow && rvec && n0 + c0 + 16 <= p.N) {
+                            const uint4 a = __ldg((const uint4 *)(rrow + c0)), b = __ldg((const uint4 *)(rrow + c0) + 1);
+                            rp[0] = a.x; rp[1] = a.y; rp[2] = a.z; rp[3] = a.w;
+                            rp[4] = b.x; rp[5] = b.y; rp[6] = b.z; rp[7] = b.w;
+                        } else {
 #pragma unroll
-                        for (int j = 0; j < 8; ++j) {
-                            const int cl = n0 + c0 + 2 * j;
-                            const uint32_t lo = (rrow && cl < p.N) ? (uint16_t)rrow[c0 + 2 * j] : 0u;
-                            const uint32_t hi = (rrow && cl + 1 < p.N) ? (uint16_t)rrow[c0 + 2 * j + 1] : 0u;
-                            rp[j] = lo | (hi << 16);
+                            for (int j = 0; j < 8; ++j) {
+                                const int cl = n0 + c0 + 2 * j;
+                                const uint32_t lo = (rrow && cl < p.N) ? (uint16_t)rrow[c0 + 2 * j] : 0u;
+                                const uint32_t hi = (rrow && cl + 1 < p.N) ? (uint16_t)rrow[c0 + 2 * j + 1] : 0u;
+                                rp[j] = lo | (hi << 16);
+                            }
                         }
                     }
-                }
-                tmem_wait_ld16(v);
-                if (p.branch_rq) {
-                    const int32_t mb = p.seg[sg].m_b, sbb = p.seg[sg].s_b;
+                    tmem_wait_ld16(v);
+                    if (p.branch_rq) {
+                        const int32_t mb = p.seg[sg].m_b, sbb = p.seg[sg].s_b;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) acc[i] += (int32_t)rq(__float2int_rn(__uint_as_float(v[i])), mb, sbb);
-                } else {
+                        for (int i = 0; i < 16; ++i) acc[i] += (int32_t)rq(__float2int_rn(__uint_as_float(v[i])), mb, sbb);
+                    } else {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) acc[i] += __float2int_rn(__uint_as_float(v[i]));  // exact: < 2^24
-                }
-                if (li + 1 < nld) {
-                    const int c1 = ((li + 1) / nseg) * 16, sg1 = (li + 1) - ((li + 1) / nseg) * nseg;
-                    tmem_ld16(tbase + (uint32_t)(sg1 * BN + c1), v);
-                } else {  // every TMEM read of this warp in this accumulator set is done
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(acc_empty(b));
-                }
-                if (sg != nseg - 1) continue;
-                int32_t cb[16], cm[16], cs[16];  // this chunk's per-column parameters
-                lds16(s_bias + c0, cb);
-                lds16(s_mult + c0, cm);
-                lds16(s_shift + c0, cs);
-                const int ncol = min(16, p.N - (n0 + c0));
-                if (row_ok && ncol > 0) {
-                    int32_t out[16];
-                    epi_chunk<KIND>(ep, fastw, has_res, rp, acc, cb, cm, cs, gtab, p.gelu_T, out);
-                    char *dst = (char *)ep.C + (row * ep.ldc + n0 + c0) * (bits / 8);
-                    const bool vec = ncol == 16 && (((uintptr_t)dst & 15) == 0);
-                    if constexpr (KIND == KIND_F16OUT) {
-                        // |v| <= 127: the fp16 bits of 1152 + v are 0x6480 + v; one half2 subtract of
-                        // 1152 leaves v exactly
-                        const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
-                        uint32_t hw[8];
+                        for (int i = 0; i < 16; ++i) acc[i] += __float2int_rn(__uint_as_float(v[i]));  // exact: < 2^24
+                    }
+                    if (li + 1 < nld) {
+                        const int c1 = ((li + 1) / nseg) * 16, sg1 = (li + 1) - ((li + 1) / nseg) * nseg;
+                        tmem_ld16(tbase + (uint32_t)(sg1 * BN + c1), v);
+                    } else {  // every TMEM read of this warp in this accumulator set is done
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(acc_empty(b));
+                    }
+                    if (sg != nseg - 1) continue;
+                    int32_t cb[16], cm[16], cs[16], cr[16];  // this chunk's per-column parameters
+                    lds16(s_bias + c0, cb);
+                    lds16(s_mult + c0, cm);
+                    lds16(s_shift + c0, cs);
+                    if (FAST) lds16(s_rnd + c0, cr);
+                    const int ncol = min(16, p.N - (n0 + c0));
+                    if (row_ok && ncol > 0) {
+                        int32_t out[16];
+                        const int8_t *gt = gtab + 32767;
+                        epi_chunk<KIND, FAST, RFAST>(ep, has_res, rp, acc, cb, cm, cs, cr, gt, out);
+                        char *dst = (char *)ep.C + (row * ep.ldc + n0 + c0) * (bits / 8);
+                        const bool vec = ncol == 16 && (((uintptr_t)dst & 15) == 0);
+                        if constexpr (KIND == KIND_F16OUT) {
+                            // |v| <= 127: the fp16 bits of 1152 + v are 0x6480 + v; one half2 subtract of
+                            // 1152 leaves v exactly
+                            const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
+                            uint32_t hw[8];
 #pragma unroll
-                        for (int j = 0; j < 8; ++j) {
-                            uint32_t x = (uint32_t)(0x6480 + out[2 * j]) | ((uint32_t)(0x6480 + out[2 * j + 1]) << 16);
-                            __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), k1152);
-                            hw[j] = *reinterpret_cast<uint32_t *>(&h);
-                        }
-                        if (vec) {
-                            ((uint4 *)dst)[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-                            ((uint4 *)dst)[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
-                        } else {
+                            for (int j = 0; j < 8; ++j) {
+                                uint32_t x = (uint32_t)(0x6480 + out[2 * j]) | ((uint32_t)(0x6480 + out[2 * j + 1]) << 16);
+                                __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), k1152);
+                                hw[j] = *reinterpret_cast<uint32_t *>(&h);
+                            }
+                            if (vec) {
+                                ((uint4 *)dst)[0] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+                                ((uint4 *)dst)[1] = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+                            } else {
 #pragma unroll
-                            for (int i = 0; i < 16; ++i)
-                                if (i < ncol) ((uint16_t *)dst)[i] = (uint16_t)((i & 1) ? hw[i >> 1] >> 16 : hw[i >> 1]);
-                        }
-                    } else if constexpr (bits == 8) {
-                        if (vec) {
-                            uint32_t w[4];
-#pragma unroll
-                            for (int u = 0; u < 4; ++u)
-                                w[u] = (uint32_t)(uint8_t)out[4 * u] | ((uint32_t)(uint8_t)out[4 * u + 1] << 8) |
-                                       ((uint32_t)(uint8_t)out[4 * u + 2] << 16) | ((uint32_t)(uint8_t)out[4 * u + 3] << 24);
-                            *(uint4 *)dst = make_uint4(w[0], w[1], w[2], w[3]);
-                        } else {
-#pragma unroll
-                            for (int i = 0; i < 16; ++i)
-                                if (i < ncol) ((int8_t *)dst)[i] = (int8_t)out[i];
-                        }
-                    } else if constexpr (bits == 16) {
-                        if (vec) {
-#pragma unroll
-                            for (int j = 0; j < 2; ++j) {
+                                for (int i = 0; i < 16; ++i)
+                                    if (i < ncol) ((uint16_t *)dst)[i] = (uint16_t)((i & 1) ? hw[i >> 1] >> 16 : hw[i >> 1]);
+                            }
+                        } else if constexpr (bits == 8) {
+                            if (vec) {
                                 uint32_t w[4];
 #pragma unroll
                                 for (int u = 0; u < 4; ++u)
-                                    w[u] = (uint32_t)(uint16_t)out[8 * j + 2 * u] | ((uint32_t)(uint16_t)out[8 * j + 2 * u + 1] << 16);
-                                ((uint4 *)dst)[j] = make_uint4(w[0], w[1], w[2], w[3]);
+                                    w[u] = (uint32_t)(uint8_t)out[4 * u] | ((uint32_t)(uint8_t)out[4 * u + 1] << 8) |
+                                           ((uint32_t)(uint8_t)out[4 * u + 2] << 16) | ((uint32_t)(uint8_t)out[4 * u + 3] << 24);
+                                *(uint4 *)dst = make_uint4(w[0], w[1], w[2], w[3]);
+                            } else {
+#pragma unroll
+                                for (int i = 0; i < 16; ++i)
+                                    if (i < ncol) ((int8_t *)dst)[i] = (int8_t)out[i];
+                            }
+                        } else if constexpr (bits == 16) {
+                            if (vec) {
+#pragma unroll
+                                for (int j = 0; j < 2; ++j) {
+                                    uint32_t w[4];
+#pragma unroll
+                                    for (int u = 0; u < 4; ++u)
+                                        w[u] = (uint32_t)(uint16_t)out[8 * j + 2 * u] | ((uint32_t)(uint16_t)out[8 * j + 2 * u + 1] << 16);
+                                    ((uint4 *)dst)[j] = make_uint4(w[0], w[1], w[2], w[3]);
+                                }
+                            } else {
+#pragma unroll
+                                for (int i = 0; i < 16; ++i)
+                                    if (i < ncol) ((int16_t *)dst)[i] = (int16_t)out[i];
                             }
                         } else {
+                            if (vec) {
 #pragma unroll
-                            for (int i = 0; i < 16; ++i)
-                                if (i < ncol) ((int16_t *)dst)[i] = (int16_t)out[i];
-                        }
-                    } else {
-                        if (vec) {
+                                for (int j = 0; j < 4; ++j)
+                                    ((int4 *)dst)[j] = make_int4(out[4 * j], out[4 * j + 1], out[4 * j + 2], out[4 * j + 3]);
+                            } else {
 #pragma unroll
-                            for (int j = 0; j < 4; ++j)
-                                ((int4 *)dst)[j] = make_int4(out[4 * j], out[4 * j + 1], out[4 * j + 2], out[4 * j + 3]);
-                        } else {
-#pragma unroll
-                            for (int i = 0; i < 16; ++i)
-                                if (i < ncol) ((int32_t *)dst)[i] = out[i];
+                                for (int i = 0; i < 16; ++i)
+                                    if (i < ncol) ((int32_t *)dst)[i] = out[i];
+                            }
                         }
                     }
-                }
 #pragma unroll
-                for (int i = 0; i < 16; ++i) acc[i] = 0;
-                __syncwarp();  // reconverge before the next warp-synchronous tcgen05 instruction
+                    for (int i = 0; i < 16; ++i) acc[i] = 0;
+                    __syncwarp();  // reconverge before the next warp-synchronous tcgen05 instruction
+                }
+            };
+            constexpr bool kRes = KIND == KIND_RQ8 || KIND == KIND_RQ16;  // kinds with a residual
+            if (fastw) {
+                if (kRes && rfast) chunks(std::integral_constant<bool, true>{}, std::integral_constant<bool, kRes>{});
+                else chunks(std::integral_constant<bool, true>{}, std::integral_constant<bool, false>{});
+            } else {
+                if (kRes && rfast) chunks(std::integral_constant<bool, false>{}, std::integral_constant<bool, kRes>{});
+                else chunks(std::integral_constant<bool, false>{}, std::integral_constant<bool, false>{});
             }
         }
     }
@@ -571,32 +576,37 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     }
 }
 
-// SD-ShiftGELU tables, one slot per parameter set: entry i is I_div(i - T) for i in [0, 2T].
+// SD-ShiftGELU output tables, one slot per parameter set (I0, k_inter, k_out, m_g, s_g): entry
+// g + 32767 is sat8(rq(g * I_div(g); m_g, s_g)) for every int16 value g (Algorithm 1 followed by the
+// output requantisation), a pure function of g.
 constexpr int kGeluSlots = 32;
-constexpr int kGeluTabBytes = 65536;  // 2T + 1 <= 65535 for T <= 32767, rounded up to 16 bytes
-__device__ __align__(16) uint8_t g_gelu_tab[kGeluSlots][kGeluTabBytes];
+constexpr int kGeluTabBytes = 65536;  // 65535 entries, padded to 16 bytes
+__device__ __align__(16) int8_t g_gelu_tab[kGeluSlots][kGeluTabBytes];
 
-__global__ void gelu_table_kernel(uint8_t *tab, int32_t T, GeluC c) {
+__global__ void gelu_table_kernel(int8_t *tab, GeluC c, int32_t m_g, int32_t s_g) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i <= 2 * T) tab[i] = (uint8_t)gelu_idiv(i - T, c);
+    if (i < kGeluTabBytes) {
+        const int32_t g = min(i, 65534) - 32767;
+        tab[i] = (int8_t)sat8(rq((int64_t)g * gelu_idiv(g, c), m_g, s_g));
+    }
 }
 
-// The table slot of (device, GELU constants, T), built on first use.  The first build of a slot is
-// waited for (unless the stream is being captured), so a slot marked built is complete for every
-// stream; a build recorded into a graph is repeated by each replay until an eager call builds it.
-const uint8_t *gelu_table(const GeluC &c, int32_t T, cudaStream_t s, cudaError_t *err) {
+// The table slot of (device, GELU constants, m_g, s_g), built on first use.  The first build of a
+// slot is waited for (unless the stream is being captured), so a slot marked built is complete for
+// every stream; a build recorded into a graph is repeated by each replay until an eager call builds it.
+const int8_t *gelu_table(const GeluC &c, int32_t m_g, int32_t s_g, cudaStream_t s, cudaError_t *err) {
     struct Key {
         int dev;
-        int32_t I0, k, out_sh, T;
+        int32_t I0, k, out_sh, m_g, s_g;
         bool operator==(const Key &o) const {
-            return dev == o.dev && I0 == o.I0 && k == o.k && out_sh == o.out_sh && T == o.T;
+            return dev == o.dev && I0 == o.I0 && k == o.k && out_sh == o.out_sh && m_g == o.m_g && s_g == o.s_g;
         }
     };
     static std::mutex mu;
     static Key keys[64][kGeluSlots];
     static bool used[64][kGeluSlots] = {}, built[64][kGeluSlots] = {};
     static int next[64] = {};
-    static uint8_t *base[64] = {};
+    static int8_t *base[64] = {};
     *err = cudaSuccess;
     int dev = 0;
     if ((*err = cudaGetDevice(&dev)) != cudaSuccess) return nullptr;
@@ -608,9 +618,9 @@ const uint8_t *gelu_table(const GeluC &c, int32_t T, cudaStream_t s, cudaError_t
     if (!base[dev]) {
         void *b = nullptr;
         if ((*err = cudaGetSymbolAddress(&b, g_gelu_tab)) != cudaSuccess) return nullptr;
-        base[dev] = (uint8_t *)b;
+        base[dev] = (int8_t *)b;
     }
-    const Key key{dev, c.se.I0, c.se.k, c.out_sh, T};
+    const Key key{dev, c.se.I0, c.se.k, c.out_sh, m_g, s_g};
     int slot = -1;
     for (int i = 0; i < kGeluSlots; ++i)
         if (used[dev][i] && keys[dev][i] == key) slot = i;
@@ -621,9 +631,9 @@ const uint8_t *gelu_table(const GeluC &c, int32_t T, cudaStream_t s, cudaError_t
         used[dev][slot] = true;
         built[dev][slot] = false;
     }
-    uint8_t *tab = base[dev] + (size_t)slot * kGeluTabBytes;
+    int8_t *tab = base[dev] + (size_t)slot * kGeluTabBytes;
     if (!built[dev][slot]) {
-        gelu_table_kernel<<<(2 * T + 1 + 255) / 256, 256, 0, s>>>(tab, T, c);
+        gelu_table_kernel<<<kGeluTabBytes / 256, 256, 0, s>>>(tab, c, m_g, s_g);
         if ((*err = cudaGetLastError()) != cudaSuccess) return nullptr;
         cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
         if ((*err = cudaStreamIsCapturing(s, &cs)) != cudaSuccess) return nullptr;
@@ -718,7 +728,7 @@ int num_sms() {
 
 template <int BN, int STAGES, int KIND, int NB>
 cudaError_t launch_tc(TcParams<NB> &tp, cudaStream_t s) {
-    const size_t smem = 1024 + (size_t)STAGES * Smem<BN>::kStage + 8 * (3 * STAGES + 4) + 32 + 4 * 3 * BN * 4 +
+    const size_t smem = 1024 + (size_t)STAGES * Smem<BN>::kStage + 8 * (3 * STAGES + 4) + 32 + 4 * 4 * BN * 4 +
                         (KIND == KIND_GELU8 ? 65536 : 0);
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
@@ -774,13 +784,8 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     if (alloc > 512) return cudaErrorInvalidValue;
     tp.tmem_cols = alloc;
     if (ep.kind == EPI_GELU) {
-        // |g| > T puts both ShiftExp inputs past the clamp: |I_p| >= 1.6875|g| - 3 and
-        // -I_e >= 1.4375|I_p| - 1 >= k I0 once |g| >= ((k I0 + 1)/1.4375 + 3)/1.6875; 0.7 (k I0 + 1) + 8
-        // is above that bound.  g is int16, so T never needs to exceed 32767.
-        const double bound = 0.7 * ((double)ep.gelu.se.kI0 + 1.0) + 8.0;
-        tp.gelu_T = bound > 32767.0 ? 32767 : (int32_t)bound;
         cudaError_t e = cudaSuccess;
-        tp.gelu_tab = gelu_table(ep.gelu, tp.gelu_T, s, &e);
+        tp.gelu_tab = gelu_table(ep.gelu, ep.m_g, ep.s_g, s, &e);
         if (!tp.gelu_tab) return e != cudaSuccess ? e : cudaErrorUnknown;
     }
     if constexpr (NB == 1) {

@@ -21,6 +21,24 @@ __device__ __forceinline__ int32_t sat8(int64_t v) { return (int32_t)(v < -127 ?
 __device__ __forceinline__ int32_t sat16(int64_t v) {
     return (int32_t)(v < -32767 ? -32767 : (v > 32767 ? 32767 : v));
 }
+__device__ __forceinline__ int32_t clamp8(int32_t v) { return max(-127, min(127, v)); }
+__device__ __forceinline__ int32_t clamp16(int32_t v) { return max(-32767, min(32767, v)); }
+
+// rq(v; m, s) for int32 v and s >= 33, given sh1 = s - 33.  With v m = H 2^32 + L (0 <= L < 2^32),
+// L / 2^32 < 1 added to an integer numerator never changes floor(. / 2^(s-32)), so
+// rq = floor((H + 2^(s-33)) / 2^(s-32)); and floor((h + 2^(k-1)) / 2^k) = (floor(h / 2^(k-1)) + 1) >> 1
+// for k >= 1, which needs no rounding constant.  |result| < 2^29.
+__device__ __forceinline__ int32_t rq_hi1(int32_t v, int32_t m, int32_t sh1) {
+    return ((__mulhi(v, m) >> sh1) + 1) >> 1;
+}
+// The same rq with the rounding folded into the multiply: rq = (h + 2^(s-33)) >> (s-32), where
+// h + 2^(s-33) is one mad.hi (high word of v m plus a constant; |h| <= 2^30, so no overflow).
+// rnd = 2^(s-33) and sh = s - 32 are precomputed by the caller (s >= 33).
+__device__ __forceinline__ int32_t rq_hi(int32_t v, int32_t m, int32_t rnd, int32_t sh) {
+    int32_t h;
+    asm("mad.hi.s32 %0, %1, %2, %3;" : "=r"(h) : "r"(v), "r"(m), "r"(rnd));
+    return h >> sh;
+}
 
 // ---- ShiftExp (Algorithm 1) with per-launch constants.
 // The integer part q = floor(n / I0) of n = -I_e in [0, k I0] is taken with the round-up
@@ -58,6 +76,17 @@ __device__ __forceinline__ uint32_t shift_exp_mag(uint32_t a, const ShiftExpC &c
     uint32_t q = (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
     uint32_t r = n - q * (uint32_t)c.I0;               // decimal part, in [0, I0)
     uint32_t Ib = (uint32_t)c.I0 - ((r + 1u) >> 1);    // ((-r) >> 1) + I0
+    return Ib << (c.k - (int32_t)q);
+}
+
+// shift_exp_mag with the single-multiply quotient (FASTQ: c.m32 set) and I0 - ceil(r/2) written as
+// ((q + 2) I0 - n) / 2 (r = n - q I0): the same value in fewer operations.
+template <bool FASTQ>
+__device__ __forceinline__ uint32_t shift_exp_mag_q(uint32_t a, const ShiftExpC &c) {
+    uint32_t n = a + ((a + 1u) >> 1) - ((a + 15u) >> 4);
+    n = min(n, (uint32_t)c.kI0);
+    const uint32_t q = FASTQ ? __umulhi(n, c.m32) : (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
+    const uint32_t Ib = ((q + 2u) * (uint32_t)c.I0 - n) >> 1;
     return Ib << (c.k - (int32_t)q);
 }
 

@@ -137,4 +137,22 @@ cudaError_t launch_deform(const DeformParams &p, cudaStream_t s);
 cudaError_t launch_patchify(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
                             int8_t *A, cudaStream_t s);
 
+// ---------------------------------------------------------------- detector: requantisation, resampling
+struct RequantParams {
+    const void *X;       // int16 or int32 [rows, ldx]
+    int32_t in_bits;     // 16 or 32
+    int64_t ldx, rows;
+    int32_t C;           // multiple of 4
+    int32_t m1, s1;
+    const int16_t *Z;    // optional second term [z_rows, ldz], row r uses r % z_rows
+    int64_t ldz, z_rows;
+    int32_t m2, s2;
+    int32_t out_bits;    // 8, 16 (saturating) or 32
+    void *Y;
+    int64_t ldy;
+};
+cudaError_t launch_requant(const RequantParams &p, cudaStream_t s);
+cudaError_t launch_resample(const int8_t *X, int64_t x_bstride, int32_t B, int32_t Hi, int32_t Wi, int32_t C,
+                            int8_t *Y, int64_t y_bstride, int32_t Ho, int32_t Wo, cudaStream_t s);
+
 }  // namespace ilw

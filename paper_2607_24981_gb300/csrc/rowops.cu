@@ -5,6 +5,7 @@
 // HBM sees each input byte once.  Rows are read with 128-bit loads when the layout allows.
 #include <climits>
 #include <cstdint>
+#include <mutex>
 
 #include "ilw_kernels.h"
 
@@ -44,8 +45,9 @@ __device__ __forceinline__ uint64_t group_sum_u64(uint64_t v) {
 }
 
 // LANES lanes own one row (32 / LANES rows per warp); NCH = 4-element chunks per lane (row length
-// <= 4 * LANES * NCH).  Vector loads need len % 4 == 0 and 16-byte aligned rows.
-template <int NCH, int LANES>
+// <= 4 * LANES * NCH).  Vector loads need len % 4 == 0 and 16-byte aligned rows.  All NCH loads of a
+// lane are issued before the first use, so each warp keeps 32 * NCH * 16 bytes in flight.
+template <int NCH, int LANES, bool FASTQ>
 __global__ void __launch_bounds__(256) shiftmax_rows_vec(const int32_t *__restrict__ X, int64_t ldx,
                                                           int64_t rows, int32_t len, const ShiftmaxC c,
                                                           uint8_t *__restrict__ P, int64_t ldp) {
@@ -56,31 +58,29 @@ __global__ void __launch_bounds__(256) shiftmax_rows_vec(const int32_t *__restri
     const int nch = live ? (len >> 2) : 0;
     const int4 *xr = (const int4 *)(X + (live ? row : 0) * ldx);
     int4 v[NCH];
-    int32_t mx = INT_MIN;
 #pragma unroll
     for (int j = 0; j < NCH; ++j) {
         const int ch = sub + LANES * j;
-        if (ch < nch) {
-            v[j] = __ldcs(xr + ch);
-            mx = max(mx, max(max(v[j].x, v[j].y), max(v[j].z, v[j].w)));
-        }
+        v[j] = ch < nch ? __ldcs(xr + ch) : make_int4(INT_MIN, INT_MIN, INT_MIN, INT_MIN);
     }
+    int32_t mx = INT_MIN;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) mx = max(mx, max(max(v[j].x, v[j].y), max(v[j].z, v[j].w)));
     mx = group_max<LANES>(mx);
-    // differences below -2^30 are deep in ShiftExp's clamp region: use -2^30 there
-    const int32_t lowb = mx > INT_MIN + (1 << 30) ? mx - (1 << 30) : INT_MIN;
+    // a = mx - x >= 0 as an unsigned difference; magnitudes beyond 2^30 are deep in ShiftExp's
+    // clamp region and are replaced by 2^30 (same value).  Padding lanes (INT_MIN) give a >= 2^30
+    // and are not summed.
     uint64_t sum = 0;
 #pragma unroll
     for (int j = 0; j < NCH; ++j) {
         const int ch = sub + LANES * j;
-        if (ch < nch) {
-            int32_t *e = (int32_t *)&v[j];
+        int32_t *e = (int32_t *)&v[j];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint32_t a = e[q] > lowb ? (uint32_t)(mx - e[q]) : (1u << 30);
-                const uint32_t ex = shift_exp_mag(a, c.se);
-                e[q] = (int32_t)ex;
-                sum += ex;
-            }
+        for (int q = 0; q < 4; ++q) {
+            const uint32_t a = min((uint32_t)mx - (uint32_t)e[q], 1u << 30);
+            const uint32_t ex = shift_exp_mag_q<FASTQ>(a, c.se);
+            e[q] = (int32_t)ex;
+            if (ch < nch) sum += ex;
         }
     }
     sum = group_sum_u64<LANES>(sum);
@@ -150,14 +150,22 @@ __global__ void __launch_bounds__(256) sdshiftgelu_table(const int4 *__restrict_
     extern __shared__ uint8_t tab[];
     for (int i = threadIdx.x; i <= 2 * T; i += blockDim.x) tab[i] = (uint8_t)gelu_idiv(i - T, c);
     __syncthreads();
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+    const uint8_t *t0 = tab + T;
+    auto f = [&](int32_t x) { return x * (int32_t)t0[min(max(x, -T), T)]; };
+    // 4 vectors per thread per step, all loaded before the first lookup (64 bytes in flight)
+    constexpr int U = 4;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    for (; i + (U - 1) * stride < n4; i += U * stride) {
+        int4 v[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) v[u] = __ldcs(X + i + u * stride);
+#pragma unroll
+        for (int u = 0; u < U; ++u) __stcs(Y + i + u * stride, make_int4(f(v[u].x), f(v[u].y), f(v[u].z), f(v[u].w)));
+    }
+    for (; i < n4; i += stride) {
         const int4 v = __ldcs(X + i);
-        int4 o;
-        o.x = v.x * (int32_t)tab[min(max(v.x, -T), T) + T];
-        o.y = v.y * (int32_t)tab[min(max(v.y, -T), T) + T];
-        o.z = v.z * (int32_t)tab[min(max(v.z, -T), T) + T];
-        o.w = v.w * (int32_t)tab[min(max(v.w, -T), T) + T];
-        __stcs(Y + i, o);
+        __stcs(Y + i, make_int4(f(v.x), f(v.y), f(v.z), f(v.w)));
     }
 }
 
@@ -187,127 +195,267 @@ __device__ __forceinline__ uint64_t newton_isqrt_early(uint64_t V, int iters) {
     return r < 1 ? 1 : r;
 }
 
-// Row storage of the multi-row kernel: int16 rows stay packed (two per 32-bit register).
-template <typename TIn> struct Chunk;
-template <> struct Chunk<int16_t> {
-    uint2 w;
-    __device__ __forceinline__ void load(const int16_t *x) { w = __ldcs((const uint2 *)x); }
-    __device__ __forceinline__ void zero() { w = make_uint2(0, 0); }
-    __device__ __forceinline__ int32_t get(int u) const {
-        const uint32_t h = u < 2 ? w.x : w.y;
-        return (u & 1) ? ((int32_t)h >> 16) : ((int32_t)(h << 16) >> 16);
-    }
-};
-template <> struct Chunk<int32_t> {
-    int4 w;
-    __device__ __forceinline__ void load(const int32_t *x) { w = __ldcs((const int4 *)x); }
-    __device__ __forceinline__ void zero() { w = make_int4(0, 0, 0, 0); }
-    __device__ __forceinline__ int32_t get(int u) const { return u == 0 ? w.x : (u == 1 ? w.y : (u == 2 ? w.z : w.w)); }
-};
-template <typename TOut>
-__device__ __forceinline__ void store4(TOut *y, const int32_t (&o)[4]);
-template <>
-__device__ __forceinline__ void store4<int8_t>(int8_t *y, const int32_t (&o)[4]) {
-    *(uint32_t *)y = (uint32_t)(uint8_t)o[0] | ((uint32_t)(uint8_t)o[1] << 8) | ((uint32_t)(uint8_t)o[2] << 16) |
-                     ((uint32_t)(uint8_t)o[3] << 24);
+// floor(V / r) for V < 2^48 and 1 <= r < 2^32 with a quotient below 2^26: a float estimate (relative
+// error < 2^-21, so absolute error < 2^5), one float refinement from the exact 64-bit remainder
+// (error < 1 on a remainder below 2^6 r), and a final +-1 test on the remainder.
+__device__ __forceinline__ uint32_t div_u48_u32(uint64_t V, uint32_t r) {
+    const float rinv = __frcp_rn(__uint2float_rn(r));
+    uint32_t q = __float2uint_rz(__ull2float_rn(V) * rinv);
+    int64_t rem = (int64_t)V - (int64_t)q * r;
+    const int32_t dq = __float2int_rd(__ll2float_rn(rem) * rinv);
+    q += dq;
+    rem -= (int64_t)dq * r;
+    if (rem < 0) --q;
+    else if (rem >= (int64_t)r) ++q;
+    return q;
 }
-template <>
-__device__ __forceinline__ void store4<int16_t>(int16_t *y, const int32_t (&o)[4]) {
-    *(uint2 *)y = make_uint2((uint32_t)(uint16_t)o[0] | ((uint32_t)(uint16_t)o[1] << 16),
-                             (uint32_t)(uint16_t)o[2] | ((uint32_t)(uint16_t)o[3] << 16));
+// newton_isqrt_early for V < 2^48: the first step from 2^16 is a shift, and every later divisor r
+// is at least isqrt(V) (a floored Newton step from any positive start lands at or above isqrt(V),
+// and the iterates then decrease), so r < 2^32 and V / r < isqrt(V) + 3 < 2^25.
+__device__ __forceinline__ uint64_t newton_isqrt_fast(uint64_t V, int iters) {
+    if (iters <= 0) return 1ull << 16;
+    uint64_t r = ((1ull << 16) + (V >> 16)) >> 1, prev = 1ull << 16;
+    if (r == prev) return r;
+    for (int it = 1; it < iters; ++it) {
+        if (r == 0) break;
+        const uint64_t nx = (r + div_u48_u32(V, (uint32_t)r)) >> 1;
+        if (nx == r) break;
+        if (nx == prev) {
+            r = ((iters - it - 1) & 1) ? r : nx;
+            break;
+        }
+        prev = r;
+        r = nx;
+    }
+    return r < 1 ? 1 : r;
 }
 
-// Sums R per-lane partials (one per row) over the warp so that lane l ends with the total of row
-// l % R: log2 R exchange steps each hand half of the rows to the partner lane (R - 1 shuffles),
-// then 5 - log2 R ordinary butterfly steps.
-template <int R, typename T>
-__device__ __forceinline__ T rows_reduce(T (&v)[R], int lane) {
-#pragma unroll
-    for (int o = 1, n = R; o < R; o <<= 1, n >>= 1) {
-        const bool up = (lane & o) != 0;
-#pragma unroll
-        for (int i = 0; i < n / 2; ++i) {
-            const T keep = up ? v[2 * i + 1] : v[2 * i];
-            const T send = up ? v[2 * i] : v[2 * i + 1];
-            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-        }
-    }
-#pragma unroll
-    for (int o = R; o < 32; o <<= 1) v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
-    return v[0];
+// I-LayerNorm over tiles of LN_RB rows (Sec. 3.3; mean, variance, Newton's
+// integer square root, F = floor((2^31 - 1) / R), n = (y F) >> 1, out = sat(rq(n + beta; m, s))):
+//  (1) cp.async copies the tile into shared memory, rows padded by 16 bytes; the CTAs are
+//      persistent and double-buffered, so the next tile streams in while one is processed;
+//  (2) each warp sums slices of the columns of all the tile's rows, one row per lane (sum x, sum x^2 in
+//      int64; the padded pitch keeps the lanes' 16-byte reads on distinct banks);
+//  (3) warp 0 finishes the statistics, one row per lane: the Newton sequences of the tile run
+//      side by side instead of once per warp;
+//  (4) each thread owns 4 fixed columns (beta, m, s in registers) and normalises one 4-element
+//      group of a row per pass, with coalesced stores.
+// 32-bit arithmetic in (4) is exact: after at least one Newton step R >= isqrt(V) >= |y| for every
+// y = x - mu of the row (a floored Newton step from any positive start lands at or above isqrt(V)),
+// so |y F| <= |y| (2^31 - 1) / R < 2^31; with |beta| <= 2^30, n + beta fits int32 and for s >= 33 the
+// requantisation takes the high-word form.  Rows or columns outside those conditions use the
+// 64-bit formulas.
+
+// acc += a * b with a 64-bit accumulator in one wide multiply-add
+__device__ __forceinline__ void madw(int64_t &acc, int32_t a, int32_t b) {
+    asm("mad.wide.s32 %0, %1, %2, %0;" : "+l"(acc) : "r"(a), "r"(b));
 }
 
-// ROWS rows per warp, held in registers.  Each lane owns 4-element chunks (lane + 32 j) of every
-// row; all loads of the warp's rows are issued before any reduction.  Lane l then holds the sums
-// of row l % ROWS and runs Newton's iteration for it, so a warp pays for one Newton sequence per
-// ROWS rows.  V = sum (x - mu)^2 = sum x^2 - 2 mu sum x + C mu^2, exactly.
-template <typename TIn, typename TOut, int NCH, int ROWS>
-__global__ void __launch_bounds__(256) layernorm_multi(const LnParams p) {
-    const int lane = threadIdx.x & 31;
-    const int64_t row0 = ((int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5)) * ROWS;
-    if (row0 >= p.rows) return;
-    const int C = p.C, nchunk = C >> 2;
-    Chunk<TIn> v[ROWS][NCH];
-#pragma unroll
-    for (int r = 0; r < ROWS; ++r) {
-        const bool ok = row0 + r < p.rows;
-        const TIn *x = (const TIn *)p.X + (ok ? row0 + r : row0) * p.ldx;
-#pragma unroll
-        for (int j = 0; j < NCH; ++j) {
-            const int ch = lane + 32 * j;
-            if (ok && ch < nchunk) v[r][j].load(x + 4 * ch);
-            else v[r][j].zero();
-        }
+struct LnRowStat {
+    int64_t mu, F;
+    int32_t fast;
+    int32_t mF;  // -mu * F in wrapping 32-bit arithmetic: (x F + mF) = (x - mu) F exactly when that fits int32
+};
+
+template <typename TIn>
+__device__ __forceinline__ void ln_get4(const uint8_t *p, int32_t (&x)[4]) {
+    if (sizeof(TIn) == 4) {
+        const int4 v = *(const int4 *)p;
+        x[0] = v.x; x[1] = v.y; x[2] = v.z; x[3] = v.w;
+    } else {
+        const uint2 v = *(const uint2 *)p;
+        x[0] = (int32_t)(v.x << 16) >> 16; x[1] = (int32_t)v.x >> 16;
+        x[2] = (int32_t)(v.y << 16) >> 16; x[3] = (int32_t)v.y >> 16;
     }
-    int64_t ps[ROWS], pq[ROWS];
-#pragma unroll
-    for (int r = 0; r < ROWS; ++r) {
-        int64_t sr = 0, qr = 0;
-#pragma unroll
-        for (int j = 0; j < NCH; ++j)
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int32_t x = v[r][j].get(u);
-                sr += x;
-                qr += (int64_t)x * x;
+}
+
+template <typename TIn, typename TOut, int LN_RB>
+__global__ void __launch_bounds__(256) layernorm_tile(const LnParams p, int32_t pitch, int64_t ntiles) {
+    extern __shared__ __align__(16) uint8_t ln_smem[];
+    constexpr int EB = sizeof(TIn);
+    const int C = p.C, nc16 = C * EB / 16, nc4 = C / 4;
+    const int T = blockDim.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int nwarps = T >> 5;  // full warps (T >= 128)
+    constexpr int SPW = 32 / LN_RB;  // column slices per warp in (2): lane = slice * LN_RB + row
+    const int nslice = nwarps * SPW;
+    uint8_t *tiles = ln_smem;                                             // [2][LN_RB * pitch]
+    int64_t *part = (int64_t *)(tiles + 2 * LN_RB * pitch);               // [nslice][LN_RB][2]
+    LnRowStat *stat = (LnRowStat *)(part + 2 * LN_RB * nslice);          // [LN_RB]
+
+    // (1) tile t -> shared buffer `buf` with cp.async (one commit group per tile)
+    // T is a multiple of the 16-byte chunks per row (T = nc4 k and nc16 = nc4 EB / 4), so a thread
+    // copies the same chunk column of rows r_c, r_c + T / nc16, ...
+    const int ch_c = tid % nc16, r_c = tid / nc16, r_step = T / nc16;
+    const int64_t ld_bytes = p.ldx * EB;
+    const uint32_t tiles_s = (uint32_t)__cvta_generic_to_shared(tiles);
+    auto issue = [&](int64_t t, int buf) {
+        if (t < ntiles) {
+            const int64_t r0 = t * LN_RB;
+            const int nr = (int)min((int64_t)LN_RB, p.rows - r0);
+            const uint8_t *src = (const uint8_t *)p.X + r0 * ld_bytes + ch_c * 16;
+            const uint32_t dst0 = tiles_s + (uint32_t)(buf * LN_RB * pitch + ch_c * 16);
+            const uint8_t *g = src + r_c * ld_bytes;
+            const int64_t g_step = r_step * ld_bytes;
+            uint32_t dst = dst0 + (uint32_t)(r_c * pitch);
+            const uint32_t d_step = (uint32_t)(r_step * pitch);
+            for (int r = r_c; r < LN_RB; r += r_step, g += g_step, dst += d_step) {
+                const bool ok = r < nr;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(ok ? g : src),
+                             "r"(ok ? 16 : 0)
+                             : "memory");
             }
-        ps[r] = sr;
-        pq[r] = qr;
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    int64_t t = blockIdx.x;
+    issue(t, 0);
+    // this thread's 4 columns and their parameters, fetched while the first copies are in flight
+    const int cc = tid % nc4, rs = tid / nc4, kpass = T / nc4;
+    int32_t be[4], mm[4], ss[4];
+    {
+        const int4 b4 = __ldg((const int4 *)(p.beta + 4 * cc)), m4 = __ldg((const int4 *)(p.mult + 4 * cc)),
+                   s4 = __ldg((const int4 *)(p.shift + 4 * cc));
+        be[0] = b4.x; be[1] = b4.y; be[2] = b4.z; be[3] = b4.w;
+        mm[0] = m4.x; mm[1] = m4.y; mm[2] = m4.z; mm[3] = m4.w;
+        ss[0] = s4.x; ss[1] = s4.y; ss[2] = s4.z; ss[3] = s4.w;
     }
-    const int64_t my_s = rows_reduce<ROWS>(ps, lane), my_q = rows_reduce<ROWS>(pq, lane);
-    // lane l: mean, variance and Newton for row l % ROWS
-    const int64_t den = 2 * (int64_t)C, num = 2 * my_s + C;
-    int64_t mu = num / den;
-    if ((num % den) != 0 && num < 0) mu -= 1;
-    const uint64_t V = (uint64_t)(my_q - 2 * mu * my_s + (int64_t)C * mu * mu);
-    const uint64_t R = newton_isqrt_early(V, p.iters);
-    const int64_t F = R < (1ull << 32) ? (int64_t)(0x7fffffffu / (uint32_t)R) : 0;
+    bool col_fast = true;
 #pragma unroll
-    for (int r = 0; r < ROWS; ++r) {
-        if (row0 + r >= p.rows) break;
-        const int64_t mur = __shfl_sync(0xffffffffu, mu, r);
-        const int64_t Fr = __shfl_sync(0xffffffffu, F, r);
-        TOut *yo = (TOut *)p.Y + (row0 + r) * p.ldy;
+    for (int u = 0; u < 4; ++u) col_fast &= ss[u] >= 33 && be[u] >= -(1 << 30) && be[u] <= (1 << 30);
+    int32_t rnd[4], sh[4];  // rq_hi constants of the 4 columns (used only when every shift is >= 33)
 #pragma unroll
-        for (int j = 0; j < NCH; ++j) {
-            const int ch = lane + 32 * j;
-            if (ch < nchunk) {
-                const int4 be = __ldg((const int4 *)(p.beta + 4 * ch));
-                const int4 mu4 = __ldg((const int4 *)(p.mult + 4 * ch));
-                const int4 sh4 = __ldg((const int4 *)(p.shift + 4 * ch));
-                const int32_t bb[4] = {be.x, be.y, be.z, be.w}, mm[4] = {mu4.x, mu4.y, mu4.z, mu4.w},
-                              ss[4] = {sh4.x, sh4.y, sh4.z, sh4.w};
-                int32_t o[4];
+    for (int u = 0; u < 4; ++u) {
+        rnd[u] = col_fast ? 1 << (ss[u] - 33) : 0;
+        sh[u] = ss[u] - 32;
+    }
+    // uniform over the CTA, so that (4) branches once per tile instead of predicating both forms
+    const bool cols_fast = __syncthreads_and(col_fast) != 0;
+    __shared__ int tile_fast;
+
+    for (int buf = 0; t < ntiles; t += gridDim.x, buf ^= 1) {
+        issue(t + gridDim.x, buf ^ 1);  // the next tile streams in while this one is processed
+        asm volatile("cp.async.wait_group 1;" ::: "memory");
+        __syncthreads();
+        const uint8_t *tile = tiles + buf * LN_RB * pitch;
+        const int64_t row0 = t * LN_RB;
+        const int nrows = (int)min((int64_t)LN_RB, p.rows - row0);
+
+        // (2) column slice `sl` of row `rr`
+        {
+            const int rr = lane % LN_RB, sl = warp * SPW + lane / LN_RB;
+            const int per = (nc16 + nslice - 1) / nslice;
+            const int c0 = sl * per, c1 = min(nc16, c0 + per);
+            int64_t sx = 0, sq = 0;
+            if (warp < nwarps) {
+                const uint8_t *rp = tile + rr * pitch;
+                for (int ch = c0; ch < c1; ++ch) {
+                    const int4 v = *(const int4 *)(rp + ch * 16);
+                    if (EB == 4) {
+                        madw(sx, v.x, 1); madw(sx, v.y, 1); madw(sx, v.z, 1); madw(sx, v.w, 1);
+                        madw(sq, v.x, v.x); madw(sq, v.y, v.y); madw(sq, v.z, v.z); madw(sq, v.w, v.w);
+                    } else {
+                        const uint32_t w[4] = {(uint32_t)v.x, (uint32_t)v.y, (uint32_t)v.z, (uint32_t)v.w};
+                        int32_t s32 = 0;
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const int32_t lo = (int32_t)(w[u] << 16) >> 16, hi = (int32_t)w[u] >> 16;
+                            s32 += lo + hi;
+                            sq += (int64_t)((uint32_t)(lo * lo) + (uint32_t)(hi * hi));  // <= 2^31
+                        }
+                        sx += s32;
+                    }
+                }
+                part[(sl * LN_RB + rr) * 2] = sx;
+                part[(sl * LN_RB + rr) * 2 + 1] = sq;
+            }
+        }
+        __syncthreads();
+
+        // (3) statistics of row `lane`, Newton's iteration side by side for the tile's rows (lanes
+        // past the tile's rows compute a dummy row)
+        if (warp == 0) {
+            const int lr = lane % LN_RB;
+            int64_t S = 0, Q = 0;
+            for (int w = 0; w < nslice; ++w) {
+                S += part[(w * LN_RB + lr) * 2];
+                Q += part[(w * LN_RB + lr) * 2 + 1];
+            }
+            const int64_t num = 2 * S + C, den = 2 * (int64_t)C;
+            int64_t mu;
+            if (num >= -(1ll << 31) && num < (1ll << 31)) {  // 32-bit floor division
+                const int32_t n32 = (int32_t)num, d32 = (int32_t)den;
+                const int32_t qt = n32 / d32;
+                mu = qt - ((n32 % d32 != 0 && n32 < 0) ? 1 : 0);
+            } else {
+                mu = num / den;
+                if ((num % den) != 0 && num < 0) mu -= 1;  // floor
+            }
+            const uint64_t V = (uint64_t)(Q - 2 * mu * S + (int64_t)C * mu * mu);
+            const uint64_t R = V < (1ull << 48) ? newton_isqrt_fast(V, p.iters) : newton_isqrt_early(V, p.iters);
+            LnRowStat st;
+            st.mu = mu;
+            st.F = R < (1ull << 32) ? (int64_t)div_int31((uint32_t)R) : 0;
+            st.fast = (p.iters >= 1 || V < (1ull << 32)) ? 1 : 0;
+            st.mF = (int32_t)(0u - (uint32_t)mu * (uint32_t)st.F);
+            if (lane < LN_RB) stat[lane] = st;
+            const bool all_fast = __all_sync(0xffffffffu, st.fast != 0);
+            if (lane == 0) tile_fast = all_fast ? 1 : 0;
+        }
+        __syncthreads();
+
+        // (4) normalise: rows rs, rs + kpass, ... of this thread's column group
+        TOut *ybase = (TOut *)p.Y + row0 * p.ldy + 4 * cc;
+        auto store = [&](int r, const int32_t (&o)[4]) {
+            TOut *y = ybase + (int64_t)r * p.ldy;
+            if (sizeof(TOut) == 1)
+                *(uint32_t *)y = (uint32_t)(uint8_t)o[0] | ((uint32_t)(uint8_t)o[1] << 8) |
+                                 ((uint32_t)(uint8_t)o[2] << 16) | ((uint32_t)(uint8_t)o[3] << 24);
+            else
+                *(uint2 *)y = make_uint2((uint32_t)(uint16_t)o[0] | ((uint32_t)(uint16_t)o[1] << 16),
+                                         (uint32_t)(uint16_t)o[2] | ((uint32_t)(uint16_t)o[3] << 16));
+        };
+        if (tile_fast && cols_fast) {
+            // (x - mu) F = x F + mF in wrapping 32-bit arithmetic (the product fits int32), and
+            // rq takes its high-word form with the rounding constant folded in
+            for (int r = rs; r < nrows; r += kpass) {
+                const int32_t F = (int32_t)stat[r].F, mF = stat[r].mF;
+                int32_t x[4], o[4];
+                ln_get4<TIn>(tile + r * pitch + cc * 4 * EB, x);
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const int64_t n = (((int64_t)v[r][j].get(u) - mur) * Fr) >> 1;
-                    const int64_t t = rq(n + bb[u], mm[u], ss[u]);
-                    o[u] = sizeof(TOut) == 1 ? sat8(t) : sat16(t);
+                    const int32_t n = (int32_t)((uint32_t)x[u] * (uint32_t)F + (uint32_t)mF) >> 1;
+                    const int32_t tq = rq_hi(n + be[u], mm[u], rnd[u], sh[u]);
+                    o[u] = sizeof(TOut) == 1 ? clamp8(tq) : clamp16(tq);
                 }
-                store4<TOut>(yo + 4 * ch, o);
+                store(r, o);
+            }
+        } else {
+            for (int r = rs; r < nrows; r += kpass) {
+                const LnRowStat st = stat[r];
+                int32_t x[4], o[4];
+                ln_get4<TIn>(tile + r * pitch + cc * 4 * EB, x);
+                if (st.fast && col_fast) {
+                    const int32_t mu = (int32_t)st.mu, F = (int32_t)st.F;
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int32_t n = ((x[u] - mu) * F) >> 1;
+                        const int32_t tq = rq_hi1(n + be[u], mm[u], ss[u] - 33);
+                        o[u] = sizeof(TOut) == 1 ? clamp8(tq) : clamp16(tq);
+                    }
+                } else {
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int64_t n = (((int64_t)x[u] - st.mu) * st.F) >> 1;
+                        const int64_t tq = rq(n + be[u], mm[u], ss[u]);
+                        o[u] = sizeof(TOut) == 1 ? sat8(tq) : sat16(tq);
+                    }
+                }
+                store(r, o);
             }
         }
+        __syncthreads();  // buffer `buf` and the statistics are free again
     }
+    asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
 template <typename TIn, typename TOut, int EPL>
@@ -359,15 +507,38 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const LnParams p) {
 template <typename TIn, typename TOut>
 cudaError_t ln_dispatch(const LnParams &p, cudaStream_t s) {
     const int eb = sizeof(TIn), ob = sizeof(TOut);
-    const bool vec = p.C % 4 == 0 && p.ldx % 4 == 0 && p.ldy % 4 == 0 && ((uintptr_t)p.X % (4 * eb)) == 0 &&
-                     ((uintptr_t)p.Y % (4 * ob)) == 0 && (((uintptr_t)p.beta | (uintptr_t)p.mult | (uintptr_t)p.shift) % 16) == 0;
-    if (vec && p.C <= 512) {  // several rows per warp in registers, vector loads, lane-parallel Newton
-        constexpr int ROWS = sizeof(TIn) == 2 ? 8 : 4;
-        dim3 g4((unsigned)((p.rows + 8 * ROWS - 1) / (8 * ROWS)));
-        if (p.C <= 128) layernorm_multi<TIn, TOut, 1, ROWS><<<g4, 256, 0, s>>>(p);
-        else if (p.C <= 256) layernorm_multi<TIn, TOut, 2, ROWS><<<g4, 256, 0, s>>>(p);
-        else if (p.C <= 384) layernorm_multi<TIn, TOut, 3, ROWS><<<g4, 256, 0, s>>>(p);
-        else layernorm_multi<TIn, TOut, 4, ROWS><<<g4, 256, 0, s>>>(p);
+    const bool tiled = p.C % 4 == 0 && (p.C * eb) % 16 == 0 && (p.ldx * eb) % 16 == 0 && p.ldy % 4 == 0 &&
+                       ((uintptr_t)p.X % 16) == 0 && ((uintptr_t)p.Y % (4 * ob)) == 0 &&
+                       (((uintptr_t)p.beta | (uintptr_t)p.mult | (uintptr_t)p.shift) % 16) == 0 && p.C * eb <= 2048;
+    if (tiled) {
+        constexpr int RB = 16;  // rows per tile
+        const int nc4 = p.C / 4, T = nc4 * (256 / nc4);
+        const int pitch = p.C * eb + 16;
+        const size_t smem =
+            (size_t)2 * RB * pitch + 2 * RB * (T / 32) * (32 / RB) * sizeof(int64_t) + RB * sizeof(LnRowStat);
+        static std::once_flag once;
+        static cudaError_t attr = cudaSuccess;
+        std::call_once(once, [] {
+            attr = cudaFuncSetAttribute(layernorm_tile<TIn, TOut, RB>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+        });
+        if (attr != cudaSuccess) return attr;
+        // persistent CTAs: as many as fit on the GPU at once, each striding over the tiles
+        static thread_local int last_T = -1, last_per_sm = 0, sms = 0;
+        static thread_local size_t last_smem = 0;
+        if (T != last_T || smem != last_smem) {
+            int dev = 0;
+            cudaError_t e = cudaGetDevice(&dev);
+            if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            if (e == cudaSuccess)
+                e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&last_per_sm, layernorm_tile<TIn, TOut, RB>, T, smem);
+            if (e != cudaSuccess) return e;
+            last_T = T;
+            last_smem = smem;
+        }
+        const int per_sm = last_per_sm;
+        const int64_t ntiles = (p.rows + RB - 1) / RB;
+        const int64_t grid = min(ntiles, (int64_t)max(per_sm, 1) * sms);
+        layernorm_tile<TIn, TOut, RB><<<(unsigned)grid, T, smem, s>>>(p, pitch, ntiles);
         return cudaGetLastError();
     }
     const int rows_per_block = 8;
@@ -391,12 +562,19 @@ cudaError_t launch_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, in
     dim3 grid2((unsigned)((rows + 15) / 16));
     bool vec = (len % 4 == 0) && (ldx % 4 == 0) && (ldp % 4 == 0) && (((uintptr_t)X & 15) == 0) &&
                (((uintptr_t)P & 3) == 0);
-    if (vec && len <= 64) shiftmax_rows_vec<1, 16><<<grid2, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 128) shiftmax_rows_vec<1, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 512) shiftmax_rows_vec<4, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 1024) shiftmax_rows_vec<8, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 1664) shiftmax_rows_vec<13, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
-    else if (vec && len <= 2048) shiftmax_rows_vec<16, 32><<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
+    const bool fq = c.se.m32 != 0;
+    // rows per CTA: 8 warps x (32 / LANES) rows
+    auto g = [&](int lanes) { return dim3((unsigned)((rows + 8 * (32 / lanes) - 1) / (8 * (32 / lanes)))); };
+#define ILW_SMX(NCH, LANES)                                                                                  \
+    (fq ? (shiftmax_rows_vec<NCH, LANES, true><<<g(LANES), 256, 0, s>>>(X, ldx, rows, len, c, P, ldp), 0)   \
+        : (shiftmax_rows_vec<NCH, LANES, false><<<g(LANES), 256, 0, s>>>(X, ldx, rows, len, c, P, ldp), 0))
+    if (vec && len <= 64) ILW_SMX(4, 4);
+    else if (vec && len <= 128) ILW_SMX(4, 8);
+    else if (vec && len <= 416) ILW_SMX(13, 8);
+    else if (vec && len <= 1024) ILW_SMX(8, 32);
+    else if (vec && len <= 1664) ILW_SMX(13, 32);
+    else if (vec && len <= 2048) ILW_SMX(16, 32);
+#undef ILW_SMX
     else shiftmax_rows_generic<<<grid, 256, 0, s>>>(X, ldx, rows, len, c, P, ldp);
     return cudaGetLastError();
 }
@@ -421,7 +599,7 @@ cudaError_t launch_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const Ge
             cudaGetDevice(&dev);
             cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
             int64_t blocks = (n4 + 255) / 256;
-            if (blocks > 3 * sms) blocks = 3 * sms;
+            if (blocks > 6 * sms) blocks = 6 * sms;
             sdshiftgelu_table<<<(unsigned)blocks, 256, smem, s>>>((const int4 *)X, (int4 *)Y, n4, c, T);
         } else if (n4) {
             int64_t blocks = (n4 + 255) / 256;

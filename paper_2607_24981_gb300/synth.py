@@ -166,6 +166,90 @@ CONFIGS = {
 }
 
 
+# Full integer detector (640x640, batch 16): the Medium backbone with its four output layers
+# tapped, a split-convolution projector at strides 8 / 16 / 32 (80x80, 40x40, 20x20 maps of 256
+# channels, concatenated as the decoder memory), and 3 decoder layers of 300 queries, dim 256,
+# 8 heads, 4 sampling points per level, MLP 1024.
+CONFIGS["detector_c4"] = dict(B=16, backbone="medium_c2", taps=(2, 4, 5, 9), grid=40,
+                              levels=((80, 80), (40, 40), (20, 20)), N=256, Q=300, Hd=8, Fd=1024,
+                              P=4, dec_layers=3)
+
+
+def _mult(seed: int, name: str) -> int:
+    return int(uniform_int(seed, name, (1,), 1 << 30, (1 << 31) - 1)[0])
+
+
+def projector_params(seed: int, nb: int, K: int, N: int = 256, levels: int = 3,
+                     sigma_tap: float = 600.0) -> dict:
+    """Tap requantisation (one per-tensor scale per tapped layer, 2^(b) apart so the branches
+    really differ) and, per level, one split convolution: branch weights int8 [N, K], per-branch
+    dyadic rescale to the largest branch scale (ratio <= 1), bias and per-channel output rq."""
+    pp: dict = {"taps": [], "levels": []}
+    s_tap = [_shift_for(sigma_tap, 40.0) + b for b in range(nb)]  # branch b: scale 2^b larger
+    for b in range(nb):
+        pp["taps"].append((_mult(seed, f"prj.t{b}.m"), s_tap[b]))
+    s_max = max(s_tap)
+    for l in range(levels):
+        lv = {"w": [], "m_b": [], "s_b": []}
+        for b in range(nb):
+            W = uniform_int(seed, f"prj.l{l}.w{b}", (N, K), -127, 127, np.int8)
+            lv["w"].append(W)
+            lv["m_b"].append(_mult(seed, f"prj.l{l}.mb{b}"))
+            lv["s_b"].append(31 + (s_max - s_tap[b]))  # m_b / 2^s_b in [2^-1, 1) * 2^(s_b' - s_max)
+        # each branch contributes ~ sqrt(K) * 40 * SIGMA_W, the largest-scale branch fully
+        lv["b"] = uniform_int(seed, f"prj.l{l}.b", (N,), -(1 << 15), 1 << 15, np.int32)
+        lv["m"] = uniform_int(seed, f"prj.l{l}.m", (N,), 1 << 30, (1 << 31) - 1, np.int32)
+        lv["s"] = np.full((N,), _shift_for(40.0 * SIGMA_W * math.sqrt(K) * 1.2, 40.0), dtype=np.int32)
+        pp["levels"].append(lv)
+    return pp
+
+
+def decoder_params(seed: int, layer: int, d: int = 256, H: int = 8, F: int = 1024, L: int = 3,
+                   P: int = 4, sigma_t: float = 2048.0) -> dict:
+    """All integer parameters of one decoder layer (post-norm self-attention, nearest-neighbour
+    deformable cross-attention, FFN with SD-ShiftGELU; I-LayerNorm with 20 Newton steps and int16
+    outputs of std ~ sigma_t)."""
+    p = f"D{layer}."
+    dp: dict = {"d": d, "H": H, "F": F, "L": L, "P": P, "ln_iters": 20}
+    s_in = _shift_for(sigma_t, 32.0)  # int16 residual stream -> int8 layer input
+    for k in ("q1", "q2", "v1", "c1", "c2", "f"):
+        dp["m_" + k] = _mult(seed, p + k + ".m")
+        dp["s_" + k] = s_in + (1 if k in ("q1", "q2", "c1", "c2") else 0)  # two terms: half each
+    dp["w_qk"], dp["b_qk"], dp["m_qk"], dp["s_qk"] = gemm_params(seed, p + "qk", 2 * d, d, 32.0, 40.0)
+    dp["w_v"], dp["b_v"], dp["m_v"], dp["s_v"] = gemm_params(seed, p + "v", d, d, 32.0, 40.0)
+    I0_s = int(uniform_int(seed, p + "smx.I0", (1,), 1 << 12, 1 << 14)[0])
+    dp["smx"] = {"I0": I0_s, "k_inter": 16, "k_out": 8, "s_d": -1, "m_p": 4, "M_hw": 31}
+    dp["m_o"], dp["s_o"] = _mult(seed, p + "o.m"), _shift_for(128.0 * 40.0, 32.0)
+    dp["w_o"], dp["b_o"], dp["m_oc"], dp["s_oc"] = gemm_params(seed, p + "out", d, d, 32.0, sigma_t / 2)
+    dp["m_r1"], dp["s_r1"] = _mult(seed, p + "r1.m"), 31
+    for i in (1, 2, 3):
+        dp[f"ln{i}_beta"], dp[f"ln{i}_mult"], dp[f"ln{i}_shift"] = ln_params(seed, p + f"ln{i}", d, target=sigma_t)
+    dp["w_val"], dp["b_val"], dp["m_val"], dp["s_val"] = gemm_params(seed, p + "val", d, d, 40.0, 40.0)
+    # sampling offsets in Q8 pixels (std ~ 2 pixels) and attention logits (std ~ 2 I0_w)
+    dp["w_off"], dp["b_off"], dp["m_off"], dp["s_off"] = gemm_params(seed, p + "off", H * L * P * 2, d, 32.0, 512.0)
+    I0_w = int(uniform_int(seed, p + "smxw.I0", (1,), 1 << 6, 1 << 8)[0])
+    dp["w_att"], dp["b_att"], dp["m_att"], dp["s_att"] = gemm_params(seed, p + "att", H * L * P, d, 32.0, 2.0 * I0_w)
+    dp["smx_w"] = {"I0": I0_w, "k_inter": 16, "k_out": 8, "s_d": -1, "m_p": 4, "M_hw": 31}
+    dp["m_s"], dp["s_s"] = _mult(seed, p + "s.m"), _shift_for(128.0 * 40.0 / 2.0, 32.0)
+    dp["w_o2"], dp["b_o2"], dp["m_o2"], dp["s_o2"] = gemm_params(seed, p + "out2", d, d, 32.0, sigma_t / 2)
+    dp["m_r2"], dp["s_r2"] = _mult(seed, p + "r2.m"), 31
+    I0_g = int(uniform_int(seed, p + "gelu.I0", (1,), 1 << 9, 1 << 11)[0])
+    dp["w_fc1"], dp["b_fc1"], dp["m_fc1"], dp["s_fc1"] = gemm_params(seed, p + "fc1", F, d, 32.0, 2.0 * I0_g)
+    dp["gelu_I0"], dp["gelu_k_inter"], dp["gelu_k_out"] = I0_g, 16, 8
+    dp["m_g"], dp["s_g"] = _mult(seed, p + "g.m"), _shift_for(2.0 * I0_g * 64.0, 32.0)
+    dp["w_fc2"], dp["b_fc2"], dp["m_fc2"], dp["s_fc2"] = gemm_params(seed, p + "fc2", d, F, 40.0, sigma_t / 2)
+    dp["m_r3"], dp["s_r3"] = _mult(seed, p + "r3.m"), 31
+    return dp
+
+
+def decoder_inputs(seed: int, B: int, Q: int, d: int = 256) -> dict:
+    """Initial queries tgt and positional queries pos (int16 [B*Q, d], uniform in +-2^11) and the
+    reference points (x, y) in Q16 of the map, fixed across the decoder layers."""
+    return {"tgt": uniform_int(seed, "dec.tgt", (B * Q, d), -(1 << 11), 1 << 11, np.int16),
+            "pos": uniform_int(seed, "dec.pos", (B * Q, d), -(1 << 11), 1 << 11, np.int16),
+            "refs": uniform_int(seed, "dec.refs", (B, Q, 2), 0, (1 << 16) - 1, np.int32)}
+
+
 def image_input(seed: int, B: int, H: int = 640, W: int = 640) -> np.ndarray:
     """int8 image [B, 3, H, W], uniform in [-127, 127]."""
     return uniform_int(seed, "img", (B, 3, H, W), -127, 127, np.int8)

@@ -27,7 +27,8 @@ def test_header_declares_the_paths_entry_points():
     syms = declared_symbols()
     for name in ("ilwdetr_gemm_requant", "ilwdetr_shiftmax_attn", "ilwdetr_sdshiftgelu",
                  "ilwdetr_int_layernorm", "ilwdetr_split_conv", "ilwdetr_deform_attn",
-                 "ilwdetr_block_forward", "ilwdetr_shiftmax_rows"):
+                 "ilwdetr_block_forward", "ilwdetr_shiftmax_rows", "ilwdetr_requant",
+                 "ilwdetr_resample_nearest", "ilwdetr_decoder_layer_forward"):
         assert name in syms
 
 
@@ -73,3 +74,9 @@ def test_host_side_validation_without_gpu(built_lib):
     assert rc == -2  # K % 16 != 0
     assert L.ilwdetr_packed_weight_bytes(3, 32) > 0
     assert L.ilwdetr_block_workspace_bytes(8, 1600, 384, 1536) > 8 * 1600 * 384 * 8
+    assert L.ilwdetr_decoder_workspace_bytes(16, 300, 8400, 256, 1024, 8, 3, 4) > 16 * 8400 * 256
+    rc = L.ilwdetr_requant(ctypes.c_void_p(16), 16, 12, 4, 10, 1 << 30, 30, None, 0, 1, 0, 1, 8,
+                           ctypes.c_void_p(16), 12, None)
+    assert rc == -2  # C % 4 != 0
+    rc = L.ilwdetr_resample_nearest(ctypes.c_void_p(16), 100, 1, 10, 10, 24, ctypes.c_void_p(16), 400, 20, 20, None)
+    assert rc == -2  # C % 16 != 0

@@ -119,3 +119,83 @@ def test_newton_early_exit_matches_fixed_iteration_count():
     for V in Vs:
         for iters in range(0, 21):
             assert _newton_early(V, iters) == _newton_fixed(V, iters), (V, iters)
+
+
+def test_shiftmax_output_from_shiftexp_parts():
+    """Attention forms the Constrained Shiftmax output (I_exp F) >> sh from ShiftExp's parts: with
+    I_exp = I_b << (k - q) and sh = 31 - k_out + 1 + s_d >= k, floor(I_exp F / 2^sh) equals
+    floor(I_b F / 2^(sh - k + q)), and a shift amount of 32 or more gives 0 (PTX shr saturates).
+    Also checked: I_b F < 2^32 under the conditions the host requires (per-row s_d,
+    m_p <= M_hw - 15), with F from the bounds of S_R."""
+    rng = np.random.default_rng(5)
+    k, k_out = 16, 8
+    for s_d in range(0, 16):
+        sh = 31 - k_out + 1 + s_d
+        Ib = rng.integers(1, 1 << 15, size=1 << 16).astype(object)
+        q = rng.integers(0, k + 1, size=Ib.size)
+        F = rng.integers(1, 1 << 15, size=Ib.size).astype(object)
+        lit = [((int(b) << (k - int(qq))) * int(f)) >> sh for b, qq, f in zip(Ib, q, F)]
+        amt = [sh - k + int(qq) for qq in q]
+        direct = [0 if n >= 32 else (((int(b) * int(f)) & 0xFFFFFFFF) >> n) for b, f, n in zip(Ib, F, amt)]
+        assert lit == direct
+    # F bounds: s_d > 0 puts S_R in [2^(M_hw - m_p - 1), 2^31) ; s_d = 0 has S_R >= I0 2^k > I_b 2^k
+    for m_p, M_hw in [(4, 31), (0, 15), (16, 31)]:
+        F_max = (2**31 - 1) // (1 << (M_hw - m_p - 1))
+        assert (2**15 - 1) * F_max < 2**32
+    I0 = np.arange(1, 1 << 15, dtype=object)
+    assert all(int(i) * ((2**31 - 1) // (int(i) << k)) < 2**32 for i in I0[: (1 << 15) >> 1])
+
+
+def _div_u48_u32(V, r):
+    """The kernels' floor(V / r) for V < 2^48, r < 2^32 (quotient < 2^26), in float32 arithmetic:
+    correctly rounded reciprocal, conversions to nearest, truncation / floor back to integers."""
+    f32 = np.float32
+    rinv = f32(1.0) / f32(r)
+    q = np.uint64(np.trunc(f32(float(V)) * rinv))
+    rem = int(V) - int(q) * int(r)
+    dq = int(np.floor(f32(float(rem)) * rinv))
+    q = int(q) + dq
+    rem -= dq * int(r)
+    if rem < 0:
+        q -= 1
+    elif rem >= r:
+        q += 1
+    return q
+
+
+def test_float_assisted_division_in_newton():
+    """I-LayerNorm's Newton steps divide V < 2^48 by r >= isqrt(V) (r < 2^32, quotient < 2^25); the
+    float-estimate division with one refinement and a +-1 test gives floor(V / r) exactly."""
+    import math
+
+    rng = np.random.default_rng(3)
+    cases = []
+    for e in range(1, 48):
+        for _ in range(300):
+            V = int(rng.integers(1 << (e - 1), 1 << e))
+            s = math.isqrt(V)
+            for r in (max(s, 1), s + 1, s + 2, 2 * s + 7, max(1, (1 << 16) + (V >> 16)) >> 1):
+                if 1 <= r < 2**32 and V // r < 2**26:
+                    cases.append((V, r))
+    for V in ((1 << 48) - 1, (1 << 47), 12345678901234):
+        s = math.isqrt(V)
+        cases += [(V, s), (V, s + 1), (V, s - 1 if s > 1 else 1)]
+    for V, r in cases:
+        assert _div_u48_u32(V, r) == V // r, (V, r)
+
+
+def test_high_word_requantisation_forms():
+    """For int32 v, |m| < 2^31 and s in [33, 62] the kernels requantise from the high word of v m:
+    rq(v; m, s) = ((hi >> (s-33)) + 1) >> 1 = (hi + 2^(s-33)) >> (s-32), hi = floor(v m / 2^32)
+    (the second form is one mad.hi plus a shift), against exact rq = floor((v m + 2^(s-1)) / 2^s)."""
+    rng = np.random.default_rng(17)
+    v = np.concatenate([rng.integers(-(2**31), 2**31, 20000), [-(2**31), 2**31 - 1, 0, 1, -1]])
+    m = np.concatenate([rng.integers(-(2**31) + 1, 2**31, 20000), [2**31 - 1, -(2**31) + 1, 2**30, -(2**30), 7]])
+    for s in (33, 34, 40, 47, 51, 62):
+        for vi, mi in zip(v.tolist(), m.tolist()):
+            p = vi * mi
+            exact = (p + (1 << (s - 1))) >> s
+            hi = p >> 32
+            assert ((hi >> (s - 33)) + 1) >> 1 == exact
+            assert (hi + (1 << (s - 33))) >> (s - 32) == exact
+            assert -(2**31) <= hi + (1 << (s - 33)) < 2**31

@@ -568,3 +568,98 @@ def test_patch_embed_is_patch_matmul(orc):
         for c in range(d):
             v = exact_rq(int(acc[i, c]), int(m[c]), int(s[c])) + exact_rq(int(pos[i % T, c]), 3 << 29, 31)
             assert x0[i, c] == max(-32767, min(32767, v))
+
+
+# ---------------------------------------------------------------- detector: requant, resample, decoder
+def test_requant_special_cases(orc):
+    """rq with m = 2^30, s = 30 is the identity and s = 29 doubles; rounding is half up; 8/16-bit
+    outputs saturate symmetrically; the second term broadcasts rows modulo z_rows and adds
+    exactly (Z = X with the same (m, s) doubles the single-term result)."""
+    rng = np.random.default_rng(21)
+    X = rng.integers(-32767, 32768, size=(37, 12)).astype(np.int16)
+    assert np.array_equal(orc.requant(X, 1 << 30, 30, out_bits=32), X.astype(np.int32))
+    assert np.array_equal(orc.requant(X, 1 << 30, 29, out_bits=32), 2 * X.astype(np.int32))
+    half = np.array([[1, -1, 3, -3]], dtype=np.int16)  # x / 2 exactly at .5: rounds up
+    assert np.array_equal(orc.requant(half, 1 << 30, 31, out_bits=32), np.array([[1, 0, 2, -1]]))
+    big = np.array([[1000, -1000, 127, -128]], dtype=np.int16)
+    assert np.array_equal(orc.requant(big, 1 << 30, 30, out_bits=8), np.array([[127, -127, 127, -127]]))
+    assert np.array_equal(orc.requant(np.array([[40000, -40000, 0, 1]], np.int32), 1 << 30, 30, out_bits=16),
+                          np.array([[32767, -32767, 0, 1]]))
+    m, s = 1555555555, 38
+    one = orc.requant(X, m, s, out_bits=32).astype(np.int64)
+    assert np.array_equal(orc.requant(X, m, s, X, m, s, out_bits=32), 2 * one)
+    Z = rng.integers(-32767, 32768, size=(1, 12)).astype(np.int16)
+    zr = orc.requant(np.repeat(Z, 37, axis=0), m, s, out_bits=32).astype(np.int64)
+    assert np.array_equal(orc.requant(X, m, s, Z, m, s, out_bits=32), one + zr)
+
+
+def test_resample_nearest_against_numpy(orc):
+    """Nearest resampling: same size is the identity, 2x upsampling is numpy repeat along both
+    axes, 2x downsampling keeps every second pixel (numpy slicing)."""
+    rng = np.random.default_rng(22)
+    B, Hi, Wi, Cn = 3, 6, 10, 32
+    X = rng.integers(-127, 128, size=(B, Hi, Wi, Cn)).astype(np.int8)
+    flat = X.reshape(B * Hi * Wi, Cn)
+    assert np.array_equal(orc.resample_nearest(flat, B, Hi, Wi, Hi, Wi), flat)
+    up = np.repeat(np.repeat(X, 2, axis=1), 2, axis=2).reshape(-1, Cn)
+    assert np.array_equal(orc.resample_nearest(flat, B, Hi, Wi, 2 * Hi, 2 * Wi), up)
+    down = X[:, ::2, ::2].reshape(-1, Cn)
+    assert np.array_equal(orc.resample_nearest(flat, B, Hi, Wi, Hi // 2, Wi // 2), down)
+
+
+def test_projector_levels_are_resampled_convolutions(orc):
+    """With the same weights at every level, the stride-8 level is the stride-16 level upsampled
+    2x (repeat) and the stride-32 level keeps every second pixel of it: the 1x1 convolution
+    commutes with nearest resampling, and the memory holds the levels image by image."""
+    from paper_2607_24981_gb300 import synth
+
+    B, g, K = 2, 8, 64
+    pp = synth.projector_params(3, 2, K, N=32)
+    for lv in pp["levels"][1:]:
+        for k in ("w", "m_b", "s_b", "b", "m", "s"):
+            lv[k] = pp["levels"][0][k]
+    taps = [synth.uniform_int(4 + i, "tap", (B * g * g, K), -2000, 2000, np.int16) for i in range(2)]
+    levels = ((2 * g, 2 * g), (g, g), (g // 2, g // 2))
+    mem = orc.projector(pp, taps, B, g, levels).reshape(B, -1, 32)
+    s8, s16, s32 = 4 * g * g, g * g, g * g // 4
+    l16 = mem[:, s8:s8 + s16].reshape(B, g, g, 32)
+    assert np.array_equal(mem[:, :s8], np.repeat(np.repeat(l16, 2, 1), 2, 2).reshape(B, s8, 32))
+    assert np.array_equal(mem[:, s8 + s16:], l16[:, ::2, ::2].reshape(B, s32, 32))
+    assert mem.shape[1] == s8 + s16 + s32
+
+
+def _small_decoder(seed=0, B=2, Q=20):
+    from paper_2607_24981_gb300 import synth
+
+    dp = synth.decoder_params(seed, 0, d=64, H=2, F=128, L=2, P=2)
+    inp = synth.decoder_inputs(seed, B, Q, 64)
+    levels = ((8, 8), (4, 4))
+    mem = synth.laplace_int(seed, "mem", (B * 80, 64), 20.0, 127, np.int8)
+    return dp, inp, levels, mem
+
+
+def test_decoder_layer_query_permutation_equivariance(orc):
+    """Every step of a decoder layer treats the queries of an image alike (global self-attention,
+    per-query sampling, per-query FFN and LayerNorm), so permuting the queries (tgt, pos and the
+    reference points together) permutes the output rows the same way."""
+    B, Q = 2, 20
+    dp, inp, levels, mem = _small_decoder(1, B, Q)
+    out = orc.decoder_layer(dp, inp["tgt"], inp["pos"], mem, levels, inp["refs"], B, Q)
+    perm = np.random.default_rng(23).permutation(Q)
+    idx = (np.arange(B)[:, None] * Q + perm[None, :]).reshape(-1)
+    out_p = orc.decoder_layer(dp, inp["tgt"][idx], inp["pos"][idx], mem, levels, inp["refs"][:, perm], B, Q)
+    assert np.array_equal(out_p, out[idx])
+    assert 10 < np.abs(out.astype(np.int64)).mean() < 30000
+
+
+def test_decoder_layer_images_are_independent(orc):
+    """Two images through one call give the same rows as each image alone (the memory, queries
+    and references of an image never meet another image's)."""
+    B, Q = 2, 20
+    dp, inp, levels, mem = _small_decoder(2, B, Q)
+    out = orc.decoder_layer(dp, inp["tgt"], inp["pos"], mem, levels, inp["refs"], B, Q)
+    for b in range(B):
+        r = slice(b * Q, (b + 1) * Q)
+        one = orc.decoder_layer(dp, inp["tgt"][r], inp["pos"][r], mem[b * 80:(b + 1) * 80], levels,
+                                inp["refs"][b:b + 1], 1, Q)
+        assert np.array_equal(one, out[r])
