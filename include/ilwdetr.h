@@ -42,8 +42,9 @@ enum {
 
 /* Activation form code: int8-range integers (|v| <= 127) stored as fp16, which holds them exactly.
  * It is the operand form of the fp16 tensor-core kernels; a producer that writes it saves its
- * consumer the int8 -> fp16 conversion.  Accepted where an argument says so (out_bits of
- * ilwdetr_gemm_requant, qkv_form of ilwdetr_shiftmax_attn); 8 denotes plain int8 there. */
+ * consumer the int8 -> fp16 conversion.  Accepted where an argument says so (out_bits of the
+ * GEMMs and of ilwdetr_int_layernorm, a_form of ilwdetr_gemm, qkv_form and o_form of
+ * ilwdetr_shiftmax_attn, a_form of ilwdetr_patch_embed's internal GEMM); 8 denotes plain int8. */
 #define ILW_I8_IN_F16 108
 
 /* Library version string, e.g. "ilwdetr 0.1 sm_103a". */
@@ -111,6 +112,33 @@ int ilwdetr_gemm_gelu(const int8_t *A, int64_t lda, const void *Wp, const int32_
                       const ilw_gelu_t *gelu, int32_t m_g, int32_t s_g, int8_t *H, int64_t ldh,
                       ilw_stream_t stream);
 
+/* The integer linear layer in its general form: the computation of ilwdetr_gemm_requant
+ * (epilogue ILW_EPI_REQUANT) or of ilwdetr_gemm_gelu (ILW_EPI_GELU), with the activation operand
+ * A either int8 (a_form 8; lda % 16 == 0) or the same int8 values carried in fp16 (a_form
+ * ILW_I8_IN_F16; fp16 [M, lda], lda % 8 == 0), which the tensor cores read directly.  out_bits:
+ * 8 / 16 / 32 / ILW_I8_IN_F16 for ILW_EPI_REQUANT, 8 or ILW_I8_IN_F16 for ILW_EPI_GELU (the int8
+ * outputs carried in fp16).  res: residual term (ILW_EPI_REQUANT, out_bits != 32), or NULL;
+ * gelu, m_g, s_g: ILW_EPI_GELU only.  struct_size = sizeof(ilw_gemm_t). */
+#define ILW_EPI_REQUANT 0
+#define ILW_EPI_GELU 1
+typedef struct {
+    uint32_t struct_size;
+    const void *A;
+    int32_t a_form;
+    int64_t lda;
+    const void *Wp;
+    const int32_t *bias, *mult, *shift;
+    int32_t M, N, K;
+    int32_t epilogue;
+    int32_t out_bits;
+    void *C;
+    int64_t ldc;
+    const ilw_residual_t *res;
+    const ilw_gelu_t *gelu;
+    int32_t m_g, s_g;
+} ilw_gemm_t;
+int ilwdetr_gemm(const ilw_gemm_t *g, ilw_stream_t stream);
+
 /* Scale-preserving split convolution (Sec. 3.2.2, Fig. 2(b)), 1x1 kernels (a per-pixel GEMM):
  *   y[i,c] = sat8(rq( sum_b rq(X_b[i,:] . W_b[c,:]; m_b[b], s_b[b]) + bias[c]; mult[c], shift[c] ))
  * Each branch keeps its own activation scale; (m_b, s_b) is the dyadic ratio S_b / max_b S_b
@@ -157,13 +185,14 @@ int ilwdetr_int_layernorm(const void *X, int32_t in_bits, int64_t ldx, int64_t r
  * Q, K, V: token-major, element (b, t, h, e) at [(b*T + t) * ld_qkv + h*dh + e] (elements), in
  * the form qkv_form: 8 = int8, ILW_I8_IN_F16 = the same integers as fp16 (16-byte aligned rows;
  * q|k|v of one [B*T, 3*H*dh] buffer is the usual case).
- * O: int8, element (b, t, h, e) at [(b*T + t) * ld_o + h*dh + e].
+ * O: element (b, t, h, e) at [(b*T + t) * ld_o + h*dh + e], in the form o_form (8 = int8,
+ * ILW_I8_IN_F16 = the int8 values as fp16).
  * win_side <= 1: global attention over the T tokens; win_side = n >= 2: the sqrt(T) x sqrt(T)
  * token grid (row-major) is cut into n x n windows and tokens attend within their window
  * (LW-DETR's window attention, Table 1).  dh must be 32 or 64. */
 int ilwdetr_shiftmax_attn(const void *Q, const void *K, const void *V, int64_t ld_qkv,
                           int32_t qkv_form, int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side,
-                          const ilw_shiftmax_t *p, int32_t m_o, int32_t s_o, int8_t *O,
+                          const ilw_shiftmax_t *p, int32_t m_o, int32_t s_o, void *O, int32_t o_form,
                           int64_t ld_o, ilw_stream_t stream);
 
 /* Integer deformable-attention sampling with nearest-neighbour lookup (Sec. 3.1.1): for each

@@ -11,7 +11,7 @@ import ctypes as C
 import os
 
 __all__ = [
-    "lib", "IlwError", "I8_IN_F16", "version", "pack_weight", "gemm_requant", "gemm_gelu", "split_conv",
+    "lib", "IlwError", "I8_IN_F16", "version", "pack_weight", "gemm_requant", "gemm_gelu", "gemm", "split_conv",
     "shiftmax_rows", "sdshiftgelu", "int_layernorm", "shiftmax_attn", "deform_attn",
     "BlockWeights", "block_forward", "block_workspace_bytes", "device_status",
     "patch_embed", "patch_embed_workspace_bytes", "Backbone", "Graphed",
@@ -64,6 +64,17 @@ class BlockParamsT(C.Structure):
     ]
 
 
+class GemmT(C.Structure):
+    _fields_ = [("struct_size", C.c_uint32), ("A", C.c_void_p), ("a_form", C.c_int32), ("lda", C.c_int64),
+                ("Wp", C.c_void_p), ("bias", C.c_void_p), ("mult", C.c_void_p), ("shift", C.c_void_p),
+                ("M", C.c_int32), ("N", C.c_int32), ("K", C.c_int32), ("epilogue", C.c_int32),
+                ("out_bits", C.c_int32), ("C", C.c_void_p), ("ldc", C.c_int64),
+                ("res", C.POINTER(ResidualT)), ("gelu", C.POINTER(GeluT)), ("m_g", C.c_int32), ("s_g", C.c_int32)]
+
+
+EPI_REQUANT, EPI_GELU = 0, 1
+
+
 class DecoderParamsT(C.Structure):
     _fields_ = [
         ("struct_size", C.c_uint32),
@@ -114,7 +125,8 @@ SIGNATURES = {
     "ilwdetr_int_layernorm": ([_VP, _I32, _I64, _I64, _I32, _VP, _VP, _VP, _I32, _VP, _I32, _I64,
                                _VP], C.c_int),
     "ilwdetr_shiftmax_attn": ([_VP, _VP, _VP, _I64, _I32, _I32, _I32, _I32, _I32, _I32,
-                               C.POINTER(ShiftmaxT), _I32, _I32, _VP, _I64, _VP], C.c_int),
+                               C.POINTER(ShiftmaxT), _I32, _I32, _VP, _I32, _I64, _VP], C.c_int),
+    "ilwdetr_gemm": ([C.POINTER(GemmT), _VP], C.c_int),
     "ilwdetr_deform_attn": ([_VP, C.POINTER(_I32), _I32, _VP, _VP, _VP, _I32, _I32, _I32, _I32,
                              _I32, _I32, _I32, _VP, _VP], C.c_int),
     "ilwdetr_patch_embed_workspace_bytes": ([_I32, _I32, _I32, _I32, _I32], C.c_size_t),
@@ -213,6 +225,27 @@ def gemm_requant(A, Wp, N, bias, mult, shift, out_bits=8, res=None, m_r=0, s_r=0
     return out
 
 
+def gemm(A, Wp, N, bias, mult, shift, out_bits=8, res=None, m_r=0, s_r=0, gelu: dict | None = None, m_g=0, s_g=1,
+         out=None):
+    """ilwdetr_gemm: A int8 or float16 (the int8 values) [M, K] x packed W [N, K]; epilogue
+    requantisation (with optional residual) or, with ``gelu``, SD-ShiftGELU; out_bits 8 / 16 / 32 /
+    I8_IN_F16."""
+    import torch
+
+    M, K = A.shape
+    dt = {8: torch.int8, 16: torch.int16, 32: torch.int32, I8_IN_F16: torch.float16}[out_bits]
+    if out is None:
+        out = torch.empty((M, N), dtype=dt, device=A.device)
+    r = None if res is None else ResidualT(res.data_ptr(), res.stride(0), res.shape[0], m_r, s_r)
+    g = None if gelu is None else GeluT(gelu["I0"], gelu.get("k_inter", 16), gelu.get("k_out", 8))
+    a_form = I8_IN_F16 if A.dtype == torch.float16 else 8
+    desc = GemmT(C.sizeof(GemmT), A.data_ptr(), a_form, A.stride(0), Wp.data_ptr(), _ptr(bias), _ptr(mult), _ptr(shift),
+                 M, N, K, EPI_GELU if gelu is not None else EPI_REQUANT, out_bits, out.data_ptr(), out.stride(0),
+                 None if r is None else C.pointer(r), None if g is None else C.pointer(g), m_g, s_g)
+    _check(lib().ilwdetr_gemm(C.byref(desc), _stream()), "gemm")
+    return out
+
+
 def gemm_gelu(A, Wp, N, bias, mult, shift, gelu: dict, m_g, s_g, out=None):
     """ilwdetr_gemm_gelu: linear + SD-ShiftGELU epilogue -> int8 [M, N]."""
     import torch
@@ -285,7 +318,7 @@ def int_layernorm(X, beta, mult, shift, iters=10, out_bits=8, out=None):
     rows, Cn = X.shape
     in_bits = {torch.int16: 16, torch.int32: 32}[X.dtype]
     if out is None:
-        out = torch.empty((rows, Cn), dtype=torch.int8 if out_bits == 8 else torch.int16,
+        out = torch.empty((rows, Cn), dtype={8: torch.int8, 16: torch.int16, I8_IN_F16: torch.float16}[out_bits],
                           device=X.device)
     _check(lib().ilwdetr_int_layernorm(_ptr(X), in_bits, X.stride(0), rows, Cn, _ptr(beta),
                                        _ptr(mult), _ptr(shift), iters, _ptr(out), out_bits,
@@ -293,20 +326,21 @@ def int_layernorm(X, beta, mult, shift, iters=10, out_bits=8, out=None):
     return out
 
 
-def shiftmax_attn(qkv, B, T, H, dh, win_side, smx: dict, m_o, s_o, out=None):
+def shiftmax_attn(qkv, B, T, H, dh, win_side, smx: dict, m_o, s_o, out=None, o_f16=False):
     """ilwdetr_shiftmax_attn on a token-major [B*T, 3*H*dh] q|k|v buffer (int8, or float16
-    holding the int8 values) -> int8 [B*T, H*dh]."""
+    holding the int8 values) -> int8 [B*T, H*dh] (float16 holding them with ``o_f16``)."""
     import torch
 
     d = H * dh
     if out is None:
-        out = torch.empty((B * T, d), dtype=torch.int8, device=qkv.device)
+        out = torch.empty((B * T, d), dtype=torch.float16 if o_f16 else torch.int8, device=qkv.device)
     form = I8_IN_F16 if qkv.dtype == torch.float16 else 8
+    o_form = I8_IN_F16 if out.dtype == torch.float16 else 8
     base, es = qkv.data_ptr(), qkv.element_size()
     p = _smx(smx)
     _check(lib().ilwdetr_shiftmax_attn(C.c_void_p(base), C.c_void_p(base + d * es), C.c_void_p(base + 2 * d * es),
                                        qkv.stride(0), form, B, T, H, dh, win_side, C.byref(p), m_o, s_o,
-                                       _ptr(out), out.stride(0), _stream()), "shiftmax_attn")
+                                       _ptr(out), o_form, out.stride(0), _stream()), "shiftmax_attn")
     return out
 
 

@@ -3,8 +3,8 @@
   python -m paper_2607_24981_gb300.cases <case> [--reps N]
 
 Each case builds its seeded inputs (shapes of the paper's Medium model and of the nonlinearity
-sweep), runs the entry point `reps` times after 3 warm-up calls and prints the mean device time
-with the case's algorithmic work.  Cases:
+sweep), runs the entry point `reps` times after 3 warm-up calls, each launch timed with CUDA
+events, and prints the median (and minimum) device time with the case's algorithmic work.  Cases:
   attn_global   attention, 2 images x 1600 tokens, 6 heads, dh 64, global (fp16-carried q|k|v);
                 --batch 8 gives the encoder's launch
   attn_window   attention, 8 images x 1600 tokens, 6 heads, 2x2 windows of 400
@@ -47,27 +47,28 @@ def build(case: str, batch: int = 0):
         win = 0 if case == "attn_global" else 2
         # q|k|v as the QKV GEMM hands them over: the int8 values carried in float16
         qkv = _dev(synth.uniform_int(0, "case.qkv", (B * T, 3 * H * dh), -127, 127, np.int8).astype(np.float16))
-        out = torch.empty((B * T, H * dh), dtype=torch.int8, device="cuda")
+        out = torch.empty((B * T, H * dh), dtype=torch.float16, device="cuda")  # the encoder's O form
         scores = B * H * (T * T if win == 0 else 4 * (T // 4) ** 2)
         return (lambda: ilw.shiftmax_attn(qkv, B, T, H, dh, win, {"I0": 6000}, 3 << 29, 36, out=out),
                 {"scores": scores})
     if case.startswith("gemm"):
         M, d, F = 12800, 384, 1536
         N, K = {"gemm_qkv": (3 * d, d), "gemm_proj": (d, d), "gemm_fc1_gelu": (F, d), "gemm_fc2": (d, F)}[case]
-        A = _dev(synth.uniform_int(1, "case.A", (M, K), -127, 127, np.int8))
+        # the activations as the encoder hands them over: int8 values carried in fp16
+        A = _dev(synth.uniform_int(1, "case.A", (M, K), -127, 127, np.int8).astype(np.float16))
         W, b, m, s = synth.gemm_params(1, "case.W", N, K, 40.0, 40.0)
         Wp = ilw.pack_weight(_dev(W))
         b, m, s = _dev(b), _dev(m), _dev(s)
-        if case == "gemm_fc1_gelu":
-            out = torch.empty((M, N), dtype=torch.int8, device="cuda")
-            fn = lambda: ilw.gemm_gelu(A, Wp, N, b, m, s, {"I0": 1000}, 3 << 29, 40, out=out)
-        elif case == "gemm_qkv":  # q|k|v written as fp16-carried int8, as the encoder block does
+        if case == "gemm_fc1_gelu":  # h written as fp16-carried int8, as the encoder block does
             out = torch.empty((M, N), dtype=torch.float16, device="cuda")
-            fn = lambda: ilw.gemm_requant(A, Wp, N, b, m, s, ilw.I8_IN_F16, out=out)
+            fn = lambda: ilw.gemm(A, Wp, N, b, m, s, ilw.I8_IN_F16, gelu={"I0": 1000}, m_g=3 << 29, s_g=40, out=out)
+        elif case == "gemm_qkv":  # q|k|v written as fp16-carried int8
+            out = torch.empty((M, N), dtype=torch.float16, device="cuda")
+            fn = lambda: ilw.gemm(A, Wp, N, b, m, s, ilw.I8_IN_F16, out=out)
         else:
             res = _dev(synth.uniform_int(1, "case.res", (M, N), -3000, 3000, np.int16))
             out = torch.empty((M, N), dtype=torch.int16, device="cuda")
-            fn = lambda: ilw.gemm_requant(A, Wp, N, b, m, s, 16, res=res, m_r=1 << 30, s_r=31, out=out)
+            fn = lambda: ilw.gemm(A, Wp, N, b, m, s, 16, res=res, m_r=1 << 30, s_r=31, out=out)
         return fn, {"flops": 2.0 * M * N * K}
     if case.startswith("smx"):
         L = int(case.split("_")[1])
@@ -81,15 +82,16 @@ def build(case: str, batch: int = 0):
     if case.startswith("ln"):
         if case == "ln_c2":
             X = _dev(synth.uniform_int(34, "case.ln", (12800, 384), -3000, 3000, np.int16))
-            per = 3.0
+            per = 3.0  # int16 in, int8 out (carried in fp16, the encoder's form)
         else:
             C = int(case.split("_")[1])
             X = _dev(synth.uniform_int(34, f"c3ln{C}", (1 << 20, C), -(1 << 14), 1 << 14))
             per = 5.0
         C = X.shape[1]
         beta, mult, shift = (_dev(a) for a in synth.ln_params(34, f"c3lnp{C}", C))
-        Y = torch.empty(X.shape, dtype=torch.int8, device="cuda")
-        return (lambda: ilw.int_layernorm(X, beta, mult, shift, 10, 8, out=Y)), {"bytes": per * X.numel()}
+        ob = ilw.I8_IN_F16 if case == "ln_c2" else 8
+        Y = torch.empty(X.shape, dtype=torch.float16 if case == "ln_c2" else torch.int8, device="cuda")
+        return (lambda: ilw.int_layernorm(X, beta, mult, shift, 10, ob, out=Y)), {"bytes": per * X.numel()}
     raise SystemExit(f"unknown case {case}")
 
 
@@ -105,14 +107,16 @@ def main(argv=None):
     for _ in range(3):
         fn()
     torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for _ in range(a.reps):
+    # every launch timed on its own (events on the launching stream), median reported
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(max(a.reps, 1))]
+    for e0, e1 in ev:
+        e0.record()
         fn()
-    e1.record()
+        e1.record()
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / max(a.reps, 1)
-    out = {"case": a.case, "us": ms * 1000.0}
+    times = sorted(e0.elapsed_time(e1) for e0, e1 in ev)
+    ms = times[len(times) // 2]
+    out = {"case": a.case, "us": ms * 1000.0, "us_min": times[0] * 1000.0}
     if "flops" in work:
         out["tflops"] = work["flops"] / (ms / 1000.0) / 1e12
     if "bytes" in work:

@@ -114,18 +114,42 @@ int ilwdetr_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, ilw
     return cuda_status(ilw::launch_pack_weight(W, N, K, packed, (cudaStream_t)stream), "pack_weight");
 }
 
-int ilwdetr_gemm_requant(const int8_t *A, int64_t lda, const void *Wp, const int32_t *bias,
-                         const int32_t *mult, const int32_t *shift, int32_t M, int32_t N, int32_t K,
-                         int32_t out_bits, void *C, int64_t ldc, const ilw_residual_t *res,
-                         ilw_stream_t stream) {
-    int rc = gemm_common(A, lda, Wp, M, N, K);
-    if (rc) return rc;
-    if (out_bits != 8 && out_bits != 16 && out_bits != 32 && out_bits != ILW_I8_IN_F16)
+namespace {
+// The common path of the GEMM entry points.
+int gemm_impl(const void *A, int32_t a_form, int64_t lda, const void *Wp, const int32_t *bias, const int32_t *mult,
+              const int32_t *shift, int32_t M, int32_t N, int32_t K, int32_t epilogue, int32_t out_bits, void *C,
+              int64_t ldc, const ilw_residual_t *res, const ilw_gelu_t *gelu, int32_t m_g, int32_t s_g,
+              ilw_stream_t stream, const char *what) {
+    if (a_form != 8 && a_form != ILW_I8_IN_F16)
+        return fail(ILW_ERR_INVALID_ARG, "%s: a_form=%d must be 8 or ILW_I8_IN_F16", what, a_form);
+    int rc;
+    if (a_form == 8) {
+        if ((rc = gemm_common((const int8_t *)A, lda, Wp, M, N, K))) return rc;
+    } else {
+        if (M < 0 || N < 0 || K < 1) return fail(ILW_ERR_INVALID_ARG, "bad GEMM sizes M=%d N=%d K=%d", M, N, K);
+        if (K % 16) return fail(ILW_ERR_UNSUPPORTED, "K=%d must be a multiple of 16", K);
+        if (M == 0 || N == 0) return ILW_OK;
+        if (!A || !Wp) return fail(ILW_ERR_INVALID_ARG, "GEMM operand is NULL");
+        if (lda < K || lda % 8 || !aligned(A, 16))
+            return fail(ILW_ERR_INVALID_ARG, "fp16 A must be 16-byte aligned with lda >= K, lda %% 8 == 0");
+        if (!aligned(Wp, 256)) return fail(ILW_ERR_INVALID_ARG, "packed weight must be 256-byte aligned");
+        if (K > (1 << 20)) return fail(ILW_ERR_UNSUPPORTED, "K too large");
+    }
+    if (epilogue == ILW_EPI_GELU) {
+        if ((rc = check_gelu(gelu))) return rc;
+        if ((rc = check_rq_scalar(s_g, "gelu output"))) return rc;
+        if (out_bits != 8 && out_bits != ILW_I8_IN_F16)
+            return fail(ILW_ERR_INVALID_ARG, "%s: GELU out_bits=%d must be 8 or ILW_I8_IN_F16", what, out_bits);
+    } else if (epilogue != ILW_EPI_REQUANT) {
+        return fail(ILW_ERR_INVALID_ARG, "%s: epilogue=%d unknown", what, epilogue);
+    } else if (out_bits != 8 && out_bits != 16 && out_bits != 32 && out_bits != ILW_I8_IN_F16) {
         return fail(ILW_ERR_INVALID_ARG, "out_bits=%d must be 8, 16, 32 or ILW_I8_IN_F16", out_bits);
+    }
     if (M == 0 || N == 0) return ILW_OK;
     if (!C || ldc < N) return fail(ILW_ERR_INVALID_ARG, "C is NULL or ldc < N");
     if (out_bits != 32 && (!mult || !shift)) return fail(ILW_ERR_INVALID_ARG, "mult/shift are NULL");
-    if (res && out_bits != 32) {
+    const bool use_res = res && epilogue == ILW_EPI_REQUANT && out_bits != 32;
+    if (use_res) {
         if (!res->x || res->rows < 1 || res->ldx < N) return fail(ILW_ERR_INVALID_ARG, "bad residual");
         if ((rc = check_rq_scalar(res->shift, "residual"))) return rc;
     }
@@ -134,51 +158,52 @@ int ilwdetr_gemm_requant(const int8_t *A, int64_t lda, const void *Wp, const int
     gp.N = N;
     gp.nb = 1;
     gp.branch_rq = false;
-    gp.br[0] = {A, lda, ilw::packed_i8(Wp), ilw::packed_f16(Wp, N, K), K, 0, 0};
+    gp.a_f16 = a_form == ILW_I8_IN_F16;
+    gp.br[0] = {(const int8_t *)A, lda, ilw::packed_i8(Wp), ilw::packed_f16(Wp, N, K), K, 0, 0};
     ilw::EpiParams ep{};
-    ep.kind = ilw::EPI_REQUANT;
+    ep.kind = epilogue == ILW_EPI_GELU ? ilw::EPI_GELU : ilw::EPI_REQUANT;
     ep.bias = bias;
     ep.mult = mult;
     ep.shift = shift;
     ep.out_bits = out_bits;
     ep.C = C;
     ep.ldc = ldc;
-    if (res && out_bits != 32) {
+    if (use_res) {
         ep.res = res->x;
         ep.ldr = res->ldx;
         ep.res_rows = res->rows;
         ep.m_r = res->mult;
         ep.s_r = res->shift;
     }
-    return cuda_status(ilw::launch_gemm(gp, ep, (cudaStream_t)stream), "gemm_requant");
+    if (epilogue == ILW_EPI_GELU) {
+        ep.gelu = ilw::make_gelu(*gelu);
+        ep.m_g = m_g;
+        ep.s_g = s_g;
+    }
+    return cuda_status(ilw::launch_gemm(gp, ep, (cudaStream_t)stream), what);
+}
+}  // namespace
+
+int ilwdetr_gemm_requant(const int8_t *A, int64_t lda, const void *Wp, const int32_t *bias,
+                         const int32_t *mult, const int32_t *shift, int32_t M, int32_t N, int32_t K,
+                         int32_t out_bits, void *C, int64_t ldc, const ilw_residual_t *res,
+                         ilw_stream_t stream) {
+    return gemm_impl(A, 8, lda, Wp, bias, mult, shift, M, N, K, ILW_EPI_REQUANT, out_bits, C, ldc, res, nullptr, 0,
+                     0, stream, "gemm_requant");
 }
 
 int ilwdetr_gemm_gelu(const int8_t *A, int64_t lda, const void *Wp, const int32_t *bias,
                       const int32_t *mult, const int32_t *shift, int32_t M, int32_t N, int32_t K,
                       const ilw_gelu_t *gelu, int32_t m_g, int32_t s_g, int8_t *H, int64_t ldh,
                       ilw_stream_t stream) {
-    int rc = gemm_common(A, lda, Wp, M, N, K);
-    if (rc) return rc;
-    if ((rc = check_gelu(gelu))) return rc;
-    if ((rc = check_rq_scalar(s_g, "gelu output"))) return rc;
-    if (M == 0 || N == 0) return ILW_OK;
-    if (!H || ldh < N || !mult || !shift) return fail(ILW_ERR_INVALID_ARG, "gemm_gelu: bad output or NULL mult/shift");
-    ilw::GemmProblem gp{};
-    gp.M = M;
-    gp.N = N;
-    gp.nb = 1;
-    gp.br[0] = {A, lda, ilw::packed_i8(Wp), ilw::packed_f16(Wp, N, K), K, 0, 0};
-    ilw::EpiParams ep{};
-    ep.kind = ilw::EPI_GELU;
-    ep.bias = bias;
-    ep.mult = mult;
-    ep.shift = shift;
-    ep.C = H;
-    ep.ldc = ldh;
-    ep.gelu = ilw::make_gelu(*gelu);
-    ep.m_g = m_g;
-    ep.s_g = s_g;
-    return cuda_status(ilw::launch_gemm(gp, ep, (cudaStream_t)stream), "gemm_gelu");
+    return gemm_impl(A, 8, lda, Wp, bias, mult, shift, M, N, K, ILW_EPI_GELU, 8, H, ldh, nullptr, gelu, m_g, s_g,
+                     stream, "gemm_gelu");
+}
+
+int ilwdetr_gemm(const ilw_gemm_t *g, ilw_stream_t stream) {
+    if (!g || g->struct_size != sizeof(ilw_gemm_t)) return fail(ILW_ERR_INVALID_ARG, "gemm: NULL or struct_size mismatch");
+    return gemm_impl(g->A, g->a_form, g->lda, g->Wp, g->bias, g->mult, g->shift, g->M, g->N, g->K, g->epilogue,
+                     g->out_bits, g->C, g->ldc, g->res, g->gelu, g->m_g, g->s_g, stream, "gemm");
 }
 
 int ilwdetr_split_conv(const int8_t *const *X, const int64_t *ldx, int32_t nb, int32_t M,
@@ -241,7 +266,8 @@ int ilwdetr_int_layernorm(const void *X, int32_t in_bits, int64_t ldx, int64_t r
                           const int32_t *beta, const int32_t *mult, const int32_t *shift,
                           int32_t iters, void *Y, int32_t out_bits, int64_t ldy, ilw_stream_t stream) {
     if (in_bits != 16 && in_bits != 32) return fail(ILW_ERR_INVALID_ARG, "in_bits=%d must be 16 or 32", in_bits);
-    if (out_bits != 8 && out_bits != 16) return fail(ILW_ERR_INVALID_ARG, "out_bits=%d must be 8 or 16", out_bits);
+    if (out_bits != 8 && out_bits != 16 && out_bits != ILW_I8_IN_F16)
+        return fail(ILW_ERR_INVALID_ARG, "out_bits=%d must be 8, 16 or ILW_I8_IN_F16", out_bits);
     if (C < 1 || C > 4096) return fail(ILW_ERR_UNSUPPORTED, "C=%d outside [1, 4096]", C);
     if (rows < 0 || iters < 0 || iters > 64) return fail(ILW_ERR_INVALID_ARG, "bad rows / iters");
     if (rows == 0) return ILW_OK;
@@ -253,7 +279,8 @@ int ilwdetr_int_layernorm(const void *X, int32_t in_bits, int64_t ldx, int64_t r
 
 static int attn_params(ilw::AttnParams &ap, const void *Q, const void *K, const void *V, int64_t ld_qkv,
                        int32_t qkv_form, int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side,
-                       const ilw_shiftmax_t *p, int32_t m_o, int32_t s_o, int8_t *O, int64_t ld_o) {
+                       const ilw_shiftmax_t *p, int32_t m_o, int32_t s_o, void *O, int32_t o_form,
+                       int64_t ld_o) {
     int rc = check_shiftmax(p);
     if (rc) return rc;
     if ((rc = check_rq_scalar(s_o, "attention output"))) return rc;
@@ -266,6 +293,9 @@ static int attn_params(ilw::AttnParams &ap, const void *Q, const void *K, const 
     if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || (ld_qkv * esz) % 16 || ld_qkv < (int64_t)H * dh)
         return fail(ILW_ERR_INVALID_ARG, "attention: q/k/v must be 16-byte aligned with 16-byte aligned rows");
     if (ld_o < (int64_t)H * dh) return fail(ILW_ERR_INVALID_ARG, "attention: ld_o < H*dh");
+    if (o_form != 8 && o_form != ILW_I8_IN_F16)
+        return fail(ILW_ERR_INVALID_ARG, "attention: o_form=%d must be 8 or ILW_I8_IN_F16", o_form);
+    if (o_form == ILW_I8_IN_F16 && !aligned(O, 4)) return fail(ILW_ERR_INVALID_ARG, "attention: fp16 O misaligned");
     ap = {};
     ap.Q = Q; ap.K = K; ap.V = V; ap.ld_qkv = ld_qkv;
     ap.qkv_f16 = qkv_form == ILW_I8_IN_F16 ? 1 : 0;
@@ -281,16 +311,16 @@ static int attn_params(ilw::AttnParams &ap, const void *Q, const void *K, const 
     }
     ap.smx = make_smx(*p);
     ap.m_o = m_o; ap.s_o = s_o;
-    ap.O = O; ap.ld_o = ld_o;
+    ap.O = O; ap.o_f16 = o_form == ILW_I8_IN_F16 ? 1 : 0; ap.ld_o = ld_o;
     return ILW_OK;
 }
 
 int ilwdetr_shiftmax_attn(const void *Q, const void *K, const void *V, int64_t ld_qkv, int32_t qkv_form,
                           int32_t B, int32_t T, int32_t H, int32_t dh, int32_t win_side, const ilw_shiftmax_t *p,
-                          int32_t m_o, int32_t s_o, int8_t *O, int64_t ld_o, ilw_stream_t stream) {
+                          int32_t m_o, int32_t s_o, void *O, int32_t o_form, int64_t ld_o, ilw_stream_t stream) {
     if (B == 0 || T == 0) return ILW_OK;
     ilw::AttnParams ap;
-    int rc = attn_params(ap, Q, K, V, ld_qkv, qkv_form, B, T, H, dh, win_side, p, m_o, s_o, O, ld_o);
+    int rc = attn_params(ap, Q, K, V, ld_qkv, qkv_form, B, T, H, dh, win_side, p, m_o, s_o, O, o_form, ld_o);
     if (rc) return rc;
     return cuda_status(ilw::launch_attention(ap, (cudaStream_t)stream), "shiftmax_attn");
 }
@@ -329,7 +359,7 @@ static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 size_t ilwdetr_patch_embed_workspace_bytes(int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p) {
     if (B < 0 || Cin < 1 || p < 1 || Hh < 0 || Ww < 0) return 0;
-    return align256((size_t)B * (Hh / p) * (Ww / p) * Cin * p * p);
+    return align256((size_t)B * (Hh / p) * (Ww / p) * Cin * p * p * 2);  // patch matrix, fp16-carried int8
 }
 
 int ilwdetr_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
@@ -344,14 +374,12 @@ int ilwdetr_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, i
         workspace_bytes < ilwdetr_patch_embed_workspace_bytes(B, Cin, Hh, Ww, p))
         return fail(ILW_ERR_INVALID_ARG, "patch_embed: workspace too small or misaligned");
     const int32_t T = (Hh / p) * (Ww / p), K = Cin * p * p;
-    int8_t *A = (int8_t *)workspace;
-    cudaError_t e = ilw::launch_patchify(img, B, Cin, Hh, Ww, p, A, (cudaStream_t)stream);
+    __half *A = (__half *)workspace;  // the patch matrix as fp16-carried int8: the GEMM reads it directly
+    cudaError_t e = ilw::launch_patchify_f16(img, B, Cin, Hh, Ww, p, A, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_status(e, "patchify");
-    if (pos) {
-        ilw_residual_t r{pos, d, T, m_pos, s_pos};
-        return ilwdetr_gemm_requant(A, K, Wp, bias, mult, shift, B * T, d, K, 16, x0, d, &r, stream);
-    }
-    return ilwdetr_gemm_requant(A, K, Wp, bias, mult, shift, B * T, d, K, 16, x0, d, nullptr, stream);
+    ilw_residual_t r{pos, d, T, m_pos, s_pos};
+    return gemm_impl(A, ILW_I8_IN_F16, K, Wp, bias, mult, shift, B * T, d, K, ILW_EPI_REQUANT, 16, x0, d,
+                     pos ? &r : nullptr, nullptr, 0, 0, stream, "patch_embed");
 }
 
 // ------------------------------------------------------------------ encoder block
@@ -359,8 +387,9 @@ int ilwdetr_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, i
 size_t ilwdetr_block_workspace_bytes(int32_t B, int32_t T, int32_t d, int32_t F) {
     if (B < 0 || T < 0 || d < 0 || F < 0) return 0;
     size_t M = (size_t)B * T;
-    return align256(M * d) /*a1*/ + align256(M * 3 * d * 2) /*qkv (fp16)*/ + align256(M * d) /*O*/ +
-           align256(M * d * 2) /*x1*/ + align256(M * d) /*a2*/ + align256(M * F) /*h*/;
+    // every int8 activation between kernels is carried in fp16 (the tensor cores' operand form)
+    return align256(M * d * 2) /*a1*/ + align256(M * 3 * d * 2) /*qkv*/ + align256(M * d * 2) /*O*/ +
+           align256(M * d * 2) /*x1 (int16)*/ + align256(M * d * 2) /*a2*/ + align256(M * F * 2) /*h*/;
 }
 
 int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t *y, int32_t B, int32_t T,
@@ -377,32 +406,35 @@ int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t
         return fail(ILW_ERR_INVALID_ARG, "block: workspace NULL, misaligned or smaller than %zu bytes",
                     ilwdetr_block_workspace_bytes(B, T, d, F));
     const int32_t M = B * T;
+    const int32_t F16 = ILW_I8_IN_F16;
     char *ws = (char *)workspace;
-    int8_t *a1 = (int8_t *)ws; ws += align256((size_t)M * d);
-    __half *qkv = (__half *)ws; ws += align256((size_t)M * 3 * d * 2);  // q|k|v as fp16 (ILW_I8_IN_F16)
-    int8_t *o = (int8_t *)ws; ws += align256((size_t)M * d);
+    __half *a1 = (__half *)ws; ws += align256((size_t)M * d * 2);
+    __half *qkv = (__half *)ws; ws += align256((size_t)M * 3 * d * 2);
+    __half *o = (__half *)ws; ws += align256((size_t)M * d * 2);
     int16_t *x1 = (int16_t *)ws; ws += align256((size_t)M * d * 2);
-    int8_t *a2 = (int8_t *)ws; ws += align256((size_t)M * d);
-    int8_t *hbuf = (int8_t *)ws;
+    __half *a2 = (__half *)ws; ws += align256((size_t)M * d * 2);
+    __half *hbuf = (__half *)ws;
     int rc;
-    if ((rc = ilwdetr_int_layernorm(x, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, a1, 8, d, stream)))
+    if ((rc = ilwdetr_int_layernorm(x, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, a1, F16, d, stream)))
         return rc;
-    if ((rc = ilwdetr_gemm_requant(a1, d, p->w_qkv, p->b_qkv, p->m_qkv, p->s_qkv, M, 3 * d, d, ILW_I8_IN_F16, qkv, 3 * d,
-                                   nullptr, stream)))
+    if ((rc = gemm_impl(a1, F16, d, p->w_qkv, p->b_qkv, p->m_qkv, p->s_qkv, M, 3 * d, d, ILW_EPI_REQUANT, F16, qkv, 3 * d,
+                        nullptr, nullptr, 0, 0, stream, "block qkv")))
         return rc;
-    if ((rc = ilwdetr_shiftmax_attn(qkv, qkv + d, qkv + 2 * d, 3 * d, ILW_I8_IN_F16, B, T, H, d / H, p->win_side, &p->smx, p->m_o,
-                                    p->s_o, o, d, stream)))
+    if ((rc = ilwdetr_shiftmax_attn(qkv, qkv + d, qkv + 2 * d, 3 * d, F16, B, T, H, d / H, p->win_side, &p->smx, p->m_o,
+                                    p->s_o, o, F16, d, stream)))
         return rc;
     ilw_residual_t r1{x, d, M, p->m_r1, p->s_r1};
-    if ((rc = ilwdetr_gemm_requant(o, d, p->w_proj, p->b_proj, p->m_proj, p->s_proj, M, d, d, 16, x1, d, &r1, stream)))
+    if ((rc = gemm_impl(o, F16, d, p->w_proj, p->b_proj, p->m_proj, p->s_proj, M, d, d, ILW_EPI_REQUANT, 16, x1, d, &r1,
+                        nullptr, 0, 0, stream, "block proj")))
         return rc;
-    if ((rc = ilwdetr_int_layernorm(x1, 16, d, M, d, p->ln2_beta, p->ln2_mult, p->ln2_shift, p->ln_iters, a2, 8, d, stream)))
+    if ((rc = ilwdetr_int_layernorm(x1, 16, d, M, d, p->ln2_beta, p->ln2_mult, p->ln2_shift, p->ln_iters, a2, F16, d, stream)))
         return rc;
-    if ((rc = ilwdetr_gemm_gelu(a2, d, p->w_fc1, p->b_fc1, p->m_fc1, p->s_fc1, M, F, d, &p->gelu, p->m_g, p->s_g, hbuf, F,
-                                stream)))
+    if ((rc = gemm_impl(a2, F16, d, p->w_fc1, p->b_fc1, p->m_fc1, p->s_fc1, M, F, d, ILW_EPI_GELU, F16, hbuf, F, nullptr,
+                        &p->gelu, p->m_g, p->s_g, stream, "block fc1")))
         return rc;
     ilw_residual_t r2{x1, d, M, p->m_r2, p->s_r2};
-    return ilwdetr_gemm_requant(hbuf, F, p->w_fc2, p->b_fc2, p->m_fc2, p->s_fc2, M, d, F, 16, y, d, &r2, stream);
+    return gemm_impl(hbuf, F16, F, p->w_fc2, p->b_fc2, p->m_fc2, p->s_fc2, M, d, F, ILW_EPI_REQUANT, 16, y, d, &r2,
+                     nullptr, 0, 0, stream, "block fc2");
 }
 
 // ------------------------------------------------------------------ detector: projector, decoder
@@ -520,7 +552,7 @@ int ilwdetr_decoder_layer_forward(const ilw_decoder_params_t *p, const int16_t *
     ILW_TRY(ilwdetr_gemm_requant(b.v_in, d, p->w_v, p->b_v, p->m_v, p->s_v, M, d, d, 8, b.qkv + 2 * d, 3 * d, nullptr,
                                  stream));
     ILW_TRY(ilwdetr_shiftmax_attn(b.qkv, b.qkv + d, b.qkv + 2 * d, 3 * d, 8, B, Q, H, d / H, 0, &p->smx, p->m_o, p->s_o,
-                                  b.o, d, stream));
+                                  b.o, 8, d, stream));
     ilw_residual_t r1{tgt, d, M, p->m_r1, p->s_r1};
     ILW_TRY(ilwdetr_gemm_requant(b.o, d, p->w_o, p->b_o, p->m_oc, p->s_oc, M, d, d, 16, b.x1, d, &r1, stream));
     ILW_TRY(ilwdetr_int_layernorm(b.x1, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, b.t1, 16, d,

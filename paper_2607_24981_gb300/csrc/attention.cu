@@ -423,21 +423,28 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     // ---- epilogue: sat8(rq(O; m_o, s_o)), written back at the tokens' own positions
     const int r0 = q0 + warp * 16 + g, r1 = r0 + 8;
     const bool ok0 = r0 < Tg, ok1 = r1 < Tg;
-    int8_t *O0 = ok0 ? p.O + gr.token(r0) * p.ld_o + hoff : nullptr;
-    int8_t *O1 = ok1 ? p.O + gr.token(r1) * p.ld_o + hoff : nullptr;
+    const int esz = p.o_f16 ? 2 : 1;
+    uint8_t *O0 = ok0 ? (uint8_t *)p.O + (gr.token(r0) * p.ld_o + hoff) * esz : nullptr;
+    uint8_t *O1 = ok1 ? (uint8_t *)p.O + (gr.token(r1) * p.ld_o + hoff) * esz : nullptr;
+    // two outputs -> int8 pair (16 bits), or the same integers as an fp16 pair: the fp16 bits of
+    // 1152 + v are 0x6480 + v (|v| <= 127), and one half2 subtract of 1152 leaves v exactly
+    const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
+    auto put = [&](uint8_t *dst, int col, int32_t a, int32_t b) {
+        if (p.o_f16) {
+            uint32_t x = (uint32_t)(0x6480 + a) | ((uint32_t)(0x6480 + b) << 16);
+            __half2 h2 = __hsub2(*reinterpret_cast<__half2 *>(&x), k1152);
+            *(uint32_t *)(dst + 2 * col) = *reinterpret_cast<uint32_t *>(&h2);
+        } else {
+            *(uint16_t *)(dst + col) = (uint16_t)((uint8_t)a | ((uint32_t)(uint8_t)b << 8));
+        }
+    };
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
         const int col = nt * 8 + 2 * t;
-        if (ok0) {
-            const int32_t a0 = sat8(rq(__float2int_rn(o[nt][0]), p.m_o, p.s_o));
-            const int32_t a1 = sat8(rq(__float2int_rn(o[nt][1]), p.m_o, p.s_o));
-            *(uint16_t *)(O0 + col) = (uint16_t)((uint8_t)a0 | ((uint32_t)(uint8_t)a1 << 8));
-        }
-        if (ok1) {
-            const int32_t a2 = sat8(rq(__float2int_rn(o[nt][2]), p.m_o, p.s_o));
-            const int32_t a3 = sat8(rq(__float2int_rn(o[nt][3]), p.m_o, p.s_o));
-            *(uint16_t *)(O1 + col) = (uint16_t)((uint8_t)a2 | ((uint32_t)(uint8_t)a3 << 8));
-        }
+        if (ok0)
+            put(O0, col, sat8(rq(__float2int_rn(o[nt][0]), p.m_o, p.s_o)), sat8(rq(__float2int_rn(o[nt][1]), p.m_o, p.s_o)));
+        if (ok1)
+            put(O1, col, sat8(rq(__float2int_rn(o[nt][2]), p.m_o, p.s_o)), sat8(rq(__float2int_rn(o[nt][3]), p.m_o, p.s_o)));
     }
 }
 

@@ -13,15 +13,18 @@
 // before the integer sum.
 //
 // Persistent kernel, one CTA per SM, 128 x BN output tiles, 14 warps:
-//   warp 0      TMA producer: int8 activation tile (128 x 64 bytes) and fp16 weight tile
-//               (BN x 64, 128-byte swizzle) per K stage, STAGES stages ahead; TMEM allocation
+//   warp 0      TMA producer: per K stage the activation tile (int8 128 x 64 bytes, or, when A is
+//               carried in fp16, the fp16 128 x 64 tile in the MMA's 128-byte swizzled layout) and
+//               the fp16 weight tile (BN x 64, 128-byte swizzle); with resident weights the CTA's
+//               BN rows of W are loaded once, before its first tile; TMEM allocation
 //   warp 1      MMA issuer (one thread): 4 x (128 x BN x 16) MMAs per 64-wide K stage
-//   warps 2-5   operand converters: int8 activation rows (smem) -> fp16 rows in the same 128-byte
-//               swizzled K-major layout TMA produces for the weights
+//   warps 2-5   operand converters (int8 A only): int8 activation rows (smem) -> fp16 rows in the
+//               same 128-byte swizzled K-major layout TMA produces for the weights
 //   warps 6-13  epilogue: TMEM -> registers -> integer epilogue -> HBM, one row per thread and
 //               half of the tile's columns per warp
 // Two TMEM accumulator sets (when they fit) let the epilogue of tile i overlap the MMAs of tile
-// i+1.  HBM sees the activations as int8 (half the bytes of fp16).
+// i+1.  With resident weights the grid is a multiple of the number of column blocks, so every
+// tile of a CTA uses the same BN rows of W and L2 serves only the activations.
 // Every mbarrier wait is bounded (about one second); on expiry the kernel latches the device
 // status word, stops issuing work, drains the loads it issued and frees its TMEM.
 #include <cuda.h>
@@ -58,6 +61,7 @@ struct TcParams {  // CUtensorMap members keep the 64-byte alignment TMA needs
     int32_t M, N;
     int32_t tiles_n, tiles;
     int32_t nbuf;       // TMEM accumulator sets (1 or 2)
+    int32_t wres_bytes; // resident weight bytes (WRES), a multiple of 1024
     int32_t tmem_cols;
     const int8_t *gelu_tab;  // SD-ShiftGELU output table in global memory (16-byte aligned, 65536 bytes)
     int *status;
@@ -161,18 +165,24 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
     hi = *reinterpret_cast<uint32_t *>(&hb);
 }
 
-// Shared memory per pipeline stage: fp16 A (128 rows x 128 B, swizzled), fp16 W (BN rows x 128 B,
-// swizzled by TMA), int8 A staging (128 rows x 64 B, written by TMA).
-template <int BN>
+// Shared memory per pipeline stage: fp16 A (128 rows x 128 B, swizzled; written by the converter
+// warps from the int8 staging rows, or by TMA directly when A arrives as fp16), fp16 W (BN rows x
+// 128 B, swizzled by TMA; absent when the CTA's weights are resident), int8 A staging (128 rows x
+// 64 B, written by TMA; absent for fp16 A).  Resident weights (WRES) keep every K block of the
+// CTA's BN rows of W after the stages.
+template <int BN, bool AF16 = false, bool WRES = false>
 struct Smem {
     static constexpr int kA16 = BM * 128;
-    static constexpr int kW = BN * 128;
-    static constexpr int kA8 = BM * 64;
+    static constexpr int kW = WRES ? 0 : BN * 128;
+    static constexpr int kA8 = AF16 ? 0 : BM * 64;
     static constexpr int kStage = kA16 + kW + kA8;
+    static constexpr int kWtile = BN * 128;  // one K block of W
 };
 
 // Output kinds: one compact epilogue per kernel instantiation.
-enum { KIND_RQ8 = 0, KIND_RQ16 = 1, KIND_RAW32 = 2, KIND_GELU8 = 3, KIND_F16OUT = 4 };  // F16OUT: RQ8 values as fp16
+// F16OUT: RQ8 values as fp16; GELU_F16: GELU8 values as fp16
+enum { KIND_RQ8 = 0, KIND_RQ16 = 1, KIND_RAW32 = 2, KIND_GELU8 = 3, KIND_F16OUT = 4, KIND_GELU_F16 = 5 };
+constexpr bool gelu_kind(int kind) { return kind == KIND_GELU8 || kind == KIND_GELU_F16; }
 
 // 16 consecutive int32 of shared memory (16-byte aligned) into registers: four 128-bit loads
 __device__ __forceinline__ void lds16(const int32_t *p, int32_t (&o)[16]) {
@@ -209,7 +219,7 @@ __device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool has_res, con
             r[i] = (int32_t)(t < -(1 << 30) ? -(1 << 30) : (t > (1 << 30) ? (1 << 30) : t));  // saturates the same
         }
     }
-    if (KIND == KIND_GELU8) {
+    if (KIND == KIND_GELU8 || KIND == KIND_GELU_F16) {
         // g = sat16(r); the table holds sat8(rq(g * I_div(g); m_g, s_g)) for every int16 g
 #pragma unroll
         for (int i = 0; i < 16; ++i) out[i] = gtab[clamp16(r[i])];
@@ -228,14 +238,16 @@ __device__ __forceinline__ void epi_chunk(const EpiParams &ep, bool has_res, con
     for (int i = 0; i < 16; ++i) out[i] = (KIND == KIND_RQ8 || KIND == KIND_F16OUT) ? clamp8(r[i]) : clamp16(r[i]);
 }
 
-template <int BN, int STAGES, int KIND, int NB>
+template <int BN, int STAGES, int KIND, int NB, bool AF16, bool WRES>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcParams<NB> p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    constexpr int kStage = Smem<BN>::kStage;
-    uint64_t *bars = (uint64_t *)(smem + STAGES * kStage);
-    // barriers: full[S], a_ready[S], empty[S], acc_full[2], acc_empty[2]
-    uint32_t *tmem_slot = (uint32_t *)(bars + 3 * STAGES + 4);
+    using SM = Smem<BN, AF16, WRES>;
+    constexpr int kStage = SM::kStage;
+    uint8_t *wres = smem + STAGES * kStage;  // resident weights (WRES)
+    uint64_t *bars = (uint64_t *)(wres + (WRES ? p.wres_bytes : 0));
+    // barriers: full[S], a_ready[S], empty[S], acc_full[2], acc_empty[2], wfull
+    uint32_t *tmem_slot = (uint32_t *)(bars + 3 * STAGES + 5);
     volatile int *abort = (volatile int *)(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -245,6 +257,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     auto empty = [&](int s) { return bar0 + 8u * (2 * STAGES + s); };
     auto acc_full = [&](int b) { return bar0 + 8u * (3 * STAGES + b); };
     auto acc_empty = [&](int b) { return bar0 + 8u * (3 * STAGES + 2 + b); };
+    const uint32_t wfull = bar0 + 8u * (3 * STAGES + 4);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -256,6 +269,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             mbar_init(acc_full(b), 1);
             mbar_init(acc_empty(b), 8);
         }
+        mbar_init(wfull, 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -273,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     // sat8(rq(g * I_div(g); m_g, s_g)) (built once per parameter set by gelu_table_kernel) is
     // copied into shared memory here.
     int8_t *gtab = (int8_t *)((int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + 16 * BN);
-    if (KIND == KIND_GELU8 && warp >= 6) {
+    if ((KIND == KIND_GELU8 || KIND == KIND_GELU_F16) && warp >= 6) {
         for (int i = threadIdx.x - 192; i < 65536 / 16; i += 256) ((uint4 *)gtab)[i] = __ldg((const uint4 *)p.gelu_tab + i);
         asm volatile("bar.sync 1, 256;" ::: "memory");  // the 8 epilogue warps only
     }
@@ -284,6 +298,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         if (lane == 0) {
             int it = 0;  // global K-block counter (ring position)
             bool ok = true;
+            if (WRES && blockIdx.x < p.tiles) {
+                // this CTA's BN rows of W, resident for all of its tiles (the grid is a multiple of
+                // tiles_n, so every tile of the CTA has the same n block)
+                const int n0 = (blockIdx.x % p.tiles_n) * BN;
+                const int nk = (p.seg[0].klen + BK - 1) / BK;
+                mbar_expect_tx(wfull, (uint32_t)(nk * SM::kWtile));
+                for (int kk = 0; kk < nk; ++kk)
+                    tma_load_2d(smem_u32(wres + kk * SM::kWtile), &p.wmap[0], p.seg[0].k0 + kk * BK, n0, wfull);
+            }
             for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x) {
                 const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN;
                 for (int sg = 0; sg < p.nseg && ok; ++sg) {
@@ -297,15 +320,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                             break;
                         }
                         uint8_t *st = smem + s * kStage;
-                        mbar_expect_tx(full(s), Smem<BN>::kW + Smem<BN>::kA8);
-                        tma_load_2d(smem_u32(st + Smem<BN>::kA16 + Smem<BN>::kW), &p.amap[S.map], S.k0 + kk * BK, m0,
+                        mbar_expect_tx(full(s), (AF16 ? SM::kA16 : SM::kA8) + SM::kW);
+                        tma_load_2d(smem_u32(AF16 ? st : st + SM::kA16 + SM::kW), &p.amap[S.map], S.k0 + kk * BK, m0,
                                     full(s));
-                        tma_load_2d(smem_u32(st + Smem<BN>::kA16), &p.wmap[S.map], S.k0 + kk * BK, n0, full(s));
+                        if (!WRES) tma_load_2d(smem_u32(st + SM::kA16), &p.wmap[S.map], S.k0 + kk * BK, n0, full(s));
                     }
                 }
             }
             if (!ok) {  // drain the loads still in flight (bounded) before the CTA can exit
                 long long t0 = clock64();
+                while (WRES && blockIdx.x < p.tiles && !mbar_try(wfull, 0) && clock64() - t0 < kWaitCycles) {
+                }
                 for (int j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
                     while (!mbar_try(full(j % STAGES), (j / STAGES) & 1) && clock64() - t0 < kWaitCycles) {
                     }
@@ -317,6 +342,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint32_t idesc = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
             int it = 0, tl = 0;
             bool ok = true;
+            if (WRES && blockIdx.x < p.tiles) {
+                ok = mbar_wait(wfull, 0, abort, p.status, kStatusTimeoutTma);
+                tc_fence_after();
+            }
             for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++tl) {
                 const int b = tl % p.nbuf;
                 const uint32_t use = (uint32_t)(tl / p.nbuf);
@@ -329,12 +358,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     for (int kk = 0; kk < nk; ++kk, ++it) {
                         const int s = it % STAGES;
                         const uint32_t ph = (it / STAGES) & 1;
-                        if (!mbar_wait(a_ready(s), ph, abort, p.status, kStatusTimeoutOperand)) {
+                        if (!mbar_wait(AF16 ? full(s) : a_ready(s), ph, abort, p.status,
+                                       AF16 ? kStatusTimeoutTma : kStatusTimeoutOperand)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
-                        const uint32_t a0 = smem_u32(smem + s * kStage), w0 = a0 + Smem<BN>::kA16;
+                        const uint32_t a0 = smem_u32(smem + s * kStage);
+                        const uint32_t w0 = WRES ? smem_u32(wres + kk * SM::kWtile) : a0 + SM::kA16;
 #pragma unroll
                         for (int k16 = 0; k16 < BK / 16; ++k16)
                             tc_mma(dt, sw128_desc(a0 + 32 * k16), sw128_desc(w0 + 32 * k16), idesc,
@@ -347,33 +378,35 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
     } else if (warp < 6) {
         // ---------------------------------------------------------------- operand converters
-        const int r = (warp - 2) * 32 + lane;  // row of the 128-row A tile
-        const int sw = (r >> 1) & 3;           // TMA's 64-byte swizzle of the int8 staging rows
-        int it = 0;
-        for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
-            for (int sg = 0; sg < p.nseg; ++sg) {
-                const int nk = (p.seg[sg].klen + BK - 1) / BK;
-                for (int kk = 0; kk < nk; ++kk, ++it) {
-                    const int s = it % STAGES;
-                    const uint32_t ph = (it / STAGES) & 1;
-                    if (!mbar_wait(full(s), ph, abort, p.status, kStatusTimeoutTma)) goto conv_done;
-                    uint8_t *st = smem + s * kStage;
-                    const uint8_t *a8 = st + Smem<BN>::kA16 + Smem<BN>::kW + r * 64;
-                    uint8_t *a16 = st + r * 128;
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {  // 16 int8 = K elements 16j .. 16j+15
-                        const uint4 v = *(const uint4 *)(a8 + 16 * (j ^ sw));
-                        uint4 o0, o1;
-                        i8x4_to_f16x4(v.x, o0.x, o0.y);
-                        i8x4_to_f16x4(v.y, o0.z, o0.w);
-                        i8x4_to_f16x4(v.z, o1.x, o1.y);
-                        i8x4_to_f16x4(v.w, o1.z, o1.w);
-                        *(uint4 *)(a16 + (((2 * j) ^ (r & 7)) << 4)) = o0;
-                        *(uint4 *)(a16 + (((2 * j + 1) ^ (r & 7)) << 4)) = o1;
+        if constexpr (!AF16) {  // fp16 A arrives in the MMA's operand layout: nothing to convert
+            const int r = (warp - 2) * 32 + lane;  // row of the 128-row A tile
+            const int sw = (r >> 1) & 3;           // TMA's 64-byte swizzle of the int8 staging rows
+            int it = 0;
+            for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
+                for (int sg = 0; sg < p.nseg; ++sg) {
+                    const int nk = (p.seg[sg].klen + BK - 1) / BK;
+                    for (int kk = 0; kk < nk; ++kk, ++it) {
+                        const int s = it % STAGES;
+                        const uint32_t ph = (it / STAGES) & 1;
+                        if (!mbar_wait(full(s), ph, abort, p.status, kStatusTimeoutTma)) goto conv_done;
+                        uint8_t *st = smem + s * kStage;
+                        const uint8_t *a8 = st + SM::kA16 + SM::kW + r * 64;
+                        uint8_t *a16 = st + r * 128;
+    #pragma unroll
+                        for (int j = 0; j < 4; ++j) {  // 16 int8 = K elements 16j .. 16j+15
+                            const uint4 v = *(const uint4 *)(a8 + 16 * (j ^ sw));
+                            uint4 o0, o1;
+                            i8x4_to_f16x4(v.x, o0.x, o0.y);
+                            i8x4_to_f16x4(v.y, o0.z, o0.w);
+                            i8x4_to_f16x4(v.z, o1.x, o1.y);
+                            i8x4_to_f16x4(v.w, o1.z, o1.w);
+                            *(uint4 *)(a16 + (((2 * j) ^ (r & 7)) << 4)) = o0;
+                            *(uint4 *)(a16 + (((2 * j + 1) ^ (r & 7)) << 4)) = o1;
+                        }
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(a_ready(s));
                     }
-                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(a_ready(s));
                 }
             }
         }
@@ -388,7 +421,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         int32_t *s_mult = s_bias + HALF;                                       // the tile's per-column
         int32_t *s_shift = s_mult + HALF;                                      // epilogue parameters
         int32_t *s_rnd = s_shift + HALF;                                       // (rq_hi rounding constants)
-        constexpr int bits = (KIND == KIND_RQ16 || KIND == KIND_F16OUT) ? 16 : (KIND == KIND_RAW32 ? 32 : 8);
+        constexpr int bits = (KIND == KIND_RQ16 || KIND == KIND_F16OUT || KIND == KIND_GELU_F16) ? 16
+                             : (KIND == KIND_RAW32 ? 32 : 8);
         constexpr int PPL = HALF / 32;  // parameters per lane and per array
         // The next tile's parameters are fetched into registers while the current tile is processed.
         int32_t pb[PPL], pm[PPL], ps[PPL];
@@ -492,7 +526,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                         epi_chunk<KIND, FAST, RFAST>(ep, has_res, rp, acc, cb, cm, cs, cr, gt, out);
                         char *dst = (char *)ep.C + (row * ep.ldc + n0 + c0) * (bits / 8);
                         const bool vec = ncol == 16 && (((uintptr_t)dst & 15) == 0);
-                        if constexpr (KIND == KIND_F16OUT) {
+                        if constexpr (KIND == KIND_F16OUT || KIND == KIND_GELU_F16) {
                             // |v| <= 127: the fp16 bits of 1152 + v are 0x6480 + v; one half2 subtract of
                             // 1152 leaves v exactly
                             const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
@@ -557,12 +591,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 }
             };
             constexpr bool kRes = KIND == KIND_RQ8 || KIND == KIND_RQ16;  // kinds with a residual
+            using T_ = std::true_type;
+            using F_ = std::false_type;
+            using R_ = std::integral_constant<bool, kRes>;
+            auto go = [&](auto f, auto r) { chunks(f, r); };
             if (fastw) {
-                if (kRes && rfast) chunks(std::integral_constant<bool, true>{}, std::integral_constant<bool, kRes>{});
-                else chunks(std::integral_constant<bool, true>{}, std::integral_constant<bool, false>{});
+                if (kRes && rfast) go(T_{}, R_{});
+                else go(T_{}, F_{});
             } else {
-                if (kRes && rfast) chunks(std::integral_constant<bool, false>{}, std::integral_constant<bool, kRes>{});
-                else chunks(std::integral_constant<bool, false>{}, std::integral_constant<bool, false>{});
+                if (kRes && rfast) go(F_{}, R_{});
+                else go(F_{}, F_{});
             }
         }
     }
@@ -726,23 +764,37 @@ int num_sms() {
     return n;
 }
 
-template <int BN, int STAGES, int KIND, int NB>
+// Dynamic shared memory of one instantiation (wres: resident weight bytes).
+template <int BN, int STAGES, int KIND, bool AF16, bool WRES>
+size_t smem_bytes(int wres) {
+    return 1024 + (size_t)STAGES * Smem<BN, AF16, WRES>::kStage + (WRES ? wres : 0) + 8 * (3 * STAGES + 5) + 32 +
+           4 * 4 * BN * 4 + (gelu_kind(KIND) ? 65536 : 0);
+}
+constexpr size_t kSmemMax = 227 * 1024;
+
+template <int BN, int STAGES, int KIND, int NB, bool AF16, bool WRES>
 cudaError_t launch_tc(TcParams<NB> &tp, cudaStream_t s) {
-    const size_t smem = 1024 + (size_t)STAGES * Smem<BN>::kStage + 8 * (3 * STAGES + 4) + 32 + 4 * 4 * BN * 4 +
-                        (KIND == KIND_GELU8 ? 65536 : 0);
+    const size_t smem = smem_bytes<BN, STAGES, KIND, AF16, WRES>(tp.wres_bytes);
+    if (smem > kSmemMax) return cudaErrorInvalidValue;
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, KIND, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)smem);
+        attr_err = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, KIND, NB, AF16, WRES>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMax);
     });
     if (attr_err != cudaSuccess) return attr_err;
-    const int grid = tp.tiles < num_sms() ? tp.tiles : num_sms();
-    gemm_tc_kernel<BN, STAGES, KIND, NB><<<grid, kThreads, smem, s>>>(tp);
+    int grid = tp.tiles < num_sms() ? tp.tiles : num_sms();
+    if (WRES) {  // a multiple of tiles_n: every CTA keeps one n block of W
+        const int tiles_m = tp.tiles / tp.tiles_n;
+        int per_n = num_sms() / tp.tiles_n;
+        per_n = per_n < 1 ? 1 : (per_n > tiles_m ? tiles_m : per_n);
+        grid = per_n * tp.tiles_n;
+    }
+    gemm_tc_kernel<BN, STAGES, KIND, NB, AF16, WRES><<<grid, kThreads, smem, s>>>(tp);
     return cudaGetLastError();
 }
 
-template <int BN, int STAGES, int NB>
+template <int BN, int STAGES, int NB, bool AF16 = false, bool WRES = false>
 cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     if (gp.nb > NB) return cudaErrorInvalidValue;
     TcParams<NB> tp;
@@ -755,8 +807,12 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     int nseg = 0;
     for (int b = 0; b < gp.nb; ++b) {
         const GemmBranch &br = gp.br[b];
-        if (!make_map(&tp.amap[b], br.A, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, gp.M, br.K, br.lda, BK, BM,
-                      CU_TENSOR_MAP_SWIZZLE_64B) ||
+        const bool amap_ok =
+            AF16 ? make_map(&tp.amap[b], br.A, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, gp.M, br.K, br.lda, BK, BM,
+                            CU_TENSOR_MAP_SWIZZLE_128B)
+                 : make_map(&tp.amap[b], br.A, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, gp.M, br.K, br.lda, BK, BM,
+                            CU_TENSOR_MAP_SWIZZLE_64B);
+        if (!amap_ok ||
             !make_map(&tp.wmap[b], br.Wp, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, gp.N, br.K, br.K, BK, BN,
                       CU_TENSOR_MAP_SWIZZLE_128B))
             return cudaErrorInvalidValue;
@@ -783,23 +839,29 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     while (alloc < tp.nbuf * one) alloc <<= 1;
     if (alloc > 512) return cudaErrorInvalidValue;
     tp.tmem_cols = alloc;
+    if (WRES) {
+        if (nseg != 1) return cudaErrorInvalidValue;
+        tp.wres_bytes = ((tp.seg[0].klen + BK - 1) / BK) * Smem<BN, AF16, WRES>::kWtile;
+    }
     if (ep.kind == EPI_GELU) {
         cudaError_t e = cudaSuccess;
         tp.gelu_tab = gelu_table(ep.gelu, ep.m_g, ep.s_g, s, &e);
         if (!tp.gelu_tab) return e != cudaSuccess ? e : cudaErrorUnknown;
     }
     if constexpr (NB == 1) {
-        if (ep.kind == EPI_GELU) return launch_tc<BN, STAGES, KIND_GELU8, NB>(tp, s);
+        if (ep.kind == EPI_GELU)
+            return ep.out_bits == kOutI8InF16 ? launch_tc<BN, STAGES, KIND_GELU_F16, NB, AF16, WRES>(tp, s)
+                                              : launch_tc<BN, STAGES, KIND_GELU8, NB, AF16, WRES>(tp, s);
     } else {
         if (ep.kind == EPI_GELU) return cudaErrorInvalidValue;  // split convolutions requantise only
     }
     if (ep.out_bits == kOutI8InF16) {
-        if constexpr (NB == 1) return launch_tc<BN, STAGES, KIND_F16OUT, NB>(tp, s);
+        if constexpr (NB == 1) return launch_tc<BN, STAGES, KIND_F16OUT, NB, AF16, WRES>(tp, s);
         else return cudaErrorInvalidValue;
     }
-    if (ep.out_bits == 8) return launch_tc<BN, STAGES, KIND_RQ8, NB>(tp, s);
-    if (ep.out_bits == 16) return launch_tc<BN, STAGES, KIND_RQ16, NB>(tp, s);
-    return launch_tc<BN, STAGES, KIND_RAW32, NB>(tp, s);
+    if (ep.out_bits == 8) return launch_tc<BN, STAGES, KIND_RQ8, NB, AF16, WRES>(tp, s);
+    if (ep.out_bits == 16) return launch_tc<BN, STAGES, KIND_RQ16, NB, AF16, WRES>(tp, s);
+    return launch_tc<BN, STAGES, KIND_RAW32, NB, AF16, WRES>(tp, s);
 }
 
 }  // namespace
@@ -814,6 +876,23 @@ cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t
     if (gp.M == 0 || gp.N == 0) return cudaSuccess;
     // 192-wide tiles when N splits evenly into them (fewer re-reads of A per flop), else 128
     if (gp.nb > 1) return run<128, 5, kMaxBranches>(gp, ep, s);
+    if (gp.a_f16) {
+        // fp16 A: no conversion stage.  Weights resident in shared memory when the CTA's BN rows
+        // of W fit next to the A stages (K <= 1024); GELU tiles are 128 wide to leave room for
+        // its 64 KB table.
+        const bool gelu = ep.kind == EPI_GELU;
+        const int K = gp.br[0].K, nkb = (K + BK - 1) / BK;
+        const bool wide = !gelu && gp.N % 192 == 0 && gp.N >= 384;
+        if (K <= kSegK) {
+            if (wide && smem_bytes<192, 3, KIND_RQ8, true, true>(nkb * 192 * 128) <= kSmemMax)
+                return run<192, 3, 1, true, true>(gp, ep, s);
+            if (!wide && smem_bytes<128, 3, KIND_GELU8, true, true>(nkb * 128 * 128) <= kSmemMax)
+                return run<128, 3, 1, true, true>(gp, ep, s);
+        }
+        if (gp.N % 192 == 0 && gp.N >= 384)
+            return gelu ? run<192, 3, 1, true, false>(gp, ep, s) : run<192, 4, 1, true, false>(gp, ep, s);
+        return gelu ? run<128, 3, 1, true, false>(gp, ep, s) : run<128, 5, 1, true, false>(gp, ep, s);
+    }
     if (gp.N % 192 == 0 && gp.N >= 768)
         return ep.kind == EPI_GELU ? run<192, 3, 1>(gp, ep, s) : run<192, 4, 1>(gp, ep, s);
     return ep.kind == EPI_GELU ? run<128, 3, 1>(gp, ep, s) : run<128, 5, 1>(gp, ep, s);

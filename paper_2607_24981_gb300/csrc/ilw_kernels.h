@@ -55,6 +55,7 @@ struct GemmProblem {
     int32_t M, N;
     int32_t nb;        // branches; 1 = plain GEMM
     bool branch_rq;    // rq each branch partial with (m_b, s_b) before the integer sum
+    bool a_f16;        // A holds the int8 values as fp16 (plain GEMM only)
     GemmBranch br[kMaxBranches];
 };
 enum EpiKind { EPI_REQUANT = 0, EPI_GELU = 1 };
@@ -113,8 +114,9 @@ struct AttnParams {
     int32_t grid_side; // sqrt(T) when nw > 1
     ShiftmaxC smx;
     int32_t m_o, s_o;
-    int8_t *O;
-    int64_t ld_o;
+    void *O;           // int8, or fp16 holding the int8 values when o_f16
+    int32_t o_f16;
+    int64_t ld_o;      // elements
 };
 cudaError_t launch_attention(const AttnParams &p, cudaStream_t s);
 
@@ -136,6 +138,8 @@ cudaError_t launch_deform(const DeformParams &p, cudaStream_t s);
 // ---------------------------------------------------------------- patch embedding
 cudaError_t launch_patchify(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
                             int8_t *A, cudaStream_t s);
+cudaError_t launch_patchify_f16(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
+                                __half *A, cudaStream_t s);
 
 // ---------------------------------------------------------------- detector: requantisation, resampling
 struct RequantParams {

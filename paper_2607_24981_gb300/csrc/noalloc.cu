@@ -55,7 +55,8 @@ extern "C" int ilwdetr_patch_embed_noalloc(const int8_t *img, int32_t B, int32_t
     if (B < 0 || Cin < 1 || p < 16 || p % 16 || Hh < p || Ww < p || Hh % p || Ww % p || Ww % 16 || d < 1)
         return ilw::report_error(ILW_ERR_UNSUPPORTED, "patch_embed_noalloc: needs p % 16 == 0, p | H, p | W");
     if (B == 0) return ILW_OK;
-    const size_t need = ilwdetr_patch_embed_workspace_bytes(B, Cin, Hh, Ww, p);
+    // the gathered patch matrix, int8 (B*T rows of Cin*p*p)
+    const size_t need = (size_t)B * (Hh / p) * (Ww / p) * Cin * p * p;
     if (need > kNoAllocScratchBytes)
         return ilw::report_error(ILW_ERR_UNSUPPORTED,
                                  "patch_embed_noalloc: this batch needs more scratch than the fixed 8 MiB "
@@ -65,6 +66,11 @@ extern "C" int ilwdetr_patch_embed_noalloc(const int8_t *img, int32_t B, int32_t
     int rc = scratch_on_current_device(&scratch);
     if (rc) return rc;
     // every byte the GEMM reads is written by the gather first: nothing needs clearing
-    return ilwdetr_patch_embed(img, B, Cin, Hh, Ww, p, Wp, bias, mult, shift, d, pos, m_pos, s_pos, x0, scratch,
-                               kNoAllocScratchBytes, stream);
+    if (!img || ((uintptr_t)img % 16) != 0 || !x0)
+        return ilw::report_error(ILW_ERR_INVALID_ARG, "patch_embed_noalloc: NULL or misaligned image");
+    cudaError_t e = ilw::launch_patchify(img, B, Cin, Hh, Ww, p, scratch, (cudaStream_t)stream);
+    if (e != cudaSuccess) return ilw::report_error(ILW_ERR_CUDA, cudaGetErrorString(e));
+    const int32_t T = (Hh / p) * (Ww / p), K = Cin * p * p;
+    ilw_residual_t r{pos, d, T, m_pos, s_pos};
+    return ilwdetr_gemm_requant(scratch, K, Wp, bias, mult, shift, B * T, d, K, 16, x0, d, pos ? &r : nullptr, stream);
 }

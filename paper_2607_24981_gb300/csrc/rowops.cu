@@ -179,7 +179,7 @@ __global__ void sdshiftgelu_tail(const int32_t *X, int32_t *Y, int64_t start, in
 // stops at 0, which only V = 0 reaches), cut short once the rest of the sequence is known: a fixed
 // point repeats forever, and once r_{i+1} = r_{i-1} the iterates alternate between two values, so
 // r_iters is read off the parity of the steps left.  Identical result, fewer 64-bit divisions.
-__device__ __forceinline__ uint64_t newton_isqrt_early(uint64_t V, int iters) {
+__device__ __noinline__ uint64_t newton_isqrt_early(uint64_t V, int iters) {
     uint64_t r = 1ull << 16, prev = ~0ull;
     for (int it = 0; it < iters; ++it) {
         if (r == 0) break;
@@ -246,6 +246,32 @@ __device__ __forceinline__ uint64_t newton_isqrt_fast(uint64_t V, int iters) {
 // requantisation takes the high-word form.  Rows or columns outside those conditions use the
 // 64-bit formulas.
 
+// Output element types of I-LayerNorm: int8, int16, or the int8 values carried in fp16.
+template <typename TOut> struct LnOut { static constexpr int bits = 8 * (int)sizeof(TOut); };
+template <> struct LnOut<__half> { static constexpr int bits = 8; };
+// 4 outputs of one row, stored at y (4-element aligned)
+template <typename TOut>
+__device__ __forceinline__ void ln_store4(TOut *y, const int32_t (&o)[4]) {
+    if constexpr (sizeof(TOut) == 1) {
+        *(uint32_t *)y = (uint32_t)(uint8_t)o[0] | ((uint32_t)(uint8_t)o[1] << 8) | ((uint32_t)(uint8_t)o[2] << 16) |
+                         ((uint32_t)(uint8_t)o[3] << 24);
+    } else if constexpr (LnOut<TOut>::bits == 16) {
+        *(uint2 *)y = make_uint2((uint32_t)(uint16_t)o[0] | ((uint32_t)(uint16_t)o[1] << 16),
+                                 (uint32_t)(uint16_t)o[2] | ((uint32_t)(uint16_t)o[3] << 16));
+    } else {
+        // |v| <= 127: the fp16 bits of 1152 + v are 0x6480 + v; one half2 subtract of 1152 leaves v
+        const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
+        uint32_t w[2];
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            uint32_t x = (uint32_t)(0x6480 + o[2 * j]) | ((uint32_t)(0x6480 + o[2 * j + 1]) << 16);
+            __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), k1152);
+            w[j] = *reinterpret_cast<uint32_t *>(&h);
+        }
+        *(uint2 *)y = make_uint2(w[0], w[1]);
+    }
+}
+
 // acc += a * b with a 64-bit accumulator in one wide multiply-add
 __device__ __forceinline__ void madw(int64_t &acc, int32_t a, int32_t b) {
     asm("mad.wide.s32 %0, %1, %2, %0;" : "+l"(acc) : "r"(a), "r"(b));
@@ -256,6 +282,19 @@ struct LnRowStat {
     int32_t fast;
     int32_t mF;  // -mu * F in wrapping 32-bit arithmetic: (x F + mF) = (x - mu) F exactly when that fits int32
 };
+
+// The normalisation of 4 elements in 64-bit arithmetic, for tiles or columns outside the 32-bit
+// fast path's conditions (kept out of line so that its registers do not weigh on the fast path).
+__device__ __noinline__ void ln_norm4_exact(const int32_t (&x)[4], int64_t mu, int64_t F, const int32_t (&be)[4],
+                                            const int32_t (&mm)[4], const int32_t (&ss)[4], int out_bits,
+                                            int32_t (&o)[4]) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int64_t n = (((int64_t)x[u] - mu) * F) >> 1;
+        const int64_t tq = rq(n + be[u], mm[u], ss[u]);
+        o[u] = out_bits == 8 ? sat8(tq) : sat16(tq);
+    }
+}
 
 template <typename TIn>
 __device__ __forceinline__ void ln_get4(const uint8_t *p, int32_t (&x)[4]) {
@@ -405,15 +444,7 @@ __global__ void __launch_bounds__(256) layernorm_tile(const LnParams p, int32_t 
 
         // (4) normalise: rows rs, rs + kpass, ... of this thread's column group
         TOut *ybase = (TOut *)p.Y + row0 * p.ldy + 4 * cc;
-        auto store = [&](int r, const int32_t (&o)[4]) {
-            TOut *y = ybase + (int64_t)r * p.ldy;
-            if (sizeof(TOut) == 1)
-                *(uint32_t *)y = (uint32_t)(uint8_t)o[0] | ((uint32_t)(uint8_t)o[1] << 8) |
-                                 ((uint32_t)(uint8_t)o[2] << 16) | ((uint32_t)(uint8_t)o[3] << 24);
-            else
-                *(uint2 *)y = make_uint2((uint32_t)(uint16_t)o[0] | ((uint32_t)(uint16_t)o[1] << 16),
-                                         (uint32_t)(uint16_t)o[2] | ((uint32_t)(uint16_t)o[3] << 16));
-        };
+        auto store = [&](int r, const int32_t (&o)[4]) { ln_store4<TOut>(ybase + (int64_t)r * p.ldy, o); };
         if (tile_fast && cols_fast) {
             // (x - mu) F = x F + mF in wrapping 32-bit arithmetic (the product fits int32), and
             // rq takes its high-word form with the rounding constant folded in
@@ -425,31 +456,15 @@ __global__ void __launch_bounds__(256) layernorm_tile(const LnParams p, int32_t 
                 for (int u = 0; u < 4; ++u) {
                     const int32_t n = (int32_t)((uint32_t)x[u] * (uint32_t)F + (uint32_t)mF) >> 1;
                     const int32_t tq = rq_hi(n + be[u], mm[u], rnd[u], sh[u]);
-                    o[u] = sizeof(TOut) == 1 ? clamp8(tq) : clamp16(tq);
+                    o[u] = LnOut<TOut>::bits == 8 ? clamp8(tq) : clamp16(tq);
                 }
                 store(r, o);
             }
         } else {
             for (int r = rs; r < nrows; r += kpass) {
-                const LnRowStat st = stat[r];
                 int32_t x[4], o[4];
                 ln_get4<TIn>(tile + r * pitch + cc * 4 * EB, x);
-                if (st.fast && col_fast) {
-                    const int32_t mu = (int32_t)st.mu, F = (int32_t)st.F;
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int32_t n = ((x[u] - mu) * F) >> 1;
-                        const int32_t tq = rq_hi1(n + be[u], mm[u], ss[u] - 33);
-                        o[u] = sizeof(TOut) == 1 ? clamp8(tq) : clamp16(tq);
-                    }
-                } else {
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int64_t n = (((int64_t)x[u] - st.mu) * st.F) >> 1;
-                        const int64_t tq = rq(n + be[u], mm[u], ss[u]);
-                        o[u] = sizeof(TOut) == 1 ? sat8(tq) : sat16(tq);
-                    }
-                }
+                ln_norm4_exact(x, stat[r].mu, stat[r].F, be, mm, ss, LnOut<TOut>::bits, o);
                 store(r, o);
             }
         }
@@ -499,7 +514,9 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const LnParams p) {
             int64_t y = (int64_t)v[j] - mu;
             int64_t n = (y * F) >> 1;
             int64_t o = rq(n + p.beta[c], p.mult[c], p.shift[c]);
-            yo[c] = (TOut)(sizeof(TOut) == 1 ? sat8(o) : sat16(o));
+            const int32_t v = LnOut<TOut>::bits == 8 ? sat8(o) : sat16(o);
+            if constexpr (sizeof(TOut) == 2 && LnOut<TOut>::bits == 8) yo[c] = __int2half_rn(v);
+            else yo[c] = (TOut)v;
         }
     }
 }
@@ -614,6 +631,8 @@ cudaError_t launch_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const Ge
 
 cudaError_t launch_layernorm(const LnParams &p, cudaStream_t s) {
     if (p.rows == 0) return cudaSuccess;
+    if (p.out_bits == kOutI8InF16)
+        return p.in_bits == 16 ? ln_dispatch<int16_t, __half>(p, s) : ln_dispatch<int32_t, __half>(p, s);
     if (p.in_bits == 16 && p.out_bits == 8) return ln_dispatch<int16_t, int8_t>(p, s);
     if (p.in_bits == 16 && p.out_bits == 16) return ln_dispatch<int16_t, int16_t>(p, s);
     if (p.in_bits == 32 && p.out_bits == 8) return ln_dispatch<int32_t, int8_t>(p, s);

@@ -61,13 +61,13 @@ def test_host_side_validation_without_gpu(built_lib):
     assert rc == -1
     smx = ilw.ShiftmaxT(100, 16, 8, -1, 4, 31)
     rc = L.ilwdetr_shiftmax_attn(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), 48, 8, 1, 64, 1, 48,
-                                 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 48, None)
+                                 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 8, 48, None)
     assert rc == -2  # dh = 48 unsupported
     rc = L.ilwdetr_shiftmax_attn(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), 64, 16, 1, 64, 1, 64,
-                                 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 64, None)
+                                 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 8, 64, None)
     assert rc == -1 and b"qkv_form" in L.ilwdetr_last_error()  # neither int8 nor ILW_I8_IN_F16
     rc = L.ilwdetr_shiftmax_attn(ctypes.c_void_p(16), ctypes.c_void_p(16), ctypes.c_void_p(16), 68, ilw.I8_IN_F16, 1,
-                                 64, 1, 64, 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 64, None)
+                                 64, 1, 64, 0, ctypes.byref(smx), 1 << 30, 30, ctypes.c_void_p(16), 8, 64, None)
     assert rc == -1  # fp16 rows of 68 elements are not 16-byte aligned
     rc = L.ilwdetr_gemm_requant(ctypes.c_void_p(16), 24, ctypes.c_void_p(256), None, None, None, 4, 4, 24, 8,
                                 ctypes.c_void_p(16), 4, None, None)

@@ -89,6 +89,40 @@ def test_gemm_gelu(ilw, orc, M, N, K, I0):
     assert_same(host(got), want, "gemm_gelu")
 
 
+# fp16-carried int8 A (ilwdetr_gemm a_form ILW_I8_IN_F16): resident-weight tiles of 192 (N % 192 == 0)
+# and 128 columns, streamed weights for K > 1024, ragged M / N, every epilogue form
+@pytest.mark.parametrize("M,N,K", [(1, 1, 16), (37, 29, 64), (300, 1152, 384), (257, 384, 1024), (130, 200, 384),
+                                   (128, 96, 256), (12800, 1536, 384), (333, 384, 1536), (64, 192, 1040)])
+@pytest.mark.parametrize("kind", ["rq8", "rq16res", "f16", "raw32", "gelu8", "gelu_f16"])
+def test_gemm_f16_operand(ilw, orc, M, N, K, kind):
+    if M * N * K > 1e9 and kind not in ("f16", "gelu_f16", "rq16res"):
+        pytest.skip("the large case runs the encoder's forms only")
+    A = synth.uniform_int(11, f"Af{M}{K}", (M, K), -127, 127, np.int8)
+    I0 = 700
+    W, b, m, s = synth.gemm_params(11, f"Wf{N}{K}", N, K, 73.0, 2.0 * I0 if kind.startswith("gelu") else 40.0)
+    Wp = ilw.pack_weight(dev(W))
+    Ad = dev(A.astype(np.float16))
+    F16 = ilw.I8_IN_F16
+    if kind.startswith("gelu"):
+        m_g, s_g = 3 << 29, 40
+        got = ilw.gemm(Ad, Wp, N, dev(b), dev(m), dev(s), F16 if kind == "gelu_f16" else 8, gelu={"I0": I0},
+                       m_g=m_g, s_g=s_g)
+        gi = orc.sdshiftgelu(orc.gemm_requant(A, W, b, m, s, 16), I0).astype(np.int64)
+        want = np.array([[orc.sat(orc.rq(int(v), m_g, s_g), 8) for v in row] for row in gi], np.int8) \
+            if M * N <= 1 << 20 else orc.requant(gi.astype(np.int32), m_g, s_g, out_bits=8)
+    elif kind == "rq16res":
+        res = synth.uniform_int(12, "resf", (M, N), -32767, 32767, np.int16)
+        got = ilw.gemm(Ad, Wp, N, dev(b), dev(m), dev(s), 16, res=dev(res), m_r=3 << 29, s_r=31)
+        want = orc.gemm_requant(A, W, b, m, s, 16, res, 3 << 29, 31)
+    else:
+        ob = {"rq8": 8, "f16": F16, "raw32": 32}[kind]
+        got = ilw.gemm(Ad, Wp, N, dev(b), dev(m), dev(s), ob)
+        want = orc.gemm_requant(A, W, b, m, s, 8 if ob == F16 else ob)
+    if kind in ("f16", "gelu_f16"):
+        assert got.dtype == torch.float16
+    assert_same(host(got), want, f"gemm fp16-A {kind}")
+
+
 # ------------------------------------------------------------------------------ Shiftmax rows
 @pytest.mark.parametrize("L", [1, 3, 4, 63, 64, 65, 128, 400, 1600, 1664, 2048, 2100])
 def test_shiftmax_rows(ilw, orc, L):
@@ -162,6 +196,18 @@ def test_int_layernorm(ilw, orc, C, in_bits, out_bits, iters):
     assert_same(host(got), want, f"ln C={C}")
 
 
+@pytest.mark.parametrize("C,in_bits", [(384, 16), (192, 32), (100, 16), (1000, 32)])
+def test_int_layernorm_f16_out(ilw, orc, C, in_bits):
+    """out_bits ILW_I8_IN_F16: the int8 outputs carried in float16 (the encoder's form)."""
+    rows = 1000
+    lim = (1 << 14) if in_bits == 32 else 32767
+    X = synth.uniform_int(9, f"lnf{C}", (rows, C), -lim, lim, np.int32 if in_bits == 32 else np.int16)
+    beta, mult, shift = synth.ln_params(9, f"lnpf{C}", C)
+    got = ilw.int_layernorm(dev(X), dev(beta), dev(mult), dev(shift), 10, ilw.I8_IN_F16)
+    assert got.dtype == torch.float16
+    assert_same(host(got), orc.int_layernorm(X, beta, mult, shift, 10, 8), f"ln f16 C={C}")
+
+
 # ------------------------------------------------------------------------------ attention
 @pytest.mark.parametrize("B,T,H,dh,win", [(1, 17, 1, 64, 0), (2, 64, 2, 64, 0), (1, 256, 3, 64, 0),
                                           (1, 300, 2, 32, 0), (2, 100, 2, 64, 2), (1, 1600, 1, 64, 2),
@@ -177,6 +223,17 @@ def test_attention(ilw, orc, B, T, H, dh, win, form):
         got = ilw.shiftmax_attn(q_dev, B, T, H, dh, win, smx, 3 << 29, 36)
         want = orc.attention(qkv, B, T, H, dh, win, smx, 3 << 29, 36)
         assert_same(host(got), want, f"attn T={T} win={win} I0={I0} {form}")
+
+
+@pytest.mark.parametrize("B,T,H,dh,win", [(2, 1600, 2, 64, 0), (2, 1600, 2, 64, 2), (1, 300, 8, 32, 0)])
+def test_attention_f16_output(ilw, orc, B, T, H, dh, win):
+    """o_form ILW_I8_IN_F16 with float16 q|k|v: the encoder block's launch form."""
+    d = H * dh
+    qkv = synth.uniform_int(13, f"qkvo{T}{dh}", (B * T, 3 * d), -127, 127, np.int8)
+    smx = {"I0": 6000, "k_inter": 16, "k_out": 8, "s_d": -1, "m_p": 4, "M_hw": 31}
+    got = ilw.shiftmax_attn(dev(qkv.astype(np.float16)), B, T, H, dh, win, smx, 3 << 29, 36, o_f16=True)
+    assert got.dtype == torch.float16
+    assert_same(host(got), orc.attention(qkv, B, T, H, dh, win, smx, 3 << 29, 36), f"attn f16 out T={T}")
 
 
 def test_attention_extreme_scores(ilw, orc):

@@ -199,3 +199,4 @@ def test_high_word_requantisation_forms():
             assert ((hi >> (s - 33)) + 1) >> 1 == exact
             assert (hi + (1 << (s - 33))) >> (s - 32) == exact
             assert -(2**31) <= hi + (1 << (s - 33)) < 2**31
+
