@@ -21,7 +21,8 @@
 //   warps 2-5   operand converters (int8 A only): int8 activation rows (smem) -> fp16 rows in the
 //               same 128-byte swizzled K-major layout TMA produces for the weights
 //   warps 6-13  epilogue: TMEM -> registers -> integer epilogue -> HBM, one row per thread and
-//               half of the tile's columns per warp
+//               half of the tile's columns per warp (fp16 A with 192-wide tiles: warps 2-13, a
+//               third of the columns each, since there is nothing to convert)
 // Two TMEM accumulator sets (when they fit) let the epilogue of tile i overlap the MMAs of tile
 // i+1.  With resident weights the grid is a multiple of the number of column blocks, so every
 // tile of a CTA uses the same BN rows of W and L2 serves only the activations.
@@ -80,12 +81,14 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
+// One try_wait; the waiting thread may be suspended (up to the hint, 20 us) until the phase completes,
+// so that waiting roles do not spin on the issue slots the epilogue needs.
 __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
-        "{\n .reg .pred P;\n mbarrier.try_wait.parity.shared::cta.b64 P, [%1], %2;\n selp.b32 %0, 1, 0, P;\n}\n"
+        "{\n .reg .pred P;\n mbarrier.try_wait.parity.shared::cta.b64 P, [%1], %2, %3;\n selp.b32 %0, 1, 0, P;\n}\n"
         : "=r"(ok)
-        : "r"(bar), "r"(parity)
+        : "r"(bar), "r"(parity), "r"(20000)
         : "memory");
     return ok != 0;
 }
@@ -244,6 +247,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     using SM = Smem<BN, AF16, WRES>;
     constexpr int kStage = SM::kStage;
+    // Epilogue warps: 8 (warps 6-13, two column parts per TMEM lane quarter), or, when A arrives in
+    // fp16 and the tile is 192 wide, the converters' warps too: 12 (warps 2-13, three parts of 64).
+    constexpr int NP = (AF16 && BN == 192) ? 3 : 2;
+    constexpr int EPI0 = NP == 3 ? 2 : 6;
+    constexpr int NWE = 4 * NP;
     uint8_t *wres = smem + STAGES * kStage;  // resident weights (WRES)
     uint64_t *bars = (uint64_t *)(wres + (WRES ? p.wres_bytes : 0));
     // barriers: full[S], a_ready[S], empty[S], acc_full[2], acc_empty[2], wfull
@@ -267,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(acc_full(b), 1);
-            mbar_init(acc_empty(b), 8);
+            mbar_init(acc_empty(b), NWE);
         }
         mbar_init(wfull, 1);
         *abort = 0;
@@ -287,9 +295,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     // sat8(rq(g * I_div(g); m_g, s_g)) (built once per parameter set by gelu_table_kernel) is
     // copied into shared memory here.
     int8_t *gtab = (int8_t *)((int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + 16 * BN);
-    if ((KIND == KIND_GELU8 || KIND == KIND_GELU_F16) && warp >= 6) {
-        for (int i = threadIdx.x - 192; i < 65536 / 16; i += 256) ((uint4 *)gtab)[i] = __ldg((const uint4 *)p.gelu_tab + i);
-        asm volatile("bar.sync 1, 256;" ::: "memory");  // the 8 epilogue warps only
+    if ((KIND == KIND_GELU8 || KIND == KIND_GELU_F16) && warp >= EPI0) {
+        for (int i = threadIdx.x - 32 * EPI0; i < 65536 / 16; i += 32 * NWE)
+            ((uint4 *)gtab)[i] = __ldg((const uint4 *)p.gelu_tab + i);
+        asm volatile("bar.sync 1, %0;" ::"r"(32 * NWE) : "memory");  // the epilogue warps only
     }
     const int acc_cols = p.nseg * BN;  // columns of one accumulator set
 
@@ -376,7 +385,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 tc_commit(acc_full(b));  // arrives once every MMA of this tile has completed
             }
         }
-    } else if (warp < 6) {
+    } else if (warp < EPI0) {
         // ---------------------------------------------------------------- operand converters
         if constexpr (!AF16) {  // fp16 A arrives in the MMA's operand layout: nothing to convert
             const int r = (warp - 2) * 32 + lane;  // row of the 128-row A tile
@@ -413,11 +422,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     conv_done:;
     } else {
         // ---------------------------------------------------------------- epilogue
-        // 8 warps: warp w reads TMEM lanes 32q..32q+31 (q = w % 4) and owns half h of the columns
-        constexpr int HALF = BN / 2;
-        const int q = warp & 3, h = (warp - 6) >> 2;
+        // NWE warps: warp w reads TMEM lanes 32q..32q+31 (q = w % 4) and owns part h of the columns
+        constexpr int HALF = BN / NP;  // columns of this warp in a tile
+        const int q = warp & 3, h = (warp - EPI0) >> 2;
         const EpiParams &ep = p.ep;
-        int32_t *s_bias = (int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + (warp - 6) * 4 * HALF;  // this warp's copy of
+        int32_t *s_bias = (int32_t *)(((uintptr_t)(tmem_slot + 4) + 15) & ~(uintptr_t)15) + (warp - EPI0) * 4 * HALF;  // this warp's copy of
         int32_t *s_mult = s_bias + HALF;                                       // the tile's per-column
         int32_t *s_shift = s_mult + HALF;                                      // epilogue parameters
         int32_t *s_rnd = s_shift + HALF;                                       // (rq_hi rounding constants)
@@ -877,21 +886,27 @@ cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t
     // 192-wide tiles when N splits evenly into them (fewer re-reads of A per flop), else 128
     if (gp.nb > 1) return run<128, 5, kMaxBranches>(gp, ep, s);
     if (gp.a_f16) {
-        // fp16 A: no conversion stage.  Weights resident in shared memory when the CTA's BN rows
-        // of W fit next to the A stages (K <= 1024); GELU tiles are 128 wide to leave room for
-        // its 64 KB table.
+        // fp16 A: no conversion stage, so 192-wide tiles get 12 epilogue warps.  Weights resident
+        // in shared memory when the CTA's BN rows of W fit next to the A stages (K <= 1024).
+        // GELU keeps its 64 KB table in shared memory, so its 192-wide tiles stream the weights.
+        // K > 1024 needs two accumulators per tile: 128-wide tiles keep two TMEM sets (overlap).
         const bool gelu = ep.kind == EPI_GELU;
         const int K = gp.br[0].K, nkb = (K + BK - 1) / BK;
-        const bool wide = !gelu && gp.N % 192 == 0 && gp.N >= 384;
-        if (K <= kSegK) {
-            if (wide && smem_bytes<192, 3, KIND_RQ8, true, true>(nkb * 192 * 128) <= kSmemMax)
-                return run<192, 3, 1, true, true>(gp, ep, s);
-            if (!wide && smem_bytes<128, 3, KIND_GELU8, true, true>(nkb * 128 * 128) <= kSmemMax)
+        const bool n192 = gp.N % 192 == 0 && gp.N >= 384;
+        if (gelu) {
+            if (n192) return run<192, 3, 1, true, false>(gp, ep, s);
+            if (K <= kSegK && smem_bytes<128, 3, KIND_GELU8, true, true>(nkb * 128 * 128) <= kSmemMax)
                 return run<128, 3, 1, true, true>(gp, ep, s);
+            return run<128, 3, 1, true, false>(gp, ep, s);
         }
-        if (gp.N % 192 == 0 && gp.N >= 384)
-            return gelu ? run<192, 3, 1, true, false>(gp, ep, s) : run<192, 4, 1, true, false>(gp, ep, s);
-        return gelu ? run<128, 3, 1, true, false>(gp, ep, s) : run<128, 5, 1, true, false>(gp, ep, s);
+        if (K <= kSegK) {
+            if (n192 && smem_bytes<192, 3, KIND_RQ8, true, true>(nkb * 192 * 128) <= kSmemMax)
+                return run<192, 3, 1, true, true>(gp, ep, s);
+            if (smem_bytes<128, 3, KIND_RQ8, true, true>(nkb * 128 * 128) <= kSmemMax)
+                return run<128, 3, 1, true, true>(gp, ep, s);
+            return n192 ? run<192, 4, 1, true, false>(gp, ep, s) : run<128, 5, 1, true, false>(gp, ep, s);
+        }
+        return run<128, 5, 1, true, false>(gp, ep, s);
     }
     if (gp.N % 192 == 0 && gp.N >= 768)
         return ep.kind == EPI_GELU ? run<192, 3, 1>(gp, ep, s) : run<192, 4, 1>(gp, ep, s);
