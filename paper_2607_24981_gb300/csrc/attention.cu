@@ -30,14 +30,14 @@ __device__ __forceinline__ void mma_f16(float (&c)[4], const uint32_t (&a)[4], u
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-// D = A B + C with C = {c0, c0, c1, c1} (rows g and g + 8 of the fragment): starts an accumulation
-// without a separate initialisation of D.
-__device__ __forceinline__ void mma_f16_init(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1, float c0,
-                                             float c1) {
+// D = A B + C with a separate C fragment: starts an accumulation from C without initialising D.
+// C is a fragment kept for the whole pass ({0,0,0,0} or {c0, c0, c1, c1} for rows g, g + 8).
+__device__ __forceinline__ void mma_f16_init(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1,
+                                             const float (&c)[4]) {
     asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%11,%11};\n"
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%11,%12,%13};\n"
         : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(c0), "f"(c1));
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(c[0]), "f"(c[1]), "f"(c[2]), "f"(c[3]));
 }
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
@@ -217,12 +217,13 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
             }
         }
     };
-    // c - s for this warp's 16 rows x the 64 keys of buffer `buf` (c0 for row g, c1 for row g + 8;
-    // exact integers in fp32, below 2^24 in magnitude)
-    auto scores = [&](int buf, float (&S)[8][4], float c0, float c1) {
-        const uint32_t ks_base = (uint32_t)__cvta_generic_to_shared(Ks[buf]);
+    // C - s for this warp's 16 rows x keys 32hf .. 32hf + 31 of buffer `buf` (C from the fragment cq;
+    // exact integers in fp32, below 2^24 in magnitude).  A key block is processed in two halves to
+    // keep the score fragments at 16 registers.
+    auto scores = [&](int buf, int hf, float (&S)[4][4], const float (&cq)[4]) {
+        const uint32_t ks_base = (uint32_t)__cvta_generic_to_shared(Ks[buf]) + (uint32_t)(32 * hf * LDH);
 #pragma unroll
-        for (int np = 0; np < 4; ++np) {      // pairs of n-tiles (16 keys)
+        for (int np = 0; np < 2; ++np) {      // pairs of n-tiles (16 keys)
 #pragma unroll
             for (int kp = 0; kp < KS; kp += 2) {  // pairs of k16 steps (32 dims)
                 // matrices: keys [16np + 8(i&1) ...], dims [16kp + 8(i>>1) ...]
@@ -232,8 +233,8 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
                 uint32_t r0, r1, r2, r3;
                 ldsm_x4(addr, r0, r1, r2, r3);  // r0: n-tile 2np, k lo; r1: 2np+1, k lo; r2, r3: k hi
                 if (kp == 0) {
-                    mma_f16_init(S[2 * np], qa[kp], r0, r2, c0, c1);
-                    mma_f16_init(S[2 * np + 1], qa[kp], r1, r3, c0, c1);
+                    mma_f16_init(S[2 * np], qa[kp], r0, r2, cq);
+                    mma_f16_init(S[2 * np + 1], qa[kp], r1, r3, cq);
                 } else {
                     mma_f16(S[2 * np], qa[kp], r0, r2);
                     mma_f16(S[2 * np + 1], qa[kp], r1, r3);
@@ -310,21 +311,25 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
 
     // ---- pass 1: exact row maxima (the MMAs give -s; max s = -min)
     float mn0 = 3.0e38f, mn1 = 3.0e38f;
+    const float cz[4] = {0.f, 0.f, 0.f, 0.f};
     sweep(false, true, false, [&](int kb, int buf, bool full) {
-        float S[8][4];
-        scores(buf, S, 0.f, 0.f);
-        if (full) {
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                mn0 = fminf(mn0, fminf(S[nt][0], S[nt][1]));
-                mn1 = fminf(mn1, fminf(S[nt][2], S[nt][3]));
-            }
-        } else {
+        for (int hf = 0; hf < 2; ++hf) {
+            float S[4][4];
+            scores(buf, hf, S, cz);
+            if (full) {
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                const int key = kb * KB + nt * 8 + 2 * t;
-                if (key < Tg) { mn0 = fminf(mn0, S[nt][0]); mn1 = fminf(mn1, S[nt][2]); }
-                if (key + 1 < Tg) { mn0 = fminf(mn0, S[nt][1]); mn1 = fminf(mn1, S[nt][3]); }
+                for (int nt = 0; nt < 4; ++nt) {
+                    mn0 = fminf(mn0, fminf(S[nt][0], S[nt][1]));
+                    mn1 = fminf(mn1, fminf(S[nt][2], S[nt][3]));
+                }
+            } else {
+#pragma unroll
+                for (int nt = 0; nt < 4; ++nt) {
+                    const int key = kb * KB + 32 * hf + nt * 8 + 2 * t;
+                    if (key < Tg) { mn0 = fminf(mn0, S[nt][0]); mn1 = fminf(mn1, S[nt][2]); }
+                    if (key + 1 < Tg) { mn0 = fminf(mn0, S[nt][1]); mn1 = fminf(mn1, S[nt][3]); }
+                }
             }
         }
     });
@@ -335,27 +340,31 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
     // ShiftExp(s - max) is read off the bits of (max + 2^23) - s (exact: integers below 2^23), which
     // the MMAs of passes 2 and 3 produce with C = max + 2^23
     const float mb0 = 8388608.0f - mn0, mb1 = 8388608.0f - mn1;
+    const float cmb[4] = {mb0, mb0, mb1, mb1};
     const ShiftExpC se = p.smx.se;
     auto sexp = [&](float d) { return shift_exp_bits<FASTQ>(__float_as_uint(d), se); };
 
     // ---- pass 2: S_sum = sum ShiftExp(s - max)
     uint64_t sum0 = 0, sum1 = 0;
     sweep(false, true, true, [&](int kb, int buf, bool full) {
-        float S[8][4];
-        scores(buf, S, mb0, mb1);
-        if (full) {
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                sum0 += (uint64_t)sexp(S[nt][0]) + sexp(S[nt][1]);
-                sum1 += (uint64_t)sexp(S[nt][2]) + sexp(S[nt][3]);
-            }
-        } else {
+        for (int hf = 0; hf < 2; ++hf) {
+            float S[4][4];
+            scores(buf, hf, S, cmb);
+            if (full) {
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                const int key = kb * KB + nt * 8 + 2 * t;
-                const bool v0 = key < Tg, v1 = key + 1 < Tg;
-                sum0 += (uint64_t)(v0 ? sexp(S[nt][0]) : 0u) + (v1 ? sexp(S[nt][1]) : 0u);
-                sum1 += (uint64_t)(v0 ? sexp(S[nt][2]) : 0u) + (v1 ? sexp(S[nt][3]) : 0u);
+                for (int nt = 0; nt < 4; ++nt) {
+                    sum0 += (uint64_t)sexp(S[nt][0]) + sexp(S[nt][1]);
+                    sum1 += (uint64_t)sexp(S[nt][2]) + sexp(S[nt][3]);
+                }
+            } else {
+#pragma unroll
+                for (int nt = 0; nt < 4; ++nt) {
+                    const int key = kb * KB + 32 * hf + nt * 8 + 2 * t;
+                    const bool v0 = key < Tg, v1 = key + 1 < Tg;
+                    sum0 += (uint64_t)(v0 ? sexp(S[nt][0]) : 0u) + (v1 ? sexp(S[nt][1]) : 0u);
+                    sum1 += (uint64_t)(v0 ? sexp(S[nt][2]) : 0u) + (v1 ? sexp(S[nt][3]) : 0u);
+                }
             }
         }
     });
@@ -373,49 +382,52 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
     sweep(true, false, false, [&](int kb, int buf, bool full) {
-        float S[8][4];
-        scores(buf, S, mb0, mb1);
-        uint32_t pa[4][4];  // A fragments of P for the 4 k16 steps (16 keys each)
         // P of one score: (I_exp F) >> sh, or its direct form from ShiftExp's parts
         auto pout0 = [&](float d) { return DIRECT ? smx_out_direct<FASTQ>(__float_as_uint(d), se, rn0.F, sh00)
                                                   : shiftmax_out(sexp(d), rn0); };
         auto pout1 = [&](float d) { return DIRECT ? smx_out_direct<FASTQ>(__float_as_uint(d), se, rn1.F, sh01)
                                                   : shiftmax_out(sexp(d), rn1); };
-        // n-tile nt covers keys 8nt..8nt+7 = half (nt & 1) of k16 step nt >> 1
-        if (full) {
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(pout0(S[nt][0]), pout0(S[nt][1]));  // row g
-                pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(pout1(S[nt][2]), pout1(S[nt][3]));  // row g + 8
-            }
-        } else {
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                const int key = kb * KB + nt * 8 + 2 * t;
-                const bool v0 = key < Tg, v1 = key + 1 < Tg;
-                const uint32_t p0 = v0 ? pout0(S[nt][0]) : 0u;
-                const uint32_t p1 = v1 ? pout0(S[nt][1]) : 0u;
-                const uint32_t p2 = v0 ? pout1(S[nt][2]) : 0u;
-                const uint32_t p3 = v1 ? pout1(S[nt][3]) : 0u;
-                pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(p0, p1);
-                pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(p2, p3);
-            }
-        }
         const uint32_t vs_base = (uint32_t)__cvta_generic_to_shared(Vs[buf]);
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-            // A fragment order for m16n8k16: {row g k lo, row g+8 k lo, row g k hi, row g+8 k hi}
-            const uint32_t a[4] = {pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3]};
+        for (int hf = 0; hf < 2; ++hf) {
+            float S[4][4];
+            scores(buf, hf, S, cmb);
+            uint32_t pa[2][4];  // A fragments of P for the half's 2 k16 steps (16 keys each)
+            // n-tile nt covers keys 8nt..8nt+7 of the half = half (nt & 1) of k16 step nt >> 1
+            if (full) {
 #pragma unroll
-            for (int np = 0; np < NT / 2; ++np) {
-                // V rows = keys 16kk.., cols = dims 16np..: transposed 8x8 matrices give B fragments
-                const int i = lane >> 3;
-                const uint32_t row = 16 * kk + 8 * (i & 1) + (lane & 7);
-                const uint32_t addr = vs_base + row * LDH + (16 * np + 8 * (i >> 1)) * 2;
-                uint32_t r0, r1, r2, r3;
-                ldsm_x4_t(addr, r0, r1, r2, r3);  // r0: k lo, n 16np..; r1: k hi, n 16np..; r2/r3: n 16np+8..
-                mma_f16(o[2 * np], a, r0, r1);
-                mma_f16(o[2 * np + 1], a, r2, r3);
+                for (int nt = 0; nt < 4; ++nt) {
+                    pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(pout0(S[nt][0]), pout0(S[nt][1]));  // row g
+                    pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(pout1(S[nt][2]), pout1(S[nt][3]));  // row g + 8
+                }
+            } else {
+#pragma unroll
+                for (int nt = 0; nt < 4; ++nt) {
+                    const int key = kb * KB + 32 * hf + nt * 8 + 2 * t;
+                    const bool v0 = key < Tg, v1 = key + 1 < Tg;
+                    const uint32_t p0 = v0 ? pout0(S[nt][0]) : 0u;
+                    const uint32_t p1 = v1 ? pout0(S[nt][1]) : 0u;
+                    const uint32_t p2 = v0 ? pout1(S[nt][2]) : 0u;
+                    const uint32_t p3 = v1 ? pout1(S[nt][3]) : 0u;
+                    pa[nt >> 1][(nt & 1) * 2 + 0] = u10x2_to_h2(p0, p1);
+                    pa[nt >> 1][(nt & 1) * 2 + 1] = u10x2_to_h2(p2, p3);
+                }
+            }
+#pragma unroll
+            for (int kk = 0; kk < 2; ++kk) {
+                // A fragment order for m16n8k16: {row g k lo, row g+8 k lo, row g k hi, row g+8 k hi}
+                const uint32_t a[4] = {pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3]};
+#pragma unroll
+                for (int np = 0; np < NT / 2; ++np) {
+                    // V rows = keys 32hf + 16kk.., cols = dims 16np..: transposed 8x8 matrices give B fragments
+                    const int i = lane >> 3;
+                    const uint32_t row = 32 * hf + 16 * kk + 8 * (i & 1) + (lane & 7);
+                    const uint32_t addr = vs_base + row * LDH + (16 * np + 8 * (i >> 1)) * 2;
+                    uint32_t r0, r1, r2, r3;
+                    ldsm_x4_t(addr, r0, r1, r2, r3);  // r0: k lo, n 16np..; r1: k hi, n 16np..; r2/r3: n 16np+8..
+                    mma_f16(o[2 * np], a, r0, r1);
+                    mma_f16(o[2 * np + 1], a, r2, r3);
+                }
             }
         }
     });
