@@ -14,6 +14,7 @@
 // score fragments of pass 3 are already laid out as the A operand of P V.
 #include <climits>
 #include <cstdint>
+#include <cstdlib>
 
 #include "ilw_kernels.h"
 
@@ -462,10 +463,26 @@ __global__ void __launch_bounds__(THREADS, 4) attn_kernel(const AttnParams p) {
 
 }  // namespace
 
-cudaError_t launch_attention(const AttnParams &p, cudaStream_t s) {
+// The tensor-memory kernel is used where it applies unless ILWDETR_ATTENTION_TC=0 is set in the
+// environment (read once per process), which selects the warp-MMA kernel for every problem.
+static bool attention_tc_enabled() {
+    static const bool on = [] {
+        const char *v = getenv("ILWDETR_ATTENTION_TC");
+        return !(v && v[0] == '0');
+    }();
+    return on;
+}
+
+cudaError_t launch_attention(const AttnParams &p0, cudaStream_t s) {
+    AttnParams p = p0;
+    p.status = status_word_ptr();
     const int G2 = p.nw > 1 ? p.nw * p.nw : 1;
     const int Tg = p.nw > 1 ? (p.grid_side / p.nw) * (p.grid_side / p.nw) : p.T;
     if (p.B == 0 || Tg == 0) return cudaSuccess;
+    if (attention_tc_enabled()) {
+        const cudaError_t e = launch_attention_tc(p, s);
+        if (e != cudaErrorNotSupported) return e;
+    }
     dim3 grid((Tg + QT - 1) / QT, p.H, p.B * G2);
     const bool fastq = p.smx.se.m32 != 0;
     // the direct output form needs per-row s_d and I_b F < 2^32 (m_p <= M_hw - 15), and sh >= k

@@ -117,8 +117,12 @@ struct AttnParams {
     void *O;           // int8, or fp16 holding the int8 values when o_f16
     int32_t o_f16;
     int64_t ld_o;      // elements
+    int *status;       // device status word (set by launch_attention)
 };
 cudaError_t launch_attention(const AttnParams &p, cudaStream_t s);
+// The tensor-memory (tcgen05) form for dh = 64 with fp16-carried q|k|v, 16-byte aligned rows and
+// windows of side <= 128; cudaErrorNotSupported when the problem is outside that.
+cudaError_t launch_attention_tc(const AttnParams &p, cudaStream_t s);
 
 // ---------------------------------------------------------------- deformable sampling
 struct DeformParams {
