@@ -188,6 +188,7 @@ struct TcArgs {
     int32_t kbk;   // keys per block: 64 (global) or R ws (windows)
     int32_t rpb;   // window rows per block R (windows)
     int32_t win;   // 1: 3-D window boxes
+    int32_t nq;    // query tiles per group
 };
 __device__ __forceinline__ uint32_t shr_clamp(uint32_t v, uint32_t n) {
     uint32_t r;
@@ -240,9 +241,24 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
     volatile int *abort = (volatile int *)(sm + TcSmem::kSlot + 4);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // CTA -> (query tile, head, group): the tiles of every group but its last come first, the last
+    // (possibly partial, hence shorter) tiles of all groups at the end, so they fill the last wave
+    int qt, head, z;
+    {
+        const int Z = p.B * p.nw * p.nw, L = blockIdx.x, F = (args.nq - 1) * p.H * Z;
+        if (L < F) {
+            qt = L % (args.nq - 1);
+            head = (L / (args.nq - 1)) % p.H;
+            z = L / ((args.nq - 1) * p.H);
+        } else {
+            qt = args.nq - 1;
+            head = (L - F) % p.H;
+            z = (L - F) / p.H;
+        }
+    }
     GroupTc gr;
     {
-        const int G2 = p.nw * p.nw, z = blockIdx.z, b = z / G2, w = z % G2;
+        const int G2 = p.nw * p.nw, b = z / G2, w = z % G2;
         gr.base = (int64_t)b * p.T;
         gr.nw = p.nw;
         gr.gs = p.grid_side;
@@ -251,7 +267,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         gr.wx = w % p.nw;
         gr.Tg = p.nw > 1 ? gr.ws * gr.ws : p.T;
     }
-    const int Tg = gr.Tg, q0 = blockIdx.x * TQ, hoff = blockIdx.y * 64, kbk = args.kbk;
+    const int Tg = gr.Tg, q0 = qt * TQ, hoff = head * 64, kbk = args.kbk;
     const int nkb = (Tg + kbk - 1) / kbk;
 
     if (threadIdx.x == 0) {
@@ -428,6 +444,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
     } else {
         // ------------------------------------------------------------------ softmax, one row per thread
         const int qw = warp & 3, cq = (warp - 4) >> 2, row = 32 * qw + lane, tok = q0 + row;
+        const bool live = q0 + 32 * qw < Tg;  // some row of this warp is a query of the group
         const uint32_t tlane = tmem + ((uint32_t)(32 * qw) << 16);
         float *red_max = (float *)(sm + TcSmem::kRedMax);
         uint64_t *red_sum = (uint64_t *)(sm + TcSmem::kRedSum);
@@ -473,9 +490,13 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     if (!ok) break;
                 }
                 const int kvalid = min(kbk, Tg - kb * kbk);
-#pragma unroll
+#pragma unroll 1
                 for (int h = 0; h < NCH; ++h) {
                     const int c0 = CPW * cq + 32 * h;  // first column of this load
+                    const int nvalid = kvalid - c0;    // valid columns of this load (may be <= 0 or > 32)
+                    // warp-uniform: a warp whose rows all lie past the group, or a load past the group's
+                    // keys, has nothing to compute (its P is zero, its other values unused)
+                    const bool work = live && nvalid > 0;
                     uint32_t s[32];
                     tld<32>(tlane + (uint32_t)(TKB * b + c0), s);
                     twait<32>(s);
@@ -484,7 +505,15 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                         __syncwarp();
                         if (lane == 0) bar_arrive(s_free(b));
                     }
-                    const int nvalid = kvalid - c0;  // valid columns of this load (may be <= 0 or > 32)
+                    if (!work) {
+                        if (pass == 2 && live) {
+                            uint8_t *prow = sm + TcSmem::kP + pb * kPB + (c0 >> 6) * (TQ * 128) + row * 128;
+                            const int k0 = (c0 & 63) >> 3;
+#pragma unroll
+                            for (int cc = 0; cc < 4; ++cc) *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                        }
+                        continue;
+                    }
                     const bool whole = nvalid >= 32;
                     if (pass == 0) {
                         float m = __uint_as_float(s[0]);
@@ -504,9 +533,10 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
 #pragma unroll
                             for (int c = 0; c < 32; ++c) e[c] = c < nvalid ? e[c] : 0u;
                         }
+                        // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits
                         uint64_t part = 0;
 #pragma unroll
-                        for (int c = 0; c < 32; c += 2) part += (uint64_t)e[c] + e[c + 1];
+                        for (int c = 0; c < 32; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
                         sum += part;
                     } else {
                         // P of the 32 keys as fp16 (exact integers below 1024): the bits of 1024 + P are
@@ -678,7 +708,8 @@ cudaError_t launch_attention_tc(const AttnParams &p, cudaStream_t s) {
     const bool fastq = p.smx.se.m32 != 0;
     const bool direct = p.smx.s_d < 0 && p.smx.m_p + 15 <= p.smx.M_hw && 32 - p.smx.k_out >= p.smx.se.k;
     const size_t smem = 1024 + TcSmem::kBytes;
-    dim3 grid((Tg + TQ - 1) / TQ, p.H, p.B * G2);
+    a.nq = (Tg + TQ - 1) / TQ;
+    const dim3 grid((unsigned)(a.nq * p.H * p.B * G2));
     if (fastq && direct) return launch_tc_kernel<true, true>(a, grid, smem, s);
     if (fastq) return launch_tc_kernel<true, false>(a, grid, smem, s);
     if (direct) return launch_tc_kernel<false, true>(a, grid, smem, s);
