@@ -30,6 +30,8 @@
 // status word, stops issuing work, drains the loads it issued and frees its TMEM.
 #include <cuda.h>
 
+#include <algorithm>
+#include <climits>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
@@ -890,21 +892,39 @@ cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t
         // in shared memory when the CTA's BN rows of W fit next to the A stages (K <= 1024).
         // GELU keeps its 64 KB table in shared memory, so its 192-wide tiles stream the weights.
         // K > 1024 needs two accumulators per tile: 128-wide tiles keep two TMEM sets (overlap).
+        // Without GELU, among the shapes that fit, the one whose busiest CTA has the fewest output
+        // columns to produce wins (tiles are uniform work, so wave quantisation decides; ties go to
+        // the wider tile, which re-reads A less).
         const bool gelu = ep.kind == EPI_GELU;
         const int K = gp.br[0].K, nkb = (K + BK - 1) / BK;
         const bool n192 = gp.N % 192 == 0 && gp.N >= 384;
-        if (gelu) {
+        const int64_t tiles_m = (gp.M + BM - 1) / BM;
+        auto cost = [&](int bn, bool wres) -> int64_t {  // output columns of the busiest CTA, per row block
+            const int64_t tiles_n = (gp.N + bn - 1) / bn, sms = num_sms();
+            if (wres) {
+                int64_t per_n = sms / tiles_n;
+                per_n = per_n < 1 ? 1 : (per_n > tiles_m ? tiles_m : per_n);
+                return (tiles_m + per_n - 1) / per_n * bn;
+            }
+            const int64_t tiles = tiles_m * tiles_n, grid = tiles < sms ? tiles : sms;
+            return (tiles + grid - 1) / grid * bn;
+        };
+        if (gelu) {  // 192-wide measured faster inside the encoder step even at 6 vs 8 rounds (FC1)
             if (n192) return run<192, 3, 1, true, false>(gp, ep, s);
             if (K <= kSegK && smem_bytes<128, 3, KIND_GELU8, true, true>(nkb * 128 * 128) <= kSmemMax)
                 return run<128, 3, 1, true, true>(gp, ep, s);
             return run<128, 3, 1, true, false>(gp, ep, s);
         }
         if (K <= kSegK) {
-            if (n192 && smem_bytes<192, 3, KIND_RQ8, true, true>(nkb * 192 * 128) <= kSmemMax)
-                return run<192, 3, 1, true, true>(gp, ep, s);
-            if (smem_bytes<128, 3, KIND_RQ8, true, true>(nkb * 128 * 128) <= kSmemMax)
-                return run<128, 3, 1, true, true>(gp, ep, s);
-            return n192 ? run<192, 4, 1, true, false>(gp, ep, s) : run<128, 5, 1, true, false>(gp, ep, s);
+            const bool w192 = n192 && smem_bytes<192, 3, KIND_RQ8, true, true>(nkb * 192 * 128) <= kSmemMax;
+            const bool w128 = smem_bytes<128, 3, KIND_RQ8, true, true>(nkb * 128 * 128) <= kSmemMax;
+            const int64_t c192w = w192 ? cost(192, true) : INT64_MAX, c128w = w128 ? cost(128, true) : INT64_MAX,
+                          c192 = n192 ? cost(192, false) : INT64_MAX, c128 = cost(128, false);
+            const int64_t best = std::min(std::min(c192w, c128w), std::min(c192, c128));
+            if (c192w == best) return run<192, 3, 1, true, true>(gp, ep, s);
+            if (c192 == best) return run<192, 4, 1, true, false>(gp, ep, s);
+            if (c128w == best) return run<128, 3, 1, true, true>(gp, ep, s);
+            return run<128, 5, 1, true, false>(gp, ep, s);
         }
         return run<128, 5, 1, true, false>(gp, ep, s);
     }
