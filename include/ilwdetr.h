@@ -52,7 +52,8 @@ const char *ilwdetr_version(void);
 /* Message of the last failing call on this thread ("" if none). */
 const char *ilwdetr_last_error(void);
 /* Synchronises `stream`, then reads and clears the device status word of the current device:
- * ILW_OK, or ILW_ERR_TIMEOUT if a kernel gave up a bounded wait since the last read. */
+ * ILW_OK, ILW_ERR_TIMEOUT if a kernel gave up a bounded wait since the last read, or
+ * ILW_ERR_INVALID_ARG if ilwdetr_gather_rows met an index outside its source since then. */
 int ilwdetr_device_status(ilw_stream_t stream);
 
 /* Constrained Shiftmax parameters (Algorithm 2 inputs; Sec. 3.3.2).
@@ -359,6 +360,38 @@ int ilwdetr_decoder_layer_forward(const ilw_decoder_params_t *p, const int16_t *
                                   const int8_t *memory, const int32_t *level_hw, int32_t L,
                                   const int32_t *ref_q16, int32_t B, int32_t Q, int16_t *out,
                                   void *workspace, size_t workspace_bytes, ilw_stream_t stream);
+
+/* ------------------------------------------------------------------ detection head, two-stage selection */
+
+/* Integer sigmoid parameters.  1 <= I0 < 2^15, 0 <= k_inter <= 16, I0 * 2^(k_inter+1) < 2^31,
+ * 1 <= k_out <= 24. */
+typedef struct {
+    int32_t I0, k_inter, k_out;
+} ilw_sigmoid_t;
+
+/* Integer sigmoid of the detection head (Table 5: the head's exponential is ShiftExp), taken in
+ * the sign-dependent form of SD-ShiftGELU's sigmoid factor (Sec. 3.3.1, Algorithm 1) with the logit
+ * itself as the argument:
+ *   I_shift = ReLU(x), I_delta = x - I_shift, E = ShiftExp(I_delta), E' = ShiftExp(-I_shift),
+ *   Y = (E * floor((2^31 - 1) / (E + E'))) >> (32 - k_out)      (scale 2^-(k_out-1))
+ * X, Y int32 [n] device (may alias), 16-byte aligned. */
+int ilwdetr_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, const ilw_sigmoid_t *p, ilw_stream_t stream);
+
+/* ReLU of int8 values: Y = max(X, 0).  X, Y device [n] (may alias), 4-byte aligned. */
+int ilwdetr_relu_i8(const int8_t *X, int8_t *Y, int64_t n, ilw_stream_t stream);
+
+/* Integer top-K (two-stage query selection): for each of `rows` rows of S (int32, leading dimension
+ * lds), the K largest of its first N values in decreasing order, equal values ordered by
+ * increasing index.  vals, idx int32 [rows, K] device.  1 <= K <= N <= 16384. */
+int ilwdetr_topk(const int32_t *S, int64_t lds, int32_t rows, int32_t N, int32_t K, int32_t *vals,
+                 int32_t *idx, ilw_stream_t stream);
+
+/* Row gather: dst row i = src row idx[i], i < n (row_bytes bytes each; leading dimensions in
+ * bytes).  src, dst, idx device; row_bytes, src_ld, dst_ld multiples of 4, pointers 4-byte
+ * aligned.  An index outside [0, src_rows) gives a zero row and is reported by the next
+ * ilwdetr_device_status. */
+int ilwdetr_gather_rows(const void *src, int64_t src_ld, int64_t src_rows, const int32_t *idx, int64_t n,
+                        int64_t row_bytes, void *dst, int64_t dst_ld, ilw_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -128,6 +128,15 @@ def lib():
         L.orc_resample_nearest.restype = C.c_int
         L.orc_resample_nearest.argtypes = [i8p, C.c_int64, C.c_int32, C.c_int32, C.c_int32,
                                            C.c_int32, i8p, C.c_int64, C.c_int32, C.c_int32]
+        L.orc_int_sigmoid1.restype = C.c_int64
+        L.orc_int_sigmoid1.argtypes = [C.c_int64, C.c_int32, C.c_int32, C.c_int32]
+        L.orc_int_sigmoid.restype = C.c_int
+        L.orc_int_sigmoid.argtypes = [i32p, i32p, C.c_int64, C.c_int32, C.c_int32, C.c_int32]
+        L.orc_topk.restype = C.c_int
+        L.orc_topk.argtypes = [i32p, C.c_int64, C.c_int32, C.c_int32, C.c_int32, i32p, i32p]
+        L.orc_gather_rows.restype = C.c_int
+        L.orc_gather_rows.argtypes = [u8p, C.c_int64, C.c_int64, i32p, C.c_int64, C.c_int64, u8p,
+                                      C.c_int64]
         _lib = L
     return _lib
 
@@ -453,3 +462,79 @@ def decoder_layer(dp: dict, tgt: np.ndarray, pos: np.ndarray, memory: np.ndarray
     h = requant(gi, dp["m_g"], dp["s_g"], out_bits=8)
     x3 = gemm_requant(h, dp["w_fc2"], dp["b_fc2"], dp["m_fc2"], dp["s_fc2"], 16, t2, dp["m_r3"], dp["s_r3"])
     return int_layernorm(x3, dp["ln3_beta"], dp["ln3_mult"], dp["ln3_shift"], it, 16).astype(np.int16)
+
+
+# ---------------------------------------------------------------- detection head, two-stage selection
+def int_sigmoid1(x: int, I0: int, k_inter: int = 16, k_out: int = 8) -> int:
+    return int(lib().orc_int_sigmoid1(int(x), int(I0), int(k_inter), int(k_out)))
+
+
+def int_sigmoid(X: np.ndarray, I0: int, k_inter: int = 16, k_out: int = 8) -> np.ndarray:
+    """Integer sigmoid (Table 5's ShiftExp in the detection head, in SD-ShiftGELU's sign-dependent
+    form): int32 logits -> int32 outputs at scale 2^-(k_out-1), same shape."""
+    X32 = np.ascontiguousarray(X, dtype=np.int32)
+    Y = np.empty_like(X32)
+    _check(lib().orc_int_sigmoid(_p(X32, i32p), _p(Y, i32p), X32.size, I0, k_inter, k_out), "int_sigmoid")
+    return Y
+
+
+def topk(S: np.ndarray, K: int):
+    """Per row of the 2-D int32 S: the K largest values in decreasing order, equal values by
+    increasing index -> (values int32 [rows, K], indices int32 [rows, K])."""
+    S32 = np.ascontiguousarray(S, dtype=np.int32)
+    rows, N = S32.shape
+    vals = np.empty((rows, K), dtype=np.int32)
+    idx = np.empty((rows, K), dtype=np.int32)
+    _check(lib().orc_topk(_p(S32, i32p), N, rows, N, K, _p(vals, i32p), _p(idx, i32p)), "topk")
+    return vals, idx
+
+
+def gather_rows(X: np.ndarray, idx: np.ndarray) -> np.ndarray:
+    """Rows idx of the 2-D X (any integer type)."""
+    X = np.ascontiguousarray(X)
+    idx = np.ascontiguousarray(idx, dtype=np.int32).reshape(-1)
+    rb = X.shape[1] * X.itemsize
+    Y = np.empty((idx.size, X.shape[1]), dtype=X.dtype)
+    _check(lib().orc_gather_rows(X.view(np.uint8).ctypes.data_as(u8p), rb, X.shape[0], _p(idx, i32p),
+                                 idx.size, rb, Y.view(np.uint8).ctypes.data_as(u8p), rb), "gather_rows")
+    return Y
+
+
+def relu(X: np.ndarray) -> np.ndarray:
+    return np.maximum(X, 0).astype(X.dtype)
+
+
+def detection_head(hp: dict, out: np.ndarray, ref16: np.ndarray):
+    """Detection head on the decoder output (reading H2; Table 5: QuantLinear and ShiftExp):
+      class scores = IntSigmoid(Linear_cls(out))               (raw int32 logits, k_out = cls_k_out)
+      box logits   z = rq(Linear_3(ReLU(Linear_2(ReLU(Linear_1(out))))); m_d, s_d) + rq(ref16; m_ref, s_ref)
+      boxes        = IntSigmoid(z) with k_out = 17             (cx, cy, w, h at scale 2^-16)
+    ReLU acts on the int8 outputs of the hidden layers.  Returns (scores, boxes, z)."""
+    logits = gemm_requant(out, hp["w_cls"], hp["b_cls"], None, None, 32)
+    scores = int_sigmoid(logits, hp["cls_I0"], hp["k_inter"], hp["cls_k_out"])
+    h1 = relu(gemm_requant(out, hp["w_b1"], hp["b_b1"], hp["m_b1"], hp["s_b1"], 8).astype(np.int8))
+    h2 = relu(gemm_requant(h1, hp["w_b2"], hp["b_b2"], hp["m_b2"], hp["s_b2"], 8).astype(np.int8))
+    d = gemm_requant(h2, hp["w_b3"], hp["b_b3"], None, None, 32)
+    z = requant(d, hp["m_d"], hp["s_d"], ref16, hp["m_ref"], hp["s_ref"], out_bits=32)
+    boxes = int_sigmoid(z, hp["box_I0"], hp["k_inter"], 17)
+    return scores, boxes, z
+
+
+def two_stage(tp: dict, memory: np.ndarray, B: int, S: int, K: int):
+    """Two-stage query selection (reading H3): encoder class logits of every memory token,
+    the token's best class logit (top-1 over classes), the K best tokens of each image
+    (top-K, ties to the lower index), and their reference-box logits
+      ref16 = sat16(rq(Linear_2(ReLU(Linear_1(memory[token]))); m_d, s_d) + rq(anchor16[token]; m_a, s_a))
+    and the reference boxes IntSigmoid(ref16) (cx, cy, w, h at scale 2^-16; the decoder samples at
+    (cx, cy)).  Returns (values [B, K], token indices [B, K], ref16 [B*K, 4], boxes [B*K, 4])."""
+    enc = gemm_requant(memory, tp["w_enc"], tp["b_enc"], None, None, 32)
+    best, _ = topk(enc, 1)
+    vals, idx = topk(best.reshape(B, S), K)
+    rows = (idx + (np.arange(B, dtype=np.int32) * S)[:, None]).reshape(-1)
+    sel = gather_rows(memory, rows)
+    anc = gather_rows(tp["anchor16"], idx.reshape(-1))
+    h1 = relu(gemm_requant(sel, tp["w_p1"], tp["b_p1"], tp["m_p1"], tp["s_p1"], 8).astype(np.int8))
+    d = gemm_requant(h1, tp["w_p2"], tp["b_p2"], None, None, 32)
+    ref16 = requant(d, tp["m_d"], tp["s_d"], anc, tp["m_a"], tp["s_a"], out_bits=16)
+    boxes = int_sigmoid(ref16, tp["ref_I0"], tp["k_inter"], 17)
+    return vals, idx, ref16, boxes

@@ -14,6 +14,7 @@
 
 #include <cstdint>
 #include <cstdlib>
+#include <algorithm>
 #include <vector>
 
 namespace {
@@ -512,6 +513,63 @@ int orc_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int32_t 
                 int8_t *dst = Y + ((int64_t)b * y_bstride + (int64_t)y * Wo + x) * C;
                 for (int32_t c = 0; c < C; ++c) dst[c] = src[c];
             }
+    return 0;
+}
+
+// Integer sigmoid of the detection head.  Table 5 lists ShiftExp as the integer form of the
+// detection head's exponential; the sigmoid is taken in the sign-dependent form SD-ShiftGELU
+// uses for its sigmoid factor (Sec. 3.3.1, Algorithm 1), with the logit as the argument
+// (reading H1: no 1.702 factor):
+//   I_shift = ReLU(I); I_delta = I - I_shift
+//   E = ShiftExp(I_delta); E' = ShiftExp(-I_shift)
+//   F = floor((2^31 - 1) / (E + E')); out = (E F) >> (31 - k_out + 1)   (scale 2^-(k_out-1))
+int64_t orc_int_sigmoid1(int64_t x, int32_t I0, int32_t k_inter, int32_t k_out) {
+    int64_t Ish = x > 0 ? x : 0;
+    int64_t Id = x - Ish;
+    int64_t E = orc_shiftexp(Id, I0, k_inter);
+    int64_t E2 = orc_shiftexp(-Ish, I0, k_inter);
+    int64_t den = clamp64(E + E2, 1, kInt31Max);
+    int64_t F = kInt31Max / den;
+    return (int64_t)(((__int128)E * F) >> (31 - k_out + 1));
+}
+
+int orc_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, int32_t I0, int32_t k_inter,
+                    int32_t k_out) {
+    if (I0 < 1 || k_inter < 0 || k_inter > 30 || k_out < 1 || k_out > 24) return -1;
+    for (int64_t i = 0; i < n; ++i) Y[i] = (int32_t)orc_int_sigmoid1(X[i], I0, k_inter, k_out);
+    return 0;
+}
+
+// Integer top-K of the two-stage query selection (reading H3): the K largest values of each row,
+// in decreasing order, equal values ordered by increasing index (a deterministic order the
+// paper leaves open).  Plain selection: K times, the first index holding the largest value not
+// yet taken.
+int orc_topk(const int32_t *S, int64_t lds, int32_t rows, int32_t N, int32_t K, int32_t *vals,
+             int32_t *idx) {
+    if (rows < 0 || N < 1 || K < 1 || K > N) return -1;
+    std::vector<char> taken((size_t)N);
+    for (int32_t r = 0; r < rows; ++r) {
+        const int32_t *s = S + (int64_t)r * lds;
+        std::fill(taken.begin(), taken.end(), 0);
+        for (int32_t k = 0; k < K; ++k) {
+            int32_t best = -1;
+            for (int32_t j = 0; j < N; ++j)
+                if (!taken[(size_t)j] && (best < 0 || s[j] > s[best])) best = j;
+            taken[(size_t)best] = 1;
+            vals[(int64_t)r * K + k] = s[best];
+            idx[(int64_t)r * K + k] = best;
+        }
+    }
+    return 0;
+}
+
+int orc_gather_rows(const uint8_t *src, int64_t src_ld, int64_t src_rows, const int32_t *idx,
+                    int64_t n, int64_t row_bytes, uint8_t *dst, int64_t dst_ld) {
+    if (n < 0 || row_bytes < 0) return -1;
+    for (int64_t i = 0; i < n; ++i) {
+        if (idx[i] < 0 || idx[i] >= src_rows) return -1;
+        for (int64_t b = 0; b < row_bytes; ++b) dst[i * dst_ld + b] = src[(int64_t)idx[i] * src_ld + b];
+    }
     return 0;
 }
 

@@ -150,6 +150,22 @@ int orc_requant(const int32_t *X, int64_t ldx, int64_t rows, int64_t C, int32_t 
 int orc_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int32_t Hi, int32_t Wi,
                          int32_t C, int8_t *Y, int64_t y_bstride, int32_t Ho, int32_t Wo);
 
+/* Integer sigmoid of the detection head (Table 5: the head's exponential is ShiftExp), in the
+ * sign-dependent form of SD-ShiftGELU's sigmoid factor (Sec. 3.3.1, Algorithm 1) with the logit
+ * itself as the argument: out = (E F) >> (32 - k_out), scale 2^-(k_out-1). */
+int64_t orc_int_sigmoid1(int64_t x, int32_t I0, int32_t k_inter, int32_t k_out);
+int orc_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, int32_t I0, int32_t k_inter,
+                    int32_t k_out);
+
+/* Integer top-K (two-stage query selection): per row r of S [rows, lds], the K largest of its
+ * first N values in decreasing order, equal values by increasing index. */
+int orc_topk(const int32_t *S, int64_t lds, int32_t rows, int32_t N, int32_t K, int32_t *vals,
+             int32_t *idx);
+
+/* Row gather: dst row i = src row idx[i] (row_bytes bytes each; strides in bytes). */
+int orc_gather_rows(const uint8_t *src, int64_t src_ld, int64_t src_rows, const int32_t *idx,
+                    int64_t n, int64_t row_bytes, uint8_t *dst, int64_t dst_ld);
+
 #ifdef __cplusplus
 }
 #endif

@@ -16,7 +16,7 @@ __all__ = [
     "BlockWeights", "block_forward", "block_workspace_bytes", "device_status",
     "patch_embed", "patch_embed_workspace_bytes", "Backbone", "Graphed",
     "requant", "resample_nearest", "DecoderWeights", "decoder_workspace_bytes", "decoder_layer_forward",
-    "Projector", "Detector",
+    "Projector", "Detector", "int_sigmoid", "relu_i8", "topk", "gather_rows", "DetectionHead", "TwoStage",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -73,6 +73,10 @@ class GemmT(C.Structure):
 
 
 EPI_REQUANT, EPI_GELU = 0, 1
+
+
+class SigmoidT(C.Structure):
+    _fields_ = [("I0", C.c_int32), ("k_inter", C.c_int32), ("k_out", C.c_int32)]
 
 
 class DecoderParamsT(C.Structure):
@@ -141,6 +145,10 @@ SIGNATURES = {
     "ilwdetr_requant": ([_VP, _I32, _I64, _I64, _I32, _I32, _I32, _VP, _I64, _I64, _I32, _I32, _I32, _VP,
                          _I64, _VP], C.c_int),
     "ilwdetr_resample_nearest": ([_VP, _I64, _I32, _I32, _I32, _I32, _VP, _I64, _I32, _I32, _VP], C.c_int),
+    "ilwdetr_int_sigmoid": ([_VP, _VP, _I64, C.POINTER(SigmoidT), _VP], C.c_int),
+    "ilwdetr_relu_i8": ([_VP, _VP, _I64, _VP], C.c_int),
+    "ilwdetr_topk": ([_VP, _I64, _I32, _I32, _I32, _VP, _VP, _VP], C.c_int),
+    "ilwdetr_gather_rows": ([_VP, _I64, _I64, _VP, _I64, _I64, _VP, _I64, _VP], C.c_int),
     "ilwdetr_decoder_workspace_bytes": ([_I32, _I32, _I64, _I32, _I32, _I32, _I32, _I32], C.c_size_t),
     "ilwdetr_decoder_layer_forward": ([C.POINTER(DecoderParamsT), _VP, _VP, _VP, C.POINTER(_I32), _I32, _VP,
                                        _I32, _I32, _VP, _VP, C.c_size_t, _VP], C.c_int),
@@ -651,3 +659,126 @@ class Detector:
             x = decoder_layer_forward(dw, x, pos, memory, self.levels, refs, self.B, self.Q, self.ws,
                                       out=self.t[i % 2])
         return x
+
+
+# ---------------------------------------------------------------- detection head, two-stage selection
+def int_sigmoid(X, sig: dict, out=None):
+    """ilwdetr_int_sigmoid: int32 logits -> int32 sigmoid at scale 2^-(k_out-1) (same shape)."""
+    import torch
+
+    if out is None:
+        out = torch.empty_like(X)
+    p = SigmoidT(sig["I0"], sig.get("k_inter", 8), sig.get("k_out", 8))
+    _check(lib().ilwdetr_int_sigmoid(_ptr(X), _ptr(out), X.numel(), C.byref(p), _stream()), "int_sigmoid")
+    return out
+
+
+def relu_i8(X, out=None):
+    """ilwdetr_relu_i8: max(X, 0) on int8 (in place when out is X)."""
+    import torch
+
+    if out is None:
+        out = torch.empty_like(X)
+    _check(lib().ilwdetr_relu_i8(_ptr(X), _ptr(out), X.numel(), _stream()), "relu_i8")
+    return out
+
+
+def topk(S, K, vals=None, idx=None):
+    """ilwdetr_topk over the rows of the 2-D int32 S -> (values int32 [rows, K], indices int32 [rows, K])."""
+    import torch
+
+    rows, N = S.shape
+    if vals is None:
+        vals = torch.empty((rows, K), dtype=torch.int32, device=S.device)
+    if idx is None:
+        idx = torch.empty((rows, K), dtype=torch.int32, device=S.device)
+    _check(lib().ilwdetr_topk(_ptr(S), S.stride(0), rows, N, K, _ptr(vals), _ptr(idx), _stream()), "topk")
+    return vals, idx
+
+
+def gather_rows(X, idx, out=None):
+    """ilwdetr_gather_rows: rows idx (int32, any shape) of the 2-D X -> [idx.numel(), X.shape[1]]."""
+    import torch
+
+    n = idx.numel()
+    rb = X.shape[1] * X.element_size()
+    if out is None:
+        out = torch.empty((n, X.shape[1]), dtype=X.dtype, device=X.device)
+    _check(lib().ilwdetr_gather_rows(_ptr(X), X.stride(0) * X.element_size(), X.shape[0], _ptr(idx), n, rb,
+                                     _ptr(out), out.stride(0) * out.element_size(), _stream()), "gather_rows")
+    return out
+
+
+class DetectionHead:
+    """The detection head on the decoder output (``synth.head_params``): class scores by the integer
+    sigmoid of a linear layer's raw logits; box logits from a 3-layer integer MLP (ReLU on the int8
+    hidden outputs) added to the reference logits at one scale, and boxes (cx, cy, w, h at scale
+    2^-16) by the integer sigmoid.  Every step is an ilwdetr_* call."""
+
+    def __init__(self, hp: dict, device="cuda"):
+        import numpy as np
+        import torch
+
+        self.hp = hp
+        dv = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)  # noqa: E731
+        self.t = {k: dv(v) for k, v in hp.items() if isinstance(v, np.ndarray)}
+        for k in ("w_cls", "w_b1", "w_b2", "w_b3"):
+            self.t[k + "_p"] = pack_weight(self.t[k])
+        self.C = hp["w_cls"].shape[0]
+
+    def forward(self, out, ref16):
+        """out int8 [M, d] (decoder output), ref16 int16 [M, 4] (reference logits) ->
+        (scores int32 [M, C], boxes int32 [M, 4], box logits z int32 [M, 4])."""
+        hp, t = self.hp, self.t
+        d = out.shape[1]
+        logits = gemm_requant(out, t["w_cls_p"], self.C, t["b_cls"], None, None, 32)
+        scores = int_sigmoid(logits, {"I0": hp["cls_I0"], "k_inter": hp["k_inter"], "k_out": hp["cls_k_out"]})
+        h1 = gemm_requant(out, t["w_b1_p"], d, t["b_b1"], t["m_b1"], t["s_b1"], 8)
+        relu_i8(h1, out=h1)
+        h2 = gemm_requant(h1, t["w_b2_p"], d, t["b_b2"], t["m_b2"], t["s_b2"], 8)
+        relu_i8(h2, out=h2)
+        dlt = gemm_requant(h2, t["w_b3_p"], 4, t["b_b3"], None, None, 32)
+        z = requant(dlt, hp["m_d"], hp["s_d"], ref16, hp["m_ref"], hp["s_ref"], out_bits=32)
+        boxes = int_sigmoid(z, {"I0": hp["box_I0"], "k_inter": hp["k_inter"], "k_out": 17})
+        return scores, boxes, z
+
+
+class TwoStage:
+    """Two-stage query selection (``synth.two_stage_params``): encoder class logits of every
+    memory token, its best class logit (top-1), the K best tokens per image (top-K, ties to the
+    lower index), and their reference logits sat16(rq(MLP(memory[token])) + rq(anchor[token])) and
+    boxes (integer sigmoid, scale 2^-16).  Every step is an ilwdetr_* call."""
+
+    def __init__(self, tp: dict, device="cuda"):
+        import numpy as np
+        import torch
+
+        self.tp = tp
+        dv = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)  # noqa: E731
+        self.t = {k: dv(v) for k, v in tp.items() if isinstance(v, np.ndarray)}
+        for k in ("w_enc", "w_p1", "w_p2"):
+            self.t[k + "_p"] = pack_weight(self.t[k])
+
+    def forward(self, memory, B, S, K):
+        """memory int8 [B*S, d] -> (values [B, K], token indices [B, K], ref16 int16 [B*K, 4],
+        boxes int32 [B*K, 4])."""
+        import torch
+
+        tp, t = self.tp, self.t
+        d = memory.shape[1]
+        Cn = tp["w_enc"].shape[0]
+        enc = gemm_requant(memory, t["w_enc_p"], Cn, t["b_enc"], None, None, 32)
+        best, _ = topk(enc, 1)
+        vals, idx = topk(best.view(B, S), K)
+        # the selected tokens' memory rows and anchors, image by image (views of the batch)
+        sel = torch.empty((B * K, d), dtype=torch.int8, device=memory.device)
+        for b in range(B):
+            gather_rows(memory[b * S:(b + 1) * S], idx[b], out=sel[b * K:(b + 1) * K])
+        anc = gather_rows(t["anchor16"], idx.view(-1))
+        h1 = gemm_requant(sel, t["w_p1_p"], d, t["b_p1"], t["m_p1"], t["s_p1"], 8)
+        relu_i8(h1, out=h1)
+        dlt = gemm_requant(h1, t["w_p2_p"], 4, t["b_p2"], None, None, 32)
+        ref16 = requant(dlt, tp["m_d"], tp["s_d"], anc, tp["m_a"], tp["s_a"], out_bits=16)
+        ref32 = requant(ref16, 1 << 30, 30, out_bits=32)
+        boxes = int_sigmoid(ref32, {"I0": tp["ref_I0"], "k_inter": tp["k_inter"], "k_out": 17})
+        return vals, idx, ref16, boxes

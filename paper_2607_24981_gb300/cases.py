@@ -8,6 +8,8 @@ events, and prints the median (and minimum) device time with the case's algorith
   attn_global   attention, 2 images x 1600 tokens, 6 heads, dh 64, global (fp16-carried q|k|v);
                 --batch 8 gives the encoder's launch
   attn_window   attention, 8 images x 1600 tokens, 6 heads, 2x2 windows of 400
+  heads         detection head (class sigmoid, 3-layer box MLP, box sigmoid), 16 x 300 queries
+  two_stage     two-stage query selection, 16 images x 8400 memory tokens, top 300
   gemm_qkv / gemm_proj / gemm_fc1_gelu / gemm_fc2
                 the block GEMMs at 12800 tokens, d 384, MLP 1536
   ln_c2         I-LayerNorm on the int16 residual stream, 12800 x 384
@@ -92,6 +94,18 @@ def build(case: str, batch: int = 0):
         ob = ilw.I8_IN_F16 if case == "ln_c2" else 8
         Y = torch.empty(X.shape, dtype=torch.float16 if case == "ln_c2" else torch.int8, device="cuda")
         return (lambda: ilw.int_layernorm(X, beta, mult, shift, 10, ob, out=Y)), {"bytes": per * X.numel()}
+    if case == "heads":  # detection head on 16 images x 300 decoder queries, 80 classes
+        B, Q, d = batch or 16, 300, 256
+        head = ilw.DetectionHead(synth.head_params(8, d=d, C=80))
+        out = _dev(synth.uniform_int(8, "case.dh.out", (B * Q, d), -127, 127, np.int8))
+        ref = _dev(synth.uniform_int(8, "case.dh.ref", (B * Q, 4), -6000, 6000, np.int16))
+        return (lambda: head.forward(out, ref)), {"queries": B * Q}
+    if case == "two_stage":  # two-stage selection over 16 images x 8400 memory tokens, top 300
+        B, K, d = batch or 16, 300, 256
+        S = 8400
+        ts = ilw.TwoStage(synth.two_stage_params(9, d=d, C=80))
+        mem = _dev(synth.uniform_int(9, "case.ts.mem", (B * S, d), -127, 127, np.int8))
+        return (lambda: ts.forward(mem, B, S, K)), {"tokens": B * S}
     raise SystemExit(f"unknown case {case}")
 
 
@@ -123,6 +137,10 @@ def main(argv=None):
         out["gbs"] = work["bytes"] / (ms / 1000.0) / 1e9
     if "scores" in work:
         out["gscores_s"] = work["scores"] / (ms / 1000.0) / 1e9
+    if "queries" in work:
+        out["mqueries_s"] = work["queries"] / (ms / 1000.0) / 1e6
+    if "tokens" in work:
+        out["mtokens_s"] = work["tokens"] / (ms / 1000.0) / 1e6
     print(json.dumps(out), flush=True)
 
 

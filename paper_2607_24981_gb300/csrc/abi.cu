@@ -97,6 +97,7 @@ int ilwdetr_device_status(ilw_stream_t stream) {
     int v = 0;
     e = ilw::read_and_clear_status(&v);
     if (e != cudaSuccess) return cuda_status(e, "read device status");
+    if (v == ilw::kStatusBadIndex) return fail(ILW_ERR_INVALID_ARG, "a gather index lay outside its source rows");
     if (v) return fail(ILW_ERR_TIMEOUT, "a kernel's bounded wait expired (code %d)", v);
     return ILW_OK;
 }
@@ -585,6 +586,54 @@ int ilwdetr_decoder_layer_forward(const ilw_decoder_params_t *p, const int16_t *
     return ilwdetr_int_layernorm(b.x3, 16, d, M, d, p->ln3_beta, p->ln3_mult, p->ln3_shift, p->ln_iters, out, 16, d,
                                  stream);
 #undef ILW_TRY
+}
+
+// ---------------------------------------------------------------- detection head, two-stage selection
+int ilwdetr_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, const ilw_sigmoid_t *p, ilw_stream_t stream) {
+    if (!p) return fail(ILW_ERR_INVALID_ARG, "int_sigmoid: params NULL");
+    if (p->I0 < 1 || p->I0 >= (1 << 15)) return fail(ILW_ERR_INVALID_ARG, "int_sigmoid I0=%d outside [1, 2^15)", p->I0);
+    if (p->k_inter < 0 || p->k_inter > 16)
+        return fail(ILW_ERR_INVALID_ARG, "int_sigmoid k_inter=%d outside [0, 16]", p->k_inter);
+    if (((int64_t)p->I0 << (p->k_inter + 1)) >= ((int64_t)1 << 31))
+        return fail(ILW_ERR_INVALID_ARG, "int_sigmoid I0 * 2^(k_inter+1) must be < 2^31");
+    if (p->k_out < 1 || p->k_out > 24) return fail(ILW_ERR_INVALID_ARG, "int_sigmoid k_out=%d outside [1, 24]", p->k_out);
+    if (n < 0) return fail(ILW_ERR_INVALID_ARG, "int_sigmoid: n < 0");
+    if (n == 0) return ILW_OK;
+    if (!X || !Y || !aligned(X, 16) || !aligned(Y, 16))
+        return fail(ILW_ERR_INVALID_ARG, "int_sigmoid: NULL or not 16-byte aligned");
+    return cuda_status(ilw::launch_int_sigmoid(X, Y, n, ilw::make_shiftexp(p->I0, p->k_inter), p->k_out,
+                                               (cudaStream_t)stream),
+                       "int_sigmoid");
+}
+
+int ilwdetr_relu_i8(const int8_t *X, int8_t *Y, int64_t n, ilw_stream_t stream) {
+    if (n < 0) return fail(ILW_ERR_INVALID_ARG, "relu_i8: n < 0");
+    if (n == 0) return ILW_OK;
+    if (!X || !Y || !aligned(X, 4) || !aligned(Y, 4)) return fail(ILW_ERR_INVALID_ARG, "relu_i8: NULL or misaligned");
+    return cuda_status(ilw::launch_relu_i8(X, Y, n, (cudaStream_t)stream), "relu_i8");
+}
+
+int ilwdetr_topk(const int32_t *S, int64_t lds, int32_t rows, int32_t N, int32_t K, int32_t *vals, int32_t *idx,
+                 ilw_stream_t stream) {
+    if (rows < 0 || N < 1 || K < 1 || K > N || lds < N)
+        return fail(ILW_ERR_INVALID_ARG, "topk: bad sizes rows=%d N=%d K=%d", rows, N, K);
+    if (N > 16384) return fail(ILW_ERR_UNSUPPORTED, "topk: N=%d above 16384", N);
+    if (rows == 0) return ILW_OK;
+    if (!S || !vals || !idx || !aligned(S, 4) || !aligned(vals, 4) || !aligned(idx, 4))
+        return fail(ILW_ERR_INVALID_ARG, "topk: NULL or misaligned");
+    return cuda_status(ilw::launch_topk(S, lds, rows, N, K, vals, idx, (cudaStream_t)stream), "topk");
+}
+
+int ilwdetr_gather_rows(const void *src, int64_t src_ld, int64_t src_rows, const int32_t *idx, int64_t n,
+                        int64_t row_bytes, void *dst, int64_t dst_ld, ilw_stream_t stream) {
+    if (n < 0 || row_bytes < 0 || src_rows < 0 || row_bytes % 4 || src_ld % 4 || dst_ld % 4 || src_ld < row_bytes ||
+        dst_ld < row_bytes)
+        return fail(ILW_ERR_INVALID_ARG, "gather_rows: bad sizes (row bytes and strides multiples of 4)");
+    if (n == 0 || row_bytes == 0) return ILW_OK;
+    if (!src || !idx || !dst || !aligned(src, 4) || !aligned(dst, 4) || !aligned(idx, 4))
+        return fail(ILW_ERR_INVALID_ARG, "gather_rows: NULL or misaligned");
+    return cuda_status(ilw::launch_gather_rows(src, src_ld, src_rows, idx, n, row_bytes, dst, dst_ld, (cudaStream_t)stream),
+                       "gather_rows");
 }
 
 }  // extern "C"

@@ -18,6 +18,7 @@ constexpr int kStatusTimeoutTma = 1;     // a wait for a TMA load ran out
 constexpr int kStatusTimeoutMma = 2;     // a wait for tensor-core completion ran out
 constexpr int kStatusTimeoutOperand = 3; // a wait for the converted operand ran out
 constexpr int kStatusTimeoutFree = 4;    // a wait for a free pipeline stage ran out
+constexpr int kStatusBadIndex = 5;       // a gather index lay outside its source
 
 // Host-side construction of the per-launch ShiftExp constants (Algorithm 1).
 inline ShiftExpC make_shiftexp(int32_t I0, int32_t k) {
@@ -144,6 +145,15 @@ cudaError_t launch_patchify(const int8_t *img, int32_t B, int32_t Cin, int32_t H
                             int8_t *A, cudaStream_t s);
 cudaError_t launch_patchify_f16(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, int32_t Ww, int32_t p,
                                 __half *A, cudaStream_t s);
+
+// ---------------------------------------------------------------- detection head, two-stage selection
+cudaError_t launch_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, const ShiftExpC &se, int32_t k_out,
+                               cudaStream_t s);
+cudaError_t launch_relu_i8(const int8_t *X, int8_t *Y, int64_t n, cudaStream_t s);
+cudaError_t launch_topk(const int32_t *S, int64_t lds, int32_t rows, int32_t N, int32_t K, int32_t *vals,
+                        int32_t *idx, cudaStream_t s);
+cudaError_t launch_gather_rows(const void *src, int64_t src_ld_bytes, int64_t src_rows, const int32_t *idx, int64_t n,
+                               int64_t row_bytes, void *dst, int64_t dst_ld_bytes, cudaStream_t s);
 
 // ---------------------------------------------------------------- detector: requantisation, resampling
 struct RequantParams {

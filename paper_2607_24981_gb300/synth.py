@@ -269,3 +269,58 @@ def backbone_params(seed: int, cfg: dict) -> list:
         win = 0 if layer in cfg["global_layers"] else 2
         out.append(block_params(seed, layer, cfg["d"], cfg["H"], cfg["F"], win, cfg["mode"]))
     return out
+
+
+def head_params(seed: int, d: int = 256, C: int = 80, sigma_in: float = 32.0, k_inter: int = 8) -> dict:
+    """Integer parameters of the detection head: class linear layer (raw int32 logits of std ~2/S
+    with I0 = 1/S), box MLP d -> d -> d -> 4 (int8 hidden outputs of std ~32), box deltas
+    requantised to the reference-logit scale 2^-10 (std ~256, i.e. 0.25 in logit units) and the
+    int16 reference logits taken at that scale (identity requantisation)."""
+    p = "H."
+    hp: dict = {"k_inter": k_inter, "cls_k_out": 8}
+    acc_std = sigma_in * 73.3 * math.sqrt(d)  # U[-127, 127] weights: std 73.3
+    hp["w_cls"], hp["b_cls"], _, _ = gemm_params(seed, p + "cls", C, d, sigma_in, 1.0)
+    hp["cls_I0"] = int(min(acc_std / 2.0, (1 << 15) - 1))
+    hp["w_b1"], hp["b_b1"], hp["m_b1"], hp["s_b1"] = gemm_params(seed, p + "b1", d, d, sigma_in, 32.0)
+    hp["w_b2"], hp["b_b2"], hp["m_b2"], hp["s_b2"] = gemm_params(seed, p + "b2", d, d, 16.0, 32.0)
+    hp["w_b3"], hp["b_b3"], _, _ = gemm_params(seed, p + "b3", 4, d, 16.0, 1.0)
+    hp["m_d"] = _mult(seed, p + "d.m")
+    hp["s_d"] = _shift_for(16.0 * 73.3 * math.sqrt(d), 256.0)
+    hp["m_ref"], hp["s_ref"] = 1 << 30, 30
+    hp["box_I0"] = 1024
+    return hp
+
+
+def anchor_logits(levels=((80, 80), (40, 40), (20, 20)), scale: float = 1024.0) -> np.ndarray:
+    """Anchor boxes of every memory token as int16 logits at scale 1/`scale`: token (y, x) of
+    level l has cx = (x + 0.5) / W_l, cy = (y + 0.5) / H_l, w = h = 0.05 * 2^l; logit(p) =
+    log(p / (1 - p)), rounded half away from zero and clipped to int16 (host-side input
+    preparation, as the projector's anchors are fixed per resolution)."""
+    rows = []
+    for l, (H, W) in enumerate(levels):
+        ys, xs = np.meshgrid(np.arange(H), np.arange(W), indexing="ij")
+        cx = (xs.reshape(-1) + 0.5) / W
+        cy = (ys.reshape(-1) + 0.5) / H
+        wh = np.full(H * W, 0.05 * 2.0 ** l)
+        rows.append(np.stack([cx, cy, wh, wh], axis=1))
+    pr = np.concatenate(rows, axis=0)
+    lg = np.log(pr / (1.0 - pr)) * scale
+    lg = np.sign(lg) * np.floor(np.abs(lg) + 0.5)
+    return np.clip(lg, -32767, 32767).astype(np.int16)
+
+
+def two_stage_params(seed: int, d: int = 256, C: int = 80, levels=((80, 80), (40, 40), (20, 20)),
+                     sigma_in: float = 40.0, k_inter: int = 8) -> dict:
+    """Integer parameters of the two-stage query selection: encoder class linear layer (raw int32
+    logits), proposal MLP d -> d -> 4 with deltas requantised to the anchor-logit scale 2^-10, the
+    anchors (``anchor_logits``) and the sigmoid constants of the reference boxes."""
+    p = "TS."
+    tp: dict = {"k_inter": k_inter, "ref_I0": 1024}
+    tp["w_enc"], tp["b_enc"], _, _ = gemm_params(seed, p + "enc", C, d, sigma_in, 1.0)
+    tp["w_p1"], tp["b_p1"], tp["m_p1"], tp["s_p1"] = gemm_params(seed, p + "p1", d, d, sigma_in, 32.0)
+    tp["w_p2"], tp["b_p2"], _, _ = gemm_params(seed, p + "p2", 4, d, 16.0, 1.0)
+    tp["m_d"] = _mult(seed, p + "d.m")
+    tp["s_d"] = _shift_for(16.0 * 73.3 * math.sqrt(d), 256.0)
+    tp["anchor16"] = anchor_logits(levels)
+    tp["m_a"], tp["s_a"] = 1 << 30, 30
+    return tp

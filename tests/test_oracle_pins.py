@@ -663,3 +663,101 @@ def test_decoder_layer_images_are_independent(orc):
         one = orc.decoder_layer(dp, inp["tgt"][r], inp["pos"][r], mem[b * 80:(b + 1) * 80], levels,
                                 inp["refs"][b:b + 1], 1, Q)
         assert np.array_equal(one, out[r])
+
+
+# ----------------------------------------------------------------------------- detection head, two-stage
+@pytest.mark.parametrize("I0,k_inter", [(256, 8), (1024, 8), (5000, 8), (18764, 8), (1024, 12)])
+def test_int_sigmoid_follows_the_logistic_function(orc, I0, k_inter):
+    """Against 1 / (1 + e^-x) (x = I / I0) over the range ShiftExp does not clamp (|x| below
+    (k_inter - 1) ln 2): ShiftExp's linear fraction errs by at most ~6 % of E and the sigmoid
+    E / (E + E') by at most a quarter of that, so 0.02 absolute holds with margin; a swapped or
+    mis-signed term errs by up to 0.5.  Also non-decreasing everywhere, 0 at the far left."""
+    lim = int((k_inter - 1) * math.log(2.0) * I0)
+    xs = np.arange(-lim, lim + 1, max(1, I0 // 97), dtype=np.int64)
+    ys = orc.int_sigmoid(xs.astype(np.int32), I0, k_inter, 17).astype(np.float64) / 2 ** 16
+    assert np.abs(ys - 1.0 / (1.0 + np.exp(-xs / I0))).max() < 0.02
+    wide = np.concatenate([np.array([-(1 << 31), -(1 << 30)]), np.arange(-40 * I0, 40 * I0, I0 // 7 + 1),
+                           np.array([(1 << 30), (1 << 31) - 1])]).astype(np.int64)
+    yw = orc.int_sigmoid(wide.astype(np.int32), I0, k_inter, 17)
+    assert np.all(np.diff(yw.astype(np.int64)) >= 0)
+    assert 0 <= yw[0] <= 2 ** 16 * 2.0 ** -k_inter and yw[-1] <= 2 ** 16
+
+
+def test_int_sigmoid_halves_and_gelu_factor(orc):
+    """sigma(x) + sigma(-x): both share F = floor((2^31 - 1) / (E + E')), so the sum lies within
+    (E + E') / 2^(32 - k_out) + 1 below 2^(k_out - 1).  And SD-ShiftGELU's sigmoid factor of x is
+    this sigmoid of 1.702 x (x + x/2 + x/8 + x/16 by shifts, Algorithm 1)."""
+    I0, k, ko = 1024, 8, 17
+    den_max = 2 * I0 << k
+    rng = np.random.default_rng(5)
+    for x in [0, 1, 7, I0, 3 * I0] + [int(v) for v in rng.integers(0, 12 * I0, 300)]:
+        s = orc.int_sigmoid1(x, I0, k, ko) + orc.int_sigmoid1(-x, I0, k, ko)
+        assert 2 ** (ko - 1) - den_max // 2 ** (32 - ko) - 1 <= s <= 2 ** (ko - 1), x
+    for x in [int(v) for v in rng.integers(-(1 << 20), 1 << 20, 500)] + [0, -1, 1, -17, 17]:
+        ip = x + (x >> 1) + (x >> 3) + (x >> 4)
+        assert orc.sdshiftgelu_idiv(x, 600, 16, 8) == orc.int_sigmoid1(ip, 600, 16, 8)
+
+
+def test_topk_against_sorting(orc):
+    """Against numpy's lexicographic sort (value descending, index ascending); K = 1 against
+    argmax (first occurrence); K = N is the whole order; heavy ties and the int32 extremes."""
+    rng = np.random.default_rng(9)
+    S = rng.integers(-5, 6, size=(7, 300)).astype(np.int32)  # many ties
+    S[0, :4] = [np.iinfo(np.int32).min, np.iinfo(np.int32).max, np.iinfo(np.int32).max, 0]
+    for K in (1, 17, 300):
+        v, i = orc.topk(S, K)
+        for r in range(S.shape[0]):
+            order = np.lexsort((np.arange(S.shape[1]), -S[r].astype(np.int64)))[:K]
+            assert np.array_equal(i[r], order) and np.array_equal(v[r], S[r, order])
+    v1, i1 = orc.topk(S, 1)
+    assert np.array_equal(i1[:, 0], np.argmax(S, axis=1))
+
+
+def test_gather_rows_against_indexing(orc):
+    X = synth.uniform_int(3, "gr", (50, 12), -30000, 30000, np.int16)
+    idx = np.array([49, 0, 7, 7, 23], dtype=np.int32)
+    assert np.array_equal(orc.gather_rows(X, idx), X[idx])
+
+
+def _small_head(seed, M):
+    hp = synth.head_params(seed, d=64, C=16)
+    out = synth.uniform_int(seed, "hd.out", (M, 64), -127, 127, np.int8)
+    ref = synth.uniform_int(seed, "hd.ref", (M, 4), -4000, 4000, np.int16)
+    return hp, out, ref
+
+
+def test_detection_head_reduces_to_reference_sigmoid_and_is_rowwise(orc):
+    """With the box MLP's last layer zero (weights and bias), the box logits are the reference
+    logits and the boxes their sigmoid; the head treats each query alone (row permutation
+    equivariance); scores and boxes stay in [0, 2^(k_out-1)]."""
+    hp, out, ref = _small_head(4, 40)
+    scores, boxes, z = orc.detection_head(hp, out, ref)
+    assert scores.min() >= 0 and scores.max() <= 2 ** (hp["cls_k_out"] - 1)
+    assert boxes.min() >= 0 and boxes.max() <= 2 ** 16
+    perm = np.random.default_rng(2).permutation(40)
+    s2, b2, z2 = orc.detection_head(hp, out[perm], ref[perm])
+    assert np.array_equal(s2, scores[perm]) and np.array_equal(b2, boxes[perm])
+    hp0 = dict(hp, w_b3=np.zeros_like(hp["w_b3"]), b_b3=np.zeros_like(hp["b_b3"]))
+    _, b0, z0 = orc.detection_head(hp0, out, ref)
+    assert np.array_equal(z0, ref.astype(np.int32))
+    assert np.array_equal(b0, orc.int_sigmoid(ref.astype(np.int32), hp["box_I0"], hp["k_inter"], 17))
+
+
+def test_two_stage_selects_the_best_tokens(orc):
+    """The selected values are each image's K largest per-token best class logits (numpy max and
+    lexicographic sort of the oracle's raw logits); with the proposal MLP's last layer zero the
+    reference logits are the selected tokens' anchors."""
+    B, S, K, d = 2, 120, 20, 64
+    levels = ((8, 10), (4, 5), (2, 10))
+    tp = synth.two_stage_params(6, d=d, C=16, levels=levels)
+    mem = synth.uniform_int(6, "ts.mem", (B * S, d), -127, 127, np.int8)
+    vals, idx, ref16, boxes = orc.two_stage(tp, mem, B, S, K)
+    logits = orc.gemm_requant(mem, tp["w_enc"], tp["b_enc"], None, None, 32)
+    best = logits.max(axis=1).reshape(B, S).astype(np.int64)
+    for b in range(B):
+        order = np.lexsort((np.arange(S), -best[b]))[:K]
+        assert np.array_equal(idx[b], order) and np.array_equal(vals[b], best[b, order])
+    tp0 = dict(tp, w_p2=np.zeros_like(tp["w_p2"]), b_p2=np.zeros_like(tp["b_p2"]))
+    _, idx0, r0, _ = orc.two_stage(tp0, mem, B, S, K)
+    assert np.array_equal(r0, tp["anchor16"][idx0.reshape(-1)])
+    assert boxes.min() >= 0 and boxes.max() <= 2 ** 16
