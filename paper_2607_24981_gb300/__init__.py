@@ -631,10 +631,13 @@ class Projector:
 
 class Detector:
     """The full integer detector forward: Backbone (with its output layers tapped) -> Projector ->
-    decoder layers (ilwdetr_decoder_layer_forward), all on fixed device buffers."""
+    decoder layers (ilwdetr_decoder_layer_forward), all on fixed device buffers.  With two-stage
+    parameters (``synth.two_stage_params``) the decoder's reference points come from the two-stage
+    query selection over the memory; with head parameters (``synth.head_params``) the decoder output
+    is requantised to int8 and the detection head gives class scores and boxes."""
 
     def __init__(self, pe: dict, blocks: list, taps, pp: dict, dps: list, B: int, Q: int, levels, grid: int = 40,
-                 device="cuda"):
+                 tsp: dict | None = None, hp: dict | None = None, device="cuda"):
         import torch
 
         self.backbone = Backbone(pe, blocks, B, device=device)
@@ -649,16 +652,34 @@ class Detector:
         self.ws = torch.empty(decoder_workspace_bytes(B, Q, self.proj.S, d, dp0["F"], dp0["H"], dp0["L"], dp0["P"]),
                               dtype=torch.uint8, device=device)
         self.t = [torch.empty((B * Q, d), dtype=torch.int16, device=device) for _ in range(2)]
+        self.ts = TwoStage(tsp, device) if tsp is not None else None
+        self.head = DetectionHead(hp, device) if hp is not None else None
+        if self.ts is not None:
+            # (cx, cy) of each selected box: a gather of the first 8 bytes of every box row
+            self.ident = torch.arange(B * Q, dtype=torch.int32, device=device)
+            self.refs_buf = torch.empty((B, Q, 2), dtype=torch.int32, device=device)
 
-    def forward(self, img, tgt, pos, refs):
-        """img int8 [B, 3, H, W]; tgt, pos int16 [B*Q, d]; refs int32 [B, Q, 2] -> int16 [B*Q, d]."""
+    def forward(self, img, tgt, pos, refs=None, ref16=None):
+        """img int8 [B, 3, H, W]; tgt, pos int16 [B*Q, d]; refs int32 [B, Q, 2] (Q16 sampling points;
+        ignored with two-stage selection) -> int16 [B*Q, d], or, with a detection head, (that output,
+        class scores int32 [B*Q, C], boxes int32 [B*Q, 4]); ref16: int16 [B*Q, 4] reference logits
+        for the head when there is no two-stage selection."""
         self.backbone.forward(img, taps=dict(zip(self.taps, self.tap_buf)))
         memory = self.proj.forward(self.tap_buf)
+        if self.ts is not None:
+            _, _, ref16, boxes = self.ts.forward(memory, self.B, self.proj.S, self.Q)
+            gather_rows(boxes[:, :2], self.ident, out=self.refs_buf.view(self.B * self.Q, 2))
+            refs = self.refs_buf
         x = tgt
         for i, dw in enumerate(self.dec):
             x = decoder_layer_forward(dw, x, pos, memory, self.levels, refs, self.B, self.Q, self.ws,
                                       out=self.t[i % 2])
-        return x
+        if self.head is None:
+            return x
+        hp = self.head.hp
+        a = requant(x, hp["m_in"], hp["s_in"], out_bits=8)
+        scores, boxes, _ = self.head.forward(a, ref16)
+        return x, scores, boxes
 
 
 # ---------------------------------------------------------------- detection head, two-stage selection

@@ -288,6 +288,8 @@ def head_params(seed: int, d: int = 256, C: int = 80, sigma_in: float = 32.0, k_
     hp["s_d"] = _shift_for(16.0 * 73.3 * math.sqrt(d), 256.0)
     hp["m_ref"], hp["s_ref"] = 1 << 30, 30
     hp["box_I0"] = 1024
+    # the requantisation of the decoder's int16 output (std ~2^11) to the head's int8 input
+    hp["m_in"], hp["s_in"] = _mult(seed, p + "in.m"), _shift_for(2048.0, 32.0)
     return hp
 
 

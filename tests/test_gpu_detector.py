@@ -121,3 +121,45 @@ def test_detector_full_batch_sampled_image(ilw, orc):
         t = orc.decoder_layer(dp, t, inp["pos"][r], mem, cfg["levels"], inp["refs"][pick:pick + 1], 1, Q)
     same(out[r], t, f"detector image {pick}")
     assert 10 < float(np.abs(out.astype(np.int64)).mean()) < 30000
+
+
+def test_detector_two_stage_and_head_sampled_image(ilw, orc):
+    """The detector with two-stage query selection (the decoder's reference points from the top-300
+    memory tokens) and the detection head (class scores, boxes) at batch 2; the oracle recomputes
+    one image end to end (backbone, projector, two-stage selection, three decoder layers, head)."""
+    cfg = synth.CONFIGS["detector_c4"]
+    bb = synth.CONFIGS[cfg["backbone"]]
+    B, Q, g = 2, cfg["Q"], cfg["grid"]
+    blocks = synth.backbone_params(0, bb)
+    pe = synth.patch_embed_params(0, bb["d"], mode=bb["mode"])
+    pp = synth.projector_params(0, len(cfg["taps"]), bb["d"], cfg["N"])
+    dps = [synth.decoder_params(0, i) for i in range(cfg["dec_layers"])]
+    tsp = synth.two_stage_params(3, d=cfg["N"], C=80, levels=cfg["levels"])
+    hp = synth.head_params(3, d=cfg["N"], C=80)
+    inp = synth.decoder_inputs(1, B, Q)
+    img = synth.image_input(1, B)
+    det = ilw.Detector(pe, blocks, cfg["taps"], pp, dps, B, Q, cfg["levels"], g, tsp=tsp, hp=hp)
+    x, scores, boxes = det.forward(dev(img), dev(inp["tgt"]), dev(inp["pos"]))
+    x, scores, boxes = host(x), host(scores), host(boxes)
+    ilw.device_status()
+    pick = 1
+    xo = orc.patch_embed(img[pick:pick + 1], pe["p"], pe["w"], pe["b"], pe["m"], pe["s"], pe["pos"], pe["m_pos"],
+                         pe["s_pos"])
+    taps = {}
+    for i, bp in enumerate(blocks):
+        xo = orc.block_forward(bp, xo, 1, bb["T"])
+        if i in cfg["taps"]:
+            taps[i] = xo
+    mem = orc.projector(pp, [taps[i] for i in cfg["taps"]], 1, g, cfg["levels"])
+    S = mem.shape[0]
+    _, _, ref16, bx = orc.two_stage(tsp, mem, 1, S, Q)
+    refs = np.ascontiguousarray(bx[:, :2]).reshape(1, Q, 2)
+    r = slice(pick * Q, (pick + 1) * Q)
+    t = inp["tgt"][r]
+    for dp in dps:
+        t = orc.decoder_layer(dp, t, inp["pos"][r], mem, cfg["levels"], refs, 1, Q)
+    same(x[r], t, f"decoder output image {pick}")
+    a = orc.requant(t, hp["m_in"], hp["s_in"], out_bits=8)
+    ws, wb, _ = orc.detection_head(hp, a, ref16)
+    same(scores[r], ws, f"scores image {pick}")
+    same(boxes[r], wb, f"boxes image {pick}")
