@@ -17,6 +17,7 @@ __all__ = [
     "patch_embed", "patch_embed_workspace_bytes", "Backbone", "Graphed",
     "requant", "resample_nearest", "DecoderWeights", "decoder_workspace_bytes", "decoder_layer_forward",
     "Projector", "Detector", "int_sigmoid", "relu_i8", "topk", "gather_rows", "DetectionHead", "TwoStage",
+    "QueryPos",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -633,11 +634,13 @@ class Detector:
     """The full integer detector forward: Backbone (with its output layers tapped) -> Projector ->
     decoder layers (ilwdetr_decoder_layer_forward), all on fixed device buffers.  With two-stage
     parameters (``synth.two_stage_params``) the decoder's reference points come from the two-stage
-    query selection over the memory; with head parameters (``synth.head_params``) the decoder output
-    is requantised to int8 and the detection head gives class scores and boxes."""
+    query selection over the memory, and with positional-query parameters as well
+    (``synth.query_pos_params``) so do its positional queries (the learnable projection of the
+    selected boxes); with head parameters (``synth.head_params``) the decoder output is requantised
+    to int8 and the detection head gives class scores and boxes."""
 
     def __init__(self, pe: dict, blocks: list, taps, pp: dict, dps: list, B: int, Q: int, levels, grid: int = 40,
-                 tsp: dict | None = None, hp: dict | None = None, device="cuda"):
+                 tsp: dict | None = None, hp: dict | None = None, pq: dict | None = None, device="cuda"):
         import torch
 
         self.backbone = Backbone(pe, blocks, B, device=device)
@@ -658,18 +661,24 @@ class Detector:
             # (cx, cy) of each selected box: a gather of the first 8 bytes of every box row
             self.ident = torch.arange(B * Q, dtype=torch.int32, device=device)
             self.refs_buf = torch.empty((B, Q, 2), dtype=torch.int32, device=device)
+        self.qp = QueryPos(pq, B * Q, device) if (pq is not None and self.ts is not None) else None
+        if self.qp is not None:
+            self.pos_buf = torch.empty((B * Q, d), dtype=torch.int16, device=device)
 
-    def forward(self, img, tgt, pos, refs=None, ref16=None):
-        """img int8 [B, 3, H, W]; tgt, pos int16 [B*Q, d]; refs int32 [B, Q, 2] (Q16 sampling points;
-        ignored with two-stage selection) -> int16 [B*Q, d], or, with a detection head, (that output,
-        class scores int32 [B*Q, C], boxes int32 [B*Q, 4]); ref16: int16 [B*Q, 4] reference logits
-        for the head when there is no two-stage selection."""
+    def forward(self, img, tgt, pos=None, refs=None, ref16=None):
+        """img int8 [B, 3, H, W]; tgt, pos int16 [B*Q, d] (pos ignored with the positional-query
+        projection); refs int32 [B, Q, 2] (Q16 sampling points; ignored with two-stage selection)
+        -> int16 [B*Q, d], or, with a detection head, (that output, class scores int32 [B*Q, C],
+        boxes int32 [B*Q, 4]); ref16: int16 [B*Q, 4] reference logits for the head when there is
+        no two-stage selection."""
         self.backbone.forward(img, taps=dict(zip(self.taps, self.tap_buf)))
         memory = self.proj.forward(self.tap_buf)
         if self.ts is not None:
             _, _, ref16, boxes = self.ts.forward(memory, self.B, self.proj.S, self.Q)
             gather_rows(boxes[:, :2], self.ident, out=self.refs_buf.view(self.B * self.Q, 2))
             refs = self.refs_buf
+            if self.qp is not None:
+                pos = self.qp.forward(boxes, out=self.pos_buf)
         x = tgt
         for i, dw in enumerate(self.dec):
             x = decoder_layer_forward(dw, x, pos, memory, self.levels, refs, self.B, self.Q, self.ws,
@@ -803,3 +812,28 @@ class TwoStage:
         ref32 = requant(ref16, 1 << 30, 30, out_bits=32)
         boxes = int_sigmoid(ref32, {"I0": tp["ref_I0"], "k_inter": tp["k_inter"], "k_out": 17})
         return vals, idx, ref16, boxes
+
+
+class QueryPos:
+    """The learnable positional-query projection (``synth.query_pos_params``): Q16 boxes [M, 4] ->
+    int8 (requantised, zero-padded to 16 columns) -> linear 16 -> hidden, ReLU -> linear hidden -> d
+    -> int16 positional queries [M, d].  Every step is an ilwdetr_* call."""
+
+    def __init__(self, pq: dict, M: int, device="cuda"):
+        import numpy as np
+        import torch
+
+        self.pq, self.M = pq, M
+        dv = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)  # noqa: E731
+        self.t = {k: dv(v) for k, v in pq.items() if isinstance(v, np.ndarray)}
+        for k in ("w_q1", "w_q2"):
+            self.t[k + "_p"] = pack_weight(self.t[k])
+        self.hidden, self.d = pq["w_q1"].shape[0], pq["w_q2"].shape[0]
+        self.b8 = torch.zeros((M, 16), dtype=torch.int8, device=device)  # columns 4..15 stay zero
+
+    def forward(self, boxes, out=None):
+        pq, t = self.pq, self.t
+        requant(boxes, pq["m_box"], pq["s_box"], out_bits=8, out=self.b8[:, :4])
+        h = gemm_requant(self.b8, t["w_q1_p"], self.hidden, t["b_q1"], t["m_q1"], t["s_q1"], 8)
+        relu_i8(h, out=h)
+        return gemm_requant(h, t["w_q2_p"], self.d, t["b_q2"], t["m_q2"], t["s_q2"], 16, out=out)

@@ -125,8 +125,9 @@ def test_detector_full_batch_sampled_image(ilw, orc):
 
 def test_detector_two_stage_and_head_sampled_image(ilw, orc):
     """The detector with two-stage query selection (the decoder's reference points from the top-300
-    memory tokens) and the detection head (class scores, boxes) at batch 2; the oracle recomputes
-    one image end to end (backbone, projector, two-stage selection, three decoder layers, head)."""
+    memory tokens, its positional queries by the learnable projection of their boxes) and the
+    detection head (class scores, boxes) at batch 2; the oracle recomputes one image end to end
+    (backbone, projector, two-stage selection, positional queries, three decoder layers, head)."""
     cfg = synth.CONFIGS["detector_c4"]
     bb = synth.CONFIGS[cfg["backbone"]]
     B, Q, g = 2, cfg["Q"], cfg["grid"]
@@ -136,10 +137,11 @@ def test_detector_two_stage_and_head_sampled_image(ilw, orc):
     dps = [synth.decoder_params(0, i) for i in range(cfg["dec_layers"])]
     tsp = synth.two_stage_params(3, d=cfg["N"], C=80, levels=cfg["levels"])
     hp = synth.head_params(3, d=cfg["N"], C=80)
+    pq = synth.query_pos_params(3, d=cfg["N"])
     inp = synth.decoder_inputs(1, B, Q)
     img = synth.image_input(1, B)
-    det = ilw.Detector(pe, blocks, cfg["taps"], pp, dps, B, Q, cfg["levels"], g, tsp=tsp, hp=hp)
-    x, scores, boxes = det.forward(dev(img), dev(inp["tgt"]), dev(inp["pos"]))
+    det = ilw.Detector(pe, blocks, cfg["taps"], pp, dps, B, Q, cfg["levels"], g, tsp=tsp, hp=hp, pq=pq)
+    x, scores, boxes = det.forward(dev(img), dev(inp["tgt"]))
     x, scores, boxes = host(x), host(scores), host(boxes)
     ilw.device_status()
     pick = 1
@@ -154,12 +156,22 @@ def test_detector_two_stage_and_head_sampled_image(ilw, orc):
     S = mem.shape[0]
     _, _, ref16, bx = orc.two_stage(tsp, mem, 1, S, Q)
     refs = np.ascontiguousarray(bx[:, :2]).reshape(1, Q, 2)
+    pos = orc.query_pos(pq, bx)
     r = slice(pick * Q, (pick + 1) * Q)
     t = inp["tgt"][r]
     for dp in dps:
-        t = orc.decoder_layer(dp, t, inp["pos"][r], mem, cfg["levels"], refs, 1, Q)
+        t = orc.decoder_layer(dp, t, pos, mem, cfg["levels"], refs, 1, Q)
     same(x[r], t, f"decoder output image {pick}")
     a = orc.requant(t, hp["m_in"], hp["s_in"], out_bits=8)
     ws, wb, _ = orc.detection_head(hp, a, ref16)
     same(scores[r], ws, f"scores image {pick}")
     same(boxes[r], wb, f"boxes image {pick}")
+
+
+def test_query_pos(ilw, orc):
+    M = 600
+    pq = synth.query_pos_params(5)
+    boxes = synth.uniform_int(5, "qp.box", (M, 4), 0, 1 << 16)
+    boxes[:3] = [[0, 0, 0, 0], [1 << 16, 1 << 16, 1 << 16, 1 << 16], [32768, 1, 65535, 2]]
+    qp = ilw.QueryPos(pq, M)
+    same(host(qp.forward(dev(boxes))), orc.query_pos(pq, boxes), "query pos")

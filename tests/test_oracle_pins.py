@@ -761,3 +761,17 @@ def test_two_stage_selects_the_best_tokens(orc):
     _, idx0, r0, _ = orc.two_stage(tp0, mem, B, S, K)
     assert np.array_equal(r0, tp["anchor16"][idx0.reshape(-1)])
     assert boxes.min() >= 0 and boxes.max() <= 2 ** 16
+
+
+def test_query_pos_is_rowwise_and_ignores_padding(orc):
+    """The positional query of a box depends on that box alone (row permutation equivariance), and
+    the weight columns facing the 12 zero-padded input columns do not matter."""
+    pq = synth.query_pos_params(7, d=64, hidden=32)
+    boxes = synth.uniform_int(7, "qp.pin", (50, 4), 0, 1 << 16)
+    pos = orc.query_pos(pq, boxes)
+    perm = np.random.default_rng(3).permutation(50)
+    assert np.array_equal(orc.query_pos(pq, boxes[perm]), pos[perm])
+    w = pq["w_q1"].copy()
+    w[:, 4:] = synth.uniform_int(8, "qp.junk", (w.shape[0], 12), -127, 127, np.int8)
+    assert np.array_equal(orc.query_pos(dict(pq, w_q1=w), boxes), pos)
+    assert np.abs(pos.astype(np.int64)).mean() > 10
