@@ -377,6 +377,15 @@ typedef struct {
  * X, Y int32 [n] device (may alias), 16-byte aligned. */
 int ilwdetr_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, const ilw_sigmoid_t *p, ilw_stream_t stream);
 
+/* I-ViT's ShiftGELU, the baseline SD-ShiftGELU replaces (Sec. 3.3.1), over rows of L values: the
+ * sigmoid's exponentials after subtracting the row maximum of 1.702 x (clamped at 0):
+ *   I_p = x + (x >> 1) + (x >> 3) + (x >> 4); M = max(max_row I_p, 0);
+ *   E = ShiftExp(I_p - M), E' = ShiftExp(-M), I_div = (E floor((2^31-1)/(E + E'))) >> (32 - k_out),
+ *   Y = x I_div (int32; values must satisfy |x| 2^(k_out-1) < 2^31).
+ * X [rows, ldx], Y [rows, ldy] int32 device, 4-byte aligned, ldx, ldy >= L >= 1. */
+int ilwdetr_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int32_t L, int32_t *Y, int64_t ldy,
+                           const ilw_gelu_t *p, ilw_stream_t stream);
+
 /* ReLU of int8 values: Y = max(X, 0).  X, Y device [n] (may alias), 4-byte aligned. */
 int ilwdetr_relu_i8(const int8_t *X, int8_t *Y, int64_t n, ilw_stream_t stream);
 

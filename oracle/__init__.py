@@ -134,6 +134,9 @@ def lib():
         L.orc_int_sigmoid.argtypes = [i32p, i32p, C.c_int64, C.c_int32, C.c_int32, C.c_int32]
         L.orc_topk.restype = C.c_int
         L.orc_topk.argtypes = [i32p, C.c_int64, C.c_int32, C.c_int32, C.c_int32, i32p, i32p]
+        L.orc_ivit_shiftgelu.restype = C.c_int
+        L.orc_ivit_shiftgelu.argtypes = [i32p, C.c_int64, C.c_int64, C.c_int64, C.c_int32, C.c_int32,
+                                         C.c_int32, i32p, C.c_int64]
         L.orc_gather_rows.restype = C.c_int
         L.orc_gather_rows.argtypes = [u8p, C.c_int64, C.c_int64, i32p, C.c_int64, C.c_int64, u8p,
                                       C.c_int64]
@@ -549,3 +552,14 @@ def query_pos(pq: dict, boxes: np.ndarray) -> np.ndarray:
     bp[:, :4] = b8
     h = relu(gemm_requant(bp, pq["w_q1"], pq["b_q1"], pq["m_q1"], pq["s_q1"], 8).astype(np.int8))
     return gemm_requant(h, pq["w_q2"], pq["b_q2"], pq["m_q2"], pq["s_q2"], 16).astype(np.int16)
+
+
+def ivit_shiftgelu(X: np.ndarray, I0: int, k_inter: int = 16, k_out: int = 8) -> np.ndarray:
+    """I-ViT's ShiftGELU over the rows of the 2-D int32 X (row-maximum subtraction; Sec. 3.3.1's
+    baseline, reading H5) -> int32 I_x * I_div."""
+    X32 = np.ascontiguousarray(X, dtype=np.int32)
+    rows, L = X32.shape
+    Y = np.empty_like(X32)
+    _check(lib().orc_ivit_shiftgelu(_p(X32, i32p), L, rows, L, I0, k_inter, k_out, _p(Y, i32p), L),
+           "ivit_shiftgelu")
+    return Y

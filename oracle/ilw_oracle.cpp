@@ -573,4 +573,34 @@ int orc_gather_rows(const uint8_t *src, int64_t src_ld, int64_t src_rows, const 
     return 0;
 }
 
+// I-ViT's ShiftGELU, the baseline SD-ShiftGELU replaces (Sec. 3.3.1): sigma(z) = e^(z - M) /
+// (e^(z - M) + e^(-M)) with the vector-wise maximum M of the row, so that every ShiftExp input is
+// non-positive.  Reading H5: M is clamped at 0 (a row whose values are all negative has M = 0,
+// where the identity holds just the same and -M stays non-positive).
+int orc_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int64_t L, int32_t I0,
+                       int32_t k_inter, int32_t k_out, int32_t *Y, int64_t ldy) {
+    if (I0 < 1 || k_inter < 0 || k_inter > 30 || k_out < 1 || k_out > 16 || L < 1) return -1;
+    std::vector<int64_t> Ip((size_t)L);
+    for (int64_t r = 0; r < rows; ++r) {
+        const int32_t *x = X + r * ldx;
+        int64_t M = 0;
+        for (int64_t c = 0; c < L; ++c) {
+            const int64_t v = x[c];
+            Ip[(size_t)c] = v + (v >> 1) + (v >> 3) + (v >> 4);
+            if (Ip[(size_t)c] > M) M = Ip[(size_t)c];
+        }
+        const int64_t E2 = orc_shiftexp(-M, I0, k_inter);
+        for (int64_t c = 0; c < L; ++c) {
+            const int64_t E = orc_shiftexp(Ip[(size_t)c] - M, I0, k_inter);
+            const int64_t den = clamp64(E + E2, 1, kInt31Max);
+            const int64_t F = kInt31Max / den;
+            const int64_t idiv = (int64_t)(((__int128)E * F) >> (31 - k_out + 1));
+            const int64_t o = (int64_t)x[c] * idiv;
+            if (o < INT32_MIN || o > INT32_MAX) return -2;
+            Y[r * ldy + c] = (int32_t)o;
+        }
+    }
+    return 0;
+}
+
 }  // extern "C"

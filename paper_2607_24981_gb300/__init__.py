@@ -17,7 +17,7 @@ __all__ = [
     "patch_embed", "patch_embed_workspace_bytes", "Backbone", "Graphed",
     "requant", "resample_nearest", "DecoderWeights", "decoder_workspace_bytes", "decoder_layer_forward",
     "Projector", "Detector", "int_sigmoid", "relu_i8", "topk", "gather_rows", "DetectionHead", "TwoStage",
-    "QueryPos",
+    "QueryPos", "ivit_shiftgelu",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -148,6 +148,7 @@ SIGNATURES = {
     "ilwdetr_resample_nearest": ([_VP, _I64, _I32, _I32, _I32, _I32, _VP, _I64, _I32, _I32, _VP], C.c_int),
     "ilwdetr_int_sigmoid": ([_VP, _VP, _I64, C.POINTER(SigmoidT), _VP], C.c_int),
     "ilwdetr_relu_i8": ([_VP, _VP, _I64, _VP], C.c_int),
+    "ilwdetr_ivit_shiftgelu": ([_VP, _I64, _I64, _I32, _VP, _I64, C.POINTER(GeluT), _VP], C.c_int),
     "ilwdetr_topk": ([_VP, _I64, _I32, _I32, _I32, _VP, _VP, _VP], C.c_int),
     "ilwdetr_gather_rows": ([_VP, _I64, _I64, _VP, _I64, _I64, _VP, _I64, _VP], C.c_int),
     "ilwdetr_decoder_workspace_bytes": ([_I32, _I32, _I64, _I32, _I32, _I32, _I32, _I32], C.c_size_t),
@@ -837,3 +838,17 @@ class QueryPos:
         h = gemm_requant(self.b8, t["w_q1_p"], self.hidden, t["b_q1"], t["m_q1"], t["s_q1"], 8)
         relu_i8(h, out=h)
         return gemm_requant(h, t["w_q2_p"], self.d, t["b_q2"], t["m_q2"], t["s_q2"], 16, out=out)
+
+
+def ivit_shiftgelu(X, gelu: dict, out=None):
+    """ilwdetr_ivit_shiftgelu: I-ViT's ShiftGELU (row-maximum subtraction) over the rows of the 2-D
+    int32 X -> int32 x * I_div (the ablation baseline of SD-ShiftGELU)."""
+    import torch
+
+    rows, L = X.shape
+    if out is None:
+        out = torch.empty_like(X)
+    g = GeluT(gelu["I0"], gelu.get("k_inter", 16), gelu.get("k_out", 8))
+    _check(lib().ilwdetr_ivit_shiftgelu(_ptr(X), X.stride(0), rows, L, _ptr(out), out.stride(0), C.byref(g), _stream()),
+           "ivit_shiftgelu")
+    return out

@@ -636,4 +636,15 @@ int ilwdetr_gather_rows(const void *src, int64_t src_ld, int64_t src_rows, const
                        "gather_rows");
 }
 
+int ilwdetr_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int32_t L, int32_t *Y, int64_t ldy,
+                           const ilw_gelu_t *p, ilw_stream_t stream) {
+    int rc = check_gelu(p);
+    if (rc) return rc;
+    if (rows < 0 || L < 1 || ldx < L || ldy < L) return fail(ILW_ERR_INVALID_ARG, "ivit_shiftgelu: bad sizes");
+    if (rows == 0) return ILW_OK;
+    if (!X || !Y || !aligned(X, 4) || !aligned(Y, 4)) return fail(ILW_ERR_INVALID_ARG, "ivit_shiftgelu: NULL or misaligned");
+    return cuda_status(ilw::launch_ivit_shiftgelu(X, ldx, rows, L, Y, ldy, ilw::make_gelu(*p), (cudaStream_t)stream),
+                       "ivit_shiftgelu");
+}
+
 }  // extern "C"

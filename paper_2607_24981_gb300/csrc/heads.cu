@@ -128,6 +128,36 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(const uint32_t *__rest
     }
 }
 
+// I-ViT's ShiftGELU (the baseline of Sec. 3.3.1), one warp per row: M = max(max_row 1.702 x, 0),
+// E = ShiftExp(I_p - M), E' = ShiftExp(-M), I_div = (E F) >> out_sh, Y = x I_div.  1.702 x by shifts
+// in 64 bits (no int32 overflow for any input); ShiftExp magnitudes clamped at 2^30 (past k I0 the
+// result no longer changes).
+__device__ __forceinline__ int64_t ip1702(int32_t x) {
+    const int64_t v = x;
+    return v + (v >> 1) + (v >> 3) + (v >> 4);
+}
+__global__ void __launch_bounds__(256) ivit_shiftgelu_kernel(const int32_t *__restrict__ X, int64_t ldx, int64_t rows,
+                                                             int32_t L, int32_t *__restrict__ Y, int64_t ldy,
+                                                             ShiftExpC se, int32_t out_sh) {
+    const int lane = threadIdx.x & 31;
+    const int64_t wpr = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t r = blockIdx.x * (int64_t)(blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += wpr) {
+        const int32_t *x = X + r * ldx;
+        int64_t M = 0;
+        for (int c = lane; c < L; c += 32) M = max(M, ip1702(x[c]));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) M = max(M, (int64_t)__shfl_xor_sync(0xffffffffu, (long long)M, o));
+        const uint32_t e2 = shift_exp_mag((uint32_t)min(M, (int64_t)1 << 30), se);
+        for (int c = lane; c < L; c += 32) {
+            const int32_t v = x[c];
+            const uint32_t E = shift_exp_mag((uint32_t)min(M - ip1702(v), (int64_t)1 << 30), se);
+            const uint32_t F = div_int31(E + e2);
+            const int64_t idiv = (int64_t)(((uint64_t)E * F) >> out_sh);
+            Y[r * ldy + c] = (int32_t)((int64_t)v * idiv);
+        }
+    }
+}
+
 unsigned grid_for(int64_t work, int per_block) {
     const int64_t g = (work + per_block - 1) / per_block;
     return (unsigned)(g < 1 ? 1 : (g > 152 * 16 ? 152 * 16 : g));
@@ -139,6 +169,13 @@ cudaError_t launch_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, const Sh
                                cudaStream_t s) {
     if (n == 0) return cudaSuccess;
     int_sigmoid_kernel<<<grid_for((n + 3) / 4, 256), 256, 0, s>>>(X, Y, n, se, 32 - k_out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int32_t L, int32_t *Y, int64_t ldy,
+                                  const GeluC &c, cudaStream_t s) {
+    if (rows == 0) return cudaSuccess;
+    ivit_shiftgelu_kernel<<<grid_for((rows + 7) / 8, 1), 256, 0, s>>>(X, ldx, rows, L, Y, ldy, c.se, c.out_sh);
     return cudaGetLastError();
 }
 

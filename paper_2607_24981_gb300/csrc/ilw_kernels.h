@@ -150,6 +150,8 @@ cudaError_t launch_patchify_f16(const int8_t *img, int32_t B, int32_t Cin, int32
 cudaError_t launch_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, const ShiftExpC &se, int32_t k_out,
                                cudaStream_t s);
 cudaError_t launch_relu_i8(const int8_t *X, int8_t *Y, int64_t n, cudaStream_t s);
+cudaError_t launch_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int32_t L, int32_t *Y, int64_t ldy,
+                                  const GeluC &c, cudaStream_t s);
 cudaError_t launch_topk(const int32_t *S, int64_t lds, int32_t rows, int32_t N, int32_t K, int32_t *vals,
                         int32_t *idx, cudaStream_t s);
 cudaError_t launch_gather_rows(const void *src, int64_t src_ld_bytes, int64_t src_rows, const int32_t *idx, int64_t n,

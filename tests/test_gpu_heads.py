@@ -117,3 +117,14 @@ def test_two_stage(ilw, orc):
     same(host(vals), wv, "selected values")
     same(host(ref16), wr, "reference logits")
     same(host(boxes), wb, "reference boxes")
+
+
+@pytest.mark.parametrize("rows,L,I0,k_inter", [(300, 1536, 600, 16), (7, 1000, 1000, 8), (1, 5, 3, 16),
+                                               (64, 64, 20000, 0)])
+def test_ivit_shiftgelu(ilw, orc, rows, L, I0, k_inter):
+    X = synth.uniform_int(76, f"ivit{L}", (rows, L), -4 * I0, 4 * I0)
+    X[0, 0] = 40 * I0  # an outlier that drives the row maximum
+    if L >= 4:
+        X[-1, :4] = [(1 << 24) - 1, -(1 << 24) + 1, 0, -1]  # the domain's extremes (k_out 8)
+    got = ilw.ivit_shiftgelu(dev(X), {"I0": I0, "k_inter": k_inter, "k_out": 8})
+    same(host(got), orc.ivit_shiftgelu(X, I0, k_inter, 8), f"ivit shiftgelu {rows}x{L}")

@@ -775,3 +775,28 @@ def test_query_pos_is_rowwise_and_ignores_padding(orc):
     w[:, 4:] = synth.uniform_int(8, "qp.junk", (w.shape[0], 12), -127, 127, np.int8)
     assert np.array_equal(orc.query_pos(dict(pq, w_q1=w), boxes), pos)
     assert np.abs(pos.astype(np.int64)).mean() > 10
+
+
+def test_ivit_shiftgelu_reduces_to_sd_shiftgelu_without_positives(orc):
+    """On a row with no positive value the row maximum clamps to 0, E' = ShiftExp(0) and E =
+    ShiftExp(1.702 x): exactly SD-ShiftGELU's sign-dependent form for negative inputs."""
+    X = synth.uniform_int(11, "iv.neg", (20, 300), -(1 << 14), 0)
+    assert np.array_equal(orc.ivit_shiftgelu(X, 600, 16, 8), orc.sdshiftgelu(X, 600, 16, 8))
+
+
+def test_ivit_shiftgelu_error_grows_with_an_outlier(orc):
+    """The paper's case for SD-ShiftGELU (Sec. 3.3.1, Fig. 3): I-ViT's row-maximum subtraction pushes
+    the other elements of a row with one large value into ShiftExp's clamped, high-error region;
+    SD-ShiftGELU treats each element alone.  Against the erf GELU on the other elements: SD-ShiftGELU
+    is unchanged by the outlier and several times more accurate than I-ViT's form with it."""
+    I0 = 600
+    X = synth.uniform_int(12, "iv.row", (50, 512), -3 * I0, 3 * I0)
+    Xo = X.copy()
+    Xo[:, 0] = 60 * I0
+    erf = np.vectorize(math.erf)
+    ref = 0.5 * (X[:, 1:] / I0) * (1 + erf(X[:, 1:] / I0 / math.sqrt(2.0)))
+    err = lambda Y: np.abs(Y[:, 1:] / I0 / 2.0 ** 7 - ref).mean()  # noqa: E731
+    sd, sdo = orc.sdshiftgelu(X, I0, 8, 8), orc.sdshiftgelu(Xo, I0, 8, 8)
+    assert np.array_equal(sd[:, 1:], sdo[:, 1:])
+    assert err(sdo) < 0.03
+    assert err(orc.ivit_shiftgelu(Xo, I0, 8, 8)) > 5 * err(sdo)
