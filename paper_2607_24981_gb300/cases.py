@@ -1,6 +1,6 @@
 """Single-kernel workloads of the path, for timing and for profiler captures.
 
-  python -m paper_2607_24981_gb300.cases <case> [--reps N]
+  python -m paper_2607_24981_gb300.cases <case> [--reps N] [--graph]
 
 Each case builds its seeded inputs (shapes of the paper's Medium model and of the nonlinearity
 sweep), runs the entry point `reps` times after 3 warm-up calls, each launch timed with CUDA
@@ -116,8 +116,13 @@ def main(argv=None):
     ap.add_argument("case")
     ap.add_argument("--reps", type=int, default=10)
     ap.add_argument("--batch", type=int, default=0, help="images of the attention cases")
+    ap.add_argument("--graph", action="store_true", help="time replays of a CUDA graph of the case (no host gaps)")
     a = ap.parse_args(argv)
     fn, work = build(a.case, a.batch)
+    if a.graph:
+        import paper_2607_24981_gb300 as ilw
+
+        fn = ilw.Graphed(fn, warmup=2).replay
     for _ in range(3):
         fn()
     torch.cuda.synchronize()
@@ -130,7 +135,7 @@ def main(argv=None):
     torch.cuda.synchronize()
     times = sorted(e0.elapsed_time(e1) for e0, e1 in ev)
     ms = times[len(times) // 2]
-    out = {"case": a.case, "us": ms * 1000.0, "us_min": times[0] * 1000.0}
+    out = {"case": a.case, "us": ms * 1000.0, "us_min": times[0] * 1000.0, "graph": bool(a.graph)}
     if "flops" in work:
         out["tflops"] = work["flops"] / (ms / 1000.0) / 1e12
     if "bytes" in work:
