@@ -508,7 +508,7 @@ def relu(X: np.ndarray) -> np.ndarray:
 
 
 def detection_head(hp: dict, out: np.ndarray, ref16: np.ndarray):
-    """Detection head on the decoder output (reading H2; Table 5: QuantLinear and ShiftExp):
+    """Detection head on the decoder output (Table 5: QuantLinear and ShiftExp; the box refinement in the logit domain is a reading, as the paper gives no integer inverse sigmoid):
       class scores = IntSigmoid(Linear_cls(out))               (raw int32 logits, k_out = cls_k_out)
       box logits   z = rq(Linear_3(ReLU(Linear_2(ReLU(Linear_1(out))))); m_d, s_d) + rq(ref16; m_ref, s_ref)
       boxes        = IntSigmoid(z) with k_out = 17             (cx, cy, w, h at scale 2^-16)
@@ -524,7 +524,7 @@ def detection_head(hp: dict, out: np.ndarray, ref16: np.ndarray):
 
 
 def two_stage(tp: dict, memory: np.ndarray, B: int, S: int, K: int):
-    """Two-stage query selection (reading H3): encoder class logits of every memory token,
+    """Two-stage query selection (a reading of the two-stage pipeline of Sec. 3.1.2): encoder class logits of every memory token,
     the token's best class logit (top-1 over classes), the K best tokens of each image
     (top-K, ties to the lower index), and their reference-box logits
       ref16 = sat16(rq(Linear_2(ReLU(Linear_1(memory[token]))); m_d, s_d) + rq(anchor16[token]; m_a, s_a))
@@ -544,7 +544,7 @@ def two_stage(tp: dict, memory: np.ndarray, B: int, S: int, K: int):
 
 
 def query_pos(pq: dict, boxes: np.ndarray) -> np.ndarray:
-    """Learnable positional-query projection (Sec. 3.1.2, reading H4): int16 query_pos [M, d] =
+    """Learnable positional-query projection (Sec. 3.1.2; the layer sizes and the int8 box input are a reading): int16 query_pos [M, d] =
     sat16(rq(Linear_2(ReLU(sat8(rq(Linear_1(b)))))) with b = sat8(rq(box; m_box, s_box)), the Q16
     box [M, 4] requantised to int8 and zero-padded to 16 columns (the GEMM's K granularity)."""
     b8 = requant(boxes, pq["m_box"], pq["s_box"], out_bits=8)
@@ -556,7 +556,7 @@ def query_pos(pq: dict, boxes: np.ndarray) -> np.ndarray:
 
 def ivit_shiftgelu(X: np.ndarray, I0: int, k_inter: int = 16, k_out: int = 8) -> np.ndarray:
     """I-ViT's ShiftGELU over the rows of the 2-D int32 X (row-maximum subtraction; Sec. 3.3.1's
-    baseline, reading H5) -> int32 I_x * I_div."""
+    baseline; the row maximum is clamped at 0) -> int32 I_x * I_div."""
     X32 = np.ascontiguousarray(X, dtype=np.int32)
     rows, L = X32.shape
     Y = np.empty_like(X32)

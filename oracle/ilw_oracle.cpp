@@ -519,7 +519,7 @@ int orc_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int32_t 
 // Integer sigmoid of the detection head.  Table 5 lists ShiftExp as the integer form of the
 // detection head's exponential; the sigmoid is taken in the sign-dependent form SD-ShiftGELU
 // uses for its sigmoid factor (Sec. 3.3.1, Algorithm 1), with the logit as the argument
-// (reading H1: no 1.702 factor):
+// (a reading: no 1.702 factor):
 //   I_shift = ReLU(I); I_delta = I - I_shift
 //   E = ShiftExp(I_delta); E' = ShiftExp(-I_shift)
 //   F = floor((2^31 - 1) / (E + E')); out = (E F) >> (31 - k_out + 1)   (scale 2^-(k_out-1))
@@ -540,7 +540,7 @@ int orc_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, int32_t I0, int32_t
     return 0;
 }
 
-// Integer top-K of the two-stage query selection (reading H3): the K largest values of each row,
+// Integer top-K of the two-stage query selection: the K largest values of each row,
 // in decreasing order, equal values ordered by increasing index (a deterministic order the
 // paper leaves open).  Plain selection: K times, the first index holding the largest value not
 // yet taken.
@@ -575,7 +575,7 @@ int orc_gather_rows(const uint8_t *src, int64_t src_ld, int64_t src_rows, const 
 
 // I-ViT's ShiftGELU, the baseline SD-ShiftGELU replaces (Sec. 3.3.1): sigma(z) = e^(z - M) /
 // (e^(z - M) + e^(-M)) with the vector-wise maximum M of the row, so that every ShiftExp input is
-// non-positive.  Reading H5: M is clamped at 0 (a row whose values are all negative has M = 0,
+// non-positive.  A reading: M is clamped at 0 (a row whose values are all negative has M = 0,
 // where the identity holds just the same and -M stays non-positive).
 int orc_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int64_t L, int32_t I0,
                        int32_t k_inter, int32_t k_out, int32_t *Y, int64_t ldy) {

@@ -167,7 +167,7 @@ int orc_gather_rows(const uint8_t *src, int64_t src_ld, int64_t src_rows, const 
                     int64_t n, int64_t row_bytes, uint8_t *dst, int64_t dst_ld);
 
 /* I-ViT's ShiftGELU (the ablation baseline of Sec. 3.3.1): per row, the sigmoid's exponentials are
- * taken after subtracting the row maximum of 1.702 x (clamped at 0, reading H5):
+ * taken after subtracting the row maximum of 1.702 x (clamped at 0, a reading):
  *   I_p = 1.702 I_x (shifts); M = max(max_row I_p, 0); E = ShiftExp(I_p - M); E' = ShiftExp(-M);
  *   I_div = (E * floor((2^31 - 1) / (E + E'))) >> (32 - k_out); Y = I_x * I_div. */
 int orc_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int64_t L, int32_t I0,
