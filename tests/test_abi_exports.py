@@ -80,3 +80,26 @@ def test_host_side_validation_without_gpu(built_lib):
     assert rc == -2  # C % 4 != 0
     rc = L.ilwdetr_resample_nearest(ctypes.c_void_p(16), 100, 1, 10, 10, 24, ctypes.c_void_p(16), 400, 20, 20, None)
     assert rc == -2  # C % 16 != 0
+
+
+def test_detection_entry_points_validate_without_gpu(built_lib):
+    """The detection-head and selection entry points reject bad arguments before any launch."""
+    import paper_2607_24981_gb300 as ilw
+
+    L = ilw.lib()
+    p = ilw.SigmoidT(1 << 14, 16, 8)  # I0 * 2^(k+1) = 2^31: overflows the IntDiv denominator
+    assert L.ilwdetr_int_sigmoid(ctypes.c_void_p(16), ctypes.c_void_p(16), 4, ctypes.byref(p), None) == -1
+    p = ilw.SigmoidT(1024, 8, 25)  # k_out above 24: the output no longer fits int32
+    assert L.ilwdetr_int_sigmoid(ctypes.c_void_p(16), ctypes.c_void_p(16), 4, ctypes.byref(p), None) == -1
+    p = ilw.SigmoidT(1024, 8, 17)
+    assert L.ilwdetr_int_sigmoid(ctypes.c_void_p(20), ctypes.c_void_p(16), 4, ctypes.byref(p), None) == -1  # not 16 B
+    assert L.ilwdetr_topk(ctypes.c_void_p(16), 10, 2, 10, 11, ctypes.c_void_p(16), ctypes.c_void_p(16), None) == -1
+    assert L.ilwdetr_topk(ctypes.c_void_p(16), 20000, 1, 20000, 5, ctypes.c_void_p(16), ctypes.c_void_p(16),
+                          None) == -2  # past the shared-memory sort's 16384 keys
+    assert b"16384" in L.ilwdetr_last_error()
+    assert L.ilwdetr_gather_rows(ctypes.c_void_p(16), 12, 5, ctypes.c_void_p(16), 3, 6, ctypes.c_void_p(16), 12,
+                                 None) == -1  # 6-byte rows
+    assert L.ilwdetr_relu_i8(ctypes.c_void_p(17), ctypes.c_void_p(16), 8, None) == -1  # misaligned
+    g = ilw.GeluT(600, 16, 8)
+    assert L.ilwdetr_ivit_shiftgelu(ctypes.c_void_p(16), 4, 3, 8, ctypes.c_void_p(16), 8, ctypes.byref(g), None) == -1
+    assert L.ilwdetr_topk(ctypes.c_void_p(16), 10, 0, 10, 3, ctypes.c_void_p(16), ctypes.c_void_p(16), None) == 0
