@@ -200,3 +200,29 @@ def test_high_word_requantisation_forms():
             assert (hi + (1 << (s - 33))) >> (s - 32) == exact
             assert -(2**31) <= hi + (1 << (s - 33)) < 2**31
 
+
+
+def test_relu_on_packed_bytes():
+    """The int8 ReLU kernel clears each byte whose sign bit is set: w & ~(((w & 0x80808080) >> 7) *
+    0xFF) (the product has no carries: one low bit per byte), against bytewise max(0, b)."""
+    rng = np.random.default_rng(0)
+    w = rng.integers(0, 1 << 32, size=200000, dtype=np.uint64)
+    w[:4] = [0, 0xFFFFFFFF, 0x80808080, 0x7F7F7F7F]
+    neg = (w & np.uint64(0x80808080)) >> np.uint64(7)
+    got = w & ~(neg * np.uint64(0xFF)) & np.uint64(0xFFFFFFFF)
+    b = w.astype(np.uint32).view(np.int8).reshape(-1, 4)
+    want = np.maximum(b, 0).astype(np.int8).view(np.uint32).reshape(-1)
+    assert np.array_equal(got.astype(np.uint32), want)
+
+
+def test_topk_key_order():
+    """The top-K sort key (value biased to unsigned) << 32 | (2^32 - 1 - index), sorted in decreasing
+    order, is the order value descending, index ascending; padding keys (0) sort after every key."""
+    rng = np.random.default_rng(1)
+    v = rng.integers(-3, 4, size=5000).astype(np.int64)
+    v[:3] = [-(1 << 31), (1 << 31) - 1, -(1 << 31)]
+    i = np.arange(v.size, dtype=np.int64)
+    key = (((v + (1 << 31)) & 0xFFFFFFFF).astype(np.uint64) << np.uint64(32)) | (np.uint64(0xFFFFFFFF) - i.astype(np.uint64))
+    by_key = sorted(range(v.size), key=lambda j: -int(key[j]))  # exact 64-bit comparisons
+    assert by_key == list(np.lexsort((i, -v)))
+    assert int(key.min()) > 0
