@@ -226,3 +226,20 @@ def test_topk_key_order():
     by_key = sorted(range(v.size), key=lambda j: -int(key[j]))  # exact 64-bit comparisons
     assert by_key == list(np.lexsort((i, -v)))
     assert int(key.min()) > 0
+
+
+@pytest.mark.parametrize("nq,H,Z", [(1, 1, 1), (13, 6, 8), (4, 6, 32), (1, 8, 3), (2, 1, 5)])
+def test_attention_cta_order_is_a_bijection(nq, H, Z):
+    """The tensor-memory attention maps CTA L to (query tile, head, group): the first (nq - 1) H Z
+    CTAs take the tiles of every group but its last (tile fastest), the remaining H Z CTAs the last
+    tiles.  Every (tile, head, group) is taken exactly once, and the last tiles come last."""
+    F = (nq - 1) * H * Z
+    seen = []
+    for L in range(nq * H * Z):
+        if L < F:
+            t = (L % (nq - 1), (L // (nq - 1)) % H, L // ((nq - 1) * H))
+        else:
+            t = (nq - 1, (L - F) % H, (L - F) // H)
+        seen.append(t)
+    assert sorted(seen) == sorted((q, h, z) for q in range(nq) for h in range(H) for z in range(Z))
+    assert all(t[0] == nq - 1 for t in seen[F:]) and all(t[0] < nq - 1 for t in seen[:F])
