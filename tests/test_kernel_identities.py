@@ -243,3 +243,27 @@ def test_attention_cta_order_is_a_bijection(nq, H, Z):
         seen.append(t)
     assert sorted(seen) == sorted((q, h, z) for q in range(nq) for h in range(H) for z in range(Z))
     assert all(t[0] == nq - 1 for t in seen[F:]) and all(t[0] < nq - 1 for t in seen[:F])
+
+
+@pytest.mark.parametrize("ws", [1, 5, 7, 12, 20, 40, 64, 100, 128])
+def test_attention_window_key_boxes(ws):
+    """Window key blocks are 3-D boxes of R = min(floor(128 / ws), ws) whole window rows: row z,
+    column y of the box of block kb is grid cell (wy ws + kb R + z, wx ws + y), which is key
+    kb R ws + z ws + y of the window in row-major order; the blocks cover every key once and the
+    keys at or past ws^2 are the ones masked."""
+    R = min(128 // ws, ws)
+    kbk = R * ws
+    nkb = -(-ws * ws // kbk)
+    wy, wx = 1, 2
+    got = {}
+    for kb in range(nkb):
+        for z in range(R):
+            for y in range(ws):
+                key = kb * kbk + z * ws + y
+                cell = (wy * ws + kb * R + z, wx * ws + y)
+                if key < ws * ws:
+                    assert cell == (wy * ws + key // ws, wx * ws + key % ws)
+                    got[key] = cell
+                else:
+                    assert kb * R + z >= ws  # past the window: a masked column
+    assert sorted(got) == list(range(ws * ws)) and kbk <= 128
