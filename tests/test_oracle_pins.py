@@ -800,3 +800,26 @@ def test_ivit_shiftgelu_error_grows_with_an_outlier(orc):
     assert np.array_equal(sd[:, 1:], sdo[:, 1:])
     assert err(sdo) < 0.03
     assert err(orc.ivit_shiftgelu(Xo, I0, 8, 8)) > 5 * err(sdo)
+
+
+def test_ivit_shiftgelu_follows_gelu_on_moderate_rows(orc):
+    """Where no element pushes the row maximum far (|x| <= 1 in real units, so every ShiftExp input
+    stays above the clamp), I-ViT's form is a GELU too: mean |error| against the erf GELU below
+    0.02 (a sigmoid shifted by the row maximum, or missing the e^-M term, errs by ~0.1)."""
+    I0 = 600
+    X = synth.uniform_int(13, "iv.mid", (40, 256), -I0, I0)
+    erf = np.vectorize(math.erf)
+    ref = 0.5 * (X / I0) * (1 + erf(X / I0 / math.sqrt(2.0)))
+    for k in (12, 16):
+        assert np.abs(orc.ivit_shiftgelu(X, I0, k, 8) / I0 / 2.0 ** 7 - ref).mean() < 0.02
+
+
+def test_detection_scores_rise_with_the_class_logit(orc):
+    """Class scores are a non-decreasing function of the raw class logit out . w_c + b_c (numpy
+    int64 matmul), over all queries and classes together."""
+    hp, out, ref = _small_head(5, 60)
+    scores, _, _ = orc.detection_head(hp, out, ref)
+    logits = out.astype(np.int64) @ hp["w_cls"].astype(np.int64).T + hp["b_cls"].astype(np.int64)
+    order = np.argsort(logits.reshape(-1), kind="stable")
+    s = scores.reshape(-1)[order].astype(np.int64)
+    assert np.all(np.diff(s) >= 0) and s[-1] > s[0]
