@@ -680,6 +680,9 @@ class Detector:
             refs = self.refs_buf
             if self.qp is not None:
                 pos = self.qp.forward(boxes, out=self.pos_buf)
+        if pos is None or refs is None:
+            raise ValueError("Detector.forward: pos and refs are needed unless the two-stage selection "
+                             "(and, for pos, the positional-query projection) provides them")
         x = tgt
         for i, dw in enumerate(self.dec):
             x = decoder_layer_forward(dw, x, pos, memory, self.levels, refs, self.B, self.Q, self.ws,
