@@ -18,14 +18,17 @@
 //               layout); then one thread of warp 1 streams the key blocks as TMA pieces (k blocks
 //               in passes 1 and 2; k and v blocks in pass 3) into a 3-slot ring.  A key block is 128
 //               consecutive tokens (global attention: a 2-D box of the q|k|v matrix) or R whole
-//               rows of a ws x ws window, R = floor(128 / ws) (a 3-D box over (channel, x, y));
-//               the slot rows a window block leaves unwritten stay zero
+//               rows of a ws x ws window, R = min(floor(128 / ws), ws) (a 3-D box over (channel,
+//               x, y)); the slot rows a window block leaves unwritten stay zero
 //   warps 4-11  softmax: warp 4 + w reads TMEM lanes 32 (w % 4) .. + 31 (one query row per
 //               thread) and score columns 64 (w / 4) .. + 63 of each block (two 32-column loads);
 //               the two halves of a row combine their max and sum once per pass through shared
 //               memory; P rows go to shared memory as fp16 operands.  The score buffer is released
 //               as soon as the last load of a block has landed, so the next block's MMAs run
-//               while the softmax works
+//               while the softmax works.  Warps whose rows all lie past the group, and 32-key
+//               loads past its keys, skip the arithmetic (their P is written as zero)
+// The CTAs holding the last (possibly partial, hence shorter) query tile of each group come after
+// all the others, so they fill the last wave.
 // Every mbarrier wait is bounded (about one second); on expiry the kernel latches the device status
 // word, every role stops, the loaders drain their copies and the TMEM is freed after every MMA
 // issued has completed.
