@@ -6,10 +6,12 @@
  * use it.  It shares no code, header, table or helper with the CUDA path.
  *
  * Every function is written from the paper ("Enabling Fully Integer-Only Inference for
- * Lightweight Detection Transformers"): Sec. 3.2 (integer linear ops, split convolution),
- * Sec. 3.3 (I-LayerNorm, SD-ShiftGELU, Constrained Shiftmax), Algorithm 1 (ShiftExp,
- * SD-ShiftGELU) and Algorithm 2 (CalibrateShift, Constrained Shiftmax).  Where the paper is
- * silent the reading used is stated beside the function.
+ * Lightweight Detection Transformers"): Sec. 3.1 (nearest-neighbour deformable sampling, the
+ * two-stage pipeline), Sec. 3.2 (integer linear ops, split convolution), Sec. 3.3 (I-LayerNorm,
+ * SD-ShiftGELU and I-ViT's ShiftGELU it replaces, Constrained Shiftmax), Table 5 (the detection
+ * head's ShiftExp), Algorithm 1 (ShiftExp, SD-ShiftGELU) and Algorithm 2 (CalibrateShift,
+ * Constrained Shiftmax).  Where the paper is silent the reading used is stated beside the
+ * function.
  *
  * Conventions
  *   - All arithmetic is exact integer arithmetic in int64 (int128 where a product needs it).
