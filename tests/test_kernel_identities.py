@@ -267,3 +267,31 @@ def test_attention_window_key_boxes(ws):
                 else:
                     assert kb * R + z >= ws  # past the window: a masked column
     assert sorted(got) == list(range(ws * ws)) and kbk <= 128
+
+
+def _shift_exp_mag_model(a, I0, k):
+    """The kernels' ShiftExp of -a in 32-bit unsigned arithmetic (a <= 2^30): n = a + ceil(a/2) -
+    ceil(a/16), clamped at k I0; q = floor(n / I0); I_b = I0 - ceil(r / 2); I_b << (k - q)."""
+    a = np.asarray(a, dtype=np.uint64)
+    n = (a + ((a + 1) >> np.uint64(1)) - ((a + 15) >> np.uint64(4))) & np.uint64(0xFFFFFFFF)
+    n = np.minimum(n, np.uint64(k * I0))
+    q = n // np.uint64(I0)
+    r = n - q * np.uint64(I0)
+    Ib = np.uint64(I0) - ((r + 1) >> np.uint64(1))
+    return (Ib << (np.uint64(k) - q)).astype(np.int64)
+
+
+@pytest.mark.parametrize("I0,k", [(1, 0), (3, 16), (600, 8), (1024, 8), (18764, 8), (32767, 0)])
+def test_clamped_magnitude_shiftexp(orc, I0, k):
+    """The detection-head and I-ViT kernels clamp the ShiftExp magnitude at 2^30 before the 32-bit
+    form: past k I0 ShiftExp sits in its clamp region, so for every a >= 0 (up to 2^31 and the
+    int32 extreme) ShiftExp(-min(a, 2^30)) in the kernels' arithmetic equals Algorithm 1's
+    ShiftExp(-a)."""
+    rng = np.random.default_rng(I0)
+    edge = np.array([0, 1, 2, 15, 16, 17, k * I0 - 1, k * I0, k * I0 + 1, (1 << 30) - 1, 1 << 30,
+                     (1 << 30) + 1, (1 << 31) - 1, 1 << 31], dtype=np.int64)
+    a = np.concatenate([edge[edge >= 0], np.arange(0, 40 * I0 + 64, max(1, I0 // 50)),
+                        rng.integers(0, 1 << 31, 2000)])
+    got = _shift_exp_mag_model(np.minimum(a, 1 << 30), I0, k)
+    want = np.array([orc.shiftexp(-int(x), I0, k) for x in a], dtype=np.int64)
+    assert np.array_equal(got, want)
