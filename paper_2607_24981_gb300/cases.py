@@ -114,7 +114,7 @@ def main(argv=None):
 
     ap = argparse.ArgumentParser()
     ap.add_argument("case")
-    ap.add_argument("--reps", type=int, default=10)
+    ap.add_argument("--reps", type=int, default=20)
     ap.add_argument("--batch", type=int, default=0, help="images of the attention cases")
     ap.add_argument("--graph", action="store_true", help="time replays of a CUDA graph of the case (no host gaps)")
     a = ap.parse_args(argv)
