@@ -20,6 +20,10 @@
  *     that domain give unspecified results.
  *   - The caller passes integer parameters only (I0 = round(1/S), dyadic pairs, shifts): the
  *     float scales of calibration never reach the device.
+ *   - The library keeps a few arrays of its own in device memory (the status word, the
+ *     SD-ShiftGELU tables, the allocation-free patch scratch) and looks up their device
+ *     addresses once per device.  A cudaDeviceReset ends the context those addresses belong
+ *     to: do not call the library across one.
  */
 #ifndef ILWDETR_H
 #define ILWDETR_H
@@ -238,7 +242,9 @@ int ilwdetr_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, i
  *   - Batches needing more than that (B * (Hh/p) * (Ww/p) * Cin * p * p bytes; e.g. more than
  *     6 images of 3 x 640 x 640) are rejected with ILW_ERR_UNSUPPORTED and a message.
  *   - The first call on each device looks up the array's device address (cudaGetSymbolAddress)
- *     with that device current; make that first call before any stream capture.
+ *     with that device current; make that first call before any stream capture.  The address is
+ *     kept for the life of the process, so do not call this across a cudaDeviceReset.
+ *   - Every argument is checked before anything is launched; errors as ilwdetr_patch_embed.
  *   - All calls share the one array and it keeps the last call's contents (each call overwrites
  *     every byte it reads, so nothing needs clearing).  Calls whose execution overlaps on the
  *     GPU (other streams, other threads) race on it: serialise them. */

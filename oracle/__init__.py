@@ -545,12 +545,10 @@ def two_stage(tp: dict, memory: np.ndarray, B: int, S: int, K: int):
 
 def query_pos(pq: dict, boxes: np.ndarray) -> np.ndarray:
     """Learnable positional-query projection (Sec. 3.1.2; the layer sizes and the int8 box input are a reading): int16 query_pos [M, d] =
-    sat16(rq(Linear_2(ReLU(sat8(rq(Linear_1(b)))))) with b = sat8(rq(box; m_box, s_box)), the Q16
-    box [M, 4] requantised to int8 and zero-padded to 16 columns (the GEMM's K granularity)."""
-    b8 = requant(boxes, pq["m_box"], pq["s_box"], out_bits=8)
-    bp = np.zeros((b8.shape[0], 16), dtype=np.int8)
-    bp[:, :4] = b8
-    h = relu(gemm_requant(bp, pq["w_q1"], pq["b_q1"], pq["m_q1"], pq["s_q1"], 8).astype(np.int8))
+    sat16(rq(Linear_2(ReLU(sat8(rq(Linear_1(b))))))) with b = sat8(rq(box; m_box, s_box)), the Q16
+    box [M, 4] requantised to int8; Linear_1 is a 4 -> hidden layer."""
+    b8 = requant(boxes, pq["m_box"], pq["s_box"], out_bits=8).astype(np.int8)
+    h = relu(gemm_requant(b8, pq["w_q1"], pq["b_q1"], pq["m_q1"], pq["s_q1"], 8).astype(np.int8))
     return gemm_requant(h, pq["w_q2"], pq["b_q2"], pq["m_q2"], pq["s_q2"], 16).astype(np.int16)
 
 

@@ -7,9 +7,13 @@
 // Parity status per function (how each is pinned is listed in tests/test_oracle_pins.py):
 //   orc_rq, orc_sat, orc_shiftexp, orc_calibrate_shift, orc_shiftmax_rows,
 //   orc_sdshiftgelu(_idiv), orc_newton_isqrt, orc_int_layernorm, orc_gemm_requant,
-//   orc_attention, orc_split_conv, orc_deform_attn : pinned.
+//   orc_attention, orc_split_conv, orc_deform_attn, orc_patch_embed, orc_requant,
+//   orc_resample_nearest, orc_int_sigmoid, orc_topk, orc_gather_rows, orc_ivit_shiftgelu : pinned.
 //   orc_block_forward : parity unpinned beyond its parts (its composition order and the
 //   residual/window conventions are readings of the paper, not stated by it).
+// Each operator is written from its mathematics as the cited passage defines it; where the paper
+// proves two forms equal (Constrained Shiftmax's reduced denominator), the plain form is used and
+// a pin checks the other.
 #include "ilw_oracle.h"
 
 #include <cstdint>
@@ -30,12 +34,21 @@ int64_t floor_div(int64_t a, int64_t b) {
 
 int64_t clamp64(int64_t v, int64_t lo, int64_t hi) { return v < lo ? lo : (v > hi ? hi : v); }
 
+// The fixed-point quotient shared by Constrained Shiftmax's normalisation (Sec. 3.3.2) and, with
+// s_d = 0, by IntDiv (a reading): num / den with k_out - 1 fractional bits, formed as a 31-bit
+// reciprocal F = floor((2^31 - 1) / den') of the denominator den' = clamp(den >> s_d, 1, 2^31 - 1)
+// and a right shift of num F by 31 - (k_out - 1) + s_d.  `den_reduced` is den >> s_d.
+int64_t fixed_point_ratio(int64_t num, int64_t den_reduced, int32_t s_d, int32_t k_out) {
+    const int64_t F = kInt31Max / clamp64(den_reduced, 1, kInt31Max);
+    return (int64_t)(((__int128)num * F) >> (31 - (k_out - 1) + s_d));
+}
+
 }  // namespace
 
 extern "C" {
 
-// Dyadic requantisation (Sec. 3.2.2: "integer dyadic multiply-and-shift").  Reading: round
-// half up, i.e. add 2^(s-1) before the arithmetic right shift.  Computed in int128 so that no
+// Dyadic requantisation (Sec. 3.2.2: a fixed rescale applied as an integer multiply followed by a
+// right shift).  Reading: round half up, i.e. add 2^(s-1) before the arithmetic right shift.  Computed in int128 so that no
 // intermediate can overflow; the callers' ranges keep the result within int64.
 int64_t orc_rq(int64_t v, int32_t m, int32_t s) {
     __int128 p = (__int128)v * (__int128)m;
@@ -50,45 +63,44 @@ int64_t orc_sat(int64_t v, int32_t bits) {
     return clamp64(v, -hi, hi);
 }
 
-// ShiftExp, Algorithm 1 (function ShiftExp), for a non-positive integer input I with the
-// integer I0 = round(1/S) supplied by the caller (the kernel never sees S).
-//   I_e  = I + (I >> 1) - (I >> 4)          (I * log2 e with shifts)
-//   I_e  = clamp_min(I_e, k_inter * (-I0))  (lower-bound clipping)
-//   q    = floor(I_e / (-I0))               (integer part)
-//   r    = -(I_e - q * (-I0))               (decimal part)
-//   I_b  = ((-r) >> 1) + I0
-//   I_exp = I_b << (k_inter - q)            (scale S / 2^k_inter)
+// ShiftExp (Algorithm 1, Sec. 3.3.1): an integer stand-in for e^(S I), I <= 0, where the caller
+// supplies I0 = round(1/S) instead of S.  Since e^(S I) = 2^(S I log2 e), the input is first
+// brought to base 2 with shifts and adds, I_e = I + floor(I/2) - floor(I/16) (log2 e ~ 1.4375,
+// each shift flooring as an arithmetic shift does).  Its magnitude t = -I_e, in units of 1/I0, is
+// clipped at k_inter I0 (powers below 2^-k_inter are all represented by the smallest one) and
+// divided with remainder, t = q I0 + r, 0 <= r < I0: 2^(-t/I0) = 2^-q 2^(-r/I0).  The fractional
+// power is replaced by its chord 2^-f ~ 1 - f/2 on [0, 1), so I0 2^(-r/I0) becomes I0 - r/2, rounded
+// the way Algorithm 1 rounds it (a floor of -r/2, i.e. I0 - ceil(r/2)).  The integer power 2^-q and
+// k_inter fractional bits of output scale (S_exp = S / 2^k_inter) leave one left shift by k_inter - q.
 int64_t orc_shiftexp(int64_t I, int64_t I0, int32_t k_inter) {
-    int64_t Ie = I + (I >> 1) - (I >> 4);
-    int64_t lo = (int64_t)k_inter * (-I0);
-    if (Ie < lo) Ie = lo;
-    int64_t q = floor_div(Ie, -I0);
-    int64_t r = -(Ie - q * (-I0));
-    int64_t Ib = ((-r) >> 1) + I0;
-    return Ib << (k_inter - q);
+    const int64_t I_e = I + floor_div(I, 2) - floor_div(I, 16);  // I log2 e
+    const int64_t t = std::min(-I_e, (int64_t)k_inter * I0);     // clipped magnitude of the exponent
+    const int64_t q = t / I0, r = t % I0;                         // t = q I0 + r (t >= 0)
+    const int64_t I_b = I0 - (r + 1) / 2;                         // I0 2^(-r/I0) by the chord
+    return I_b << (k_inter - q);
 }
 
-// CalibrateShift, Algorithm 2:  M_req = ceil(log2 S_sum), M_target = M_req + m_p,
-// s_d = max(M_target - M_hw, 0).  ceil(log2 S) is the smallest m with 2^m >= S.
+// CalibrateShift (Algorithm 2, Sec. 3.3.2): the smallest denominator shift s_d >= 0 that leaves a
+// sum of ceil(log2 S_sum) bits with m_p bits of headroom below the M_hw-bit division:
+// s_d = max(ceil(log2 S_sum) + m_p - M_hw, 0), where ceil(log2 S) is the least m with 2^m >= S.
 int32_t orc_calibrate_shift(int64_t S_sum, int32_t m_p, int32_t M_hw) {
-    int32_t M_req = 0;
-    while (M_req < 62 && (int64_t(1) << M_req) < S_sum) ++M_req;
-    int32_t M_target = M_req + m_p;
-    int32_t s_d = M_target - M_hw;
-    return s_d > 0 ? s_d : 0;
+    int32_t bits_needed = 0;
+    while (bits_needed < 62 && (int64_t(1) << bits_needed) < S_sum) ++bits_needed;
+    return std::max(bits_needed + m_p - M_hw, 0);
 }
 
 void orc_shiftexp_vec(const int32_t *I, int64_t n, int32_t I0, int32_t k_inter, int64_t *out) {
     for (int64_t i = 0; i < n; ++i) out[i] = orc_shiftexp(I[i], I0, k_inter);
 }
 
-// Constrained Shiftmax, Algorithm 2 (function ConstrainedShiftmax) applied to each row:
-//   I_max = max(I_x); I_delta = I_x - I_max; I_exp = ShiftExp(I_delta)
-//   S_sum = sum I_exp; s_d = CalibrateShift(S_sum) (or the static s_d)
-//   Q_i = I_exp_i >> s_d; r_i = I_exp_i - (Q_i << s_d); S_R = sum Q_i + (sum r_i >> s_d)
-//   S_R = clamp(S_R, 1, 2^31-1); F = floor((2^31-1) / S_R)
-//   I_out_i = (I_exp_i * F) >> (31 - k_out + 1 + s_d)       (scale 2^-(k_out-1))
-// The output is stored as u8; every value is < 2^k_out for k_out <= 8 (checked, error -3).
+// Constrained Shiftmax (Algorithm 2, Sec. 3.3.2): softmax_i = e^(x_i - max) / sum_j e^(x_j - max)
+// over each row, every exponential by ShiftExp (its argument x_i - max is never positive).  The
+// exponentials are summed exactly (S_sum, int64).  The sum is reduced by 2^s_d -- s_d from
+// CalibrateShift per row, or a fixed s_d >= 0 -- so that the 31-bit reciprocal keeps precision: the
+// paper accumulates the reduced sum as quotients plus the floored sum of remainders and shows that
+// this equals floor(S_sum / 2^s_d), which is what is taken here.  The quotient is then the fixed-point
+// ratio above with k_out - 1 fractional bits (outputs stored as u8: every one is < 2^k_out for
+// k_out <= 8; a larger value is reported as error -3).
 int orc_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, int64_t len,
                       const orc_shiftmax_t *p, uint8_t *P, int64_t ldp, int64_t *S_sum_out,
                       int32_t *s_d_out, int64_t *S_R_out) {
@@ -105,27 +117,16 @@ int orc_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, int64_t len,
             if (S_R_out) S_R_out[row] = 0;
             continue;
         }
-        int64_t I_max = x[0];
-        for (int64_t i = 1; i < len; ++i)
-            if (x[i] > I_max) I_max = x[i];
-        for (int64_t i = 0; i < len; ++i) e[i] = orc_shiftexp((int64_t)x[i] - I_max, p->I0, p->k_inter);
+        const int64_t x_max = *std::max_element(x, x + len);
         int64_t S_sum = 0;
-        for (int64_t i = 0; i < len; ++i) S_sum += e[i];
-        int32_t s_d = p->s_d >= 0 ? p->s_d : orc_calibrate_shift(S_sum, p->m_p, p->M_hw);
-        int64_t sum_Q = 0, sum_r = 0;
         for (int64_t i = 0; i < len; ++i) {
-            int64_t Q = e[i] >> s_d;
-            int64_t r = e[i] - (Q << s_d);
-            sum_Q += Q;
-            sum_r += r;
+            e[i] = orc_shiftexp((int64_t)x[i] - x_max, p->I0, p->k_inter);
+            S_sum += e[i];
         }
-        int64_t S_R = sum_Q + (sum_r >> s_d);
-        S_R = clamp64(S_R, 1, kInt31Max);
-        int64_t F = kInt31Max / S_R;
-        int32_t sh = 31 - p->k_out + 1 + s_d;
+        const int32_t s_d = p->s_d >= 0 ? p->s_d : orc_calibrate_shift(S_sum, p->m_p, p->M_hw);
+        const int64_t S_R = clamp64(S_sum >> s_d, 1, kInt31Max);
         for (int64_t i = 0; i < len; ++i) {
-            __int128 prod = (__int128)e[i] * F;
-            int64_t o = (int64_t)(prod >> sh);
+            const int64_t o = fixed_point_ratio(e[i], S_sum >> s_d, s_d, p->k_out);
             if (o < 0 || o > 255) return -3;
             out[i] = (uint8_t)o;
         }
@@ -136,23 +137,19 @@ int orc_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, int64_t len,
     return 0;
 }
 
-// SD-ShiftGELU, Algorithm 1 (function SD-ShiftGELU) and Sec. 3.3.1:
-//   I_p = x + (x>>1) + (x>>3) + (x>>4)                 (1.702 x)
-//   I_shift = ReLU(I_p); I_delta = I_p - I_shift        (<= 0)
-//   E = ShiftExp(I_delta); E' = ShiftExp(-I_shift)
-//   I_div = IntDiv(E, E + E', k_out)                    (sigmoid, scale 2^-(k_out-1))
-// IntDiv is not defined in the paper; reading: the fixed-point division of Algorithm 2 with
-// s_d = 0, i.e. den = clamp(E + E', 1, 2^31-1), F = floor((2^31-1)/den),
-// I_div = (E * F) >> (31 - k_out + 1).  Returns I_div; the GELU output is x * I_div.
+// SD-ShiftGELU (Algorithm 1, Sec. 3.3.1): GELU(x) ~ x sigma(1.702 x).  The sigmoid is evaluated in
+// its sign-split form sigma(z) = e^min(z,0) / (e^min(z,0) + e^-max(z,0)), in which neither
+// exponential sees a positive argument, so no row maximum is needed and each element stands alone.
+// z = 1.702 x is formed with shifts, I_p = x + floor(x/2) + floor(x/8) + floor(x/16) (1.6875 x);
+// both exponentials come from ShiftExp; the quotient (IntDiv, which the paper does not define) is
+// read as the fixed-point ratio of Constrained Shiftmax with s_d = 0.  Returns the sigmoid factor
+// I_div (scale 2^-(k_out-1)); the GELU output is x I_div.
 int64_t orc_sdshiftgelu_idiv(int64_t x, int32_t I0, int32_t k_inter, int32_t k_out) {
-    int64_t Ip = x + (x >> 1) + (x >> 3) + (x >> 4);
-    int64_t Ish = Ip > 0 ? Ip : 0;
-    int64_t Id = Ip - Ish;
-    int64_t E = orc_shiftexp(Id, I0, k_inter);
-    int64_t E2 = orc_shiftexp(-Ish, I0, k_inter);
-    int64_t den = clamp64(E + E2, 1, kInt31Max);
-    int64_t F = kInt31Max / den;
-    return (int64_t)(((__int128)E * F) >> (31 - k_out + 1));
+    const int64_t I_p = x + floor_div(x, 2) + floor_div(x, 8) + floor_div(x, 16);
+    const int64_t I_shift = std::max<int64_t>(I_p, 0);
+    const int64_t e_neg = orc_shiftexp(I_p - I_shift, I0, k_inter);  // e^min(z, 0)
+    const int64_t e_pos = orc_shiftexp(-I_shift, I0, k_inter);       // e^-max(z, 0)
+    return fixed_point_ratio(e_neg, e_neg + e_pos, 0, k_out);
 }
 
 int orc_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, int32_t I0, int32_t k_inter,
@@ -517,20 +514,15 @@ int orc_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int32_t 
 }
 
 // Integer sigmoid of the detection head.  Table 5 lists ShiftExp as the integer form of the
-// detection head's exponential; the sigmoid is taken in the sign-dependent form SD-ShiftGELU
-// uses for its sigmoid factor (Sec. 3.3.1, Algorithm 1), with the logit as the argument
-// (a reading: no 1.702 factor):
-//   I_shift = ReLU(I); I_delta = I - I_shift
-//   E = ShiftExp(I_delta); E' = ShiftExp(-I_shift)
-//   F = floor((2^31 - 1) / (E + E')); out = (E F) >> (31 - k_out + 1)   (scale 2^-(k_out-1))
+// detection head's exponential; the sigmoid is taken in the sign-split form SD-ShiftGELU uses for
+// its sigmoid factor (Sec. 3.3.1), sigma(z) = e^min(z,0) / (e^min(z,0) + e^-max(z,0)), with the logit
+// itself as z (a reading: no 1.702 factor), and the same fixed-point quotient (k_out - 1 fractional
+// bits).
 int64_t orc_int_sigmoid1(int64_t x, int32_t I0, int32_t k_inter, int32_t k_out) {
-    int64_t Ish = x > 0 ? x : 0;
-    int64_t Id = x - Ish;
-    int64_t E = orc_shiftexp(Id, I0, k_inter);
-    int64_t E2 = orc_shiftexp(-Ish, I0, k_inter);
-    int64_t den = clamp64(E + E2, 1, kInt31Max);
-    int64_t F = kInt31Max / den;
-    return (int64_t)(((__int128)E * F) >> (31 - k_out + 1));
+    const int64_t x_pos = std::max<int64_t>(x, 0);
+    const int64_t e_neg = orc_shiftexp(x - x_pos, I0, k_inter);  // e^min(z, 0)
+    const int64_t e_pos = orc_shiftexp(-x_pos, I0, k_inter);     // e^-max(z, 0)
+    return fixed_point_ratio(e_neg, e_neg + e_pos, 0, k_out);
 }
 
 int orc_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, int32_t I0, int32_t k_inter,
@@ -573,10 +565,11 @@ int orc_gather_rows(const uint8_t *src, int64_t src_ld, int64_t src_rows, const 
     return 0;
 }
 
-// I-ViT's ShiftGELU, the baseline SD-ShiftGELU replaces (Sec. 3.3.1): sigma(z) = e^(z - M) /
-// (e^(z - M) + e^(-M)) with the vector-wise maximum M of the row, so that every ShiftExp input is
-// non-positive.  A reading: M is clamped at 0 (a row whose values are all negative has M = 0,
-// where the identity holds just the same and -M stays non-positive).
+// I-ViT's ShiftGELU, the baseline SD-ShiftGELU replaces (Sec. 3.3.1): the same sigmoid factor of
+// 1.702 x, but with every exponential made non-positive by the row's maximum M of I_p instead of by
+// each element's sign, sigma(z) = e^(z - M) / (e^(z - M) + e^-M).  A reading: M is clamped at 0 (a
+// row whose values are all negative has M = 0, where the identity holds just the same and -M stays
+// non-positive).
 int orc_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int64_t L, int32_t I0,
                        int32_t k_inter, int32_t k_out, int32_t *Y, int64_t ldy) {
     if (I0 < 1 || k_inter < 0 || k_inter > 30 || k_out < 1 || k_out > 16 || L < 1) return -1;
@@ -586,16 +579,13 @@ int orc_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int64_t L, i
         int64_t M = 0;
         for (int64_t c = 0; c < L; ++c) {
             const int64_t v = x[c];
-            Ip[(size_t)c] = v + (v >> 1) + (v >> 3) + (v >> 4);
-            if (Ip[(size_t)c] > M) M = Ip[(size_t)c];
+            Ip[(size_t)c] = v + floor_div(v, 2) + floor_div(v, 8) + floor_div(v, 16);
+            M = std::max(M, Ip[(size_t)c]);
         }
-        const int64_t E2 = orc_shiftexp(-M, I0, k_inter);
+        const int64_t e_max = orc_shiftexp(-M, I0, k_inter);  // e^-M
         for (int64_t c = 0; c < L; ++c) {
-            const int64_t E = orc_shiftexp(Ip[(size_t)c] - M, I0, k_inter);
-            const int64_t den = clamp64(E + E2, 1, kInt31Max);
-            const int64_t F = kInt31Max / den;
-            const int64_t idiv = (int64_t)(((__int128)E * F) >> (31 - k_out + 1));
-            const int64_t o = (int64_t)x[c] * idiv;
+            const int64_t e = orc_shiftexp(Ip[(size_t)c] - M, I0, k_inter);
+            const int64_t o = (int64_t)x[c] * fixed_point_ratio(e, e + e_max, 0, k_out);
             if (o < INT32_MIN || o > INT32_MAX) return -2;
             Y[r * ldy + c] = (int32_t)o;
         }

@@ -820,8 +820,10 @@ class TwoStage:
 
 class QueryPos:
     """The learnable positional-query projection (``synth.query_pos_params``): Q16 boxes [M, 4] ->
-    int8 (requantised, zero-padded to 16 columns) -> linear 16 -> hidden, ReLU -> linear hidden -> d
-    -> int16 positional queries [M, d].  Every step is an ilwdetr_* call."""
+    int8 (requantised) -> linear 4 -> hidden, ReLU -> linear hidden -> d -> int16 positional queries
+    [M, d].  Every step is an ilwdetr_* call.  The GEMM takes K in multiples of 16, so the 4-column
+    layer runs as a 16-column one: the int8 boxes sit in columns 0..3 of a zeroed [M, 16] buffer and
+    the packed weight has zero columns 4..15 (zero products, the same integers)."""
 
     def __init__(self, pq: dict, M: int, device="cuda"):
         import numpy as np
@@ -830,8 +832,11 @@ class QueryPos:
         self.pq, self.M = pq, M
         dv = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)  # noqa: E731
         self.t = {k: dv(v) for k, v in pq.items() if isinstance(v, np.ndarray)}
-        for k in ("w_q1", "w_q2"):
-            self.t[k + "_p"] = pack_weight(self.t[k])
+        w1 = pq["w_q1"]
+        w1p = np.zeros((w1.shape[0], 16), dtype=np.int8)
+        w1p[:, :w1.shape[1]] = w1
+        self.t["w_q1_p"] = pack_weight(dv(w1p))
+        self.t["w_q2_p"] = pack_weight(self.t["w_q2"])
         self.hidden, self.d = pq["w_q1"].shape[0], pq["w_q2"].shape[0]
         self.b8 = torch.zeros((M, 16), dtype=torch.int8, device=device)  # columns 4..15 stay zero
 

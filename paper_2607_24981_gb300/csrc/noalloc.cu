@@ -26,7 +26,9 @@ std::mutex g_mu;
 int8_t *g_scratch_addr[kMaxDevices] = {};
 
 // Device address of the scratch array on the current device; looked up once per device (the
-// first call on each device), with that device current.
+// first call on each device), with that device current, and kept for the life of the process: a
+// cudaDeviceReset ends the context the address belongs to, so the entry point is not to be used
+// across one.
 int scratch_on_current_device(int8_t **out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -52,9 +54,17 @@ extern "C" int ilwdetr_patch_embed_noalloc(const int8_t *img, int32_t B, int32_t
                                            int32_t p, const void *Wp, const int32_t *bias, const int32_t *mult,
                                            const int32_t *shift, int32_t d, const int16_t *pos, int32_t m_pos,
                                            int32_t s_pos, int16_t *x0, ilw_stream_t stream) {
+    // every argument is checked before anything is launched
     if (B < 0 || Cin < 1 || p < 16 || p % 16 || Hh < p || Ww < p || Hh % p || Ww % p || Ww % 16 || d < 1)
         return ilw::report_error(ILW_ERR_UNSUPPORTED, "patch_embed_noalloc: needs p % 16 == 0, p | H, p | W");
     if (B == 0) return ILW_OK;
+    if (!img || ((uintptr_t)img % 16) != 0 || !x0)
+        return ilw::report_error(ILW_ERR_INVALID_ARG, "patch_embed_noalloc: NULL or misaligned image, or NULL x0");
+    if (!Wp || ((uintptr_t)Wp % 256) != 0)
+        return ilw::report_error(ILW_ERR_INVALID_ARG, "patch_embed_noalloc: packed weight NULL or not 256-byte aligned");
+    if (!mult || !shift) return ilw::report_error(ILW_ERR_INVALID_ARG, "patch_embed_noalloc: mult/shift are NULL");
+    if (pos && (s_pos < 1 || s_pos > 62))
+        return ilw::report_error(ILW_ERR_INVALID_ARG, "patch_embed_noalloc: position shift outside [1, 62]");
     // the gathered patch matrix, int8 (B*T rows of Cin*p*p)
     const size_t need = (size_t)B * (Hh / p) * (Ww / p) * Cin * p * p;
     if (need > kNoAllocScratchBytes)
@@ -66,8 +76,6 @@ extern "C" int ilwdetr_patch_embed_noalloc(const int8_t *img, int32_t B, int32_t
     int rc = scratch_on_current_device(&scratch);
     if (rc) return rc;
     // every byte the GEMM reads is written by the gather first: nothing needs clearing
-    if (!img || ((uintptr_t)img % 16) != 0 || !x0)
-        return ilw::report_error(ILW_ERR_INVALID_ARG, "patch_embed_noalloc: NULL or misaligned image");
     cudaError_t e = ilw::launch_patchify(img, B, Cin, Hh, Ww, p, scratch, (cudaStream_t)stream);
     if (e != cudaSuccess) return ilw::report_error(ILW_ERR_CUDA, cudaGetErrorString(e));
     const int32_t T = (Hh / p) * (Ww / p), K = Cin * p * p;

@@ -331,13 +331,11 @@ def two_stage_params(seed: int, d: int = 256, C: int = 80, levels=((80, 80), (40
 def query_pos_params(seed: int, d: int = 256, hidden: int = 256, sigma_pos: float = 2048.0) -> dict:
     """Integer parameters of the learnable positional-query projection (Sec. 3.1.2: linear layers
     on the reference-box coordinates in place of the sinusoidal encoding): the Q16 box (cx, cy, w,
-    h) requantised to int8 (box / 512, in [0, 128]) and zero-padded to 16 columns, a linear layer
-    16 -> hidden with ReLU on its int8 outputs (std ~32), a linear layer hidden -> d to the decoder's
-    int16 positional query (std ~sigma_pos).  The padded weight columns are zero."""
+    h) requantised to int8 (box / 512, in [0, 128]), a linear layer 4 -> hidden with ReLU on its
+    int8 outputs (std ~32), a linear layer hidden -> d to the decoder's int16 positional query
+    (std ~sigma_pos)."""
     p = "QP."
     pq: dict = {"m_box": 1 << 30, "s_box": 39}
-    w1, pq["b_q1"], pq["m_q1"], pq["s_q1"] = gemm_params(seed, p + "q1", hidden, 16, 40.0, 32.0)
-    w1[:, 4:] = 0
-    pq["w_q1"] = w1
+    pq["w_q1"], pq["b_q1"], pq["m_q1"], pq["s_q1"] = gemm_params(seed, p + "q1", hidden, 4, 40.0, 32.0)
     pq["w_q2"], pq["b_q2"], pq["m_q2"], pq["s_q2"] = gemm_params(seed, p + "q2", d, hidden, 16.0, sigma_pos)
     return pq

@@ -103,3 +103,29 @@ def test_detection_entry_points_validate_without_gpu(built_lib):
     g = ilw.GeluT(600, 16, 8)
     assert L.ilwdetr_ivit_shiftgelu(ctypes.c_void_p(16), 4, 3, 8, ctypes.c_void_p(16), 8, ctypes.byref(g), None) == -1
     assert L.ilwdetr_topk(ctypes.c_void_p(16), 10, 0, 10, 3, ctypes.c_void_p(16), ctypes.c_void_p(16), None) == 0
+
+
+def test_int8_tcgen05_mma_is_not_available_on_sm103a(tmp_path):
+    """The reason the integer GEMMs and attention run on kind::f16 (int8 values carried exactly in
+    fp16, fp32 accumulation kept below 2^24): ptxas of this toolkit rejects the int8 tensor-core
+    MMA for sm_103a while accepting the fp16 form.  Compiles a one-instruction kernel of each kind."""
+    from paper_2607_24981_gb300 import build
+
+    def compile_kind(kind):
+        src = tmp_path / f"probe_{kind}.cu"
+        src.write_text(
+            "#include <cstdint>\n"
+            "__global__ void k(uint32_t d, uint64_t a, uint64_t b, uint32_t i) {\n"
+            "  asm volatile(\"{\\n .reg .pred p;\\n setp.ne.b32 p, %4, 0;\\n"
+            f" tcgen05.mma.cta_group::1.kind::{kind} [%0], %1, %2, %3, p;\\n}}\\n\""
+            " :: \"r\"(d), \"l\"(a), \"l\"(b), \"r\"(i), \"r\"(1u) : \"memory\");\n}\n")
+        import subprocess
+
+        r = subprocess.run([build.nvcc()] + build.ARCH + ["-c", str(src), "-o", str(tmp_path / f"{kind}.o")],
+                           capture_output=True, text=True)
+        return r.returncode, r.stdout + r.stderr
+
+    rc16, _ = compile_kind("f16")
+    rc8, msg = compile_kind("i8")
+    assert rc16 == 0
+    assert rc8 != 0 and "kind::i8" in msg and "sm_103a" in msg, msg

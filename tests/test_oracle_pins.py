@@ -60,6 +60,43 @@ def test_shiftexp_closed_form_multiples(orc):
         assert orc.shiftexp(-16 * j, 23, 16) == want, j
 
 
+def _golden_lines(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return [line.split() for line in f if line.strip() and not line.startswith("#")]
+
+
+def test_shiftexp_golden_odd_remainders(orc):
+    """Hand-derived ShiftExp values at odd remainders, even non-multiple-of-16 inputs, q > 0 and the
+    clip boundary (tests/golden/shiftexp_odd_remainders.txt, each derived there from Algorithm 1).
+    The intermediate columns are re-derived here with Python's floor division as a check of the
+    file itself."""
+    for I, I0, k, Ie, t, q, r, Ib, Iexp in ([int(v) for v in row] for row in _golden_lines("shiftexp_odd_remainders.txt")):
+        assert I + I // 2 - I // 16 == Ie and min(-Ie, k * I0) == t and divmod(t, I0) == (q, r)
+        assert Ib == I0 - (r + 1) // 2 and Iexp == Ib << (k - q)
+        assert orc.shiftexp(I, I0, k) == Iexp, (I, I0, k)
+        assert orc.shiftexp_vec(np.array([I], dtype=np.int32), I0, k)[0] == Iexp
+
+
+def test_shiftmax_and_gelu_golden_odd_remainders(orc):
+    """A Shiftmax row and SD-ShiftGELU factors whose ShiftExp has an odd remainder
+    (tests/golden/odd_remainder_rows.txt, derived by hand from Algorithms 1 and 2)."""
+    for row in _golden_lines("odd_remainder_rows.txt"):
+        if row[0] == "shiftmax":
+            I0, Ssum, sd, SR, F = (int(v) for v in row[1:6])
+            bar1 = row.index("|")
+            bar2 = row.index("|", bar1 + 1)
+            X = np.array([[int(v) for v in row[bar1 + 1:bar2]]], dtype=np.int32)
+            want = [int(v) for v in row[bar2 + 1:]]
+            P, S, sdv, SRv = orc.shiftmax_rows(X, I0)
+            assert (S[0], sdv[0], SRv[0]) == (Ssum, sd, SR)
+            assert (2**31 - 1) // SR == F
+            assert P[0].tolist() == want
+        else:
+            x, I0, idiv, out = (int(v) for v in row[1:])
+            assert orc.sdshiftgelu_idiv(x, I0) == idiv
+            assert orc.sdshiftgelu(np.array([x], dtype=np.int32), I0)[0] == out
+
+
 def test_shiftexp_brute_force_properties(orc):
     """Every Delta in [-1.5 k I0, 0] for several I0: top value I0 2^k, monotone, clamp value I0
     below the threshold, and the float bound of the shift-add exponential:
@@ -150,6 +187,10 @@ def test_shiftmax_qr_identity_and_range(orc):
             assert (2**31 - 1) // SR[r] >= 15
             e = orc.shiftexp_vec(X[r] - X[r].max(), I0)
             assert int(e.sum()) == S[r]
+            # the paper's quotient-remainder accumulation, term by term, lands on the same S_R
+            Q = [int(v) >> int(sd[r]) for v in e]
+            rem = [int(v) - (qq << int(sd[r])) for v, qq in zip(e, Q)]
+            assert min(max(sum(Q) + (sum(rem) >> int(sd[r])), 1), 2**31 - 1) == SR[r]
         assert P.max() < 256
 
 
@@ -763,17 +804,25 @@ def test_two_stage_selects_the_best_tokens(orc):
     assert boxes.min() >= 0 and boxes.max() <= 2 ** 16
 
 
-def test_query_pos_is_rowwise_and_ignores_padding(orc):
+def test_query_pos_is_rowwise(orc):
     """The positional query of a box depends on that box alone (row permutation equivariance), and
-    the weight columns facing the 12 zero-padded input columns do not matter."""
+    the first layer is the plain 4-column integer product of the requantised boxes."""
     pq = synth.query_pos_params(7, d=64, hidden=32)
     boxes = synth.uniform_int(7, "qp.pin", (50, 4), 0, 1 << 16)
     pos = orc.query_pos(pq, boxes)
     perm = np.random.default_rng(3).permutation(50)
     assert np.array_equal(orc.query_pos(pq, boxes[perm]), pos[perm])
-    w = pq["w_q1"].copy()
-    w[:, 4:] = synth.uniform_int(8, "qp.junk", (w.shape[0], 12), -127, 127, np.int8)
-    assert np.array_equal(orc.query_pos(dict(pq, w_q1=w), boxes), pos)
+    assert pq["w_q1"].shape == (32, 4)
+    b8 = np.clip((boxes.astype(np.int64) * (1 << 30) + (1 << 38)) >> 39, -127, 127)
+    def rq(v, m, s):  # exact round-half-up dyadic rescale, in Python integers
+        return np.array([[(int(a) * int(mm) + (1 << (int(ss) - 1))) >> int(ss) for a, mm, ss in zip(row, m, s)]
+                         for row in v], dtype=np.int64)
+
+    acc = b8 @ pq["w_q1"].astype(np.int64).T + pq["b_q1"]
+    h = np.maximum(np.clip(rq(acc, pq["m_q1"], pq["s_q1"]), -127, 127), 0)
+    acc2 = h @ pq["w_q2"].astype(np.int64).T + pq["b_q2"]
+    want = np.clip(rq(acc2, pq["m_q2"], pq["s_q2"]), -32767, 32767)
+    assert np.array_equal(pos, want)
     assert np.abs(pos.astype(np.int64)).mean() > 10
 
 
