@@ -18,9 +18,7 @@ import argparse
 import json
 import os
 import statistics
-import subprocess
 import sys
-import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -42,6 +40,7 @@ def parse_args(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ilw", choices=["ilw", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-legs", action="store_true", help="skip the block-variant, sweep and detector legs")
     return ap.parse_args(argv)
 
 
@@ -67,60 +66,6 @@ def barrier(world: int) -> None:
         import torch.distributed as dist
 
         dist.barrier()
-
-
-# ------------------------------------------------------------------------------ clocks
-class ClockSampler:
-    """nvidia-smi samples (every 200 ms) of SM clock and throttle reasons while running."""
-
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
-
-    def __init__(self, index: int):
-        self.index = index
-        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
-        self.p = None
-
-    def __enter__(self):
-        try:
-            self.p = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
-                                       "--format=csv,noheader,nounits", "-lms", "200"],
-                                      stdout=self.f, stderr=subprocess.DEVNULL)
-        except OSError:
-            self.p = None
-        return self
-
-    def __exit__(self, *a):
-        if self.p is not None:
-            self.p.terminate()
-            try:
-                self.p.wait(timeout=5)
-            except subprocess.TimeoutExpired:
-                self.p.kill()
-
-    def summary(self) -> dict:
-        self.f.flush()
-        self.f.seek(0)
-        sm, mx, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.f.read().splitlines():
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) < 9:
-                continue
-            try:
-                sm.append(float(parts[1]))
-                mx.append(float(parts[2]))
-            except ValueError:
-                continue
-            for n, v in zip(names, parts[5:9]):
-                if v.lower().startswith("active"):
-                    reasons.add(n)
-        os.unlink(self.f.name)
-        if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
 
 
 # ------------------------------------------------------------------------------ workload
@@ -227,56 +172,196 @@ def kernel_work(cfg, B):
     }
 
 
-def run_cpu_sample(cfg, pe, blocks) -> dict:
-    """The oracle as it stands, single-threaded: one image through blocks 0..CPU_SAMPLE_BLOCKS-1."""
-    import numpy as np
+def host_cpu() -> dict:
+    """The host's usable cores and CPU model (lscpu's model name, when lscpu answers)."""
+    import subprocess
 
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    model = "unknown"
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.TimeoutExpired):
+        pass
+    return {"cores": cores, "model": model}
+
+
+def _oracle_image(job):
+    """One image through the given encoder blocks in the oracle (a spawned worker process);
+    returns the seconds the blocks took."""
+    seed, pe, blocks, T = job
     import oracle
     from paper_2607_24981_gb300 import synth
 
-    oracle.build()
-    img = synth.image_input(SEED, 1)
+    img = synth.image_input(seed, 1)
     x = oracle.patch_embed(img, pe["p"], pe["w"], pe["b"], pe["m"], pe["s"], pe["pos"], pe["m_pos"], pe["s_pos"])
     t0 = time.perf_counter()
-    for bp in blocks[:CPU_SAMPLE_BLOCKS]:
-        x = oracle.block_forward(bp, x, 1, cfg["T"])
-    dt = time.perf_counter() - t0
+    for bp in blocks:
+        x = oracle.block_forward(bp, x, 1, T)
+    return time.perf_counter() - t0
+
+
+def oracle_pool(n):
+    """A pool of n spawned processes for the oracle (spawn: safe after the CUDA context exists)."""
+    import multiprocessing as mp
+
+    import oracle
+
+    oracle.build()  # built once here, so the workers only load it
+    return mp.get_context("spawn").Pool(n)
+
+
+def run_cpu_sample(cfg, pe, blocks) -> dict:
+    """The oracle as it stands, timed on the host's cores: single-threaded (one image through
+    blocks 0..CPU_SAMPLE_BLOCKS-1), then on every core (one image per core, in separate processes,
+    each through the same blocks; the loops of the oracle stay plain)."""
+    host = host_cpu()
+    sub = blocks[:CPU_SAMPLE_BLOCKS]
+    with oracle_pool(host["cores"]) as pool:
+        t1 = pool.apply(_oracle_image, ((SEED, pe, sub, cfg["T"]),))
+        t0 = time.perf_counter()
+        pool.map(_oracle_image, [(SEED + 1 + i, pe, sub, cfg["T"]) for i in range(host["cores"])], chunksize=1)
+        tall = time.perf_counter() - t0
     units = CPU_SAMPLE_BLOCKS * cfg["T"]
-    assert np.isfinite(dt)
-    return {"value": units / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"1 image x encoder blocks 0-{CPU_SAMPLE_BLOCKS - 1} (3 window + 2 global), "
-                      f"{units} block-tokens, {dt:.1f} s, single-threaded C++ oracle (-O2)"}
+    blocks_desc = f"encoder blocks 0-{CPU_SAMPLE_BLOCKS - 1} (3 window + 2 global)"
+    return {"value": host["cores"] * units / tall, "unit": UNIT, "cores": host["cores"], "kind": "oracle",
+            "cpu": host["model"],
+            "sample": f"{host['cores']} images (one per core, separate processes) x {blocks_desc}: "
+                      f"{host['cores'] * units} block-tokens in {tall:.1f} s wall; C++ oracle (g++ -O2)",
+            "single_thread": {"value": units / t1, "unit": UNIT, "cores": 1,
+                              "sample": f"1 image x {blocks_desc}, {units} block-tokens, {t1:.1f} s"}}
+
+
+# ------------------------------------------------------------------------------ further legs
+def _time_launches(torch, fn, reps, flush=None):
+    """Median and minimum device time (ms) of `reps` calls of fn, each bracketed by CUDA events on
+    the current stream; `flush` (a buffer larger than L2) is rewritten before each call."""
+    ts = []
+    for _ in range(reps):
+        if flush is not None:
+            flush.fill_(1)
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record()
+        fn()
+        e.record()
+        e.synchronize()
+        ts.append(s.elapsed_time(e))
+    ts.sort()
+    return ts[len(ts) // 2], ts[0]
+
+
+def leg_blocks(ilw, torch, bb, img, reps, flush):
+    """One global-attention block and one window block of the backbone, each a CUDA graph of one
+    ilwdetr_block_forward on the patch embedding of the batch; block tokens/s = B T / block time."""
+    pe = bb.pe
+    x0 = torch.empty((bb.B * bb.T, bb.d), dtype=torch.int16, device=img.device)
+    ilw.patch_embed(img, bb.p, pe["w_p"], bb.d, pe["b"], pe["m"], pe["s"], pe["pos"], bb.pe_s["m_pos"],
+                    bb.pe_s["s_pos"], bb.ws_pe, x0)
+    out = torch.empty_like(x0)
+    res = {}
+    for kind in ("global", "window"):
+        i = next(j for j, bw in enumerate(bb.blocks) if (bw.bp["win_side"] <= 1) == (kind == "global"))
+        bw = bb.blocks[i]
+        g = ilw.Graphed(lambda: ilw.block_forward(bw, x0, bb.B, bb.T, bb.ws_blk, out=out))
+        med, best = _time_launches(torch, g.replay, reps, flush)
+        res[kind] = {"block": i, "ms": med, "ms_best": best, "tokens_per_s": bb.B * bb.T / (med / 1000.0)}
+    return res
+
+
+def leg_c3(ilw, torch, dev, reps):
+    """The nonlinearity sweep at its workload sizes: Constrained Shiftmax over 2^27 int32 scores in
+    rows of 64 / 400 / 1600, SD-ShiftGELU over 2^28 int32 values, I-LayerNorm over 2^20 int32 rows
+    of 192 / 384.  Inputs drawn on the device from a seeded generator with the workload's ranges;
+    every working set is larger than L2, so no flush is needed.  GB/s counts the algorithmic bytes
+    (4 B in + 1 B out per Shiftmax or LayerNorm element, 4 B + 4 B per GELU element)."""
+    from paper_2607_24981_gb300 import synth
+
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(SEED)
+    res = {}
+
+    def draw(shape, lo, hi):
+        return torch.randint(lo, hi + 1, shape, generator=gen, device=dev, dtype=torch.int32)
+
+    for L in (64, 400, 1600):
+        X = draw(((1 << 27) // L, L), -(1 << 15), 1 << 15)
+        P = torch.empty(X.shape, dtype=torch.uint8, device=dev)
+        med, best = _time_launches(torch, lambda: ilw.shiftmax_rows(X, {"I0": 3000}, out=P), reps)
+        res[f"shiftmax_{L}"] = {"ms": med, "gbs": 5.0 * X.numel() / (med / 1000.0) / 1e9}
+        del X, P
+    X = draw((1 << 28,), -(1 << 12), 1 << 12)
+    Y = torch.empty_like(X)
+    med, best = _time_launches(torch, lambda: ilw.sdshiftgelu(X, {"I0": 600}, out=Y), reps)
+    res["sdshiftgelu"] = {"ms": med, "gbs": 8.0 * X.numel() / (med / 1000.0) / 1e9}
+    del X, Y
+    for C in (192, 384):
+        X = draw((1 << 20, C), -(1 << 14), 1 << 14)
+        beta, mult, shift = (torch.from_numpy(a).to(dev) for a in synth.ln_params(34, f"c3lnp{C}", C))
+        Y = torch.empty(X.shape, dtype=torch.int8, device=dev)
+        med, best = _time_launches(torch, lambda: ilw.int_layernorm(X, beta, mult, shift, 10, 8, out=Y), reps)
+        res[f"layernorm_{C}"] = {"ms": med, "gbs": 5.0 * X.numel() / (med / 1000.0) / 1e9}
+        del X, Y
+    return res
+
+
+def leg_detector(ilw, torch, dev, reps, flush):
+    """The full integer detector forward at batch 16 (Medium backbone with its four output layers
+    tapped, split-convolution projector, two-stage query selection with the positional-query
+    projection, three decoder layers, detection head), one CUDA graph per forward."""
+    from paper_2607_24981_gb300 import synth
+
+    cfg = synth.CONFIGS["detector_c4"]
+    bbc = synth.CONFIGS[cfg["backbone"]]
+    B, Q, g = cfg["B"], cfg["Q"], cfg["grid"]
+    det = ilw.Detector(synth.patch_embed_params(SEED, bbc["d"], mode=bbc["mode"]), synth.backbone_params(SEED, bbc),
+                       cfg["taps"], synth.projector_params(SEED, len(cfg["taps"]), bbc["d"], cfg["N"]),
+                       [synth.decoder_params(SEED, i) for i in range(cfg["dec_layers"])], B, Q, cfg["levels"], g,
+                       tsp=synth.two_stage_params(SEED, d=cfg["N"], C=80, levels=cfg["levels"]),
+                       hp=synth.head_params(SEED, d=cfg["N"], C=80), pq=synth.query_pos_params(SEED, d=cfg["N"]),
+                       device=dev)
+    img = torch.from_numpy(synth.image_input(SEED, B)).to(dev)
+    tgt = torch.from_numpy(synth.decoder_inputs(SEED, B, Q)["tgt"]).to(dev)
+    graph = ilw.Graphed(lambda: det.forward(img, tgt))
+    med, best = _time_launches(torch, graph.replay, reps, flush)
+    return {"B": B, "queries": Q, "ms": med, "ms_best": best, "images_per_s": B / (med / 1000.0),
+            "stages": "patch embed + 10 blocks, projector (3 levels), two-stage top-300 with positional "
+                      "queries, 3 decoder layers, detection head (80 classes)"}
 
 
 # ------------------------------------------------------------------------------ reference arm
 def run_reference(args) -> None:
+    """The oracle as it stands on the host's cores: each step runs one image per core (separate
+    processes) through one encoder block, cycling over the backbone's 10 blocks step by step."""
     rank, world, _ = dist_env()
     if rank != 0:
         return
     cfg, pe, blocks = build_host_params()
-    import oracle
-    from paper_2607_24981_gb300 import synth
-
-    oracle.build()
-    img = synth.image_input(SEED, 1)
-    x0 = oracle.patch_embed(img, pe["p"], pe["w"], pe["b"], pe["m"], pe["s"], pe["pos"], pe["m_pos"], pe["s_pos"])
+    host = host_cpu()
+    n = host["cores"]
     times = []
-    for step in range(args.warmup + args.steps):
-        bp = blocks[step % len(blocks)]
-        t0 = time.perf_counter()
-        oracle.block_forward(bp, x0, 1, cfg["T"])
-        if step >= args.warmup:
-            times.append(time.perf_counter() - t0)
+    with oracle_pool(n) as pool:
+        for step in range(args.warmup + args.steps):
+            bp = blocks[step % len(blocks)]
+            t0 = time.perf_counter()
+            pool.map(_oracle_image, [(SEED + i, pe, [bp], cfg["T"]) for i in range(n)], chunksize=1)
+            if step >= args.warmup:
+                times.append(time.perf_counter() - t0)
     ms = 1000.0 * statistics.mean(times)
-    value = cfg["T"] / (ms / 1000.0)
-    sample = (f"per step: 1 image (1600 tokens) through one encoder block, cycling over the 10 "
-              f"blocks (6 window, 4 global) step by step; single-threaded C++ oracle")
+    value = n * cfg["T"] / (ms / 1000.0)
+    sample = (f"per step: {n} images (one per core, separate processes, 1600 tokens each) through one "
+              f"encoder block, cycling over the 10 blocks (6 window, 4 global) step by step; the patch "
+              f"embedding is outside the timed region; C++ oracle (g++ -O2)")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-            "config": {"workload": "medium_c2 backbone (CPU oracle sample)", "B": 1, "T": cfg["T"],
+            "config": {"workload": "medium_c2 backbone (CPU oracle sample)", "B": n, "T": cfg["T"],
                        "d": cfg["d"], "H": cfg["H"], "F": cfg["F"]},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": n, "kind": "oracle", "cpu": host["model"],
+                             "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -350,6 +435,8 @@ def main(argv=None):
             per[name] = (tot + s_.elapsed_time(e_), cnt + 1, ln + n)
 
     barrier(world)
+    from paper_2607_24981_gb300.clocks import ClockSampler
+
     with ClockSampler(local) as clk:
         for _ in range(args.steps):
             flush.fill_(1)  # evict L2 before every timed step
@@ -396,7 +483,8 @@ def main(argv=None):
         else:
             kernels[name]["gscores_s"] = w / (avg_ms / 1000.0) / 1e9
     dom = max(per, key=lambda k: per[k][0])
-    roofline = roofline_entry(dom, kernels[dom], work[dom], peaks, clocks)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    roofline = roofline_entry(dom, kernels[dom], work[dom], peaks, clocks, sms)
 
     # end to end through the public API: pinned host image -> device, backbone, result -> host
     pin_in = torch.from_numpy(img_h).pin_memory()
@@ -422,6 +510,25 @@ def main(argv=None):
     e2e = {"value": world * units_per_step / (e2e_t / 1000.0), "unit": UNIT,
            "h2d_bytes_per_step": int(pin_in.numel()), "d2h_bytes_per_step": int(pin_out.numel() * 2)}
 
+    # further legs, timed in this run under their own clock record: the two block variants of the
+    # headline metric, the nonlinearity sweep and the full detector
+    legs = None
+    if not args.no_legs:
+        reps = max(args.steps, 10)
+        with ClockSampler(local) as clk2:
+            legs = {"blocks": leg_blocks(ilw, torch, bb, img, reps, flush)}
+            del bb, step, inst, e2e_step
+            torch.cuda.empty_cache()
+            legs["nonlinearity_sweep"] = leg_c3(ilw, torch, dev, reps)
+            legs["detector"] = leg_detector(ilw, torch, dev, reps, flush)
+            torch.cuda.synchronize()
+        legs["clocks"] = clk2.summary()
+        hbm = peaks.get("hbm_gbs") or 6800.0
+        for v in legs["nonlinearity_sweep"].values():
+            v["frac_of_measured_hbm"] = v["gbs"] / hbm
+            v["frac_of_8tbs"] = v["gbs"] / 8000.0
+        ilw.device_status()
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = run_cpu_sample(cfg, pe, blocks)
@@ -438,7 +545,7 @@ def main(argv=None):
                        "units": "block-tokens = blocks x images x tokens per step",
                        "l2": "flushed between timed steps (256 MB write)", "parallelism": f"replicas x{world}"},
             "clocks": clocks, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
-            "roofline": roofline, "kernels": kernels, "cpu_baseline": cpu,
+            "roofline": roofline, "kernels": kernels, "legs": legs, "cpu_baseline": cpu,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -452,7 +559,7 @@ def main(argv=None):
 NCU_TRAFFIC = {"attention_global": 29563136 + 0}
 
 
-def roofline_entry(name, k, work, peaks, clocks):
+def roofline_entry(name, k, work, peaks, clocks, sms):
     bound, w = work
     avg_s = k["avg_ms"] / 1000.0
     if bound == "hbm":
@@ -469,15 +576,18 @@ def roofline_entry(name, k, work, peaks, clocks):
         a = w / avg_s / 1e12
         return {"kernel": name, "bound": "tensor", "achieved": a, "peak": peak, "unit": "TFLOP/s",
                 "frac": a / peak, "traffic": NCU_TRAFFIC.get(name), "peak_source": src}
-    # ALU: integer ops per score (minimum the method needs with ShiftExp evaluated once per score:
-    # max 1, ShiftExp 12, sum 1, output multiply+shift 2) against SMs x 128 lanes x SM clock
-    ops_per_score = 16.0
+    # ALU: integer operations per score of the exact three-pass method (row maximum; ShiftExp and the
+    # int64 sum; ShiftExp again, the normalising multiply and shift, the fp16 P), the midpoint of the
+    # 30-40 that the method needs, against SMs x 128 lanes x the median SM clock; the figure at 16
+    # operations (ShiftExp counted once per score) is reported beside it
+    ops_per_score = 35.0
     mhz = clocks.get("sm_mhz") or 1500.0
-    peak = 152 * 128 * mhz * 1e6 / 1e12
+    peak = sms * 128 * mhz * 1e6 / 1e12
     a = w * ops_per_score / avg_s / 1e12
     return {"kernel": name, "bound": "alu", "achieved": a, "peak": peak, "unit": "Tops/s", "frac": a / peak,
-            "traffic": NCU_TRAFFIC.get(name), "peak_source": f"derived: 152 SMs x 128 int32 lanes x {mhz:.0f} MHz (median SM clock)",
-            "ops_per_score": ops_per_score}
+            "traffic": NCU_TRAFFIC.get(name),
+            "peak_source": f"derived: {sms} SMs (read from the device) x 128 int32 lanes x {mhz:.0f} MHz (median SM clock)",
+            "ops_per_score": ops_per_score, "frac_at_16_ops_per_score": a / peak * 16.0 / ops_per_score}
 
 
 if __name__ == "__main__":

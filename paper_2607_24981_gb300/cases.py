@@ -55,15 +55,21 @@ def build(case: str, batch: int = 0):
                 {"scores": scores})
     if case.startswith("gemm"):
         M, d, F = 12800, 384, 1536
-        N, K = {"gemm_qkv": (3 * d, d), "gemm_proj": (d, d), "gemm_fc1_gelu": (F, d), "gemm_fc2": (d, F)}[case]
-        # the activations as the encoder hands them over: int8 values carried in fp16
-        A = _dev(synth.uniform_int(1, "case.A", (M, K), -127, 127, np.int8).astype(np.float16))
+        N, K = {"gemm_qkv": (3 * d, d), "gemm_proj": (d, d), "gemm_fc1_gelu": (F, d), "gemm_fc2": (d, F),
+                "gemm_fc2_i8": (d, F), "gemm_fc1_gelu_i8": (F, d)}[case]
+        # the activations as the encoder hands them over: int8 values carried in fp16 (the _i8 cases:
+        # plain int8, converted to the fp16 operand inside the GEMM)
+        A8 = synth.uniform_int(1, "case.A", (M, K), -127, 127, np.int8)
+        A = _dev(A8) if case.endswith("_i8") else _dev(A8.astype(np.float16))
         W, b, m, s = synth.gemm_params(1, "case.W", N, K, 40.0, 40.0)
         Wp = ilw.pack_weight(_dev(W))
         b, m, s = _dev(b), _dev(m), _dev(s)
         if case == "gemm_fc1_gelu":  # h written as fp16-carried int8, as the encoder block does
             out = torch.empty((M, N), dtype=torch.float16, device="cuda")
             fn = lambda: ilw.gemm(A, Wp, N, b, m, s, ilw.I8_IN_F16, gelu={"I0": 1000}, m_g=3 << 29, s_g=40, out=out)
+        elif case == "gemm_fc1_gelu_i8":  # int8 a2 in, int8 h out
+            out = torch.empty((M, N), dtype=torch.int8, device="cuda")
+            fn = lambda: ilw.gemm(A, Wp, N, b, m, s, 8, gelu={"I0": 1000}, m_g=3 << 29, s_g=40, out=out)
         elif case == "gemm_qkv":  # q|k|v written as fp16-carried int8
             out = torch.empty((M, N), dtype=torch.float16, device="cuda")
             fn = lambda: ilw.gemm(A, Wp, N, b, m, s, ilw.I8_IN_F16, out=out)
@@ -126,16 +132,21 @@ def main(argv=None):
     for _ in range(3):
         fn()
     torch.cuda.synchronize()
-    # every launch timed on its own (events on the launching stream), median reported
+    # every launch timed on its own (events on the launching stream), median reported; the SM clock
+    # and throttle reasons are sampled over the timed launches
+    from .clocks import ClockSampler
+
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(max(a.reps, 1))]
-    for e0, e1 in ev:
-        e0.record()
-        fn()
-        e1.record()
-    torch.cuda.synchronize()
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        for e0, e1 in ev:
+            e0.record()
+            fn()
+            e1.record()
+        torch.cuda.synchronize()
     times = sorted(e0.elapsed_time(e1) for e0, e1 in ev)
     ms = times[len(times) // 2]
-    out = {"case": a.case, "us": ms * 1000.0, "us_min": times[0] * 1000.0, "graph": bool(a.graph)}
+    out = {"case": a.case, "us": ms * 1000.0, "us_min": times[0] * 1000.0, "graph": bool(a.graph),
+           "clocks": clk.summary()}
     if "flops" in work:
         out["tflops"] = work["flops"] / (ms / 1000.0) / 1e12
     if "bytes" in work:

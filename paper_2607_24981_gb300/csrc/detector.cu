@@ -74,7 +74,8 @@ __global__ void __launch_bounds__(256) resample_kernel(const int8_t *__restrict_
 
 unsigned grid_for(int64_t items) {
     int64_t g = (items + 255) / 256;
-    return (unsigned)(g < 1 ? 1 : (g > 152 * 16 ? 152 * 16 : g));
+    const int64_t cap = (int64_t)sm_count() * 16;  // grid-stride loops: 16 CTAs of 256 threads per SM
+    return (unsigned)(g < 1 ? 1 : (g > cap ? cap : g));
 }
 
 }  // namespace

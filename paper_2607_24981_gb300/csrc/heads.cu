@@ -160,7 +160,8 @@ __global__ void __launch_bounds__(256) ivit_shiftgelu_kernel(const int32_t *__re
 
 unsigned grid_for(int64_t work, int per_block) {
     const int64_t g = (work + per_block - 1) / per_block;
-    return (unsigned)(g < 1 ? 1 : (g > 152 * 16 ? 152 * 16 : g));
+    const int64_t cap = (int64_t)sm_count() * 16;  // grid-stride loops: 16 CTAs of 256 threads per SM
+    return (unsigned)(g < 1 ? 1 : (g > cap ? cap : g));
 }
 
 }  // namespace

@@ -14,6 +14,8 @@ int report_error(int code, const char *msg);
 // the current device (nullptr on failure), and a synchronous read-and-clear.
 int *status_word_ptr();
 cudaError_t read_and_clear_status(int *value);
+// Streaming multiprocessors of the current device (read from the device once per device).
+int sm_count();
 constexpr int kStatusTimeoutTma = 1;     // a wait for a TMA load ran out
 constexpr int kStatusTimeoutMma = 2;     // a wait for tensor-core completion ran out
 constexpr int kStatusTimeoutOperand = 3; // a wait for the converted operand ran out

@@ -1,5 +1,6 @@
 // status.cu -- the device status word that kernels with bounded waits latch when a wait runs
 // out, and the host side that reads and clears it (ilwdetr_device_status).
+#include <atomic>
 #include <cstdint>
 #include <mutex>
 
@@ -31,6 +32,18 @@ int *status_word_ptr() {
     last_dev = dev;
     last_ptr = g_addr[dev];
     return g_addr[dev];
+}
+
+int sm_count() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return 1;
+    static std::atomic<int> count[kMaxDev];  // 0 until read; every writer stores the same value
+    int v = count[dev].load(std::memory_order_relaxed);
+    if (!v) {
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1) return 1;
+        count[dev].store(v, std::memory_order_relaxed);
+    }
+    return v;
 }
 
 cudaError_t read_and_clear_status(int *value) {
