@@ -64,11 +64,16 @@ struct TcSmem {  // offsets from the 1024-aligned base
     static constexpr int kQ = 0;
     static constexpr int kRing = kQ + TQ * 128;
     static constexpr int kP = kRing + NP * kSlotB;
-    static constexpr int kRedMax = kP + NPB * kPB;         // float [NCQ][128]
+    // the constant-term operands of passes 2 and 3 (K = 16, 32-byte rows, 32-byte swizzle):
+    // A: -(2^23 + max + 1) of each query row as fp16 terms, B: the matching weights for every key
+    static constexpr int kAugA = kP + NPB * kPB;
+    static constexpr int kAugB = kAugA + TQ * 32;
+    static constexpr int kRedMax = kAugB + TKB * 32;       // float [NCQ][128]
     static constexpr int kRedSum = kRedMax + NCQ * TQ * 4; // uint64 [NCQ][128]
     static constexpr int kBar = kRedSum + NCQ * TQ * 8;
-    // barriers: q_full, full[NP], empty[NP], s_full[NS], s_free[NS], p_full[NPB], p_free[NPB], o_full, drain, xchg
-    static constexpr int kNBar = 1 + 2 * NP + 2 * NS + 2 * NPB + 3;
+    // barriers: q_full, full[NP], empty[NP], s_full[NS], s_free[NS], p_full[NPB], p_free[NPB], o_full, drain,
+    // xchg, aug_full
+    static constexpr int kNBar = 1 + 2 * NP + 2 * NS + 2 * NPB + 4;
     static constexpr int kSlot = kBar + 8 * kNBar;  // TMEM address, abort flag
     static constexpr int kBytes = kSlot + 16;
 };
@@ -119,6 +124,15 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr) {
     d |= (uint64_t)(1024 >> 4) << 32;
     d |= (uint64_t)1 << 46;
     d |= (uint64_t)2 << 61;
+    return d;
+}
+// 32-byte swizzled K-major operand of K = 16: rows of 32 bytes, 8-row groups 256 bytes apart
+__device__ __forceinline__ uint64_t desc_sw32(uint32_t saddr) {
+    uint64_t d = (uint64_t)((saddr >> 4) & 0x3FFFu);
+    d |= (uint64_t)1 << 16;
+    d |= (uint64_t)(256 >> 4) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)6 << 61;
     return d;
 }
 __device__ __forceinline__ void mma(uint32_t dt, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
@@ -199,10 +213,10 @@ __device__ __forceinline__ uint32_t shr_clamp(uint32_t v, uint32_t n) {
     return r;
 }
 // Constrained Shiftmax output from ShiftExp's parts (see attention.cu): floor(I_b F / 2^(sh0 + q)),
-// b = bits of the fp32 value (max + 2^23) - s
+// w = bits of the fp32 value s - (2^23 + max + 1) that the score MMA of passes 2 and 3 leaves in TMEM
 template <bool FASTQ>
-__device__ __forceinline__ uint32_t p_direct(uint32_t b, const ShiftExpC &c, uint32_t F, uint32_t sh0) {
-    uint32_t n = b + ((b + 1u) >> 1) - ((b + 15u) >> 4) - 1808793600u;
+__device__ __forceinline__ uint32_t p_direct(uint32_t w, const ShiftExpC &c, uint32_t F, uint32_t sh0) {
+    uint32_t n = exp_arg_from_neg_bits(w);
     n = min(n, (uint32_t)c.kI0);
     const uint32_t q = FASTQ ? __umulhi(n, c.m32) : (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
     const uint32_t Ib = ((q + 2u) * (uint32_t)c.I0 - n) >> 1;
@@ -220,13 +234,14 @@ struct GroupTc {
 
 // P of one score: (I_exp F) >> sh, or its direct form from ShiftExp's parts (DIRECT)
 template <bool FASTQ, bool DIRECT>
-__device__ __forceinline__ uint32_t p_of(uint32_t b, const ShiftExpC &se, const RowNorm &rn, uint32_t sh0) {
-    return DIRECT ? p_direct<FASTQ>(b, se, rn.F, sh0) : shiftmax_out(shift_exp_bits<FASTQ>(b, se), rn);
+__device__ __forceinline__ uint32_t p_of(uint32_t w, const ShiftExpC &se, const RowNorm &rn, uint32_t sh0) {
+    return DIRECT ? p_direct<FASTQ>(w, se, rn.F, sh0) : shiftmax_out(shift_exp_nbits<FASTQ>(w, se), rn);
 }
 
 // DIRECT: per-row s_d with I_b F < 2^32 (the host's condition), so P comes straight from ShiftExp's
-// parts; otherwise P = (I_exp F) >> sh from the 64-bit product.
-template <bool FASTQ, bool DIRECT>
+// parts; otherwise P = (I_exp F) >> sh from the 64-bit product.  SUM4: every ShiftExp value is below
+// 2^30 (I0 2^k_inter < 2^30, the host's condition), so four of them add up in 32 bits.
+template <bool FASTQ, bool DIRECT, bool SUM4>
 __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const __grid_constant__ TcArgs args) {
     const AttnParams &p = args.p;
     extern __shared__ uint8_t smem_raw[];
@@ -239,7 +254,8 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
     auto s_free = [&](int b) { return bq_full + 8u * (1 + 2 * NP + NS + b); };
     auto p_full = [&](int b) { return bq_full + 8u * (1 + 2 * NP + 2 * NS + b); };
     auto p_free = [&](int b) { return bq_full + 8u * (1 + 2 * NP + 2 * NS + NPB + b); };
-    const uint32_t o_full = bq_full + 8u * (1 + 2 * NP + 2 * NS + 2 * NPB), drain = o_full + 8u, xchg = o_full + 16u;
+    const uint32_t o_full = bq_full + 8u * (1 + 2 * NP + 2 * NS + 2 * NPB), drain = o_full + 8u, xchg = o_full + 16u,
+                   aug_full = o_full + 24u;
     uint32_t *tmem_slot = (uint32_t *)(sm + TcSmem::kSlot);
     volatile int *abort = (volatile int *)(sm + TcSmem::kSlot + 4);
 
@@ -290,6 +306,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         bar_init(o_full, 1);
         bar_init(drain, 1);
         bar_init(xchg, NSMX / 32);
+        bar_init(aug_full, 4);  // the four warps of the first column group write the constant-term rows
         *abort = 0;
         if (kbk < TKB)  // slot rows no window box writes: zero k rows give masked scores, zero v rows add nothing
             for (int sl = 0; sl < NP; ++sl)
@@ -319,7 +336,8 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             const uint32_t id_o = (1u << 4) | (1u << 16) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
             // descriptors: an address step of 16 bytes is 1 in the low word (addresses < 256 KB, no carry)
             const uint64_t dq = desc_sw128(sbase + TcSmem::kQ), dring = desc_sw128(sbase + TcSmem::kRing),
-                           dp = desc_sw128(sbase + TcSmem::kP);
+                           dp = desc_sw128(sbase + TcSmem::kP), daa = desc_sw32(sbase + TcSmem::kAugA),
+                           dab = desc_sw32(sbase + TcSmem::kAugB);
             // consumption state: the S buffer, the ring slot of the next k piece (and, in pass 3, of the
             // next v piece) and the P buffer, each with its phase bit
             int sb = 0, ks = 0, vs = 0, pb = 0;
@@ -331,8 +349,9 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     ph ^= 1u;
                 }
             };
-            // scores of the next key block into S[sb]; the k piece is released when they complete
-            auto issue_s = [&]() -> bool {
+            // scores of the next key block into S[sb] (aug: plus the constant term -(2^23 + max + 1) of
+            // each row, passes 2 and 3); the k piece is released when they complete
+            auto issue_s = [&](bool aug) -> bool {
                 if (!bar_wait(full(ks), kph, abort, p.status, kStatusTimeoutTma)) return false;
                 if (!bar_wait(s_free(sb), sph ^ 1u, abort, p.status, kStatusTimeoutOperand)) return false;
                 fence_after();
@@ -342,6 +361,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 mma(dt, dq + 2, dk + 2, id_s, 1u);
                 mma(dt, dq + 4, dk + 4, id_s, 1u);
                 mma(dt, dq + 6, dk + 6, id_s, 1u);
+                if (aug) mma(dt, daa, dab, id_s, 1u);
                 commit(s_full(sb));
                 commit(empty(ks));
                 if (++sb == NS) {
@@ -372,9 +392,10 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             };
             bool ok = bar_wait(bq_full, 0, abort, p.status, kStatusTimeoutTma);
             fence_after();
-            // passes 1 and 2: the k pieces in order
+            // passes 1 and 2: the k pieces in order; pass 2 waits for the rows' constant terms
             for (int j = 0; j < 2 * nkb && ok; ++j) {
-                ok = issue_s();
+                if (j == nkb) ok = bar_wait(aug_full, 0, abort, p.status, kStatusTimeoutOperand);
+                if (ok) ok = issue_s(j >= nkb);
                 adv(ks, kph, 1);
             }
             // pass 3: k piece of block kb, then its v piece; the P V of block kb is issued after the
@@ -383,7 +404,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             vph = kph;
             adv(vs, vph, 1);
             for (int kb = 0; kb < nkb && ok; ++kb) {
-                ok = issue_s();
+                ok = issue_s(true);
                 adv(ks, kph, 2);
                 if (ok && kb > 0) ok = issue_pv(kb == 1);
             }
@@ -457,7 +478,6 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         uint64_t sum = 0;
         RowNorm rn{};
         uint32_t sh0 = 0;
-        float mb = 0.f;
         // the other column groups' contributions to the row, through shared memory and the xchg barrier
         auto exchange = [&](int phase) -> bool {
             __syncwarp();
@@ -473,7 +493,28 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 if (!(ok = exchange(0))) break;
 #pragma unroll
                 for (int o = 1; o < NCQ; ++o) mx = fmaxf(mx, red_max[((cq + o) % NCQ) * TQ + row]);
-                mb = mx + 8388608.0f;  // ShiftExp(s - max) is read off (max + 2^23) - s
+                if (cq == 0) {
+                    // this row's constant term -(2^23 + max + 1) as fp16 terms against the key weights
+                    // (1, 2048, 2048, 2048): max + 1 = 2048 a3 + a0 with a0 in [0, 2047], |a3| <= 512,
+                    // every term exact in fp16 and every partial sum of the MMA an integer below 2^24.
+                    // Both 16-byte halves of the row hold the same terms and the key rows carry their
+                    // weights in one half only, so the product does not depend on which half the
+                    // swizzle puts where.  Rows past the group get zeros.
+                    const int m1 = tok < Tg ? __float2int_rn(mx) + 1 : 0;
+                    const int a3 = m1 >> 11, a0 = m1 - (a3 << 11);
+                    const uint32_t h0 = (uint32_t)__half_as_ushort(__int2half_rn(-a0)),
+                                   h3 = (uint32_t)__half_as_ushort(__int2half_rn(-a3));
+                    const uint32_t n2048 = tok < Tg ? 0xE800u : 0u;  // -2048
+                    const uint4 ra = make_uint4(h0 | (n2048 << 16), n2048 | (h3 << 16), 0u, 0u);
+                    *(uint4 *)(sm + TcSmem::kAugA + row * 32) = ra;
+                    *(uint4 *)(sm + TcSmem::kAugA + row * 32 + 16) = ra;
+                    // key row `row`: (1, 2048, 2048, 2048) in the first half, zeros in the second
+                    *(uint4 *)(sm + TcSmem::kAugB + row * 32) = make_uint4(0x3C00u | (0x6800u << 16), 0x6800u | (0x6800u << 16), 0u, 0u);
+                    *(uint4 *)(sm + TcSmem::kAugB + row * 32 + 16) = make_uint4(0u, 0u, 0u, 0u);
+                    fence_async_smem();
+                    __syncwarp();
+                    if (lane == 0) bar_arrive(aug_full);
+                }
             }
             if (pass == 2) {
                 red_sum[cq * TQ + row] = sum;
@@ -531,22 +572,28 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     } else if (pass == 1) {
                         uint32_t e[32];
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) e[c] = shift_exp_bits<FASTQ>(__float_as_uint(mb - __uint_as_float(s[c])), se);
+                        for (int c = 0; c < 32; ++c) e[c] = shift_exp_nbits<FASTQ>(s[c], se);
                         if (!whole) {
 #pragma unroll
                             for (int c = 0; c < 32; ++c) e[c] = c < nvalid ? e[c] : 0u;
                         }
-                        // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits
+                        // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits;
+                        // with SUM4 (I0 2^k < 2^30) four do
                         uint64_t part = 0;
+                        if constexpr (SUM4) {
 #pragma unroll
-                        for (int c = 0; c < 32; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
+                            for (int c = 0; c < 32; c += 4) part += (uint64_t)(e[c] + e[c + 1] + e[c + 2] + e[c + 3]);
+                        } else {
+#pragma unroll
+                            for (int c = 0; c < 32; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
+                        }
                         sum += part;
                     } else {
                         // P of the 32 keys as fp16 (exact integers below 1024): the bits of 1024 + P are
                         // 0x6400 | P, and one half2 subtraction of 1024 leaves P
                         uint32_t pw[32];
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) pw[c] = p_of<FASTQ, DIRECT>(__float_as_uint(mb - __uint_as_float(s[c])), se, rn, sh0);
+                        for (int c = 0; c < 32; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
                         if (!whole) {
 #pragma unroll
                             for (int c = 0; c < 32; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
@@ -673,15 +720,16 @@ bool kv_map(CUtensorMap *m, const void *base, const AttnParams &p, bool win, int
 }
 
 // One instantiation's launch; its shared-memory limit is raised once.
-template <bool FASTQ, bool DIRECT>
+template <bool FASTQ, bool DIRECT, bool SUM4>
 cudaError_t launch_tc_kernel(const TcArgs &a, dim3 grid, size_t smem, cudaStream_t s) {
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;
     std::call_once(once, [&] {
-        attr = cudaFuncSetAttribute(attn_tc_kernel<FASTQ, DIRECT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        attr = cudaFuncSetAttribute(attn_tc_kernel<FASTQ, DIRECT, SUM4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)smem);
     });
     if (attr != cudaSuccess) return attr;
-    attn_tc_kernel<FASTQ, DIRECT><<<grid, kThreadsTc, smem, s>>>(a);
+    attn_tc_kernel<FASTQ, DIRECT, SUM4><<<grid, kThreadsTc, smem, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -713,10 +761,12 @@ cudaError_t launch_attention_tc(const AttnParams &p, cudaStream_t s) {
     const size_t smem = 1024 + TcSmem::kBytes;
     a.nq = (Tg + TQ - 1) / TQ;
     const dim3 grid((unsigned)(a.nq * p.H * p.B * G2));
-    if (fastq && direct) return launch_tc_kernel<true, true>(a, grid, smem, s);
-    if (fastq) return launch_tc_kernel<true, false>(a, grid, smem, s);
-    if (direct) return launch_tc_kernel<false, true>(a, grid, smem, s);
-    return launch_tc_kernel<false, false>(a, grid, smem, s);
+    const bool sum4 = ((int64_t)p.smx.se.I0 << p.smx.se.k) < ((int64_t)1 << 30);
+    if (fastq && direct)
+        return sum4 ? launch_tc_kernel<true, true, true>(a, grid, smem, s) : launch_tc_kernel<true, true, false>(a, grid, smem, s);
+    if (fastq) return launch_tc_kernel<true, false, false>(a, grid, smem, s);
+    if (direct) return launch_tc_kernel<false, true, false>(a, grid, smem, s);
+    return launch_tc_kernel<false, false, false>(a, grid, smem, s);
 }
 
 }  // namespace ilw

@@ -105,6 +105,24 @@ __device__ __forceinline__ uint32_t shift_exp_bits(uint32_t b, const ShiftExpC &
     return Ib << (c.k - (int32_t)q);
 }
 
+// The same ShiftExp of the magnitude a = max - s, taken from w = bits of the fp32 value s - C with
+// C = 2^23 + max + 1 (the attention kernel's score MMA adds -C to q.k directly).  For integer scores
+// with 0 <= a < 2^23 - 1 that value is -(2^23 + a + 1), exact, so w = 0xCB000000 + a + 1.  Both
+// 0xCB000000 terms are multiples of 16, so w >> 1 and (w + 14) >> 4 are ceil(a/2) and ceil(a/16)
+// plus fixed constants, and with 32-bit wrap-around n = a + ceil(a/2) - ceil(a/16) is
+// w + (w >> 1) - ((w + 14) >> 4) - 0x23D00001.
+__device__ __forceinline__ uint32_t exp_arg_from_neg_bits(uint32_t w) {
+    return w + (w >> 1) - ((w + 14u) >> 4) - 0x23D00001u;
+}
+template <bool FASTQ>
+__device__ __forceinline__ uint32_t shift_exp_nbits(uint32_t w, const ShiftExpC &c) {
+    uint32_t n = exp_arg_from_neg_bits(w);
+    n = min(n, (uint32_t)c.kI0);
+    const uint32_t q = FASTQ ? __umulhi(n, c.m32) : (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
+    const uint32_t Ib = ((q + 2u) * (uint32_t)c.I0 - n) >> 1;
+    return Ib << (c.k - (int32_t)q);
+}
+
 // ---- Constrained Shiftmax row constants (Algorithm 2): from S_sum to (F, output shift).
 struct RowNorm {
     uint32_t F;

@@ -295,3 +295,23 @@ def test_clamped_magnitude_shiftexp(orc, I0, k):
     got = _shift_exp_mag_model(np.minimum(a, 1 << 30), I0, k)
     want = np.array([orc.shiftexp(-int(x), I0, k) for x in a], dtype=np.int64)
     assert np.array_equal(got, want)
+
+
+def test_shiftexp_exponent_from_negative_biased_bits():
+    """The attention kernel's score MMA adds -C = -(2^23 + max + 1) to q.k, so TMEM holds the fp32
+    value s - C = -(2^23 + a + 1) for a = max - s.  For every integer score pair with a in
+    [0, 2^22] (|scores| < 2^20, so a <= 2^21 in practice) that value is exact, its bits are
+    0xCB000000 + a + 1, and w + (w >> 1) - ((w + 14) >> 4) - 0x23D00001 (32-bit wrap-around) equals
+    a + ceil(a/2) - ceil(a/16)."""
+    a = np.arange(0, (1 << 22) + 1, dtype=np.int64)
+    mx = np.int64(12345)
+    s = mx - a
+    C = (1 << 23) + mx + 1
+    val = (s - C).astype(np.float32)  # exact: |s - C| < 2^24
+    assert np.array_equal(val.astype(np.int64), s - C)
+    w = val.view(np.uint32).astype(np.uint64)
+    assert np.array_equal(w, 0xCB000000 + a + 1)
+    M32 = np.uint64(0xFFFFFFFF)
+    n = (w + (w >> np.uint64(1)) - ((w + np.uint64(14)) >> np.uint64(4)) - np.uint64(0x23D00001)) & M32
+    assert np.array_equal(n.astype(np.int64), a + ((a + 1) >> 1) - ((a + 15) >> 4))
+
