@@ -3,6 +3,7 @@
 //
 // One warp owns one row; the row stays in registers between the two dependent reductions, so
 // HBM sees each input byte once.  Rows are read with 128-bit loads when the layout allows.
+#include <algorithm>
 #include <climits>
 #include <cstdint>
 #include <mutex>
@@ -196,13 +197,21 @@ __device__ __noinline__ uint64_t newton_isqrt_early(uint64_t V, int iters) {
 }
 
 // floor(V / r) for V < 2^48 and 1 <= r < 2^32 with a quotient below 2^26: a float estimate (relative
-// error < 2^-21, so absolute error < 2^5), one float refinement from the exact 64-bit remainder
-// (error < 1 on a remainder below 2^6 r), and a final +-1 test on the remainder.
+// error < 2^-20, so absolute error < 2^6), one float refinement from the exact 64-bit remainder
+// (error < 1 on a remainder below 2^7 r), and a final +-1 test on the remainder.
+// A 64-bit integer of magnitude below 2^62 as a float from its two 32-bit halves (two 32-bit
+// conversions and one multiply-add: relative error below 2^-22), instead of a 64-bit conversion.
+__device__ __forceinline__ float u64_to_float(uint64_t v) {
+    return fmaf(__uint2float_rn((uint32_t)(v >> 32)), 4294967296.0f, __uint2float_rn((uint32_t)v));
+}
+__device__ __forceinline__ float i64_to_float(int64_t v) {
+    return fmaf(__int2float_rn((int32_t)(v >> 32)), 4294967296.0f, __uint2float_rn((uint32_t)v));
+}
 __device__ __forceinline__ uint32_t div_u48_u32(uint64_t V, uint32_t r) {
     const float rinv = __frcp_rn(__uint2float_rn(r));
-    uint32_t q = __float2uint_rz(__ull2float_rn(V) * rinv);
+    uint32_t q = __float2uint_rz(u64_to_float(V) * rinv);
     int64_t rem = (int64_t)V - (int64_t)q * r;
-    const int32_t dq = __float2int_rd(__ll2float_rn(rem) * rinv);
+    const int32_t dq = __float2int_rd(i64_to_float(rem) * rinv);
     q += dq;
     rem -= (int64_t)dq * r;
     if (rem < 0) --q;
@@ -229,22 +238,6 @@ __device__ __forceinline__ uint64_t newton_isqrt_fast(uint64_t V, int iters) {
     }
     return r < 1 ? 1 : r;
 }
-
-// I-LayerNorm over tiles of LN_RB rows (Sec. 3.3; mean, variance, Newton's
-// integer square root, F = floor((2^31 - 1) / R), n = (y F) >> 1, out = sat(rq(n + beta; m, s))):
-//  (1) cp.async copies the tile into shared memory, rows padded by 16 bytes; the CTAs are
-//      persistent and double-buffered, so the next tile streams in while one is processed;
-//  (2) each warp sums slices of the columns of all the tile's rows, one row per lane (sum x, sum x^2 in
-//      int64; the padded pitch keeps the lanes' 16-byte reads on distinct banks);
-//  (3) warp 0 finishes the statistics, one row per lane: the Newton sequences of the tile run
-//      side by side instead of once per warp;
-//  (4) each thread owns 4 fixed columns (beta, m, s in registers) and normalises one 4-element
-//      group of a row per pass, with coalesced stores.
-// 32-bit arithmetic in (4) is exact: after at least one Newton step R >= isqrt(V) >= |y| for every
-// y = x - mu of the row (a floored Newton step from any positive start lands at or above isqrt(V)),
-// so |y F| <= |y| (2^31 - 1) / R < 2^31; with |beta| <= 2^30, n + beta fits int32 and for s >= 33 the
-// requantisation takes the high-word form.  Rows or columns outside those conditions use the
-// 64-bit formulas.
 
 // Output element types of I-LayerNorm: int8, int16, or the int8 values carried in fp16.
 template <typename TOut> struct LnOut { static constexpr int bits = 8 * (int)sizeof(TOut); };
@@ -277,13 +270,7 @@ __device__ __forceinline__ void madw(int64_t &acc, int32_t a, int32_t b) {
     asm("mad.wide.s32 %0, %1, %2, %0;" : "+l"(acc) : "r"(a), "r"(b));
 }
 
-struct LnRowStat {
-    int64_t mu, F;
-    int32_t fast;
-    int32_t mF;  // -mu * F in wrapping 32-bit arithmetic: (x F + mF) = (x - mu) F exactly when that fits int32
-};
-
-// The normalisation of 4 elements in 64-bit arithmetic, for tiles or columns outside the 32-bit
+// The normalisation of 4 elements in 64-bit arithmetic, for rows or columns outside the 32-bit
 // fast path's conditions (kept out of line so that its registers do not weigh on the fast path).
 __device__ __noinline__ void ln_norm4_exact(const int32_t (&x)[4], int64_t mu, int64_t F, const int32_t (&be)[4],
                                             const int32_t (&mm)[4], const int32_t (&ss)[4], int out_bits,
@@ -296,181 +283,150 @@ __device__ __noinline__ void ln_norm4_exact(const int32_t (&x)[4], int64_t mu, i
     }
 }
 
-template <typename TIn>
-__device__ __forceinline__ void ln_get4(const uint8_t *p, int32_t (&x)[4]) {
-    if (sizeof(TIn) == 4) {
-        const int4 v = *(const int4 *)p;
-        x[0] = v.x; x[1] = v.y; x[2] = v.z; x[3] = v.w;
-    } else {
-        const uint2 v = *(const uint2 *)p;
-        x[0] = (int32_t)(v.x << 16) >> 16; x[1] = (int32_t)v.x >> 16;
-        x[2] = (int32_t)(v.y << 16) >> 16; x[3] = (int32_t)v.y >> 16;
+// I-LayerNorm by row groups (Sec. 3.3; mean, variance, Newton's integer square root,
+// F = floor((2^31 - 1) / R), n = (y F) >> 1, out = sat(rq(n + beta; m, s))).  LPR lanes own one row,
+// 32 / LPR rows per warp, and every warp walks its own rows (persistent grid, no CTA barrier in the
+// loop).  A lane reads 16-byte chunks sub, sub + LPR, ... of its row (CPL at most; the LPR lanes of a
+// row read adjacent chunks, so a warp's load covers 32 / LPR row segments of LPR * 16 bytes), sums x
+// and x^2 (int64), and the LPR lanes combine them with shuffles; each lane then runs the row's Newton
+// sequence (the lanes of a row compute the same values, side by side with the other rows of the warp)
+// and normalises its own chunks with the per-column parameters from shared memory.
+// 32-bit normalisation: after at least one Newton step R >= isqrt(V) >= |y| for every y = x - mu of
+// the row (a floored Newton step from any positive start lands at or above isqrt(V)), so
+// |y F| <= |y| (2^31 - 1) / R < 2^31 and y F fits int32; with one shift s >= 33 for every column and
+// |beta| <= 2^30 the requantisation is the high-word form with a scalar rounding constant; otherwise
+// (or for rows with iters = 0 and V >= 2^32) the 64-bit formulas run.
+template <typename TIn, typename TOut, int LPR, int CPL>
+__global__ void __launch_bounds__(256) layernorm_rows(const LnParams p) {
+    extern __shared__ __align__(16) int32_t ln_par[];  // beta[C], mult[C], shift[C]
+    constexpr int EB = sizeof(TIn), EPC = 16 / EB;      // elements per 16-byte chunk
+    constexpr int RPW = 32 / LPR;
+    const int C = p.C, nch = C / EPC;
+    int32_t *s_beta = ln_par, *s_mult = ln_par + C, *s_shift = ln_par + 2 * C;
+    for (int i = threadIdx.x; i < C / 4; i += blockDim.x) {
+        ((int4 *)s_beta)[i] = __ldg((const int4 *)p.beta + i);
+        ((int4 *)s_mult)[i] = __ldg((const int4 *)p.mult + i);
+        ((int4 *)s_shift)[i] = __ldg((const int4 *)p.shift + i);
     }
-}
-
-template <typename TIn, typename TOut, int LN_RB>
-__global__ void __launch_bounds__(256) layernorm_tile(const LnParams p, int32_t pitch, int64_t ntiles) {
-    extern __shared__ __align__(16) uint8_t ln_smem[];
-    constexpr int EB = sizeof(TIn);
-    const int C = p.C, nc16 = C * EB / 16, nc4 = C / 4;
-    const int T = blockDim.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int nwarps = T >> 5;  // full warps (T >= 128)
-    constexpr int SPW = 32 / LN_RB;  // column slices per warp in (2): lane = slice * LN_RB + row
-    const int nslice = nwarps * SPW;
-    uint8_t *tiles = ln_smem;                                             // [2][LN_RB * pitch]
-    int64_t *part = (int64_t *)(tiles + 2 * LN_RB * pitch);               // [nslice][LN_RB][2]
-    LnRowStat *stat = (LnRowStat *)(part + 2 * LN_RB * nslice);          // [LN_RB]
-
-    // (1) tile t -> shared buffer `buf` with cp.async (one commit group per tile)
-    // T is a multiple of the 16-byte chunks per row (T = nc4 k and nc16 = nc4 EB / 4), so a thread
-    // copies the same chunk column of rows r_c, r_c + T / nc16, ...
-    const int ch_c = tid % nc16, r_c = tid / nc16, r_step = T / nc16;
-    const int64_t ld_bytes = p.ldx * EB;
-    const uint32_t tiles_s = (uint32_t)__cvta_generic_to_shared(tiles);
-    auto issue = [&](int64_t t, int buf) {
-        if (t < ntiles) {
-            const int64_t r0 = t * LN_RB;
-            const int nr = (int)min((int64_t)LN_RB, p.rows - r0);
-            const uint8_t *src = (const uint8_t *)p.X + r0 * ld_bytes + ch_c * 16;
-            const uint32_t dst0 = tiles_s + (uint32_t)(buf * LN_RB * pitch + ch_c * 16);
-            const uint8_t *g = src + r_c * ld_bytes;
-            const int64_t g_step = r_step * ld_bytes;
-            uint32_t dst = dst0 + (uint32_t)(r_c * pitch);
-            const uint32_t d_step = (uint32_t)(r_step * pitch);
-            for (int r = r_c; r < LN_RB; r += r_step, g += g_step, dst += d_step) {
-                const bool ok = r < nr;
-                asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(ok ? g : src),
-                             "r"(ok ? 16 : 0)
-                             : "memory");
-            }
-        }
-        asm volatile("cp.async.commit_group;" ::: "memory");
-    };
-    int64_t t = blockIdx.x;
-    issue(t, 0);
-    // this thread's 4 columns and their parameters, fetched while the first copies are in flight
-    const int cc = tid % nc4, rs = tid / nc4, kpass = T / nc4;
-    int32_t be[4], mm[4], ss[4];
-    {
-        const int4 b4 = __ldg((const int4 *)(p.beta + 4 * cc)), m4 = __ldg((const int4 *)(p.mult + 4 * cc)),
-                   s4 = __ldg((const int4 *)(p.shift + 4 * cc));
-        be[0] = b4.x; be[1] = b4.y; be[2] = b4.z; be[3] = b4.w;
-        mm[0] = m4.x; mm[1] = m4.y; mm[2] = m4.z; mm[3] = m4.w;
-        ss[0] = s4.x; ss[1] = s4.y; ss[2] = s4.z; ss[3] = s4.w;
-    }
+    __syncthreads();
+    const int32_t uniform_shift = s_shift[0];  // the fast form needs one shift >= 33 for every column
     bool col_fast = true;
-#pragma unroll
-    for (int u = 0; u < 4; ++u) col_fast &= ss[u] >= 33 && be[u] >= -(1 << 30) && be[u] <= (1 << 30);
-    int32_t rnd[4], sh[4];  // rq_hi constants of the 4 columns (used only when every shift is >= 33)
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-        rnd[u] = col_fast ? 1 << (ss[u] - 33) : 0;
-        sh[u] = ss[u] - 32;
-    }
-    // uniform over the CTA, so that (4) branches once per tile instead of predicating both forms
-    const bool cols_fast = __syncthreads_and(col_fast) != 0;
-    __shared__ int tile_fast;
+    for (int c = threadIdx.x; c < C; c += blockDim.x)
+        col_fast &= s_beta[c] >= -(1 << 30) && s_beta[c] <= (1 << 30) && s_shift[c] == uniform_shift;
+    const bool cols_fast = __syncthreads_and(col_fast) != 0 && uniform_shift >= 33;
+    const int32_t rnd = cols_fast ? 1 << (uniform_shift - 33) : 0, sh = uniform_shift - 32;
 
-    for (int buf = 0; t < ntiles; t += gridDim.x, buf ^= 1) {
-        issue(t + gridDim.x, buf ^ 1);  // the next tile streams in while this one is processed
-        asm volatile("cp.async.wait_group 1;" ::: "memory");
-        __syncthreads();
-        const uint8_t *tile = tiles + buf * LN_RB * pitch;
-        const int64_t row0 = t * LN_RB;
-        const int nrows = (int)min((int64_t)LN_RB, p.rows - row0);
-
-        // (2) column slice `sl` of row `rr`
-        {
-            const int rr = lane % LN_RB, sl = warp * SPW + lane / LN_RB;
-            const int per = (nc16 + nslice - 1) / nslice;
-            const int c0 = sl * per, c1 = min(nc16, c0 + per);
-            int64_t sx = 0, sq = 0;
-            if (warp < nwarps) {
-                const uint8_t *rp = tile + rr * pitch;
-                for (int ch = c0; ch < c1; ++ch) {
-                    const int4 v = *(const int4 *)(rp + ch * 16);
-                    if (EB == 4) {
-                        madw(sx, v.x, 1); madw(sx, v.y, 1); madw(sx, v.z, 1); madw(sx, v.w, 1);
-                        madw(sq, v.x, v.x); madw(sq, v.y, v.y); madw(sq, v.z, v.z); madw(sq, v.w, v.w);
-                    } else {
-                        const uint32_t w[4] = {(uint32_t)v.x, (uint32_t)v.y, (uint32_t)v.z, (uint32_t)v.w};
-                        int32_t s32 = 0;
+    const int lane = threadIdx.x & 31, sub = lane % LPR, rr = lane / LPR;
+    const int64_t ngroups = (p.rows + RPW - 1) / RPW;
+    const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t g = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); g < ngroups; g += wstride) {
+        const int64_t row = g * RPW + rr;
+        const bool live = row < p.rows;  // every lane stays for the shuffles
+        const uint8_t *xr = (const uint8_t *)p.X + (live ? row : 0) * p.ldx * EB;
+        int4 v[CPL];
 #pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const int32_t lo = (int32_t)(w[u] << 16) >> 16, hi = (int32_t)w[u] >> 16;
-                            s32 += lo + hi;
-                            sq += (int64_t)((uint32_t)(lo * lo) + (uint32_t)(hi * hi));  // <= 2^31
-                        }
-                        sx += s32;
-                    }
-                }
-                part[(sl * LN_RB + rr) * 2] = sx;
-                part[(sl * LN_RB + rr) * 2 + 1] = sq;
-            }
+        for (int i = 0; i < CPL; ++i) {
+            const int j = sub + LPR * i;
+            v[i] = (live && j < nch) ? __ldg((const int4 *)xr + j) : make_int4(0, 0, 0, 0);
         }
-        __syncthreads();
-
-        // (3) statistics of row `lane`, Newton's iteration side by side for the tile's rows (lanes
-        // past the tile's rows compute a dummy row)
-        if (warp == 0) {
-            const int lr = lane % LN_RB;
-            int64_t S = 0, Q = 0;
-            for (int w = 0; w < nslice; ++w) {
-                S += part[(w * LN_RB + lr) * 2];
-                Q += part[(w * LN_RB + lr) * 2 + 1];
-            }
-            const int64_t num = 2 * S + C, den = 2 * (int64_t)C;
-            int64_t mu;
-            if (num >= -(1ll << 31) && num < (1ll << 31)) {  // 32-bit floor division
-                const int32_t n32 = (int32_t)num, d32 = (int32_t)den;
-                const int32_t qt = n32 / d32;
-                mu = qt - ((n32 % d32 != 0 && n32 < 0) ? 1 : 0);
-            } else {
-                mu = num / den;
-                if ((num % den) != 0 && num < 0) mu -= 1;  // floor
-            }
-            const uint64_t V = (uint64_t)(Q - 2 * mu * S + (int64_t)C * mu * mu);
-            const uint64_t R = V < (1ull << 48) ? newton_isqrt_fast(V, p.iters) : newton_isqrt_early(V, p.iters);
-            LnRowStat st;
-            st.mu = mu;
-            st.F = R < (1ull << 32) ? (int64_t)div_int31((uint32_t)R) : 0;
-            st.fast = (p.iters >= 1 || V < (1ull << 32)) ? 1 : 0;
-            st.mF = (int32_t)(0u - (uint32_t)mu * (uint32_t)st.F);
-            if (lane < LN_RB) stat[lane] = st;
-            const bool all_fast = __all_sync(0xffffffffu, st.fast != 0);
-            if (lane == 0) tile_fast = all_fast ? 1 : 0;
-        }
-        __syncthreads();
-
-        // (4) normalise: rows rs, rs + kpass, ... of this thread's column group
-        TOut *ybase = (TOut *)p.Y + row0 * p.ldy + 4 * cc;
-        auto store = [&](int r, const int32_t (&o)[4]) { ln_store4<TOut>(ybase + (int64_t)r * p.ldy, o); };
-        if (tile_fast && cols_fast) {
-            // (x - mu) F = x F + mF in wrapping 32-bit arithmetic (the product fits int32), and
-            // rq takes its high-word form with the rounding constant folded in
-            for (int r = rs; r < nrows; r += kpass) {
-                const int32_t F = (int32_t)stat[r].F, mF = stat[r].mF;
-                int32_t x[4], o[4];
-                ln_get4<TIn>(tile + r * pitch + cc * 4 * EB, x);
+        // sum x and sum x^2 of the lane's chunks
+        int64_t S = 0, Q = 0;
+#pragma unroll
+        for (int i = 0; i < CPL; ++i) {
+            if constexpr (EB == 2) {
+                const uint32_t w[4] = {(uint32_t)v[i].x, (uint32_t)v[i].y, (uint32_t)v[i].z, (uint32_t)v[i].w};
+                int32_t s32 = 0;
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const int32_t n = (int32_t)((uint32_t)x[u] * (uint32_t)F + (uint32_t)mF) >> 1;
-                    const int32_t tq = rq_hi(n + be[u], mm[u], rnd[u], sh[u]);
-                    o[u] = LnOut<TOut>::bits == 8 ? clamp8(tq) : clamp16(tq);
+                    const int32_t lo = (int32_t)(w[u] << 16) >> 16, hi = (int32_t)w[u] >> 16;
+                    s32 += lo + hi;
+                    Q += (int64_t)((uint32_t)(lo * lo) + (uint32_t)(hi * hi));  // <= 2^31
                 }
-                store(r, o);
-            }
-        } else {
-            for (int r = rs; r < nrows; r += kpass) {
-                int32_t x[4], o[4];
-                ln_get4<TIn>(tile + r * pitch + cc * 4 * EB, x);
-                ln_norm4_exact(x, stat[r].mu, stat[r].F, be, mm, ss, LnOut<TOut>::bits, o);
-                store(r, o);
+                S += s32;
+            } else {
+                const int32_t e[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    madw(S, e[u], 1);
+                    madw(Q, e[u], e[u]);
+                }
             }
         }
-        __syncthreads();  // buffer `buf` and the statistics are free again
+#pragma unroll
+        for (int o = LPR / 2; o; o >>= 1) {
+            S += __shfl_xor_sync(0xffffffffu, S, o, LPR);
+            Q += __shfl_xor_sync(0xffffffffu, Q, o, LPR);
+        }
+        // mu = floor((2S + C) / (2C)); V = Q - 2 mu S + C mu^2 (= sum (x - mu)^2 exactly)
+        const int64_t num = 2 * S + C, den = 2 * (int64_t)C;
+        int64_t mu;
+        if (num >= -(1ll << 31) && num < (1ll << 31)) {
+            const int32_t n32 = (int32_t)num, d32 = (int32_t)den;
+            const int32_t qt = n32 / d32;
+            mu = qt - ((n32 % d32 != 0 && n32 < 0) ? 1 : 0);
+        } else {
+            mu = num / den;
+            if ((num % den) != 0 && num < 0) mu -= 1;
+        }
+        const uint64_t V = (uint64_t)(Q - 2 * mu * S + (int64_t)C * mu * mu);
+        const uint64_t R = V < (1ull << 48) ? newton_isqrt_fast(V, p.iters) : newton_isqrt_early(V, p.iters);
+        const int64_t F = R < (1ull << 32) ? (int64_t)div_int31((uint32_t)R) : 0;
+        const bool fast = cols_fast && __all_sync(0xffffffffu, p.iters >= 1 || V < (1ull << 32));
+        const int32_t F32 = (int32_t)F, mF = (int32_t)(0u - (uint32_t)mu * (uint32_t)F);
+        TOut *yr = (TOut *)p.Y + (live ? row : 0) * p.ldy;
+#pragma unroll
+        for (int i = 0; i < CPL; ++i) {
+            const int j = sub + LPR * i;
+            if (!live || j >= nch) continue;
+            int32_t x[EPC];
+            if constexpr (EB == 2) {
+                const uint32_t w[4] = {(uint32_t)v[i].x, (uint32_t)v[i].y, (uint32_t)v[i].z, (uint32_t)v[i].w};
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    x[2 * u] = (int32_t)(w[u] << 16) >> 16;
+                    x[2 * u + 1] = (int32_t)w[u] >> 16;
+                }
+            } else {
+                x[0] = v[i].x; x[1] = v[i].y; x[2] = v[i].z; x[3] = v[i].w;
+            }
+            const int c0 = j * EPC;
+            int32_t o[EPC];
+            if (fast) {
+#pragma unroll
+                for (int u4 = 0; u4 < EPC; u4 += 4) {
+                    const int4 b4 = *(const int4 *)(s_beta + c0 + u4), m4 = *(const int4 *)(s_mult + c0 + u4);
+                    const int32_t be[4] = {b4.x, b4.y, b4.z, b4.w}, mm[4] = {m4.x, m4.y, m4.z, m4.w};
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        // (x - mu) F = x F + mF in wrapping 32-bit arithmetic (the product fits int32)
+                        const int32_t n = (int32_t)((uint32_t)x[u4 + u] * (uint32_t)F32 + (uint32_t)mF) >> 1;
+                        const int32_t tq = rq_hi(n + be[u], mm[u], rnd, sh);
+                        o[u4 + u] = LnOut<TOut>::bits == 8 ? clamp8(tq) : clamp16(tq);
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int u4 = 0; u4 < EPC; u4 += 4) {
+                    int32_t xx[4], be[4], mm[4], ss[4], oo[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        xx[u] = x[u4 + u];
+                        be[u] = s_beta[c0 + u4 + u];
+                        mm[u] = s_mult[c0 + u4 + u];
+                        ss[u] = s_shift[c0 + u4 + u];
+                    }
+                    ln_norm4_exact(xx, mu, F, be, mm, ss, LnOut<TOut>::bits, oo);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) o[u4 + u] = oo[u];
+                }
+            }
+#pragma unroll
+            for (int u4 = 0; u4 < EPC; u4 += 4) {
+                const int32_t oo[4] = {o[u4], o[u4 + 1], o[u4 + 2], o[u4 + 3]};
+                ln_store4<TOut>(yr + c0 + u4, oo);
+            }
+        }
     }
-    asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
 template <typename TIn, typename TOut, int EPL>
@@ -528,35 +484,27 @@ cudaError_t ln_dispatch(const LnParams &p, cudaStream_t s) {
                        ((uintptr_t)p.X % 16) == 0 && ((uintptr_t)p.Y % (4 * ob)) == 0 &&
                        (((uintptr_t)p.beta | (uintptr_t)p.mult | (uintptr_t)p.shift) % 16) == 0 && p.C * eb <= 2048;
     if (tiled) {
-        constexpr int RB = 16;  // rows per tile
-        const int nc4 = p.C / 4, T = nc4 * (256 / nc4);
-        const int pitch = p.C * eb + 16;
-        const size_t smem =
-            (size_t)2 * RB * pitch + 2 * RB * (T / 32) * (32 / RB) * sizeof(int64_t) + RB * sizeof(LnRowStat);
-        static std::once_flag once;
-        static cudaError_t attr = cudaSuccess;
-        std::call_once(once, [] {
-            attr = cudaFuncSetAttribute(layernorm_tile<TIn, TOut, RB>, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
-        });
-        if (attr != cudaSuccess) return attr;
-        // persistent CTAs: as many as fit on the GPU at once, each striding over the tiles
-        static thread_local int last_T = -1, last_per_sm = 0, sms = 0;
-        static thread_local size_t last_smem = 0;
-        if (T != last_T || smem != last_smem) {
-            int dev = 0;
+        const int nch = p.C * eb / 16;
+        const size_t smem = (size_t)3 * p.C * sizeof(int32_t);
+        auto go = [&](auto kern) -> cudaError_t {
+            int dev = 0, sms = 0, per_sm = 0;
             cudaError_t e = cudaGetDevice(&dev);
             if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-            if (e == cudaSuccess)
-                e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&last_per_sm, layernorm_tile<TIn, TOut, RB>, T, smem);
+            if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, smem);
             if (e != cudaSuccess) return e;
-            last_T = T;
-            last_smem = smem;
-        }
-        const int per_sm = last_per_sm;
-        const int64_t ntiles = (p.rows + RB - 1) / RB;
-        const int64_t grid = min(ntiles, (int64_t)max(per_sm, 1) * sms);
-        layernorm_tile<TIn, TOut, RB><<<(unsigned)grid, T, smem, s>>>(p, pitch, ntiles);
-        return cudaGetLastError();
+            // persistent CTAs of 8 warps, at most one warp per row (each warp covers 32 / LPR rows)
+            const int64_t grid = std::max<int64_t>(1, std::min<int64_t>((int64_t)std::max(per_sm, 1) * sms,
+                                                                        (p.rows + 7) / 8));
+            kern<<<(unsigned)grid, 256, smem, s>>>(p);
+            return cudaGetLastError();
+        };
+        // chunks per lane: 6 for int16 rows (8 values each), 12 for int32 rows (4 values each), so a
+        // lane holds at most 48 values; lanes per row from the row's chunk count
+        constexpr int CPL = sizeof(TIn) == 2 ? 6 : 12;
+        if (nch <= 4 * CPL) return go(layernorm_rows<TIn, TOut, 4, CPL>);
+        if (nch <= 8 * CPL) return go(layernorm_rows<TIn, TOut, 8, CPL>);
+        if (nch <= 16 * CPL) return go(layernorm_rows<TIn, TOut, 16, CPL>);
+        if (nch <= 32 * CPL) return go(layernorm_rows<TIn, TOut, 32, CPL>);
     }
     const int rows_per_block = 8;
     dim3 grid((unsigned)((p.rows + rows_per_block - 1) / rows_per_block));

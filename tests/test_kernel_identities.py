@@ -148,12 +148,18 @@ def test_shiftmax_output_from_shiftexp_parts():
 
 def _div_u48_u32(V, r):
     """The kernels' floor(V / r) for V < 2^48, r < 2^32 (quotient < 2^26), in float32 arithmetic:
-    correctly rounded reciprocal, conversions to nearest, truncation / floor back to integers."""
+    correctly rounded reciprocal, 64-bit integers converted as two 32-bit halves joined by one fma,
+    truncation / floor back to integers."""
     f32 = np.float32
+
+    def to_f32(v):  # the kernels' conversion of a 64-bit integer: two 32-bit halves and one fma
+        hi, lo = v >> 32, v & 0xFFFFFFFF
+        return f32(float(f32(hi)) * 4294967296.0 + float(f32(lo)))  # exact in float64, rounded once
+
     rinv = f32(1.0) / f32(r)
-    q = np.uint64(np.trunc(f32(float(V)) * rinv))
+    q = np.uint64(np.trunc(to_f32(int(V)) * rinv))
     rem = int(V) - int(q) * int(r)
-    dq = int(np.floor(f32(float(rem)) * rinv))
+    dq = int(np.floor(to_f32(rem) * rinv))
     q = int(q) + dq
     rem -= dq * int(r)
     if rem < 0:
