@@ -56,6 +56,8 @@ constexpr int BM = 128, BK = 64;
 constexpr int kThreads = 448;
 constexpr int kMaxSeg = 8;
 constexpr int kSegK = 1024;  // max K per accumulator for exact fp32 accumulation
+constexpr int kMaxWk = kSegK / 64;  // K blocks of resident weights (one barrier each)
+constexpr int kStageBytes = 1024;   // per epilogue warp: the 32 x 16 output box of the TMA store
 constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
 
 struct Seg {
@@ -76,6 +78,8 @@ struct TcParams {  // CUtensorMap members keep the 64-byte alignment TMA needs
     int32_t nbuf;       // TMEM accumulator sets (1 or 2)
     int32_t wres_bytes; // resident weight bytes (WRES), a multiple of 1024
     int32_t tmem_cols;
+    int32_t tma_store;  // 1: outputs go out by TMA tensor stores of 32 x 16 boxes through shared memory
+    CUtensorMap cmap;   // C [M, N] with 16 x 32 boxes (2-byte outputs: 32-byte swizzle)
     const int8_t *gelu_tab;  // SD-ShiftGELU output table in global memory (16-byte aligned, 65536 bytes)
     int *status;
     EpiParams ep;
@@ -127,6 +131,16 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar)
         : "memory");
 }
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, int32_t x, int32_t y, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"((uint64_t)map),
+                 "r"(x), "r"(y), "r"(src)
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void fence_async_smem_g() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+__device__ __forceinline__ void tma_store_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void tma_store_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -338,6 +352,40 @@ __device__ __forceinline__ void store16(char *dst, const int32_t (&out)[16], int
     }
 }
 
+// 16 epilogue outputs of one row into row `lane` of the warp's 32 x 16 TMA-store box: 2-byte outputs
+// (fp16-carried int8, int16) as two 16-byte halves in the 32-byte swizzle the tensor map declares
+// (half j of row r at ((j ^ ((r >> 2) & 1)) << 4): no bank conflicts), 1-byte outputs as one 16-byte row.
+template <int KIND>
+__device__ __forceinline__ void box_row16(uint8_t *box, int lane, const int32_t (&out)[16]) {
+    if constexpr (KIND == KIND_F16OUT || KIND == KIND_GELU_F16) {
+        const __half2 k1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
+        uint32_t hw[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            uint32_t x = (uint32_t)(0x6480 + out[2 * j]) | ((uint32_t)(0x6480 + out[2 * j + 1]) << 16);
+            __half2 h = __hsub2(*reinterpret_cast<__half2 *>(&x), k1152);
+            hw[j] = *reinterpret_cast<uint32_t *>(&h);
+        }
+        const int sw = (lane >> 2) & 1;
+        *(uint4 *)(box + lane * 32 + (sw << 4)) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        *(uint4 *)(box + lane * 32 + ((sw ^ 1) << 4)) = make_uint4(hw[4], hw[5], hw[6], hw[7]);
+    } else if constexpr (KIND == KIND_RQ16) {
+        uint32_t w[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) w[j] = (uint32_t)(uint16_t)out[2 * j] | ((uint32_t)(uint16_t)out[2 * j + 1] << 16);
+        const int sw = (lane >> 2) & 1;
+        *(uint4 *)(box + lane * 32 + (sw << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+        *(uint4 *)(box + lane * 32 + ((sw ^ 1) << 4)) = make_uint4(w[4], w[5], w[6], w[7]);
+    } else {
+        uint32_t w[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            w[u] = (uint32_t)(uint8_t)out[4 * u] | ((uint32_t)(uint8_t)out[4 * u + 1] << 8) |
+                   ((uint32_t)(uint8_t)out[4 * u + 2] << 16) | ((uint32_t)(uint8_t)out[4 * u + 3] << 24);
+        *(uint4 *)(box + lane * 16) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
 // Waits for this thread's TMEM loads; every register of v is marked as written by the wait.
 template <int NSEG>
 __device__ __forceinline__ void tmem_wait_all(uint32_t (&v)[NSEG][16]) {
@@ -379,11 +427,15 @@ __device__ __forceinline__ void res_group(const int16_t *rrow, int c0, int ncol,
     }
 }
 
+// box: this warp's TMA-store box (nullptr: plain stores at dst), written out at column x0 + 16 c, row
+// y0 of cmap by lane 0 once every lane has written its row; the box is rewritten only after the
+// previous store has read it (that wait comes after the next chunk's arithmetic).
 template <int KIND, int BN, int HALF, int NSEG, bool RES>
 __device__ __forceinline__ void epi_fast(const EpiParams &ep, uint32_t tbase, const int32_t *s_bias,
                                          const int32_t *s_mult, int32_t rnd, int32_t sh, uint32_t (&rp)[16],
                                          const int16_t *rrow, bool rvec, char *dst, int ncol_row, bool vec_ok,
-                                         const int8_t *gt, uint32_t empty_bar, int lane) {
+                                         const int8_t *gt, uint32_t empty_bar, int lane, uint8_t *box,
+                                         const CUtensorMap *cmap, int x0, int y0) {
     static_assert(HALF % 32 == 0, "32-column groups");
     constexpr int NG = HALF / 32;                    // 32-column groups of the part
     // groups read per TMEM pass (32 registers per group and segment): the whole part for one segment
@@ -440,7 +492,14 @@ __device__ __forceinline__ void epi_fast(const EpiParams &ep, uint32_t tbase, co
                     out[i] = (KIND == KIND_RQ8 || KIND == KIND_F16OUT) ? clamp8(r) : clamp16(r);
                 }
             }
-            if (dst) {
+            if (box) {
+                if (lane == 0) tma_store_wait_read();  // the previous chunk's box has been read
+                __syncwarp();
+                box_row16<KIND>(box, lane, out);
+                fence_async_smem_g();
+                __syncwarp();
+                if (lane == 0 && 16 * c < ncol_row) tma_store_2d(cmap, x0 + 16 * c, y0, smem_u32(box));
+            } else if (dst) {
                 const int ncol = ncol_row - 16 * c;
                 if (ncol > 0) store16<KIND>(dst + 16 * c * esz, out, ncol, vec_ok && ncol >= 16);
             }
@@ -462,8 +521,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     constexpr int NWE = 4 * NP;
     uint8_t *wres = smem + STAGES * kStage;  // resident weights (WRES)
     uint64_t *bars = (uint64_t *)(wres + (WRES ? p.wres_bytes : 0));
-    // barriers: full[S], a_ready[S], empty[S], acc_full[2], acc_empty[2], wfull
-    uint32_t *tmem_slot = (uint32_t *)(bars + 3 * STAGES + 5);
+    // barriers: full[S], a_ready[S], empty[S], acc_full[2], acc_empty[2], wfull[kMaxWk] (one per K block
+    // of the resident weights, so the first MMAs start as soon as their own block has landed)
+    uint32_t *tmem_slot = (uint32_t *)(bars + 3 * STAGES + 4 + kMaxWk);
     volatile int *abort = (volatile int *)(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -473,7 +533,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     auto empty = [&](int s) { return bar0 + 8u * (2 * STAGES + s); };
     auto acc_full = [&](int b) { return bar0 + 8u * (3 * STAGES + b); };
     auto acc_empty = [&](int b) { return bar0 + 8u * (3 * STAGES + 2 + b); };
-    const uint32_t wfull = bar0 + 8u * (3 * STAGES + 4);
+    auto wfull = [&](int kk) { return bar0 + 8u * (3 * STAGES + 4 + kk); };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -485,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             mbar_init(acc_full(b), 1);
             mbar_init(acc_empty(b), NWE);
         }
-        mbar_init(wfull, 1);
+        for (int kk = 0; kk < kMaxWk; ++kk) mbar_init(wfull(kk), 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -509,21 +569,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         asm volatile("bar.sync 1, %0;" ::"r"(32 * NWE) : "memory");  // the epilogue warps only
     }
     const int acc_cols = p.nseg * BN;  // columns of one accumulator set
+    // the epilogue warps' TMA-store boxes (1024-byte aligned, after the parameters and the GELU table)
+    uint8_t *stg = (uint8_t *)(((uintptr_t)gtab + (gelu_kind(KIND) ? 65536 : 0) + 1023) & ~(uintptr_t)1023);
 
     if (warp == 0) {
         // ---------------------------------------------------------------- TMA producer
         if (lane == 0) {
             int it = 0;  // global K-block counter (ring position)
+            int wk = 0;  // K blocks of the resident weights issued
             bool ok = true;
-            if (WRES && blockIdx.x < p.tiles) {
-                // this CTA's BN rows of W, resident for all of its tiles (the grid is a multiple of
-                // tiles_n, so every tile of the CTA has the same n block)
-                const int n0 = (blockIdx.x % p.tiles_n) * BN;
-                const int nk = (p.seg[0].klen + BK - 1) / BK;
-                mbar_expect_tx(wfull, (uint32_t)(nk * SM::kWtile));
-                for (int kk = 0; kk < nk; ++kk)
-                    tma_load_2d(smem_u32(wres + kk * SM::kWtile), &p.wmap[0], p.seg[0].k0 + kk * BK, n0, wfull);
-            }
             for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x) {
                 const int m0 = (t / p.tiles_n) * BM, n0 = (t % p.tiles_n) * BN;
                 for (int sg = 0; sg < p.nseg && ok; ++sg) {
@@ -532,6 +586,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     for (int kk = 0; kk < nk; ++kk, ++it) {
                         const int s = it % STAGES;
                         const uint32_t ph = (it / STAGES) & 1;
+                        if (WRES && t == (int)blockIdx.x && kk < STAGES) {
+                            // the CTA's BN rows of W, resident for all of its tiles (the grid is a
+                            // multiple of tiles_n, so every tile of the CTA has the same n block): the
+                            // first K blocks travel with the first tile's activations of the same K block,
+                            // the rest follow at once (they have shared memory of their own)
+                            const int last = kk == (STAGES < nk ? STAGES : nk) - 1 ? nk - 1 : kk;
+                            for (int j = kk; j <= last; ++j) {
+                                mbar_expect_tx(wfull(j), (uint32_t)SM::kWtile);
+                                tma_load_2d(smem_u32(wres + j * SM::kWtile), &p.wmap[0], p.seg[0].k0 + j * BK, n0,
+                                            wfull(j));
+                            }
+                            wk = last + 1;
+                        }
                         if (!mbar_wait(empty(s), ph ^ 1, abort, p.status, kStatusTimeoutFree)) {
                             ok = false;
                             break;
@@ -546,8 +613,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             }
             if (!ok) {  // drain the loads still in flight (bounded) before the CTA can exit
                 long long t0 = clock64();
-                while (WRES && blockIdx.x < p.tiles && !mbar_try(wfull, 0) && clock64() - t0 < kWaitCycles) {
-                }
+                for (int kk = 0; kk < wk; ++kk)
+                    while (!mbar_try(wfull(kk), 0) && clock64() - t0 < kWaitCycles) {
+                    }
                 for (int j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
                     while (!mbar_try(full(j % STAGES), (j / STAGES) & 1) && clock64() - t0 < kWaitCycles) {
                     }
@@ -559,10 +627,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             const uint32_t idesc = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
             int it = 0, tl = 0;
             bool ok = true;
-            if (WRES && blockIdx.x < p.tiles) {
-                ok = mbar_wait(wfull, 0, abort, p.status, kStatusTimeoutTma);
-                tc_fence_after();
-            }
             for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++tl) {
                 const int b = tl % p.nbuf;
                 const uint32_t use = (uint32_t)(tl / p.nbuf);
@@ -576,7 +640,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                         const int s = it % STAGES;
                         const uint32_t ph = (it / STAGES) & 1;
                         if (!mbar_wait(AF16 ? full(s) : a_ready(s), ph, abort, p.status,
-                                       AF16 ? kStatusTimeoutTma : kStatusTimeoutOperand)) {
+                                       AF16 ? kStatusTimeoutTma : kStatusTimeoutOperand) ||
+                            (WRES && tl == 0 && !mbar_wait(wfull(kk), 0, abort, p.status, kStatusTimeoutTma))) {
                             ok = false;
                             break;
                         }
@@ -707,20 +772,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     const int32_t rnd = 1 << (s_0 - 33), sh = s_0 - 32;
                     const int8_t *gt = gtab + 32767;
                     const uint32_t eb = acc_empty(b);
+                    uint8_t *box = p.tma_store ? stg + (warp - EPI0) * kStageBytes : nullptr;
                     if (p.nseg == 1) {
                         if (kResKind && has_res)
                             epi_fast<KIND, BN, HALF, 1, kResKind>(ep, tbase, s_bias, s_mult, rnd, sh, rpa, rrow, rvec, dst,
-                                                                   ncol_row, vec_ok, gt, eb, lane);
+                                                                   ncol_row, vec_ok, gt, eb, lane, box, &p.cmap, n0,
+                                                                   m0 + 32 * q);
                         else
                             epi_fast<KIND, BN, HALF, 1, false>(ep, tbase, s_bias, s_mult, rnd, sh, rpa, rrow, rvec, dst,
-                                                               ncol_row, vec_ok, gt, eb, lane);
+                                                               ncol_row, vec_ok, gt, eb, lane, box, &p.cmap, n0,
+                                                               m0 + 32 * q);
                     } else {
                         if (kResKind && has_res)
                             epi_fast<KIND, BN, HALF, 2, kResKind>(ep, tbase, s_bias, s_mult, rnd, sh, rpa, rrow, rvec, dst,
-                                                                   ncol_row, vec_ok, gt, eb, lane);
+                                                                   ncol_row, vec_ok, gt, eb, lane, box, &p.cmap, n0,
+                                                                   m0 + 32 * q);
                         else
                             epi_fast<KIND, BN, HALF, 2, false>(ep, tbase, s_bias, s_mult, rnd, sh, rpa, rrow, rvec, dst,
-                                                               ncol_row, vec_ok, gt, eb, lane);
+                                                               ncol_row, vec_ok, gt, eb, lane, box, &p.cmap, n0,
+                                                               m0 + 32 * q);
                     }
                     continue;
                 }
@@ -862,6 +932,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 else go(F_{}, F_{});
             }
         }
+        if (p.tma_store && lane == 0) tma_store_wait_all();  // this warp's stores are complete
     }
 
     tc_fence_before();
@@ -876,16 +947,22 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 inline int num_sms() { return sm_count(); }
 
 // Dynamic shared memory of one instantiation (wres: resident weight bytes).
+// stg: the epilogue warps' TMA-store boxes (0 without TMA stores).
 template <int BN, int STAGES, int KIND, bool AF16, bool WRES>
-size_t smem_bytes(int wres) {
-    return 1024 + (size_t)STAGES * Smem<BN, AF16, WRES>::kStage + (WRES ? wres : 0) + 8 * (3 * STAGES + 5) + 32 +
-           4 * 4 * BN * 4 + (gelu_kind(KIND) ? 65536 : 0);
+size_t smem_bytes(int wres, int stg = 0) {
+    return 1024 + (size_t)STAGES * Smem<BN, AF16, WRES>::kStage + (WRES ? wres : 0) + 8 * (3 * STAGES + 4 + kMaxWk) +
+           32 + 4 * 4 * BN * 4 + (gelu_kind(KIND) ? 65536 : 0) + (stg ? 1024 + stg : 0);
 }
+template <int BN, bool AF16>
+constexpr int epi_warps() { return 4 * ((AF16 && BN == 192) ? 3 : 2); }
 constexpr size_t kSmemMax = 227 * 1024;
 
 template <int BN, int STAGES, int KIND, int NB, bool AF16, bool WRES>
 cudaError_t launch_tc(TcParams<NB> &tp, cudaStream_t s) {
-    const size_t smem = smem_bytes<BN, STAGES, KIND, AF16, WRES>(tp.wres_bytes);
+    // TMA stores when the output allows them (set up by run) and their boxes fit next to the rest
+    constexpr int stg = epi_warps<BN, AF16>() * kStageBytes;
+    if (tp.tma_store && smem_bytes<BN, STAGES, KIND, AF16, WRES>(tp.wres_bytes, stg) > kSmemMax) tp.tma_store = 0;
+    const size_t smem = smem_bytes<BN, STAGES, KIND, AF16, WRES>(tp.wres_bytes, tp.tma_store ? stg : 0);
     if (smem > kSmemMax) return cudaErrorInvalidValue;
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
@@ -952,6 +1029,18 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     while (alloc < tp.nbuf * one) alloc <<= 1;
     if (alloc > 512) return cudaErrorInvalidValue;
     tp.tmem_cols = alloc;
+    // TMA tensor stores of the outputs: 16 x 32 boxes of C (1-byte outputs: 16-byte box rows; 2-byte
+    // outputs: 32-byte rows in the 32-byte swizzle), for a C whose rows start on 16-byte boundaries
+    tp.tma_store = 0;
+    if (NB == 1 && ep.out_bits != 32) {
+        const int esz = ep.out_bits == 8 ? 1 : 2;  // int8, or int16 / fp16-carried int8
+        if (((uintptr_t)ep.C % 16) == 0 && (ep.ldc * esz) % 16 == 0 && gp.N * esz >= 16)
+            tp.tma_store = gemm_make_map(&tp.cmap, ep.C, esz == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16,
+                                         esz, gp.M, gp.N, ep.ldc, 16, 32,
+                                         esz == 1 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_32B)
+                               ? 1
+                               : 0;
+    }
     if (WRES) {
         if (nseg != 1) return cudaErrorInvalidValue;
         tp.wres_bytes = ((tp.seg[0].klen + BK - 1) / BK) * Smem<BN, AF16, WRES>::kWtile;
