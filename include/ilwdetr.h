@@ -254,6 +254,16 @@ int ilwdetr_patch_embed_noalloc(const int8_t *img, int32_t B, int32_t Cin, int32
                                 const int32_t *shift, int32_t d, const int16_t *pos, int32_t m_pos,
                                 int32_t s_pos, int16_t *x0, ilw_stream_t stream);
 
+/* Test hook of the bounded device waits (the paper has no counterpart; off by default).  Every
+ * wait inside the kernels is bounded; when one runs out the kernel latches the device status word,
+ * stops, drains the copies it issued, frees its tensor memory and returns, and
+ * ilwdetr_device_status() then reports ILW_ERR_TIMEOUT.  This call makes that path testable
+ * without a fault: GEMM launches made after it skip the operand load of their K-block counter
+ * `skip_load` (so the wait for it never completes; -1 = none) and bound every wait by
+ * `wait_cycles` SM clock cycles (0 = the default, about one second).  Process-wide; not for use
+ * while other threads launch GEMMs.  Call ilwdetr_debug_gemm_wait(-1, 0) to restore. */
+int ilwdetr_debug_gemm_wait(int32_t skip_load, int64_t wait_cycles);
+
 /* ------------------------------------------------------------------ encoder block */
 
 /* Integer parameters of one encoder block (all pointers are device pointers; weights packed

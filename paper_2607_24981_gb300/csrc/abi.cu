@@ -102,6 +102,12 @@ int ilwdetr_device_status(ilw_stream_t stream) {
     return ILW_OK;
 }
 
+int ilwdetr_debug_gemm_wait(int32_t skip_load, int64_t wait_cycles) {
+    if (skip_load < -1 || wait_cycles < 0) return fail(ILW_ERR_INVALID_ARG, "debug_gemm_wait: skip_load >= -1, wait_cycles >= 0");
+    ilw::gemm_set_debug_wait(skip_load, (long long)wait_cycles);
+    return ILW_OK;
+}
+
 size_t ilwdetr_packed_weight_bytes(int32_t N, int32_t K) {
     if (N < 0 || K < 0) return 0;
     return ilw::packed_weight_bytes(N, K);

@@ -1,6 +1,8 @@
 // gemm_tc.cu -- host side of the tensor-core integer GEMM (tensor maps, SD-ShiftGELU output tables,
 // weight packing, launch-shape choice) and its fp16-A launch shapes; the kernel is in gemm_tc.cuh,
 // the int8-A launch shapes in gemm_tc_i8.cu.
+#include <atomic>
+
 #include "gemm_tc.cuh"
 
 namespace ilw {
@@ -153,6 +155,20 @@ bool gemm_make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int
 }
 const int8_t *gemm_gelu_table(const GeluC &c, int32_t m_g, int32_t s_g, cudaStream_t s, cudaError_t *err) {
     return gelu_table_impl(c, m_g, s_g, s, err);
+}
+
+namespace {
+std::atomic<int32_t> g_dbg_skip{-1};
+std::atomic<long long> g_dbg_cycles{0};
+}  // namespace
+void gemm_debug_wait(int32_t *skip, long long *cycles) {
+    *skip = g_dbg_skip.load(std::memory_order_relaxed);
+    const long long c = g_dbg_cycles.load(std::memory_order_relaxed);
+    *cycles = c > 0 ? c : kWaitCycles;
+}
+void gemm_set_debug_wait(int32_t skip, long long cycles) {
+    g_dbg_skip.store(skip, std::memory_order_relaxed);
+    g_dbg_cycles.store(cycles, std::memory_order_relaxed);
 }
 
 cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, cudaStream_t s) {

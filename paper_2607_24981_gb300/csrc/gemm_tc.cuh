@@ -45,6 +45,9 @@ namespace ilw {
 bool gemm_make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int esize, int64_t rows, int64_t cols,
                    int64_t ld, int box_cols, int box_rows, CUtensorMapSwizzle sw);
 const int8_t *gemm_gelu_table(const GeluC &c, int32_t m_g, int32_t s_g, cudaStream_t s, cudaError_t *err);
+// The wait bound of the next GEMM launches and the K block whose load the producer skips (-1: none),
+// as set by ilwdetr_debug_gemm_wait (defaults: about one second, none).
+void gemm_debug_wait(int32_t *skip, long long *cycles);
 struct GemmProblem;
 struct EpiParams;
 // The int8-A launch shapes (gemm_tc_i8.cu): run<BN, STAGES, NB, false, false, GELU>.
@@ -58,7 +61,7 @@ constexpr int kMaxSeg = 8;
 constexpr int kSegK = 1024;  // max K per accumulator for exact fp32 accumulation
 constexpr int kMaxWk = kSegK / 64;  // K blocks of resident weights (one barrier each)
 constexpr int kStageBytes = 1024;   // per epilogue warp: the 32 x 16 output box of the TMA store
-constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz
+constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at 2 GHz: the default bound of every wait
 
 struct Seg {
     int32_t k0, klen;   // K range of this accumulator (same columns of A and W)
@@ -79,6 +82,8 @@ struct TcParams {  // CUtensorMap members keep the 64-byte alignment TMA needs
     int32_t wres_bytes; // resident weight bytes (WRES), a multiple of 1024
     int32_t tmem_cols;
     int32_t tma_store;  // 1: outputs go out by TMA tensor stores of 32 x 16 boxes through shared memory
+    int32_t dbg_skip;   // test hook: the producer issues no load for this K-block counter value (-1: none)
+    long long wait_cycles;  // the bound of every wait (about one second, shorter for the test hook)
     CUtensorMap cmap;   // C [M, N] with 16 x 32 boxes (2-byte outputs: 32-byte swizzle)
     const int8_t *gelu_tab;  // SD-ShiftGELU output table in global memory (16-byte aligned, 65536 bytes)
     int *status;
@@ -110,13 +115,14 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
 }
 // Bounded wait: true when the phase completed; false (after latching `code` in the status word
 // and raising the CTA's abort flag) when it ran out, or when another role already aborted.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort, int *status, int code) {
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort, int *status, int code,
+                                          long long limit) {
     long long t0 = clock64();
     for (uint32_t i = 0;; ++i) {
         if (mbar_try(bar, parity)) return true;
         if ((i & 255) == 255) {
             if (*abort) return false;
-            if (clock64() - t0 > kWaitCycles) {
+            if (clock64() - t0 > limit) {
                 if (status) atomicExch(status, code);
                 *abort = 1;
                 return false;
@@ -523,7 +529,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     uint64_t *bars = (uint64_t *)(wres + (WRES ? p.wres_bytes : 0));
     // barriers: full[S], a_ready[S], empty[S], acc_full[2], acc_empty[2], wfull[kMaxWk] (one per K block
     // of the resident weights, so the first MMAs start as soon as their own block has landed)
-    uint32_t *tmem_slot = (uint32_t *)(bars + 3 * STAGES + 4 + kMaxWk);
+    uint32_t *tmem_slot = (uint32_t *)(bars + 3 * STAGES + 5 + kMaxWk);
     volatile int *abort = (volatile int *)(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -534,6 +540,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     auto acc_full = [&](int b) { return bar0 + 8u * (3 * STAGES + b); };
     auto acc_empty = [&](int b) { return bar0 + 8u * (3 * STAGES + 2 + b); };
     auto wfull = [&](int kk) { return bar0 + 8u * (3 * STAGES + 4 + kk); };
+    const uint32_t drain = bar0 + 8u * (3 * STAGES + 4 + kMaxWk);  // every MMA issued has completed
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -546,6 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             mbar_init(acc_empty(b), NWE);
         }
         for (int kk = 0; kk < kMaxWk; ++kk) mbar_init(wfull(kk), 1);
+        mbar_init(drain, 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -599,11 +607,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                             }
                             wk = last + 1;
                         }
-                        if (!mbar_wait(empty(s), ph ^ 1, abort, p.status, kStatusTimeoutFree)) {
+                        if (!mbar_wait(empty(s), ph ^ 1, abort, p.status, kStatusTimeoutFree, p.wait_cycles)) {
                             ok = false;
                             break;
                         }
                         uint8_t *st = smem + s * kStage;
+                        if (it == p.dbg_skip) continue;  // test hook: this stage's barrier never completes
                         mbar_expect_tx(full(s), (AF16 ? SM::kA16 : SM::kA8) + SM::kW);
                         tma_load_2d(smem_u32(AF16 ? st : st + SM::kA16 + SM::kW), &p.amap[S.map], S.k0 + kk * BK, m0,
                                     full(s));
@@ -611,13 +620,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     }
                 }
             }
-            if (!ok) {  // drain the loads still in flight (bounded) before the CTA can exit
+            if (!ok || *abort) {  // drain the loads still in flight (bounded) before the CTA can exit
                 long long t0 = clock64();
                 for (int kk = 0; kk < wk; ++kk)
-                    while (!mbar_try(wfull(kk), 0) && clock64() - t0 < kWaitCycles) {
+                    while (!mbar_try(wfull(kk), 0) && clock64() - t0 < p.wait_cycles) {
                     }
                 for (int j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
-                    while (!mbar_try(full(j % STAGES), (j / STAGES) & 1) && clock64() - t0 < kWaitCycles) {
+                    while (j != p.dbg_skip && !mbar_try(full(j % STAGES), (j / STAGES) & 1) &&
+                           clock64() - t0 < p.wait_cycles) {
                     }
             }
         }
@@ -630,7 +640,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
             for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++tl) {
                 const int b = tl % p.nbuf;
                 const uint32_t use = (uint32_t)(tl / p.nbuf);
-                if (!mbar_wait(acc_empty(b), (use & 1) ^ 1, abort, p.status, kStatusTimeoutMma)) break;
+                if (!mbar_wait(acc_empty(b), (use & 1) ^ 1, abort, p.status, kStatusTimeoutMma, p.wait_cycles)) break;
                 tc_fence_after();
                 for (int sg = 0; sg < p.nseg && ok; ++sg) {
                     const Seg &S = p.seg[sg];
@@ -640,8 +650,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                         const int s = it % STAGES;
                         const uint32_t ph = (it / STAGES) & 1;
                         if (!mbar_wait(AF16 ? full(s) : a_ready(s), ph, abort, p.status,
-                                       AF16 ? kStatusTimeoutTma : kStatusTimeoutOperand) ||
-                            (WRES && tl == 0 && !mbar_wait(wfull(kk), 0, abort, p.status, kStatusTimeoutTma))) {
+                                       AF16 ? kStatusTimeoutTma : kStatusTimeoutOperand, p.wait_cycles) ||
+                            (WRES && tl == 0 && !mbar_wait(wfull(kk), 0, abort, p.status, kStatusTimeoutTma, p.wait_cycles))) {
                             ok = false;
                             break;
                         }
@@ -657,6 +667,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                 }
                 tc_commit(acc_full(b));  // arrives once every MMA of this tile has completed
             }
+            // every MMA issued has completed before the CTA can reach the TMEM release (also after an
+            // abort, when the epilogue no longer waits for the accumulators)
+            tc_commit(drain);
+            const long long t0 = clock64();
+            while (!mbar_try(drain, 0) && clock64() - t0 < p.wait_cycles) {
+            }
         }
     } else if (warp < EPI0) {
         // ---------------------------------------------------------------- operand converters
@@ -670,7 +686,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     for (int kk = 0; kk < nk; ++kk, ++it) {
                         const int s = it % STAGES;
                         const uint32_t ph = (it / STAGES) & 1;
-                        if (!mbar_wait(full(s), ph, abort, p.status, kStatusTimeoutTma)) goto conv_done;
+                        if (!mbar_wait(full(s), ph, abort, p.status, kStatusTimeoutTma, p.wait_cycles)) goto conv_done;
                         uint8_t *st = smem + s * kStage;
                         const uint8_t *a8 = st + SM::kA16 + SM::kW + r * 64;
                         uint8_t *a16 = st + r * 128;
@@ -764,7 +780,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
 #pragma unroll
                     for (int j = 0; j < 16; ++j) rpa[j] = 0;
                     if (kResKind && has_res) res_group(rrow, 0, p.N - n0, rvec, rpa);
-                    if (!mbar_wait(acc_full(b), use & 1, abort, p.status, kStatusTimeoutMma)) break;
+                    if (!mbar_wait(acc_full(b), use & 1, abort, p.status, kStatusTimeoutMma, p.wait_cycles)) break;
                     tc_fence_after();
                     char *dst = row_ok ? (char *)ep.C + (row * ep.ldc + n0) * (bits / 8) : nullptr;
                     const bool vec_ok = ((uintptr_t)dst & 15) == 0;
@@ -795,7 +811,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     continue;
                 }
             }
-            if (!mbar_wait(acc_full(b), use & 1, abort, p.status, kStatusTimeoutMma)) break;
+            if (!mbar_wait(acc_full(b), use & 1, abort, p.status, kStatusTimeoutMma, p.wait_cycles)) break;
             tc_fence_after();
             uint32_t rp[8];
             // The tile's chunks, with the requantisation forms fixed for the whole tile (a branch per
@@ -950,7 +966,7 @@ inline int num_sms() { return sm_count(); }
 // stg: the epilogue warps' TMA-store boxes (0 without TMA stores).
 template <int BN, int STAGES, int KIND, bool AF16, bool WRES>
 size_t smem_bytes(int wres, int stg = 0) {
-    return 1024 + (size_t)STAGES * Smem<BN, AF16, WRES>::kStage + (WRES ? wres : 0) + 8 * (3 * STAGES + 4 + kMaxWk) +
+    return 1024 + (size_t)STAGES * Smem<BN, AF16, WRES>::kStage + (WRES ? wres : 0) + 8 * (3 * STAGES + 5 + kMaxWk) +
            32 + 4 * 4 * BN * 4 + (gelu_kind(KIND) ? 65536 : 0) + (stg ? 1024 + stg : 0);
 }
 template <int BN, bool AF16>
@@ -1029,6 +1045,7 @@ cudaError_t run(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s) {
     while (alloc < tp.nbuf * one) alloc <<= 1;
     if (alloc > 512) return cudaErrorInvalidValue;
     tp.tmem_cols = alloc;
+    gemm_debug_wait(&tp.dbg_skip, &tp.wait_cycles);
     // TMA tensor stores of the outputs: 16 x 32 boxes of C (1-byte outputs: 16-byte box rows; 2-byte
     // outputs: 32-byte rows in the 32-byte swizzle), for a C whose rows start on 16-byte boundaries
     tp.tma_store = 0;

@@ -85,6 +85,9 @@ inline const void *packed_f16(const void *p, int32_t, int32_t) { return p; }
 cudaError_t launch_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, cudaStream_t s);
 // tcgen05 tensor-core GEMM (exact integer via fp16 operands, fp32 TMEM accumulators)
 cudaError_t launch_gemm(const GemmProblem &gp, const EpiParams &ep, cudaStream_t s);
+// Test hook of the bounded waits (ilwdetr_debug_gemm_wait): later GEMM launches skip the load of
+// K-block counter `skip` (-1: none) and bound every wait by `cycles` (0: the default, about 1 s).
+void gemm_set_debug_wait(int32_t skip, long long cycles);
 
 // ---------------------------------------------------------------- row / element kernels
 struct ShiftmaxC {
