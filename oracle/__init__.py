@@ -523,6 +523,42 @@ def detection_head(hp: dict, out: np.ndarray, ref16: np.ndarray):
     return scores, boxes, z
 
 
+def refine_references(rp: dict, t: np.ndarray, ref16: np.ndarray):
+    """Box refinement after a decoder layer (the two-stage pipeline's references refined layer by
+    layer, Sec. 3.1.2; the head rows of Table 5; the logit-domain update is a reading, as the paper
+    gives no integer inverse sigmoid):
+      a      = sat8(rq(t; m_in, s_in))                              (decoder output, int16 -> int8)
+      d      = Linear_3(ReLU(Linear_2(ReLU(Linear_1(a)))))          (raw int32 deltas)
+      ref16' = sat16(rq(d; m_d, s_d) + rq(ref16; m_ref, s_ref))     (new reference logits, scale 2^-10)
+      boxes  = IntSigmoid(ref16') with k_out = 17                   (cx, cy, w, h at scale 2^-16)
+    Returns (ref16' int16 [M, 4], boxes int32 [M, 4])."""
+    a = requant(t, rp["m_in"], rp["s_in"], out_bits=8).astype(np.int8)
+    h1 = relu(gemm_requant(a, rp["w_b1"], rp["b_b1"], rp["m_b1"], rp["s_b1"], 8).astype(np.int8))
+    h2 = relu(gemm_requant(h1, rp["w_b2"], rp["b_b2"], rp["m_b2"], rp["s_b2"], 8).astype(np.int8))
+    d = gemm_requant(h2, rp["w_b3"], rp["b_b3"], None, None, 32)
+    ref = requant(d, rp["m_d"], rp["s_d"], ref16, rp["m_ref"], rp["s_ref"], out_bits=16).astype(np.int16)
+    boxes = int_sigmoid(ref.astype(np.int32), rp["box_I0"], rp["k_inter"], 17)
+    return ref, boxes
+
+
+def decoder_stack(dps: list, tgt: np.ndarray, memory: np.ndarray, level_hw, ref16: np.ndarray,
+                  boxes: np.ndarray, B: int, Q: int, pq: dict | None = None, pos: np.ndarray | None = None,
+                  rps: list | None = None):
+    """The decoder layers with the references refined between them: layer l samples at the (cx, cy)
+    of the current boxes with positional queries from the learnable projection of those boxes (pq),
+    or the fixed `pos`; after every layer but the last, the box branch rps[l] gives the next
+    references (refine_references).  Without rps the references stay fixed.  Returns (decoder output
+    int16 [B*Q, d], the last layer's input reference logits int16 [B*Q, 4])."""
+    t = tgt
+    for l, dp in enumerate(dps):
+        refs = np.ascontiguousarray(boxes[:, :2]).reshape(B, Q, 2).astype(np.int32)
+        p = query_pos(pq, boxes) if pq is not None else pos
+        t = decoder_layer(dp, t, p, memory, level_hw, refs, B, Q)
+        if rps is not None and l + 1 < len(dps):
+            ref16, boxes = refine_references(rps[l], t, ref16)
+    return t, ref16
+
+
 def two_stage(tp: dict, memory: np.ndarray, B: int, S: int, K: int):
     """Two-stage query selection (a reading of the two-stage pipeline of Sec. 3.1.2): encoder class logits of every memory token,
     the token's best class logit (top-1 over classes), the K best tokens of each image

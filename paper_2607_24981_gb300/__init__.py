@@ -17,7 +17,7 @@ __all__ = [
     "patch_embed", "patch_embed_workspace_bytes", "Backbone", "Graphed",
     "requant", "resample_nearest", "DecoderWeights", "decoder_workspace_bytes", "decoder_layer_forward",
     "Projector", "Detector", "int_sigmoid", "relu_i8", "topk", "gather_rows", "DetectionHead", "TwoStage",
-    "QueryPos", "ivit_shiftgelu",
+    "QueryPos", "BoxRefine", "ivit_shiftgelu",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -638,11 +638,14 @@ class Detector:
     parameters (``synth.two_stage_params``) the decoder's reference points come from the two-stage
     query selection over the memory, and with positional-query parameters as well
     (``synth.query_pos_params``) so do its positional queries (the learnable projection of the
-    selected boxes); with head parameters (``synth.head_params``) the decoder output is requantised
+    selected boxes); with refinement parameters (``synth.refine_params``) the references are
+    refined after every layer but the last (BoxRefine), and each layer samples at, and projects, the
+    current boxes; with head parameters (``synth.head_params``) the decoder output is requantised
     to int8 and the detection head gives class scores and boxes."""
 
     def __init__(self, pe: dict, blocks: list, taps, pp: dict, dps: list, B: int, Q: int, levels, grid: int = 40,
-                 tsp: dict | None = None, hp: dict | None = None, pq: dict | None = None, device="cuda"):
+                 tsp: dict | None = None, hp: dict | None = None, pq: dict | None = None, rps: list | None = None,
+                 device="cuda"):
         import torch
 
         self.backbone = Backbone(pe, blocks, B, device=device)
@@ -664,6 +667,9 @@ class Detector:
             self.ident = torch.arange(B * Q, dtype=torch.int32, device=device)
             self.refs_buf = torch.empty((B, Q, 2), dtype=torch.int32, device=device)
         self.qp = QueryPos(pq, B * Q, device) if (pq is not None and self.ts is not None) else None
+        if rps is not None and self.ts is None:
+            raise ValueError("Detector: box refinement needs the two-stage references (tsp)")
+        self.refine = [BoxRefine(rp, device) for rp in rps[: len(dps) - 1]] if rps is not None else None
         if self.qp is not None:
             self.pos_buf = torch.empty((B * Q, d), dtype=torch.int16, device=device)
 
@@ -675,19 +681,23 @@ class Detector:
         no two-stage selection."""
         self.backbone.forward(img, taps=dict(zip(self.taps, self.tap_buf)))
         memory = self.proj.forward(self.tap_buf)
+        boxes = None
         if self.ts is not None:
             _, _, ref16, boxes = self.ts.forward(memory, self.B, self.proj.S, self.Q)
-            gather_rows(boxes[:, :2], self.ident, out=self.refs_buf.view(self.B * self.Q, 2))
-            refs = self.refs_buf
-            if self.qp is not None:
-                pos = self.qp.forward(boxes, out=self.pos_buf)
-        if pos is None or refs is None:
-            raise ValueError("Detector.forward: pos and refs are needed unless the two-stage selection "
-                             "(and, for pos, the positional-query projection) provides them")
         x = tgt
         for i, dw in enumerate(self.dec):
+            if boxes is not None:  # this layer's sampling points and positional queries from the current boxes
+                gather_rows(boxes[:, :2], self.ident, out=self.refs_buf.view(self.B * self.Q, 2))
+                refs = self.refs_buf
+                if self.qp is not None:
+                    pos = self.qp.forward(boxes, out=self.pos_buf)
+            if pos is None or refs is None:
+                raise ValueError("Detector.forward: pos and refs are needed unless the two-stage selection "
+                                 "(and, for pos, the positional-query projection) provides them")
             x = decoder_layer_forward(dw, x, pos, memory, self.levels, refs, self.B, self.Q, self.ws,
                                       out=self.t[i % 2])
+            if self.refine is not None and i + 1 < len(self.dec):
+                ref16, boxes = self.refine[i].forward(x, ref16)
         if self.head is None:
             return x
         hp = self.head.hp
@@ -776,6 +786,39 @@ class DetectionHead:
         z = requant(dlt, hp["m_d"], hp["s_d"], ref16, hp["m_ref"], hp["s_ref"], out_bits=32)
         boxes = int_sigmoid(z, {"I0": hp["box_I0"], "k_inter": hp["k_inter"], "k_out": 17})
         return scores, boxes, z
+
+
+class BoxRefine:
+    """The box refinement after a decoder layer (``synth.refine_params``, one per layer): the decoder
+    output requantised to int8, a 3-layer integer MLP (ReLU on the int8 hidden outputs), the deltas
+    requantised to the reference-logit scale and added to the current reference logits (saturated
+    to int16), and the new boxes by the integer sigmoid (scale 2^-16).  Every step is an ilwdetr_*
+    call."""
+
+    def __init__(self, rp: dict, device="cuda"):
+        import numpy as np
+        import torch
+
+        self.rp = rp
+        dv = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)  # noqa: E731
+        self.t = {k: dv(v) for k, v in rp.items() if isinstance(v, np.ndarray)}
+        for k in ("w_b1", "w_b2", "w_b3"):
+            self.t[k + "_p"] = pack_weight(self.t[k])
+
+    def forward(self, x, ref16):
+        """x int16 [M, d] (decoder output), ref16 int16 [M, 4] -> (new ref16 int16 [M, 4], boxes int32 [M, 4])."""
+        rp, t = self.rp, self.t
+        d = x.shape[1]
+        a = requant(x, rp["m_in"], rp["s_in"], out_bits=8)
+        h1 = gemm_requant(a, t["w_b1_p"], d, t["b_b1"], t["m_b1"], t["s_b1"], 8)
+        relu_i8(h1, out=h1)
+        h2 = gemm_requant(h1, t["w_b2_p"], d, t["b_b2"], t["m_b2"], t["s_b2"], 8)
+        relu_i8(h2, out=h2)
+        dlt = gemm_requant(h2, t["w_b3_p"], 4, t["b_b3"], None, None, 32)
+        ref = requant(dlt, rp["m_d"], rp["s_d"], ref16, rp["m_ref"], rp["s_ref"], out_bits=16)
+        ref32 = requant(ref, 1 << 30, 30, out_bits=32)
+        boxes = int_sigmoid(ref32, {"I0": rp["box_I0"], "k_inter": rp["k_inter"], "k_out": 17})
+        return ref, boxes
 
 
 class TwoStage:

@@ -293,6 +293,31 @@ def head_params(seed: int, d: int = 256, C: int = 80, sigma_in: float = 32.0, k_
     return hp
 
 
+def refine_params(seed: int, layers: int, d: int = 256, sigma_in: float = 32.0, k_inter: int = 8) -> list:
+    """Integer parameters of the box refinement between decoder layers (one box branch per layer
+    whose output feeds another layer): the decoder output requantised to int8, a box MLP
+    d -> d -> d -> 4 with ReLU on its int8 hidden outputs, the deltas requantised to the
+    reference-logit scale 2^-10 (std ~256) and added to the current reference logits, the result
+    saturated to int16 and passed through the integer sigmoid (scale 2^-16).  Same recipe as the
+    detection head's box branch, drawn per layer."""
+    out = []
+    acc_std = sigma_in * 73.3 * math.sqrt(d)
+    for l in range(layers):
+        p = f"RB{l}."
+        rp: dict = {"k_inter": k_inter}
+        rp["w_b1"], rp["b_b1"], rp["m_b1"], rp["s_b1"] = gemm_params(seed, p + "b1", d, d, sigma_in, 32.0)
+        rp["w_b2"], rp["b_b2"], rp["m_b2"], rp["s_b2"] = gemm_params(seed, p + "b2", d, d, 16.0, 32.0)
+        rp["w_b3"], rp["b_b3"], _, _ = gemm_params(seed, p + "b3", 4, d, 16.0, 1.0)
+        rp["m_d"] = _mult(seed, p + "d.m")
+        rp["s_d"] = _shift_for(16.0 * 73.3 * math.sqrt(d), 256.0)
+        rp["m_ref"], rp["s_ref"] = 1 << 30, 30
+        rp["box_I0"] = 1024
+        rp["m_in"], rp["s_in"] = _mult(seed, p + "in.m"), _shift_for(2048.0, 32.0)
+        assert acc_std > 0
+        out.append(rp)
+    return out
+
+
 def anchor_logits(levels=((80, 80), (40, 40), (20, 20)), scale: float = 1024.0) -> np.ndarray:
     """Anchor boxes of every memory token as int16 logits at scale 1/`scale`: token (y, x) of
     level l has cx = (x + 0.5) / W_l, cy = (y + 0.5) / H_l, w = h = 0.05 * 2^l; logit(p) =

@@ -123,11 +123,12 @@ def test_detector_full_batch_sampled_image(ilw, orc):
     assert 10 < float(np.abs(out.astype(np.int64)).mean()) < 30000
 
 
-def test_detector_two_stage_and_head_sampled_image(ilw, orc):
+def test_detector_two_stage_refinement_and_head_sampled_image(ilw, orc):
     """The detector with two-stage query selection (the decoder's reference points from the top-300
-    memory tokens, its positional queries by the learnable projection of their boxes) and the
-    detection head (class scores, boxes) at batch 2; the oracle recomputes one image end to end
-    (backbone, projector, two-stage selection, positional queries, three decoder layers, head)."""
+    memory tokens, its positional queries by the learnable projection of their boxes), the reference
+    boxes refined after each decoder layer but the last, and the detection head (class scores,
+    boxes) at batch 2; the oracle recomputes one image end to end (backbone, projector, two-stage
+    selection, three decoder layers with refinement and positional queries, head)."""
     cfg = synth.CONFIGS["detector_c4"]
     bb = synth.CONFIGS[cfg["backbone"]]
     B, Q, g = 2, cfg["Q"], cfg["grid"]
@@ -138,9 +139,10 @@ def test_detector_two_stage_and_head_sampled_image(ilw, orc):
     tsp = synth.two_stage_params(3, d=cfg["N"], C=80, levels=cfg["levels"])
     hp = synth.head_params(3, d=cfg["N"], C=80)
     pq = synth.query_pos_params(3, d=cfg["N"])
+    rps = synth.refine_params(3, cfg["dec_layers"] - 1, d=cfg["N"])
     inp = synth.decoder_inputs(1, B, Q)
     img = synth.image_input(1, B)
-    det = ilw.Detector(pe, blocks, cfg["taps"], pp, dps, B, Q, cfg["levels"], g, tsp=tsp, hp=hp, pq=pq)
+    det = ilw.Detector(pe, blocks, cfg["taps"], pp, dps, B, Q, cfg["levels"], g, tsp=tsp, hp=hp, pq=pq, rps=rps)
     x, scores, boxes = det.forward(dev(img), dev(inp["tgt"]))
     x, scores, boxes = host(x), host(scores), host(boxes)
     ilw.device_status()
@@ -155,15 +157,12 @@ def test_detector_two_stage_and_head_sampled_image(ilw, orc):
     mem = orc.projector(pp, [taps[i] for i in cfg["taps"]], 1, g, cfg["levels"])
     S = mem.shape[0]
     _, _, ref16, bx = orc.two_stage(tsp, mem, 1, S, Q)
-    refs = np.ascontiguousarray(bx[:, :2]).reshape(1, Q, 2)
-    pos = orc.query_pos(pq, bx)
     r = slice(pick * Q, (pick + 1) * Q)
-    t = inp["tgt"][r]
-    for dp in dps:
-        t = orc.decoder_layer(dp, t, pos, mem, cfg["levels"], refs, 1, Q)
+    t, ref_last = orc.decoder_stack(dps, inp["tgt"][r], mem, cfg["levels"], ref16, bx, 1, Q, pq=pq, rps=rps)
     same(x[r], t, f"decoder output image {pick}")
+    assert not np.array_equal(ref_last, ref16)  # the references did move
     a = orc.requant(t, hp["m_in"], hp["s_in"], out_bits=8)
-    ws, wb, _ = orc.detection_head(hp, a, ref16)
+    ws, wb, _ = orc.detection_head(hp, a, ref_last)
     same(scores[r], ws, f"scores image {pick}")
     same(boxes[r], wb, f"boxes image {pick}")
 

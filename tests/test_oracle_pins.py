@@ -872,3 +872,35 @@ def test_detection_scores_rise_with_the_class_logit(orc):
     order = np.argsort(logits.reshape(-1), kind="stable")
     s = scores.reshape(-1)[order].astype(np.int64)
     assert np.all(np.diff(s) >= 0) and s[-1] > s[0]
+
+
+def test_box_refinement_reduces_to_fixed_references(orc):
+    """Box refinement between decoder layers (a reading of the two-stage pipeline's references,
+    Sec. 3.1.2): with the last layer of every refinement MLP zero the deltas vanish, the references
+    are requantised by the identity (m 2^30, s 30) and stay what they were, so the decoder stack
+    equals the one with fixed references; with the drawn weights they move, and the output differs."""
+    Q, levels = 20, ((8, 8), (4, 4), (2, 2))
+    S = sum(h * w for h, w in levels)
+    dps = [synth.decoder_params(0, i) for i in range(3)]
+    rps = synth.refine_params(4, 2)
+    pq = synth.query_pos_params(4)
+    tgt = synth.decoder_inputs(4, 1, Q)["tgt"]
+    mem = synth.laplace_int(4, "rf.mem", (S, 256), 20.0, 127, np.int8)
+    ref16 = synth.uniform_int(4, "rf.ref", (Q, 4), -3000, 3000, np.int16)
+    boxes = orc.int_sigmoid(ref16.astype(np.int32), 1024, 8, 17)
+    fixed, r_fixed = orc.decoder_stack(dps, tgt, mem, levels, ref16, boxes, 1, Q, pq=pq)
+    zero = [dict(rp, w_b3=np.zeros_like(rp["w_b3"]), b_b3=np.zeros_like(rp["b_b3"])) for rp in rps]
+    same, r_same = orc.decoder_stack(dps, tgt, mem, levels, ref16, boxes, 1, Q, pq=pq, rps=zero)
+    assert np.array_equal(same, fixed) and np.array_equal(r_same, r_fixed) and np.array_equal(r_fixed, ref16)
+    moved, r_moved = orc.decoder_stack(dps, tgt, mem, levels, ref16, boxes, 1, Q, pq=pq, rps=rps)
+    assert not np.array_equal(r_moved, ref16) and not np.array_equal(moved, fixed)
+    # one refinement step by hand: the box branch's deltas added to the logits, then the sigmoid
+    ref1, box1 = orc.refine_references(rps[0], fixed, ref16)
+    a = orc.requant(fixed, rps[0]["m_in"], rps[0]["s_in"], out_bits=8).astype(np.int8)
+    h = orc.relu(orc.gemm_requant(a, rps[0]["w_b1"], rps[0]["b_b1"], rps[0]["m_b1"], rps[0]["s_b1"], 8).astype(np.int8))
+    h = orc.relu(orc.gemm_requant(h, rps[0]["w_b2"], rps[0]["b_b2"], rps[0]["m_b2"], rps[0]["s_b2"], 8).astype(np.int8))
+    dl = orc.gemm_requant(h, rps[0]["w_b3"], rps[0]["b_b3"], None, None, 32).astype(np.int64)
+    rqd = (dl * rps[0]["m_d"] + (1 << (rps[0]["s_d"] - 1))) >> rps[0]["s_d"]
+    assert np.array_equal(ref1, np.clip(rqd + ref16, -32767, 32767))
+    assert np.array_equal(box1, orc.int_sigmoid(ref1.astype(np.int32), 1024, 8, 17))
+
