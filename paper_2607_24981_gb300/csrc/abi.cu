@@ -481,6 +481,8 @@ int ilwdetr_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int3
 namespace {
 struct DecBufs {
     int8_t *qk_in, *v_in, *qkv, *o, *qc, *value, *samp, *fin, *h;
+    __half *qkv64;  // heads of dh < 64: q|k|v widened to 64 columns per head (fp16-carried int8)
+    int8_t *o64;    // and the attention output at 64 columns per head
     int16_t *x1, *t1, *off16, *att16, *x2, *t2, *x3;
     int32_t *off32, *att32;
     uint8_t *w;
@@ -500,6 +502,10 @@ DecBufs dec_layout(char *ws, int32_t B, int32_t Q, int64_t S_total, int32_t d, i
     b.v_in = (int8_t *)take(M * d);
     b.qkv = (int8_t *)take(M * 3 * d);
     b.o = (int8_t *)take(M * d);
+    if (d / H < 64) {
+        b.qkv64 = (__half *)take(M * 3 * (size_t)H * 64 * 2);
+        b.o64 = (int8_t *)take(M * (size_t)H * 64);
+    }
     b.x1 = (int16_t *)take(M * d * 2);
     b.t1 = (int16_t *)take(M * d * 2);
     b.qc = (int8_t *)take(M * d);
@@ -558,8 +564,20 @@ int ilwdetr_decoder_layer_forward(const ilw_decoder_params_t *p, const int16_t *
                                  stream));
     ILW_TRY(ilwdetr_gemm_requant(b.v_in, d, p->w_v, p->b_v, p->m_v, p->s_v, M, d, d, 8, b.qkv + 2 * d, 3 * d, nullptr,
                                  stream));
-    ILW_TRY(ilwdetr_shiftmax_attn(b.qkv, b.qkv + d, b.qkv + 2 * d, 3 * d, 8, B, Q, H, d / H, 0, &p->smx, p->m_o, p->s_o,
-                                  b.o, 8, d, stream));
+    if (d / H < 64) {
+        // heads of 32 columns run on the tensor-memory attention of 64-column heads: q|k|v widened with
+        // zero columns (nothing added to q.k, zero outputs), the output narrowed back
+        const int64_t w = (int64_t)H * 64;
+        cudaError_t e = ilw::launch_head_pad64(b.qkv, 3 * d, M, 3 * H, d / H, b.qkv64, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_status(e, "decoder head pad");
+        ILW_TRY(ilwdetr_shiftmax_attn(b.qkv64, b.qkv64 + w, b.qkv64 + 2 * w, 3 * w, ILW_I8_IN_F16, B, Q, H, 64, 0, &p->smx,
+                                      p->m_o, p->s_o, b.o64, 8, w, stream));
+        e = ilw::launch_head_compact(b.o64, w, M, H, d / H, b.o, d, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_status(e, "decoder head compact");
+    } else {
+        ILW_TRY(ilwdetr_shiftmax_attn(b.qkv, b.qkv + d, b.qkv + 2 * d, 3 * d, 8, B, Q, H, d / H, 0, &p->smx, p->m_o,
+                                      p->s_o, b.o, 8, d, stream));
+    }
     ilw_residual_t r1{tgt, d, M, p->m_r1, p->s_r1};
     ILW_TRY(ilwdetr_gemm_requant(b.o, d, p->w_o, p->b_o, p->m_oc, p->s_oc, M, d, d, 16, b.x1, d, &r1, stream));
     ILW_TRY(ilwdetr_int_layernorm(b.x1, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, b.t1, 16, d,

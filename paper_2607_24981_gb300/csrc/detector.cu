@@ -72,6 +72,43 @@ __global__ void __launch_bounds__(256) resample_kernel(const int8_t *__restrict_
     }
 }
 
+// Heads of dh < 64 columns widened to 64: Y[m, (p H + h) 64 + c] = X[m, (p H + h) dh + c] for c < dh,
+// 0 above (the int8 values carried in fp16), for nparts consecutive groups of H heads.  Eight
+// outputs (16 bytes) per item.
+__global__ void head_pad64_kernel(const int8_t *__restrict__ X, int64_t ldx, int64_t M, int32_t nh, int32_t dh,
+                                  __half *__restrict__ Y) {
+    const int64_t per_row = (int64_t)nh * 8;  // 16-byte chunks of a padded row
+    const int64_t items = M * per_row;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < items; i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t m = i / per_row;
+        const int32_t j = (int32_t)(i - m * per_row), head = j >> 3, c0 = (j & 7) * 8;
+        uint32_t w[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int c = c0 + 2 * u;
+            const int8_t *x = X + m * ldx + (int64_t)head * dh + c;
+            const int32_t a = c < dh ? (int32_t)x[0] : 0, b = c + 1 < dh ? (int32_t)x[1] : 0;
+            // |v| <= 127: 1152 + v has the fp16 bits 0x6480 + v; subtracting 1152 leaves v
+            uint32_t hb = (uint32_t)(0x6480 + a) | ((uint32_t)(0x6480 + b) << 16);
+            const __half2 hh = __hsub2(*reinterpret_cast<__half2 *>(&hb), __half2half2(__ushort_as_half((unsigned short)0x6480)));
+            w[u] = *reinterpret_cast<const uint32_t *>(&hh);
+        }
+        *(uint4 *)(Y + m * (per_row * 8) + (int64_t)j * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+// The inverse for int8 rows: O[m, h dh + c] = Y[m, h 64 + c] for c < dh.
+__global__ void head_compact_kernel(const int8_t *__restrict__ Y, int64_t ldy, int64_t M, int32_t H, int32_t dh,
+                                    int8_t *__restrict__ O, int64_t ldo) {
+    const int64_t per_row = (int64_t)H * dh;
+    const int64_t items = M * per_row;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < items; i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t m = i / per_row;
+        const int32_t j = (int32_t)(i - m * per_row), head = j / dh, c = j - head * dh;
+        O[m * ldo + j] = Y[m * ldy + (int64_t)head * 64 + c];
+    }
+}
+
 unsigned grid_for(int64_t items) {
     int64_t g = (items + 255) / 256;
     const int64_t cap = (int64_t)sm_count() * 16;  // grid-stride loops: 16 CTAs of 256 threads per SM
@@ -93,6 +130,19 @@ cudaError_t launch_requant(const RequantParams &p, cudaStream_t s) {
         else if (p.out_bits == 16) requant_kernel<int32_t, int16_t><<<g, 256, 0, s>>>(p);
         else requant_kernel<int32_t, int32_t><<<g, 256, 0, s>>>(p);
     }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_head_pad64(const int8_t *X, int64_t ldx, int64_t M, int32_t nh, int32_t dh, __half *Y,
+                              cudaStream_t s) {
+    if (M == 0 || nh == 0) return cudaSuccess;
+    head_pad64_kernel<<<grid_for(M * nh * 8), 256, 0, s>>>(X, ldx, M, nh, dh, Y);
+    return cudaGetLastError();
+}
+cudaError_t launch_head_compact(const int8_t *Y, int64_t ldy, int64_t M, int32_t H, int32_t dh, int8_t *O, int64_t ldo,
+                                cudaStream_t s) {
+    if (M == 0 || H == 0) return cudaSuccess;
+    head_compact_kernel<<<grid_for(M * H * dh), 256, 0, s>>>(Y, ldy, M, H, dh, O, ldo);
     return cudaGetLastError();
 }
 

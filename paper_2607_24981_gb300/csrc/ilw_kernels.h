@@ -179,5 +179,12 @@ struct RequantParams {
 cudaError_t launch_requant(const RequantParams &p, cudaStream_t s);
 cudaError_t launch_resample(const int8_t *X, int64_t x_bstride, int32_t B, int32_t Hi, int32_t Wi, int32_t C,
                             int8_t *Y, int64_t y_bstride, int32_t Ho, int32_t Wo, cudaStream_t s);
+// Attention heads of dh < 64 widened to 64 columns for the tensor-memory attention (zero columns
+// add nothing to q.k and give zero outputs): nh heads of int8 rows -> fp16-carried [M, nh 64]; and
+// the int8 outputs narrowed back to dh columns per head.
+cudaError_t launch_head_pad64(const int8_t *X, int64_t ldx, int64_t M, int32_t nh, int32_t dh, __half *Y,
+                              cudaStream_t s);
+cudaError_t launch_head_compact(const int8_t *Y, int64_t ldy, int64_t M, int32_t H, int32_t dh, int8_t *O, int64_t ldo,
+                                cudaStream_t s);
 
 }  // namespace ilw
