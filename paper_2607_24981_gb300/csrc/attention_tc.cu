@@ -326,8 +326,8 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
     const uint32_t tmem = *tmem_slot;  // columns: S[b] TKB b .. TKB b + TKB - 1, O TKB NS .. TKB NS + 63
     constexpr uint32_t kOcol = (uint32_t)(TKB * NS);
 
-    // Piece sequence: pieces 0 .. 2 nkb - 1 are the k blocks of passes 1 and 2; in pass 3 key block
-    // kb has the k piece 2 nkb + 2 kb and the v piece 2 nkb + 2 kb + 1.
+    // Piece sequence: pieces 0 .. 2 nkb - 1 are the k blocks of passes 1 and 2; pass 3 streams
+    // k0, k1, v0, k2, v1, ..., k(nkb - 1), v(nkb - 2), v(nkb - 1), the order in which the MMA uses them.
     if (warp == 0) {
         // ------------------------------------------------------------------ MMA issuer
         if (lane == 0) {
@@ -338,10 +338,10 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             const uint64_t dq = desc_sw128(sbase + TcSmem::kQ), dring = desc_sw128(sbase + TcSmem::kRing),
                            dp = desc_sw128(sbase + TcSmem::kP), daa = desc_sw32(sbase + TcSmem::kAugA),
                            dab = desc_sw32(sbase + TcSmem::kAugB);
-            // consumption state: the S buffer, the ring slot of the next k piece (and, in pass 3, of the
-            // next v piece) and the P buffer, each with its phase bit
-            int sb = 0, ks = 0, vs = 0, pb = 0;
-            uint32_t sph = 0, kph = 0, vph = 0, pph = 0;
+            // consumption state: the S buffer, the ring slot of the next piece and the P buffer, each
+            // with its phase bit
+            int sb = 0, ks = 0, pb = 0;
+            uint32_t sph = 0, kph = 0, pph = 0;
             auto adv = [](int &slot, uint32_t &ph, int by) {
                 slot += by;
                 while (slot >= NP) {
@@ -373,17 +373,17 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             // O += P V for the next key block of pass 3 (TKB / 16 steps; P sub-tile t / 4 holds keys
             // 64 (t / 4) ..); releases P[pb] and the v piece
             auto issue_pv = [&](bool first) -> bool {
-                if (!bar_wait(full(vs), vph, abort, p.status, kStatusTimeoutTma)) return false;
+                if (!bar_wait(full(ks), kph, abort, p.status, kStatusTimeoutTma)) return false;
                 if (!bar_wait(p_full(pb), pph, abort, p.status, kStatusTimeoutOperand)) return false;
                 fence_after();
-                const uint64_t da = dp + (uint64_t)(pb * (kPB / 16)), dv = dring + (uint64_t)(vs * (kSlotB / 16));
+                const uint64_t da = dp + (uint64_t)(pb * (kPB / 16)), dv = dring + (uint64_t)(ks * (kSlotB / 16));
 #pragma unroll
                 for (int t = 0; t < TKB / 16; ++t)
                     mma(tmem + kOcol, da + (uint64_t)((t >> 2) * (TQ * 128 / 16) + 2 * (t & 3)), dv + (uint64_t)(128 * t),
                         id_o, (first && t == 0) ? 0u : 1u);
                 commit(p_free(pb));
-                commit(empty(vs));
-                adv(vs, vph, 2);
+                commit(empty(ks));
+                adv(ks, kph, 1);
                 if (++pb == NPB) {
                     pb = 0;
                     pph ^= 1u;
@@ -398,15 +398,15 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 if (ok) ok = issue_s(j >= nkb);
                 adv(ks, kph, 1);
             }
-            // pass 3: k piece of block kb, then its v piece; the P V of block kb is issued after the
-            // scores of block kb + 1, so the softmax warps always have the next scores waiting
-            vs = ks;
-            vph = kph;
-            adv(vs, vph, 1);
-            for (int kb = 0; kb < nkb && ok; ++kb) {
+            // pass 3: the scores of block kb + 1 are issued before the P V of block kb, so the softmax
+            // warps always have the next scores waiting; the loaders stream the pieces in exactly this
+            // order (k0, k1, v0, k2, v1, ..., v(n-1)), so a slot is refilled as soon as it is consumed
+            if (ok) ok = issue_s(true);
+            adv(ks, kph, 1);
+            for (int kb = 0; kb + 1 < nkb && ok; ++kb) {
                 ok = issue_s(true);
-                adv(ks, kph, 2);
-                if (ok && kb > 0) ok = issue_pv(kb == 1);
+                adv(ks, kph, 1);
+                if (ok) ok = issue_pv(kb == 0);
             }
             if (ok) ok = issue_pv(nkb == 1);
             if (ok) commit(o_full);
@@ -433,14 +433,27 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         fence_async_smem();
         bar_arrive(bq_full);
         if (tl == 0) {
-            // the key-block stream: piece i into slot i % NP once the piece before it there is consumed
+            // the key-block stream: piece i into slot i % NP once the piece before it there is consumed.
+            // Pieces 0 .. 2 nkb - 1 are the k blocks of passes 1 and 2; pass 3 follows the MMA's order:
+            // k0, then k(j + 1), v(j) for j = 0 .. nkb - 2, then v(nkb - 1)
             const uint32_t bytes = (uint32_t)kbk * 128u;
             const int bimg = gr.base / p.T, npiece = 4 * nkb;
-            int issued = 0, slot = 0, kb = 0;
+            int issued = 0, slot = 0;
             uint32_t ph = 0;
             for (int i = 0; i < npiece; ++i) {
                 if (!bar_wait(empty(slot), ph ^ 1u, abort, p.status, kStatusTimeoutFree)) break;
-                const CUtensorMap *m = (i >= 2 * nkb && ((i - 2 * nkb) & 1)) ? &args.vmap : &args.kmap;
+                bool isv = false;
+                int kb;
+                if (i < 2 * nkb) {
+                    kb = i < nkb ? i : i - nkb;
+                } else {
+                    const int j = i - 2 * nkb;
+                    if (j == 0) kb = 0;
+                    else if (j == 2 * nkb - 1) { kb = nkb - 1; isv = true; }
+                    else if (j & 1) kb = (j + 1) >> 1;
+                    else { kb = (j - 2) >> 1; isv = true; }
+                }
+                const CUtensorMap *m = isv ? &args.vmap : &args.kmap;
                 const uint32_t dst = sbase + TcSmem::kRing + slot * kSlotB;
                 bar_expect_tx(full(slot), bytes);
                 if (args.win)
@@ -452,10 +465,6 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     slot = 0;
                     ph ^= 1u;
                 }
-                // next piece's key block: k blocks 0 .. nkb - 1 twice, then k, v of each block
-                if (i < 2 * nkb - 1) kb = kb + 1 == nkb ? 0 : kb + 1;
-                else if (i == 2 * nkb - 1) kb = 0;
-                else if ((i - 2 * nkb) & 1) ++kb;
             }
             // after an abort, the pieces still in flight land before the CTA exits
             if (*abort)
@@ -529,10 +538,9 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 ok = __all_sync(0xffffffffu, bar_wait(s_full(b), sph, abort, p.status, kStatusTimeoutMma));
                 if (!ok) break;
                 fence_after();
-                if (pass == 2) {  // the P V that read the P buffer before has completed
-                    ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
-                    if (!ok) break;
-                }
+                // pass 3 writes P into the buffer the previous block's P V reads: that MMA must have
+                // completed, which is waited for just before the first store, after the arithmetic
+                bool p_ready = pass != 2;
                 const int kvalid = min(kbk, Tg - kb * kbk);
 #pragma unroll 1
                 for (int h = 0; h < NCH; ++h) {
@@ -551,6 +559,11 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     }
                     if (!work) {
                         if (pass == 2 && live) {
+                            if (!p_ready) {
+                                p_ready = true;
+                                ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
+                                if (!ok) break;
+                            }
                             uint8_t *prow = sm + TcSmem::kP + pb * kPB + (c0 >> 6) * (TQ * 128) + row * 128;
                             const int k0 = (c0 & 63) >> 3;
 #pragma unroll
@@ -605,6 +618,11 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                             __half2 hh = __hsub2(*reinterpret_cast<__half2 *>(&x), h1024);
                             w[c] = *reinterpret_cast<uint32_t *>(&hh);
                         }
+                        if (!p_ready) {
+                            p_ready = true;
+                            ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
+                            if (!ok) break;
+                        }
                         // keys c0 .. c0 + 31 sit in sub-tile c0 / 64, chunks (c0 % 64) / 8 .. + 3 of the row;
                         // 16-byte chunk k of a row sits at k ^ (row & 7)
                         uint8_t *prow = sm + TcSmem::kP + pb * kPB + (c0 >> 6) * (TQ * 128) + row * 128;
@@ -620,6 +638,13 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     sph ^= 1u;
                 }
                 if (pass == 2) {
+                    // every warp (also one that stored nothing) arrives for this block only after the
+                    // previous block's P V completed, so arrivals never run a phase ahead
+                    if (!p_ready) {
+                        p_ready = true;
+                        ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
+                        if (!ok) break;
+                    }
                     fence_async_smem();
                     __syncwarp();
                     if (lane == 0) bar_arrive(p_full(pb));
