@@ -10,25 +10,32 @@
 //
 // One CTA = 128 queries of one (image, head, group), 12 warps, two CTAs per SM:
 //   warp 0      TMEM allocation; MMA issuer (one thread): per key block of 128, 4 MMAs
-//               128 x 128 x 16 into the score buffer, and in pass 3 8 MMAs O += P V (P from shared
-//               memory in two 64-key sub-tiles, v as an N-major operand, exactly the rows it was
-//               loaded with), issued after the scores of the next block.  The cost of one MMA barely
-//               depends on N here, so 128-key blocks halve the MMA time of 64-key blocks
+//               128 x 128 x 16 into a score buffer (passes 2 and 3: plus one K = 16 MMA that adds
+//               each row's constant term), and in pass 3 8 MMAs O += P V (P from shared memory in
+//               two 64-key sub-tiles, v as an N-major operand, exactly the rows it was loaded with),
+//               issued after the scores of the next block.  Passes 1 and 2 alternate between two
+//               score buffers; pass 3 has one, O taking the second one's columns
 //   warps 1-3   the CTA's 128 q rows once (cp.async, in the tensor cores' 128-byte swizzled
-//               layout); then one thread of warp 1 streams the key blocks as TMA pieces (k blocks
-//               in passes 1 and 2; k and v blocks in pass 3) into a 3-slot ring.  A key block is 128
-//               consecutive tokens (global attention: a 2-D box of the q|k|v matrix) or R whole
-//               rows of a ws x ws window, R = min(floor(128 / ws), ws) (a 3-D box over (channel,
-//               x, y)); the slot rows a window block leaves unwritten stay zero
+//               layout); then one thread of warp 1 streams the key blocks as TMA pieces into a
+//               3-slot ring, in the order the MMA consumes them (k blocks in passes 1 and 2; then
+//               k0, k1, v0, k2, v1, ...).  A key block is 128 consecutive tokens (global attention:
+//               a 2-D box of the q|k|v matrix) or R whole rows of a ws x ws window,
+//               R = min(floor(128 / ws), ws) (a 3-D box over (channel, x, y)); the slot rows a window
+//               block leaves unwritten stay zero
 //   warps 4-11  softmax: warp 4 + w reads TMEM lanes 32 (w % 4) .. + 31 (one query row per
 //               thread) and score columns 64 (w / 4) .. + 63 of each block (two 32-column loads);
 //               the two halves of a row combine their max and sum once per pass through shared
-//               memory; P rows go to shared memory as fp16 operands.  The score buffer is released
+//               memory; P rows go to shared memory as fp16 operands (P < 1024 written as its own
+//               bits, the subnormal P 2^-24; O is scaled back by 2^24).  A score buffer is released
 //               as soon as the last load of a block has landed, so the next block's MMAs run
 //               while the softmax works.  Warps whose rows all lie past the group, and 32-key
 //               loads past its keys, skip the arithmetic (their P is written as zero)
 // The CTAs holding the last (possibly partial, hence shorter) query tile of each group come after
-// all the others, so they fill the last wave.
+// all the others, so they fill the last wave.  Global attention whose last tile has at most 64
+// queries puts the last tiles of two (image, head) units in one CTA (rows 0-63 and 64-127): a key
+// block is then 64 keys of each unit (two N = 64 score MMAs, each unit's rows reading their own
+// half of the columns), and each unit has its own O.  At 1600 tokens this turns 8 x 6 x 13 = 624
+// CTAs (2.05 waves of two per SM) into 600 (two waves).
 // Every mbarrier wait is bounded (about one second); on expiry the kernel latches the device status
 // word, every role stops, the loaders drain their copies and the TMEM is freed after every MMA
 // issued has completed.
@@ -45,16 +52,20 @@ namespace {
 constexpr int TQ = 128;      // queries per CTA
 constexpr int TKB = 128;     // keys per block (global attention)
 constexpr int NP = 3;        // ring slots of TKB x 128 bytes (one k or v block)
-constexpr int NS = 1;        // score buffers (TMEM, TKB columns each); O follows them
+// score buffers (TMEM, TKB columns each): two in passes 1 and 2, when O is not yet accumulated and
+// the second buffer takes its columns; one in pass 3, with O in the columns after it
+constexpr int NS = 2;
 constexpr int NPB = 1;       // P buffers (shared memory, TQ x TKB fp16)
 constexpr int NCQ = 2;       // softmax warps per TMEM lane quarter, each on CPW columns of a block
 constexpr int CPW = TKB / NCQ;
-constexpr int NCH = CPW / 32;  // 32-column TMEM loads per block and thread
+constexpr int CW = 32;          // columns per TMEM load (one softmax chunk)
+constexpr int NCH = CPW / CW;   // chunks per block and thread
 constexpr int OPW = 64 / NCQ;  // output columns per softmax thread
 constexpr int kSlotB = TKB * 128;
 constexpr int kPB = TQ * TKB * 2;  // bytes of one P buffer: TKB / 64 sub-tiles of 128 rows x 128 bytes
-constexpr int kTmemCols = NS * TKB + 64 <= 256 ? 256 : 512;
-constexpr int kMinBlocks = kTmemCols == 256 ? 2 : 1;
+constexpr int kTmemCols = 256;  // S[0] | S[1] or O (64 columns; paired tiles: 128)
+constexpr int kMinBlocks = 2;
+static_assert(NS * TKB <= kTmemCols && TKB + 128 <= kTmemCols, "TMEM columns");
 constexpr int NLOAD = 96;        // q loader threads (warps 1-3)
 constexpr int NSMX = 128 * NCQ;  // softmax threads (warps 4 ..)
 constexpr int kThreadsTc = 128 + NSMX;
@@ -200,12 +211,14 @@ __device__ __forceinline__ void tma_3d(uint32_t dst, const CUtensorMap *m, int32
 
 // Kernel arguments: the attention problem and the tensor maps of its k and v columns.
 struct TcArgs {
-    CUtensorMap kmap, vmap;  // 2-D {64 H, B T} (global) or 3-D {64 H, gs, B gs} (windows), 128-byte swizzle
+    CUtensorMap kmap, vmap;      // 2-D {64 H, B T} (global) or 3-D {64 H, gs, B gs} (windows), 128-byte swizzle
+    CUtensorMap kmap64, vmap64;  // global, paired last tiles: the same with 64-row boxes
     AttnParams p;
-    int32_t kbk;   // keys per block: 64 (global) or R ws (windows)
+    int32_t kbk;   // keys per block: 128 (global) or R ws (windows)
     int32_t rpb;   // window rows per block R (windows)
     int32_t win;   // 1: 3-D window boxes
     int32_t nq;    // query tiles per group
+    int32_t pair;  // 1: the last tiles (<= 64 queries each) of two (image, head) units share a CTA
 };
 __device__ __forceinline__ uint32_t shr_clamp(uint32_t v, uint32_t n) {
     uint32_t r;
@@ -262,17 +275,29 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // CTA -> (query tile, head, group): the tiles of every group but its last come first, the last
     // (possibly partial, hence shorter) tiles of all groups at the end, so they fill the last wave
-    int qt, head, z;
+    // (pair: the CTA holds the last tiles of units 2 j and 2 j + 1, unit = (image, head), rows
+    // 0-63 for the first and 64-127 for the second; a key block is then 64 keys of each unit)
+    int qt, head, z, head1 = 0, z1 = 0;
+    bool pair = false, has1 = false;
     {
         const int Z = p.B * p.nw * p.nw, L = blockIdx.x, F = (args.nq - 1) * p.H * Z;
         if (L < F) {
             qt = L % (args.nq - 1);
             head = (L / (args.nq - 1)) % p.H;
             z = L / ((args.nq - 1) * p.H);
-        } else {
+        } else if (!args.pair) {
             qt = args.nq - 1;
             head = (L - F) % p.H;
             z = (L - F) / p.H;
+        } else {
+            const int u0 = 2 * (L - F), u1 = u0 + 1;
+            pair = true;
+            qt = args.nq - 1;
+            head = u0 % p.H;
+            z = u0 / p.H;
+            has1 = u1 < p.H * Z;
+            head1 = has1 ? u1 % p.H : head;
+            z1 = has1 ? u1 / p.H : z;
         }
     }
     GroupTc gr;
@@ -286,8 +311,11 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         gr.wx = w % p.nw;
         gr.Tg = p.nw > 1 ? gr.ws * gr.ws : p.T;
     }
-    const int Tg = gr.Tg, q0 = qt * TQ, hoff = head * 64, kbk = args.kbk;
+    const int Tg = gr.Tg, q0 = qt * TQ, hoff = head * 64, kbk = pair ? 64 : args.kbk;
     const int nkb = (Tg + kbk - 1) / kbk;
+    // pair: the second unit's first token (global attention: image z1) and head offset
+    const int64_t base1 = (int64_t)z1 * p.T;
+    const int hoff1 = head1 * 64;
 
     if (threadIdx.x == 0) {
         bar_init(bq_full, NLOAD);
@@ -323,8 +351,8 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
     fence_before();
     __syncthreads();
     fence_after();
-    const uint32_t tmem = *tmem_slot;  // columns: S[b] TKB b .. TKB b + TKB - 1, O TKB NS .. TKB NS + 63
-    constexpr uint32_t kOcol = (uint32_t)(TKB * NS);
+    const uint32_t tmem = *tmem_slot;  // columns: S[b] at TKB b; O at TKB (pass 3)
+    constexpr uint32_t kOcol = (uint32_t)TKB;  // O shares its columns with S[1], used before pass 3 only
 
     // Piece sequence: pieces 0 .. 2 nkb - 1 are the k blocks of passes 1 and 2; pass 3 streams
     // k0, k1, v0, k2, v1, ..., k(nkb - 1), v(nkb - 2), v(nkb - 1), the order in which the MMA uses them.
@@ -333,6 +361,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         if (lane == 0) {
             // D f32, A/B f16, both K-major, M = 128, N = TKB (scores) or 64 (O, B = v N-major)
             const uint32_t id_s = (1u << 4) | ((uint32_t)(TKB >> 3) << 17) | ((128u >> 4) << 24);
+            const uint32_t id_s64 = (1u << 4) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
             const uint32_t id_o = (1u << 4) | (1u << 16) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
             // descriptors: an address step of 16 bytes is 1 in the low word (addresses < 256 KB, no carry)
             const uint64_t dq = desc_sw128(sbase + TcSmem::kQ), dring = desc_sw128(sbase + TcSmem::kRing),
@@ -350,21 +379,33 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 }
             };
             // scores of the next key block into S[sb] (aug: plus the constant term -(2^23 + max + 1) of
-            // each row, passes 2 and 3); the k piece is released when they complete
-            auto issue_s = [&](bool aug) -> bool {
+            // each row, passes 2 and 3); the k piece is released when they complete.  Passes 1 and 2
+            // alternate between the two buffers (ring), pass 3 uses S[0] alone
+            auto issue_s = [&](bool aug, bool ring) -> bool {
                 if (!bar_wait(full(ks), kph, abort, p.status, kStatusTimeoutTma)) return false;
                 if (!bar_wait(s_free(sb), sph ^ 1u, abort, p.status, kStatusTimeoutOperand)) return false;
                 fence_after();
                 const uint64_t dk = dring + (uint64_t)(ks * (kSlotB / 16));
                 const uint32_t dt = tmem + (uint32_t)(TKB * sb);
-                mma(dt, dq, dk, id_s, 0u);
-                mma(dt, dq + 2, dk + 2, id_s, 1u);
-                mma(dt, dq + 4, dk + 4, id_s, 1u);
-                mma(dt, dq + 6, dk + 6, id_s, 1u);
+                if (!pair) {
+                    mma(dt, dq, dk, id_s, 0u);
+                    mma(dt, dq + 2, dk + 2, id_s, 1u);
+                    mma(dt, dq + 4, dk + 4, id_s, 1u);
+                    mma(dt, dq + 6, dk + 6, id_s, 1u);
+                } else {
+                    // columns 0-63: every q row against the first unit's 64 keys (slot rows 0-63),
+                    // columns 64-127: against the second unit's (slot rows 64-127, 8 KB on)
+#pragma unroll
+                    for (int u = 0; u < 2; ++u)
+#pragma unroll
+                        for (int t = 0; t < 4; ++t)
+                            mma(dt + 64u * u, dq + 2 * t, dk + (uint64_t)(u * 512 + 2 * t), id_s64, t ? 1u : 0u);
+                }
                 if (aug) mma(dt, daa, dab, id_s, 1u);
                 commit(s_full(sb));
                 commit(empty(ks));
-                if (++sb == NS) {
+                if (!ring) sph ^= 1u;
+                else if (++sb == NS) {
                     sb = 0;
                     sph ^= 1u;
                 }
@@ -377,10 +418,21 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 if (!bar_wait(p_full(pb), pph, abort, p.status, kStatusTimeoutOperand)) return false;
                 fence_after();
                 const uint64_t da = dp + (uint64_t)(pb * (kPB / 16)), dv = dring + (uint64_t)(ks * (kSlotB / 16));
+                if (!pair) {
 #pragma unroll
-                for (int t = 0; t < TKB / 16; ++t)
-                    mma(tmem + kOcol, da + (uint64_t)((t >> 2) * (TQ * 128 / 16) + 2 * (t & 3)), dv + (uint64_t)(128 * t),
-                        id_o, (first && t == 0) ? 0u : 1u);
+                    for (int t = 0; t < TKB / 16; ++t)
+                        mma(tmem + kOcol, da + (uint64_t)((t >> 2) * (TQ * 128 / 16) + 2 * (t & 3)), dv + (uint64_t)(128 * t),
+                            id_o, (first && t == 0) ? 0u : 1u);
+                } else {
+                    // P holds 64 keys per row (sub-tile 0); O of unit u (TMEM columns kOcol + 64 u) takes
+                    // the P rows against that unit's v rows; only its own q rows are read back
+#pragma unroll
+                    for (int u = 0; u < 2; ++u)
+#pragma unroll
+                        for (int t = 0; t < 4; ++t)
+                            mma(tmem + kOcol + 64u * u, da + (uint64_t)(2 * t), dv + (uint64_t)(u * 512 + 128 * t), id_o,
+                                (first && t == 0) ? 0u : 1u);
+                }
                 commit(p_free(pb));
                 commit(empty(ks));
                 adv(ks, kph, 1);
@@ -395,16 +447,17 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             // passes 1 and 2: the k pieces in order; pass 2 waits for the rows' constant terms
             for (int j = 0; j < 2 * nkb && ok; ++j) {
                 if (j == nkb) ok = bar_wait(aug_full, 0, abort, p.status, kStatusTimeoutOperand);
-                if (ok) ok = issue_s(j >= nkb);
+                if (ok) ok = issue_s(j >= nkb, true);
                 adv(ks, kph, 1);
             }
             // pass 3: the scores of block kb + 1 are issued before the P V of block kb, so the softmax
             // warps always have the next scores waiting; the loaders stream the pieces in exactly this
             // order (k0, k1, v0, k2, v1, ..., v(n-1)), so a slot is refilled as soon as it is consumed
-            if (ok) ok = issue_s(true);
+            // (after 2 nkb blocks the ring is back at S[0], whose phase bit sph now holds)
+            if (ok) ok = issue_s(true, false);
             adv(ks, kph, 1);
             for (int kb = 0; kb + 1 < nkb && ok; ++kb) {
-                ok = issue_s(true);
+                ok = issue_s(true, false);
                 adv(ks, kph, 1);
                 if (ok) ok = issue_pv(kb == 0);
             }
@@ -423,10 +476,11 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         const __half *Qg = (const __half *)p.Q;
         // one 16-byte chunk c of a 128-byte row r per item, swizzled: chunk c of row r at c ^ (r & 7)
         for (int it = tl; it < TQ * 8; it += NLOAD) {
-            const int r = it >> 3, c = it & 7, tok = q0 + r;
-            const bool okr = tok < Tg;
-            cpa16(sbase + TcSmem::kQ + r * 128 + ((c ^ (r & 7)) << 4),
-                  Qg + (okr ? gr.token(tok) * ld : 0) + hoff + 8 * c, okr ? 16u : 0u);
+            const int r = it >> 3, c = it & 7, u = pair ? r >> 6 : 0, tok = q0 + (pair ? r & 63 : r);
+            const bool okr = tok < Tg && (u == 0 || has1);
+            const int64_t t = !okr ? 0 : u ? base1 + tok : gr.token(tok);
+            cpa16(sbase + TcSmem::kQ + r * 128 + ((c ^ (r & 7)) << 4), Qg + t * ld + (u ? hoff1 : hoff) + 8 * c,
+                  okr ? 16u : 0u);
         }
         cpa_commit();
         asm volatile("cp.async.wait_all;" ::: "memory");
@@ -436,7 +490,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             // the key-block stream: piece i into slot i % NP once the piece before it there is consumed.
             // Pieces 0 .. 2 nkb - 1 are the k blocks of passes 1 and 2; pass 3 follows the MMA's order:
             // k0, then k(j + 1), v(j) for j = 0 .. nkb - 2, then v(nkb - 1)
-            const uint32_t bytes = (uint32_t)kbk * 128u;
+            const uint32_t bytes = pair ? 2u * 64u * 128u : (uint32_t)kbk * 128u;
             const int bimg = gr.base / p.T, npiece = 4 * nkb;
             int issued = 0, slot = 0;
             uint32_t ph = 0;
@@ -456,7 +510,13 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 const CUtensorMap *m = isv ? &args.vmap : &args.kmap;
                 const uint32_t dst = sbase + TcSmem::kRing + slot * kSlotB;
                 bar_expect_tx(full(slot), bytes);
-                if (args.win)
+                if (pair) {
+                    // 64 keys of each unit: rows 0-63 and 64-127 of the slot (the second unit's rows
+                    // repeat the first's when there is none; nothing reads them then)
+                    const CUtensorMap *m64 = isv ? &args.vmap64 : &args.kmap64;
+                    tma_2d(dst, m64, hoff, (int32_t)(gr.base + kb * 64), full(slot));
+                    tma_2d(dst + 8192u, m64, has1 ? hoff1 : hoff, (int32_t)((has1 ? base1 : gr.base) + kb * 64), full(slot));
+                } else if (args.win)
                     tma_3d(dst, m, hoff, gr.wx * gr.ws, bimg * gr.gs + gr.wy * gr.ws + kb * args.rpb, full(slot));
                 else
                     tma_2d(dst, m, hoff, bimg * p.T + kb * TKB, full(slot));
@@ -476,8 +536,11 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         }
     } else {
         // ------------------------------------------------------------------ softmax, one row per thread
-        const int qw = warp & 3, cq = (warp - 4) >> 2, row = 32 * qw + lane, tok = q0 + row;
-        const bool live = q0 + 32 * qw < Tg;  // some row of this warp is a query of the group
+        // pair: rows 64-127 are the second unit's, row & 63 the query's place in its unit's tile
+        const int qw = warp & 3, cq = (warp - 4) >> 2, row = 32 * qw + lane, unit = pair ? qw >> 1 : 0;
+        const int urow = pair ? row & 63 : row, tok = q0 + urow;
+        // some row of this warp is a query of the group
+        const bool live = q0 + (urow & ~31) < Tg && (unit == 0 || has1);
         const uint32_t tlane = tmem + ((uint32_t)(32 * qw) << 16);
         float *red_max = (float *)(sm + TcSmem::kRedMax);
         uint64_t *red_sum = (uint64_t *)(sm + TcSmem::kRedSum);
@@ -495,7 +558,6 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         };
         int b = 0, pb = 0;  // S and P buffers of the next block, with their phase bits
         uint32_t sph = 0, pph = 0;
-        const __half2 h1024 = __half2half2(__ushort_as_half((unsigned short)0x6400));
         for (int pass = 0; pass < 3 && ok; ++pass) {
             if (pass == 1) {
                 red_max[cq * TQ + row] = mx;
@@ -509,11 +571,11 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     // Both 16-byte halves of the row hold the same terms and the key rows carry their
                     // weights in one half only, so the product does not depend on which half the
                     // swizzle puts where.  Rows past the group get zeros.
-                    const int m1 = tok < Tg ? __float2int_rn(mx) + 1 : 0;
+                    const int m1 = live && tok < Tg ? __float2int_rn(mx) + 1 : 0;
                     const int a3 = m1 >> 11, a0 = m1 - (a3 << 11);
                     const uint32_t h0 = (uint32_t)__half_as_ushort(__int2half_rn(-a0)),
                                    h3 = (uint32_t)__half_as_ushort(__int2half_rn(-a3));
-                    const uint32_t n2048 = tok < Tg ? 0xE800u : 0u;  // -2048
+                    const uint32_t n2048 = live && tok < Tg ? 0xE800u : 0u;  // -2048
                     const uint4 ra = make_uint4(h0 | (n2048 << 16), n2048 | (h3 << 16), 0u, 0u);
                     *(uint4 *)(sm + TcSmem::kAugA + row * 32) = ra;
                     *(uint4 *)(sm + TcSmem::kAugA + row * 32 + 16) = ra;
@@ -542,17 +604,20 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 // completed, which is waited for just before the first store, after the arithmetic
                 bool p_ready = pass != 2;
                 const int kvalid = min(kbk, Tg - kb * kbk);
+                // pair: 32 columns per block, from the unit's half of the score columns
+                const int nch = pair ? 32 / CW : NCH;
 #pragma unroll 1
-                for (int h = 0; h < NCH; ++h) {
-                    const int c0 = CPW * cq + 32 * h;  // first column of this load
-                    const int nvalid = kvalid - c0;    // valid columns of this load (may be <= 0 or > 32)
+                for (int h = 0; h < nch; ++h) {
+                    const int kc = (pair ? 32 * cq : CPW * cq) + CW * h;  // first key of this load in the block
+                    const int c0 = pair ? 64 * unit + kc : kc;           // its first score column
+                    const int nvalid = kvalid - kc;  // valid columns of this load (may be <= 0 or > CW)
                     // warp-uniform: a warp whose rows all lie past the group, or a load past the group's
                     // keys, has nothing to compute (its P is zero, its other values unused)
                     const bool work = live && nvalid > 0;
-                    uint32_t s[32];
-                    tld<32>(tlane + (uint32_t)(TKB * b + c0), s);
-                    twait<32>(s);
-                    if (h == NCH - 1) {  // the scores are in registers: the buffer is free
+                    uint32_t s[CW];
+                    tld<CW>(tlane + (uint32_t)(TKB * b + c0), s);
+                    twait<CW>(s);
+                    if (h == nch - 1) {  // the scores are in registers: the buffer is free
                         fence_before();
                         __syncwarp();
                         if (lane == 0) bar_arrive(s_free(b));
@@ -564,76 +629,74 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                                 ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
                                 if (!ok) break;
                             }
-                            uint8_t *prow = sm + TcSmem::kP + pb * kPB + (c0 >> 6) * (TQ * 128) + row * 128;
-                            const int k0 = (c0 & 63) >> 3;
+                            uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
+                            const int k0 = (kc & 63) >> 3;
 #pragma unroll
-                            for (int cc = 0; cc < 4; ++cc) *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                            for (int cc = 0; cc < CW / 8; ++cc) *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
                         }
                         continue;
                     }
-                    const bool whole = nvalid >= 32;
+                    const bool whole = nvalid >= CW;
                     if (pass == 0) {
                         float m = __uint_as_float(s[0]);
 #pragma unroll
-                        for (int c = 1; c < 32; ++c) m = fmaxf(m, __uint_as_float(s[c]));
+                        for (int c = 1; c < CW; ++c) m = fmaxf(m, __uint_as_float(s[c]));
                         if (!whole) {
                             m = -3.0e38f;
 #pragma unroll
-                            for (int c = 0; c < 32; ++c) m = c < nvalid ? fmaxf(m, __uint_as_float(s[c])) : m;
+                            for (int c = 0; c < CW; ++c) m = c < nvalid ? fmaxf(m, __uint_as_float(s[c])) : m;
                         }
                         mx = fmaxf(mx, m);
                     } else if (pass == 1) {
-                        uint32_t e[32];
+                        uint32_t e[CW];
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) e[c] = shift_exp_nbits<FASTQ>(s[c], se);
+                        for (int c = 0; c < CW; ++c) e[c] = shift_exp_nbits<FASTQ>(s[c], se);
                         if (!whole) {
 #pragma unroll
-                            for (int c = 0; c < 32; ++c) e[c] = c < nvalid ? e[c] : 0u;
+                            for (int c = 0; c < CW; ++c) e[c] = c < nvalid ? e[c] : 0u;
                         }
                         // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits;
                         // with SUM4 (I0 2^k < 2^30) four do
                         uint64_t part = 0;
                         if constexpr (SUM4) {
 #pragma unroll
-                            for (int c = 0; c < 32; c += 4) part += (uint64_t)(e[c] + e[c + 1] + e[c + 2] + e[c + 3]);
+                            for (int c = 0; c < CW; c += 4) part += (uint64_t)(e[c] + e[c + 1] + e[c + 2] + e[c + 3]);
                         } else {
 #pragma unroll
-                            for (int c = 0; c < 32; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
+                            for (int c = 0; c < CW; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
                         }
                         sum += part;
                     } else {
-                        // P of the 32 keys as fp16 (exact integers below 1024): the bits of 1024 + P are
-                        // 0x6400 | P, and one half2 subtraction of 1024 leaves P
-                        uint32_t pw[32];
+                        // P of the CW keys as fp16 operands: P < 1024, so its own bits are the fp16
+                        // subnormal P 2^-24, exact; O then accumulates 2^-24 P V (also exact) and is
+                        // scaled back by 2^24 when read
+                        uint32_t pw[CW];
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
+                        for (int c = 0; c < CW; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
                         if (!whole) {
 #pragma unroll
-                            for (int c = 0; c < 32; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
+                            for (int c = 0; c < CW; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
                         }
-                        uint32_t w[16];
+                        uint32_t w[CW / 2];
 #pragma unroll
-                        for (int c = 0; c < 16; ++c) {
-                            uint32_t x = (0x6400u | pw[2 * c]) | ((0x6400u | pw[2 * c + 1]) << 16);
-                            __half2 hh = __hsub2(*reinterpret_cast<__half2 *>(&x), h1024);
-                            w[c] = *reinterpret_cast<uint32_t *>(&hh);
-                        }
+                        for (int c = 0; c < CW / 2; ++c) w[c] = __byte_perm(pw[2 * c], pw[2 * c + 1], 0x5410);
                         if (!p_ready) {
                             p_ready = true;
                             ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
                             if (!ok) break;
                         }
-                        // keys c0 .. c0 + 31 sit in sub-tile c0 / 64, chunks (c0 % 64) / 8 .. + 3 of the row;
+                        // keys kc .. kc + CW - 1 sit in sub-tile kc / 64, chunks (kc % 64) / 8 .. of the row;
                         // 16-byte chunk k of a row sits at k ^ (row & 7)
-                        uint8_t *prow = sm + TcSmem::kP + pb * kPB + (c0 >> 6) * (TQ * 128) + row * 128;
-                        const int k0 = (c0 & 63) >> 3;
+                        uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
+                        const int k0 = (kc & 63) >> 3;
 #pragma unroll
-                        for (int cc = 0; cc < 4; ++cc)
+                        for (int cc = 0; cc < CW / 8; ++cc)
                             *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) =
                                 make_uint4(w[4 * cc], w[4 * cc + 1], w[4 * cc + 2], w[4 * cc + 3]);
                     }
                 }
-                if (++b == NS) {
+                if (pass == 2) sph ^= 1u;  // pass 3: S[0] alone
+                else if (++b == NS) {
                     b = 0;
                     sph ^= 1u;
                 }
@@ -660,13 +723,15 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         if (ok) {
             fence_after();
             uint32_t o[OPW];
-            tld<OPW>(tlane + kOcol + (uint32_t)(OPW * cq), o);
+            tld<OPW>(tlane + kOcol + (uint32_t)(64 * unit + OPW * cq), o);
             twait<OPW>(o);
-            if (tok < Tg) {
+            if (live && tok < Tg) {
                 int32_t r[OPW];
 #pragma unroll
-                for (int c = 0; c < OPW; ++c) r[c] = sat8(rq(__float2int_rn(__uint_as_float(o[c])), p.m_o, p.s_o));
-                const int64_t t = gr.token(tok);
+                for (int c = 0; c < OPW; ++c)
+                    r[c] = sat8(rq(__float2int_rn(__uint_as_float(o[c]) * 16777216.0f), p.m_o, p.s_o));  // O = 2^24 acc
+                const int64_t t = unit ? base1 + tok : gr.token(tok);
+                const int ho = unit ? hoff1 : hoff;
                 if (p.o_f16) {
                     // 1152 + r (|r| <= 127) has the fp16 bits 0x6480 + r; subtracting 1152 leaves r
                     const __half2 h1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
@@ -677,7 +742,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                         __half2 hh = __hsub2(*reinterpret_cast<__half2 *>(&x), h1152);
                         hw[c] = *reinterpret_cast<uint32_t *>(&hh);
                     }
-                    uint4 *dst = (uint4 *)((__half *)p.O + t * p.ld_o + hoff + OPW * cq);
+                    uint4 *dst = (uint4 *)((__half *)p.O + t * p.ld_o + ho + OPW * cq);
 #pragma unroll
                     for (int c = 0; c < OPW / 8; ++c) dst[c] = make_uint4(hw[4 * c], hw[4 * c + 1], hw[4 * c + 2], hw[4 * c + 3]);
                 } else {
@@ -686,7 +751,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     for (int c = 0; c < OPW / 4; ++c)
                         bw[c] = (uint32_t)(uint8_t)r[4 * c] | ((uint32_t)(uint8_t)r[4 * c + 1] << 8) |
                                 ((uint32_t)(uint8_t)r[4 * c + 2] << 16) | ((uint32_t)(uint8_t)r[4 * c + 3] << 24);
-                    uint4 *dst = (uint4 *)((int8_t *)p.O + t * p.ld_o + hoff + OPW * cq);
+                    uint4 *dst = (uint4 *)((int8_t *)p.O + t * p.ld_o + ho + OPW * cq);
 #pragma unroll
                     for (int c = 0; c < OPW / 16; ++c) dst[c] = make_uint4(bw[4 * c], bw[4 * c + 1], bw[4 * c + 2], bw[4 * c + 3]);
                 }
@@ -720,15 +785,15 @@ EncodeTiledTc encode_tc() {
 }
 
 // Tensor map over the 64 H fp16 columns of k (or v) starting at `base`: 2-D {64 H, B T} with
-// 64 x 64 boxes, or (win) 3-D {64 H, gs, B gs} with 64 x ws x R boxes; 128-byte swizzle, zero fill.
-bool kv_map(CUtensorMap *m, const void *base, const AttnParams &p, bool win, int ws, int R) {
+// 64 x `rows` boxes, or (win) 3-D {64 H, gs, B gs} with 64 x ws x R boxes; 128-byte swizzle, zero fill.
+bool kv_map(CUtensorMap *m, const void *base, const AttnParams &p, bool win, int ws, int R, int rows = TKB) {
     EncodeTiledTc fn = encode_tc();
     if (!fn) return false;
     const cuuint64_t row = (cuuint64_t)p.ld_qkv * 2;
     if (!win) {
         cuuint64_t dims[2] = {(cuuint64_t)p.H * 64, (cuuint64_t)p.B * p.T};
         cuuint64_t str[1] = {row};
-        cuuint32_t box[2] = {64, (cuuint32_t)TKB};
+        cuuint32_t box[2] = {64, (cuuint32_t)rows};
         cuuint32_t es[2] = {1, 1};
         return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(base), dims, str, box, es,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -785,7 +850,13 @@ cudaError_t launch_attention_tc(const AttnParams &p, cudaStream_t s) {
     const bool direct = p.smx.s_d < 0 && p.smx.m_p + 15 <= p.smx.M_hw && 32 - p.smx.k_out >= p.smx.se.k;
     const size_t smem = 1024 + TcSmem::kBytes;
     a.nq = (Tg + TQ - 1) / TQ;
-    const dim3 grid((unsigned)(a.nq * p.H * p.B * G2));
+    // global attention whose last query tile has at most 64 rows: two units' last tiles per CTA
+    // (T = 1600: 48 half tiles become 24 CTAs, so 8 x 6 units fill two waves of two CTAs per SM)
+    a.pair = !win && Tg - (a.nq - 1) * TQ <= 64 ? 1 : 0;
+    if (a.pair && (!kv_map(&a.kmap64, p.K, p, false, 0, 0, 64) || !kv_map(&a.vmap64, p.V, p, false, 0, 0, 64)))
+        return cudaErrorNotSupported;
+    const int units = p.H * p.B * G2;
+    const dim3 grid((unsigned)((a.nq - 1) * units + (a.pair ? (units + 1) / 2 : units)));
     const bool sum4 = ((int64_t)p.smx.se.I0 << p.smx.se.k) < ((int64_t)1 << 30);
     if (fastq && direct)
         return sum4 ? launch_tc_kernel<true, true, true>(a, grid, smem, s) : launch_tc_kernel<true, true, false>(a, grid, smem, s);

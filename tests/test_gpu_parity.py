@@ -237,14 +237,17 @@ def test_attention_f16_output(ilw, orc, B, T, H, dh, win):
 
 
 @pytest.mark.parametrize("B,T,H,dh,win", [(1, 128, 2, 64, 0), (1, 129, 1, 64, 0), (2, 257, 2, 64, 0),
-                                          (1, 130, 8, 64, 0), (1, 196, 1, 64, 2), (1, 1296, 1, 64, 3),
-                                          (2, 6400, 1, 64, 2)])
+                                          (1, 130, 8, 64, 0), (3, 900, 3, 64, 0), (1, 196, 1, 64, 2),
+                                          (1, 1296, 1, 64, 3), (2, 6400, 1, 64, 2)])
 @pytest.mark.parametrize("o_f16", [False, True])
 def test_attention_tensor_memory_shapes(ilw, orc, B, T, H, dh, win, o_f16):
     """Shapes at the tensor-memory kernel's block edges with fp16-carried q|k|v: a group of exactly
     one query tile, one query past it (a tile whose warps but one have no query), several images,
     8 heads, window sides 7 (one key block of 49), 12 (two blocks of 120 keys) and 40 (14 blocks;
-    the last key box reaches past the window and, for the last image, past the matrix)."""
+    the last key box reaches past the window and, for the last image, past the matrix).  Global
+    groups whose last tile has at most 64 queries put two (image, head) units' last tiles in one
+    CTA: T = 129, 257, 130 and 900 run that form, 3 x 3 units at T = 900 with pairs that span two
+    images and a last CTA with one unit."""
     d = H * dh
     qkv = synth.uniform_int(14, f"qkvtc{T}{H}{win}", (B * T, 3 * d), -127, 127, np.int8)
     smx = {"I0": 5000, "k_inter": 16, "k_out": 8, "s_d": -1, "m_p": 4, "M_hw": 31}

@@ -251,6 +251,56 @@ def test_attention_cta_order_is_a_bijection(nq, H, Z):
     assert all(t[0] == nq - 1 for t in seen[F:]) and all(t[0] < nq - 1 for t in seen[:F])
 
 
+@pytest.mark.parametrize("nq,H,Z", [(1, 1, 1), (1, 3, 3), (13, 6, 8), (8, 3, 3), (2, 8, 1)])
+def test_attention_paired_last_tiles_cover_every_unit(nq, H, Z):
+    """Global attention whose last tile has at most 64 queries: the first (nq - 1) H Z CTAs keep the
+    one-tile mapping, CTA F + j holds the last tiles of units 2 j and 2 j + 1 (unit = head + H
+    image), the second absent when H Z is odd.  Every (tile, unit) is taken once, pairs may span two
+    images, and the grid shrinks by floor(H Z / 2) CTAs."""
+    F = (nq - 1) * H * Z
+    units = H * Z
+    grid = F + (units + 1) // 2
+    seen = []
+    for L in range(grid):
+        if L < F:
+            seen.append((L % (nq - 1), (L // (nq - 1)) % H, L // ((nq - 1) * H)))
+        else:
+            u0 = 2 * (L - F)
+            seen.append((nq - 1, u0 % H, u0 // H))
+            if u0 + 1 < units:
+                seen.append((nq - 1, (u0 + 1) % H, (u0 + 1) // H))
+            else:
+                assert L == grid - 1 and units % 2 == 1
+    assert sorted(seen) == sorted((q, h, z) for q in range(nq) for h in range(H) for z in range(Z))
+    assert grid == nq * units - units // 2
+
+
+@pytest.mark.parametrize("nkb", [1, 2, 3, 13, 25])
+def test_attention_piece_stream_matches_mma_order(nkb):
+    """The loader's piece sequence (k blocks of passes 1 and 2, then k0, k(j + 1), v(j) ..., v(nkb - 1))
+    is exactly the order in which the MMA issuer consumes ring slots: scores of block kb + 1 before
+    the P V of block kb in pass 3."""
+    loads = []
+    for i in range(4 * nkb):
+        if i < 2 * nkb:
+            loads.append(("k", i if i < nkb else i - nkb))
+        else:
+            j = i - 2 * nkb
+            if j == 0:
+                loads.append(("k", 0))
+            elif j == 2 * nkb - 1:
+                loads.append(("v", nkb - 1))
+            elif j & 1:
+                loads.append(("k", (j + 1) >> 1))
+            else:
+                loads.append(("v", (j - 2) >> 1))
+    mma = [("k", j % nkb) for j in range(2 * nkb)] + [("k", 0)]
+    for kb in range(nkb - 1):
+        mma += [("k", kb + 1), ("v", kb)]
+    mma.append(("v", nkb - 1))
+    assert loads == mma
+
+
 @pytest.mark.parametrize("ws", [1, 5, 7, 12, 20, 40, 64, 100, 128])
 def test_attention_window_key_boxes(ws):
     """Window key blocks are 3-D boxes of R = min(floor(128 / ws), ws) whole window rows: row z,
