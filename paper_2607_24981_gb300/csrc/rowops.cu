@@ -45,10 +45,34 @@ __device__ __forceinline__ uint64_t group_sum_u64(uint64_t v) {
     return v;
 }
 
+// The output floor(e F / 2^sh) as one high-word product: for sh <= 32 and F < 2^sh,
+// F 2^(32 - sh) < 2^32 and floor(e F 2^(32 - sh) / 2^32) is the same floor; for sh > 32 the high word
+// of e F shifted right by sh - 32 (floors compose).  `ok` is false for the rows neither form covers
+// (sh < 32 with F >= 2^sh, i.e. a reduced denominator below 2^(31 - sh)), which take shiftmax_out.
+struct RowOut {
+    uint32_t Fs;
+    uint32_t rs;
+    bool ok;
+};
+__device__ __forceinline__ RowOut row_out(const RowNorm &rn) {
+    RowOut o;
+    if (rn.sh <= 32) {
+        o.ok = rn.sh == 32 || (rn.F >> rn.sh) == 0;
+        o.Fs = o.ok ? rn.F << (32 - rn.sh) : 0u;
+        o.rs = 0;
+    } else {
+        o.ok = true;
+        o.Fs = rn.F;
+        o.rs = (uint32_t)min(rn.sh - 32, 31);
+    }
+    return o;
+}
+
 // LANES lanes own one row (32 / LANES rows per warp); NCH = 4-element chunks per lane (row length
 // <= 4 * LANES * NCH).  Vector loads need len % 4 == 0 and 16-byte aligned rows.  All NCH loads of a
 // lane are issued before the first use, so each warp keeps 32 * NCH * 16 bytes in flight.
-template <int NCH, int LANES, bool FASTQ>
+// SUM4: I0 2^k < 2^30, so four ShiftExp values add up in 32 bits (two always do: I0 2^k < 2^31).
+template <int NCH, int LANES, bool FASTQ, bool SUM4>
 __global__ void __launch_bounds__(256) shiftmax_rows_vec(const int32_t *__restrict__ X, int64_t ldx,
                                                           int64_t rows, int32_t len, const ShiftmaxC c,
                                                           uint8_t *__restrict__ P, int64_t ldp) {
@@ -75,27 +99,44 @@ __global__ void __launch_bounds__(256) shiftmax_rows_vec(const int32_t *__restri
 #pragma unroll
     for (int j = 0; j < NCH; ++j) {
         const int ch = sub + LANES * j;
-        int32_t *e = (int32_t *)&v[j];
+        uint32_t *e = (uint32_t *)&v[j];
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-            const uint32_t a = min((uint32_t)mx - (uint32_t)e[q], 1u << 30);
-            const uint32_t ex = shift_exp_mag_q<FASTQ>(a, c.se);
-            e[q] = (int32_t)ex;
-            if (ch < nch) sum += ex;
+            const uint32_t a = min((uint32_t)mx - e[q], 1u << 30);
+            e[q] = shift_exp_mag_q<FASTQ>(a, c.se);
+        }
+        if (ch < nch) {
+            if constexpr (SUM4) sum += (uint64_t)(e[0] + e[1] + e[2] + e[3]);
+            else sum += (uint64_t)(e[0] + e[1]) + (uint64_t)(e[2] + e[3]);
         }
     }
     sum = group_sum_u64<LANES>(sum);
     if (!live) return;
     const RowNorm rn = shiftmax_norm(sum, c.s_d, c.m_p, c.M_hw, c.k_out);
+    const RowOut ro = row_out(rn);
     uint32_t *pr = (uint32_t *)(P + row * ldp);
+    // every output is below 2^k_out <= 256: the four bytes of a chunk by two byte permutations
+    if (ro.ok) {
 #pragma unroll
-    for (int j = 0; j < NCH; ++j) {
-        const int ch = sub + LANES * j;
-        if (ch < nch) {
-            const int32_t *e = (const int32_t *)&v[j];
-            const uint32_t o = shiftmax_out((uint32_t)e[0], rn) | (shiftmax_out((uint32_t)e[1], rn) << 8) |
-                               (shiftmax_out((uint32_t)e[2], rn) << 16) | (shiftmax_out((uint32_t)e[3], rn) << 24);
-            __stcs(pr + ch, o);
+        for (int j = 0; j < NCH; ++j) {
+            const int ch = sub + LANES * j;
+            if (ch < nch) {
+                const uint32_t *e = (const uint32_t *)&v[j];
+                const uint32_t b01 = __byte_perm(__umulhi(e[0], ro.Fs) >> ro.rs, __umulhi(e[1], ro.Fs) >> ro.rs, 0x0040);
+                const uint32_t b23 = __byte_perm(__umulhi(e[2], ro.Fs) >> ro.rs, __umulhi(e[3], ro.Fs) >> ro.rs, 0x0040);
+                __stcs(pr + ch, __byte_perm(b01, b23, 0x5410));
+            }
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) {
+            const int ch = sub + LANES * j;
+            if (ch < nch) {
+                const uint32_t *e = (const uint32_t *)&v[j];
+                const uint32_t o = shiftmax_out(e[0], rn) | (shiftmax_out(e[1], rn) << 8) |
+                                   (shiftmax_out(e[2], rn) << 16) | (shiftmax_out(e[3], rn) << 24);
+                __stcs(pr + ch, o);
+            }
         }
     }
 }
@@ -297,7 +338,7 @@ __device__ __noinline__ void ln_norm4_exact(const int32_t (&x)[4], int64_t mu, i
 // |beta| <= 2^30 the requantisation is the high-word form with a scalar rounding constant; otherwise
 // (or for rows with iters = 0 and V >= 2^32) the 64-bit formulas run.
 template <typename TIn, typename TOut, int LPR, int CPL>
-__global__ void __launch_bounds__(256) layernorm_rows(const LnParams p) {
+__global__ void __launch_bounds__(256, 3) layernorm_rows(const LnParams p) {
     extern __shared__ __align__(16) int32_t ln_par[];  // beta[C], mult[C], shift[C]
     constexpr int EB = sizeof(TIn), EPC = 16 / EB;      // elements per 16-byte chunk
     constexpr int RPW = 32 / LPR;
@@ -530,9 +571,12 @@ cudaError_t launch_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, in
     const bool fq = c.se.m32 != 0;
     // rows per CTA: 8 warps x (32 / LANES) rows
     auto g = [&](int lanes) { return dim3((unsigned)((rows + 8 * (32 / lanes) - 1) / (8 * (32 / lanes)))); };
-#define ILW_SMX(NCH, LANES)                                                                                  \
-    (fq ? (shiftmax_rows_vec<NCH, LANES, true><<<g(LANES), 256, 0, s>>>(X, ldx, rows, len, c, P, ldp), 0)   \
-        : (shiftmax_rows_vec<NCH, LANES, false><<<g(LANES), 256, 0, s>>>(X, ldx, rows, len, c, P, ldp), 0))
+    const bool s4 = ((int64_t)c.se.I0 << c.se.k) < ((int64_t)1 << 30);
+#define ILW_SMX(NCH, LANES)                                                                                         \
+    (fq ? (s4 ? (shiftmax_rows_vec<NCH, LANES, true, true><<<g(LANES), 256, 0, s>>>(X, ldx, rows, len, c, P, ldp), 0)  \
+              : (shiftmax_rows_vec<NCH, LANES, true, false><<<g(LANES), 256, 0, s>>>(X, ldx, rows, len, c, P, ldp), 0)) \
+        : (s4 ? (shiftmax_rows_vec<NCH, LANES, false, true><<<g(LANES), 256, 0, s>>>(X, ldx, rows, len, c, P, ldp), 0) \
+              : (shiftmax_rows_vec<NCH, LANES, false, false><<<g(LANES), 256, 0, s>>>(X, ldx, rows, len, c, P, ldp), 0)))
     if (vec && len <= 64) ILW_SMX(4, 4);
     else if (vec && len <= 128) ILW_SMX(4, 8);
     else if (vec && len <= 416) ILW_SMX(13, 8);

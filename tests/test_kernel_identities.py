@@ -371,3 +371,30 @@ def test_shiftexp_exponent_from_negative_biased_bits():
     n = (w + (w >> np.uint64(1)) - ((w + np.uint64(14)) >> np.uint64(4)) - np.uint64(0x23D00001)) & M32
     assert np.array_equal(n.astype(np.int64), a + ((a + 1) >> 1) - ((a + 15) >> 4))
 
+
+
+def test_shiftmax_rows_one_multiply_output():
+    """The standalone Shiftmax rows kernel writes floor(e F / 2^sh) as umulhi(e, Fs) >> rs: for
+    sh <= 32 and F < 2^sh, Fs = F 2^(32 - sh), rs = 0; for sh > 32, Fs = F, rs = min(sh - 32, 31);
+    other rows take the 64-bit form.  Checked against the exact floor for e < 2^31 over the whole
+    range of F and sh, extremes included."""
+    rng = np.random.default_rng(7)
+    es = np.concatenate([rng.integers(0, 1 << 31, 4000), [0, 1, (1 << 31) - 1, (1 << 30), 12345]])
+    checked = 0
+    for sh in list(range(17, 64)):
+        Fs_list = np.concatenate([rng.integers(1, 1 << 31, 60), [1, 2, 31, 32, (1 << 31) - 1, 1 << 24]])
+        for F in Fs_list:
+            F = int(F)
+            if sh <= 32:
+                ok = sh == 32 or (F >> sh) == 0
+                Fs, rs = (F << (32 - sh)) if ok else 0, 0
+            else:
+                ok, Fs, rs = True, F, min(sh - 32, 31)
+            if not ok:
+                continue
+            assert Fs < (1 << 32)
+            for e in es:
+                e = int(e)
+                assert ((e * Fs) >> 32) >> rs == (e * F) >> sh
+                checked += 1
+    assert checked > 100000
