@@ -31,12 +31,11 @@
 //               while the softmax works.  Warps whose rows all lie past the group, and 32-key
 //               loads past its keys, skip the arithmetic (their P is written as zero)
 // The CTAs holding the last (possibly partial, hence shorter) query tile of each group come after
-// all the others, so they fill the last wave.  When the last tile has at most 64 queries, the
-// last tiles of two (image, head, group) units share one CTA (rows 0-63 and 64-127): a key block
-// is then up to 64 keys of each unit (64 tokens, or min(floor(64 / ws), ws) whole window rows), two
-// N = 64 score MMAs, each unit's rows reading their own half of the columns, and each unit has its
-// own O.  Global attention at 1600 tokens goes from 8 x 6 x 13 = 624 CTAs (2.05 waves of two per
-// SM) to 600 (two waves).
+// all the others, so they fill the last wave.  Global attention whose last tile has at most 64
+// queries puts the last tiles of two (image, head) units in one CTA (rows 0-63 and 64-127): a key
+// block is then 64 keys of each unit (two N = 64 score MMAs, each unit's rows reading their own
+// half of the columns), and each unit has its own O.  At 1600 tokens this turns 8 x 6 x 13 = 624
+// CTAs (2.05 waves of two per SM) into 600 (two waves).
 // Every mbarrier wait is bounded (about one second); on expiry the kernel latches the device status
 // word, every role stops, the loaders drain their copies and the TMEM is freed after every MMA
 // issued has completed.
@@ -213,15 +212,13 @@ __device__ __forceinline__ void tma_3d(uint32_t dst, const CUtensorMap *m, int32
 // Kernel arguments: the attention problem and the tensor maps of its k and v columns.
 struct TcArgs {
     CUtensorMap kmap, vmap;      // 2-D {64 H, B T} (global) or 3-D {64 H, gs, B gs} (windows), 128-byte swizzle
-    CUtensorMap kmap64, vmap64;  // paired last tiles: 64-row boxes (global) or boxes of rpb2 window rows
+    CUtensorMap kmap64, vmap64;  // global, paired last tiles: the same with 64-row boxes
     AttnParams p;
     int32_t kbk;   // keys per block: 128 (global) or R ws (windows)
     int32_t rpb;   // window rows per block R (windows)
     int32_t win;   // 1: 3-D window boxes
     int32_t nq;    // query tiles per group
-    int32_t pair;  // 1: the last tiles (<= 64 queries each) of two (image, head, group) units share a CTA
-    int32_t kbk2;  // paired tiles: keys per block and unit (64, or rpb2 ws <= 64 for windows)
-    int32_t rpb2;  // paired tiles: window rows per block, min(floor(64 / ws), ws)
+    int32_t pair;  // 1: the last tiles (<= 64 queries each) of two (image, head) units share a CTA
 };
 __device__ __forceinline__ uint32_t shr_clamp(uint32_t v, uint32_t n) {
     uint32_t r;
@@ -303,23 +300,22 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             z1 = has1 ? u1 / p.H : z;
         }
     }
-    // the group of the CTA's (first) unit, and of the second unit of a paired CTA
-    auto group_of = [&](int zz) {
-        GroupTc g;
-        const int G2 = p.nw * p.nw, b = zz / G2, w = zz % G2;
-        g.base = (int64_t)b * p.T;
-        g.nw = p.nw;
-        g.gs = p.grid_side;
-        g.ws = p.nw > 1 ? p.grid_side / p.nw : 0;
-        g.wy = w / p.nw;
-        g.wx = w % p.nw;
-        g.Tg = p.nw > 1 ? g.ws * g.ws : p.T;
-        return g;
-    };
-    const GroupTc gr = group_of(z), gr1 = group_of(z1);
-    const int Tg = gr.Tg, q0 = qt * TQ, hoff = head * 64, kbk = pair ? args.kbk2 : args.kbk;
+    GroupTc gr;
+    {
+        const int G2 = p.nw * p.nw, b = z / G2, w = z % G2;
+        gr.base = (int64_t)b * p.T;
+        gr.nw = p.nw;
+        gr.gs = p.grid_side;
+        gr.ws = p.nw > 1 ? p.grid_side / p.nw : 0;
+        gr.wy = w / p.nw;
+        gr.wx = w % p.nw;
+        gr.Tg = p.nw > 1 ? gr.ws * gr.ws : p.T;
+    }
+    const int Tg = gr.Tg, q0 = qt * TQ, hoff = head * 64, kbk = pair ? 64 : args.kbk;
     const int nkb = (Tg + kbk - 1) / kbk;
-    const int hoff1 = head1 * 64;  // pair: the second unit's head offset
+    // pair: the second unit's first token (global attention: image z1) and head offset
+    const int64_t base1 = (int64_t)z1 * p.T;
+    const int hoff1 = head1 * 64;
 
     if (threadIdx.x == 0) {
         bar_init(bq_full, NLOAD);
@@ -482,7 +478,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
         for (int it = tl; it < TQ * 8; it += NLOAD) {
             const int r = it >> 3, c = it & 7, u = pair ? r >> 6 : 0, tok = q0 + (pair ? r & 63 : r);
             const bool okr = tok < Tg && (u == 0 || has1);
-            const int64_t t = !okr ? 0 : u ? gr1.token(tok) : gr.token(tok);
+            const int64_t t = !okr ? 0 : u ? base1 + tok : gr.token(tok);
             cpa16(sbase + TcSmem::kQ + r * 128 + ((c ^ (r & 7)) << 4), Qg + t * ld + (u ? hoff1 : hoff) + 8 * c,
                   okr ? 16u : 0u);
         }
@@ -494,7 +490,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             // the key-block stream: piece i into slot i % NP once the piece before it there is consumed.
             // Pieces 0 .. 2 nkb - 1 are the k blocks of passes 1 and 2; pass 3 follows the MMA's order:
             // k0, then k(j + 1), v(j) for j = 0 .. nkb - 2, then v(nkb - 1)
-            const uint32_t bytes = (pair ? 2u : 1u) * (uint32_t)kbk * 128u;
+            const uint32_t bytes = pair ? 2u * 64u * 128u : (uint32_t)kbk * 128u;
             const int bimg = gr.base / p.T, npiece = 4 * nkb;
             int issued = 0, slot = 0;
             uint32_t ph = 0;
@@ -515,20 +511,11 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 const uint32_t dst = sbase + TcSmem::kRing + slot * kSlotB;
                 bar_expect_tx(full(slot), bytes);
                 if (pair) {
-                    // kbk <= 64 keys of each unit: from rows 0 and 64 of the slot (the second unit's
-                    // rows repeat the first's when there is none; nothing reads them then; rows a
-                    // window block leaves unwritten stay zero)
+                    // 64 keys of each unit: rows 0-63 and 64-127 of the slot (the second unit's rows
+                    // repeat the first's when there is none; nothing reads them then)
                     const CUtensorMap *m64 = isv ? &args.vmap64 : &args.kmap64;
-                    const GroupTc &g1 = has1 ? gr1 : gr;
-                    const int h1 = has1 ? hoff1 : hoff;
-                    if (args.win) {
-                        tma_3d(dst, m64, hoff, gr.wx * gr.ws, bimg * gr.gs + gr.wy * gr.ws + kb * args.rpb2, full(slot));
-                        tma_3d(dst + 8192u, m64, h1, g1.wx * g1.ws,
-                               (int32_t)(g1.base / p.T) * g1.gs + g1.wy * g1.ws + kb * args.rpb2, full(slot));
-                    } else {
-                        tma_2d(dst, m64, hoff, (int32_t)(gr.base + kb * 64), full(slot));
-                        tma_2d(dst + 8192u, m64, h1, (int32_t)(g1.base + kb * 64), full(slot));
-                    }
+                    tma_2d(dst, m64, hoff, (int32_t)(gr.base + kb * 64), full(slot));
+                    tma_2d(dst + 8192u, m64, has1 ? hoff1 : hoff, (int32_t)((has1 ? base1 : gr.base) + kb * 64), full(slot));
                 } else if (args.win)
                     tma_3d(dst, m, hoff, gr.wx * gr.ws, bimg * gr.gs + gr.wy * gr.ws + kb * args.rpb, full(slot));
                 else
@@ -743,7 +730,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
 #pragma unroll
                 for (int c = 0; c < OPW; ++c)
                     r[c] = sat8(rq(__float2int_rn(__uint_as_float(o[c]) * 16777216.0f), p.m_o, p.s_o));  // O = 2^24 acc
-                const int64_t t = unit ? gr1.token(tok) : gr.token(tok);
+                const int64_t t = unit ? base1 + tok : gr.token(tok);
                 const int ho = unit ? hoff1 : hoff;
                 if (p.o_f16) {
                     // 1152 + r (|r| <= 127) has the fp16 bits 0x6480 + r; subtracting 1152 leaves r
@@ -863,14 +850,10 @@ cudaError_t launch_attention_tc(const AttnParams &p, cudaStream_t s) {
     const bool direct = p.smx.s_d < 0 && p.smx.m_p + 15 <= p.smx.M_hw && 32 - p.smx.k_out >= p.smx.se.k;
     const size_t smem = 1024 + TcSmem::kBytes;
     a.nq = (Tg + TQ - 1) / TQ;
-    // a last query tile of at most 64 rows: two units' last tiles per CTA (global T = 1600: 48 half
-    // tiles become 24 CTAs, so 8 x 6 units fill two waves of two CTAs per SM; 2 x 2 windows of 400:
-    // 192 tiles of 16 queries become 96 CTAs)
-    // (windows: blocks of rpb2 whole window rows, at most 64 keys, so windows of side <= 64)
-    a.pair = Tg - (a.nq - 1) * TQ <= 64 && (!win || ws <= 64) ? 1 : 0;
-    a.rpb2 = win ? (64 / ws < ws ? 64 / ws : ws) : 0;
-    a.kbk2 = win ? a.rpb2 * ws : 64;
-    if (a.pair && (!kv_map(&a.kmap64, p.K, p, win, ws, a.rpb2, 64) || !kv_map(&a.vmap64, p.V, p, win, ws, a.rpb2, 64)))
+    // global attention whose last query tile has at most 64 rows: two units' last tiles per CTA
+    // (T = 1600: 48 half tiles become 24 CTAs, so 8 x 6 units fill two waves of two CTAs per SM)
+    a.pair = !win && Tg - (a.nq - 1) * TQ <= 64 ? 1 : 0;
+    if (a.pair && (!kv_map(&a.kmap64, p.K, p, false, 0, 0, 64) || !kv_map(&a.vmap64, p.V, p, false, 0, 0, 64)))
         return cudaErrorNotSupported;
     const int units = p.H * p.B * G2;
     const dim3 grid((unsigned)((a.nq - 1) * units + (a.pair ? (units + 1) / 2 : units)));

@@ -244,11 +244,10 @@ def test_attention_tensor_memory_shapes(ilw, orc, B, T, H, dh, win, o_f16):
     """Shapes at the tensor-memory kernel's block edges with fp16-carried q|k|v: a group of exactly
     one query tile, one query past it (a tile whose warps but one have no query), several images,
     8 heads, window sides 7 (one key block of 49), 12 (two blocks of 120 keys) and 40 (14 blocks;
-    the last key box reaches past the window and, for the last image, past the matrix).  Groups
-    whose last tile has at most 64 queries put two (image, head, group) units' last tiles in one
-    CTA: global T = 129, 257, 130 and 900 (3 x 3 units with pairs that span two images and a last
-    CTA with one unit) and windows of side 7 (4 units), 12 (9 units: one alone) and 40 (one
-    window row of 40 keys per paired block) run that form."""
+    the last key box reaches past the window and, for the last image, past the matrix).  Global
+    groups whose last tile has at most 64 queries put two (image, head) units' last tiles in one
+    CTA: T = 129, 257, 130 and 900 run that form, 3 x 3 units at T = 900 with pairs that span two
+    images and a last CTA with one unit."""
     d = H * dh
     qkv = synth.uniform_int(14, f"qkvtc{T}{H}{win}", (B * T, 3 * d), -127, 127, np.int8)
     smx = {"I0": 5000, "k_inter": 16, "k_out": 8, "s_d": -1, "m_p": 4, "M_hw": 31}
