@@ -49,6 +49,16 @@
 namespace ilw {
 namespace {
 
+// The CTA form seen by the softmax warps: fixed at compile time (launches without paired tiles) or
+// read at run time (launches with them, where one code path serves both forms: two specialised
+// copies measured slower there, the SMs running both).
+template <bool B> struct FixedForm {
+    __device__ constexpr bool operator()() const { return B; }
+};
+struct RuntimeForm {
+    bool pair;
+    __device__ bool operator()() const { return pair; }
+};
 constexpr int TQ = 128;      // queries per CTA
 constexpr int TKB = 128;     // keys per block (global attention)
 constexpr int NP = 3;        // ring slots of TKB x 128 bytes (one k or v block)
@@ -254,7 +264,8 @@ __device__ __forceinline__ uint32_t p_of(uint32_t w, const ShiftExpC &se, const 
 // DIRECT: per-row s_d with I_b F < 2^32 (the host's condition), so P comes straight from ShiftExp's
 // parts; otherwise P = (I_exp F) >> sh from the 64-bit product.  SUM4: every ShiftExp value is below
 // 2^30 (I0 2^k_inter < 2^30, the host's condition), so four of them add up in 32 bits.
-template <bool FASTQ, bool DIRECT, bool SUM4>
+// MAYPAIR: the launch may hold paired last tiles (args.pair).
+template <bool FASTQ, bool DIRECT, bool SUM4, bool MAYPAIR>
 __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const __grid_constant__ TcArgs args) {
     const AttnParams &p = args.p;
     extern __shared__ uint8_t smem_raw[];
@@ -285,7 +296,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             qt = L % (args.nq - 1);
             head = (L / (args.nq - 1)) % p.H;
             z = L / ((args.nq - 1) * p.H);
-        } else if (!args.pair) {
+        } else if (!MAYPAIR || !args.pair) {
             qt = args.nq - 1;
             head = (L - F) % p.H;
             z = (L - F) / p.H;
@@ -535,228 +546,234 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 }
         }
     } else {
-        // ------------------------------------------------------------------ softmax, one row per thread
-        // pair: rows 64-127 are the second unit's, row & 63 the query's place in its unit's tile
-        const int qw = warp & 3, cq = (warp - 4) >> 2, row = 32 * qw + lane, unit = pair ? qw >> 1 : 0;
-        const int urow = pair ? row & 63 : row, tok = q0 + urow;
-        // some row of this warp is a query of the group
-        const bool live = q0 + (urow & ~31) < Tg && (unit == 0 || has1);
-        const uint32_t tlane = tmem + ((uint32_t)(32 * qw) << 16);
-        float *red_max = (float *)(sm + TcSmem::kRedMax);
-        uint64_t *red_sum = (uint64_t *)(sm + TcSmem::kRedSum);
-        const ShiftExpC se = p.smx.se;
-        bool ok = true;
-        float mx = -3.0e38f;
-        uint64_t sum = 0;
-        RowNorm rn{};
-        uint32_t sh0 = 0;
-        // the other column groups' contributions to the row, through shared memory and the xchg barrier
-        auto exchange = [&](int phase) -> bool {
-            __syncwarp();
-            if (lane == 0) bar_arrive(xchg);
-            return __all_sync(0xffffffffu, bar_wait(xchg, phase, abort, p.status, kStatusTimeoutOperand));
-        };
-        int b = 0, pb = 0;  // S and P buffers of the next block, with their phase bits
-        uint32_t sph = 0, pph = 0;
-        for (int pass = 0; pass < 3 && ok; ++pass) {
-            if (pass == 1) {
-                red_max[cq * TQ + row] = mx;
-                if (!(ok = exchange(0))) break;
-#pragma unroll
-                for (int o = 1; o < NCQ; ++o) mx = fmaxf(mx, red_max[((cq + o) % NCQ) * TQ + row]);
-                if (cq == 0) {
-                    // this row's constant term -(2^23 + max + 1) as fp16 terms against the key weights
-                    // (1, 2048, 2048, 2048): max + 1 = 2048 a3 + a0 with a0 in [0, 2047], |a3| <= 512,
-                    // every term exact in fp16 and every partial sum of the MMA an integer below 2^24.
-                    // Both 16-byte halves of the row hold the same terms and the key rows carry their
-                    // weights in one half only, so the product does not depend on which half the
-                    // swizzle puts where.  Rows past the group get zeros.
-                    const int m1 = live && tok < Tg ? __float2int_rn(mx) + 1 : 0;
-                    const int a3 = m1 >> 11, a0 = m1 - (a3 << 11);
-                    const uint32_t h0 = (uint32_t)__half_as_ushort(__int2half_rn(-a0)),
-                                   h3 = (uint32_t)__half_as_ushort(__int2half_rn(-a3));
-                    const uint32_t n2048 = live && tok < Tg ? 0xE800u : 0u;  // -2048
-                    const uint4 ra = make_uint4(h0 | (n2048 << 16), n2048 | (h3 << 16), 0u, 0u);
-                    *(uint4 *)(sm + TcSmem::kAugA + row * 32) = ra;
-                    *(uint4 *)(sm + TcSmem::kAugA + row * 32 + 16) = ra;
-                    // key row `row`: (1, 2048, 2048, 2048) in the first half, zeros in the second
-                    *(uint4 *)(sm + TcSmem::kAugB + row * 32) = make_uint4(0x3C00u | (0x6800u << 16), 0x6800u | (0x6800u << 16), 0u, 0u);
-                    *(uint4 *)(sm + TcSmem::kAugB + row * 32 + 16) = make_uint4(0u, 0u, 0u, 0u);
-                    fence_async_smem();
-                    __syncwarp();
-                    if (lane == 0) bar_arrive(aug_full);
-                }
-            }
-            if (pass == 2) {
-                red_sum[cq * TQ + row] = sum;
-                if (!(ok = exchange(1))) break;
-#pragma unroll
-                for (int o = 1; o < NCQ; ++o) sum += red_sum[((cq + o) % NCQ) * TQ + row];
-                rn = shiftmax_norm(sum ? sum : 1, p.smx.s_d, p.smx.m_p, p.smx.M_hw, p.smx.k_out);
-                sh0 = (uint32_t)(rn.sh - se.k);
-            }
-            for (int kb = 0; kb < nkb; ++kb) {
-                // warp-uniform outcome: the TMEM loads below need the whole warp
-                ok = __all_sync(0xffffffffu, bar_wait(s_full(b), sph, abort, p.status, kStatusTimeoutMma));
-                if (!ok) break;
-                fence_after();
-                // pass 3 writes P into the buffer the previous block's P V reads: that MMA must have
-                // completed, which is waited for just before the first store, after the arithmetic
-                bool p_ready = pass != 2;
-                const int kvalid = min(kbk, Tg - kb * kbk);
-                // pair: 32 columns per block, from the unit's half of the score columns
-                const int nch = pair ? 32 / CW : NCH;
-#pragma unroll 1
-                for (int h = 0; h < nch; ++h) {
-                    const int kc = (pair ? 32 * cq : CPW * cq) + CW * h;  // first key of this load in the block
-                    const int c0 = pair ? 64 * unit + kc : kc;           // its first score column
-                    const int nvalid = kvalid - kc;  // valid columns of this load (may be <= 0 or > CW)
-                    // warp-uniform: a warp whose rows all lie past the group, or a load past the group's
-                    // keys, has nothing to compute (its P is zero, its other values unused)
-                    const bool work = live && nvalid > 0;
-                    uint32_t s[CW];
-                    tld<CW>(tlane + (uint32_t)(TKB * b + c0), s);
-                    twait<CW>(s);
-                    if (h == nch - 1) {  // the scores are in registers: the buffer is free
-                        fence_before();
+        // the softmax warps' work for the CTA's form (one unit, or two paired last tiles)
+        auto softmax = [&](auto form) {
+            const bool PAIR = form();
+            // ------------------------------------------------------------------ softmax, one row per thread
+            // pair: rows 64-127 are the second unit's, row & 63 the query's place in its unit's tile
+            const int qw = warp & 3, cq = (warp - 4) >> 2, row = 32 * qw + lane, unit = PAIR ? qw >> 1 : 0;
+            const int urow = PAIR ? row & 63 : row, tok = q0 + urow;
+            // some row of this warp is a query of the group
+            const bool live = q0 + (urow & ~31) < Tg && (!PAIR || unit == 0 || has1);
+            const uint32_t tlane = tmem + ((uint32_t)(32 * qw) << 16);
+            float *red_max = (float *)(sm + TcSmem::kRedMax);
+            uint64_t *red_sum = (uint64_t *)(sm + TcSmem::kRedSum);
+            const ShiftExpC se = p.smx.se;
+            bool ok = true;
+            float mx = -3.0e38f;
+            uint64_t sum = 0;
+            RowNorm rn{};
+            uint32_t sh0 = 0;
+            // the other column groups' contributions to the row, through shared memory and the xchg barrier
+            auto exchange = [&](int phase) -> bool {
+                __syncwarp();
+                if (lane == 0) bar_arrive(xchg);
+                return __all_sync(0xffffffffu, bar_wait(xchg, phase, abort, p.status, kStatusTimeoutOperand));
+            };
+            int b = 0, pb = 0;  // S and P buffers of the next block, with their phase bits
+            uint32_t sph = 0, pph = 0;
+            for (int pass = 0; pass < 3 && ok; ++pass) {
+                if (pass == 1) {
+                    red_max[cq * TQ + row] = mx;
+                    if (!(ok = exchange(0))) break;
+    #pragma unroll
+                    for (int o = 1; o < NCQ; ++o) mx = fmaxf(mx, red_max[((cq + o) % NCQ) * TQ + row]);
+                    if (cq == 0) {
+                        // this row's constant term -(2^23 + max + 1) as fp16 terms against the key weights
+                        // (1, 2048, 2048, 2048): max + 1 = 2048 a3 + a0 with a0 in [0, 2047], |a3| <= 512,
+                        // every term exact in fp16 and every partial sum of the MMA an integer below 2^24.
+                        // Both 16-byte halves of the row hold the same terms and the key rows carry their
+                        // weights in one half only, so the product does not depend on which half the
+                        // swizzle puts where.  Rows past the group get zeros.
+                        const int m1 = live && tok < Tg ? __float2int_rn(mx) + 1 : 0;
+                        const int a3 = m1 >> 11, a0 = m1 - (a3 << 11);
+                        const uint32_t h0 = (uint32_t)__half_as_ushort(__int2half_rn(-a0)),
+                                       h3 = (uint32_t)__half_as_ushort(__int2half_rn(-a3));
+                        const uint32_t n2048 = live && tok < Tg ? 0xE800u : 0u;  // -2048
+                        const uint4 ra = make_uint4(h0 | (n2048 << 16), n2048 | (h3 << 16), 0u, 0u);
+                        *(uint4 *)(sm + TcSmem::kAugA + row * 32) = ra;
+                        *(uint4 *)(sm + TcSmem::kAugA + row * 32 + 16) = ra;
+                        // key row `row`: (1, 2048, 2048, 2048) in the first half, zeros in the second
+                        *(uint4 *)(sm + TcSmem::kAugB + row * 32) = make_uint4(0x3C00u | (0x6800u << 16), 0x6800u | (0x6800u << 16), 0u, 0u);
+                        *(uint4 *)(sm + TcSmem::kAugB + row * 32 + 16) = make_uint4(0u, 0u, 0u, 0u);
+                        fence_async_smem();
                         __syncwarp();
-                        if (lane == 0) bar_arrive(s_free(b));
+                        if (lane == 0) bar_arrive(aug_full);
                     }
-                    if (!work) {
-                        if (pass == 2 && live) {
+                }
+                if (pass == 2) {
+                    red_sum[cq * TQ + row] = sum;
+                    if (!(ok = exchange(1))) break;
+    #pragma unroll
+                    for (int o = 1; o < NCQ; ++o) sum += red_sum[((cq + o) % NCQ) * TQ + row];
+                    rn = shiftmax_norm(sum ? sum : 1, p.smx.s_d, p.smx.m_p, p.smx.M_hw, p.smx.k_out);
+                    sh0 = (uint32_t)(rn.sh - se.k);
+                }
+                for (int kb = 0; kb < nkb; ++kb) {
+                    // warp-uniform outcome: the TMEM loads below need the whole warp
+                    ok = __all_sync(0xffffffffu, bar_wait(s_full(b), sph, abort, p.status, kStatusTimeoutMma));
+                    if (!ok) break;
+                    fence_after();
+                    // pass 3 writes P into the buffer the previous block's P V reads: that MMA must have
+                    // completed, which is waited for just before the first store, after the arithmetic
+                    bool p_ready = pass != 2;
+                    const int kvalid = min(kbk, Tg - kb * kbk);
+                    // pair: 32 columns per block, from the unit's half of the score columns
+                    const int nch = PAIR ? 32 / CW : NCH;
+    #pragma unroll 1
+                    for (int h = 0; h < nch; ++h) {
+                        const int kc = (PAIR ? 32 * cq : CPW * cq) + CW * h;  // first key of this load in the block
+                        const int c0 = PAIR ? 64 * unit + kc : kc;           // its first score column
+                        const int nvalid = kvalid - kc;  // valid columns of this load (may be <= 0 or > CW)
+                        // warp-uniform: a warp whose rows all lie past the group, or a load past the group's
+                        // keys, has nothing to compute (its P is zero, its other values unused)
+                        const bool work = live && nvalid > 0;
+                        uint32_t s[CW];
+                        tld<CW>(tlane + (uint32_t)(TKB * b + c0), s);
+                        twait<CW>(s);
+                        if (h == nch - 1) {  // the scores are in registers: the buffer is free
+                            fence_before();
+                            __syncwarp();
+                            if (lane == 0) bar_arrive(s_free(b));
+                        }
+                        if (!work) {
+                            if (pass == 2 && live) {
+                                if (!p_ready) {
+                                    p_ready = true;
+                                    ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
+                                    if (!ok) break;
+                                }
+                                uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
+                                const int k0 = (kc & 63) >> 3;
+    #pragma unroll
+                                for (int cc = 0; cc < CW / 8; ++cc) *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                            }
+                            continue;
+                        }
+                        const bool whole = nvalid >= CW;
+                        if (pass == 0) {
+                            float m = __uint_as_float(s[0]);
+    #pragma unroll
+                            for (int c = 1; c < CW; ++c) m = fmaxf(m, __uint_as_float(s[c]));
+                            if (!whole) {
+                                m = -3.0e38f;
+    #pragma unroll
+                                for (int c = 0; c < CW; ++c) m = c < nvalid ? fmaxf(m, __uint_as_float(s[c])) : m;
+                            }
+                            mx = fmaxf(mx, m);
+                        } else if (pass == 1) {
+                            uint32_t e[CW];
+    #pragma unroll
+                            for (int c = 0; c < CW; ++c) e[c] = shift_exp_nbits<FASTQ>(s[c], se);
+                            if (!whole) {
+    #pragma unroll
+                                for (int c = 0; c < CW; ++c) e[c] = c < nvalid ? e[c] : 0u;
+                            }
+                            // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits;
+                            // with SUM4 (I0 2^k < 2^30) four do
+                            uint64_t part = 0;
+                            if constexpr (SUM4) {
+    #pragma unroll
+                                for (int c = 0; c < CW; c += 4) part += (uint64_t)(e[c] + e[c + 1] + e[c + 2] + e[c + 3]);
+                            } else {
+    #pragma unroll
+                                for (int c = 0; c < CW; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
+                            }
+                            sum += part;
+                        } else {
+                            // P of the CW keys as fp16 operands: P < 1024, so its own bits are the fp16
+                            // subnormal P 2^-24, exact; O then accumulates 2^-24 P V (also exact) and is
+                            // scaled back by 2^24 when read
+                            uint32_t pw[CW];
+    #pragma unroll
+                            for (int c = 0; c < CW; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
+                            if (!whole) {
+    #pragma unroll
+                                for (int c = 0; c < CW; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
+                            }
+                            uint32_t w[CW / 2];
+    #pragma unroll
+                            for (int c = 0; c < CW / 2; ++c) w[c] = __byte_perm(pw[2 * c], pw[2 * c + 1], 0x5410);
                             if (!p_ready) {
                                 p_ready = true;
                                 ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
                                 if (!ok) break;
                             }
+                            // keys kc .. kc + CW - 1 sit in sub-tile kc / 64, chunks (kc % 64) / 8 .. of the row;
+                            // 16-byte chunk k of a row sits at k ^ (row & 7)
                             uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
                             const int k0 = (kc & 63) >> 3;
-#pragma unroll
-                            for (int cc = 0; cc < CW / 8; ++cc) *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+    #pragma unroll
+                            for (int cc = 0; cc < CW / 8; ++cc)
+                                *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) =
+                                    make_uint4(w[4 * cc], w[4 * cc + 1], w[4 * cc + 2], w[4 * cc + 3]);
                         }
-                        continue;
                     }
-                    const bool whole = nvalid >= CW;
-                    if (pass == 0) {
-                        float m = __uint_as_float(s[0]);
-#pragma unroll
-                        for (int c = 1; c < CW; ++c) m = fmaxf(m, __uint_as_float(s[c]));
-                        if (!whole) {
-                            m = -3.0e38f;
-#pragma unroll
-                            for (int c = 0; c < CW; ++c) m = c < nvalid ? fmaxf(m, __uint_as_float(s[c])) : m;
-                        }
-                        mx = fmaxf(mx, m);
-                    } else if (pass == 1) {
-                        uint32_t e[CW];
-#pragma unroll
-                        for (int c = 0; c < CW; ++c) e[c] = shift_exp_nbits<FASTQ>(s[c], se);
-                        if (!whole) {
-#pragma unroll
-                            for (int c = 0; c < CW; ++c) e[c] = c < nvalid ? e[c] : 0u;
-                        }
-                        // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits;
-                        // with SUM4 (I0 2^k < 2^30) four do
-                        uint64_t part = 0;
-                        if constexpr (SUM4) {
-#pragma unroll
-                            for (int c = 0; c < CW; c += 4) part += (uint64_t)(e[c] + e[c + 1] + e[c + 2] + e[c + 3]);
-                        } else {
-#pragma unroll
-                            for (int c = 0; c < CW; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
-                        }
-                        sum += part;
-                    } else {
-                        // P of the CW keys as fp16 operands: P < 1024, so its own bits are the fp16
-                        // subnormal P 2^-24, exact; O then accumulates 2^-24 P V (also exact) and is
-                        // scaled back by 2^24 when read
-                        uint32_t pw[CW];
-#pragma unroll
-                        for (int c = 0; c < CW; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
-                        if (!whole) {
-#pragma unroll
-                            for (int c = 0; c < CW; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
-                        }
-                        uint32_t w[CW / 2];
-#pragma unroll
-                        for (int c = 0; c < CW / 2; ++c) w[c] = __byte_perm(pw[2 * c], pw[2 * c + 1], 0x5410);
+                    if (pass == 2) sph ^= 1u;  // pass 3: S[0] alone
+                    else if (++b == NS) {
+                        b = 0;
+                        sph ^= 1u;
+                    }
+                    if (pass == 2) {
+                        // every warp (also one that stored nothing) arrives for this block only after the
+                        // previous block's P V completed, so arrivals never run a phase ahead
                         if (!p_ready) {
                             p_ready = true;
                             ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
                             if (!ok) break;
                         }
-                        // keys kc .. kc + CW - 1 sit in sub-tile kc / 64, chunks (kc % 64) / 8 .. of the row;
-                        // 16-byte chunk k of a row sits at k ^ (row & 7)
-                        uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
-                        const int k0 = (kc & 63) >> 3;
-#pragma unroll
-                        for (int cc = 0; cc < CW / 8; ++cc)
-                            *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) =
-                                make_uint4(w[4 * cc], w[4 * cc + 1], w[4 * cc + 2], w[4 * cc + 3]);
-                    }
-                }
-                if (pass == 2) sph ^= 1u;  // pass 3: S[0] alone
-                else if (++b == NS) {
-                    b = 0;
-                    sph ^= 1u;
-                }
-                if (pass == 2) {
-                    // every warp (also one that stored nothing) arrives for this block only after the
-                    // previous block's P V completed, so arrivals never run a phase ahead
-                    if (!p_ready) {
-                        p_ready = true;
-                        ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
-                        if (!ok) break;
-                    }
-                    fence_async_smem();
-                    __syncwarp();
-                    if (lane == 0) bar_arrive(p_full(pb));
-                    if (++pb == NPB) {
-                        pb = 0;
-                        pph ^= 1u;
+                        fence_async_smem();
+                        __syncwarp();
+                        if (lane == 0) bar_arrive(p_full(pb));
+                        if (++pb == NPB) {
+                            pb = 0;
+                            pph ^= 1u;
+                        }
                     }
                 }
             }
-        }
-        // ---- O = P V from TMEM: sat8(rq(O; m_o, s_o)) at the token's own position (OPW columns)
-        if (ok) ok = __all_sync(0xffffffffu, bar_wait(o_full, 0, abort, p.status, kStatusTimeoutMma));
-        if (ok) {
-            fence_after();
-            uint32_t o[OPW];
-            tld<OPW>(tlane + kOcol + (uint32_t)(64 * unit + OPW * cq), o);
-            twait<OPW>(o);
-            if (live && tok < Tg) {
-                int32_t r[OPW];
-#pragma unroll
-                for (int c = 0; c < OPW; ++c)
-                    r[c] = sat8(rq(__float2int_rn(__uint_as_float(o[c]) * 16777216.0f), p.m_o, p.s_o));  // O = 2^24 acc
-                const int64_t t = unit ? base1 + tok : gr.token(tok);
-                const int ho = unit ? hoff1 : hoff;
-                if (p.o_f16) {
-                    // 1152 + r (|r| <= 127) has the fp16 bits 0x6480 + r; subtracting 1152 leaves r
-                    const __half2 h1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
-                    uint32_t hw[OPW / 2];
-#pragma unroll
-                    for (int c = 0; c < OPW / 2; ++c) {
-                        uint32_t x = (uint32_t)(0x6480 + r[2 * c]) | ((uint32_t)(0x6480 + r[2 * c + 1]) << 16);
-                        __half2 hh = __hsub2(*reinterpret_cast<__half2 *>(&x), h1152);
-                        hw[c] = *reinterpret_cast<uint32_t *>(&hh);
+            // ---- O = P V from TMEM: sat8(rq(O; m_o, s_o)) at the token's own position (OPW columns)
+            if (ok) ok = __all_sync(0xffffffffu, bar_wait(o_full, 0, abort, p.status, kStatusTimeoutMma));
+            if (ok) {
+                fence_after();
+                uint32_t o[OPW];
+                tld<OPW>(tlane + kOcol + (uint32_t)(64 * unit + OPW * cq), o);
+                twait<OPW>(o);
+                if (live && tok < Tg) {
+                    int32_t r[OPW];
+    #pragma unroll
+                    for (int c = 0; c < OPW; ++c)
+                        r[c] = sat8(rq(__float2int_rn(__uint_as_float(o[c]) * 16777216.0f), p.m_o, p.s_o));  // O = 2^24 acc
+                    const int64_t t = unit ? base1 + tok : gr.token(tok);
+                    const int ho = unit ? hoff1 : hoff;
+                    if (p.o_f16) {
+                        // 1152 + r (|r| <= 127) has the fp16 bits 0x6480 + r; subtracting 1152 leaves r
+                        const __half2 h1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
+                        uint32_t hw[OPW / 2];
+    #pragma unroll
+                        for (int c = 0; c < OPW / 2; ++c) {
+                            uint32_t x = (uint32_t)(0x6480 + r[2 * c]) | ((uint32_t)(0x6480 + r[2 * c + 1]) << 16);
+                            __half2 hh = __hsub2(*reinterpret_cast<__half2 *>(&x), h1152);
+                            hw[c] = *reinterpret_cast<uint32_t *>(&hh);
+                        }
+                        uint4 *dst = (uint4 *)((__half *)p.O + t * p.ld_o + ho + OPW * cq);
+    #pragma unroll
+                        for (int c = 0; c < OPW / 8; ++c) dst[c] = make_uint4(hw[4 * c], hw[4 * c + 1], hw[4 * c + 2], hw[4 * c + 3]);
+                    } else {
+                        uint32_t bw[OPW / 4];
+    #pragma unroll
+                        for (int c = 0; c < OPW / 4; ++c)
+                            bw[c] = (uint32_t)(uint8_t)r[4 * c] | ((uint32_t)(uint8_t)r[4 * c + 1] << 8) |
+                                    ((uint32_t)(uint8_t)r[4 * c + 2] << 16) | ((uint32_t)(uint8_t)r[4 * c + 3] << 24);
+                        uint4 *dst = (uint4 *)((int8_t *)p.O + t * p.ld_o + ho + OPW * cq);
+    #pragma unroll
+                        for (int c = 0; c < OPW / 16; ++c) dst[c] = make_uint4(bw[4 * c], bw[4 * c + 1], bw[4 * c + 2], bw[4 * c + 3]);
                     }
-                    uint4 *dst = (uint4 *)((__half *)p.O + t * p.ld_o + ho + OPW * cq);
-#pragma unroll
-                    for (int c = 0; c < OPW / 8; ++c) dst[c] = make_uint4(hw[4 * c], hw[4 * c + 1], hw[4 * c + 2], hw[4 * c + 3]);
-                } else {
-                    uint32_t bw[OPW / 4];
-#pragma unroll
-                    for (int c = 0; c < OPW / 4; ++c)
-                        bw[c] = (uint32_t)(uint8_t)r[4 * c] | ((uint32_t)(uint8_t)r[4 * c + 1] << 8) |
-                                ((uint32_t)(uint8_t)r[4 * c + 2] << 16) | ((uint32_t)(uint8_t)r[4 * c + 3] << 24);
-                    uint4 *dst = (uint4 *)((int8_t *)p.O + t * p.ld_o + ho + OPW * cq);
-#pragma unroll
-                    for (int c = 0; c < OPW / 16; ++c) dst[c] = make_uint4(bw[4 * c], bw[4 * c + 1], bw[4 * c + 2], bw[4 * c + 3]);
                 }
             }
-        }
+        };
+        if constexpr (MAYPAIR) softmax(RuntimeForm{pair});
+        else softmax(FixedForm<false>{});
     }
 
     fence_before();
@@ -810,17 +827,22 @@ bool kv_map(CUtensorMap *m, const void *base, const AttnParams &p, bool win, int
 }
 
 // One instantiation's launch; its shared-memory limit is raised once.
-template <bool FASTQ, bool DIRECT, bool SUM4>
-cudaError_t launch_tc_kernel(const TcArgs &a, dim3 grid, size_t smem, cudaStream_t s) {
+template <bool FASTQ, bool DIRECT, bool SUM4, bool MAYPAIR>
+cudaError_t launch_tc_one(const TcArgs &a, dim3 grid, size_t smem, cudaStream_t s) {
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;
     std::call_once(once, [&] {
-        attr = cudaFuncSetAttribute(attn_tc_kernel<FASTQ, DIRECT, SUM4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)smem);
+        attr = cudaFuncSetAttribute(attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     });
     if (attr != cudaSuccess) return attr;
-    attn_tc_kernel<FASTQ, DIRECT, SUM4><<<grid, kThreadsTc, smem, s>>>(a);
+    attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR><<<grid, kThreadsTc, smem, s>>>(a);
     return cudaGetLastError();
+}
+template <bool FASTQ, bool DIRECT, bool SUM4>
+cudaError_t launch_tc_kernel(const TcArgs &a, dim3 grid, size_t smem, cudaStream_t s) {
+    return a.pair ? launch_tc_one<FASTQ, DIRECT, SUM4, true>(a, grid, smem, s)
+                  : launch_tc_one<FASTQ, DIRECT, SUM4, false>(a, grid, smem, s);
 }
 
 }  // namespace
