@@ -55,6 +55,7 @@ namespace {
 template <bool B> struct FixedForm {
     __device__ constexpr bool operator()() const { return B; }
 };
+template <int P> struct PassTag { static constexpr int value = P; };
 struct RuntimeForm {
     bool pair;
     __device__ bool operator()() const { return pair; }
@@ -572,11 +573,138 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             };
             int b = 0, pb = 0;  // S and P buffers of the next block, with their phase bits
             uint32_t sph = 0, pph = 0;
-            for (int pass = 0; pass < 3 && ok; ++pass) {
-                if (pass == 1) {
+            // the three passes over the key blocks, each compiled for its own pass
+            auto run_pass = [&](auto pass_tag) {
+                constexpr int pass = decltype(pass_tag)::value;
+                for (int kb = 0; kb < nkb; ++kb) {
+                        // warp-uniform outcome: the TMEM loads below need the whole warp
+                        ok = __all_sync(0xffffffffu, bar_wait(s_full(b), sph, abort, p.status, kStatusTimeoutMma));
+                        if (!ok) break;
+                        fence_after();
+                        // pass 3 writes P into the buffer the previous block's P V reads: that MMA must have
+                        // completed, which is waited for just before the first store, after the arithmetic
+                        bool p_ready = pass != 2;
+                        const int kvalid = min(kbk, Tg - kb * kbk);
+                        // pair: 32 columns per block, from the unit's half of the score columns
+                        const int nch = PAIR ? 32 / CW : NCH;
+    #pragma unroll 1
+                        for (int h = 0; h < nch; ++h) {
+                            const int kc = (PAIR ? 32 * cq : CPW * cq) + CW * h;  // first key of this load in the block
+                            const int c0 = PAIR ? 64 * unit + kc : kc;           // its first score column
+                            const int nvalid = kvalid - kc;  // valid columns of this load (may be <= 0 or > CW)
+                            // warp-uniform: a warp whose rows all lie past the group, or a load past the group's
+                            // keys, has nothing to compute (its P is zero, its other values unused)
+                            const bool work = live && nvalid > 0;
+                            uint32_t s[CW];
+                            tld<CW>(tlane + (uint32_t)(TKB * b + c0), s);
+                            twait<CW>(s);
+                            if (h == nch - 1) {  // the scores are in registers: the buffer is free
+                                fence_before();
+                                __syncwarp();
+                                if (lane == 0) bar_arrive(s_free(b));
+                            }
+                            if (!work) {
+                                if (pass == 2 && live) {
+                                    if (!p_ready) {
+                                        p_ready = true;
+                                        ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
+                                        if (!ok) break;
+                                    }
+                                    uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
+                                    const int k0 = (kc & 63) >> 3;
+    #pragma unroll
+                                    for (int cc = 0; cc < CW / 8; ++cc) *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+                                }
+                                continue;
+                            }
+                            const bool whole = nvalid >= CW;
+                            if (pass == 0) {
+                                float m = __uint_as_float(s[0]);
+    #pragma unroll
+                                for (int c = 1; c < CW; ++c) m = fmaxf(m, __uint_as_float(s[c]));
+                                if (!whole) {
+                                    m = -3.0e38f;
+    #pragma unroll
+                                    for (int c = 0; c < CW; ++c) m = c < nvalid ? fmaxf(m, __uint_as_float(s[c])) : m;
+                                }
+                                mx = fmaxf(mx, m);
+                            } else if (pass == 1) {
+                                uint32_t e[CW];
+    #pragma unroll
+                                for (int c = 0; c < CW; ++c) e[c] = shift_exp_nbits<FASTQ>(s[c], se);
+                                if (!whole) {
+    #pragma unroll
+                                    for (int c = 0; c < CW; ++c) e[c] = c < nvalid ? e[c] : 0u;
+                                }
+                                // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits;
+                                // with SUM4 (I0 2^k < 2^30) four do
+                                uint64_t part = 0;
+                                if constexpr (SUM4) {
+    #pragma unroll
+                                    for (int c = 0; c < CW; c += 4) part += (uint64_t)(e[c] + e[c + 1] + e[c + 2] + e[c + 3]);
+                                } else {
+    #pragma unroll
+                                    for (int c = 0; c < CW; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
+                                }
+                                sum += part;
+                            } else {
+                                // P of the CW keys as fp16 operands: P < 1024, so its own bits are the fp16
+                                // subnormal P 2^-24, exact; O then accumulates 2^-24 P V (also exact) and is
+                                // scaled back by 2^24 when read
+                                uint32_t pw[CW];
+    #pragma unroll
+                                for (int c = 0; c < CW; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
+                                if (!whole) {
+    #pragma unroll
+                                    for (int c = 0; c < CW; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
+                                }
+                                uint32_t w[CW / 2];
+    #pragma unroll
+                                for (int c = 0; c < CW / 2; ++c) w[c] = __byte_perm(pw[2 * c], pw[2 * c + 1], 0x5410);
+                                if (!p_ready) {
+                                    p_ready = true;
+                                    ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
+                                    if (!ok) break;
+                                }
+                                // keys kc .. kc + CW - 1 sit in sub-tile kc / 64, chunks (kc % 64) / 8 .. of the row;
+                                // 16-byte chunk k of a row sits at k ^ (row & 7)
+                                uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
+                                const int k0 = (kc & 63) >> 3;
+    #pragma unroll
+                                for (int cc = 0; cc < CW / 8; ++cc)
+                                    *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) =
+                                        make_uint4(w[4 * cc], w[4 * cc + 1], w[4 * cc + 2], w[4 * cc + 3]);
+                            }
+                        }
+                        if (pass == 2) sph ^= 1u;  // pass 3: S[0] alone
+                        else if (++b == NS) {
+                            b = 0;
+                            sph ^= 1u;
+                        }
+                        if (pass == 2) {
+                            // every warp (also one that stored nothing) arrives for this block only after the
+                            // previous block's P V completed, so arrivals never run a phase ahead
+                            if (!p_ready) {
+                                p_ready = true;
+                                ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
+                                if (!ok) break;
+                            }
+                            fence_async_smem();
+                            __syncwarp();
+                            if (lane == 0) bar_arrive(p_full(pb));
+                            if (++pb == NPB) {
+                                pb = 0;
+                                pph ^= 1u;
+                            }
+                        }
+                    }
+            };
+            run_pass(PassTag<0>{});
+            do {  // pass 2 prologue: the row maxima meet; the constant-term rows
+                if (!ok) break;
                     red_max[cq * TQ + row] = mx;
                     if (!(ok = exchange(0))) break;
-    #pragma unroll
+#pragma unroll
                     for (int o = 1; o < NCQ; ++o) mx = fmaxf(mx, red_max[((cq + o) % NCQ) * TQ + row]);
                     if (cq == 0) {
                         // this row's constant term -(2^23 + max + 1) as fp16 terms against the key weights
@@ -600,138 +728,18 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                         __syncwarp();
                         if (lane == 0) bar_arrive(aug_full);
                     }
-                }
-                if (pass == 2) {
+            } while (0);
+            if (ok) run_pass(PassTag<1>{});
+            do {  // pass 3 prologue: the row sums meet; s_d and F
+                if (!ok) break;
                     red_sum[cq * TQ + row] = sum;
                     if (!(ok = exchange(1))) break;
-    #pragma unroll
+#pragma unroll
                     for (int o = 1; o < NCQ; ++o) sum += red_sum[((cq + o) % NCQ) * TQ + row];
                     rn = shiftmax_norm(sum ? sum : 1, p.smx.s_d, p.smx.m_p, p.smx.M_hw, p.smx.k_out);
                     sh0 = (uint32_t)(rn.sh - se.k);
-                }
-                for (int kb = 0; kb < nkb; ++kb) {
-                    // warp-uniform outcome: the TMEM loads below need the whole warp
-                    ok = __all_sync(0xffffffffu, bar_wait(s_full(b), sph, abort, p.status, kStatusTimeoutMma));
-                    if (!ok) break;
-                    fence_after();
-                    // pass 3 writes P into the buffer the previous block's P V reads: that MMA must have
-                    // completed, which is waited for just before the first store, after the arithmetic
-                    bool p_ready = pass != 2;
-                    const int kvalid = min(kbk, Tg - kb * kbk);
-                    // pair: 32 columns per block, from the unit's half of the score columns
-                    const int nch = PAIR ? 32 / CW : NCH;
-    #pragma unroll 1
-                    for (int h = 0; h < nch; ++h) {
-                        const int kc = (PAIR ? 32 * cq : CPW * cq) + CW * h;  // first key of this load in the block
-                        const int c0 = PAIR ? 64 * unit + kc : kc;           // its first score column
-                        const int nvalid = kvalid - kc;  // valid columns of this load (may be <= 0 or > CW)
-                        // warp-uniform: a warp whose rows all lie past the group, or a load past the group's
-                        // keys, has nothing to compute (its P is zero, its other values unused)
-                        const bool work = live && nvalid > 0;
-                        uint32_t s[CW];
-                        tld<CW>(tlane + (uint32_t)(TKB * b + c0), s);
-                        twait<CW>(s);
-                        if (h == nch - 1) {  // the scores are in registers: the buffer is free
-                            fence_before();
-                            __syncwarp();
-                            if (lane == 0) bar_arrive(s_free(b));
-                        }
-                        if (!work) {
-                            if (pass == 2 && live) {
-                                if (!p_ready) {
-                                    p_ready = true;
-                                    ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
-                                    if (!ok) break;
-                                }
-                                uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
-                                const int k0 = (kc & 63) >> 3;
-    #pragma unroll
-                                for (int cc = 0; cc < CW / 8; ++cc) *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
-                            }
-                            continue;
-                        }
-                        const bool whole = nvalid >= CW;
-                        if (pass == 0) {
-                            float m = __uint_as_float(s[0]);
-    #pragma unroll
-                            for (int c = 1; c < CW; ++c) m = fmaxf(m, __uint_as_float(s[c]));
-                            if (!whole) {
-                                m = -3.0e38f;
-    #pragma unroll
-                                for (int c = 0; c < CW; ++c) m = c < nvalid ? fmaxf(m, __uint_as_float(s[c])) : m;
-                            }
-                            mx = fmaxf(mx, m);
-                        } else if (pass == 1) {
-                            uint32_t e[CW];
-    #pragma unroll
-                            for (int c = 0; c < CW; ++c) e[c] = shift_exp_nbits<FASTQ>(s[c], se);
-                            if (!whole) {
-    #pragma unroll
-                                for (int c = 0; c < CW; ++c) e[c] = c < nvalid ? e[c] : 0u;
-                            }
-                            // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits;
-                            // with SUM4 (I0 2^k < 2^30) four do
-                            uint64_t part = 0;
-                            if constexpr (SUM4) {
-    #pragma unroll
-                                for (int c = 0; c < CW; c += 4) part += (uint64_t)(e[c] + e[c + 1] + e[c + 2] + e[c + 3]);
-                            } else {
-    #pragma unroll
-                                for (int c = 0; c < CW; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
-                            }
-                            sum += part;
-                        } else {
-                            // P of the CW keys as fp16 operands: P < 1024, so its own bits are the fp16
-                            // subnormal P 2^-24, exact; O then accumulates 2^-24 P V (also exact) and is
-                            // scaled back by 2^24 when read
-                            uint32_t pw[CW];
-    #pragma unroll
-                            for (int c = 0; c < CW; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
-                            if (!whole) {
-    #pragma unroll
-                                for (int c = 0; c < CW; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
-                            }
-                            uint32_t w[CW / 2];
-    #pragma unroll
-                            for (int c = 0; c < CW / 2; ++c) w[c] = __byte_perm(pw[2 * c], pw[2 * c + 1], 0x5410);
-                            if (!p_ready) {
-                                p_ready = true;
-                                ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
-                                if (!ok) break;
-                            }
-                            // keys kc .. kc + CW - 1 sit in sub-tile kc / 64, chunks (kc % 64) / 8 .. of the row;
-                            // 16-byte chunk k of a row sits at k ^ (row & 7)
-                            uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
-                            const int k0 = (kc & 63) >> 3;
-    #pragma unroll
-                            for (int cc = 0; cc < CW / 8; ++cc)
-                                *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) =
-                                    make_uint4(w[4 * cc], w[4 * cc + 1], w[4 * cc + 2], w[4 * cc + 3]);
-                        }
-                    }
-                    if (pass == 2) sph ^= 1u;  // pass 3: S[0] alone
-                    else if (++b == NS) {
-                        b = 0;
-                        sph ^= 1u;
-                    }
-                    if (pass == 2) {
-                        // every warp (also one that stored nothing) arrives for this block only after the
-                        // previous block's P V completed, so arrivals never run a phase ahead
-                        if (!p_ready) {
-                            p_ready = true;
-                            ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
-                            if (!ok) break;
-                        }
-                        fence_async_smem();
-                        __syncwarp();
-                        if (lane == 0) bar_arrive(p_full(pb));
-                        if (++pb == NPB) {
-                            pb = 0;
-                            pph ^= 1u;
-                        }
-                    }
-                }
-            }
+            } while (0);
+            if (ok) run_pass(PassTag<2>{});
             // ---- O = P V from TMEM: sat8(rq(O; m_o, s_o)) at the token's own position (OPW columns)
             if (ok) ok = __all_sync(0xffffffffu, bar_wait(o_full, 0, abort, p.status, kStatusTimeoutMma));
             if (ok) {
@@ -741,7 +749,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                 twait<OPW>(o);
                 if (live && tok < Tg) {
                     int32_t r[OPW];
-    #pragma unroll
+#pragma unroll
                     for (int c = 0; c < OPW; ++c)
                         r[c] = sat8(rq(__float2int_rn(__uint_as_float(o[c]) * 16777216.0f), p.m_o, p.s_o));  // O = 2^24 acc
                     const int64_t t = unit ? base1 + tok : gr.token(tok);
@@ -750,23 +758,23 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                         // 1152 + r (|r| <= 127) has the fp16 bits 0x6480 + r; subtracting 1152 leaves r
                         const __half2 h1152 = __half2half2(__ushort_as_half((unsigned short)0x6480));
                         uint32_t hw[OPW / 2];
-    #pragma unroll
+#pragma unroll
                         for (int c = 0; c < OPW / 2; ++c) {
                             uint32_t x = (uint32_t)(0x6480 + r[2 * c]) | ((uint32_t)(0x6480 + r[2 * c + 1]) << 16);
                             __half2 hh = __hsub2(*reinterpret_cast<__half2 *>(&x), h1152);
                             hw[c] = *reinterpret_cast<uint32_t *>(&hh);
                         }
                         uint4 *dst = (uint4 *)((__half *)p.O + t * p.ld_o + ho + OPW * cq);
-    #pragma unroll
+#pragma unroll
                         for (int c = 0; c < OPW / 8; ++c) dst[c] = make_uint4(hw[4 * c], hw[4 * c + 1], hw[4 * c + 2], hw[4 * c + 3]);
                     } else {
                         uint32_t bw[OPW / 4];
-    #pragma unroll
+#pragma unroll
                         for (int c = 0; c < OPW / 4; ++c)
                             bw[c] = (uint32_t)(uint8_t)r[4 * c] | ((uint32_t)(uint8_t)r[4 * c + 1] << 8) |
                                     ((uint32_t)(uint8_t)r[4 * c + 2] << 16) | ((uint32_t)(uint8_t)r[4 * c + 3] << 24);
                         uint4 *dst = (uint4 *)((int8_t *)p.O + t * p.ld_o + ho + OPW * cq);
-    #pragma unroll
+#pragma unroll
                         for (int c = 0; c < OPW / 16; ++c) dst[c] = make_uint4(bw[4 * c], bw[4 * c + 1], bw[4 * c + 2], bw[4 * c + 3]);
                     }
                 }
