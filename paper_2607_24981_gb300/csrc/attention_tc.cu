@@ -56,6 +56,7 @@ template <bool B> struct FixedForm {
     __device__ constexpr bool operator()() const { return B; }
 };
 template <int P> struct PassTag { static constexpr int value = P; };
+template <bool B> struct BoolTag { static constexpr bool value = B; };
 struct RuntimeForm {
     bool pair;
     __device__ bool operator()() const { return pair; }
@@ -265,8 +266,9 @@ __device__ __forceinline__ uint32_t p_of(uint32_t w, const ShiftExpC &se, const 
 // DIRECT: per-row s_d with I_b F < 2^32 (the host's condition), so P comes straight from ShiftExp's
 // parts; otherwise P = (I_exp F) >> sh from the 64-bit product.  SUM4: every ShiftExp value is below
 // 2^30 (I0 2^k_inter < 2^30, the host's condition), so four of them add up in 32 bits.
-// MAYPAIR: the launch may hold paired last tiles (args.pair).
-template <bool FASTQ, bool DIRECT, bool SUM4, bool MAYPAIR>
+// MAYPAIR: the launch may hold paired last tiles (args.pair).  MAYFULL: key blocks of 128 tokens
+// (global attention), whose full blocks are compiled without the masking of partial ones.
+template <bool FASTQ, bool DIRECT, bool SUM4, bool MAYPAIR, bool MAYFULL>
 __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const __grid_constant__ TcArgs args) {
     const AttnParams &p = args.p;
     extern __shared__ uint8_t smem_raw[];
@@ -576,10 +578,13 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             // the three passes over the key blocks, each compiled for its own pass
             auto run_pass = [&](auto pass_tag) {
                 constexpr int pass = decltype(pass_tag)::value;
-                for (int kb = 0; kb < nkb; ++kb) {
+                // one key block; FULL: the warp is live and every chunk of the block is whole (compiled
+                // without the masking)
+                auto block = [&](int kb, auto full_tag) -> bool {
+                    constexpr bool FULL = decltype(full_tag)::value;
                         // warp-uniform outcome: the TMEM loads below need the whole warp
                         ok = __all_sync(0xffffffffu, bar_wait(s_full(b), sph, abort, p.status, kStatusTimeoutMma));
-                        if (!ok) break;
+                        if (!ok) return false;
                         fence_after();
                         // pass 3 writes P into the buffer the previous block's P V reads: that MMA must have
                         // completed, which is waited for just before the first store, after the arithmetic
@@ -587,14 +592,14 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                         const int kvalid = min(kbk, Tg - kb * kbk);
                         // pair: 32 columns per block, from the unit's half of the score columns
                         const int nch = PAIR ? 32 / CW : NCH;
-    #pragma unroll 1
+#pragma unroll 1
                         for (int h = 0; h < nch; ++h) {
                             const int kc = (PAIR ? 32 * cq : CPW * cq) + CW * h;  // first key of this load in the block
                             const int c0 = PAIR ? 64 * unit + kc : kc;           // its first score column
                             const int nvalid = kvalid - kc;  // valid columns of this load (may be <= 0 or > CW)
                             // warp-uniform: a warp whose rows all lie past the group, or a load past the group's
                             // keys, has nothing to compute (its P is zero, its other values unused)
-                            const bool work = live && nvalid > 0;
+                            const bool work = FULL || (live && nvalid > 0);
                             uint32_t s[CW];
                             tld<CW>(tlane + (uint32_t)(TKB * b + c0), s);
                             twait<CW>(s);
@@ -612,38 +617,38 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                                     }
                                     uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
                                     const int k0 = (kc & 63) >> 3;
-    #pragma unroll
+#pragma unroll
                                     for (int cc = 0; cc < CW / 8; ++cc) *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
                                 }
                                 continue;
                             }
-                            const bool whole = nvalid >= CW;
+                            const bool whole = FULL || nvalid >= CW;
                             if (pass == 0) {
                                 float m = __uint_as_float(s[0]);
-    #pragma unroll
+#pragma unroll
                                 for (int c = 1; c < CW; ++c) m = fmaxf(m, __uint_as_float(s[c]));
                                 if (!whole) {
                                     m = -3.0e38f;
-    #pragma unroll
+#pragma unroll
                                     for (int c = 0; c < CW; ++c) m = c < nvalid ? fmaxf(m, __uint_as_float(s[c])) : m;
                                 }
                                 mx = fmaxf(mx, m);
                             } else if (pass == 1) {
                                 uint32_t e[CW];
-    #pragma unroll
+#pragma unroll
                                 for (int c = 0; c < CW; ++c) e[c] = shift_exp_nbits<FASTQ>(s[c], se);
                                 if (!whole) {
-    #pragma unroll
+#pragma unroll
                                     for (int c = 0; c < CW; ++c) e[c] = c < nvalid ? e[c] : 0u;
                                 }
                                 // I0 2^k < 2^31 (checked by the host), so a pair of ShiftExp values fits in 32 bits;
                                 // with SUM4 (I0 2^k < 2^30) four do
                                 uint64_t part = 0;
                                 if constexpr (SUM4) {
-    #pragma unroll
+#pragma unroll
                                     for (int c = 0; c < CW; c += 4) part += (uint64_t)(e[c] + e[c + 1] + e[c + 2] + e[c + 3]);
                                 } else {
-    #pragma unroll
+#pragma unroll
                                     for (int c = 0; c < CW; c += 2) part += (uint64_t)(e[c] + e[c + 1]);
                                 }
                                 sum += part;
@@ -652,14 +657,14 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                                 // subnormal P 2^-24, exact; O then accumulates 2^-24 P V (also exact) and is
                                 // scaled back by 2^24 when read
                                 uint32_t pw[CW];
-    #pragma unroll
+#pragma unroll
                                 for (int c = 0; c < CW; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
                                 if (!whole) {
-    #pragma unroll
+#pragma unroll
                                     for (int c = 0; c < CW; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
                                 }
                                 uint32_t w[CW / 2];
-    #pragma unroll
+#pragma unroll
                                 for (int c = 0; c < CW / 2; ++c) w[c] = __byte_perm(pw[2 * c], pw[2 * c + 1], 0x5410);
                                 if (!p_ready) {
                                     p_ready = true;
@@ -670,7 +675,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                                 // 16-byte chunk k of a row sits at k ^ (row & 7)
                                 uint8_t *prow = sm + TcSmem::kP + pb * kPB + (kc >> 6) * (TQ * 128) + row * 128;
                                 const int k0 = (kc & 63) >> 3;
-    #pragma unroll
+#pragma unroll
                                 for (int cc = 0; cc < CW / 8; ++cc)
                                     *(uint4 *)(prow + (((k0 + cc) ^ (row & 7)) << 4)) =
                                         make_uint4(w[4 * cc], w[4 * cc + 1], w[4 * cc + 2], w[4 * cc + 3]);
@@ -687,7 +692,7 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                             if (!p_ready) {
                                 p_ready = true;
                                 ok = __all_sync(0xffffffffu, bar_wait(p_free(pb), pph ^ 1u, abort, p.status, kStatusTimeoutMma));
-                                if (!ok) break;
+                                if (!ok) return false;
                             }
                             fence_async_smem();
                             __syncwarp();
@@ -697,7 +702,16 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                                 pph ^= 1u;
                             }
                         }
-                    }
+                                        return true;
+                };
+                if constexpr (MAYFULL) {
+                    const int nfull = live && kbk % CW == 0 ? Tg / kbk : 0;
+                    for (int kb = 0; kb < nkb; ++kb)
+                        if (!(kb < nfull ? block(kb, BoolTag<true>{}) : block(kb, BoolTag<false>{}))) break;
+                } else {
+                    for (int kb = 0; kb < nkb; ++kb)
+                        if (!block(kb, BoolTag<false>{})) break;
+                }
             };
             run_pass(PassTag<0>{});
             do {  // pass 2 prologue: the row maxima meet; the constant-term rows
@@ -835,22 +849,25 @@ bool kv_map(CUtensorMap *m, const void *base, const AttnParams &p, bool win, int
 }
 
 // One instantiation's launch; its shared-memory limit is raised once.
-template <bool FASTQ, bool DIRECT, bool SUM4, bool MAYPAIR>
+template <bool FASTQ, bool DIRECT, bool SUM4, bool MAYPAIR, bool MAYFULL>
 cudaError_t launch_tc_one(const TcArgs &a, dim3 grid, size_t smem, cudaStream_t s) {
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;
     std::call_once(once, [&] {
-        attr = cudaFuncSetAttribute(attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR>,
+        attr = cudaFuncSetAttribute(attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR, MAYFULL>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     });
     if (attr != cudaSuccess) return attr;
-    attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR><<<grid, kThreadsTc, smem, s>>>(a);
+    attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR, MAYFULL><<<grid, kThreadsTc, smem, s>>>(a);
     return cudaGetLastError();
 }
+// windows: one form; global attention: full blocks compiled apart, and paired last tiles when the
+// last tile has at most 64 queries
 template <bool FASTQ, bool DIRECT, bool SUM4>
 cudaError_t launch_tc_kernel(const TcArgs &a, dim3 grid, size_t smem, cudaStream_t s) {
-    return a.pair ? launch_tc_one<FASTQ, DIRECT, SUM4, true>(a, grid, smem, s)
-                  : launch_tc_one<FASTQ, DIRECT, SUM4, false>(a, grid, smem, s);
+    if (a.win) return launch_tc_one<FASTQ, DIRECT, SUM4, false, false>(a, grid, smem, s);
+    return a.pair ? launch_tc_one<FASTQ, DIRECT, SUM4, true, true>(a, grid, smem, s)
+                  : launch_tc_one<FASTQ, DIRECT, SUM4, false, true>(a, grid, smem, s);
 }
 
 }  // namespace
