@@ -116,7 +116,18 @@ __global__ void __launch_bounds__(256) shiftmax_rows_vec(const int32_t *__restri
     const RowOut ro = row_out(rn);
     uint32_t *pr = (uint32_t *)(P + row * ldp);
     // every output is below 2^k_out <= 256: the four bytes of a chunk by two byte permutations
-    if (ro.ok) {
+    if (ro.ok && ro.rs == 0) {  // sh <= 32: one high-word product per output
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) {
+            const int ch = sub + LANES * j;
+            if (ch < nch) {
+                const uint32_t *e = (const uint32_t *)&v[j];
+                const uint32_t b01 = __byte_perm(__umulhi(e[0], ro.Fs), __umulhi(e[1], ro.Fs), 0x0040);
+                const uint32_t b23 = __byte_perm(__umulhi(e[2], ro.Fs), __umulhi(e[3], ro.Fs), 0x0040);
+                __stcs(pr + ch, __byte_perm(b01, b23, 0x5410));
+            }
+        }
+    } else if (ro.ok) {
 #pragma unroll
         for (int j = 0; j < NCH; ++j) {
             const int ch = sub + LANES * j;
