@@ -248,6 +248,18 @@ __device__ __forceinline__ uint32_t p_direct(uint32_t w, const ShiftExpC &c, uin
     return shr_clamp(Ib * F, sh0 + q);
 }
 
+// The same P as one high-word product: floor(I_b F / 2^(sh0 + q)) = umulhi(I_b, G) >> q with
+// G = F 2^(32 - sh0) when sh0 <= 32 and F < 2^sh0 (floors compose), and G = 0 when sh0 > 32 (then
+// I_b F < 2^32 <= 2^sh0 and every P is 0).  q <= k_inter < 32.
+template <bool FASTQ>
+__device__ __forceinline__ uint32_t p_direct_hi(uint32_t w, const ShiftExpC &c, uint32_t G) {
+    uint32_t n = exp_arg_from_neg_bits(w);
+    n = min(n, (uint32_t)c.kI0);
+    const uint32_t q = FASTQ ? __umulhi(n, c.m32) : (__umulhi(n, c.m_lo) + n * c.m_hi) >> 8;
+    const uint32_t Ib = ((q + 2u) * (uint32_t)c.I0 - n) >> 1;
+    return __umulhi(Ib, G) >> q;
+}
+
 struct GroupTc {
     int64_t base;
     int32_t Tg, nw, ws, gs, wy, wx;
@@ -566,7 +578,8 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
             float mx = -3.0e38f;
             uint64_t sum = 0;
             RowNorm rn{};
-            uint32_t sh0 = 0;
+            uint32_t sh0 = 0, hiG = 0;
+            bool hi_form = false;
             // the other column groups' contributions to the row, through shared memory and the xchg barrier
             auto exchange = [&](int phase) -> bool {
                 __syncwarp();
@@ -657,8 +670,13 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                                 // subnormal P 2^-24, exact; O then accumulates 2^-24 P V (also exact) and is
                                 // scaled back by 2^24 when read
                                 uint32_t pw[CW];
+                                if (DIRECT && hi_form) {
 #pragma unroll
-                                for (int c = 0; c < CW; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
+                                    for (int c = 0; c < CW; ++c) pw[c] = p_direct_hi<FASTQ>(s[c], se, hiG);
+                                } else {
+#pragma unroll
+                                    for (int c = 0; c < CW; ++c) pw[c] = p_of<FASTQ, DIRECT>(s[c], se, rn, sh0);
+                                }
                                 if (!whole) {
 #pragma unroll
                                     for (int c = 0; c < CW; ++c) pw[c] = c < nvalid ? pw[c] : 0u;
@@ -752,6 +770,12 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
                     for (int o = 1; o < NCQ; ++o) sum += red_sum[((cq + o) % NCQ) * TQ + row];
                     rn = shiftmax_norm(sum ? sum : 1, p.smx.s_d, p.smx.m_p, p.smx.M_hw, p.smx.k_out);
                     sh0 = (uint32_t)(rn.sh - se.k);
+                    {
+                        // the high-word form when every row of the warp allows it
+                        const bool row_ok = sh0 >= 32 || (rn.F >> sh0) == 0u;
+                        hiG = sh0 > 32 ? 0u : sh0 == 32 ? rn.F : rn.F << (32 - sh0);
+                        hi_form = __all_sync(0xffffffffu, row_ok);
+                    }
             } while (0);
             if (ok) run_pass(PassTag<2>{});
             // ---- O = P V from TMEM: sat8(rq(O; m_o, s_o)) at the token's own position (OPW columns)

@@ -256,6 +256,19 @@ def test_attention_tensor_memory_shapes(ilw, orc, B, T, H, dh, win, o_f16):
     assert_same(host(got), want, f"attn tc T={T} win={win} o_f16={o_f16}")
 
 
+@pytest.mark.parametrize("I0", [1, 16, 200])
+def test_attention_small_sums(ilw, orc, I0):
+    """Small I0 gives row sums below 2^23, so F >= 2^(sh0) for some rows and the tensor-memory
+    kernel's pass 3 takes the P form without the high-word product (every warp whose rows all allow
+    it takes the other); global and windowed, fp16-carried q|k|v."""
+    for B, T, H, win in ((1, 300, 2, 0), (1, 400, 1, 2)):
+        d = H * 64
+        qkv = synth.uniform_int(15, f"qkvsm{T}{I0}", (B * T, 3 * d), -40, 40, np.int8)
+        smx = {"I0": I0, "k_inter": 16, "k_out": 8, "s_d": -1, "m_p": 4, "M_hw": 31}
+        got = ilw.shiftmax_attn(dev(qkv.astype(np.float16)), B, T, H, 64, win, smx, 3 << 29, 36)
+        assert_same(host(got), orc.attention(qkv, B, T, H, 64, win, smx, 3 << 29, 36), f"attn small I0={I0} T={T}")
+
+
 def test_attention_extreme_scores(ilw, orc):
     """All q, k = +127 (largest scores, every row uniform) and alternating signs."""
     B, T, H, dh = 1, 130, 2, 64

@@ -398,3 +398,29 @@ def test_shiftmax_rows_one_multiply_output():
                 assert ((e * Fs) >> 32) >> rs == (e * F) >> sh
                 checked += 1
     assert checked > 100000
+
+
+def test_attention_p_as_one_high_word_product():
+    """Attention's pass 3 writes P = floor(I_b F / 2^(sh0 + q)) as umulhi(I_b, G) >> q, with
+    G = F 2^(32 - sh0) when sh0 <= 32 and F < 2^sh0, and G = 0 when sh0 > 32 (there I_b F < 2^32
+    <= 2^sh0, so every P is 0).  Checked against the exact floor over I_b < 2^15, the F and sh0 a
+    row can have, and every q <= 31."""
+    rng = np.random.default_rng(11)
+    ibs = np.concatenate([rng.integers(0, 1 << 15, 300), [0, 1, (1 << 15) - 1, 1 << 14]])
+    checked = 0
+    for sh0 in range(0, 48):
+        for F in np.concatenate([rng.integers(1, 1 << 31, 40), [1, 2, 31, 32, 255, 256, (1 << 31) - 1]]):
+            F = int(F)
+            ok = sh0 >= 32 or (F >> sh0) == 0
+            if not ok:
+                continue
+            G = 0 if sh0 > 32 else (F if sh0 == 32 else F << (32 - sh0))
+            assert G < (1 << 32)
+            for ib in ibs:
+                ib = int(ib)
+                if sh0 > 32 and ib * F >= (1 << 32):
+                    continue  # outside the kernel's condition I_b F < 2^32
+                for q in (0, 1, 7, 15, 16, 31):
+                    assert ((ib * G) >> 32) >> q == (ib * F) >> (sh0 + q)
+                    checked += 1
+    assert checked > 100000
