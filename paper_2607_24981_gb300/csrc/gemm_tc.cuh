@@ -117,6 +117,7 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
 // and raising the CTA's abort flag) when it ran out, or when another role already aborted.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort, int *status, int code,
                                           long long limit) {
+    if (mbar_try(bar, parity)) return true;  // the common case, without reading the clock
     long long t0 = clock64();
     for (uint32_t i = 0;; ++i) {
         if (mbar_try(bar, parity)) return true;
@@ -635,7 +636,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
         // ---------------------------------------------------------------- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-            int it = 0, tl = 0;
+            // operand descriptors from two precomputed bases: a 16-byte step of the address is 1 in
+            // the descriptor's low word (shared-memory offsets stay below 256 KB, so nothing carries)
+            const uint64_t a_desc0 = sw128_desc(smem_u32(smem)), w_desc0 = sw128_desc(smem_u32(wres));
+            int it = 0, tl = 0, s = 0;
+            uint32_t ph = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++tl) {
                 const int b = tl % p.nbuf;
@@ -647,8 +652,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                     const int nk = (S.klen + BK - 1) / BK;
                     const uint32_t dt = tmem + (uint32_t)(b * acc_cols + sg * BN);
                     for (int kk = 0; kk < nk; ++kk, ++it) {
-                        const int s = it % STAGES;
-                        const uint32_t ph = (it / STAGES) & 1;
                         if (!mbar_wait(AF16 ? full(s) : a_ready(s), ph, abort, p.status,
                                        AF16 ? kStatusTimeoutTma : kStatusTimeoutOperand, p.wait_cycles) ||
                             (WRES && tl == 0 && !mbar_wait(wfull(kk), 0, abort, p.status, kStatusTimeoutTma, p.wait_cycles))) {
@@ -656,13 +659,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
                             break;
                         }
                         tc_fence_after();
-                        const uint32_t a0 = smem_u32(smem + s * kStage);
-                        const uint32_t w0 = WRES ? smem_u32(wres + kk * SM::kWtile) : a0 + SM::kA16;
+                        const uint64_t da = a_desc0 + (uint64_t)((s * kStage) >> 4);
+                        const uint64_t dw = WRES ? w_desc0 + (uint64_t)((kk * SM::kWtile) >> 4) : da + (uint64_t)(SM::kA16 >> 4);
 #pragma unroll
                         for (int k16 = 0; k16 < BK / 16; ++k16)
-                            tc_mma(dt, sw128_desc(a0 + 32 * k16), sw128_desc(w0 + 32 * k16), idesc,
-                                   (kk > 0 || k16 > 0) ? 1u : 0u);
+                            tc_mma(dt, da + 2 * k16, dw + 2 * k16, idesc, (kk > 0 || k16 > 0) ? 1u : 0u);
                         tc_commit(empty(s));
+                        if (++s == STAGES) {
+                            s = 0;
+                            ph ^= 1u;
+                        }
                     }
                 }
                 tc_commit(acc_full(b));  // arrives once every MMA of this tile has completed
