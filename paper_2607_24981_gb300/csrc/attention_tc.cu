@@ -36,6 +36,10 @@
 // block is then 64 keys of each unit (two N = 64 score MMAs, each unit's rows reading their own
 // half of the columns), and each unit has its own O.  At 1600 tokens this turns 8 x 6 x 13 = 624
 // CTAs (2.05 waves of two per SM) into 600 (two waves).
+// The softmax warps' loop is compiled per pass, per launch form (with or without paired tiles) and,
+// for global attention, separately for full key blocks, so the hot loop carries no branch for the
+// cases it cannot meet.  In pass 3, P is one high-word product umulhi(I_b, F 2^(32 - sh0)) >> q when
+// every row of the warp allows it.
 // Every mbarrier wait is bounded (about one second); on expiry the kernel latches the device status
 // word, every role stops, the loaders drain their copies and the TMEM is freed after every MMA
 // issued has completed.
