@@ -31,7 +31,7 @@
 //               while the softmax works.  Warps whose rows all lie past the group, and 32-key
 //               loads past its keys, skip the arithmetic (their P is written as zero)
 // The CTAs holding the last (possibly partial, hence shorter) query tile of each group come after
-// all the others, so they fill the last wave.  Global attention whose last tile has at most 64
+// all the others, so they fill the last wave; paired last tiles (below) come before all the others.  Global attention whose last tile has at most 64
 // queries puts the last tiles of two (image, head) units in one CTA (rows 0-63 and 64-127): a key
 // block is then 64 keys of each unit (two N = 64 score MMAs, each unit's rows reading their own
 // half of the columns), and each unit has its own O.  At 1600 tokens this turns 8 x 6 x 13 = 624
@@ -310,7 +310,11 @@ __global__ void __launch_bounds__(kThreadsTc, kMinBlocks) attn_tc_kernel(const _
     int qt, head, z, head1 = 0, z1 = 0;
     bool pair = false, has1 = false;
     {
-        const int Z = p.B * p.nw * p.nw, L = blockIdx.x, F = (args.nq - 1) * p.H * Z;
+        // paired CTAs (the longest: every block twice the MMA and key traffic) come first, so they
+        // do not form the tail of the last wave; the unpaired last tiles (shorter) come last
+        const int Z = p.B * p.nw * p.nw, F = (args.nq - 1) * p.H * Z;
+        const int NPR = (MAYPAIR && args.pair) ? (p.H * Z + 1) / 2 : 0;
+        const int L = (int)blockIdx.x < NPR ? F + (int)blockIdx.x : (int)blockIdx.x - NPR;
         if (L < F) {
             qt = L % (args.nq - 1);
             head = (L / (args.nq - 1)) % p.H;

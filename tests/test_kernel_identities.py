@@ -253,15 +253,18 @@ def test_attention_cta_order_is_a_bijection(nq, H, Z):
 
 @pytest.mark.parametrize("nq,H,Z", [(1, 1, 1), (1, 3, 3), (13, 6, 8), (8, 3, 3), (2, 8, 1)])
 def test_attention_paired_last_tiles_cover_every_unit(nq, H, Z):
-    """Global attention whose last tile has at most 64 queries: the first (nq - 1) H Z CTAs keep the
-    one-tile mapping, CTA F + j holds the last tiles of units 2 j and 2 j + 1 (unit = head + H
-    image), the second absent when H Z is odd.  Every (tile, unit) is taken once, pairs may span two
-    images, and the grid shrinks by floor(H Z / 2) CTAs."""
+    """Global attention whose last tile has at most 64 queries: CTA j < ceil(H Z / 2) holds the last
+    tiles of units 2 j and 2 j + 1 (unit = head + H image; the second absent when H Z is odd), the
+    paired CTAs first; the remaining (nq - 1) H Z CTAs keep the one-tile mapping.  Every
+    (tile, unit) is taken once, pairs may span two images, and the grid shrinks by floor(H Z / 2)
+    CTAs."""
     F = (nq - 1) * H * Z
     units = H * Z
-    grid = F + (units + 1) // 2
+    npr = (units + 1) // 2
+    grid = F + npr
     seen = []
-    for L in range(grid):
+    for cta in range(grid):
+        L = F + cta if cta < npr else cta - npr
         if L < F:
             seen.append((L % (nq - 1), (L // (nq - 1)) % H, L // ((nq - 1) * H)))
         else:
@@ -270,7 +273,7 @@ def test_attention_paired_last_tiles_cover_every_unit(nq, H, Z):
             if u0 + 1 < units:
                 seen.append((nq - 1, (u0 + 1) % H, (u0 + 1) // H))
             else:
-                assert L == grid - 1 and units % 2 == 1
+                assert cta == npr - 1 and units % 2 == 1
     assert sorted(seen) == sorted((q, h, z) for q in range(nq) for h in range(H) for z in range(Z))
     assert grid == nq * units - units // 2
 
