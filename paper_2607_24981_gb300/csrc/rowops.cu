@@ -337,12 +337,14 @@ __device__ __noinline__ void ln_norm4_exact(const int32_t (&x)[4], int64_t mu, i
 
 // I-LayerNorm by row groups (Sec. 3.3; mean, variance, Newton's integer square root,
 // F = floor((2^31 - 1) / R), n = (y F) >> 1, out = sat(rq(n + beta; m, s))).  LPR lanes own one row,
-// 32 / LPR rows per warp, and every warp walks its own rows (persistent grid, no CTA barrier in the
-// loop).  A lane reads 16-byte chunks sub, sub + LPR, ... of its row (CPL at most; the LPR lanes of a
-// row read adjacent chunks, so a warp's load covers 32 / LPR row segments of LPR * 16 bytes), sums x
-// and x^2 (int64), and the LPR lanes combine them with shuffles; each lane then runs the row's Newton
-// sequence (the lanes of a row compute the same values, side by side with the other rows of the warp)
-// and normalises its own chunks with the per-column parameters from shared memory.
+// 32 / LPR rows per warp, 256 / LPR rows per CTA and step (persistent grid).  A lane reads 16-byte
+// chunks sub, sub + LPR, ... of its row (CPL at most; the LPR lanes of a row read adjacent chunks, so
+// a warp's load covers 32 / LPR row segments of LPR * 16 bytes) and keeps them in registers, sums x
+// and x^2 (int64), and the LPR lanes combine them with shuffles; the row's sums go to shared memory.
+// The per-row scalar work (mean, variance, Newton, F) then runs once per row, one row per thread of
+// the first 256 / LPR threads, instead of on every lane of the row: it is most of the instructions
+// when each of the LPR lanes repeats it.  Every lane reads its row's mean and F back and normalises
+// its own chunks with the per-column parameters from shared memory.
 // 32-bit normalisation: after at least one Newton step R >= isqrt(V) >= |y| for every y = x - mu of
 // the row (a floored Newton step from any positive start lands at or above isqrt(V)), so
 // |y F| <= |y| (2^31 - 1) / R < 2^31 and y F fits int32; with one shift s >= 33 for every column and
@@ -368,12 +370,14 @@ __global__ void __launch_bounds__(256, 3) layernorm_rows(const LnParams p) {
     const bool cols_fast = __syncthreads_and(col_fast) != 0 && uniform_shift >= 33;
     const int32_t rnd = cols_fast ? 1 << (uniform_shift - 33) : 0, sh = uniform_shift - 32;
 
+    constexpr int RPC = 8 * RPW;  // rows per CTA and step (256 threads)
+    __shared__ int64_t s_S[RPC], s_Q[RPC], s_mu[RPC], s_F[RPC];
+    __shared__ int32_t s_ok[RPC];
     const int lane = threadIdx.x & 31, sub = lane % LPR, rr = lane / LPR;
-    const int64_t ngroups = (p.rows + RPW - 1) / RPW;
-    const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
-    for (int64_t g = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); g < ngroups; g += wstride) {
-        const int64_t row = g * RPW + rr;
-        const bool live = row < p.rows;  // every lane stays for the shuffles
+    const int lrow = (threadIdx.x >> 5) * RPW + rr;  // the lane's row within the CTA's rows
+    for (int64_t r0 = (int64_t)blockIdx.x * RPC; r0 < p.rows; r0 += (int64_t)gridDim.x * RPC) {
+        const int64_t row = r0 + lrow;
+        const bool live = row < p.rows;  // every lane stays for the shuffles and the barriers
         const uint8_t *xr = (const uint8_t *)p.X + (live ? row : 0) * p.ldx * EB;
         int4 v[CPL];
 #pragma unroll
@@ -409,21 +413,33 @@ __global__ void __launch_bounds__(256, 3) layernorm_rows(const LnParams p) {
             S += __shfl_xor_sync(0xffffffffu, S, o, LPR);
             Q += __shfl_xor_sync(0xffffffffu, Q, o, LPR);
         }
-        // mu = floor((2S + C) / (2C)); V = Q - 2 mu S + C mu^2 (= sum (x - mu)^2 exactly)
-        const int64_t num = 2 * S + C, den = 2 * (int64_t)C;
-        int64_t mu;
-        if (num >= -(1ll << 31) && num < (1ll << 31)) {
-            const int32_t n32 = (int32_t)num, d32 = (int32_t)den;
-            const int32_t qt = n32 / d32;
-            mu = qt - ((n32 % d32 != 0 && n32 < 0) ? 1 : 0);
-        } else {
-            mu = num / den;
-            if ((num % den) != 0 && num < 0) mu -= 1;
+        if (sub == 0) {
+            s_S[lrow] = S;
+            s_Q[lrow] = Q;
         }
-        const uint64_t V = (uint64_t)(Q - 2 * mu * S + (int64_t)C * mu * mu);
-        const uint64_t R = V < (1ull << 48) ? newton_isqrt_fast(V, p.iters) : newton_isqrt_early(V, p.iters);
-        const int64_t F = R < (1ull << 32) ? (int64_t)div_int31((uint32_t)R) : 0;
-        const bool fast = cols_fast && __all_sync(0xffffffffu, p.iters >= 1 || V < (1ull << 32));
+        __syncthreads();
+        if (threadIdx.x < RPC) {
+            // one row per thread: mu = floor((2S + C) / (2C)); V = Q - 2 mu S + C mu^2 (= sum (x - mu)^2)
+            const int64_t S1 = s_S[threadIdx.x], Q1 = s_Q[threadIdx.x];
+            const int64_t num = 2 * S1 + C, den = 2 * (int64_t)C;
+            int64_t mu;
+            if (num >= -(1ll << 31) && num < (1ll << 31)) {
+                const int32_t n32 = (int32_t)num, d32 = (int32_t)den;
+                const int32_t qt = n32 / d32;
+                mu = qt - ((n32 % d32 != 0 && n32 < 0) ? 1 : 0);
+            } else {
+                mu = num / den;
+                if ((num % den) != 0 && num < 0) mu -= 1;
+            }
+            const uint64_t V = (uint64_t)(Q1 - 2 * mu * S1 + (int64_t)C * mu * mu);
+            const uint64_t R = V < (1ull << 48) ? newton_isqrt_fast(V, p.iters) : newton_isqrt_early(V, p.iters);
+            s_mu[threadIdx.x] = mu;
+            s_F[threadIdx.x] = R < (1ull << 32) ? (int64_t)div_int31((uint32_t)R) : 0;
+            s_ok[threadIdx.x] = p.iters >= 1 || V < (1ull << 32);
+        }
+        __syncthreads();
+        const int64_t mu = s_mu[lrow], F = s_F[lrow];
+        const bool fast = cols_fast && __all_sync(0xffffffffu, s_ok[lrow] != 0);
         const int32_t F32 = (int32_t)F, mF = (int32_t)(0u - (uint32_t)mu * (uint32_t)F);
         TOut *yr = (TOut *)p.Y + (live ? row : 0) * p.ldy;
 #pragma unroll
@@ -538,25 +554,26 @@ cudaError_t ln_dispatch(const LnParams &p, cudaStream_t s) {
     if (tiled) {
         const int nch = p.C * eb / 16;
         const size_t smem = (size_t)3 * p.C * sizeof(int32_t);
-        auto go = [&](auto kern) -> cudaError_t {
+        auto go = [&](auto kern, int lpr) -> cudaError_t {
             int dev = 0, sms = 0, per_sm = 0;
             cudaError_t e = cudaGetDevice(&dev);
             if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
             if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, smem);
             if (e != cudaSuccess) return e;
-            // persistent CTAs of 8 warps, at most one warp per row (each warp covers 32 / LPR rows)
+            // persistent CTAs of 8 warps, each step of a CTA covering 256 / LPR rows
+            const int64_t rpc = 256 / lpr;
             const int64_t grid = std::max<int64_t>(1, std::min<int64_t>((int64_t)std::max(per_sm, 1) * sms,
-                                                                        (p.rows + 7) / 8));
+                                                                        (p.rows + rpc - 1) / rpc));
             kern<<<(unsigned)grid, 256, smem, s>>>(p);
             return cudaGetLastError();
         };
         // chunks per lane: 6 for int16 rows (8 values each), 12 for int32 rows (4 values each), so a
         // lane holds at most 48 values; lanes per row from the row's chunk count
         constexpr int CPL = sizeof(TIn) == 2 ? 6 : 12;
-        if (nch <= 4 * CPL) return go(layernorm_rows<TIn, TOut, 4, CPL>);
-        if (nch <= 8 * CPL) return go(layernorm_rows<TIn, TOut, 8, CPL>);
-        if (nch <= 16 * CPL) return go(layernorm_rows<TIn, TOut, 16, CPL>);
-        if (nch <= 32 * CPL) return go(layernorm_rows<TIn, TOut, 32, CPL>);
+        if (nch <= 4 * CPL) return go(layernorm_rows<TIn, TOut, 4, CPL>, 4);
+        if (nch <= 8 * CPL) return go(layernorm_rows<TIn, TOut, 8, CPL>, 8);
+        if (nch <= 16 * CPL) return go(layernorm_rows<TIn, TOut, 16, CPL>, 16);
+        if (nch <= 32 * CPL) return go(layernorm_rows<TIn, TOut, 32, CPL>, 32);
     }
     const int rows_per_block = 8;
     dim3 grid((unsigned)((p.rows + rows_per_block - 1) / rows_per_block));
