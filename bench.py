@@ -590,7 +590,8 @@ def main(argv=None):
 
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one ncu capture of the
 # kernel at this launch size, for the kernels whose code has not changed since that capture
-NCU_TRAFFIC = {"attention_global": 29609472}  # attn_tc_kernel, batch 8 global launch (profiles/attn_tc_kernel_global_b8.md)
+# (the global attention's capture, 29.61 MB per launch, predates its current CTA order: none listed)
+NCU_TRAFFIC = {}
 
 
 def roofline_entry(name, k, work, peaks, clocks, sms):
