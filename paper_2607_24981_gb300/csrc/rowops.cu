@@ -632,15 +632,12 @@ cudaError_t launch_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const Ge
                 if (e != cudaSuccess) return e;
                 attr = true;
             }
-            int dev = 0, sms = 148;
-            cudaGetDevice(&dev);
-            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
             int64_t blocks = (n4 + 255) / 256;
-            if (blocks > 6 * sms) blocks = 6 * sms;
+            if (blocks > 6 * (int64_t)sm_count()) blocks = 6 * (int64_t)sm_count();
             sdshiftgelu_table<<<(unsigned)blocks, 256, smem, s>>>((const int4 *)X, (int4 *)Y, n4, c, T);
         } else if (n4) {
             int64_t blocks = (n4 + 255) / 256;
-            if (blocks > 152 * 16) blocks = 152 * 16;
+            if (blocks > 16 * (int64_t)sm_count()) blocks = 16 * (int64_t)sm_count();
             sdshiftgelu_vec<<<(unsigned)blocks, 256, 0, s>>>((const int4 *)X, (int4 *)Y, n4, c);
         }
     }
