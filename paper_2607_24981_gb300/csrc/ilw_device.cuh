@@ -67,9 +67,9 @@ __device__ __forceinline__ int32_t asr(int32_t v, int32_t s) {
 // Algorithm 1's I_e = I + (I >> 1) - (I >> 4) floors negative values; with I = -a,
 // floor(-a/2) = -((a+1) >> 1) and floor(-a/16) = -((a+15) >> 4), so
 //   -I_e = a + ((a+1) >> 1) - ((a+15) >> 4)
-// exactly, and every shift here acts on a non-negative value.  (Shifting the negated value
-// directly is not safe to leave to the compiler: CUDA 13.0 turned (-|x|) >> 4 into a truncating
-// shift when it could infer the operand's sign.)
+// exactly, and every shift here acts on a non-negative value.  (A device probe of the direct form,
+// (-|x|) >> 4 with the operand's sign known to the compiler, returned truncated rather than floored
+// results; the cause was not pursued, and the magnitude form does not depend on it.)
 __device__ __forceinline__ uint32_t shift_exp_mag(uint32_t a, const ShiftExpC &c) {
     uint32_t n = a + ((a + 1u) >> 1) - ((a + 15u) >> 4);  // -I_e (I * log2 e with shifts)
     n = min(n, (uint32_t)c.kI0);                            // -clamp_min(I_e, -k I0)
