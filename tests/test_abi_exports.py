@@ -105,6 +105,41 @@ def test_detection_entry_points_validate_without_gpu(built_lib):
     assert L.ilwdetr_topk(ctypes.c_void_p(16), 10, 0, 10, 3, ctypes.c_void_p(16), ctypes.c_void_p(16), None) == 0
 
 
+def test_layernorm_and_noalloc_validate_without_gpu(built_lib):
+    """I-LayerNorm and the allocation-free patch embedding reject bad arguments before any CUDA
+    call (so with no device at all): the no-alloc entry checks its weights and its scratch bound
+    before it looks up the scratch array or launches the gather."""
+    import paper_2607_24981_gb300 as ilw
+
+    L = ilw.lib()
+    v = ctypes.c_void_p(256)
+
+    def ln(in_bits=16, rows=4, C=64, beta=v, iters=10, out_bits=8):
+        return L.ilwdetr_int_layernorm(v, in_bits, C, rows, C, beta, v, v, iters, v, out_bits, C, None)
+
+    assert ln(in_bits=8) == -1
+    assert ln(out_bits=12) == -1
+    assert ln(C=5000) == -2 and b"4096" in L.ilwdetr_last_error()
+    assert ln(iters=65) == -1
+    assert ln(beta=None) == -1
+    assert ln(rows=0) == 0  # nothing to do, nothing launched
+
+    def pe(img=v, B=1, Cin=3, H=640, W=640, p=16, Wp=v, mult=v, pos=None, s_pos=10):
+        return L.ilwdetr_patch_embed_noalloc(img, B, Cin, H, W, p, Wp, v, mult, v, 384, pos, 1 << 30, s_pos, v, None)
+
+    assert pe(p=15) == -2  # the patch must be a multiple of 16
+    assert pe(H=632) == -2  # p must divide H
+    assert pe(img=ctypes.c_void_p(257)) == -1  # misaligned image
+    assert pe(Wp=None) == -1 and b"weight" in L.ilwdetr_last_error()
+    assert pe(Wp=ctypes.c_void_p(272)) == -1  # packed weight not 256-byte aligned
+    assert pe(mult=None) == -1
+    assert pe(pos=v, s_pos=63) == -1  # position-term shift outside [1, 62]
+    assert pe(B=0) == 0
+    # 7 images of 3 x 640 x 640 gather 8.6 MB of patches: more than the fixed scratch
+    assert 6 * 3 * 640 * 640 <= L.ilwdetr_patch_embed_noalloc_max_bytes() < 7 * 3 * 640 * 640
+    assert pe(B=7) == -2 and b"8 MiB" in L.ilwdetr_last_error()
+
+
 def test_int8_tcgen05_mma_is_not_available_on_sm103a(tmp_path):
     """The reason the integer GEMMs and attention run on kind::f16 (int8 values carried exactly in
     fp16, fp32 accumulation kept below 2^24): ptxas of this toolkit rejects the int8 tensor-core
