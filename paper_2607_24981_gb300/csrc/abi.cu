@@ -23,6 +23,24 @@ int fail(int code, const char *fmt, ...) {
     return code;
 }
 
+// Composite entry points (the patch embedding, the encoder block, the decoder layer) run their
+// steps twice: first with every launch suppressed, which checks each step's arguments with the
+// step's own validation, then for real; so an argument error in a later step is reported before
+// the first launch.  Each entry point's launch is skipped (ILW_OK) while g_check_only is set.
+thread_local bool g_check_only = false;
+struct CheckPass {
+    CheckPass() { g_check_only = true; }
+    ~CheckPass() { g_check_only = false; }
+};
+template <typename Body> int checked_then_run(Body body) {
+    if (g_check_only) return body();  // inside another composite's checking pass
+    {
+        CheckPass pass;
+        if (const int rc = body()) return rc;
+    }
+    return body();
+}
+
 int cuda_status(cudaError_t e, const char *what) {
     if (e == cudaSuccess) return ILW_OK;
     return fail(ILW_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
@@ -187,6 +205,7 @@ int gemm_impl(const void *A, int32_t a_form, int64_t lda, const void *Wp, const 
         ep.m_g = m_g;
         ep.s_g = s_g;
     }
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_gemm(gp, ep, (cudaStream_t)stream), what);
 }
 }  // namespace
@@ -245,6 +264,7 @@ int ilwdetr_split_conv(const int8_t *const *X, const int64_t *ldx, int32_t nb, i
     ep.out_bits = 8;
     ep.C = Y;
     ep.ldc = ldy;
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_gemm(gp, ep, (cudaStream_t)stream), "split_conv");
 }
 
@@ -256,6 +276,7 @@ int ilwdetr_shiftmax_rows(const int32_t *X, int64_t ldx, int64_t rows, int32_t l
     if (rows == 0 || len == 0) return ILW_OK;
     if (!X || !P || ldx < len || ldp < len) return fail(ILW_ERR_INVALID_ARG, "shiftmax_rows: NULL pointer or ld < len");
     if (!aligned(X, 4)) return fail(ILW_ERR_INVALID_ARG, "shiftmax_rows: X must be 4-byte aligned");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_shiftmax_rows(X, ldx, rows, len, make_smx(*p), P, ldp, (cudaStream_t)stream),
                        "shiftmax_rows");
 }
@@ -266,6 +287,7 @@ int ilwdetr_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const ilw_gelu_
     if (n < 0) return fail(ILW_ERR_INVALID_ARG, "sdshiftgelu: n < 0");
     if (n == 0) return ILW_OK;
     if (!X || !Y || !aligned(X, 4) || !aligned(Y, 4)) return fail(ILW_ERR_INVALID_ARG, "sdshiftgelu: NULL or misaligned");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_sdshiftgelu(X, Y, n, ilw::make_gelu(*p), (cudaStream_t)stream), "sdshiftgelu");
 }
 
@@ -281,6 +303,7 @@ int ilwdetr_int_layernorm(const void *X, int32_t in_bits, int64_t ldx, int64_t r
     if (!X || !Y || !beta || !mult || !shift || ldx < C || ldy < C)
         return fail(ILW_ERR_INVALID_ARG, "int_layernorm: NULL pointer or ld < C");
     ilw::LnParams lp{X, in_bits, ldx, rows, C, beta, mult, shift, iters, Y, out_bits, ldy};
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_layernorm(lp, (cudaStream_t)stream), "int_layernorm");
 }
 
@@ -329,6 +352,7 @@ int ilwdetr_shiftmax_attn(const void *Q, const void *K, const void *V, int64_t l
     ilw::AttnParams ap;
     int rc = attn_params(ap, Q, K, V, ld_qkv, qkv_form, B, T, H, dh, win_side, p, m_o, s_o, O, o_form, ld_o);
     if (rc) return rc;
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_attention(ap, (cudaStream_t)stream), "shiftmax_attn");
 }
 
@@ -358,6 +382,7 @@ int ilwdetr_deform_attn(const int8_t *value, const int32_t *level_hw, int32_t L,
     dp.B = B; dp.Q = Q; dp.H = H; dp.P = P; dp.dh = dh;
     dp.m = m; dp.s = s;
     dp.out = out;
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_deform(dp, (cudaStream_t)stream), "deform_attn");
 }
 
@@ -382,11 +407,15 @@ int ilwdetr_patch_embed(const int8_t *img, int32_t B, int32_t Cin, int32_t Hh, i
         return fail(ILW_ERR_INVALID_ARG, "patch_embed: workspace too small or misaligned");
     const int32_t T = (Hh / p) * (Ww / p), K = Cin * p * p;
     __half *A = (__half *)workspace;  // the patch matrix as fp16-carried int8: the GEMM reads it directly
-    cudaError_t e = ilw::launch_patchify_f16(img, B, Cin, Hh, Ww, p, A, (cudaStream_t)stream);
-    if (e != cudaSuccess) return cuda_status(e, "patchify");
-    ilw_residual_t r{pos, d, T, m_pos, s_pos};
-    return gemm_impl(A, ILW_I8_IN_F16, K, Wp, bias, mult, shift, B * T, d, K, ILW_EPI_REQUANT, 16, x0, d,
-                     pos ? &r : nullptr, nullptr, 0, 0, stream, "patch_embed");
+    return checked_then_run([&]() -> int {
+        if (!g_check_only) {
+            cudaError_t e = ilw::launch_patchify_f16(img, B, Cin, Hh, Ww, p, A, (cudaStream_t)stream);
+            if (e != cudaSuccess) return cuda_status(e, "patchify");
+        }
+        ilw_residual_t r{pos, d, T, m_pos, s_pos};
+        return gemm_impl(A, ILW_I8_IN_F16, K, Wp, bias, mult, shift, B * T, d, K, ILW_EPI_REQUANT, 16, x0, d,
+                         pos ? &r : nullptr, nullptr, 0, 0, stream, "patch_embed");
+    });
 }
 
 // ------------------------------------------------------------------ encoder block
@@ -421,27 +450,29 @@ int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t
     int16_t *x1 = (int16_t *)ws; ws += align256((size_t)M * d * 2);
     __half *a2 = (__half *)ws; ws += align256((size_t)M * d * 2);
     __half *hbuf = (__half *)ws;
-    int rc;
-    if ((rc = ilwdetr_int_layernorm(x, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, a1, F16, d, stream)))
-        return rc;
-    if ((rc = gemm_impl(a1, F16, d, p->w_qkv, p->b_qkv, p->m_qkv, p->s_qkv, M, 3 * d, d, ILW_EPI_REQUANT, F16, qkv, 3 * d,
-                        nullptr, nullptr, 0, 0, stream, "block qkv")))
-        return rc;
-    if ((rc = ilwdetr_shiftmax_attn(qkv, qkv + d, qkv + 2 * d, 3 * d, F16, B, T, H, d / H, p->win_side, &p->smx, p->m_o,
-                                    p->s_o, o, F16, d, stream)))
-        return rc;
-    ilw_residual_t r1{x, d, M, p->m_r1, p->s_r1};
-    if ((rc = gemm_impl(o, F16, d, p->w_proj, p->b_proj, p->m_proj, p->s_proj, M, d, d, ILW_EPI_REQUANT, 16, x1, d, &r1,
-                        nullptr, 0, 0, stream, "block proj")))
-        return rc;
-    if ((rc = ilwdetr_int_layernorm(x1, 16, d, M, d, p->ln2_beta, p->ln2_mult, p->ln2_shift, p->ln_iters, a2, F16, d, stream)))
-        return rc;
-    if ((rc = gemm_impl(a2, F16, d, p->w_fc1, p->b_fc1, p->m_fc1, p->s_fc1, M, F, d, ILW_EPI_GELU, F16, hbuf, F, nullptr,
-                        &p->gelu, p->m_g, p->s_g, stream, "block fc1")))
-        return rc;
-    ilw_residual_t r2{x1, d, M, p->m_r2, p->s_r2};
-    return gemm_impl(hbuf, F16, F, p->w_fc2, p->b_fc2, p->m_fc2, p->s_fc2, M, d, F, ILW_EPI_REQUANT, 16, y, d, &r2,
-                     nullptr, 0, 0, stream, "block fc2");
+    return checked_then_run([&]() -> int {
+        int rc;
+        if ((rc = ilwdetr_int_layernorm(x, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, a1, F16, d, stream)))
+            return rc;
+        if ((rc = gemm_impl(a1, F16, d, p->w_qkv, p->b_qkv, p->m_qkv, p->s_qkv, M, 3 * d, d, ILW_EPI_REQUANT, F16, qkv, 3 * d,
+                            nullptr, nullptr, 0, 0, stream, "block qkv")))
+            return rc;
+        if ((rc = ilwdetr_shiftmax_attn(qkv, qkv + d, qkv + 2 * d, 3 * d, F16, B, T, H, d / H, p->win_side, &p->smx, p->m_o,
+                                        p->s_o, o, F16, d, stream)))
+            return rc;
+        ilw_residual_t r1{x, d, M, p->m_r1, p->s_r1};
+        if ((rc = gemm_impl(o, F16, d, p->w_proj, p->b_proj, p->m_proj, p->s_proj, M, d, d, ILW_EPI_REQUANT, 16, x1, d, &r1,
+                            nullptr, 0, 0, stream, "block proj")))
+            return rc;
+        if ((rc = ilwdetr_int_layernorm(x1, 16, d, M, d, p->ln2_beta, p->ln2_mult, p->ln2_shift, p->ln_iters, a2, F16, d, stream)))
+            return rc;
+        if ((rc = gemm_impl(a2, F16, d, p->w_fc1, p->b_fc1, p->m_fc1, p->s_fc1, M, F, d, ILW_EPI_GELU, F16, hbuf, F, nullptr,
+                            &p->gelu, p->m_g, p->s_g, stream, "block fc1")))
+            return rc;
+        ilw_residual_t r2{x1, d, M, p->m_r2, p->s_r2};
+        return gemm_impl(hbuf, F16, F, p->w_fc2, p->b_fc2, p->m_fc2, p->s_fc2, M, d, F, ILW_EPI_REQUANT, 16, y, d, &r2,
+                         nullptr, 0, 0, stream, "block fc2");
+    });
 }
 
 // ------------------------------------------------------------------ detector: projector, decoder
@@ -463,6 +494,7 @@ int ilwdetr_requant(const void *X, int32_t in_bits, int64_t ldx, int64_t rows, i
     if (Z && (z_rows < 1 || ldz < C || !aligned(Z, 8) || ldz % 4))
         return fail(ILW_ERR_INVALID_ARG, "requant: bad second term");
     ilw::RequantParams p{X, in_bits, ldx, rows, C, m1, s1, Z, ldz, Z ? z_rows : 1, m2, Z ? s2 : 1, out_bits, Y, ldy};
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_requant(p, (cudaStream_t)stream), "requant");
 }
 
@@ -474,6 +506,7 @@ int ilwdetr_resample_nearest(const int8_t *X, int64_t x_bstride, int32_t B, int3
     if (B == 0) return ILW_OK;
     if (!X || !Y || !aligned(X, 16) || !aligned(Y, 16) || x_bstride < (int64_t)Hi * Wi || y_bstride < (int64_t)Ho * Wo)
         return fail(ILW_ERR_INVALID_ARG, "resample: NULL, misaligned or overlapping batch strides");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_resample(X, x_bstride, B, Hi, Wi, C, Y, y_bstride, Ho, Wo, (cudaStream_t)stream),
                        "resample_nearest");
 }
@@ -554,62 +587,68 @@ int ilwdetr_decoder_layer_forward(const ilw_decoder_params_t *p, const int16_t *
     const DecBufs b = dec_layout((char *)workspace, B, Q, S_total, d, F, H, L, P);
     const int32_t M = B * Q, LP = L * P, HLP = H * LP;
     const int64_t MS = (int64_t)B * S_total;
-    int rc;
+    return checked_then_run([&]() -> int {
+        int rc;
 #define ILW_TRY(x) \
-    if ((rc = (x))) return rc
-    // self-attention
-    ILW_TRY(ilwdetr_requant(tgt, 16, d, M, d, p->m_q1, p->s_q1, pos, d, M, p->m_q2, p->s_q2, 8, b.qk_in, d, stream));
-    ILW_TRY(ilwdetr_requant(tgt, 16, d, M, d, p->m_v1, p->s_v1, nullptr, 0, 1, 0, 1, 8, b.v_in, d, stream));
-    ILW_TRY(ilwdetr_gemm_requant(b.qk_in, d, p->w_qk, p->b_qk, p->m_qk, p->s_qk, M, 2 * d, d, 8, b.qkv, 3 * d, nullptr,
-                                 stream));
-    ILW_TRY(ilwdetr_gemm_requant(b.v_in, d, p->w_v, p->b_v, p->m_v, p->s_v, M, d, d, 8, b.qkv + 2 * d, 3 * d, nullptr,
-                                 stream));
-    if (d / H < 64) {
-        // heads of 32 columns run on the tensor-memory attention of 64-column heads: q|k|v widened with
-        // zero columns (nothing added to q.k, zero outputs), the output narrowed back
-        const int64_t w = (int64_t)H * 64;
-        cudaError_t e = ilw::launch_head_pad64(b.qkv, 3 * d, M, 3 * H, d / H, b.qkv64, (cudaStream_t)stream);
-        if (e != cudaSuccess) return cuda_status(e, "decoder head pad");
-        ILW_TRY(ilwdetr_shiftmax_attn(b.qkv64, b.qkv64 + w, b.qkv64 + 2 * w, 3 * w, ILW_I8_IN_F16, B, Q, H, 64, 0, &p->smx,
-                                      p->m_o, p->s_o, b.o64, 8, w, stream));
-        e = ilw::launch_head_compact(b.o64, w, M, H, d / H, b.o, d, (cudaStream_t)stream);
-        if (e != cudaSuccess) return cuda_status(e, "decoder head compact");
-    } else {
-        ILW_TRY(ilwdetr_shiftmax_attn(b.qkv, b.qkv + d, b.qkv + 2 * d, 3 * d, 8, B, Q, H, d / H, 0, &p->smx, p->m_o,
-                                      p->s_o, b.o, 8, d, stream));
-    }
-    ilw_residual_t r1{tgt, d, M, p->m_r1, p->s_r1};
-    ILW_TRY(ilwdetr_gemm_requant(b.o, d, p->w_o, p->b_o, p->m_oc, p->s_oc, M, d, d, 16, b.x1, d, &r1, stream));
-    ILW_TRY(ilwdetr_int_layernorm(b.x1, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, b.t1, 16, d,
-                                  stream));
-    // deformable cross-attention
-    ILW_TRY(ilwdetr_requant(b.t1, 16, d, M, d, p->m_c1, p->s_c1, pos, d, M, p->m_c2, p->s_c2, 8, b.qc, d, stream));
-    ILW_TRY(ilwdetr_gemm_requant(memory, d, p->w_val, p->b_val, p->m_val, p->s_val, (int32_t)MS, d, d, 8, b.value, d,
-                                 nullptr, stream));
-    ILW_TRY(ilwdetr_gemm_requant(b.qc, d, p->w_off, p->b_off, p->m_off, p->s_off, M, 2 * HLP, d, 16, b.off16, 2 * HLP,
-                                 nullptr, stream));
-    ILW_TRY(ilwdetr_gemm_requant(b.qc, d, p->w_att, p->b_att, p->m_att, p->s_att, M, HLP, d, 16, b.att16, HLP, nullptr,
-                                 stream));
-    // int16 -> int32 containers (rq with m = 2^30, s = 30 is the identity)
-    ILW_TRY(ilwdetr_requant(b.off16, 16, 2 * HLP, M, 2 * HLP, 1 << 30, 30, nullptr, 0, 1, 0, 1, 32, b.off32, 2 * HLP,
-                            stream));
-    ILW_TRY(ilwdetr_requant(b.att16, 16, HLP, M, HLP, 1 << 30, 30, nullptr, 0, 1, 0, 1, 32, b.att32, HLP, stream));
-    ILW_TRY(ilwdetr_shiftmax_rows(b.att32, LP, (int64_t)M * H, LP, &p->smx_w, b.w, LP, stream));
-    ILW_TRY(ilwdetr_deform_attn(b.value, level_hw, L, ref_q16, b.off32, b.w, B, Q, H, P, d / H, p->m_s, p->s_s, b.samp,
+        if ((rc = (x))) return rc
+        // self-attention
+        ILW_TRY(ilwdetr_requant(tgt, 16, d, M, d, p->m_q1, p->s_q1, pos, d, M, p->m_q2, p->s_q2, 8, b.qk_in, d, stream));
+        ILW_TRY(ilwdetr_requant(tgt, 16, d, M, d, p->m_v1, p->s_v1, nullptr, 0, 1, 0, 1, 8, b.v_in, d, stream));
+        ILW_TRY(ilwdetr_gemm_requant(b.qk_in, d, p->w_qk, p->b_qk, p->m_qk, p->s_qk, M, 2 * d, d, 8, b.qkv, 3 * d, nullptr,
+                                     stream));
+        ILW_TRY(ilwdetr_gemm_requant(b.v_in, d, p->w_v, p->b_v, p->m_v, p->s_v, M, d, d, 8, b.qkv + 2 * d, 3 * d, nullptr,
+                                     stream));
+        if (d / H < 64) {
+            // heads of 32 columns run on the tensor-memory attention of 64-column heads: q|k|v widened with
+            // zero columns (nothing added to q.k, zero outputs), the output narrowed back
+            const int64_t w = (int64_t)H * 64;
+            if (!g_check_only) {
+                cudaError_t e = ilw::launch_head_pad64(b.qkv, 3 * d, M, 3 * H, d / H, b.qkv64, (cudaStream_t)stream);
+                if (e != cudaSuccess) return cuda_status(e, "decoder head pad");
+            }
+            ILW_TRY(ilwdetr_shiftmax_attn(b.qkv64, b.qkv64 + w, b.qkv64 + 2 * w, 3 * w, ILW_I8_IN_F16, B, Q, H, 64, 0, &p->smx,
+                                          p->m_o, p->s_o, b.o64, 8, w, stream));
+            if (!g_check_only) {
+                cudaError_t e = ilw::launch_head_compact(b.o64, w, M, H, d / H, b.o, d, (cudaStream_t)stream);
+                if (e != cudaSuccess) return cuda_status(e, "decoder head compact");
+            }
+        } else {
+            ILW_TRY(ilwdetr_shiftmax_attn(b.qkv, b.qkv + d, b.qkv + 2 * d, 3 * d, 8, B, Q, H, d / H, 0, &p->smx, p->m_o,
+                                          p->s_o, b.o, 8, d, stream));
+        }
+        ilw_residual_t r1{tgt, d, M, p->m_r1, p->s_r1};
+        ILW_TRY(ilwdetr_gemm_requant(b.o, d, p->w_o, p->b_o, p->m_oc, p->s_oc, M, d, d, 16, b.x1, d, &r1, stream));
+        ILW_TRY(ilwdetr_int_layernorm(b.x1, 16, d, M, d, p->ln1_beta, p->ln1_mult, p->ln1_shift, p->ln_iters, b.t1, 16, d,
+                                      stream));
+        // deformable cross-attention
+        ILW_TRY(ilwdetr_requant(b.t1, 16, d, M, d, p->m_c1, p->s_c1, pos, d, M, p->m_c2, p->s_c2, 8, b.qc, d, stream));
+        ILW_TRY(ilwdetr_gemm_requant(memory, d, p->w_val, p->b_val, p->m_val, p->s_val, (int32_t)MS, d, d, 8, b.value, d,
+                                     nullptr, stream));
+        ILW_TRY(ilwdetr_gemm_requant(b.qc, d, p->w_off, p->b_off, p->m_off, p->s_off, M, 2 * HLP, d, 16, b.off16, 2 * HLP,
+                                     nullptr, stream));
+        ILW_TRY(ilwdetr_gemm_requant(b.qc, d, p->w_att, p->b_att, p->m_att, p->s_att, M, HLP, d, 16, b.att16, HLP, nullptr,
+                                     stream));
+        // int16 -> int32 containers (rq with m = 2^30, s = 30 is the identity)
+        ILW_TRY(ilwdetr_requant(b.off16, 16, 2 * HLP, M, 2 * HLP, 1 << 30, 30, nullptr, 0, 1, 0, 1, 32, b.off32, 2 * HLP,
                                 stream));
-    ilw_residual_t r2{b.t1, d, M, p->m_r2, p->s_r2};
-    ILW_TRY(ilwdetr_gemm_requant(b.samp, d, p->w_o2, p->b_o2, p->m_o2, p->s_o2, M, d, d, 16, b.x2, d, &r2, stream));
-    ILW_TRY(ilwdetr_int_layernorm(b.x2, 16, d, M, d, p->ln2_beta, p->ln2_mult, p->ln2_shift, p->ln_iters, b.t2, 16, d,
-                                  stream));
-    // FFN
-    ILW_TRY(ilwdetr_requant(b.t2, 16, d, M, d, p->m_f, p->s_f, nullptr, 0, 1, 0, 1, 8, b.fin, d, stream));
-    ILW_TRY(ilwdetr_gemm_gelu(b.fin, d, p->w_fc1, p->b_fc1, p->m_fc1, p->s_fc1, M, F, d, &p->gelu, p->m_g, p->s_g, b.h,
-                              F, stream));
-    ilw_residual_t r3{b.t2, d, M, p->m_r3, p->s_r3};
-    ILW_TRY(ilwdetr_gemm_requant(b.h, F, p->w_fc2, p->b_fc2, p->m_fc2, p->s_fc2, M, d, F, 16, b.x3, d, &r3, stream));
-    return ilwdetr_int_layernorm(b.x3, 16, d, M, d, p->ln3_beta, p->ln3_mult, p->ln3_shift, p->ln_iters, out, 16, d,
-                                 stream);
+        ILW_TRY(ilwdetr_requant(b.att16, 16, HLP, M, HLP, 1 << 30, 30, nullptr, 0, 1, 0, 1, 32, b.att32, HLP, stream));
+        ILW_TRY(ilwdetr_shiftmax_rows(b.att32, LP, (int64_t)M * H, LP, &p->smx_w, b.w, LP, stream));
+        ILW_TRY(ilwdetr_deform_attn(b.value, level_hw, L, ref_q16, b.off32, b.w, B, Q, H, P, d / H, p->m_s, p->s_s, b.samp,
+                                    stream));
+        ilw_residual_t r2{b.t1, d, M, p->m_r2, p->s_r2};
+        ILW_TRY(ilwdetr_gemm_requant(b.samp, d, p->w_o2, p->b_o2, p->m_o2, p->s_o2, M, d, d, 16, b.x2, d, &r2, stream));
+        ILW_TRY(ilwdetr_int_layernorm(b.x2, 16, d, M, d, p->ln2_beta, p->ln2_mult, p->ln2_shift, p->ln_iters, b.t2, 16, d,
+                                      stream));
+        // FFN
+        ILW_TRY(ilwdetr_requant(b.t2, 16, d, M, d, p->m_f, p->s_f, nullptr, 0, 1, 0, 1, 8, b.fin, d, stream));
+        ILW_TRY(ilwdetr_gemm_gelu(b.fin, d, p->w_fc1, p->b_fc1, p->m_fc1, p->s_fc1, M, F, d, &p->gelu, p->m_g, p->s_g, b.h,
+                                  F, stream));
+        ilw_residual_t r3{b.t2, d, M, p->m_r3, p->s_r3};
+        ILW_TRY(ilwdetr_gemm_requant(b.h, F, p->w_fc2, p->b_fc2, p->m_fc2, p->s_fc2, M, d, F, 16, b.x3, d, &r3, stream));
+        return ilwdetr_int_layernorm(b.x3, 16, d, M, d, p->ln3_beta, p->ln3_mult, p->ln3_shift, p->ln_iters, out, 16, d,
+                                     stream);
 #undef ILW_TRY
+    });
 }
 
 // ---------------------------------------------------------------- detection head, two-stage selection

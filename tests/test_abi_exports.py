@@ -1,5 +1,6 @@
 """The C-ABI library builds, loads without a GPU and exports every entry point declared in
-include/ilwdetr.h; the Python binding covers the same names.  No compute call is made here."""
+include/ilwdetr.h; the Python binding covers the same names.  No kernel runs here: argument checks
+are exercised up to the first CUDA call, which fails on a machine without a device."""
 import ctypes
 import os
 import re
@@ -138,6 +139,102 @@ def test_layernorm_and_noalloc_validate_without_gpu(built_lib):
     # 7 images of 3 x 640 x 640 gather 8.6 MB of patches: more than the fixed scratch
     assert 6 * 3 * 640 * 640 <= L.ilwdetr_patch_embed_noalloc_max_bytes() < 7 * 3 * 640 * 640
     assert pe(B=7) == -2 and b"8 MiB" in L.ilwdetr_last_error()
+
+
+def _no_cuda_device():
+    try:
+        import torch
+    except ImportError:
+        return True
+    return not torch.cuda.is_available()
+
+
+# Fake device addresses: these tests only run where no CUDA device exists, so nothing can be
+# launched on them (the first real launch fails with ILW_ERR_CUDA before touching memory).
+no_device = pytest.mark.skipif(not _no_cuda_device(), reason="checks the no-device behaviour")
+
+
+def _fake_ptrs(struct, base):
+    """Every pointer field of a ctypes struct set to a distinct 256-byte aligned fake address."""
+    k = 0
+    for name, typ in struct._fields_:
+        if typ is ctypes.c_void_p:
+            setattr(struct, name, base + 0x10000 * k)
+            k += 1
+
+
+@no_device
+def test_composite_entry_points_check_every_step_before_launching(built_lib):
+    """The encoder block, the decoder layer and the patch embedding check the arguments of all
+    their steps before the first launch: a bad parameter of a late step (the attention's Shiftmax,
+    the FFN's GELU, a residual shift, the deformable weights' Shiftmax) is an argument error, not a
+    CUDA error from a launch already made; with valid arguments the checking pass succeeds and the
+    first real launch fails only for want of a device."""
+    import paper_2607_24981_gb300 as ilw
+
+    L = ilw.lib()
+    B, T, d, H, F = 2, 1600, 384, 6, 1536
+
+    def block(**over):
+        bp = ilw.BlockParamsT()
+        _fake_ptrs(bp, 0x7000000)
+        bp.struct_size = ctypes.sizeof(ilw.BlockParamsT)
+        bp.d, bp.H, bp.F, bp.win_side, bp.ln_iters = d, H, F, 2, 10
+        bp.smx = ilw.ShiftmaxT(3000, 16, 8, -1, 4, 31)
+        bp.gelu = ilw.GeluT(600, 16, 8)
+        bp.m_o, bp.s_o, bp.m_r1, bp.s_r1, bp.m_g, bp.s_g, bp.m_r2, bp.s_r2 = (1 << 30, 34) * 4
+        for k, val in over.items():
+            setattr(bp, k, val)
+        ws = L.ilwdetr_block_workspace_bytes(B, T, d, F)
+        return L.ilwdetr_block_forward(ctypes.byref(bp), ctypes.c_void_p(0x100000), ctypes.c_void_p(0x200000),
+                                       B, T, ctypes.c_void_p(0x300000), ws, None)
+
+    assert block() == -3  # ILW_ERR_CUDA: every step's arguments passed, the first launch has no device
+    assert block(smx=ilw.ShiftmaxT(0, 16, 8, -1, 4, 31)) == -1 and b"I0" in L.ilwdetr_last_error()
+    assert block(gelu=ilw.GeluT(1 << 15, 16, 8)) == -1
+    assert block(s_r2=63) == -1 and b"residual" in L.ilwdetr_last_error()
+    assert block(s_g=0) == -1
+    assert block(win_side=7) == -1 and b"window" in L.ilwdetr_last_error()  # 40 x 40 grid, 7 does not divide 40
+
+    lvl = (ctypes.c_int32 * 6)(80, 80, 40, 40, 20, 20)
+    Bd, Q, dd, Hd, Fd, Ld, Pd = 2, 300, 256, 8, 1024, 3, 4
+
+    def decoder(**over):
+        dp = ilw.DecoderParamsT()
+        _fake_ptrs(dp, 0x9000000)
+        dp.struct_size = ctypes.sizeof(ilw.DecoderParamsT)
+        dp.d, dp.H, dp.F, dp.L, dp.P, dp.ln_iters = dd, Hd, Fd, Ld, Pd, 20
+        for name, typ in ilw.DecoderParamsT._fields_:
+            if typ is ctypes.c_int32 and name.startswith("s_"):
+                setattr(dp, name, 34)
+            elif typ is ctypes.c_int32 and name.startswith("m_"):
+                setattr(dp, name, 1 << 30)
+        dp.smx = ilw.ShiftmaxT(3000, 16, 8, -1, 4, 31)
+        dp.smx_w = ilw.ShiftmaxT(3000, 16, 8, -1, 4, 31)
+        dp.gelu = ilw.GeluT(600, 16, 8)
+        for k, val in over.items():
+            setattr(dp, k, val)
+        ws = L.ilwdetr_decoder_workspace_bytes(Bd, Q, 8400, dd, Fd, Hd, Ld, Pd)
+        return L.ilwdetr_decoder_layer_forward(ctypes.byref(dp), ctypes.c_void_p(0x100000), ctypes.c_void_p(0x200000),
+                                               ctypes.c_void_p(0x300000), lvl, Ld, ctypes.c_void_p(0x400000), Bd, Q,
+                                               ctypes.c_void_p(0x500000), ctypes.c_void_p(0x600000), ws, None)
+
+    assert decoder() == -3
+    assert decoder(smx_w=ilw.ShiftmaxT(0, 16, 8, -1, 4, 31)) == -1  # the deformable weights, late in the layer
+    assert decoder(s_s=0) == -1 and b"deform" in L.ilwdetr_last_error()
+    assert decoder(gelu=ilw.GeluT(1 << 15, 16, 8)) == -1
+    assert decoder(s_r3=63) == -1
+
+    def patch(Wp=0x200000, s_pos=10):
+        ws = L.ilwdetr_patch_embed_workspace_bytes(2, 3, 640, 640, 16)
+        return L.ilwdetr_patch_embed(ctypes.c_void_p(0x100000), 2, 3, 640, 640, 16, ctypes.c_void_p(Wp),
+                                     ctypes.c_void_p(0x300000), ctypes.c_void_p(0x400000), ctypes.c_void_p(0x500000),
+                                     384, ctypes.c_void_p(0x600000), 1 << 30, s_pos, ctypes.c_void_p(0x700000),
+                                     ctypes.c_void_p(0x800000), ws, None)
+
+    assert patch() == -3
+    assert patch(Wp=0x200010) == -1 and b"256-byte" in L.ilwdetr_last_error()  # the GEMM's check, before the gather
+    assert patch(s_pos=63) == -1 and b"residual" in L.ilwdetr_last_error()
 
 
 def test_int8_tcgen05_mma_is_not_available_on_sm103a(tmp_path):
