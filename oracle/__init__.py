@@ -8,6 +8,13 @@ Every function takes and returns numpy arrays; the integer semantics are those o
 oracle (see ``ilw_oracle.h``): Algorithm 1 (ShiftExp, SD-ShiftGELU), Algorithm 2
 (CalibrateShift, Constrained Shiftmax), Sec. 3.2 (integer linear layers, split convolution),
 Sec. 3.3 (I-LayerNorm) and Sec. 3.1.1 (nearest-neighbour deformable sampling).
+
+Parity status of the compositions written here in Python from the pinned C++ operators:
+``projector``, ``decoder_layer``, ``detection_head``, ``refine_references``, ``decoder_stack``,
+``two_stage`` and ``query_pos`` are parity unpinned beyond their parts and the invariants that
+tests/test_oracle_pins.py checks for them (query-permutation equivariance, image independence,
+reduction to the reference sigmoid and to fixed references, selection of the best tokens,
+row-wise application): their structure is a reading of the paper, which does not state it.
 """
 from __future__ import annotations
 
