@@ -427,3 +427,40 @@ def test_attention_p_as_one_high_word_product():
                     assert ((ib * G) >> 32) >> q == (ib * F) >> (sh0 + q)
                     checked += 1
     assert checked > 100000
+
+
+@pytest.mark.parametrize("LPR,CPL,C,EPC", [(4, 12, 192, 4), (8, 12, 384, 4), (8, 6, 384, 8), (16, 6, 704, 8),
+                                            (32, 6, 1024, 8)])
+@pytest.mark.parametrize("rows,grid", [(1, 1), (77, 3), (12800, 400), (1000, 7)])
+def test_layernorm_rows_mapping(LPR, CPL, C, EPC, rows, grid):
+    """The I-LayerNorm row kernel: 256 threads, LPR lanes per row, RPW = 32 / LPR rows per warp and
+    RPC = 8 RPW rows per CTA step; CTA b takes the steps at rows r0 = b RPC + k grid RPC.  Lane l
+    of warp w owns row r0 + lrow, lrow = w RPW + l / LPR, and chunks sub + LPR i (i < CPL, sub =
+    l % LPR) of its C / EPC 16-byte chunks.  Every element of every row is read by exactly one
+    thread, once; the lanes with sub = 0 write one sum slot per row of the step (slots 0 .. RPC-1,
+    each once), and the per-row threads t < RPC read exactly those slots."""
+    RPW = 32 // LPR
+    RPC = 8 * RPW
+    nch = C // EPC
+    assert nch <= LPR * CPL  # the launcher's choice of LPR for this row length
+    hits = np.zeros((rows, nch), dtype=np.int64)
+    for b in range(grid):
+        r0 = b * RPC
+        while r0 < rows:
+            slots = []
+            for t in range(256):
+                w, l = divmod(t, 32)
+                sub, rr = l % LPR, l // LPR
+                lrow = w * RPW + rr
+                row = r0 + lrow
+                if sub == 0:
+                    slots.append(lrow)
+                if row >= rows:
+                    continue
+                for i in range(CPL):
+                    j = sub + LPR * i
+                    if j < nch:
+                        hits[row, j] += 1
+            assert sorted(slots) == list(range(RPC))  # the slots the per-row threads t < RPC read
+            r0 += grid * RPC
+    assert (hits == 1).all()
