@@ -464,3 +464,22 @@ def test_layernorm_rows_mapping(LPR, CPL, C, EPC, rows, grid):
             assert sorted(slots) == list(range(RPC))  # the slots the per-row threads t < RPC read
             r0 += grid * RPC
     assert (hits == 1).all()
+
+
+@pytest.mark.parametrize("tiles_m,tiles_n", [(1, 1), (100, 6), (100, 3), (50, 8), (3, 200), (7, 152), (200, 1)])
+def test_gemm_resident_weight_grid(tiles_m, tiles_n, sms=152):
+    """The persistent GEMM with resident weights: tile t is (row block t / tiles_n, column block
+    t % tiles_n) and CTA b takes the tiles b, b + grid, ...; the launcher makes the grid a multiple
+    of tiles_n (per_n = clamp(sms / tiles_n, 1, tiles_m) CTAs per column block).  So every tile is
+    computed once and each CTA only ever needs the one column block of W it keeps in shared memory;
+    the column blocks' tiles are spread over their per_n CTAs within one tile of each other."""
+    tiles = tiles_m * tiles_n
+    per_n = min(max(sms // tiles_n, 1), tiles_m)
+    grid = per_n * tiles_n
+    seen = np.zeros(tiles, dtype=np.int64)
+    for b in range(grid):
+        mine = list(range(b, tiles, grid))
+        seen[mine] += 1
+        assert len({t % tiles_n for t in mine}) <= 1  # one resident column block per CTA
+        assert tiles_m // per_n <= len(mine) <= -(-tiles_m // per_n)
+    assert (seen == 1).all()
