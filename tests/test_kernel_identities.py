@@ -1,5 +1,7 @@
 """Integer identities the CUDA kernels use in place of the paper's literal steps, checked
 exhaustively on the CPU over the ranges the kernels admit (numpy int64 arithmetic)."""
+import math
+
 import numpy as np
 import pytest
 
@@ -483,3 +485,49 @@ def test_gemm_resident_weight_grid(tiles_m, tiles_n, sms=152):
         assert len({t % tiles_n for t in mine}) <= 1  # one resident column block per CTA
         assert tiles_m // per_n <= len(mine) <= -(-tiles_m // per_n)
     assert (seen == 1).all()
+
+
+def test_layernorm_fast_normalisation_fits_int32():
+    """I-LayerNorm's 32-bit normalisation: after at least one Newton step from 2^16 the iterate R is
+    at least isqrt(V) >= |y| for every y = x - mu of the row, so F = floor((2^31 - 1) / R) gives
+    |y F| < 2^31; the kernel then forms (y F) >> 1 as the wrapping 32-bit x F + mF (mF = -mu F mod
+    2^32), and n + beta stays in int32 for |beta| <= 2^30.  Checked on random, constant and
+    single-spike rows of int16 and int32 inputs for 1 to 20 Newton steps."""
+    rng = np.random.default_rng(23)
+
+    def newton(V, iters):
+        r = 1 << 16
+        for _ in range(iters):
+            if r == 0:
+                break
+            r = (r + V // r) >> 1
+        return max(r, 1)
+
+    def wrap32(v):
+        v &= 0xFFFFFFFF
+        return v - (1 << 32) if v >= 1 << 31 else v
+
+    rows = []
+    for C in (1, 7, 64, 192, 384, 1024):
+        for lim in (127, 32767, 1 << 24):
+            rows.append(rng.integers(-lim, lim + 1, C))
+            spike = np.zeros(C, dtype=np.int64)
+            spike[0] = lim
+            rows.append(spike)
+            rows.append(np.full(C, -lim, dtype=np.int64))
+    for x in rows:
+        x = [int(t) for t in x]
+        C = len(x)
+        mu = (2 * sum(x) + C) // (2 * C)
+        V = sum((t - mu) ** 2 for t in x)
+        for iters in (1, 2, 3, 10, 20):
+            R = newton(V, iters)
+            assert R >= math.isqrt(V) >= max(abs(t - mu) for t in x)
+            F = ((1 << 31) - 1) // R
+            mF = wrap32(-mu * F)
+            for t in x:
+                y = t - mu
+                assert abs(y * F) < 1 << 31
+                n = (y * F) >> 1
+                assert wrap32(wrap32(t * F) + mF) >> 1 == n
+                assert -(1 << 31) <= n - (1 << 30) and n + (1 << 30) < 1 << 31
