@@ -102,7 +102,10 @@ int ilwdetr_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, ilw
  *   out_bits 8 / 16: C[i,c] = satN(rq(acc; mult[c], shift[c]) [+ rq(res...)]) (int8 / int16)
  *   out_bits 32    : C[i,c] = acc (int32; mult, shift and res ignored and may be NULL)
  *   out_bits ILW_I8_IN_F16: the out_bits 8 values, stored as fp16 (C is fp16 [M, ldc])
- *   bias may be NULL (0).  C has leading dimension ldc (elements). */
+ *   bias may be NULL (0).  C has leading dimension ldc (elements).
+ *   K: a multiple of 16.  Each output tile keeps one exact fp32 accumulator per 1024 terms of K in
+ *   tensor memory, so K <= 2048 in every tile shape and K <= 4096 where 128-wide tiles are chosen;
+ *   a K the chosen shape cannot hold is refused before any launch (ILW_ERR_CUDA, invalid argument). */
 int ilwdetr_gemm_requant(const int8_t *A, int64_t lda, const void *Wp, const int32_t *bias,
                          const int32_t *mult, const int32_t *shift, int32_t M, int32_t N,
                          int32_t K, int32_t out_bits, void *C, int64_t ldc,
