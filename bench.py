@@ -75,6 +75,17 @@ def workload_cfg():
     return dict(synth.CONFIGS[WORKLOAD])
 
 
+def workload_config(cfg, world):
+    """The `config` of the bench line: the workload both arms report on (the reference arm times a
+    bounded sample of it, described in its cpu_baseline)."""
+    return {"workload": "medium_c2: Medium integer ViT backbone (patch embed + 10 blocks)",
+            "B": cfg["B"], "T": cfg["T"], "d": cfg["d"], "H": cfg["H"], "F": cfg["F"], "blocks": cfg["layers"],
+            "global_layers": list(cfg["global_layers"]), "window": "2x2 windows of 400 tokens",
+            "image": "640x640 int8, 16x16 patches", "per_gpu_batch": cfg["B"],
+            "units": "block-tokens = blocks x images x tokens per step",
+            "l2": "flushed between timed steps (256 MB write)", "parallelism": f"replicas x{world}"}
+
+
 def build_host_params():
     from paper_2607_24981_gb300 import synth
 
@@ -385,8 +396,7 @@ def run_reference(args) -> None:
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-            "config": {"workload": "medium_c2 backbone (CPU oracle sample)", "B": n, "T": cfg["T"],
-                       "d": cfg["d"], "H": cfg["H"], "F": cfg["F"]},
+            "config": workload_config(cfg, world),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": n, "kind": "oracle", "cpu": host["model"],
                              "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -568,12 +578,7 @@ def main(argv=None):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int8", "data": "synthetic",
-            "config": {"workload": "medium_c2: Medium integer ViT backbone (patch embed + 10 blocks)",
-                       "B": B, "T": T, "d": cfg["d"], "H": cfg["H"], "F": cfg["F"], "blocks": L,
-                       "global_layers": list(cfg["global_layers"]), "window": "2x2 windows of 400 tokens",
-                       "image": "640x640 int8, 16x16 patches", "per_gpu_batch": B,
-                       "units": "block-tokens = blocks x images x tokens per step",
-                       "l2": "flushed between timed steps (256 MB write)", "parallelism": f"replicas x{world}"},
+            "config": workload_config(cfg, world),
             "clocks": clocks, "e2e": e2e, "gpu_launches": launches_per_step * args.steps,
             "roofline": roofline, "kernels": kernels, "kernel_timing": {
                 "method": "CUDA events around each call inside a graph replay of the step, L2 flushed; "
