@@ -9,8 +9,11 @@
 //   orc_sdshiftgelu(_idiv), orc_newton_isqrt, orc_int_layernorm, orc_gemm_requant,
 //   orc_attention, orc_split_conv, orc_deform_attn, orc_patch_embed, orc_requant,
 //   orc_resample_nearest, orc_int_sigmoid, orc_topk, orc_gather_rows, orc_ivit_shiftgelu : pinned.
-//   orc_block_forward : parity unpinned beyond its parts (its composition order and the
-//   residual/window conventions are readings of the paper, not stated by it).
+//   orc_block_forward : its structure (a pre-norm block, two-term residual requantisation, windows
+//   cut from the row-major token grid) is a reading; pinned by reductions and invariants: with
+//   constant branches it is two residual adds, with uniform scores its attention is a closed
+//   form, with a constant hidden layer its MLP is one SD-ShiftGELU value per column, a per-token
+//   offset passes through it, windowed equals global per window, tokens are equivariant.
 // Each operator is written from its mathematics as the cited passage defines it; where the paper
 // proves two forms equal (Constrained Shiftmax's reduced denominator), the plain form is used and
 // a pin checks the other.

@@ -591,6 +591,152 @@ def test_block_equals_composition_of_pinned_parts(orc):
     assert np.array_equal(y2, y)
 
 
+def test_block_with_constant_branches_is_two_residual_adds(orc):
+    """A pre-norm encoder block is x1 = x + Attn(LN1(x)) and y = x1 + MLP(LN2(x1)) (the ViT
+    encoder of Sec. 3.1.1; each add is the two-term requantisation of Sec. 3.2.2).  With the proj
+    and FC2 weights zero, each branch's output is its requantised bias whatever the attention and
+    the MLP compute.  With the first residual scale the identity (m = 2^30, s = 30) and the second
+    3/2 (m = 3 * 2^29, s = 30) the block reduces to per-column constant adds,
+    y = sat16(rq(sat16(x + rq(b_proj)); 3/2) + rq(b_fc2)), computed here with exact rationals.  A
+    residual taken from the wrong tensor (an LN output, or x instead of x1 in the second add), a
+    dropped add or the two residual scales exchanged fails it; two columns saturate on purpose."""
+    B, T, d, H, F = 2, 16, 64, 2, 128
+    bp = synth.block_params(23, 0, d, H, F, 0, "calibrated")
+    bp["w_proj"] = np.zeros_like(bp["w_proj"])
+    bp["w_fc2"] = np.zeros_like(bp["w_fc2"])
+    bp["b_proj"] = synth.uniform_int(23, "cb_proj", (d,), -(1 << 22), 1 << 22)
+    bp["b_fc2"] = synth.uniform_int(23, "cb_fc2", (d,), -(1 << 22), 1 << 22)
+    bp["b_proj"][0], bp["b_fc2"][1] = (1 << 31) - 1, -(1 << 31) + 1
+    bp["m_r1"], bp["s_r1"] = 1 << 30, 30
+    bp["m_r2"], bp["s_r2"] = 3 << 29, 30
+    x = synth.block_input(23, B, T, d)
+    y = orc.block_forward(bp, x, B, T)
+    c1 = [exact_rq(int(bp["b_proj"][c]), int(bp["m_proj"][c]), int(bp["s_proj"][c])) for c in range(d)]
+    c2 = [exact_rq(int(bp["b_fc2"][c]), int(bp["m_fc2"][c]), int(bp["s_fc2"][c])) for c in range(d)]
+    assert max(abs(v) for v in c1) > 0 and max(abs(v) for v in c2) > 0
+    sat = lambda v: max(-32767, min(32767, v))
+    want = np.array([[sat(exact_rq(sat(int(x[i, c]) + c1[c]), 3 << 29, 30) + c2[c]) for c in range(d)]
+                     for i in range(B * T)])
+    assert np.array_equal(y, want)
+    assert want[:, 0].max() == 32767 or want[:, 1].min() == -32767
+
+
+@pytest.mark.parametrize("T,I0", [(4, 1), (64, 1024)])
+def test_block_attention_branch_with_uniform_scores(orc, T, I0):
+    """With the QKV weights zero and the q and k biases zero, every score is 0, so every Shiftmax
+    row is uniform and its outputs are the hand-derived closed forms of
+    tests/golden/shiftmax_closed_forms.txt (rows of T equal scores at this I0).  Attention then
+    averages v, which is the requantised v bias alone: O = sat8(rq(sum_j P * v)), the same for
+    every token and head, and the block's first half is x1 = sat16(rq(W_proj O + b_proj) + rq(x))
+    (numpy int64 matmul, exact rationals).  The MLP branch is silenced (FC1 weights and bias and the
+    FC2 bias zero: SD-ShiftGELU of 0 is 0) with an identity second residual, so y = x1.  v routed from the wrong
+    third of qkv, P ignored, or the proj applied to anything but O fails it."""
+    golden = {(n, i0): out for n, i0, _, _, _, _, _, out in _golden_rows()}
+    P = golden[(T, I0)]
+    B, d, H, F = 2, 64, 2, 128
+    bp = synth.block_params(26, 0, d, H, F, 0, "calibrated")
+    bp["smx"] = dict(bp["smx"], I0=I0)
+    bp["w_qkv"] = np.zeros_like(bp["w_qkv"])
+    bp["b_qkv"] = np.concatenate([np.zeros(2 * d, np.int32),
+                                  synth.uniform_int(26, "bv", (d,), -(1 << 15), 1 << 15)])
+    bp["m_o"], bp["s_o"] = 1 << 30, 37
+    bp["w_fc1"] = np.zeros_like(bp["w_fc1"])
+    bp["b_fc1"] = np.zeros_like(bp["b_fc1"])
+    bp["b_fc2"] = np.zeros_like(bp["b_fc2"])
+    bp["m_r2"], bp["s_r2"] = 1 << 30, 30
+    x = synth.block_input(26, B, T, d)
+    y = orc.block_forward(bp, x, B, T)
+    sat = lambda v, bits: max(-(2 ** (bits - 1) - 1), min(2 ** (bits - 1) - 1, v))
+    v = [sat(exact_rq(int(bp["b_qkv"][2 * d + k]), int(bp["m_qkv"][2 * d + k]), int(bp["s_qkv"][2 * d + k])), 8)
+         for k in range(d)]
+    O = np.array([sat(exact_rq(T * P * v[k], 1 << 30, 37), 8) for k in range(d)], dtype=np.int64)
+    assert len(set(O.tolist())) > 8
+    acc = bp["w_proj"].astype(np.int64) @ O + bp["b_proj"].astype(np.int64)
+    proj = [exact_rq(int(acc[c]), int(bp["m_proj"][c]), int(bp["s_proj"][c])) for c in range(d)]
+    want = np.array([[sat(proj[c] + exact_rq(int(x[i, c]), bp["m_r1"], bp["s_r1"]), 16) for c in range(d)]
+                     for i in range(B * T)])
+    assert np.array_equal(y, want)
+
+
+def test_block_mlp_branch_with_constant_hidden_layer(orc):
+    """With the FC1 weights zero, the hidden layer is the requantised FC1 bias g (one int16 per
+    column, the same for every token), SD-ShiftGELU turns it into h = sat8(rq(g * I_div(g))) (the
+    element-wise operator pinned by brute force above), and the block's second half is
+    y = sat16(rq(W_fc2 h + b_fc2) + rq(x1)) (numpy int64 matmul, exact rationals).  The attention
+    branch is silenced (proj weights and bias zero) with an identity first residual, so x1 = x.
+    The GELU skipped or applied after FC2, or FC2 fed anything but h, fails it."""
+    B, T, d, H, F = 2, 16, 64, 2, 128
+    bp = synth.block_params(27, 0, d, H, F, 0, "calibrated")
+    bp["w_proj"] = np.zeros_like(bp["w_proj"])
+    bp["b_proj"] = np.zeros_like(bp["b_proj"])
+    bp["m_r1"], bp["s_r1"] = 1 << 30, 30
+    bp["w_fc1"] = np.zeros_like(bp["w_fc1"])
+    x = synth.block_input(27, B, T, d)
+    y = orc.block_forward(bp, x, B, T)
+    sat = lambda v, bits: max(-(2 ** (bits - 1) - 1), min(2 ** (bits - 1) - 1, v))
+    g = np.array([[sat(exact_rq(int(bp["b_fc1"][c]), int(bp["m_fc1"][c]), int(bp["s_fc1"][c])), 16)
+                   for c in range(F)]], dtype=np.int32)
+    gi = orc.sdshiftgelu(g, bp["gelu_I0"]).astype(np.int64)[0]
+    h = np.array([sat(exact_rq(int(v), bp["m_g"], bp["s_g"]), 8) for v in gi], dtype=np.int64)
+    assert len(set(h.tolist())) > 8 and h.min() < 0 < h.max()
+    acc = bp["w_fc2"].astype(np.int64) @ h + bp["b_fc2"].astype(np.int64)
+    fc2 = [exact_rq(int(acc[c]), int(bp["m_fc2"][c]), int(bp["s_fc2"][c])) for c in range(d)]
+    want = np.array([[sat(fc2[c] + exact_rq(int(x[i, c]), bp["m_r2"], bp["s_r2"]), 16) for c in range(d)]
+                     for i in range(B * T)])
+    assert np.array_equal(y, want)
+
+
+def test_prenorm_block_follows_a_per_token_offset(orc):
+    """Both branches of a pre-norm block read their token through a LayerNorm, which subtracts the
+    token's mean: adding an integer c to every channel of a token moves its mean by exactly c
+    (the rounded mean of x + c is the rounded mean of x plus c) and leaves the normalised values
+    unchanged.  With identity residual scales the offset then passes through both residual adds
+    alone: block(x + c) = block(x) + c per token, exactly, while no value saturates.  A LayerNorm
+    skipped, placed after a residual add, or a residual taken from a normalised tensor breaks it."""
+    B, T, d, H, F = 2, 16, 64, 2, 128
+    bp = synth.block_params(28, 0, d, H, F, 0, "calibrated")
+    bp["m_r1"], bp["s_r1"] = 1 << 30, 30
+    bp["m_r2"], bp["s_r2"] = 1 << 30, 30
+    x = synth.block_input(28, B, T, d)
+    c = synth.uniform_int(28, "offset", (B * T, 1), -3000, 3000, np.int16)
+    y = orc.block_forward(bp, x, B, T)
+    yc = orc.block_forward(bp, (x + c).astype(np.int16), B, T)
+    assert np.abs(y).max() + 3000 < 32767
+    assert np.array_equal(yc.astype(np.int64), y.astype(np.int64) + c)
+
+
+def test_windowed_block_is_global_block_per_window(orc):
+    """Everything in the block but attention acts on each token alone (LayerNorm over a token's
+    channels, linear layers, SD-ShiftGELU), so a block with 2x2 windowed attention on a 6x6 token
+    grid equals the global-attention block run on each window's tokens, gathered by numpy
+    indexing independently of the oracle's window arithmetic."""
+    B, G, nw, d, H, F = 2, 6, 2, 64, 2, 128
+    T, ws = G * G, G // nw
+    bpw = synth.block_params(24, 0, d, H, F, nw, "calibrated")
+    bpg = dict(bpw, win_side=0)
+    x = synth.block_input(24, B, T, d)
+    yw = orc.block_forward(bpw, x, B, T)
+    for b in range(B):
+        for wy in range(nw):
+            for wx in range(nw):
+                idx = np.array([b * T + (wy * ws + ly) * G + wx * ws + lx for ly in range(ws) for lx in range(ws)])
+                assert np.array_equal(yw[idx], orc.block_forward(bpg, x[idx], 1, ws * ws))
+
+
+def test_global_block_is_token_permutation_equivariant(orc):
+    """Global attention has no token order (the Shiftmax maximum and integer sums over the keys do
+    not depend on their order) and every other step is per token, so permuting an image's tokens
+    permutes the block's output the same way; images are independent of each other."""
+    B, T, d, H, F = 2, 24, 64, 2, 128
+    bp = synth.block_params(25, 0, d, H, F, 0, "calibrated")
+    x = synth.block_input(25, B, T, d)
+    y = orc.block_forward(bp, x, B, T)
+    perm = np.random.default_rng(25).permutation(T)
+    idx = np.concatenate([b * T + perm for b in range(B)])
+    assert np.array_equal(orc.block_forward(bp, x[idx], B, T), y[idx])
+    assert np.array_equal(orc.block_forward(bp, x[T:], 1, T), y[T:])
+
+
 # ----------------------------------------------------------------------------- patch embedding
 def test_patch_embed_is_patch_matmul(orc):
     """A stride-p, kernel-p convolution equals a matmul of non-overlapping patches: numpy
