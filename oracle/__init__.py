@@ -11,10 +11,12 @@ Sec. 3.3 (I-LayerNorm) and Sec. 3.1.1 (nearest-neighbour deformable sampling).
 
 Parity status of the compositions written here in Python from the pinned C++ operators:
 ``projector``, ``decoder_layer``, ``detection_head``, ``refine_references``, ``decoder_stack``,
-``two_stage`` and ``query_pos`` are parity unpinned beyond their parts and the invariants that
-tests/test_oracle_pins.py checks for them (query-permutation equivariance, image independence,
-reduction to the reference sigmoid and to fixed references, selection of the best tokens,
-row-wise application): their structure is a reading of the paper, which does not state it.
+``two_stage`` and ``query_pos`` follow a reading of the paper, which does not state their
+structure; tests/test_oracle_pins.py pins them by reductions to closed forms (the decoder layer
+with constant branches, uniform self-attention scores, or one sampling point at pixel centres; the
+projector with identity scales; the head and the refinement with a zero last box layer; the
+plain 4-column query projection) and by invariants (query-permutation equivariance, image
+independence, selection of the best tokens, row-wise application).
 """
 from __future__ import annotations
 

@@ -815,6 +815,28 @@ def test_projector_levels_are_resampled_convolutions(orc):
     assert mem.shape[1] == s8 + s16 + s32
 
 
+def test_projector_with_identity_scales_is_one_conv_over_the_concatenated_taps(orc):
+    """With every tap's requantisation and every branch rescale the identity (m = 2^30, s = 30;
+    tap values inside the int8 range), a projector level at the tapped grid's own size is one 1x1
+    convolution over the taps' channels concatenated in tap order, sat8(rq(sum_b X_b W_b^T + bias))
+    (Table 7's single-convolution baseline; numpy int64 matmul, exact rationals), laid out image by
+    image.  Taps taken in another order, branches paired with the wrong weights or a dropped bias
+    fail it."""
+    B, g, K, N = 2, 6, 32, 24
+    pp = synth.projector_params(8, 3, K, N=N, levels=1)
+    pp["taps"] = [(1 << 30, 30)] * 3
+    lv = pp["levels"][0]
+    lv["m_b"], lv["s_b"] = [1 << 30] * 3, [30] * 3
+    lv["s"] = np.full(N, 40, np.int32)
+    taps = [synth.uniform_int(8 + i, "tap", (B * g * g, K), -127, 127, np.int16) for i in range(3)]
+    mem = orc.projector(pp, taps, B, g, ((g, g),))
+    X = np.concatenate(taps, axis=1)
+    W = np.concatenate(lv["w"], axis=1)
+    want = _exact_linear(X, W, lv["b"], lv["m"], lv["s"], 8)
+    assert len(np.unique(want)) > 50
+    assert np.array_equal(mem.astype(np.int64), want)
+
+
 def _small_decoder(seed=0, B=2, Q=20):
     from paper_2607_24981_gb300 import synth
 
@@ -850,6 +872,126 @@ def test_decoder_layer_images_are_independent(orc):
         one = orc.decoder_layer(dp, inp["tgt"][r], inp["pos"][r], mem[b * 80:(b + 1) * 80], levels,
                                 inp["refs"][b:b + 1], 1, Q)
         assert np.array_equal(one, out[r])
+
+
+def _exact_linear(A, W, bias, mult, shift, bits):
+    """sat_bits(rq(A W^T + bias)) per element: numpy int64 matmul, exact rational rounding."""
+    acc = A.astype(np.int64) @ W.astype(np.int64).T + np.asarray(bias, np.int64)
+    lim = 2 ** (bits - 1) - 1
+    return np.array([[max(-lim, min(lim, exact_rq(int(acc[i, c]), int(mult[c]), int(shift[c]))))
+                      for c in range(acc.shape[1])] for i in range(acc.shape[0])], dtype=np.int64)
+
+
+def _exact_requant(X, m, s, bits):
+    lim = 2 ** (bits - 1) - 1
+    return np.array([[max(-lim, min(lim, exact_rq(int(v), m, s))) for v in row] for row in X], dtype=np.int64)
+
+
+def _silence(dp, *branches):
+    """Zero the output projection (weights and bias) of the named decoder branches and make their
+    residual scale the identity (m = 2^30, s = 30), so each named branch passes its input through."""
+    names = {"self": ("w_o", "b_o", "r1"), "cross": ("w_o2", "b_o2", "r2"), "ffn": ("w_fc2", "b_fc2", "r3")}
+    for b in branches:
+        w, bias, r = names[b]
+        dp[w] = np.zeros_like(dp[w])
+        dp[bias] = np.zeros_like(dp[bias])
+        dp["m_" + r], dp["s_" + r] = 1 << 30, 30
+
+
+def _ln(orc, dp, i, x):
+    """The decoder's LayerNorm i (the pinned operator; 20 Newton steps, int16 out)."""
+    return orc.int_layernorm(x, dp[f"ln{i}_beta"], dp[f"ln{i}_mult"], dp[f"ln{i}_shift"], 20, 16).astype(np.int64)
+
+
+def test_decoder_layer_with_constant_branches_is_a_post_norm_chain(orc):
+    """A post-norm decoder layer (Deformable-DETR order, Sec. 3.1.1) is t1 = LN1(tgt + SelfAttn),
+    t2 = LN2(t1 + CrossAttn), out = LN3(t2 + FFN).  With every branch's output projection zero
+    its output is its requantised bias, and with identity residual scales the layer reduces to
+    LayerNorms (the operator pinned above) of constant per-column adds:
+    out = LN3(LN2(LN1(tgt + c1) + c2) + c3).  A residual from the wrong tensor, a LayerNorm
+    skipped or moved before its branch (pre-norm) fails it."""
+    B, Q = 2, 20
+    dp, inp, levels, mem = _small_decoder(3, B, Q)
+    _silence(dp, "self", "cross", "ffn")
+    d = dp["d"]
+    cs = {}
+    for k, (b, m, s_) in {"c1": ("b_o", "m_oc", "s_oc"), "c2": ("b_o2", "m_o2", "s_o2"),
+                          "c3": ("b_fc2", "m_fc2", "s_fc2")}.items():
+        dp[b] = synth.uniform_int(29, k, (d,), -(1 << 15), 1 << 15)
+        cs[k] = np.array([exact_rq(int(dp[b][c]), int(dp[m][c]), int(dp[s_][c])) for c in range(d)], np.int64)
+        assert 100 < np.abs(cs[k]).max() < 8000
+    out = orc.decoder_layer(dp, inp["tgt"], inp["pos"], mem, levels, inp["refs"], B, Q)
+    sat = lambda v: np.clip(v, -32767, 32767)
+    x1 = inp["tgt"].astype(np.int64) + cs["c1"]
+    assert np.abs(x1).max() < 32767
+    t1 = _ln(orc, dp, 1, x1)
+    t2 = _ln(orc, dp, 2, sat(t1 + cs["c2"]))
+    want = _ln(orc, dp, 3, sat(t2 + cs["c3"]))
+    assert np.array_equal(out.astype(np.int64), want)
+
+
+@pytest.mark.parametrize("Q,I0", [(4, 1), (64, 1024)])
+def test_decoder_self_attention_with_uniform_scores_averages_v(orc, Q, I0):
+    """With the q|k projection zero every score is 0 and every Shiftmax row of the Q queries is
+    uniform, its outputs the hand-derived closed form of tests/golden/shiftmax_closed_forms.txt.
+    Self-attention then gives every query of an image the same O = sat8(rq(P sum_j v_j)), with
+    v = sat8(rq(W_v sat8(rq(tgt)) + b_v)) from tgt alone (no positional term), and
+    t1 = LN1(sat16(rq(W_o O + b_o) + rq(tgt))); the other two branches pass through, so
+    out = LN3(LN2(t1)).  Recomputed with numpy int64 matmuls and exact rationals; v taken from the
+    positional query, P ignored or the residual from the wrong tensor fails it."""
+    golden = {(n, i0): out for n, i0, _, _, _, _, _, out in _golden_rows()}
+    P = golden[(Q, I0)]
+    B = 2
+    dp, inp, levels, mem = _small_decoder(4, B, Q)
+    d, H = dp["d"], dp["H"]
+    _silence(dp, "cross", "ffn")
+    dp["w_qk"] = np.zeros_like(dp["w_qk"])
+    dp["b_qk"] = np.zeros_like(dp["b_qk"])
+    dp["smx"] = dict(dp["smx"], I0=I0)
+    dp["m_o"], dp["s_o"] = 1 << 30, 37
+    out = orc.decoder_layer(dp, inp["tgt"], inp["pos"], mem, levels, inp["refs"], B, Q)
+    v_in = _exact_requant(inp["tgt"], dp["m_v1"], dp["s_v1"], 8)
+    v = _exact_linear(v_in, dp["w_v"], dp["b_v"], dp["m_v"], dp["s_v"], 8)
+    O = np.concatenate([np.tile([max(-127, min(127, exact_rq(int(P * t), 1 << 30, 37)))
+                                 for t in v[b * Q:(b + 1) * Q].sum(0)], (Q, 1)) for b in range(B)])
+    assert len(set(O[0].tolist())) > 8
+    x1 = np.clip(_exact_linear(O, dp["w_o"], dp["b_o"], dp["m_oc"], dp["s_oc"], 64)
+                 + _exact_requant(inp["tgt"], dp["m_r1"], dp["s_r1"], 64), -32767, 32767)
+    want = _ln(orc, dp, 3, _ln(orc, dp, 2, _ln(orc, dp, 1, x1)))
+    assert np.array_equal(out.astype(np.int64), want)
+
+
+def test_decoder_cross_attention_at_pixel_centres_reads_the_reference_pixel(orc):
+    """Deformable cross-attention with one level and one point per head (L = P = 1) and zero
+    offsets samples the value map at the reference point alone; with references at pixel centres
+    ((2x + 1) / 2W of the width) that is pixel (x, y) under any nearest-neighbour rule, and a
+    Shiftmax row of one element is the closed form for n = 1 (every weight 127 at I0 = 1, from
+    tests/golden/shiftmax_closed_forms.txt).  So samp = sat8(rq(127 value[pixel])) with
+    value = sat8(rq(memory W_val + b_val)), t2 = LN2(sat16(rq(W_o2 samp + b_o2) + rq(t1))) with
+    t1 = LN1(tgt) (self-attention silenced) and out = LN3(t2) (FFN silenced).  Recomputed with
+    numpy indexing and int64 matmuls; a wrong level offset, the x and y axes exchanged, the value
+    projection skipped or the residual from the wrong tensor fails it."""
+    B, Q, Hl, Wl = 2, 12, 8, 8
+    dp = synth.decoder_params(5, 0, d=64, H=2, F=128, L=1, P=1)
+    inp = synth.decoder_inputs(5, B, Q, 64)
+    d, H = dp["d"], dp["H"]
+    mem = synth.laplace_int(5, "mem", (B * Hl * Wl, d), 20.0, 127, np.int8)
+    _silence(dp, "self", "ffn")
+    dp["w_off"] = np.zeros_like(dp["w_off"])
+    dp["b_off"] = np.zeros_like(dp["b_off"])
+    dp["smx_w"] = dict(dp["smx_w"], I0=1)
+    px = synth.uniform_int(5, "px", (B, Q, 2), 0, Wl - 1)
+    refs = ((2 * px + 1) << 15) // Wl
+    out = orc.decoder_layer(dp, inp["tgt"], inp["pos"], mem, ((Hl, Wl),), refs.astype(np.int32), B, Q)
+    value = _exact_linear(mem, dp["w_val"], dp["b_val"], dp["m_val"], dp["s_val"], 8)
+    rows = np.array([b * Hl * Wl + px[b, q, 1] * Wl + px[b, q, 0] for b in range(B) for q in range(Q)])
+    samp = _exact_requant(127 * value[rows], dp["m_s"], dp["s_s"], 8)
+    assert np.abs(samp).max() > 20
+    t1 = _ln(orc, dp, 1, inp["tgt"].astype(np.int64))
+    x2 = np.clip(_exact_linear(samp, dp["w_o2"], dp["b_o2"], dp["m_o2"], dp["s_o2"], 64)
+                 + _exact_requant(t1, dp["m_r2"], dp["s_r2"], 64), -32767, 32767)
+    want = _ln(orc, dp, 3, _ln(orc, dp, 2, x2))
+    assert np.array_equal(out.astype(np.int64), want)
 
 
 # ----------------------------------------------------------------------------- detection head, two-stage
