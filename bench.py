@@ -28,8 +28,8 @@ METRIC = "int-only encoder block tokens/s (1600 tok, d=384)"
 UNIT = "block-tokens/s"
 WORKLOAD = "medium_c2"
 SEED = 0
-# cpu baseline / reference arm sample: one image through blocks 0..4 (3 window + 2 global, the
-# backbone's 6:4 window/global ratio)
+# cpu baseline sample: each image through blocks 0..4 (3 window + 2 global, the backbone's 6:4
+# window/global ratio); the reference arm instead cycles over all 10 blocks, one block per step
 CPU_SAMPLE_BLOCKS = 5
 
 
