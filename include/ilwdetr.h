@@ -14,6 +14,8 @@
  *     ilwdetr_last_error() (thread-local).  Argument errors are reported before anything is
  *     launched.  Device-side failures that the kernels detect (a bounded wait that ran out)
  *     are latched in a device status word and reported by ilwdetr_device_status().
+ *   - A call whose batch, row, token or element count is 0 checks its scalar parameters, returns
+ *     ILW_OK and launches nothing; its tensor pointers may then be NULL.
  *   - rq(v; m, s) = (v*m + 2^(s-1)) >> s, arithmetic shift (dyadic requantisation, Sec. 3.2.2,
  *     round half up); satN clips to the symmetric range [-(2^(N-1)-1), 2^(N-1)-1] (Sec. 3.2.1).
  *     Per-channel `mult` is int32 (sign allowed), `shift` is int32 in [1, 62]; values outside

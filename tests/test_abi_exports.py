@@ -261,3 +261,41 @@ def test_int8_tcgen05_mma_is_not_available_on_sm103a(tmp_path):
     rc8, msg = compile_kind("i8")
     assert rc16 == 0
     assert rc8 != 0 and "kind::i8" in msg and "sm_103a" in msg, msg
+
+
+def test_empty_extents_return_ok_without_a_launch(built_lib):
+    """A call whose batch, row, token or element count is 0 checks its scalar parameters and
+    returns ILW_OK without launching anything (its tensor pointers may be NULL), so it also
+    succeeds on a machine without a device."""
+    import paper_2607_24981_gb300 as ilw
+
+    L = ilw.lib()
+    smx = ctypes.byref(ilw.ShiftmaxT(100, 16, 8, -1, 4, 31))
+    g = ctypes.byref(ilw.GeluT(600, 16, 8))
+    calls = {
+        "gemm_requant M=0": lambda: L.ilwdetr_gemm_requant(None, 16, None, None, None, None, 0, 4, 16, 8, None, 4, None, None),
+        "gemm_requant N=0": lambda: L.ilwdetr_gemm_requant(None, 16, None, None, None, None, 4, 0, 16, 8, None, 4, None, None),
+        "gemm_gelu M=0": lambda: L.ilwdetr_gemm_gelu(None, 16, None, None, None, None, 0, 4, 16, g, 1 << 30, 31, None, 4, None),
+        "shiftmax_rows rows=0": lambda: L.ilwdetr_shiftmax_rows(None, 4, 0, 4, smx, None, 4, None),
+        "shiftmax_rows len=0": lambda: L.ilwdetr_shiftmax_rows(None, 4, 4, 0, smx, None, 4, None),
+        "sdshiftgelu n=0": lambda: L.ilwdetr_sdshiftgelu(None, None, 0, g, None),
+        "int_layernorm rows=0": lambda: L.ilwdetr_int_layernorm(None, 16, 64, 0, 64, None, None, None, 10, None, 8, 64, None),
+        "shiftmax_attn B=0": lambda: L.ilwdetr_shiftmax_attn(None, None, None, 192, 8, 0, 64, 3, 64, 0, smx, 1 << 30, 31,
+                                                             None, 8, 192, None),
+        "shiftmax_attn T=0": lambda: L.ilwdetr_shiftmax_attn(None, None, None, 192, 8, 1, 0, 3, 64, 0, smx, 1 << 30, 31,
+                                                             None, 8, 192, None),
+        "int_sigmoid n=0": lambda: L.ilwdetr_int_sigmoid(None, None, 0, ctypes.byref(ilw.SigmoidT(1024, 8, 17)), None),
+        "relu_i8 n=0": lambda: L.ilwdetr_relu_i8(None, None, 0, None),
+        "topk rows=0": lambda: L.ilwdetr_topk(None, 10, 0, 10, 3, None, None, None),
+        "gather_rows n=0": lambda: L.ilwdetr_gather_rows(None, 16, 5, None, 0, 16, None, 16, None),
+        "requant rows=0": lambda: L.ilwdetr_requant(None, 16, 16, 0, 16, 1 << 30, 30, None, 0, 1, 0, 1, 8, None, 16, None),
+        "resample_nearest B=0": lambda: L.ilwdetr_resample_nearest(None, 100, 0, 10, 10, 16, None, 400, 20, 20, None),
+        "ivit_shiftgelu rows=0": lambda: L.ilwdetr_ivit_shiftgelu(None, 8, 0, 8, None, 8, g, None),
+        "patch_embed B=0": lambda: L.ilwdetr_patch_embed(None, 0, 3, 640, 640, 16, None, None, None, None, 384, None,
+                                                         1 << 30, 31, None, None, 0, None),
+        "patch_embed_noalloc B=0": lambda: L.ilwdetr_patch_embed_noalloc(None, 0, 3, 640, 640, 16, None, None, None, None,
+                                                                         384, None, 1 << 30, 31, None, None),
+        "pack_weight N=0": lambda: L.ilwdetr_pack_weight(None, 0, 16, None, None),
+    }
+    for name, call in calls.items():
+        assert call() == 0, (name, L.ilwdetr_last_error())
