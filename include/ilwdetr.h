@@ -25,7 +25,10 @@
  *   - The library keeps a few arrays of its own in device memory (the status word, the
  *     SD-ShiftGELU tables, the allocation-free patch scratch) and looks up their device
  *     addresses once per device.  A cudaDeviceReset ends the context those addresses belong
- *     to: do not call the library across one.
+ *     to: do not call the library across one.  The SD-ShiftGELU GEMM epilogue keeps one 64 KB
+ *     output table per distinct (I0, k_inter, k_out, m_g, s_g) for the life of the process, up
+ *     to 256 per device; a GEMM with a further parameter set fails with ILW_ERR_CUDA (out of
+ *     memory) and launches nothing.
  */
 #ifndef ILWDETR_H
 #define ILWDETR_H

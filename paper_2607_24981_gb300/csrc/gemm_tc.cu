@@ -10,8 +10,10 @@ namespace {
 
 // SD-ShiftGELU output tables, one slot per parameter set (I0, k_inter, k_out, m_g, s_g): entry
 // g + 32767 is sat8(rq(g * I_div(g); m_g, s_g)) for every int16 value g (Algorithm 1 followed by the
-// output requantisation), a pure function of g.
-constexpr int kGeluSlots = 32;
+// output requantisation), a pure function of g.  A slot, once given to a parameter set, keeps it
+// for the life of the process: kernels in flight on other streams and captured graphs hold its
+// address, so it is never rebuilt for another set.  A parameter set beyond the last slot is refused.
+constexpr int kGeluSlots = 256;  // 16 MiB per device
 constexpr int kGeluTabBytes = 65536;  // 65535 entries, padded to 16 bytes
 __device__ __align__(16) int8_t g_gelu_tab[kGeluSlots][kGeluTabBytes];
 
@@ -25,7 +27,9 @@ __global__ void gelu_table_kernel(int8_t *tab, GeluC c, int32_t m_g, int32_t s_g
 
 // The table slot of (device, GELU constants, m_g, s_g), built on first use.  The first build of a
 // slot is waited for (unless the stream is being captured), so a slot marked built is complete for
-// every stream; a build recorded into a graph is repeated by each replay until an eager call builds it.
+// every stream; a build recorded into a graph is repeated by each replay until an eager call builds it
+// (every replay writes the same bytes, since the slot never changes hands).  With every slot taken,
+// a new parameter set gets cudaErrorMemoryAllocation and nothing is launched.
 const int8_t *gelu_table_impl(const GeluC &c, int32_t m_g, int32_t s_g, cudaStream_t s, cudaError_t *err) {
     struct Key {
         int dev;
@@ -36,8 +40,8 @@ const int8_t *gelu_table_impl(const GeluC &c, int32_t m_g, int32_t s_g, cudaStre
     };
     static std::mutex mu;
     static Key keys[64][kGeluSlots];
-    static bool used[64][kGeluSlots] = {}, built[64][kGeluSlots] = {};
-    static int next[64] = {};
+    static bool built[64][kGeluSlots] = {};
+    static int nused[64] = {};
     static int8_t *base[64] = {};
     *err = cudaSuccess;
     int dev = 0;
@@ -54,13 +58,15 @@ const int8_t *gelu_table_impl(const GeluC &c, int32_t m_g, int32_t s_g, cudaStre
     }
     const Key key{dev, c.se.I0, c.se.k, c.out_sh, m_g, s_g};
     int slot = -1;
-    for (int i = 0; i < kGeluSlots; ++i)
-        if (used[dev][i] && keys[dev][i] == key) slot = i;
+    for (int i = 0; i < nused[dev]; ++i)
+        if (keys[dev][i] == key) slot = i;
     if (slot < 0) {
-        slot = next[dev];
-        next[dev] = (next[dev] + 1) % kGeluSlots;
+        if (nused[dev] >= kGeluSlots) {
+            *err = cudaErrorMemoryAllocation;
+            return nullptr;
+        }
+        slot = nused[dev]++;
         keys[dev][slot] = key;
-        used[dev][slot] = true;
         built[dev][slot] = false;
     }
     int8_t *tab = base[dev] + (size_t)slot * kGeluTabBytes;
