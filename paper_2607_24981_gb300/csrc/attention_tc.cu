@@ -880,15 +880,13 @@ bool kv_map(CUtensorMap *m, const void *base, const AttnParams &p, bool win, int
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// One instantiation's launch; its shared-memory limit is raised once.
+// One instantiation's launch; its shared-memory limit (the same for every launch) is raised once
+// per device.
 template <bool FASTQ, bool DIRECT, bool SUM4, bool MAYPAIR, bool MAYFULL>
 cudaError_t launch_tc_one(const TcArgs &a, dim3 grid, size_t smem, cudaStream_t s) {
-    static std::once_flag once;
-    static cudaError_t attr = cudaSuccess;
-    std::call_once(once, [&] {
-        attr = cudaFuncSetAttribute(attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR, MAYFULL>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    });
+    static SmemLimit limit;
+    const cudaError_t attr =
+        raise_smem_limit(limit, (const void *)attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR, MAYFULL>, (int)smem);
     if (attr != cudaSuccess) return attr;
     attn_tc_kernel<FASTQ, DIRECT, SUM4, MAYPAIR, MAYFULL><<<grid, kThreadsTc, smem, s>>>(a);
     return cudaGetLastError();

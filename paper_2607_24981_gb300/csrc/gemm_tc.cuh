@@ -986,12 +986,9 @@ cudaError_t launch_tc(TcParams<NB> &tp, cudaStream_t s) {
     if (tp.tma_store && smem_bytes<BN, STAGES, KIND, AF16, WRES>(tp.wres_bytes, stg) > kSmemMax) tp.tma_store = 0;
     const size_t smem = smem_bytes<BN, STAGES, KIND, AF16, WRES>(tp.wres_bytes, tp.tma_store ? stg : 0);
     if (smem > kSmemMax) return cudaErrorInvalidValue;
-    static std::once_flag once;
-    static cudaError_t attr_err = cudaSuccess;
-    std::call_once(once, [&] {
-        attr_err = cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, KIND, NB, AF16, WRES>,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMax);
-    });
+    static SmemLimit limit;
+    const cudaError_t attr_err =
+        raise_smem_limit(limit, (const void *)gemm_tc_kernel<BN, STAGES, KIND, NB, AF16, WRES>, (int)kSmemMax);
     if (attr_err != cudaSuccess) return attr_err;
     int grid = tp.tiles < num_sms() ? tp.tiles : num_sms();
     if (WRES) {  // a multiple of tiles_n: every CTA keeps one n block of W

@@ -1,6 +1,7 @@
 // ilw_kernels.h -- internal launch interface between the C-ABI layer and the kernels.
 #pragma once
 #include <cstdint>
+#include <mutex>
 #include <cuda_runtime.h>
 
 #include "ilw_device.cuh"
@@ -16,6 +17,25 @@ int *status_word_ptr();
 cudaError_t read_and_clear_status(int *value);
 // Streaming multiprocessors of the current device (read from the device once per device).
 int sm_count();
+
+// A kernel's dynamic shared-memory limit, raised once per device: a function attribute belongs
+// to the device it was set on, so each device of the process gets its own call.  One SmemLimit
+// (a function-local static) per kernel; later calls on a device return its first call's result.
+constexpr int kMaxAttrDevices = 64;
+struct SmemLimit {
+    std::once_flag once[kMaxAttrDevices];
+    cudaError_t err[kMaxAttrDevices] = {};
+};
+inline cudaError_t raise_smem_limit(SmemLimit &st, const void *kernel, int bytes) {
+    int dev = 0;
+    const cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxAttrDevices) return cudaErrorInvalidDevice;
+    std::call_once(st.once[dev], [&] {
+        st.err[dev] = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    });
+    return st.err[dev];
+}
 constexpr int kStatusTimeoutTma = 1;     // a wait for a TMA load ran out
 constexpr int kStatusTimeoutMma = 2;     // a wait for tensor-core completion ran out
 constexpr int kStatusTimeoutOperand = 3; // a wait for the converted operand ran out

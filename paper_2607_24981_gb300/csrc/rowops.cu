@@ -626,12 +626,9 @@ cudaError_t launch_sdshiftgelu(const int32_t *X, int32_t *Y, int64_t n, const Ge
         if (n4 && bound <= 32767.0 && n4 >= (1 << 16)) {
             const int32_t T = (int32_t)bound;
             const int smem = 2 * T + 1;
-            static bool attr = false;
-            if (!attr) {
-                cudaError_t e = cudaFuncSetAttribute(sdshiftgelu_table, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536);
-                if (e != cudaSuccess) return e;
-                attr = true;
-            }
+            static SmemLimit limit;
+            const cudaError_t e = raise_smem_limit(limit, (const void *)sdshiftgelu_table, 65536);
+            if (e != cudaSuccess) return e;
             int64_t blocks = (n4 + 255) / 256;
             if (blocks > 6 * (int64_t)sm_count()) blocks = 6 * (int64_t)sm_count();
             sdshiftgelu_table<<<(unsigned)blocks, 256, smem, s>>>((const int4 *)X, (int4 *)Y, n4, c, T);
