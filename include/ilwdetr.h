@@ -95,8 +95,9 @@ typedef struct {
 /* Bytes of the packed form of an int8 weight W[N, K] (row-major, K contiguous). */
 size_t ilwdetr_packed_weight_bytes(int32_t N, int32_t K);
 /* Packs W (device, int8 [N, K], leading dimension K) into `packed` (device, bytes given by
- * ilwdetr_packed_weight_bytes).  Done once per weight; the values stay the same integers.
- * K must be a multiple of 16. */
+ * ilwdetr_packed_weight_bytes).  Done once per weight; the values stay the same integers (the
+ * paper has no counterpart: this is the tensor cores' operand form of the int8 weights of
+ * Sec. 3.2.1's integer linear layers).  K must be a multiple of 16. */
 int ilwdetr_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, ilw_stream_t stream);
 
 /* Integer linear layer with fused bias and dyadic requantisation (Sec. 3.2.1, the equation
@@ -125,7 +126,7 @@ int ilwdetr_gemm_gelu(const int8_t *A, int64_t lda, const void *Wp, const int32_
                       const ilw_gelu_t *gelu, int32_t m_g, int32_t s_g, int8_t *H, int64_t ldh,
                       ilw_stream_t stream);
 
-/* The integer linear layer in its general form: the computation of ilwdetr_gemm_requant
+/* The integer linear layer (Sec. 3.2.1) in its general form: the computation of ilwdetr_gemm_requant
  * (epilogue ILW_EPI_REQUANT) or of ilwdetr_gemm_gelu (ILW_EPI_GELU), with the activation operand
  * A either int8 (a_form 8; lda % 16 == 0) or the same int8 values carried in fp16 (a_form
  * ILW_I8_IN_F16; fp16 [M, lda], lda % 8 == 0), which the tensor cores read directly.  out_bits:
@@ -300,7 +301,9 @@ typedef struct {
 
 /* Workspace bytes ilwdetr_block_forward needs for B*T tokens. */
 size_t ilwdetr_block_workspace_bytes(int32_t B, int32_t T, int32_t d, int32_t F);
-/* One encoder block: x int16 [B*T, d] -> y int16 [B*T, d] (x and y may not alias).
+/* One encoder block (the ViT encoder of Sec. 3.1.1 with the integer operators of Sec. 3.2-3.3;
+ * global or window attention as Table 1 assigns per layer): x int16 [B*T, d] -> y int16
+ * [B*T, d] (x and y may not alias).
  * `workspace` is a device buffer of at least ilwdetr_block_workspace_bytes (256-byte aligned). */
 int ilwdetr_block_forward(const ilw_block_params_t *p, const int16_t *x, int16_t *y, int32_t B,
                           int32_t T, void *workspace, size_t workspace_bytes, ilw_stream_t stream);
@@ -321,8 +324,9 @@ int ilwdetr_requant(const void *X, int32_t in_bits, int64_t ldx, int64_t rows, i
                     int32_t s1, const int16_t *Z, int64_t ldz, int64_t z_rows, int32_t m2, int32_t s2,
                     int32_t out_bits, void *Y, int64_t ldy, ilw_stream_t stream);
 
-/* Nearest-neighbour resampling of B int8 feature maps (the projector's strides 8 / 16 / 32 read as
- * nearest resampling of the stride-16 encoder grid; a 1x1 convolution commutes with it):
+/* Nearest-neighbour resampling of B int8 feature maps (the multi-scale projector of Sec. 3.2.2 and
+ * Table 1: its strides 8 / 16 / 32 read as nearest resampling of the stride-16 encoder grid; a 1x1
+ * convolution commutes with it):
  *   Y[b][y*Wo + x, :] = X[b][floor(y*Hi/Ho)*Wi + floor(x*Wi/Wo), :]
  *   X int8, map b starts at row b*x_bstride of C channels; Y likewise with y_bstride (so the
  *   levels can be written into one concatenated decoder memory).  C % 16 == 0, 16-byte aligned. */
@@ -410,16 +414,18 @@ int ilwdetr_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, const ilw_sigmo
 int ilwdetr_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int32_t L, int32_t *Y, int64_t ldy,
                            const ilw_gelu_t *p, ilw_stream_t stream);
 
-/* ReLU of int8 values: Y = max(X, 0).  X, Y device [n] (may alias), 4-byte aligned. */
+/* ReLU of int8 values (the hidden layers of the detection head's box branch, Table 5):
+ * Y = max(X, 0).  X, Y device [n] (may alias), 4-byte aligned. */
 int ilwdetr_relu_i8(const int8_t *X, int8_t *Y, int64_t n, ilw_stream_t stream);
 
-/* Integer top-K (two-stage query selection): for each of `rows` rows of S (int32, leading dimension
+/* Integer top-K (the two-stage query selection of Sec. 3.1.2): for each of `rows` rows of S (int32, leading dimension
  * lds), the K largest of its first N values in decreasing order, equal values ordered by
  * increasing index.  vals, idx int32 [rows, K] device.  1 <= K <= N <= 16384. */
 int ilwdetr_topk(const int32_t *S, int64_t lds, int32_t rows, int32_t N, int32_t K, int32_t *vals,
                  int32_t *idx, ilw_stream_t stream);
 
-/* Row gather: dst row i = src row idx[i], i < n (row_bytes bytes each; leading dimensions in
+/* Row gather (the selected tokens' memory rows and anchors of the two-stage selection, Sec. 3.1.2):
+ * dst row i = src row idx[i], i < n (row_bytes bytes each; leading dimensions in
  * bytes).  src, dst, idx device; row_bytes, src_ld, dst_ld multiples of 4, pointers 4-byte
  * aligned.  An index outside [0, src_rows) gives a zero row and is reported by the next
  * ilwdetr_device_status. */
