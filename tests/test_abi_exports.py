@@ -299,3 +299,27 @@ def test_empty_extents_return_ok_without_a_launch(built_lib):
     }
     for name, call in calls.items():
         assert call() == 0, (name, L.ilwdetr_last_error())
+
+
+def test_product_fails_loudly_without_the_library(monkeypatch):
+    """With libilwdetr.so absent the binding raises instead of computing anything elsewhere: there
+    is no CPU fallback."""
+    import paper_2607_24981_gb300 as ilw
+
+    monkeypatch.setattr(ilw, "_lib", None)
+    monkeypatch.setattr(ilw, "LIB_PATH", os.path.join(os.path.dirname(ilw.LIB_PATH), "absent", "libilwdetr.so"))
+    with pytest.raises(ilw.IlwError, match="missing"):
+        ilw.lib()
+
+
+def test_product_sources_never_reach_the_oracle():
+    """The product package and the C-ABI header neither import, link nor name the oracle."""
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    pkg = os.path.join(root, "paper_2607_24981_gb300")
+    files = [os.path.join(dp, f) for dp, _, fs in os.walk(pkg) for f in fs if f.endswith((".py", ".cu", ".cuh", ".h"))]
+    files.append(os.path.join(root, "include", "ilwdetr.h"))
+    assert len(files) > 10
+    for path in files:
+        text = open(path).read()
+        for needle in ("import oracle", "from oracle", "ilw_oracle", "libilw_oracle"):
+            assert needle not in text, (path, needle)
