@@ -323,3 +323,16 @@ def test_product_sources_never_reach_the_oracle():
         text = open(path).read()
         for needle in ("import oracle", "from oracle", "ilw_oracle", "libilw_oracle"):
             assert needle not in text, (path, needle)
+
+
+def test_oracle_sources_never_reach_the_product():
+    """The oracle (Python wrapper and C++ source) neither imports nor links the product package or
+    its CUDA library; tests hand it the same seeded arrays they hand the GPU path."""
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    odir = os.path.join(root, "oracle")
+    files = [os.path.join(odir, f) for f in os.listdir(odir) if f.endswith((".py", ".cpp", ".h"))]
+    assert len(files) >= 3
+    for path in files:
+        text = open(path).read()
+        for needle in ("paper_2607_24981_gb300", "libilwdetr", "ilwdetr.h", "cuda"):
+            assert needle not in text, (path, needle)
