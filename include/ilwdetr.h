@@ -263,6 +263,15 @@ int ilwdetr_patch_embed_noalloc(const int8_t *img, int32_t B, int32_t Cin, int32
                                 const int32_t *shift, int32_t d, const int16_t *pos, int32_t m_pos,
                                 int32_t s_pos, int16_t *x0, ilw_stream_t stream);
 
+/* Argument validation without launching (the paper has no counterpart; off by default).  While
+ * `on` is non-zero for the calling thread, every entry point that launches kernels (the operators,
+ * the composite block, decoder-layer and patch-embedding calls, ilwdetr_patch_embed_noalloc and
+ * ilwdetr_pack_weight) checks its arguments exactly as usual and then returns ILW_OK, or the error
+ * it found, without any CUDA call that launches work or touches device memory.  Composite calls
+ * check every step.  Lets a host runtime validate a whole schedule ahead of time, and works on a
+ * machine without a device.  Call ilwdetr_validate_only(0) to launch again.  Always ILW_OK. */
+int ilwdetr_validate_only(int32_t on);
+
 /* Test hook of the bounded device waits (the paper has no counterpart; off by default).  Every
  * wait inside the kernels is bounded; when one runs out the kernel latches the device status word,
  * stops, drains the copies it issued, frees its tensor memory and returns, and

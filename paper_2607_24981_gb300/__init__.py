@@ -116,6 +116,7 @@ SIGNATURES = {
     "ilwdetr_version": ([], C.c_char_p),
     "ilwdetr_last_error": ([], C.c_char_p),
     "ilwdetr_device_status": ([_VP], C.c_int),
+    "ilwdetr_validate_only": ([_I32], C.c_int),
     "ilwdetr_debug_gemm_wait": ([_I32, C.c_int64], C.c_int),
     "ilwdetr_packed_weight_bytes": ([_I32, _I32], C.c_size_t),
     "ilwdetr_pack_weight": ([_VP, _I32, _I32, _VP, _VP], C.c_int),

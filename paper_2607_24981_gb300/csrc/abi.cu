@@ -26,7 +26,8 @@ int fail(int code, const char *fmt, ...) {
 // Composite entry points (the patch embedding, the encoder block, the decoder layer) run their
 // steps twice: first with every launch suppressed, which checks each step's arguments with the
 // step's own validation, then for real; so an argument error in a later step is reported before
-// the first launch.  Each entry point's launch is skipped (ILW_OK) while g_check_only is set.
+// the first launch.  Each entry point's launch is skipped (ILW_OK) while g_check_only is set;
+// ilwdetr_validate_only sets it for the calling thread until it is cleared again.
 thread_local bool g_check_only = false;
 struct CheckPass {
     CheckPass() { g_check_only = true; }
@@ -103,6 +104,7 @@ int gemm_common(const int8_t *A, int64_t lda, const void *Wp, int32_t M, int32_t
 }  // namespace
 
 int ilw::report_error(int code, const char *msg) { return fail(code, "%s", msg); }
+bool ilw::validate_only() { return g_check_only; }
 
 extern "C" {
 
@@ -117,6 +119,11 @@ int ilwdetr_device_status(ilw_stream_t stream) {
     if (e != cudaSuccess) return cuda_status(e, "read device status");
     if (v == ilw::kStatusBadIndex) return fail(ILW_ERR_INVALID_ARG, "a gather index lay outside its source rows");
     if (v) return fail(ILW_ERR_TIMEOUT, "a kernel's bounded wait expired (code %d)", v);
+    return ILW_OK;
+}
+
+int ilwdetr_validate_only(int32_t on) {
+    g_check_only = on != 0;
     return ILW_OK;
 }
 
@@ -136,6 +143,7 @@ int ilwdetr_pack_weight(const int8_t *W, int32_t N, int32_t K, void *packed, ilw
     if (N == 0) return ILW_OK;
     if (!W || !packed) return fail(ILW_ERR_INVALID_ARG, "pack: NULL pointer");
     if (!aligned(packed, 256)) return fail(ILW_ERR_INVALID_ARG, "pack: output must be 256-byte aligned");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_pack_weight(W, N, K, packed, (cudaStream_t)stream), "pack_weight");
 }
 
@@ -664,6 +672,7 @@ int ilwdetr_int_sigmoid(const int32_t *X, int32_t *Y, int64_t n, const ilw_sigmo
     if (n == 0) return ILW_OK;
     if (!X || !Y || !aligned(X, 16) || !aligned(Y, 16))
         return fail(ILW_ERR_INVALID_ARG, "int_sigmoid: NULL or not 16-byte aligned");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_int_sigmoid(X, Y, n, ilw::make_shiftexp(p->I0, p->k_inter), p->k_out,
                                                (cudaStream_t)stream),
                        "int_sigmoid");
@@ -673,6 +682,7 @@ int ilwdetr_relu_i8(const int8_t *X, int8_t *Y, int64_t n, ilw_stream_t stream) 
     if (n < 0) return fail(ILW_ERR_INVALID_ARG, "relu_i8: n < 0");
     if (n == 0) return ILW_OK;
     if (!X || !Y || !aligned(X, 4) || !aligned(Y, 4)) return fail(ILW_ERR_INVALID_ARG, "relu_i8: NULL or misaligned");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_relu_i8(X, Y, n, (cudaStream_t)stream), "relu_i8");
 }
 
@@ -684,6 +694,7 @@ int ilwdetr_topk(const int32_t *S, int64_t lds, int32_t rows, int32_t N, int32_t
     if (rows == 0) return ILW_OK;
     if (!S || !vals || !idx || !aligned(S, 4) || !aligned(vals, 4) || !aligned(idx, 4))
         return fail(ILW_ERR_INVALID_ARG, "topk: NULL or misaligned");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_topk(S, lds, rows, N, K, vals, idx, (cudaStream_t)stream), "topk");
 }
 
@@ -695,6 +706,7 @@ int ilwdetr_gather_rows(const void *src, int64_t src_ld, int64_t src_rows, const
     if (n == 0 || row_bytes == 0) return ILW_OK;
     if (!src || !idx || !dst || !aligned(src, 4) || !aligned(dst, 4) || !aligned(idx, 4))
         return fail(ILW_ERR_INVALID_ARG, "gather_rows: NULL or misaligned");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_gather_rows(src, src_ld, src_rows, idx, n, row_bytes, dst, dst_ld, (cudaStream_t)stream),
                        "gather_rows");
 }
@@ -706,6 +718,7 @@ int ilwdetr_ivit_shiftgelu(const int32_t *X, int64_t ldx, int64_t rows, int32_t 
     if (rows < 0 || L < 1 || ldx < L || ldy < L) return fail(ILW_ERR_INVALID_ARG, "ivit_shiftgelu: bad sizes");
     if (rows == 0) return ILW_OK;
     if (!X || !Y || !aligned(X, 4) || !aligned(Y, 4)) return fail(ILW_ERR_INVALID_ARG, "ivit_shiftgelu: NULL or misaligned");
+    if (g_check_only) return ILW_OK;
     return cuda_status(ilw::launch_ivit_shiftgelu(X, ldx, rows, L, Y, ldy, ilw::make_gelu(*p), (cudaStream_t)stream),
                        "ivit_shiftgelu");
 }

@@ -10,6 +10,9 @@ namespace ilw {
 
 // Records `msg` as this thread's ilwdetr_last_error() text and returns `code`.
 int report_error(int code, const char *msg);
+// True while the calling thread's entry points only check their arguments (ilwdetr_validate_only,
+// or a composite entry point's checking pass): they return before any CUDA call that launches.
+bool validate_only();
 
 // Device status word (latched by kernels whose bounded waits expire): its device address on
 // the current device (nullptr on failure), and a synchronous read-and-clear.

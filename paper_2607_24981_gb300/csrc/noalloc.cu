@@ -72,13 +72,16 @@ extern "C" int ilwdetr_patch_embed_noalloc(const int8_t *img, int32_t B, int32_t
                                  "patch_embed_noalloc: this batch needs more scratch than the fixed 8 MiB "
                                  "(B * (H/p) * (W/p) * Cin * p * p bytes); split the batch or use "
                                  "ilwdetr_patch_embed with a workspace");
+    const int32_t T = (Hh / p) * (Ww / p), K = Cin * p * p;
+    ilw_residual_t r{pos, d, T, m_pos, s_pos};
+    if (ilw::validate_only())  // the GEMM's own checks; Wp (256-byte aligned) stands in for the scratch
+        return ilwdetr_gemm_requant((const int8_t *)Wp, K, Wp, bias, mult, shift, B * T, d, K, 16, x0, d,
+                                    pos ? &r : nullptr, stream);
     int8_t *scratch = nullptr;
     int rc = scratch_on_current_device(&scratch);
     if (rc) return rc;
     // every byte the GEMM reads is written by the gather first: nothing needs clearing
     cudaError_t e = ilw::launch_patchify(img, B, Cin, Hh, Ww, p, scratch, (cudaStream_t)stream);
     if (e != cudaSuccess) return ilw::report_error(ILW_ERR_CUDA, cudaGetErrorString(e));
-    const int32_t T = (Hh / p) * (Ww / p), K = Cin * p * p;
-    ilw_residual_t r{pos, d, T, m_pos, s_pos};
     return ilwdetr_gemm_requant(scratch, K, Wp, bias, mult, shift, B * T, d, K, 16, x0, d, pos ? &r : nullptr, stream);
 }

@@ -24,6 +24,18 @@ def built_lib():
     return path
 
 
+@pytest.fixture
+def validate_only(built_lib):
+    """Validate-only mode for the calling thread during one test: the argument checks run as usual
+    and nothing can be launched, so the fake addresses these tests pass are never used."""
+    import paper_2607_24981_gb300 as ilw
+
+    L = ilw.lib()
+    assert L.ilwdetr_validate_only(1) == 0
+    yield L
+    L.ilwdetr_validate_only(0)
+
+
 def test_header_declares_the_paths_entry_points():
     syms = declared_symbols()
     for name in ("ilwdetr_gemm_requant", "ilwdetr_shiftmax_attn", "ilwdetr_sdshiftgelu",
@@ -49,7 +61,7 @@ def test_binding_signatures_cover_the_header(built_lib):
     assert ilw.version().startswith("ilwdetr")
 
 
-def test_host_side_validation_without_gpu(built_lib):
+def test_host_side_validation_without_gpu(validate_only):
     """Argument errors are reported before any launch, so they work with no device at all."""
     import paper_2607_24981_gb300 as ilw
 
@@ -83,7 +95,7 @@ def test_host_side_validation_without_gpu(built_lib):
     assert rc == -2  # C % 16 != 0
 
 
-def test_detection_entry_points_validate_without_gpu(built_lib):
+def test_detection_entry_points_validate_without_gpu(validate_only):
     """The detection-head and selection entry points reject bad arguments before any launch."""
     import paper_2607_24981_gb300 as ilw
 
@@ -106,7 +118,7 @@ def test_detection_entry_points_validate_without_gpu(built_lib):
     assert L.ilwdetr_topk(ctypes.c_void_p(16), 10, 0, 10, 3, ctypes.c_void_p(16), ctypes.c_void_p(16), None) == 0
 
 
-def test_layernorm_and_noalloc_validate_without_gpu(built_lib):
+def test_layernorm_and_noalloc_validate_without_gpu(validate_only):
     """I-LayerNorm and the allocation-free patch embedding reject bad arguments before any CUDA
     call (so with no device at all): the no-alloc entry checks its weights and its scratch bound
     before it looks up the scratch array or launches the gather."""
@@ -141,19 +153,8 @@ def test_layernorm_and_noalloc_validate_without_gpu(built_lib):
     assert pe(B=7) == -2 and b"8 MiB" in L.ilwdetr_last_error()
 
 
-def _no_cuda_device():
-    try:
-        import torch
-    except ImportError:
-        return True
-    return not torch.cuda.is_available()
-
-
-# Fake device addresses: these tests only run where no CUDA device exists, so nothing can be
-# launched on them (the first real launch fails with ILW_ERR_CUDA before touching memory).
-no_device = pytest.mark.skipif(not _no_cuda_device(), reason="checks the no-device behaviour")
-
-
+# Fake device addresses: only ever passed to calls that fail their argument checks or run in
+# validate-only mode (ilwdetr_validate_only), so nothing is launched on them on any machine.
 def _fake_ptrs(struct, base):
     """Every pointer field of a ctypes struct set to a distinct 256-byte aligned fake address."""
     k = 0
@@ -163,16 +164,23 @@ def _fake_ptrs(struct, base):
             k += 1
 
 
-@no_device
 def test_composite_entry_points_check_every_step_before_launching(built_lib):
     """The encoder block, the decoder layer and the patch embedding check the arguments of all
-    their steps before the first launch: a bad parameter of a late step (the attention's Shiftmax,
-    the FFN's GELU, a residual shift, the deformable weights' Shiftmax) is an argument error, not a
-    CUDA error from a launch already made; with valid arguments the checking pass succeeds and the
-    first real launch fails only for want of a device."""
+    their steps (the pass a real call makes before its first launch): a bad parameter of a late step
+    (the attention's Shiftmax, the FFN's GELU, a residual shift, the deformable weights' Shiftmax) is
+    an argument error, and valid arguments pass every step.  Run in validate-only mode, so nothing is
+    launched whether or not a device is present."""
     import paper_2607_24981_gb300 as ilw
 
     L = ilw.lib()
+    assert L.ilwdetr_validate_only(1) == 0
+    try:
+        _composite_checks(ilw, L)
+    finally:
+        L.ilwdetr_validate_only(0)
+
+
+def _composite_checks(ilw, L):
     B, T, d, H, F = 2, 1600, 384, 6, 1536
 
     def block(**over):
@@ -189,7 +197,7 @@ def test_composite_entry_points_check_every_step_before_launching(built_lib):
         return L.ilwdetr_block_forward(ctypes.byref(bp), ctypes.c_void_p(0x100000), ctypes.c_void_p(0x200000),
                                        B, T, ctypes.c_void_p(0x300000), ws, None)
 
-    assert block() == -3  # ILW_ERR_CUDA: every step's arguments passed, the first launch has no device
+    assert block() == 0  # every step's arguments pass
     assert block(smx=ilw.ShiftmaxT(0, 16, 8, -1, 4, 31)) == -1 and b"I0" in L.ilwdetr_last_error()
     assert block(gelu=ilw.GeluT(1 << 15, 16, 8)) == -1
     assert block(s_r2=63) == -1 and b"residual" in L.ilwdetr_last_error()
@@ -219,7 +227,7 @@ def test_composite_entry_points_check_every_step_before_launching(built_lib):
                                                ctypes.c_void_p(0x300000), lvl, Ld, ctypes.c_void_p(0x400000), Bd, Q,
                                                ctypes.c_void_p(0x500000), ctypes.c_void_p(0x600000), ws, None)
 
-    assert decoder() == -3
+    assert decoder() == 0
     assert decoder(smx_w=ilw.ShiftmaxT(0, 16, 8, -1, 4, 31)) == -1  # the deformable weights, late in the layer
     assert decoder(s_s=0) == -1 and b"deform" in L.ilwdetr_last_error()
     assert decoder(gelu=ilw.GeluT(1 << 15, 16, 8)) == -1
@@ -232,7 +240,7 @@ def test_composite_entry_points_check_every_step_before_launching(built_lib):
                                      384, ctypes.c_void_p(0x600000), 1 << 30, s_pos, ctypes.c_void_p(0x700000),
                                      ctypes.c_void_p(0x800000), ws, None)
 
-    assert patch() == -3
+    assert patch() == 0
     assert patch(Wp=0x200010) == -1 and b"256-byte" in L.ilwdetr_last_error()  # the GEMM's check, before the gather
     assert patch(s_pos=63) == -1 and b"residual" in L.ilwdetr_last_error()
 
@@ -336,3 +344,44 @@ def test_oracle_sources_never_reach_the_product():
         text = open(path).read()
         for needle in ("paper_2607_24981_gb300", "libilwdetr", "ilwdetr.h", "cuda"):
             assert needle not in text, (path, needle)
+
+
+def test_validate_only_mode_checks_without_launching(built_lib):
+    """In validate-only mode every launching entry point runs its usual checks and returns ILW_OK
+    (or the error found) without launching: valid calls on fake, aligned addresses succeed and bad
+    ones still fail, on any machine."""
+    import paper_2607_24981_gb300 as ilw
+
+    L = ilw.lib()
+    v, w = ctypes.c_void_p(0x100000), ctypes.c_void_p(0x200000)
+    smx = ctypes.byref(ilw.ShiftmaxT(3000, 16, 8, -1, 4, 31))
+    g = ctypes.byref(ilw.GeluT(600, 16, 8))
+    sg = ctypes.byref(ilw.SigmoidT(1024, 8, 17))
+    assert L.ilwdetr_validate_only(1) == 0
+    try:
+        ok = {
+            "pack_weight": L.ilwdetr_pack_weight(v, 64, 64, w, None),
+            "gemm_requant": L.ilwdetr_gemm_requant(v, 64, w, v, v, v, 100, 64, 64, 8, v, 64, None, None),
+            "gemm_gelu": L.ilwdetr_gemm_gelu(v, 64, w, v, v, v, 100, 64, 64, g, 1 << 30, 35, v, 64, None),
+            "shiftmax_rows": L.ilwdetr_shiftmax_rows(v, 400, 10, 400, smx, w, 400, None),
+            "sdshiftgelu": L.ilwdetr_sdshiftgelu(v, w, 1000, g, None),
+            "int_layernorm": L.ilwdetr_int_layernorm(v, 16, 384, 10, 384, v, v, v, 10, w, 8, 384, None),
+            "shiftmax_attn": L.ilwdetr_shiftmax_attn(v, v, v, 192, 8, 1, 64, 3, 64, 0, smx, 1 << 30, 35, w, 8, 192, None),
+            "requant": L.ilwdetr_requant(v, 16, 64, 10, 64, 1 << 30, 30, None, 0, 1, 0, 1, 8, w, 64, None),
+            "resample": L.ilwdetr_resample_nearest(v, 100, 1, 10, 10, 16, w, 400, 20, 20, None),
+            "int_sigmoid": L.ilwdetr_int_sigmoid(v, w, 100, sg, None),
+            "relu_i8": L.ilwdetr_relu_i8(v, w, 100, None),
+            "topk": L.ilwdetr_topk(v, 100, 2, 100, 10, w, v, None),
+            "gather_rows": L.ilwdetr_gather_rows(v, 16, 10, w, 5, 16, v, 16, None),
+            "ivit_shiftgelu": L.ilwdetr_ivit_shiftgelu(v, 64, 4, 64, w, 64, g, None),
+            "patch_embed_noalloc": L.ilwdetr_patch_embed_noalloc(v, 2, 3, 640, 640, 16, w, v, v, v, 384, None,
+                                                                 1 << 30, 31, ctypes.c_void_p(0x300000), None),
+        }
+        assert all(rc == 0 for rc in ok.values()), ok
+        # the checks themselves still run
+        assert L.ilwdetr_gemm_requant(v, 24, w, v, v, v, 100, 64, 24, 8, v, 64, None, None) == -2  # K % 16
+        assert L.ilwdetr_topk(v, 100, 2, 100, 101, w, v, None) == -1  # K > N
+        assert L.ilwdetr_patch_embed_noalloc(v, 7, 3, 640, 640, 16, w, v, v, v, 384, None, 1 << 30, 31,
+                                             ctypes.c_void_p(0x300000), None) == -2  # beyond the 8 MiB scratch
+    finally:
+        L.ilwdetr_validate_only(0)
