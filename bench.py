@@ -26,7 +26,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "int-only encoder block tokens/s (1600 tok, d=384)"
 UNIT = "block-tokens/s"
-WORKLOAD = "medium_c2"
+WORKLOAD = "medium_backbone_b8"
 SEED = 0
 # cpu baseline sample: each image through blocks 0..4 (3 window + 2 global, the backbone's 6:4
 # window/global ratio); the reference arm instead cycles over all 10 blocks, one block per step
@@ -78,7 +78,7 @@ def workload_cfg():
 def workload_config(cfg, world):
     """The `config` of the bench line: the workload both arms report on (the reference arm times a
     bounded sample of it, described in its cpu_baseline)."""
-    return {"workload": "medium_c2: Medium integer ViT backbone (patch embed + 10 blocks)",
+    return {"workload": "medium_backbone_b8: Medium integer ViT backbone (patch embed + 10 blocks)",
             "B": cfg["B"], "T": cfg["T"], "d": cfg["d"], "H": cfg["H"], "F": cfg["F"], "blocks": cfg["layers"],
             "global_layers": list(cfg["global_layers"]), "window": "2x2 windows of 400 tokens",
             "image": "640x640 int8, 16x16 patches", "per_gpu_batch": cfg["B"],
@@ -307,7 +307,7 @@ def leg_blocks(ilw, torch, bb, img, reps, flush):
     return res
 
 
-def leg_c3(ilw, torch, dev, reps):
+def leg_sweep(ilw, torch, dev, reps):
     """The nonlinearity sweep at its workload sizes: Constrained Shiftmax over 2^27 int32 scores in
     rows of 64 / 400 / 1600, SD-ShiftGELU over 2^28 int32 values, I-LayerNorm over 2^20 int32 rows
     of 192 / 384.  Inputs drawn on the device from a seeded generator with the workload's ranges;
@@ -351,7 +351,7 @@ def leg_detector(ilw, torch, dev, reps, flush):
     projection, three decoder layers, detection head), one CUDA graph per forward."""
     from paper_2607_24981_gb300 import synth
 
-    cfg = synth.CONFIGS["detector_c4"]
+    cfg = synth.CONFIGS["medium_detector_b16"]
     bbc = synth.CONFIGS[cfg["backbone"]]
     B, Q, g = cfg["B"], cfg["Q"], cfg["grid"]
     det = ilw.Detector(synth.patch_embed_params(SEED, bbc["d"], mode=bbc["mode"]), synth.backbone_params(SEED, bbc),
@@ -559,7 +559,7 @@ def main(argv=None):
             legs = {"blocks": leg_blocks(ilw, torch, bb, img, reps, flush)}
             del bb, step, inst, e2e_step
             torch.cuda.empty_cache()
-            legs["nonlinearity_sweep"] = leg_c3(ilw, torch, dev, reps)
+            legs["nonlinearity_sweep"] = leg_sweep(ilw, torch, dev, reps)
             legs["detector"] = leg_detector(ilw, torch, dev, reps, flush)
             torch.cuda.synchronize()
         legs["clocks"] = clk2.summary()

@@ -15,10 +15,10 @@ launches of a few tens of microseconds).  Cases:
   two_stage     two-stage query selection, 16 images x 8400 memory tokens, top 300
   gemm_qkv / gemm_proj / gemm_fc1_gelu / gemm_fc2
                 the block GEMMs at 12800 tokens, d 384, MLP 1536
-  ln_c2         I-LayerNorm on the int16 residual stream, 12800 x 384
+  ln_encoder    I-LayerNorm on the int16 residual stream, 12800 x 384
   smx_64 / smx_400 / smx_1600
                 Constrained Shiftmax over 2^27 int32 scores in rows of 64 / 400 / 1600
-  gelu_c3       SD-ShiftGELU over 2^28 int32 values
+  gelu_2p28     SD-ShiftGELU over 2^28 int32 values
   ln_192 / ln_384
                 I-LayerNorm over 2^20 int32 rows of dim 192 / 384
 """
@@ -86,12 +86,12 @@ def build(case: str, batch: int = 0):
         X = _dev(synth.uniform_int(30, f"c3smx{L}", ((1 << 27) // L, L), -(1 << 15), 1 << 15))
         P = torch.empty(X.shape, dtype=torch.uint8, device="cuda")
         return (lambda: ilw.shiftmax_rows(X, {"I0": 3000}, out=P)), {"bytes": 5.0 * X.numel()}
-    if case == "gelu_c3":
+    if case == "gelu_2p28":
         X = _dev(synth.uniform_int(32, "c3gelu", (1 << 28,), -(1 << 12), 1 << 12))
         Y = torch.empty_like(X)
         return (lambda: ilw.sdshiftgelu(X, {"I0": 600}, out=Y)), {"bytes": 8.0 * X.numel()}
     if case.startswith("ln"):
-        if case == "ln_c2":
+        if case == "ln_encoder":
             X = _dev(synth.uniform_int(34, "case.ln", (12800, 384), -3000, 3000, np.int16))
             per = 3.0  # int16 in, int8 out (carried in fp16, the encoder's form)
         else:
@@ -100,8 +100,8 @@ def build(case: str, batch: int = 0):
             per = 5.0
         C = X.shape[1]
         beta, mult, shift = (_dev(a) for a in synth.ln_params(34, f"c3lnp{C}", C))
-        ob = ilw.I8_IN_F16 if case == "ln_c2" else 8
-        Y = torch.empty(X.shape, dtype=torch.float16 if case == "ln_c2" else torch.int8, device="cuda")
+        ob = ilw.I8_IN_F16 if case == "ln_encoder" else 8
+        Y = torch.empty(X.shape, dtype=torch.float16 if case == "ln_encoder" else torch.int8, device="cuda")
         return (lambda: ilw.int_layernorm(X, beta, mult, shift, 10, ob, out=Y)), {"bytes": per * X.numel()}
     if case == "heads":  # detection head on 16 images x 300 decoder queries, 80 classes
         B, Q, d = batch or 16, 300, 256

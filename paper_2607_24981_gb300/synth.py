@@ -155,14 +155,14 @@ def block_input(seed: int, B: int, T: int, d: int, dist: str = "uniform") -> np.
 # ------------------------------------------------------------------------------------------
 CONFIGS = {
     # single block, batch 1, 256 tokens, dim 192, 3 heads, MLP 768, global attention
-    "block_c0": dict(B=1, T=256, d=192, H=3, F=768, layers=1, global_layers=(0,), mode="literal",
-                     dist="uniform"),
+    "block_256tok_d192": dict(B=1, T=256, d=192, H=3, F=768, layers=1, global_layers=(0,), mode="literal",
+                              dist="uniform"),
     # Tiny-scale backbone: 6 blocks alternating window (2x2 windows of 400 tokens) / global
-    "tiny_c1": dict(B=8, T=1600, d=192, H=3, F=768, layers=6, global_layers=(1, 3, 5),
-                    mode="calibrated", dist="uniform"),
+    "tiny_backbone_b8": dict(B=8, T=1600, d=192, H=3, F=768, layers=6, global_layers=(1, 3, 5),
+                             mode="calibrated", dist="uniform"),
     # Medium-scale backbone: 10 blocks, global attention at the output layers 2, 4, 5, 9
-    "medium_c2": dict(B=8, T=1600, d=384, H=6, F=1536, layers=10, global_layers=(2, 4, 5, 9),
-                      mode="calibrated", dist="laplace"),
+    "medium_backbone_b8": dict(B=8, T=1600, d=384, H=6, F=1536, layers=10, global_layers=(2, 4, 5, 9),
+                               mode="calibrated", dist="laplace"),
 }
 
 
@@ -170,9 +170,9 @@ CONFIGS = {
 # tapped, a split-convolution projector at strides 8 / 16 / 32 (80x80, 40x40, 20x20 maps of 256
 # channels, concatenated as the decoder memory), and 3 decoder layers of 300 queries, dim 256,
 # 8 heads, 4 sampling points per level, MLP 1024.
-CONFIGS["detector_c4"] = dict(B=16, backbone="medium_c2", taps=(2, 4, 5, 9), grid=40,
-                              levels=((80, 80), (40, 40), (20, 20)), N=256, Q=300, Hd=8, Fd=1024,
-                              P=4, dec_layers=3)
+CONFIGS["medium_detector_b16"] = dict(B=16, backbone="medium_backbone_b8", taps=(2, 4, 5, 9), grid=40,
+                                      levels=((80, 80), (40, 40), (20, 20)), N=256, Q=300, Hd=8, Fd=1024,
+                                      P=4, dec_layers=3)
 
 
 def _mult(seed: int, name: str) -> int:

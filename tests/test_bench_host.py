@@ -65,6 +65,6 @@ def test_both_arms_report_one_config(bench):
     the workload and the L2 policy and carries no model keys."""
     cfg = bench.workload_cfg()
     c = bench.workload_config(cfg, 1)
-    assert c["workload"].startswith("medium_c2") and c["B"] == 8 and c["T"] == 1600 and "l2" in c
+    assert c["workload"].startswith("medium_backbone_b8") and c["B"] == 8 and c["T"] == 1600 and "l2" in c
     assert "model" not in c
     assert bench.workload_config(cfg, 4)["parallelism"] == "replicas x4"

@@ -62,7 +62,7 @@ def test_resample_nearest(ilw, orc):
 
 
 def test_projector(ilw, orc):
-    cfg = synth.CONFIGS["detector_c4"]
+    cfg = synth.CONFIGS["medium_detector_b16"]
     B, g, K = 2, cfg["grid"], 384
     pp = synth.projector_params(0, 4, K)
     taps = [synth.uniform_int(63 + i, "pj.tap", (B * g * g, K), -3000, 3000, np.int16) for i in range(4)]
@@ -74,7 +74,7 @@ def test_projector(ilw, orc):
 
 @pytest.mark.parametrize("B,Q", [(2, 300), (1, 37)])
 def test_decoder_layer(ilw, orc, B, Q):
-    cfg = synth.CONFIGS["detector_c4"]
+    cfg = synth.CONFIGS["medium_detector_b16"]
     levels = cfg["levels"]
     S = sum(h * w for h, w in levels)
     dp = synth.decoder_params(0, 1)
@@ -94,7 +94,7 @@ def test_detector_full_batch_sampled_image(ilw, orc):
     """The full integer detector forward at its workload size (batch 16) on the GPU; the oracle
     recomputes one image end to end (patch embedding, 10 blocks, the four taps, projector, three
     decoder layers)."""
-    cfg = synth.CONFIGS["detector_c4"]
+    cfg = synth.CONFIGS["medium_detector_b16"]
     bb = synth.CONFIGS[cfg["backbone"]]
     B, Q, g = cfg["B"], cfg["Q"], cfg["grid"]
     blocks = synth.backbone_params(0, bb)
@@ -129,7 +129,7 @@ def test_detector_two_stage_refinement_and_head_sampled_image(ilw, orc):
     boxes refined after each decoder layer but the last, and the detection head (class scores,
     boxes) at batch 2; the oracle recomputes one image end to end (backbone, projector, two-stage
     selection, three decoder layers with refinement and positional queries, head)."""
-    cfg = synth.CONFIGS["detector_c4"]
+    cfg = synth.CONFIGS["medium_detector_b16"]
     bb = synth.CONFIGS[cfg["backbone"]]
     B, Q, g = 2, cfg["Q"], cfg["grid"]
     blocks = synth.backbone_params(0, bb)

@@ -34,7 +34,7 @@ def same(got, want, what):
     assert len(bad) == 0, f"{what}: {len(bad)} mismatches, first {tuple(bad[0])}"
 
 
-@pytest.mark.parametrize("workload", ["medium_c2", "tiny_c1"])
+@pytest.mark.parametrize("workload", ["medium_backbone_b8", "tiny_backbone_b8"])
 def test_backbone_full_batch_sampled_images(ilw, orc, workload):
     """Full batch of 8 images through the whole backbone on the GPU (Backbone.forward, the call
     bench.py times); the oracle recomputes one sampled image end to end."""
@@ -59,7 +59,7 @@ def test_backbone_full_batch_sampled_images(ilw, orc, workload):
     y2 = bb.forward(dimg).cpu().numpy()
     same(y2g, y2, f"{workload} graph replay, second input")
     assert not np.array_equal(y2, yh.reshape(y2.shape))
-    pick = 5 if workload == "medium_c2" else 2
+    pick = 5 if workload == "medium_backbone_b8" else 2
     x = orc.patch_embed(img[pick:pick + 1], pe["p"], pe["w"], pe["b"], pe["m"], pe["s"], pe["pos"],
                         pe["m_pos"], pe["s_pos"])
     for bp in blocks:
@@ -82,7 +82,7 @@ def test_patch_embed_full_batch(ilw, orc):
 
 
 @pytest.mark.parametrize("L", [64, 400, 1600])
-def test_shiftmax_rows_c3_sampled(ilw, orc, L):
+def test_shiftmax_rows_sweep_sampled(ilw, orc, L):
     """2^27 int32 scores uniform in [-2^15, 2^15] as rows of length L; 4096 rows checked."""
     rows = (1 << 27) // L
     X = synth.uniform_int(30, f"c3smx{L}", (rows, L), -(1 << 15), 1 << 15)
@@ -94,7 +94,7 @@ def test_shiftmax_rows_c3_sampled(ilw, orc, L):
     same(P[idx], want, f"shiftmax L={L}")
 
 
-def test_sdshiftgelu_c3_sampled(ilw, orc):
+def test_sdshiftgelu_sweep_sampled(ilw, orc):
     """2^28 int32 values uniform in [-2^12, 2^12]; 2^20 sampled elements checked."""
     n = 1 << 28
     X = synth.uniform_int(32, "c3gelu", (n,), -(1 << 12), 1 << 12)
@@ -106,7 +106,7 @@ def test_sdshiftgelu_c3_sampled(ilw, orc):
 
 
 @pytest.mark.parametrize("C", [192, 384])
-def test_layernorm_c3_sampled(ilw, orc, C):
+def test_layernorm_sweep_sampled(ilw, orc, C):
     """2^20 rows of dim C, int32 uniform in [-2^14, 2^14]; 2048 rows checked."""
     rows = 1 << 20
     X = synth.uniform_int(34, f"c3ln{C}", (rows, C), -(1 << 14), 1 << 14)

@@ -312,9 +312,9 @@ def test_deform_attn(ilw, orc):
 
 
 # ------------------------------------------------------------------------------ block
-@pytest.mark.parametrize("cfg", ["c0_literal", "c0_calibrated", "small_window"])
+@pytest.mark.parametrize("cfg", ["block256_literal", "block256_calibrated", "small_window"])
 def test_block_forward(ilw, orc, cfg):
-    if cfg.startswith("c0"):
+    if cfg.startswith("block256"):
         B, T, d, H, F, win, mode = 1, 256, 192, 3, 768, 0, cfg.split("_")[1]
     else:
         B, T, d, H, F, win, mode = 2, 400, 128, 2, 256, 2, "calibrated"
