@@ -1100,8 +1100,9 @@ def _float_decoder_layer(dp, tgt, pos, memory, levels, refs, B, Q):
     return ln(clip(lin(hid, "w_fc2", "b_fc2", "m_fc2", "s_fc2", 64) + sc(t2, dp["m_r3"], dp["s_r3"]), 16), 3)
 
 
+@pytest.mark.parametrize("sharp", [False, True])
 @pytest.mark.parametrize("seed", [11, 12, 13])
-def test_decoder_layer_follows_the_real_valued_layer(orc, seed):
+def test_decoder_layer_follows_the_real_valued_layer(orc, seed, sharp):
     """The integer decoder layer against the real-valued layer it approximates (no rounding; exp
     and sigmoid exact; the same weights, scales, references and memory).  Beyond the block's error
     sources (Shiftmax outputs at scale 2^-7 with a 4-5 bit reciprocal, ShiftExp's chord, rounding),
@@ -1110,11 +1111,17 @@ def test_decoder_layer_follows_the_real_valued_layer(orc, seed):
     at correlation >= 0.99 and relative RMS deviation <= 0.15 (these seeds measure 0.9955-0.9991
     and 0.04-0.095; 0.993 and 0.12 at worst over seeds 11-15).  A residual from the wrong tensor,
     the sampling offsets' x and y exchanged, the GELU dropped, flat sampling weights or the
-    positional query left out of the cross-attention query fails it.  The self-attention's inner
-    wiring is not resolved here: at these weights its output is close to an average over the
-    queries whatever the scores are (the closed-form pins above cover it)."""
+    positional query left out of the cross-attention query fails it.  At the drawn weights the
+    self-attention output is close to an average over the queries whatever the scores are, so the
+    `sharp` cases make it decide: I0 = 256 (scores / I0 of several units, each query attending to a
+    few keys) and the first residual scaled by 2^-6 (x1 mostly the self-attention branch); there
+    the q|k input taken after LN1 (a pre-norm layer) or without the positional query fails it too
+    (seeds 11-20 of the sharp form measure at worst 0.993 and 0.117)."""
     B, Q = 2, 20
     dp, inp, levels, mem = _small_decoder(seed, B, Q)
+    if sharp:
+        dp["smx"] = dict(dp["smx"], I0=256)
+        dp["m_r1"], dp["s_r1"] = 1 << 30, 36
     out = orc.decoder_layer(dp, inp["tgt"], inp["pos"], mem, levels, inp["refs"], B, Q).astype(np.float64)
     ref = _float_decoder_layer(dp, inp["tgt"], inp["pos"], mem, levels, inp["refs"], B, Q)
     corr = np.corrcoef(out.ravel(), ref.ravel())[0, 1]
