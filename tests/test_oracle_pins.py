@@ -465,6 +465,25 @@ def test_attention_matches_composed_reference(orc):
             assert np.array_equal(O[rows, h * dh:(h + 1) * dh], want)
 
 
+def test_attention_output_saturates_symmetrically(orc):
+    """O = sat8(rq(P V)): with q = k = 0 every row is the uniform closed form of
+    tests/golden/shiftmax_closed_forms.txt (4 keys at I0 = 1: P = 31 each), so with v = +-127 and
+    the identity rescale (m = 2^30, s = 30) the exact outputs 124 * (+-127) clip to +-127, and a
+    smaller v passes through: v = 1 gives 124 / 2^3 = 15.5, rounded half up to 16 (s = 33)."""
+    golden = {(n, i0): out for n, i0, _, _, _, _, _, out in _golden_rows()}
+    P = golden[(4, 1)]
+    T, H, dh = 4, 1, 32
+    qkv = np.zeros((T, 3 * dh), np.int8)
+    qkv[:, 2 * dh:2 * dh + 16] = 127
+    qkv[:, 2 * dh + 16:] = -127
+    O = orc.attention(qkv, 1, T, H, dh, 0, _smx(1), 1 << 30, 30)
+    assert 4 * P * 127 > 127
+    assert np.all(O[:, :16] == 127) and np.all(O[:, 16:] == -127)
+    qkv[:, 2 * dh:] = 1
+    O1 = orc.attention(qkv, 1, T, H, dh, 0, _smx(1), 1 << 30, 33)
+    assert np.all(O1 == exact_rq(4 * P, 1 << 30, 33)) and exact_rq(4 * P, 1 << 30, 33) == 16
+
+
 def test_window_attention_is_global_attention_per_window(orc):
     """Windowed attention on a 6x6 token grid with 2x2 windows equals global attention run on
     each window's gathered tokens (numpy fancy indexing, independent of the oracle's index maths)."""
