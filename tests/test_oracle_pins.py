@@ -1242,6 +1242,43 @@ def _small_head(seed, M):
     return hp, out, ref
 
 
+def _float_head(hp, out, ref):
+    """The real-valued detection head: class scores 2^(k_out-1) sigmoid(logit / cls_I0) of the
+    raw class logits; box MLP with ReLU on its 8-bit hidden layers (no rounding); box logits
+    z = d m_d / 2^s_d + ref m_ref / 2^s_ref; boxes 2^16 sigmoid(z / box_I0)."""
+    out = out.astype(np.float64)
+    ref = ref.astype(np.float64)
+
+    def lin(a, w, b, m=None, s_=None):
+        acc = a @ hp[w].astype(np.float64).T + hp[b]
+        return acc if m is None else np.clip(acc * hp[m] / 2.0 ** hp[s_], -127, 127)
+
+    def sig(z):
+        return 1.0 / (1.0 + np.exp(-z))
+
+    scores = 2 ** (hp["cls_k_out"] - 1) * sig(lin(out, "w_cls", "b_cls") / hp["cls_I0"])
+    h1 = np.maximum(lin(out, "w_b1", "b_b1", "m_b1", "s_b1"), 0)
+    h2 = np.maximum(lin(h1, "w_b2", "b_b2", "m_b2", "s_b2"), 0)
+    z = lin(h2, "w_b3", "b_b3") * hp["m_d"] / 2.0 ** hp["s_d"] + ref * hp["m_ref"] / 2.0 ** hp["s_ref"]
+    return scores, 65536.0 * sig(z / hp["box_I0"]), z
+
+
+@pytest.mark.parametrize("seed", [4, 5])
+def test_detection_head_follows_the_real_valued_head(orc, seed):
+    """Against the real-valued head: the class logits are exact integers on both sides, so the
+    scores differ only by the integer sigmoid, within 0.02 of the logistic function (the bound
+    pinned above at k_inter = 8) plus the output floor: |score - 128 sigmoid| <= 0.02 * 128 + 1.
+    The box branch rounds its two hidden layers to integers, which moves z by well under 1 %
+    (relative RMS <= 0.01), so the boxes stay within 0.02 + 0.005 of 2^16 sigmoid(z / I0).  The
+    class sigmoid at the box branch's I0, a dropped hidden ReLU or a missing reference term fails it."""
+    hp, out, ref = _small_head(seed, 200)
+    scores, boxes, z = orc.detection_head(hp, out, ref)
+    sf, bf, zf = _float_head(hp, out, ref)
+    assert np.abs(scores - sf).max() <= 0.02 * 128 + 1
+    assert np.sqrt(((z - zf) ** 2).mean()) <= 0.01 * zf.std()
+    assert np.abs(boxes - bf).max() <= (0.02 + 0.005) * 65536
+
+
 def test_detection_head_reduces_to_reference_sigmoid_and_is_rowwise(orc):
     """With the box MLP's last layer zero (weights and bias), the box logits are the reference
     logits and the boxes their sigmoid; the head treats each query alone (row permutation
@@ -1257,6 +1294,20 @@ def test_detection_head_reduces_to_reference_sigmoid_and_is_rowwise(orc):
     _, b0, z0 = orc.detection_head(hp0, out, ref)
     assert np.array_equal(z0, ref.astype(np.int32))
     assert np.array_equal(b0, orc.int_sigmoid(ref.astype(np.int32), hp["box_I0"], hp["k_inter"], 17))
+
+
+def test_two_stage_images_are_independent(orc):
+    """Each image's selection, reference logits and boxes depend on its own memory rows only: the
+    batch of two gives, image by image, what each image gives alone."""
+    B, S, K, d = 2, 120, 20, 64
+    levels = ((8, 10), (4, 5), (2, 10))
+    tp = synth.two_stage_params(7, d=d, C=16, levels=levels)
+    mem = synth.uniform_int(7, "ts.mem2", (B * S, d), -127, 127, np.int8)
+    vals, idx, ref16, boxes = orc.two_stage(tp, mem, B, S, K)
+    for b in range(B):
+        v1, i1, r1, b1 = orc.two_stage(tp, mem[b * S:(b + 1) * S], 1, S, K)
+        assert np.array_equal(v1[0], vals[b]) and np.array_equal(i1[0], idx[b])
+        assert np.array_equal(r1, ref16[b * K:(b + 1) * K]) and np.array_equal(b1, boxes[b * K:(b + 1) * K])
 
 
 def test_two_stage_selects_the_best_tokens(orc):
@@ -1379,3 +1430,50 @@ def test_box_refinement_reduces_to_fixed_references(orc):
     assert np.array_equal(ref1, np.clip(rqd + ref16, -32767, 32767))
     assert np.array_equal(box1, orc.int_sigmoid(ref1.astype(np.int32), 1024, 8, 17))
 
+
+
+def _small_stack(seed, Q=12, layers=2):
+    levels = ((8, 8), (4, 4))
+    S = sum(h * w for h, w in levels)
+    dps = [synth.decoder_params(seed, i, d=64, H=2, F=128, L=2, P=2) for i in range(layers)]
+    rps = synth.refine_params(seed, layers - 1, d=64)
+    pq = synth.query_pos_params(seed, d=64, hidden=32)
+    tgt = synth.decoder_inputs(seed, 1, Q, 64)["tgt"]
+    mem = synth.laplace_int(seed, "st.mem", (S, 64), 20.0, 127, np.int8)
+    ref16 = synth.uniform_int(seed, "st.ref", (Q, 4), -3000, 3000, np.int16)
+    return dps, rps, pq, tgt, mem, levels, ref16
+
+
+def test_decoder_stack_is_a_chain_of_single_layers(orc):
+    """Refinement makes the stack a chain: two layers with the references refined between them
+    equal one layer, then the refinement of its output, then one layer started from the refined
+    references and boxes.  Layer 2 must take its positional queries and sampling points from the
+    refined boxes, not from the first layer's."""
+    dps, rps, pq, tgt, mem, levels, ref16 = _small_stack(31)
+    Q = tgt.shape[0]
+    boxes = orc.int_sigmoid(ref16.astype(np.int32), 1024, 8, 17)
+    two, r_two = orc.decoder_stack(dps, tgt, mem, levels, ref16, boxes, 1, Q, pq=pq, rps=rps)
+    t0, _ = orc.decoder_stack(dps[:1], tgt, mem, levels, ref16, boxes, 1, Q, pq=pq)
+    ref1, box1 = orc.refine_references(rps[0], t0, ref16)
+    assert not np.array_equal(box1, boxes)
+    one, r_one = orc.decoder_stack(dps[1:], t0, mem, levels, ref1, box1, 1, Q, pq=pq)
+    assert np.array_equal(two, one) and np.array_equal(r_two, r_one)
+
+
+def test_decoder_layers_sample_at_box_centres(orc):
+    """With fixed positional queries the boxes enter a decoder layer only through their centres
+    (cx, cy), the deformable sampling points (the two-stage pipeline's reference points): boxes that
+    share their centres but not their sizes give the same output; moving the centres changes it."""
+    dps, _, _, tgt, mem, levels, ref16 = _small_stack(32, layers=1)
+    Q = tgt.shape[0]
+    pos = synth.decoder_inputs(32, 1, Q, 64)["pos"]
+    boxes = orc.int_sigmoid(ref16.astype(np.int32), 1024, 8, 17)
+    other = boxes.copy()
+    other[:, 2:] = synth.uniform_int(32, "st.wh", (Q, 2), 0, 1 << 16)
+    a, _ = orc.decoder_stack(dps, tgt, mem, levels, ref16, boxes, 1, Q, pos=pos)
+    b, _ = orc.decoder_stack(dps, tgt, mem, levels, ref16, other, 1, Q, pos=pos)
+    assert np.array_equal(a, b)
+    moved = boxes.copy()
+    moved[:, :2] = (moved[:, :2] + (1 << 14)) % (1 << 16)
+    c, _ = orc.decoder_stack(dps, tgt, mem, levels, ref16, moved, 1, Q, pos=pos)
+    assert not np.array_equal(a, c)
