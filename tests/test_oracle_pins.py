@@ -905,6 +905,22 @@ def test_projector_levels_are_resampled_convolutions(orc):
     assert mem.shape[1] == s8 + s16 + s32
 
 
+def test_projector_taps_keep_their_own_scales(orc):
+    """Each tapped layer is requantised with its own scale: doubling one tap's values while
+    halving its scale (s + 1) leaves every output unchanged, because rq(2x; m, s + 1) = rq(x; m, s)
+    exactly, whereas doubling it under an unchanged scale changes the output."""
+    B, g, K, N = 1, 4, 32, 24
+    pp = synth.projector_params(9, 3, K, N=N, levels=1)
+    taps = [synth.uniform_int(9 + i, "tap", (B * g * g, K), -4000, 4000, np.int16) for i in range(3)]
+    base = orc.projector(pp, taps, B, g, ((g, g),))
+    for b in range(3):
+        t2 = [t.copy() for t in taps]
+        t2[b] = (2 * t2[b].astype(np.int32)).astype(np.int16)
+        pp2 = dict(pp, taps=[(m, s_ + (1 if i == b else 0)) for i, (m, s_) in enumerate(pp["taps"])])
+        assert np.array_equal(orc.projector(pp2, t2, B, g, ((g, g),)), base)
+        assert not np.array_equal(orc.projector(pp, t2, B, g, ((g, g),)), base)
+
+
 def test_projector_with_identity_scales_is_one_conv_over_the_concatenated_taps(orc):
     """With every tap's requantisation and every branch rescale the identity (m = 2^30, s = 30;
     tap values inside the int8 range), a projector level at the tapped grid's own size is one 1x1
@@ -999,7 +1015,9 @@ def test_decoder_layer_with_constant_branches_is_a_post_norm_chain(orc):
     its output is its requantised bias, and with identity residual scales the layer reduces to
     LayerNorms (the operator pinned above) of constant per-column adds:
     out = LN3(LN2(LN1(tgt + c1) + c2) + c3).  A residual from the wrong tensor, a LayerNorm
-    skipped or moved before its branch (pre-norm) fails it."""
+    skipped or moved before its branch (pre-norm) fails it.  Three queries get tgt = -c1 + {0, 1}
+    so that LN1 sees rows of variance below 2^6, where Newton from 2^16 needs more than 10 of the
+    decoder's 20 steps: LayerNorms run with fewer steps fail it too."""
     B, Q = 2, 20
     dp, inp, levels, mem = _small_decoder(3, B, Q)
     _silence(dp, "self", "cross", "ffn")
@@ -1010,6 +1028,10 @@ def test_decoder_layer_with_constant_branches_is_a_post_norm_chain(orc):
         dp[b] = synth.uniform_int(29, k, (d,), -(1 << 15), 1 << 15)
         cs[k] = np.array([exact_rq(int(dp[b][c]), int(dp[m][c]), int(dp[s_][c])) for c in range(d)], np.int64)
         assert 100 < np.abs(cs[k]).max() < 8000
+    low = synth.uniform_int(29, "low", (3, d), 0, 1, np.int64)
+    inp["tgt"][:3] = (low - cs["c1"]).astype(np.int16)
+    assert orc.newton_isqrt(int(((low[0] - low[0].mean()) ** 2).sum()), 10) != orc.newton_isqrt(
+        int(((low[0] - low[0].mean()) ** 2).sum()), 20)
     out = orc.decoder_layer(dp, inp["tgt"], inp["pos"], mem, levels, inp["refs"], B, Q)
     sat = lambda v: np.clip(v, -32767, 32767)
     x1 = inp["tgt"].astype(np.int64) + cs["c1"]
