@@ -589,6 +589,10 @@ def test_block_equals_composition_of_pinned_parts(orc):
     B, T, d, H, F = 1, 16, 64, 2, 128
     bp = synth.block_params(19, 0, d, H, F, 0, "calibrated")
     x = synth.block_input(19, B, T, d)
+    # three tokens of variance below 2^6, where the encoder's 10 Newton steps from 2^16 have not
+    # converged (20 would give another R): the block must run the LayerNorms with its ln_iters
+    x[:3] = synth.uniform_int(19, "lowvar", (3, d), 0, 1, np.int16)
+    assert orc.newton_isqrt(32, 10) != orc.newton_isqrt(32, 20)
     y, taps = orc.block_forward(bp, x, B, T, taps=True)
     a1 = orc.int_layernorm(x, bp["ln1_beta"], bp["ln1_mult"], bp["ln1_shift"], 10, 8)
     assert np.array_equal(a1, taps["a1"])
