@@ -78,16 +78,22 @@ def test_shiftexp_golden_odd_remainders(orc):
 
 
 def test_shiftmax_and_gelu_golden_odd_remainders(orc):
-    """A Shiftmax row and SD-ShiftGELU factors whose ShiftExp has an odd remainder
-    (tests/golden/odd_remainder_rows.txt, derived by hand from Algorithms 1 and 2)."""
+    """Shiftmax rows (one with a static denominator shift) and SD-ShiftGELU factors whose
+    ShiftExp has an odd remainder (tests/golden/odd_remainder_rows.txt, derived by hand from
+    Algorithms 1 and 2)."""
     for row in _golden_lines("odd_remainder_rows.txt"):
-        if row[0] == "shiftmax":
-            I0, Ssum, sd, SR, F = (int(v) for v in row[1:6])
+        if row[0] in ("shiftmax", "shiftmax_static"):
+            if row[0] == "shiftmax":
+                I0, Ssum, sd, SR, F = (int(v) for v in row[1:6])
+                static = -1
+            else:
+                I0, static, Ssum, SR, F = (int(v) for v in row[1:6])
+                sd = static
             bar1 = row.index("|")
             bar2 = row.index("|", bar1 + 1)
             X = np.array([[int(v) for v in row[bar1 + 1:bar2]]], dtype=np.int32)
             want = [int(v) for v in row[bar2 + 1:]]
-            P, S, sdv, SRv = orc.shiftmax_rows(X, I0)
+            P, S, sdv, SRv = orc.shiftmax_rows(X, I0, 16, 8, static)
             assert (S[0], sdv[0], SRv[0]) == (Ssum, sd, SR)
             assert (2**31 - 1) // SR == F
             assert P[0].tolist() == want
@@ -516,19 +522,20 @@ def test_split_conv_equal_scales_is_concat_conv(orc):
 
 
 def test_split_conv_branch_rescale(orc):
-    """Each branch partial is rescaled by its own dyadic ratio before the integer sum."""
+    """Each branch partial is rescaled by its own dyadic ratio before the integer sum, and the bias
+    (at the common scale) is added after it, unscaled (reading Z18)."""
     M, N = 20, 8
     Xs = [synth.uniform_int(17, f"x{i}", (M, 16), -127, 127, np.int8) for i in range(2)]
     Ws = [synth.uniform_int(17, f"w{i}", (N, 16), -127, 127, np.int8) for i in range(2)]
-    bias = np.zeros(N, np.int32)
+    bias = synth.uniform_int(17, "bias", (N,), -(1 << 14), 1 << 14)
     mult = np.full(N, 1 << 30, np.int32)
     shift = np.full(N, 38, np.int32)
-    mb, sb = [1 << 30, 3 << 28], [30, 31]  # ratios 1 and 3/8
+    mb, sb = [3 << 28, 1 << 30], [31, 30]  # ratios 3/8 and 1
     Y = orc.split_conv(Xs, Ws, mb, sb, bias, mult, shift)
     for i in range(M):
         for c in range(N):
             t = sum(exact_rq(int(Xs[b][i].astype(np.int64) @ Ws[b][c].astype(np.int64)), mb[b], sb[b])
-                    for b in range(2))
+                    for b in range(2)) + int(bias[c])
             assert Y[i, c] == max(-127, min(127, exact_rq(t, 1 << 30, 38)))
 
 
