@@ -68,3 +68,25 @@ def test_both_arms_report_one_config(bench):
     assert c["workload"].startswith("medium_backbone_b8") and c["B"] == 8 and c["T"] == 1600 and "l2" in c
     assert "model" not in c
     assert bench.workload_config(cfg, 4)["parallelism"] == "replicas x4"
+
+
+def test_reference_arm_prints_one_contract_line():
+    """`bench.py --impl reference` (the oracle on the host's cores) prints one JSON line with the
+    metric, unit and config of the GPU arm, its own CPU baseline and a zero-copy e2e block."""
+    import json
+    import subprocess
+    import sys
+
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+                        "--warmup", "0"], capture_output=True, text=True, timeout=900, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["unit"] == "block-tokens/s" and line["value"] > 0
+    assert line["higher_is_better"] is True and line["steps"] == 1 and line["warmup"] == 0
+    assert line["config"]["workload"].startswith("medium_backbone_b8")
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == line["value"] and cb["sample"]
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
