@@ -446,6 +446,21 @@ def test_gemm_matches_numpy_int64_and_exact_rq(orc, out_bits):
             assert C[i, c] == want
 
 
+def test_gemm_extreme_accumulators(orc):
+    """All-127 operands drive the accumulator to K * 127^2 (+ bias): the raw 32-bit output is that
+    sum exactly (2,064,512 + 5 at K = 128, well past 2^20), and an accumulator beyond int32 (K =
+    140,000: 2.26e9) is an error, not a wrapped value."""
+    A = np.full((3, 128), 127, np.int8)
+    W = np.full((2, 128), 127, np.int8)
+    b = np.array([5, -5], np.int32)
+    C = orc.gemm_requant(A, W, b, None, None, 32)
+    assert np.array_equal(C, np.array([[128 * 127 * 127 + 5, 128 * 127 * 127 - 5]] * 3))
+    A2 = np.full((1, 140000), 127, np.int8)
+    W2 = np.full((1, 140000), 127, np.int8)
+    with pytest.raises(ValueError, match="rc=-2"):
+        orc.gemm_requant(A2, W2, None, None, None, 32)
+
+
 # ----------------------------------------------------------------------------- attention
 def _smx(I0):
     return {"I0": I0, "k_inter": 16, "k_out": 8, "s_d": -1, "m_p": 4, "M_hw": 31}
@@ -488,6 +503,17 @@ def test_attention_output_saturates_symmetrically(orc):
     qkv[:, 2 * dh:] = 1
     O1 = orc.attention(qkv, 1, T, H, dh, 0, _smx(1), 1 << 30, 33)
     assert np.all(O1 == exact_rq(4 * P, 1 << 30, 33)) and exact_rq(4 * P, 1 << 30, 33) == 16
+
+
+def test_window_attention_needs_a_divisible_square_grid(orc):
+    """Windows cut the sqrt(T) x sqrt(T) token grid into nw x nw equal squares: a grid side that
+    nw does not divide (6 tokens, 4 windows per side), or a T that is not a square, is refused."""
+    qkv = np.zeros((36, 3 * 32), np.int8)
+    with pytest.raises(ValueError, match="rc=-1"):
+        orc.attention(qkv, 1, 36, 1, 32, 4, _smx(100), 1 << 30, 30)
+    with pytest.raises(ValueError, match="rc=-1"):
+        orc.attention(np.zeros((35, 3 * 32), np.int8), 1, 35, 1, 32, 2, _smx(100), 1 << 30, 30)
+    assert orc.attention(qkv, 1, 36, 1, 32, 3, _smx(100), 1 << 30, 30).shape == (36, 32)
 
 
 def test_window_attention_is_global_attention_per_window(orc):
