@@ -905,6 +905,26 @@ def test_requant_special_cases(orc):
     Z = rng.integers(-32767, 32768, size=(1, 12)).astype(np.int16)
     zr = orc.requant(np.repeat(Z, 37, axis=0), m, s, out_bits=32).astype(np.int64)
     assert np.array_equal(orc.requant(X, m, s, Z, m, s, out_bits=32), one + zr)
+    # a 32-bit result beyond int32 is an error, not a wrapped value: 2^31 - 1 doubled
+    with pytest.raises(ValueError, match="rc=-2"):
+        orc.requant(np.array([[(1 << 31) - 1]], np.int32), 1 << 30, 29, out_bits=32)
+
+
+def test_gather_and_split_conv_refuse_out_of_range(orc):
+    """A gather index outside the source rows is an error (the CUDA path reports it through the
+    device status word), and a split-convolution branch accumulator beyond int32 (all-127 operands,
+    K = 140,000 per branch) is an error, not a wrapped value."""
+    src = np.arange(20, dtype=np.int32).reshape(5, 4)
+    assert np.array_equal(orc.gather_rows(src, np.array([4, 0])), src[[4, 0]])
+    with pytest.raises(ValueError, match="rc=-1"):
+        orc.gather_rows(src, np.array([5]))
+    with pytest.raises(ValueError, match="rc=-1"):
+        orc.gather_rows(src, np.array([-1]))
+    X = [np.full((1, 140000), 127, np.int8)]
+    W = [np.full((1, 140000), 127, np.int8)]
+    with pytest.raises(ValueError, match="rc=-2"):
+        orc.split_conv(X, W, [1 << 30], [30], np.zeros(1, np.int32), np.full(1, 1 << 30, np.int32),
+                       np.full(1, 40, np.int32))
 
 
 def test_resample_nearest_against_numpy(orc):
